@@ -1,0 +1,189 @@
+"""CPU oracle for multipoint quantization (arXiv 2002.09049) -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline / reference arm may
+import this package.  The product path (``paper_2002_09049_gb300``) never imports, links or runs it,
+and the two share no code: this package compiles ``mpq_oracle.c`` with the host C compiler and calls
+it through ctypes on numpy arrays.
+
+Each wrapper names the passage of the paper it follows; the C file states every reading of the text.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "mpq_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB = os.path.join(_BUILD, "libmpq_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+CFLAGS = ["-std=c99", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with the host C compiler (gcc/cc).  Returns the library path."""
+    with _lock:
+        if not force and os.path.exists(_LIB) and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC):
+            return _LIB
+        os.makedirs(_BUILD, exist_ok=True)
+        cc = os.environ.get("CC", "cc")
+        tmp = _LIB + f".{os.getpid()}.tmp"
+        subprocess.run([cc, *CFLAGS, _SRC, "-o", tmp, "-lm"], check=True)
+        os.replace(tmp, _LIB)
+        return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        I = ctypes.c_int
+        L = ctypes.c_long
+        D = ctypes.c_double
+        lib.mpqo_candidate_errors.argtypes = [P, I, I, I, P, P, P]
+        lib.mpqo_candidate_errors.restype = None
+        lib.mpqo_quantize_layer.argtypes = [P, I, I, I, I, P, I, P, P, P, P, P, P, P, I, I, P]
+        lib.mpqo_quantize_layer.restype = None
+        lib.mpqo_output_error.argtypes = [P, I, I, P, P, P, I, I, I, P, I, I, P]
+        lib.mpqo_output_error.restype = None
+        lib.mpqo_allocate_budget.argtypes = [P, I, I, D, P]
+        lib.mpqo_allocate_budget.restype = L
+        lib.mpqo_allocate_threshold.argtypes = [P, I, I, D, P]
+        lib.mpqo_allocate_threshold.restype = L
+        lib.mpqo_reconstruct.argtypes = [P, P, P, I, I, I, P]
+        lib.mpqo_reconstruct.restype = None
+        _lib = lib
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def _ranges(C: int, threads: int):
+    threads = max(1, min(threads, C))
+    step = (C + threads - 1) // threads
+    return [(c0, min(C, c0 + step)) for c0 in range(0, C, step)]
+
+
+def candidate_errors(r, bits: int, G: int, grid_frac=None):
+    """Eq. 9 objective ||r - s_g [r/s_g]_Q||^2 for every grid point g (double), and s_g (fp32)."""
+    lib = _load()
+    r = _c(r, np.float32)
+    gf = None if grid_frac is None else _c(grid_frac, np.float32)
+    E = np.empty(G, np.float64)
+    s = np.empty(G, np.float32)
+    lib.mpqo_candidate_errors(_p(r), r.size, bits, G, _p(gf), _p(E), _p(s))
+    return E, s
+
+
+def quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, channels=None,
+                   want_residuals: bool = True, threads: int = 1):
+    """Algorithm 1 (Eq. 7-9) for every channel of W (C x d, fp32), run to k_max points.
+
+    Returns a dict with codes [k_max][C][d] int8, scales [C][k_max] fp32, resid_sq [C][k_max+1]
+    float64, residuals [k_max][C][d] fp32 (or None), gstar/best/second [C][k_max].
+    ``channels`` = (c0, c1) restricts the work to a channel range (other rows stay zero).
+    """
+    lib = _load()
+    W = _c(W, np.float32)
+    C, d = W.shape
+    gf = None if grid_frac is None else _c(grid_frac, np.float32)
+    out = dict(
+        codes=np.zeros((k_max, C, d), np.int8),
+        scales=np.zeros((C, k_max), np.float32),
+        resid_sq=np.zeros((C, k_max + 1), np.float64),
+        residuals=np.zeros((k_max, C, d), np.float32) if want_residuals else None,
+        gstar=np.zeros((C, k_max), np.int32),
+        best=np.zeros((C, k_max), np.float64),
+        second=np.zeros((C, k_max), np.float64),
+    )
+    c0, c1 = channels if channels is not None else (0, C)
+
+    def run(rng):
+        work = np.empty(d, np.float32)
+        lib.mpqo_quantize_layer(_p(W), C, d, bits, G, _p(gf), k_max, _p(out["codes"]),
+                                _p(out["scales"]), _p(out["resid_sq"]), _p(out["residuals"]),
+                                _p(out["gstar"]), _p(out["best"]), _p(out["second"]), rng[0], rng[1],
+                                _p(work))
+
+    _parallel(run, [(a + c0, b + c0) for a, b in _ranges(c1 - c0, threads)], threads)
+    return out
+
+
+def output_error(X, groups: int, W, codes, scales, k_max: int, channels=None, threads: int = 1):
+    """Eq. 11 for n = 0..k_max points: err[k][n] = mean_t (x_t . r_{k,n+1})^2, in double.
+
+    groups = 1: X is N x d (shared); groups = C: X is C x N x d (one block per channel).
+    """
+    lib = _load()
+    W = _c(W, np.float32)
+    C, d = W.shape
+    X = _c(X, np.float32)
+    N = X.shape[-2]
+    codes = _c(codes, np.int8)
+    scales = _c(scales, np.float32)
+    err = np.zeros((C, k_max + 1), np.float64)
+    c0, c1 = channels if channels is not None else (0, C)
+
+    def run(rng):
+        work = np.empty(d, np.float32)
+        lib.mpqo_output_error(_p(X), N, groups, _p(W), _p(codes), _p(scales), C, d, k_max,
+                              _p(err), rng[0], rng[1], _p(work))
+
+    _parallel(run, [(a + c0, b + c0) for a, b in _ranges(c1 - c0, threads)], threads)
+    return err
+
+
+def allocate_budget(err32, k_max: int, beta: float):
+    """Budget reading of Algorithm 2: sequential marginal-gain loop on the fp32 error table."""
+    lib = _load()
+    err32 = _c(err32, np.float32)
+    C = err32.shape[0]
+    n = np.zeros(C, np.int32)
+    used = lib.mpqo_allocate_budget(_p(err32), C, k_max, float(beta), _p(n))
+    return n, int(used)
+
+
+def allocate_threshold(err32, k_max: int, eps: float):
+    """Algorithm 2: smallest n with e(n) < eps, else k_max."""
+    lib = _load()
+    err32 = _c(err32, np.float32)
+    C = err32.shape[0]
+    n = np.zeros(C, np.int32)
+    used = lib.mpqo_allocate_threshold(_p(err32), C, k_max, float(eps), _p(n))
+    return n, int(used)
+
+
+def reconstruct(codes, scales, npoints):
+    """Eq. 4: w~_k = sum_{i<=n_k} s_{k,i} q_{k,i} (fmaf chain from 0)."""
+    lib = _load()
+    codes = _c(codes, np.int8)
+    scales = _c(scales, np.float32)
+    npoints = _c(npoints, np.int32)
+    k_max, C, d = codes.shape
+    W_hat = np.zeros((C, d), np.float32)
+    lib.mpqo_reconstruct(_p(codes), _p(scales), _p(npoints), C, d, k_max, _p(W_hat))
+    return W_hat
+
+
+def _parallel(fn, ranges, threads):
+    """Channels are independent: ranges run on a thread pool (ctypes drops the GIL in C calls)."""
+    if threads <= 1 or len(ranges) == 1:
+        for rng in ranges:
+            fn(rng)
+        return
+    with ThreadPoolExecutor(max_workers=threads) as ex:
+        list(ex.map(fn, ranges))

@@ -1,0 +1,309 @@
+/*
+ * Multipoint quantization oracle -- plain, slow, single-threaded CPU restatement of the method
+ * (Liu et al., "Post-training Quantization with Multiple Points", arXiv 2002.09049).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product path links, loads or calls this file: only the
+ * tests, __graft_entry__.smoke() and bench.py's CPU-baseline / reference arm use it.  It shares no
+ * code, header, table or helper with the CUDA path.
+ *
+ * Build: cc -std=c99 -O2 -ffp-contract=off -fno-fast-math -fPIC -shared (see oracle/__init__.py).
+ * -ffp-contract=off keeps every a*b+c below as a rounded multiply followed by a rounded add, except
+ * where fmaf() is written out on purpose.
+ *
+ * Notation follows the paper: residual r_i (Eq. 7), scale a and codes [r/a]_Q (Eq. 8), scale search
+ * (Eq. 9), Algorithm 1 (greedy points), output error e(w, w~, D_L) (Eq. 11), Algorithm 2 (per-channel
+ * point count), multipoint sum w~ = sum_i a_i w~_i (Eq. 4).  The paper's a_i [r/a_i]_{[-1:eps_b:1]}
+ * is written here as s_i q_i with integer codes q_i in {-Qmax..Qmax}, Qmax = 2^(b-1)-1 and
+ * s_i = a_i / Qmax (Eq. 1, symmetric set, B = 0).
+ *
+ * Readings where the paper is silent (each one is also listed in the design doc):
+ *  - exact half-way ties of the nearest rounding (Eq. 2) go to the even integer (C nearbyintf);
+ *  - r / a is one correctly rounded fp32 division (Eq. 8 writes a division);
+ *  - the scale grid is G points s_g = f_g * (max|r| / Qmax), f_g = (g+1)/G in fp32 unless the caller
+ *    gives its own increasing fractions in (0, 1] (replaces the adaptive grid of Eq. 10);
+ *  - the scale search keeps the FIRST (lowest g) minimiser;
+ *  - a candidate whose fp32 scale underflows to 0 gives all-zero codes;
+ *  - a residual that is exactly zero gives a "null point": scale 0, codes 0, residual unchanged;
+ *  - a channel holding a NaN or Inf weight gets scales NaN, codes 0, residuals = w, errors NaN;
+ *  - the residual update is r <- fmaf(-s, q, r), one correctly rounded fp32 operation;
+ *  - the expectation of Eq. 11 is the sample mean over the N calibration rows, evaluated on the
+ *    residual r_{n+1} = w - w~(n) produced by the same fp32 recursion;
+ *  - the per-channel point budget: see mpqo_allocate_budget.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stddef.h>
+
+/* Eq. 1 with b bits: the symmetric integer grid {-Qmax..Qmax}, Qmax = 2^(b-1) - 1. */
+static int qmax_of(int bits) { return (1 << (bits - 1)) - 1; }
+
+/* Eq. 2-3 and Eq. 8: nearest element of s * {-Qmax..Qmax} to r, returned as the integer code.
+ * Rounding to the nearest integer and then clipping to [-Qmax, Qmax] gives the nearest grid
+ * element because the grid is a contiguous run of integers. */
+static int nearest_code(float r, float s, int qmax)
+{
+    if (s == 0.0f) return 0;
+    float t = nearbyintf(r / s);
+    if (t > (float)qmax) t = (float)qmax;
+    if (t < (float)(-qmax)) t = (float)(-qmax);
+    return (int)t;
+}
+
+/* The g-th candidate scale of the search grid (0-based g). */
+static float candidate_scale(int g, int G, const float *grid_frac, float smax)
+{
+    float f = grid_frac ? grid_frac[g] : (float)(g + 1) / (float)G;
+    return f * smax;
+}
+
+static int all_finite(const float *w, int d)
+{
+    for (int j = 0; j < d; ++j)
+        if (!isfinite(w[j])) return 0;
+    return 1;
+}
+
+/* The objective of Eq. 9 for one candidate scale: || r - s [r/s]_Q ||^2, summed in double in
+ * index order.  s*q is exact in double (24-bit times <=8-bit). */
+static double candidate_error(const float *r, int d, float s, int qmax)
+{
+    double E = 0.0;
+    for (int j = 0; j < d; ++j) {
+        int q = nearest_code(r[j], s, qmax);
+        double e = (double)r[j] - (double)s * (double)q;
+        E += e * e;
+    }
+    return E;
+}
+
+/* All G candidate errors of Eq. 9 for one residual (used by the brute-force tests).
+ * E[g] and s[g] are written for g = 0..G-1.  A zero residual gives s = 0 and E = 0 everywhere. */
+void mpqo_candidate_errors(const float *r, int d, int bits, int G, const float *grid_frac,
+                           double *E, float *s)
+{
+    int qmax = qmax_of(bits);
+    float m = 0.0f;
+    for (int j = 0; j < d; ++j) {
+        float a = fabsf(r[j]);
+        if (a > m) m = a;
+    }
+    float smax = m / (float)qmax;
+    for (int g = 0; g < G; ++g) {
+        float sg = (m == 0.0f) ? 0.0f : candidate_scale(g, G, grid_frac, smax);
+        s[g] = sg;
+        E[g] = candidate_error(r, d, sg, qmax);
+    }
+}
+
+/* Algorithm 1 for one channel w (length d), run to k_max points.
+ *   codes     [k_max][code_stride]  int8  (row i holds q_{i+1}; only the first d entries are written)
+ *   scales    [k_max]               fp32  (s_{i+1})
+ *   resid_sq  [k_max+1]             double, ||r_{n+1}||^2 for n = 0..k_max (n = 0 is ||w||^2)
+ *   residuals [k_max][res_stride]   fp32  r_{n+1} for n = 1..k_max, nullable
+ *   gstar     [k_max]               chosen grid index, -1 for a null point, nullable
+ *   best, second [k_max]            smallest and second smallest E_g of each step, nullable
+ * Every step: m = max|r| (exact), smax = m / Qmax, candidates s_g, codes [r/s_g]_Q, the first g with
+ * the smallest error (Eq. 9), then r <- r - s q (Eq. 7) as one fmaf per element. */
+void mpqo_quantize_channel(const float *w, int d, int bits, int G, const float *grid_frac,
+                           int k_max, int8_t *codes, long code_stride, float *scales,
+                           double *resid_sq, float *residuals, long res_stride, float *r,
+                           int *gstar, double *best, double *second)
+{
+    int qmax = qmax_of(bits);
+    for (int j = 0; j < d; ++j) r[j] = w[j];
+    int finite = all_finite(w, d);
+
+    double r2 = 0.0;
+    for (int j = 0; j < d; ++j) r2 += (double)r[j] * (double)r[j];
+    if (resid_sq) resid_sq[0] = finite ? r2 : NAN;
+
+    for (int i = 0; i < k_max; ++i) {
+        int8_t *qi = codes + (long)i * code_stride;
+        double E1 = INFINITY, E2 = INFINITY;
+        int gbest = -1;
+        float sbest = 0.0f;
+
+        if (!finite) {
+            for (int j = 0; j < d; ++j) qi[j] = 0;
+            scales[i] = NAN;
+        } else {
+            float m = 0.0f;
+            for (int j = 0; j < d; ++j) {
+                float a = fabsf(r[j]);
+                if (a > m) m = a;
+            }
+            if (m == 0.0f) {
+                /* null point: nothing left to represent */
+                for (int j = 0; j < d; ++j) qi[j] = 0;
+                scales[i] = 0.0f;
+                E1 = E2 = 0.0;
+            } else {
+                float smax = m / (float)qmax;
+                for (int g = 0; g < G; ++g) {
+                    float sg = candidate_scale(g, G, grid_frac, smax);
+                    double E = candidate_error(r, d, sg, qmax);
+                    if (E < E1) {
+                        E2 = E1;
+                        E1 = E;
+                        gbest = g;
+                        sbest = sg;
+                    } else if (E < E2) {
+                        E2 = E;
+                    }
+                }
+                for (int j = 0; j < d; ++j) {
+                    int q = nearest_code(r[j], sbest, qmax);
+                    qi[j] = (int8_t)q;
+                    r[j] = fmaf(-sbest, (float)q, r[j]);
+                }
+                scales[i] = sbest;
+            }
+        }
+        if (gstar) gstar[i] = gbest;
+        if (best) best[i] = E1;
+        if (second) second[i] = E2;
+        if (residuals) {
+            float *ri = residuals + (long)i * res_stride;
+            for (int j = 0; j < d; ++j) ri[j] = r[j];
+        }
+        if (resid_sq) {
+            double s2 = 0.0;
+            for (int j = 0; j < d; ++j) s2 += (double)r[j] * (double)r[j];
+            resid_sq[i + 1] = finite ? s2 : NAN;
+        }
+    }
+}
+
+/* Algorithm 1 for channels [c0, c1) of a C x d layer (row-major W).  Output layouts match the
+ * library's: codes [k_max][C][d], scales [C][k_max], resid_sq [C][k_max+1] (double here),
+ * residuals [k_max][C][d] (nullable), gstar/best/second [C][k_max] (nullable).
+ * work: scratch of d floats. */
+void mpqo_quantize_layer(const float *W, int C, int d, int bits, int G, const float *grid_frac,
+                         int k_max, int8_t *codes, float *scales, double *resid_sq,
+                         float *residuals, int *gstar, double *best, double *second, int c0, int c1,
+                         float *work)
+{
+    long plane = (long)C * d;
+    for (int k = c0; k < c1; ++k) {
+        mpqo_quantize_channel(W + (long)k * d, d, bits, G, grid_frac, k_max,
+                              codes + (long)k * d, plane, scales + (long)k * k_max,
+                              resid_sq ? resid_sq + (long)k * (k_max + 1) : NULL,
+                              residuals ? residuals + (long)k * d : NULL, plane, work,
+                              gstar ? gstar + (long)k * k_max : NULL,
+                              best ? best + (long)k * k_max : NULL,
+                              second ? second + (long)k * k_max : NULL);
+    }
+}
+
+/* Eq. 11 for channels [c0, c1): err[k][n] = (1/N) sum_t (x_t . r_{k,n+1})^2, n = 0..k_max, with
+ * r_{k,1} = w_k and r_{k,n+1} = fmaf(-s_{k,n}, q_{k,n}, r_{k,n}) (the recursion of Eq. 7).
+ * groups = 1: X is N x d, shared by every channel.  groups = C: X is [C][N][d], channel k reads
+ * its own N x d block (depthwise convolution: each channel sees its own input patches).
+ * Dot products and the mean are taken in double.  work: scratch of d floats. */
+void mpqo_output_error(const float *X, int N, int groups, const float *W, const int8_t *codes,
+                       const float *scales, int C, int d, int k_max, double *err, int c0, int c1,
+                       float *work)
+{
+    long plane = (long)C * d;
+    for (int k = c0; k < c1; ++k) {
+        const float *Xk = (groups == 1) ? X : X + (long)k * N * d;
+        float *r = work;
+        for (int j = 0; j < d; ++j) r[j] = W[(long)k * d + j];
+        for (int n = 0; n <= k_max; ++n) {
+            if (n > 0) {
+                float s = scales[(long)k * k_max + (n - 1)];
+                const int8_t *q = codes + (long)(n - 1) * plane + (long)k * d;
+                for (int j = 0; j < d; ++j) r[j] = fmaf(-s, (float)q[j], r[j]);
+            }
+            double acc = 0.0;
+            for (int t = 0; t < N; ++t) {
+                const float *x = Xk + (long)t * d;
+                double y = 0.0;
+                for (int j = 0; j < d; ++j) y += (double)x[j] * (double)r[j];
+                acc += y * y;
+            }
+            err[(long)k * (k_max + 1) + n] = acc / (double)N;
+        }
+    }
+}
+
+/* Gain of the (n+1)-th point of channel k: e_k(n) - e_k(n+1), one fp32 subtraction of the fp32
+ * error table (the same table the GPU allocator receives).  NaN is read as "no gain". */
+static float point_gain(const float *err, int k_max, int k, int n)
+{
+    const float *e = err + (long)k * (k_max + 1);
+    float g = e[n] - e[n + 1];
+    return isnan(g) ? -INFINITY : g;
+}
+
+/* Point allocation with a total budget (the marginal-gain reading of Algorithm 2).
+ * Every channel starts with one point.  P_total = floor(beta*C + 0.5); the extra P_total - C points
+ * (at most C*(k_max-1)) are handed out one at a time, each to the channel whose next point lowers
+ * its output error the most (largest e_k(n_k) - e_k(n_k+1), lowest k on ties), among channels with
+ * n_k < k_max.  The loop stops early when the best remaining gain is <= 0.
+ * Writes npoints[C]; returns the total number of points used. */
+long mpqo_allocate_budget(const float *err, int C, int k_max, double beta, int *npoints)
+{
+    long total = (long)floor(beta * (double)C + 0.5);
+    long extra = total - C;
+    long cap = (long)C * (k_max - 1);
+    if (extra < 0) extra = 0;
+    if (extra > cap) extra = cap;
+    for (int k = 0; k < C; ++k) npoints[k] = 1;
+    long used = C;
+    for (long it = 0; it < extra; ++it) {
+        float bestg = -INFINITY;
+        int bk = -1;
+        for (int k = 0; k < C; ++k) {
+            if (npoints[k] >= k_max) continue;
+            float g = point_gain(err, k_max, k, npoints[k]);
+            if (bk < 0 || g > bestg) {
+                bestg = g;
+                bk = k;
+            }
+        }
+        if (bk < 0 || !(bestg > 0.0f)) break;
+        npoints[bk] += 1;
+        used += 1;
+    }
+    return used;
+}
+
+/* Algorithm 2 with a threshold: n_k is the smallest n in 1..k_max with e_k(n) < eps (compared in
+ * double), else k_max.  Returns the total number of points. */
+long mpqo_allocate_threshold(const float *err, int C, int k_max, double eps, int *npoints)
+{
+    long used = 0;
+    for (int k = 0; k < C; ++k) {
+        int n = k_max;
+        for (int m = 1; m <= k_max; ++m) {
+            if ((double)err[(long)k * (k_max + 1) + m] < eps) {
+                n = m;
+                break;
+            }
+        }
+        npoints[k] = n;
+        used += n;
+    }
+    return used;
+}
+
+/* Eq. 4: w~_k = sum_{i=1..n_k} s_{k,i} q_{k,i}, accumulated as acc = fmaf(s_i, q_i, acc) from
+ * acc = 0 in the order i = 1, 2, ...  n_k is clamped to [0, k_max]. */
+void mpqo_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C, int d,
+                      int k_max, float *W_hat)
+{
+    long plane = (long)C * d;
+    for (int k = 0; k < C; ++k) {
+        int n = npoints[k];
+        if (n < 0) n = 0;
+        if (n > k_max) n = k_max;
+        for (int j = 0; j < d; ++j) {
+            float acc = 0.0f;
+            for (int i = 0; i < n; ++i)
+                acc = fmaf(scales[(long)k * k_max + i], (float)codes[(long)i * plane + (long)k * d + j],
+                           acc);
+            W_hat[(long)k * d + j] = acc;
+        }
+    }
+}

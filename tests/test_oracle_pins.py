@@ -1,0 +1,311 @@
+"""Pins of the CPU oracle to facts fixed by the paper and by mathematics (no GPU needed).
+
+Each test checks the oracle against something other than itself: a hand-worked example, exhaustive
+enumeration, a closed form, an invariance of the method, or a library routine used as a step.
+"""
+import itertools
+import json
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+from paper_2002_09049_gb300 import workloads as wlm
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _grid(m, qmax, G, grid_frac=None):
+    """The candidate-scale grid as stated in the method description (fp32)."""
+    smax = np.float32(m) / np.float32(qmax)
+    f = (np.arange(1, G + 1, dtype=np.float32) / np.float32(G)) if grid_frac is None else \
+        np.asarray(grid_frac, np.float32)
+    return (f * smax).astype(np.float32)
+
+
+# --- Algorithm 1 / Eq. 7-9 --------------------------------------------------------------------
+
+def test_hand_worked_example(oracle):
+    """Sec. 3.2 Eq. 7-9: matches a two-step example worked by hand."""
+    ex = json.load(open(os.path.join(GOLDEN, "greedy_hand_example.json")))
+    W = np.array([ex["w"]], np.float32)
+    out = oracle.quantize_layer(W, ex["bits"], ex["G"], ex["k_max"])
+    r = W[0].copy()
+    for i, st in enumerate(ex["steps"]):
+        E, s = oracle.candidate_errors(r, ex["bits"], ex["G"])
+        np.testing.assert_allclose(s, st["scales"], rtol=1e-6)
+        np.testing.assert_allclose(E, st["E"], rtol=1e-6)
+        assert out["gstar"][0, i] == st["gstar"]
+        assert out["codes"][i, 0].tolist() == st["codes"]
+        np.testing.assert_allclose(out["residuals"][i, 0], st["residual_after"], atol=1e-7)
+        r = out["residuals"][i, 0]
+
+
+@pytest.mark.parametrize("bits,d", [(2, 1), (2, 2), (2, 3), (2, 4), (3, 2), (3, 3)])
+@pytest.mark.parametrize("seed", range(6))
+def test_brute_force_step_is_grid_optimal(oracle, bits, d, seed):
+    """Eq. 8-9: for every grid scale the rounded codes are the best code vector (exhaustive over
+    all (2Qmax+1)^d vectors), and the chosen scale attains the exhaustive minimum over
+    (scale, code).  The one allowed slack: the codes come from an fp32 quotient r/s, so an element
+    whose exact r/s lies within half an fp32 ulp of a half-integer may take the other neighbour,
+    costing at most 2 s^2 (Qmax+1) 2^-24 of error per element."""
+    qmax = 2 ** (bits - 1) - 1
+    G = 16
+    W = wlm.random_weights(1, d, 100 + seed, "normal")
+    out = oracle.quantize_layer(W, bits, G, 3)
+    r = W[0].copy()
+    levels = range(-qmax, qmax + 1)
+    for i in range(3):
+        m = np.abs(r).max()
+        if m == 0:
+            assert out["scales"][0, i] == 0
+            break
+        scales = _grid(m, qmax, G)
+        rd = r.astype(np.float64)
+        exhaustive = []
+        for s in scales:
+            best = min(float(np.sum((rd - float(s) * np.array(q, np.float64)) ** 2))
+                       for q in itertools.product(levels, repeat=d))
+            exhaustive.append(best)
+        exhaustive = np.array(exhaustive)
+        slack = d * 2.0 * scales.astype(np.float64) ** 2 * (qmax + 1) * 2.0 ** -24
+        E, s_or = oracle.candidate_errors(r, bits, G)
+        np.testing.assert_array_equal(s_or, scales)
+        assert np.all(E >= exhaustive * (1 - 1e-14))
+        assert np.all(E - exhaustive <= slack + 1e-14 * exhaustive)
+        g = out["gstar"][0, i]
+        assert g == int(np.argmin(E))                       # first minimiser
+        assert E[g] <= exhaustive.min() + slack[g] + 1e-14 * exhaustive.min()
+        assert out["scales"][0, i] == scales[g]
+        r = out["residuals"][i, 0]
+
+
+def test_one_point_is_plain_per_channel_quantization(oracle):
+    """Eq. 9 with n = 1: the first point is ordinary symmetric per-channel b-bit quantization with
+    the best scale of the grid (vectorised textbook quantizer over all candidate scales at once)."""
+    for bits, G, dist in ((4, 64, "normal"), (3, 32, "laplace"), (8, 16, "t")):
+        qmax = 2 ** (bits - 1) - 1
+        W = wlm.random_weights(24, 97, 7 + bits, dist)
+        out = oracle.quantize_layer(W, bits, G, 1)
+        for k in range(W.shape[0]):
+            w = W[k]
+            s = _grid(np.abs(w).max(), qmax, G)                        # [G]
+            q = np.clip(np.rint(w[None, :] / s[:, None]), -qmax, qmax)  # [G, d]
+            err = ((w[None, :].astype(np.float64) - s[:, None].astype(np.float64) * q) ** 2).sum(1)
+            g = int(np.argmin(err))
+            assert out["scales"][k, 0] == s[g]
+            np.testing.assert_array_equal(out["codes"][0, k], q[g].astype(np.int8))
+
+
+def test_residual_norm_non_increasing_and_strict(oracle):
+    """Eq. 7 with the scale search of Eq. 9: ||r_{i+1}|| <= ||r_i||, strictly while r_i != 0
+    (at the largest grid scale the largest element is represented, so some candidate improves)."""
+    for dist in ("normal", "laplace", "t"):
+        W = wlm.random_weights(32, 200, 11, dist)
+        out = oracle.quantize_layer(W, 4, 64, 8)
+        rs = out["resid_sq"]
+        step = np.diff(rs, axis=1)
+        assert np.all(step <= 0)
+        assert np.all((step < 0) | (rs[:, :-1] == 0))
+
+
+def test_exponential_decay_theorem1(oracle):
+    """Theorem 1 (b = 2, fine grid): ||r_i||^2 decays geometrically; every step removes at least a
+    fixed fraction of the residual energy for the first steps."""
+    W = wlm.random_weights(8, 32, 5, "normal")
+    out = oracle.quantize_layer(W, 2, 4096, 10)
+    ratios = out["resid_sq"][:, 1:] / out["resid_sq"][:, :-1]
+    assert np.all(ratios < 0.9)
+    # log-linear: after 10 points the energy is down by orders of magnitude
+    assert np.all(out["resid_sq"][:, -1] < 1e-3 * out["resid_sq"][:, 0])
+
+
+def test_scale_equivariance(oracle):
+    """The method is scale-equivariant: w -> 2^k w multiplies every scale by 2^k and leaves every
+    code unchanged, bit for bit (all fp32 operations commute with exact power-of-two scaling)."""
+    W = wlm.random_weights(16, 150, 3, "t")
+    base = oracle.quantize_layer(W, 4, 128, 6)
+    for k in (-20, -3, 5, 30):
+        out = oracle.quantize_layer(np.ldexp(W, k).astype(np.float32), 4, 128, 6)
+        np.testing.assert_array_equal(out["codes"], base["codes"])
+        np.testing.assert_array_equal(out["scales"], np.ldexp(base["scales"], k).astype(np.float32))
+
+
+def test_exactly_representable_channel(oracle):
+    """If w = s0 * q0 with integer q0 and max|q0| = Qmax, the largest grid scale reproduces w
+    exactly: the first point is exact and every later point is a null point."""
+    rng = np.random.default_rng(0)
+    q0 = rng.integers(-7, 8, size=(4, 33))
+    q0[:, 0] = 7
+    W = (q0 * 0.125).astype(np.float32)
+    out = oracle.quantize_layer(W, 4, 64, 3)
+    np.testing.assert_array_equal(out["codes"][0], q0.astype(np.int8))
+    np.testing.assert_array_equal(out["scales"][:, 0], np.float32(0.125))
+    assert np.all(out["gstar"][:, 0] == 63)
+    assert np.all(out["resid_sq"][:, 1:] == 0)
+    assert np.all(out["scales"][:, 1:] == 0) and np.all(out["codes"][1:] == 0)
+
+
+def test_zero_and_nonfinite_channels(oracle):
+    """Readings for degenerate channels: an all-zero channel gives null points; a channel with a
+    NaN/Inf weight gives NaN scales and zero codes."""
+    W = np.zeros((3, 5), np.float32)
+    W[1] = [1, 2, 3, 4, 5]
+    W[2, 3] = np.nan
+    out = oracle.quantize_layer(W, 4, 8, 2)
+    assert np.all(out["scales"][0] == 0) and np.all(out["codes"][:, 0] == 0)
+    assert np.all(out["resid_sq"][0] == 0)
+    assert np.all(np.isnan(out["scales"][2])) and np.all(out["codes"][:, 2] == 0)
+    assert out["scales"][1, 0] > 0
+
+
+def test_user_grid(oracle):
+    """A caller-supplied grid of fractions replaces f_g = g/G: the chosen scale is one of them."""
+    W = wlm.random_weights(10, 64, 21, "normal")
+    gf = np.array([0.3, 0.5, 0.55, 0.7, 0.9, 1.0], np.float32)
+    out = oracle.quantize_layer(W, 4, gf.size, 2, grid_frac=gf)
+    for k in range(10):
+        s = _grid(np.abs(W[k]).max(), 7, gf.size, gf)
+        assert out["scales"][k, 0] in s
+
+
+# --- Eq. 4: reconstruction ----------------------------------------------------------------------
+
+def test_reconstruct_matches_exact_sum(oracle):
+    """Eq. 4: w~(n) = sum_i s_i q_i; the fmaf chain is within n half-ulps of the exact rational
+    sum, and w - w~(n) equals the residual r_{n+1} up to the same rounding."""
+    W = wlm.random_weights(6, 40, 9, "normal")
+    K = 4
+    out = oracle.quantize_layer(W, 4, 64, K)
+    for n in range(K + 1):
+        npts = np.full(6, n, np.int32)
+        What = oracle.reconstruct(out["codes"], out["scales"], npts)
+        for k in range(6):
+            for j in range(0, 40, 7):
+                exact = sum(Fraction(float(out["scales"][k, i])) * int(out["codes"][i, k, j])
+                            for i in range(n))
+                got = Fraction(float(What[k, j]))
+                ulp = float(np.spacing(np.abs(W[k]).max().astype(np.float32)))  # fp32 ulp
+                assert abs(float(got - exact)) <= max(n, 1) * ulp
+                if n > 0:
+                    resid = Fraction(float(out["residuals"][n - 1, k, j]))
+                    assert abs(float(Fraction(float(W[k, j])) - exact - resid)) <= n * ulp
+
+
+# --- Eq. 11: output error -----------------------------------------------------------------------
+
+def _quantized(oracle, C=6, d=64, K=3, seed=4):
+    W = wlm.random_weights(C, d, seed, "normal")
+    return W, oracle.quantize_layer(W, 4, 32, K)
+
+
+def test_output_error_identity_input(oracle):
+    """Eq. 11 with X = sqrt(N) I (N = d = 64): e(n) = ||r_{n+1}||^2 = resid_sq."""
+    W, q = _quantized(oracle)
+    X = (np.eye(64) * 8.0).astype(np.float32)
+    err = oracle.output_error(X, 1, W, q["codes"], q["scales"], 3)
+    np.testing.assert_allclose(err, q["resid_sq"], rtol=1e-13)
+
+
+def test_output_error_single_column(oracle):
+    """Eq. 11 with one nonzero input column j0 of value c: e(n) = c^2 r_{n+1,j0}^2."""
+    W, q = _quantized(oracle)
+    j0, c = 17, 3.0
+    X = np.zeros((10, 64), np.float32)
+    X[:, j0] = c
+    err = oracle.output_error(X, 1, W, q["codes"], q["scales"], 3)
+    R = np.concatenate([W[None], q["residuals"]], 0)   # [K+1][C][d]
+    expect = (c * R[:, :, j0].astype(np.float64)) ** 2
+    np.testing.assert_allclose(err, expect.T, rtol=1e-13)
+
+
+def test_output_error_matches_library_matmul(oracle):
+    """Eq. 11 against a double-precision library matmul of X with the residuals."""
+    W, q = _quantized(oracle, C=5, d=70, K=4, seed=8)
+    X = wlm.random_calibration(33, 70, 2)
+    err = oracle.output_error(X, 1, W, q["codes"], q["scales"], 4)
+    R = np.concatenate([W[None], q["residuals"]], 0).astype(np.float64)  # [K+1][C][d]
+    Y = np.einsum("td,ncd->nct", X.astype(np.float64), R)
+    np.testing.assert_allclose(err, (Y ** 2).mean(-1).T, rtol=1e-12)
+
+
+def test_output_error_depthwise_blocks(oracle):
+    """groups = C: channel k reads its own N x d input block (depthwise convolution)."""
+    W, q = _quantized(oracle, C=4, d=9, K=3, seed=12)
+    X = wlm.random_calibration(20, 9, 3, groups=4)
+    err = oracle.output_error(X, 4, W, q["codes"], q["scales"], 3)
+    R = np.concatenate([W[None], q["residuals"]], 0).astype(np.float64)
+    for k in range(4):
+        Y = X[k].astype(np.float64) @ R[:, k, :].T     # [N][K+1]
+        np.testing.assert_allclose(err[k], (Y ** 2).mean(0), rtol=1e-12)
+
+
+# --- Algorithm 2: point allocation --------------------------------------------------------------
+
+def test_allocation_hand_example(oracle):
+    ex = json.load(open(os.path.join(GOLDEN, "allocation_hand_example.json")))
+    err = np.array(ex["err"], np.float32)
+    for case in ex["budget_cases"]:
+        n, used = oracle.allocate_budget(err, ex["k_max"], case["beta"])
+        assert n.tolist() == case["npoints"], case["why"]
+        assert used == case["used"]
+    for case in ex["threshold_cases"]:
+        n, used = oracle.allocate_threshold(err, ex["k_max"], case["eps"])
+        assert n.tolist() == case["npoints"], case["why"]
+        assert used == case["used"]
+
+
+def test_allocation_budget_extremes(oracle):
+    """beta = 1 gives one point everywhere; beta = k_max with positive gains gives k_max."""
+    rng = np.random.default_rng(3)
+    C, K = 50, 5
+    err = np.sort(rng.random((C, K + 1)), axis=1)[:, ::-1].astype(np.float32) + 1
+    n, used = oracle.allocate_budget(err, K, 1.0)
+    assert np.all(n == 1) and used == C
+    n, used = oracle.allocate_budget(err, K, float(K))
+    assert np.all(n == K) and used == C * K
+
+
+def test_allocation_greedy_is_optimal_for_concave_gains(oracle):
+    """With diminishing returns (decreasing gains per channel) the marginal-gain loop maximises
+    the total output-error reduction for its budget: exhaustive check on small tables."""
+    rng = np.random.default_rng(5)
+    for trial in range(20):
+        C, K = 3, 4
+        gains = np.sort(rng.integers(1, 50, size=(C, K - 1)), axis=1)[:, ::-1]   # decreasing
+        e1 = rng.integers(200, 300, size=(C, 1))
+        err = np.concatenate([e1 + 100, e1 - np.concatenate(
+            [np.zeros((C, 1), int), np.cumsum(gains, 1)], 1)], 1).astype(np.float32)
+        for extra in range(0, C * (K - 1) + 1):
+            beta = (C + extra) / C
+            n, used = oracle.allocate_budget(err, K, beta)
+            best = max(sum(err[k, 1] - err[k, a[k]] for k in range(C))
+                       for a in itertools.product(range(1, K + 1), repeat=C)
+                       if sum(a) == C + extra)
+            got = sum(err[k, 1] - err[k, n[k]] for k in range(C))
+            assert used == C + extra
+            assert got == best
+
+
+def test_allocation_stops_at_nonpositive_gain(oracle):
+    err = np.array([[5, 4, 4.5, 1], [5, 3, 3, 3]], np.float32)
+    n, used = oracle.allocate_budget(err, 3, 3.0)
+    # ch0 head gain 4-4.5 < 0, ch1 head gain 0: nothing is worth adding
+    assert n.tolist() == [1, 1] and used == 2
+
+
+# --- Table 1: overhead closed forms -------------------------------------------------------------
+
+def test_table1_overhead_closed_forms():
+    """Table 1: naive vs multipoint memory / MULs / ADDs; n = 1 reduces to naive plus the
+    32-bit coefficient."""
+    from paper_2002_09049_gb300 import overhead
+    d, Nb = 576, 4
+    naive = overhead.naive_cost(d, Nb)
+    assert naive == dict(memory_bits=d * Nb, muls=d * Nb * Nb, adds=(d - 1) * Nb)
+    mp = overhead.multipoint_cost(d, Nb, 3)
+    assert mp == dict(memory_bits=3 * d * Nb + 96, muls=3 * (d * Nb * Nb + 1024),
+                      adds=3 * (d - 1) * Nb + 64)
+    one = overhead.multipoint_cost(d, Nb, 1)
+    assert one["memory_bits"] - naive["memory_bits"] == 32 and one["adds"] == naive["adds"]
