@@ -1,0 +1,456 @@
+#!/usr/bin/env python3
+"""Throughput of the multipoint-quantization hot path on GB300.
+
+One step = every layer of the workload through the whole path: greedy points (mpq_quantize_layer),
+output error (mpq_output_error), point allocation (mpq_allocate_points, budget mode) and
+multipoint weights (mpq_reconstruct).  Metric: weight-elements x scale-candidates x points per
+second, i.e. sum over layers of C*d*G*k_max per step / step time.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config c2] [--impl ours|reference]
+
+Prints ONE JSON line on rank 0.  Multi-GPU (torchrun): every rank quantizes its own copy of the
+workload (independent problems, no collective on the data path; weak scaling); value = units of
+all ranks / max-over-ranks time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "weight-elements x scale-candidates x points / s"
+UNIT = "elem*cand*pt/s"
+PROFILES = os.path.join(ROOT, "profiles")
+KERNEL_SOURCES = {
+    "output_error": "paper_2002_09049_gb300/csrc/output_error.cu",
+    "quantize": "paper_2002_09049_gb300/csrc/quantize.cu",
+    "allocate": "paper_2002_09049_gb300/csrc/allocate.cu",
+    "reconstruct": "paper_2002_09049_gb300/csrc/reconstruct.cu",
+}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default="c2", choices=["c1", "c2", "c3", "c4", "c5"])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="target CPU time of the oracle baseline sample")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------------------------------------
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def src_hash(rel):
+    with open(os.path.join(ROOT, rel), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "sm_max_mhz": 2070.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.15)
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------------
+def layer_inputs(wl, li):
+    from paper_2002_09049_gb300 import workloads as wlm
+    return wlm.make_weights(wl, li), wlm.make_calibration(wl, li)
+
+
+def kernel_units(wl, layer):
+    return layer.C * layer.d * wl.G * wl.k_max
+
+
+def contraction_flops(wl, layer):
+    """Algorithmic flops of Eq. 11 for one layer: 2 * N * d * C * (k_max + 1)."""
+    return 2 * wl.n_calib * layer.d * layer.C * (wl.k_max + 1)
+
+
+def run_ours(args, world, rank, local):
+    import torch
+    from paper_2002_09049_gb300 import _build, binding, pipeline, workloads as wlm
+
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0 or world == 1:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    binding.load()
+
+    wl = wlm.WORKLOADS[args.config]
+    bits = wl.bits[0]
+    runs = []  # (spec, plan, W_dev, X_dev, W_host, X_host, layer)
+    for li, layer in enumerate(wl.layers):
+        W, X = layer_inputs(wl, li)
+        spec = pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, groups=layer.groups,
+                                  bits=bits, G=wl.G, k_max=wl.k_max, budget_or_eps=wl.beta)
+        plan = pipeline.LayerPlan(spec, dev)
+        Wh = torch.from_numpy(W).pin_memory()
+        Xh = torch.from_numpy(X).pin_memory()
+        runs.append((spec, plan, Wh.to(dev), Xh.to(dev), Wh, Xh, layer))
+    units_per_step = sum(kernel_units(wl, r[6]) for r in runs) * len(wl.bits)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 512 MB > L2
+    stream = torch.cuda.current_stream()
+
+    families = ["quantize", "output_error", "allocate", "reconstruct"]
+
+    def step(record=None):
+        for b in wl.bits:
+            for spec, plan, Wd, Xd, _, _, layer in runs:
+                spec.bits = b
+                s = plan.spec
+                ev = record is not None
+                if ev:
+                    e = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+                    e[0].record(stream)
+                binding.mpq_quantize_layer(Wd, s.bits, s.G, s.k_max, codes=plan.codes,
+                                           scales=plan.scales, resid_sq=plan.resid_sq)
+                if ev:
+                    e[1].record(stream)
+                binding.mpq_output_error(Xd, Wd, plan.codes, plan.scales, s.k_max,
+                                         groups=s.groups, err=plan.err)
+                if ev:
+                    e[2].record(stream)
+                binding.mpq_allocate_points(plan.err, s.k_max, s.mode, s.budget_or_eps,
+                                            npoints=plan.npoints, points_used=plan.points_used)
+                if ev:
+                    e[3].record(stream)
+                binding.mpq_reconstruct(plan.codes, plan.scales, plan.npoints, W_hat=plan.W_hat)
+                if ev:
+                    e[4].record(stream)
+                    record.append((layer, e))
+
+    launches_per_step = 4 * len(runs) * len(wl.bits)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    peaks, peak_src = measured_peaks()
+    step_ms = []
+    recs = []
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for _ in range(args.steps):
+            flush.fill_(1.0)                    # evict L2 between steps (outside the timing)
+            a = torch.cuda.Event(enable_timing=True)
+            z = torch.cuda.Event(enable_timing=True)
+            rec = []
+            a.record(stream)
+            step(rec)
+            z.record(stream)
+            recs.append(rec)
+            torch.cuda.synchronize()
+            step_ms.append(a.elapsed_time(z))
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    ms = float(np.mean(step_ms))
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    value = units_per_step * world / (ms / 1e3)
+
+    # per-kernel-family device time from the events around each call
+    fam_ms = {f: 0.0 for f in families}
+    fam_work = {"output_error": 0.0, "quantize": 0.0, "reconstruct": 0.0, "allocate": 0.0}
+    for rec in recs:
+        for layer, e in rec:
+            for i, f in enumerate(families):
+                fam_ms[f] += e[i].elapsed_time(e[i + 1])
+            fam_work["output_error"] += contraction_flops(wl, layer)
+            fam_work["quantize"] += kernel_units(wl, layer)
+            fam_work["reconstruct"] += layer.C * layer.d * (4 + 1 + 4 / wl.k_max)  # bytes, approx
+    total_fam = sum(fam_ms.values())
+    dominant = max(fam_ms, key=fam_ms.get)
+
+    roofline = dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args)
+    roofline["share"] = fam_ms[dominant] / total_fam if total_fam else None
+    roofline["family_ms_per_step"] = {f: fam_ms[f] / args.steps for f in families}
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": f"{args.config}: {wl.title}", "layers": len(wl.layers),
+                   "weights": wl.n_weights, "channels": wl.n_channels, "bits": list(wl.bits),
+                   "G": wl.G, "k_max": wl.k_max, "budget": wl.beta, "calib_rows": wl.n_calib,
+                   "units_per_step": units_per_step, "l2": "flushed between steps (512 MB write)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roofline,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk.summary(),
+    }
+
+    if not args.no_e2e:
+        out["e2e"] = run_e2e(runs, wl, args, stream, world, units_per_step)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    return out if rank == 0 else None
+
+
+def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
+    traffic = None
+    tfile = os.path.join(PROFILES, "roofline_traffic.json")
+    if os.path.exists(tfile):
+        with open(tfile) as f:
+            tr = json.load(f)
+        ent = tr.get(args.config, {}).get(dominant)
+        if ent and ent.get("source_sha") == src_hash(KERNEL_SOURCES[dominant]):
+            traffic = ent.get("dram_bytes_per_step")
+    t_s = fam_ms[dominant] / 1e3
+    if dominant == "output_error":
+        # fp32 CUDA-core contraction: peak = 2 flops x 128 FFMA lanes x SMs x max SM clock
+        import torch
+        sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+        peak = 2 * 128 * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        ach = fam_work[dominant] / t_s / 1e12
+        return {"kernel": "output_error (Eq. 11 contraction, fp32 FFMA)", "bound": "alu",
+                "achieved": ach, "peak": peak, "unit": "TFLOP/s", "frac": ach / peak,
+                "traffic": traffic, "peak_source": f"derived: 2*128*{sms} SMs*max SM clock "
+                                                   f"({peak_src} clock)"}
+    if dominant == "quantize":
+        import torch
+        sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+        ops_per_unit = 8  # minimal fp32/int ops per (element, candidate) of the direct search
+        peak = 128 * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        ach = fam_work[dominant] * ops_per_unit / t_s / 1e12
+        return {"kernel": "quantize (Eq. 9 scale search)", "bound": "alu", "achieved": ach,
+                "peak": peak, "unit": "Tops/s", "frac": ach / peak, "traffic": traffic,
+                "peak_source": f"derived: 128 lanes*{sms} SMs*max SM clock ({peak_src} clock)"}
+    hbm = peaks["hbm_gbs"]
+    ach = fam_work.get(dominant, 0.0) / t_s / 1e9
+    return {"kernel": dominant, "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+            "frac": ach / hbm, "traffic": traffic, "peak_source": peak_src}
+
+
+def run_e2e(runs, wl, args, stream, world, units_per_step):
+    """Same metric through the public per-layer call with host buffers: H2D of W and X from
+    pinned memory, the path, D2H of codes / scales / point counts -- all inside the timing."""
+    import torch
+    h2d = sum(r[4].numel() * 4 + r[5].numel() * 4 for r in runs) * len(wl.bits)
+    d2h = sum(r[1].d2h_bytes() for r in runs) * len(wl.bits)
+
+    def step():
+        for b in wl.bits:
+            for spec, plan, Wd, Xd, Wh, Xh, _ in runs:
+                spec.bits = b
+                plan.run_host(Wh, Xh, Wd, Xd, stream=stream)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(args.steps):
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        z = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        step()
+        z.record(stream)
+        z.synchronize()
+        times.append(a.elapsed_time(z))
+    ms = float(np.mean(times))
+    return {"value": units_per_step / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+
+# ------------------------------------------------------------------------------------------------
+def oracle_sample(wl, target_s):
+    """A bounded, proportional sample of the workload for the CPU oracle: every layer keeps the
+    channels k = 0, stride, 2*stride, ...  Returns (sample list, stride)."""
+    total_ch = wl.n_channels
+    # rough oracle cost per channel (s, single core): quantize d*G*k_max*6ns + error d*N*(k+1)*1ns
+    est = sum(l.C * (l.d * wl.G * wl.k_max * 6e-9 + l.d * wl.n_calib * (wl.k_max + 1) * 1.2e-9)
+              for l in wl.layers) * len(wl.bits)
+    cores = host_cores()
+    stride = max(1, int(np.ceil(est / cores / target_s)))
+    return stride
+
+
+def run_oracle_step(wl, stride, threads, inputs):
+    """The oracle over the sampled channels of every layer: Algorithm 1, Eq. 11, Algorithm 2
+    (budget, per layer, on the sample), Eq. 4.  Returns the metric units processed."""
+    import oracle
+    units = 0
+    for b in wl.bits:
+        for li, layer in enumerate(wl.layers):
+            W, X = inputs[li]
+            q = oracle.quantize_layer(W, b, wl.G, wl.k_max, want_residuals=False, threads=threads)
+            groups = W.shape[0] if layer.groups > 1 else 1
+            err = oracle.output_error(X, groups, W, q["codes"], q["scales"], wl.k_max,
+                                      threads=threads)
+            n, _ = oracle.allocate_budget(err.astype(np.float32), wl.k_max, wl.beta)
+            oracle.reconstruct(q["codes"], q["scales"], n)
+            units += W.shape[0] * layer.d * wl.G * wl.k_max
+    return units
+
+
+def sample_inputs(wl, stride):
+    from paper_2002_09049_gb300 import workloads as wlm
+    inputs = []
+    for li, layer in enumerate(wl.layers):
+        W, X = layer_inputs(wl, li)
+        sel = np.arange(0, layer.C, stride)
+        Ws = np.ascontiguousarray(W[sel])
+        Xs = np.ascontiguousarray(X[sel]) if layer.groups > 1 else X
+        inputs.append((Ws, Xs))
+    return inputs
+
+
+def cpu_baseline(wl, target_s):
+    import oracle
+    oracle.build()
+    stride = oracle_sample(wl, target_s)
+    threads = host_cores()
+    inputs = sample_inputs(wl, stride)
+    t0 = time.perf_counter()
+    units = run_oracle_step(wl, stride, threads, inputs)
+    dt = time.perf_counter() - t0
+    return {"value": units / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "seconds": dt,
+            "sample": f"every {stride}th channel of every layer of the same workload "
+                      f"({units:.3e} units), oracle threads over channels"}
+
+
+def run_reference(args, world, rank):
+    """The oracle as the reference arm, on the host cores; rank 0 only."""
+    if rank != 0:
+        return None
+    import oracle
+    from paper_2002_09049_gb300 import workloads as wlm
+    oracle.build()
+    wl = wlm.WORKLOADS[args.config]
+    per_step = max(2.0, 150.0 / max(1, args.steps + args.warmup))
+    stride = oracle_sample(wl, per_step)
+    threads = host_cores()
+    inputs = sample_inputs(wl, stride)
+    for _ in range(args.warmup):
+        run_oracle_step(wl, stride, threads, inputs)
+    times, units = [], 0
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        units = run_oracle_step(wl, stride, threads, inputs)
+        times.append(time.perf_counter() - t0)
+    s = float(np.mean(times))
+    value = units / s
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": f"{args.config}: {wl.title}", "bits": list(wl.bits), "G": wl.G,
+                       "k_max": wl.k_max, "budget": wl.beta},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"every {stride}th channel of every layer per step"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        out = run_reference(args, world, rank)
+    else:
+        out = run_ours(args, world, rank, local)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

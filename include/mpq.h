@@ -1,0 +1,154 @@
+/*
+ * mpq.h -- C ABI of the GB300 multipoint post-training quantization library (libmpq.so).
+ *
+ * Method: Liu et al., "Post-training Quantization with Multiple Points: Mixed Precision without
+ * Mixed Precision" (arXiv 2002.09049).  A weight channel w (d values) is approximated by
+ * n points, w~ = sum_i a_i w~_i (Eq. 4), built greedily one point at a time from the residual
+ * (Eq. 6-9, Algorithm 1); the number of points of each channel is chosen from its output error on
+ * calibration inputs (Eq. 11, Algorithm 2).
+ *
+ * Representation.  A point i of channel k is a pair (s_{k,i}, q_{k,i}): an fp32 scale and a
+ * vector of d integer codes in {-Qmax..Qmax}, Qmax = 2^(b-1) - 1, stored as int8.  The paper's
+ * a_i * [r/a_i]_Q with Q = [-1 : 1/Qmax : 1] (Eq. 1) is s_i * q_i with s_i = a_i / Qmax.
+ *
+ * Conventions shared by every entry point:
+ *  - All array arguments are DEVICE pointers, allocated and owned by the caller, row-major,
+ *    on the device that is current when the call is made, unless an argument says "host".
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Every call
+ *    only enqueues work on `stream` and returns; results are ready when the stream reaches them.
+ *    No entry point allocates device memory or synchronizes.
+ *  - Arguments are validated on the host before anything is enqueued; an invalid argument
+ *    returns MPQ_ERR_INVALID_ARG / MPQ_ERR_UNSUPPORTED and leaves every output untouched.
+ *    A failed kernel launch returns MPQ_ERR_CUDA.  mpq_last_error() gives a message for the
+ *    most recent failure on the calling thread.  No C++ exception crosses this boundary.
+ *  - Outputs must not alias inputs.  C = 0 is a valid empty call that enqueues nothing.
+ *  - Non-finite data cannot be checked on the host without a synchronization, so it is handled
+ *    on the device, visibly: a channel with a NaN/Inf weight gets NaN scales and zero codes, and
+ *    NaN propagates into its output errors; the allocator treats a NaN gain as "no gain".
+ */
+#ifndef MPQ_H
+#define MPQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MPQ_OK = 0,
+    MPQ_ERR_INVALID_ARG = 1,  /* a size, pointer or parameter is out of its documented range */
+    MPQ_ERR_NONFINITE = 2,    /* a host-side numeric parameter is NaN/Inf */
+    MPQ_ERR_UNSUPPORTED = 3,  /* valid for the method but beyond this library's limits below */
+    MPQ_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
+    MPQ_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up (reserved) */
+    MPQ_ERR_NOMEM = 6         /* reserved: no entry point allocates */
+} mpq_status;
+
+/* Library limits. */
+#define MPQ_MIN_BITS 2        /* b = 2 gives Q = {-1, 0, 1}, the smallest set of Eq. 1 */
+#define MPQ_MAX_BITS 8        /* codes are stored as int8 */
+#define MPQ_MAX_POINTS 16     /* k_max */
+#define MPQ_MAX_GRID 1024     /* G, candidate scales per greedy step */
+#define MPQ_MAX_DIM 8192      /* d for mpq_quantize_layer: one channel's residual lives on chip */
+
+/* Allocation modes of mpq_allocate_points. */
+#define MPQ_ALLOC_BUDGET 0
+#define MPQ_ALLOC_THRESHOLD 1
+
+/*
+ * mpq_quantize_layer -- greedy multipoint construction (Sec. 3.2, Eq. 6-9, Algorithm 1) for every
+ * channel of one layer, run to k_max points.
+ *
+ * For each channel k and step i = 1..k_max, with residual r (r_1 = w_k, Eq. 7):
+ *   m = max_j |r_j|; smax = m / Qmax (fp32 division);
+ *   candidate scales s_g = f_g * smax (fp32), g = 1..G, where f_g = g/G (fp32 division) when
+ *     grid_frac is NULL, else f_g = grid_frac[g-1];
+ *   codes of candidate g: q_j = clamp(rint(r_j / s_g), -Qmax, Qmax) (Eq. 8; fp32 division,
+ *     ties of rint to even);
+ *   the chosen candidate minimises ||r - s_g q||^2 (Eq. 9), the lowest g on ties;
+ *   r <- fmaf(-s*, q*, r) elementwise (Eq. 7).
+ * A residual that is exactly zero yields a null point (scale 0, codes 0).
+ *
+ *   W          [C][d] fp32, the layer's weights, one output channel per row.
+ *   C, d       channels and weights per channel; 1 <= d <= MPQ_MAX_DIM.
+ *   bits       b in [MPQ_MIN_BITS, MPQ_MAX_BITS]; Qmax = 2^(b-1) - 1.
+ *   G          candidate scales per step, 1..MPQ_MAX_GRID.
+ *   grid_frac  HOST array of G fp32 fractions, strictly increasing, in (0, 1]; or NULL for the
+ *              linear grid g/G.  Copied into the launch; the caller may free it on return.
+ *   k_max      points per channel, 1..MPQ_MAX_POINTS.
+ *   codes      out [k_max][C][d] int8: codes[i][k][:] = q_{k,i+1}.
+ *   scales     out [C][k_max] fp32: scales[k][i] = s_{k,i+1}.
+ *   resid_sq   out [C][k_max+1] fp32, nullable: ||r_{k,n+1}||^2 for n = 0..k_max points
+ *              (n = 0 is ||w_k||^2).
+ *   residuals  out [k_max][C][d] fp32, nullable: residuals[i][k][:] = r_{k,i+2}.
+ */
+mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
+                              const float *grid_frac, int k_max, int8_t *codes, float *scales,
+                              float *resid_sq, float *residuals, void *stream);
+
+/*
+ * mpq_output_error -- output error of every channel for every point count (Sec. 3.3, Eq. 11):
+ *   err[k][n] = (1/N) sum_{t=1..N} (x_t . (w_k - w~_k(n)))^2,  n = 0..k_max,
+ * where w_k - w~_k(n) is the residual r_{k,n+1} regenerated from W, codes and scales by the
+ * recursion of Eq. 7 (r_{k,1} = w_k, r_{k,i+1} = fmaf(-s_{k,i}, q_{k,i}, r_{k,i})).
+ *
+ *   X       calibration inputs D_L.  groups == 1: [N][d], shared by all channels.
+ *           groups == C: [C][N][d], channel k uses its own block (depthwise convolution, where
+ *           each output channel sees only its own input patches).
+ *   N       calibration rows, >= 1.
+ *   groups  1 or C.
+ *   W, codes, scales, C, d, k_max   as produced by / passed to mpq_quantize_layer.
+ *   err     out [C][k_max+1] fp32.
+ */
+mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
+                            const int8_t *codes, const float *scales, int C, int d, int k_max,
+                            float *err, void *stream);
+
+/*
+ * mpq_allocate_points -- per-channel point counts from the output-error table (Sec. 3.3,
+ * Algorithm 2).
+ *
+ * mode MPQ_ALLOC_THRESHOLD (Algorithm 2 as printed): npoints[k] = the smallest n in 1..k_max with
+ *   err[k][n] < eps (compared in double), else k_max.  budget_or_eps = eps (not NaN).
+ * mode MPQ_ALLOC_BUDGET: a total of P = floor(beta*C + 0.5) points (beta = budget_or_eps, finite,
+ *   >= 0).  Every channel starts with one point; the P - C extra points (clamped to
+ *   [0, C*(k_max-1)]) go one at a time to the channel whose next point lowers its output error
+ *   most: gain_k = err[k][n_k] - err[k][n_k+1] (fp32 subtraction; NaN counts as no gain), lowest k
+ *   on ties, stopping early when the best remaining gain is <= 0.  Computed in one device-wide
+ *   selection that gives exactly the result of that sequential loop.
+ *
+ *   err          [C][k_max+1] fp32 (from mpq_output_error).
+ *   npoints      out [C] int32.
+ *   points_used  out, nullable: one device int32, the total sum_k npoints[k].
+ */
+mpq_status mpq_allocate_points(const float *err, int C, int k_max, int mode, double budget_or_eps,
+                               int *npoints, int *points_used, void *stream);
+
+/*
+ * mpq_reconstruct -- multipoint weights (Eq. 4): W_hat[k][j] = sum_{i=1..n_k} s_{k,i} q_{k,i,j},
+ * accumulated as acc = fmaf(s_{k,i}, q_{k,i,j}, acc) from acc = 0 in the order i = 1, 2, ...
+ * n_k = npoints[k] clamped to [0, k_max] (npoints lives on the device and is not checked on the
+ * host).
+ *
+ *   codes [k_max][C][d] int8, scales [C][k_max] fp32, npoints [C] int32.
+ *   W_hat out [C][d] fp32.
+ */
+mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C,
+                           int d, int k_max, float *W_hat, void *stream);
+
+/* Name of a status code (static string). */
+const char *mpq_status_string(mpq_status s);
+
+/* Message describing the most recent failure on the calling thread ("" if none). */
+const char *mpq_last_error(void);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int mpq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MPQ_H */

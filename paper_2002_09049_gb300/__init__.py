@@ -1,17 +1,11 @@
 """GB300-native multipoint post-training quantization (arXiv 2002.09049).
 
 The compute path lives in the C-ABI library ``libmpq.so`` (hand-written CUDA for sm_103a, built
-from ``csrc/``); ``binding`` marshals torch tensors into its entry points.  There is no CPU
-fallback: calling an entry point without the compiled library raises.
+from ``csrc/``); ``binding`` marshals torch tensors into its entry points and loads the library
+on first use.  There is no CPU fallback: calling an entry point without the compiled library
+raises.
 """
-from . import workloads, overhead  # noqa: F401
-
-__all__ = ["workloads", "overhead"]
-
-
-def __getattr__(name):
-    # the binding loads the CUDA library lazily, on first use
-    if name in ("binding",) or name.startswith("mpq_"):
-        from . import binding
-        return binding if name == "binding" else getattr(binding, name)
-    raise AttributeError(name)
+from . import overhead, workloads  # noqa: F401
+from .binding import (MPQ_ALLOC_BUDGET, MPQ_ALLOC_THRESHOLD, MPQError,  # noqa: F401
+                      mpq_allocate_points, mpq_output_error, mpq_quantize_layer, mpq_reconstruct,
+                      mpq_status_string, mpq_version)

@@ -1,0 +1,196 @@
+"""Thin Python binding of libmpq.so (include/mpq.h): torch tensors in, C-ABI calls out.
+
+Every function here only checks tensor placement/shape/dtype, allocates outputs with torch when
+the caller did not pass them, and forwards raw device pointers plus the current CUDA stream to the
+library.  All arithmetic happens in the library's CUDA kernels; there is no CPU fallback -- if the
+library is missing or fails to load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import _build
+
+MPQ_ALLOC_BUDGET = 0
+MPQ_ALLOC_THRESHOLD = 1
+
+MPQ_STATUS = {0: "MPQ_OK", 1: "MPQ_ERR_INVALID_ARG", 2: "MPQ_ERR_NONFINITE",
+              3: "MPQ_ERR_UNSUPPORTED", 4: "MPQ_ERR_CUDA", 5: "MPQ_ERR_TIMEOUT",
+              6: "MPQ_ERR_NOMEM"}
+
+# name -> (argtypes, restype), in the order of include/mpq.h
+_P, _I, _D = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+SIGNATURES = {
+    "mpq_quantize_layer": ([_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P], _I),
+    "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
+    "mpq_reconstruct": ([_P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "mpq_status_string": ([_I], ctypes.c_char_p),
+    "mpq_last_error": ([], ctypes.c_char_p),
+    "mpq_version": ([], _I),
+}
+
+_lib = None
+
+
+class MPQError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        self.status = status
+        super().__init__(f"{where}: {MPQ_STATUS.get(status, status)}: {detail}")
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load(path: str | None = None):
+    """Loads libmpq.so (built by __graft_entry__.build() / paper_2002_09049_gb300._build)."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or _build.LIB
+    if not os.path.exists(p):
+        raise RuntimeError(f"{p} is missing: build it with paper_2002_09049_gb300._build.build() "
+                           "(there is no CPU fallback)")
+    lib = ctypes.CDLL(p)
+    for name, (argt, rest) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.argtypes = argt
+        fn.restype = rest
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        detail = load().mpq_last_error().decode(errors="replace")
+        raise MPQError(status, where, detail)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t, name, dtype, shape=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    return t
+
+
+def mpq_quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, codes=None,
+                       scales=None, resid_sq=None, residuals=None, want_resid_sq=True,
+                       stream=None):
+    """Greedy multipoint construction (Algorithm 1) of every channel of W [C][d] fp32.
+
+    Returns (codes [k_max][C][d] int8, scales [C][k_max] fp32, resid_sq [C][k_max+1] or None,
+    residuals or None).  grid_frac: optional host sequence of G fractions in (0, 1]."""
+    _dev(W, "W", torch.float32)
+    C, d = W.shape
+    dev = W.device
+    codes = codes if codes is not None else torch.empty((k_max, C, d), dtype=torch.int8, device=dev)
+    scales = scales if scales is not None else torch.empty((C, k_max), dtype=torch.float32,
+                                                           device=dev)
+    if resid_sq is None and want_resid_sq:
+        resid_sq = torch.empty((C, k_max + 1), dtype=torch.float32, device=dev)
+    _dev(codes, "codes", torch.int8, (k_max, C, d))
+    _dev(scales, "scales", torch.float32, (C, k_max))
+    if resid_sq is not None:
+        _dev(resid_sq, "resid_sq", torch.float32, (C, k_max + 1))
+    if residuals is not None:
+        _dev(residuals, "residuals", torch.float32, (k_max, C, d))
+    gf = None
+    if grid_frac is not None:
+        gf_list = [float(x) for x in grid_frac]
+        if len(gf_list) != G:
+            raise ValueError("grid_frac must have G entries")
+        gf = (ctypes.c_float * G)(*gf_list)
+    st = load().mpq_quantize_layer(_ptr(W), C, d, bits, G, gf, k_max, _ptr(codes), _ptr(scales),
+                                   _ptr(resid_sq), _ptr(residuals), _stream(stream))
+    _check(st, "mpq_quantize_layer")
+    return codes, scales, resid_sq, residuals
+
+
+def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None, stream=None):
+    """Output error (Eq. 11) for n = 0..k_max points: err [C][k_max+1] fp32."""
+    _dev(W, "W", torch.float32)
+    C, d = W.shape
+    _dev(X, "X", torch.float32)
+    if groups == 1:
+        if X.dim() != 2 or X.shape[1] != d:
+            raise ValueError("X must be [N][d] for groups = 1")
+        N = X.shape[0]
+    else:
+        if X.dim() != 3 or X.shape[0] != C or X.shape[2] != d:
+            raise ValueError("X must be [C][N][d] for groups = C")
+        N = X.shape[1]
+    _dev(codes, "codes", torch.int8, (k_max, C, d))
+    _dev(scales, "scales", torch.float32, (C, k_max))
+    err = err if err is not None else torch.empty((C, k_max + 1), dtype=torch.float32,
+                                                  device=W.device)
+    _dev(err, "err", torch.float32, (C, k_max + 1))
+    st = load().mpq_output_error(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales), C, d,
+                                 k_max, _ptr(err), _stream(stream))
+    _check(st, "mpq_output_error")
+    return err
+
+
+def mpq_allocate_points(err, k_max: int, mode: int = MPQ_ALLOC_BUDGET,
+                        budget_or_eps: float = 1.0, npoints=None, points_used=None, stream=None):
+    """Per-channel point counts (Algorithm 2, budget or threshold mode).
+
+    Returns (npoints [C] int32, points_used [1] int32) on the device."""
+    _dev(err, "err", torch.float32)
+    C = err.shape[0]
+    if tuple(err.shape) != (C, k_max + 1):
+        raise ValueError("err must be [C][k_max+1]")
+    npoints = npoints if npoints is not None else torch.empty((C,), dtype=torch.int32,
+                                                              device=err.device)
+    points_used = points_used if points_used is not None else torch.empty(
+        (1,), dtype=torch.int32, device=err.device)
+    _dev(npoints, "npoints", torch.int32, (C,))
+    _dev(points_used, "points_used", torch.int32, (1,))
+    st = load().mpq_allocate_points(_ptr(err), C, k_max, mode, float(budget_or_eps),
+                                    _ptr(npoints), _ptr(points_used), _stream(stream))
+    _check(st, "mpq_allocate_points")
+    return npoints, points_used
+
+
+def mpq_reconstruct(codes, scales, npoints, W_hat=None, stream=None):
+    """Multipoint weights (Eq. 4): W_hat [C][d] fp32."""
+    _dev(codes, "codes", torch.int8)
+    k_max, C, d = codes.shape
+    _dev(scales, "scales", torch.float32, (C, k_max))
+    _dev(npoints, "npoints", torch.int32, (C,))
+    W_hat = W_hat if W_hat is not None else torch.empty((C, d), dtype=torch.float32,
+                                                        device=codes.device)
+    _dev(W_hat, "W_hat", torch.float32, (C, d))
+    st = load().mpq_reconstruct(_ptr(codes), _ptr(scales), _ptr(npoints), C, d, k_max,
+                                _ptr(W_hat), _stream(stream))
+    _check(st, "mpq_reconstruct")
+    return W_hat
+
+
+def mpq_status_string(status: int) -> str:
+    return load().mpq_status_string(status).decode()
+
+
+def mpq_version() -> int:
+    return load().mpq_version()

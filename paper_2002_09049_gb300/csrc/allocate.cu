@@ -1,0 +1,177 @@
+// Per-channel point counts from the output-error table (Sec. 3.3, Algorithm 2).
+//
+// Budget mode.  The sequential rule -- hand each extra point to the channel whose next point has
+// the largest gain e_k(n_k) - e_k(n_k+1), lowest k on ties, stop when no gain is positive -- is
+// computed as one selection.  For channel k and n = 2..k_max let
+//   gain_k(n) = e_k(n-1) - e_k(n)      (fp32 subtraction; NaN reads as -inf)
+//   p_k(n)    = min_{2<=m<=n} gain_k(m) (prefix minimum)
+// and order the pairs (k, n) by (p desc, k asc, n asc).  The sequential loop takes exactly the
+// first `extra` pairs of this order that have p > 0: a channel's (n+1)-th gain becomes its head
+// only after the n-th was taken, its priority never exceeds the priorities before it, and a head
+// at or above every other head is taken next -- so both rules visit the pairs in the same order.
+// Each pair becomes one unique 64-bit key (~bits(p) in the high word, k*(k_max-1)+(n-2) in the
+// low word); an MSB-first radix select finds the extra-th smallest key T, and
+// n_k = 1 + #{n : key(k, n) <= T}.  Keys are recomputed from the error table on every pass, so
+// nothing but a 256-bin histogram in shared memory is needed.
+#include <math.h>
+
+#include "mpq_internal.cuh"
+
+namespace mpq {
+namespace {
+
+constexpr int AB_THREADS = 1024;
+constexpr unsigned long long NO_KEY = ~0ULL;
+
+// The keys of channel k for n = 2..k_max, in n order, via callback.
+template <typename F>
+__device__ __forceinline__ void channel_keys(const float *__restrict__ err, int k, int k_max, F f)
+{
+    const float *e = err + (size_t)k * (k_max + 1);
+    float p = INFINITY;
+    float prev = e[1];
+    for (int n = 2; n <= k_max; ++n) {
+        const float cur = e[n];
+        float g = __fsub_rn(prev, cur);
+        if (isnan(g)) g = -INFINITY;
+        p = fminf(p, g);
+        prev = cur;
+        unsigned long long key = NO_KEY;
+        if (p > 0.0f) {
+            const unsigned hi = ~__float_as_uint(p);
+            const unsigned lo = (unsigned)((unsigned long long)k * (k_max - 1) + (n - 2));
+            key = ((unsigned long long)hi << 32) | lo;
+        }
+        f(n, key);
+    }
+}
+
+__global__ void __launch_bounds__(AB_THREADS)
+allocate_budget_kernel(const float *__restrict__ err, int C, int k_max, long long extra,
+                       int *__restrict__ npoints, int *__restrict__ points_used)
+{
+    __shared__ unsigned int hist[256];
+    __shared__ unsigned long long s_prefix;
+    __shared__ long long s_rem;
+    __shared__ unsigned long long s_total;
+    const int tid = threadIdx.x;
+
+    // number of selectable keys (p > 0)
+    if (tid == 0) s_total = 0;
+    __syncthreads();
+    unsigned long long mine = 0;
+    for (int k = tid; k < C; k += AB_THREADS)
+        channel_keys(err, k, k_max, [&](int, unsigned long long key) { mine += key != NO_KEY; });
+    atomicAdd(&s_total, mine);
+    __syncthreads();
+    const long long total = (long long)s_total;
+    const long long take = extra < total ? extra : total;
+
+    unsigned long long T = 0;  // threshold key; selected = keys <= T (when take > 0)
+    if (take == 0) {
+        T = 0;
+    } else if (take == total) {
+        T = NO_KEY - 1;
+    } else {
+        if (tid == 0) {
+            s_prefix = 0;
+            s_rem = take;  // 1-based rank of the key we look for
+        }
+        for (int shift = 56; shift >= 0; shift -= 8) {
+            for (int b = tid; b < 256; b += AB_THREADS) hist[b] = 0;
+            __syncthreads();
+            const unsigned long long prefix = s_prefix;
+            const int hs = shift + 8;
+            for (int k = tid; k < C; k += AB_THREADS)
+                channel_keys(err, k, k_max, [&](int, unsigned long long key) {
+                    if (key == NO_KEY) return;
+                    if (hs < 64 && ((key ^ prefix) >> hs) != 0) return;
+                    atomicAdd(&hist[(key >> shift) & 255u], 1u);
+                });
+            __syncthreads();
+            if (tid == 0) {
+                long long rem = s_rem, cum = 0;
+                int b = 0;
+                for (; b < 256; ++b) {
+                    if (cum + (long long)hist[b] >= rem) break;
+                    cum += hist[b];
+                }
+                s_rem = rem - cum;
+                s_prefix = prefix | ((unsigned long long)b << shift);
+            }
+            __syncthreads();
+        }
+        T = s_prefix;
+    }
+
+    // n_k = 1 + number of selected keys of channel k (a prefix n = 2..n_k, since p is monotone)
+    int used = 0;
+    for (int k = tid; k < C; k += AB_THREADS) {
+        int n_k = 1;
+        channel_keys(err, k, k_max, [&](int, unsigned long long key) {
+            if (take > 0 && key != NO_KEY && key <= T) ++n_k;
+        });
+        npoints[k] = n_k;
+        used += n_k;
+    }
+    if (points_used) {
+        __shared__ int s_used;
+        if (tid == 0) s_used = 0;
+        __syncthreads();
+        atomicAdd(&s_used, used);
+        __syncthreads();
+        if (tid == 0) *points_used = s_used;
+    }
+}
+
+constexpr int AT_THREADS = 256;
+
+__global__ void __launch_bounds__(AT_THREADS)
+allocate_threshold_kernel(const float *__restrict__ err, int C, int k_max, double eps,
+                          int *__restrict__ npoints, int *__restrict__ points_used)
+{
+    int used = 0;
+    for (int k = blockIdx.x * AT_THREADS + threadIdx.x; k < C; k += gridDim.x * AT_THREADS) {
+        const float *e = err + (size_t)k * (k_max + 1);
+        int n = k_max;
+        for (int m = 1; m <= k_max; ++m) {
+            if ((double)e[m] < eps) {
+                n = m;
+                break;
+            }
+        }
+        npoints[k] = n;
+        used += n;
+    }
+    if (points_used) {
+        for (int o = 16; o > 0; o >>= 1) used += __shfl_xor_sync(0xffffffffu, used, o);
+        if ((threadIdx.x & 31) == 0) atomicAdd(points_used, used);  // integer sum: order-free
+    }
+}
+
+}  // namespace
+
+mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
+                                  int *npoints, int *points_used, cudaStream_t stream)
+{
+    allocate_budget_kernel<<<1, AB_THREADS, 0, stream>>>(err, C, k_max, extra, npoints,
+                                                         points_used);
+    return cuda_status(cudaGetLastError(), "allocation kernel launch");
+}
+
+mpq_status launch_allocate_threshold(const float *err, int C, int k_max, double eps,
+                                     int *npoints, int *points_used, cudaStream_t stream)
+{
+    if (points_used) {
+        cudaError_t e = cudaMemsetAsync(points_used, 0, sizeof(int), stream);
+        if (e != cudaSuccess) return cuda_status(e, "cudaMemsetAsync");
+    }
+    int blocks = (C + AT_THREADS - 1) / AT_THREADS;
+    const int cap = sm_count() * 4;
+    if (blocks > cap) blocks = cap;
+    allocate_threshold_kernel<<<blocks, AT_THREADS, 0, stream>>>(err, C, k_max, eps, npoints,
+                                                                  points_used);
+    return cuda_status(cudaGetLastError(), "allocation kernel launch");
+}
+
+}  // namespace mpq

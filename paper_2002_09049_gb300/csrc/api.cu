@@ -1,0 +1,198 @@
+// Host side of the C ABI (include/mpq.h): argument validation, error reporting, dispatch to the
+// kernel launchers.  Nothing here allocates device memory or synchronizes.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "mpq_internal.cuh"
+
+namespace mpq {
+
+static thread_local char g_msg[512];
+
+void set_error(const char *fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof(g_msg), fmt, ap);
+    va_end(ap);
+}
+
+mpq_status cuda_status(cudaError_t e, const char *what)
+{
+    if (e == cudaSuccess) return MPQ_OK;
+    set_error("%s: %s (%s)", what, cudaGetErrorString(e), cudaGetErrorName(e));
+    return MPQ_ERR_CUDA;
+}
+
+static const int kMaxDevices = 64;
+
+int sm_count()
+{
+    static int cache[kMaxDevices];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 148;
+    if (cache[dev] == 0) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+        cache[dev] = v > 0 ? v : 148;
+    }
+    return cache[dev];
+}
+
+int max_smem_optin()
+{
+    static int cache[kMaxDevices];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 48 * 1024;
+    if (cache[dev] == 0) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+        cache[dev] = v > 0 ? v : 48 * 1024;
+    }
+    return cache[dev];
+}
+
+}  // namespace mpq
+
+using namespace mpq;
+
+#define REQUIRE(cond, status, ...)  \
+    do {                            \
+        if (!(cond)) {              \
+            set_error(__VA_ARGS__); \
+            return (status);        \
+        }                           \
+    } while (0)
+
+static mpq_status check_common(int C, int d, int k_max)
+{
+    REQUIRE(C >= 0, MPQ_ERR_INVALID_ARG, "C = %d must be >= 0", C);
+    REQUIRE(d >= 1, MPQ_ERR_INVALID_ARG, "d = %d must be >= 1", d);
+    REQUIRE(k_max >= 1, MPQ_ERR_INVALID_ARG, "k_max = %d must be >= 1", k_max);
+    REQUIRE(k_max <= MPQ_MAX_POINTS, MPQ_ERR_UNSUPPORTED, "k_max = %d exceeds MPQ_MAX_POINTS = %d",
+            k_max, MPQ_MAX_POINTS);
+    REQUIRE((long long)C * d <= (1LL << 40), MPQ_ERR_UNSUPPORTED, "C*d = %lld too large",
+            (long long)C * d);
+    return MPQ_OK;
+}
+
+extern "C" mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
+                                         const float *grid_frac, int k_max, int8_t *codes,
+                                         float *scales, float *resid_sq, float *residuals,
+                                         void *stream)
+{
+    g_msg[0] = 0;
+    mpq_status st = check_common(C, d, k_max);
+    if (st != MPQ_OK) return st;
+    REQUIRE(bits >= MPQ_MIN_BITS && bits <= MPQ_MAX_BITS,
+            (bits > MPQ_MAX_BITS ? MPQ_ERR_UNSUPPORTED : MPQ_ERR_INVALID_ARG),
+            "bits = %d outside [%d, %d]", bits, MPQ_MIN_BITS, MPQ_MAX_BITS);
+    REQUIRE(G >= 1, MPQ_ERR_INVALID_ARG, "G = %d must be >= 1", G);
+    REQUIRE(G <= MPQ_MAX_GRID, MPQ_ERR_UNSUPPORTED, "G = %d exceeds MPQ_MAX_GRID = %d", G,
+            MPQ_MAX_GRID);
+    REQUIRE(d <= MPQ_MAX_DIM, MPQ_ERR_UNSUPPORTED, "d = %d exceeds MPQ_MAX_DIM = %d", d,
+            MPQ_MAX_DIM);
+    if (C == 0) return MPQ_OK;
+    REQUIRE(W && codes && scales, MPQ_ERR_INVALID_ARG, "W, codes and scales must be non-NULL");
+
+    GridFrac gf;
+    if (grid_frac) {
+        float prev = 0.0f;
+        for (int g = 0; g < G; ++g) {
+            float f = grid_frac[g];
+            REQUIRE(isfinite(f) && f > 0.0f && f <= 1.0f, MPQ_ERR_INVALID_ARG,
+                    "grid_frac[%d] = %g must be in (0, 1]", g, (double)f);
+            REQUIRE(f > prev, MPQ_ERR_INVALID_ARG, "grid_frac must be strictly increasing at %d",
+                    g);
+            gf.f[g] = f;
+            prev = f;
+        }
+    }
+    int qmax = (1 << (bits - 1)) - 1;
+    return launch_quantize(W, C, d, qmax, G, grid_frac ? &gf : nullptr, k_max, codes, scales,
+                           resid_sq, residuals, (cudaStream_t)stream);
+}
+
+extern "C" mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
+                                       const int8_t *codes, const float *scales, int C, int d,
+                                       int k_max, float *err, void *stream)
+{
+    g_msg[0] = 0;
+    mpq_status st = check_common(C, d, k_max);
+    if (st != MPQ_OK) return st;
+    REQUIRE(N >= 1, MPQ_ERR_INVALID_ARG, "N = %d must be >= 1", N);
+    REQUIRE(groups == 1 || groups == C, MPQ_ERR_INVALID_ARG, "groups = %d must be 1 or C = %d",
+            groups, C);
+    REQUIRE((long long)N * d <= (1LL << 40), MPQ_ERR_UNSUPPORTED, "N*d too large");
+    if (C == 0) return MPQ_OK;
+    REQUIRE(X && W && codes && scales && err, MPQ_ERR_INVALID_ARG,
+            "X, W, codes, scales and err must be non-NULL");
+    return launch_output_error(X, N, groups, W, codes, scales, C, d, k_max, err,
+                               (cudaStream_t)stream);
+}
+
+extern "C" mpq_status mpq_allocate_points(const float *err, int C, int k_max, int mode,
+                                          double budget_or_eps, int *npoints, int *points_used,
+                                          void *stream)
+{
+    g_msg[0] = 0;
+    mpq_status st = check_common(C, 1, k_max);
+    if (st != MPQ_OK) return st;
+    REQUIRE(mode == MPQ_ALLOC_BUDGET || mode == MPQ_ALLOC_THRESHOLD, MPQ_ERR_INVALID_ARG,
+            "mode = %d must be MPQ_ALLOC_BUDGET (0) or MPQ_ALLOC_THRESHOLD (1)", mode);
+    REQUIRE(!isnan(budget_or_eps), MPQ_ERR_NONFINITE, "budget_or_eps is NaN");
+    if (mode == MPQ_ALLOC_BUDGET) {
+        REQUIRE(isfinite(budget_or_eps), MPQ_ERR_NONFINITE, "budget must be finite");
+        REQUIRE(budget_or_eps >= 0.0, MPQ_ERR_INVALID_ARG, "budget = %g must be >= 0",
+                budget_or_eps);
+    }
+    if (C == 0) {
+        if (points_used)
+            return cuda_status(cudaMemsetAsync(points_used, 0, sizeof(int), (cudaStream_t)stream),
+                               "cudaMemsetAsync");
+        return MPQ_OK;
+    }
+    REQUIRE(err && npoints, MPQ_ERR_INVALID_ARG, "err and npoints must be non-NULL");
+    if (mode == MPQ_ALLOC_THRESHOLD)
+        return launch_allocate_threshold(err, C, k_max, budget_or_eps, npoints, points_used,
+                                         (cudaStream_t)stream);
+    long long total = (long long)floor(budget_or_eps * (double)C + 0.5);
+    long long extra = total - (long long)C;
+    long long cap = (long long)C * (k_max - 1);
+    if (extra < 0) extra = 0;
+    if (extra > cap) extra = cap;
+    return launch_allocate_budget(err, C, k_max, extra, npoints, points_used,
+                                  (cudaStream_t)stream);
+}
+
+extern "C" mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
+                                      int C, int d, int k_max, float *W_hat, void *stream)
+{
+    g_msg[0] = 0;
+    mpq_status st = check_common(C, d, k_max);
+    if (st != MPQ_OK) return st;
+    if (C == 0) return MPQ_OK;
+    REQUIRE(codes && scales && npoints && W_hat, MPQ_ERR_INVALID_ARG,
+            "codes, scales, npoints and W_hat must be non-NULL");
+    return launch_reconstruct(codes, scales, npoints, C, d, k_max, W_hat, (cudaStream_t)stream);
+}
+
+extern "C" const char *mpq_status_string(mpq_status s)
+{
+    switch (s) {
+    case MPQ_OK: return "MPQ_OK";
+    case MPQ_ERR_INVALID_ARG: return "MPQ_ERR_INVALID_ARG";
+    case MPQ_ERR_NONFINITE: return "MPQ_ERR_NONFINITE";
+    case MPQ_ERR_UNSUPPORTED: return "MPQ_ERR_UNSUPPORTED";
+    case MPQ_ERR_CUDA: return "MPQ_ERR_CUDA";
+    case MPQ_ERR_TIMEOUT: return "MPQ_ERR_TIMEOUT";
+    case MPQ_ERR_NOMEM: return "MPQ_ERR_NOMEM";
+    }
+    return "MPQ_ERR_UNKNOWN";
+}
+
+extern "C" const char *mpq_last_error(void) { return g_msg; }
+
+extern "C" int mpq_version(void) { return 100; }

@@ -1,0 +1,45 @@
+// Internal declarations shared by the CUDA translation units of libmpq.so (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/mpq.h"
+
+namespace mpq {
+
+// Records a formatted failure message for mpq_last_error() on the calling thread.
+void set_error(const char *fmt, ...);
+
+// Maps a CUDA error to MPQ_ERR_CUDA (recording its text), cudaSuccess to MPQ_OK.
+mpq_status cuda_status(cudaError_t e, const char *what);
+
+// Multiprocessor count of the current device (cached per device).
+int sm_count();
+
+// Opt-in dynamic shared memory limit per block of the current device (cached per device).
+int max_smem_optin();
+
+struct GridFrac {
+    float f[MPQ_MAX_GRID];
+};
+
+// --- launchers, one per kernel family; arguments are already validated ----------------------
+mpq_status launch_quantize(const float *W, int C, int d, int qmax, int G, const GridFrac *grid,
+                           int k_max, int8_t *codes, float *scales, float *resid_sq,
+                           float *residuals, cudaStream_t stream);
+
+mpq_status launch_output_error(const float *X, int N, int groups, const float *W,
+                               const int8_t *codes, const float *scales, int C, int d, int k_max,
+                               float *err, cudaStream_t stream);
+
+mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
+                                  int *npoints, int *points_used, cudaStream_t stream);
+
+mpq_status launch_allocate_threshold(const float *err, int C, int k_max, double eps,
+                                     int *npoints, int *points_used, cudaStream_t stream);
+
+mpq_status launch_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C,
+                              int d, int k_max, float *W_hat, cudaStream_t stream);
+
+}  // namespace mpq

@@ -1,0 +1,93 @@
+"""One layer through the whole hot path: greedy points (Algorithm 1), output error (Eq. 11),
+point allocation (Algorithm 2), multipoint weights (Eq. 4).
+
+``LayerPlan`` owns the device output buffers of one layer so that repeated runs allocate nothing;
+``run_device`` enqueues the four C-ABI calls on one stream; ``run_host`` is the end-to-end call
+for host data: copies W and X in from (pinned) host memory, runs the path and copies the durable
+result (codes, scales, point counts) back out.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import torch
+
+from . import binding
+
+
+@dataclass
+class LayerSpec:
+    C: int
+    d: int
+    N: int
+    groups: int = 1
+    bits: int = 4
+    G: int = 64
+    k_max: int = 4
+    mode: int = binding.MPQ_ALLOC_BUDGET
+    budget_or_eps: float = 1.5
+
+
+class LayerPlan:
+    def __init__(self, spec: LayerSpec, device, with_reconstruct: bool = True):
+        self.spec = spec
+        s = spec
+        dev = torch.device(device)
+        self.codes = torch.empty((s.k_max, s.C, s.d), dtype=torch.int8, device=dev)
+        self.scales = torch.empty((s.C, s.k_max), dtype=torch.float32, device=dev)
+        self.resid_sq = torch.empty((s.C, s.k_max + 1), dtype=torch.float32, device=dev)
+        self.err = torch.empty((s.C, s.k_max + 1), dtype=torch.float32, device=dev)
+        self.npoints = torch.empty((s.C,), dtype=torch.int32, device=dev)
+        self.points_used = torch.empty((1,), dtype=torch.int32, device=dev)
+        self.W_hat = torch.empty((s.C, s.d), dtype=torch.float32, device=dev) \
+            if with_reconstruct else None
+        self._host = None
+
+    # -- device-resident inputs ---------------------------------------------------------------
+    def run_device(self, W, X, stream=None, grid_frac=None):
+        s = self.spec
+        binding.mpq_quantize_layer(W, s.bits, s.G, s.k_max, grid_frac=grid_frac, codes=self.codes,
+                                   scales=self.scales, resid_sq=self.resid_sq, stream=stream)
+        binding.mpq_output_error(X, W, self.codes, self.scales, s.k_max, groups=s.groups,
+                                 err=self.err, stream=stream)
+        binding.mpq_allocate_points(self.err, s.k_max, s.mode, s.budget_or_eps,
+                                    npoints=self.npoints, points_used=self.points_used,
+                                    stream=stream)
+        if self.W_hat is not None:
+            binding.mpq_reconstruct(self.codes, self.scales, self.npoints, W_hat=self.W_hat,
+                                    stream=stream)
+        return self
+
+    # -- host inputs / outputs (end to end) ----------------------------------------------------
+    def host_buffers(self, pin: bool = True):
+        """Pinned host buffers for the durable result of one run."""
+        if self._host is None:
+            s = self.spec
+            mk = lambda shape, dt: torch.empty(shape, dtype=dt, pin_memory=pin)
+            self._host = dict(codes=mk((s.k_max, s.C, s.d), torch.int8),
+                              scales=mk((s.C, s.k_max), torch.float32),
+                              npoints=mk((s.C,), torch.int32),
+                              points_used=mk((1,), torch.int32))
+        return self._host
+
+    def run_host(self, W_host, X_host, W_dev, X_dev, stream=None):
+        """H2D copy of W and X, the path, D2H copy of codes / scales / npoints / points_used.
+        Returns the host dict; the caller synchronizes ``stream`` before reading it."""
+        st = stream or torch.cuda.current_stream()
+        h = self.host_buffers()
+        with torch.cuda.stream(st):
+            W_dev.copy_(W_host, non_blocking=True)
+            X_dev.copy_(X_host, non_blocking=True)
+            self.run_device(W_dev, X_dev, stream=st)
+            h["codes"].copy_(self.codes, non_blocking=True)
+            h["scales"].copy_(self.scales, non_blocking=True)
+            h["npoints"].copy_(self.npoints, non_blocking=True)
+            h["points_used"].copy_(self.points_used, non_blocking=True)
+        return h
+
+    def h2d_bytes(self, W, X) -> int:
+        return W.numel() * W.element_size() + X.numel() * X.element_size()
+
+    def d2h_bytes(self) -> int:
+        s = self.spec
+        return s.k_max * s.C * s.d + 4 * s.C * s.k_max + 4 * s.C + 4

@@ -17,3 +17,14 @@ def oracle():
     import oracle as o
     o.build()
     return o
+
+
+@pytest.fixture(scope="session")
+def gpu():
+    """cuda:0 with libmpq.so built and loaded (the CUDA path; no fallback)."""
+    import torch
+    from paper_2002_09049_gb300 import _build, binding
+    assert torch.cuda.is_available(), "gpu tests need a CUDA device"
+    _build.build()
+    binding.load()
+    return torch.device("cuda:0")

@@ -1,0 +1,104 @@
+"""The C-ABI library builds, loads without a GPU, exports every symbol include/*.h declares, and
+rejects invalid arguments on the host before touching the device (no GPU needed)."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+from paper_2002_09049_gb300 import _build, binding
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = []
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        names += re.findall(r"^[A-Za-z_][\w \t\*]*?\b(mpq_\w+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    return binding.load()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for n in ("mpq_quantize_layer", "mpq_output_error", "mpq_allocate_points", "mpq_reconstruct"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    raw = ctypes.CDLL(_build.LIB)
+    for name in declared_functions():
+        assert hasattr(raw, name), name
+        assert name in binding.SIGNATURES, name
+
+
+def test_status_strings(lib):
+    assert lib.mpq_status_string(0) == b"MPQ_OK"
+    assert lib.mpq_status_string(3) == b"MPQ_ERR_UNSUPPORTED"
+    assert lib.mpq_version() >= 100
+
+
+P = ctypes.c_void_p
+FAKE = P(0x1000)  # never dereferenced: every call below fails validation on the host first
+
+
+@pytest.mark.parametrize("kwargs,status", [
+    (dict(bits=1), 1), (dict(bits=9), 3), (dict(G=0), 1), (dict(G=1025), 3), (dict(k_max=0), 1),
+    (dict(k_max=17), 3), (dict(d=0), 1), (dict(d=8193), 3), (dict(C=-1), 1),
+    (dict(W=None), 1), (dict(codes=None), 1), (dict(scales=None), 1),
+])
+def test_quantize_validation(lib, kwargs, status):
+    a = dict(W=FAKE, C=4, d=16, bits=4, G=8, grid=None, k_max=2, codes=FAKE, scales=FAKE)
+    a.update(kwargs)
+    st = lib.mpq_quantize_layer(a["W"], a["C"], a["d"], a["bits"], a["G"], a["grid"], a["k_max"],
+                                a["codes"], a["scales"], None, None, None)
+    assert st == status
+    assert lib.mpq_last_error() != b""
+
+
+@pytest.mark.parametrize("grid", [[0.5, 0.25, 1.0], [0.0, 0.5, 1.0], [0.5, 0.5, 1.0],
+                                  [0.5, 0.75, 1.5], [0.5, float("nan"), 1.0]])
+def test_quantize_rejects_bad_grid(lib, grid):
+    g = (ctypes.c_float * 3)(*grid)
+    st = lib.mpq_quantize_layer(FAKE, 4, 16, 4, 3, g, 2, FAKE, FAKE, None, None, None)
+    assert st == 1
+
+
+def test_empty_layer_is_a_no_op(lib):
+    assert lib.mpq_quantize_layer(None, 0, 16, 4, 8, None, 2, None, None, None, None, None) == 0
+    assert lib.mpq_output_error(None, 5, 1, None, None, None, 0, 16, 2, None, None) == 0
+    assert lib.mpq_reconstruct(None, None, None, 0, 16, 2, None, None) == 0
+
+
+@pytest.mark.parametrize("args,status", [
+    ((FAKE, 0, 1, FAKE, FAKE, FAKE, 4, 16, 2, FAKE), 1),    # N = 0
+    ((FAKE, 8, 3, FAKE, FAKE, FAKE, 4, 16, 2, FAKE), 1),    # groups not in {1, C}
+    ((None, 8, 1, FAKE, FAKE, FAKE, 4, 16, 2, FAKE), 1),    # X NULL
+    ((FAKE, 8, 1, FAKE, FAKE, FAKE, 4, 16, 2, None), 1),    # err NULL
+])
+def test_output_error_validation(lib, args, status):
+    assert lib.mpq_output_error(*args, None) == status
+
+
+@pytest.mark.parametrize("mode,val,status", [
+    (2, 1.0, 1), (0, float("nan"), 2), (0, float("inf"), 2), (0, -0.5, 1), (1, float("nan"), 2),
+])
+def test_allocate_validation(lib, mode, val, status):
+    assert lib.mpq_allocate_points(FAKE, 4, 3, mode, val, FAKE, None, None) == status
+
+
+def test_allocate_requires_outputs(lib):
+    assert lib.mpq_allocate_points(FAKE, 4, 3, 0, 1.5, None, None, None) == 1
+
+
+def test_reconstruct_validation(lib):
+    assert lib.mpq_reconstruct(FAKE, FAKE, None, 4, 16, 2, FAKE, None) == 1
+    assert lib.mpq_reconstruct(FAKE, FAKE, FAKE, 4, 16, 0, FAKE, None) == 1

@@ -1,0 +1,69 @@
+"""Parity of mpq_output_error (Eq. 11) with the oracle, through the C ABI."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2002_09049_gb300 import binding, workloads as wlm
+from _parity import compare_err
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_err(X, W, codes, scales, k_max, groups=1, dev="cuda:0"):
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    err = binding.mpq_output_error(t(X), t(W), t(codes), t(scales), k_max, groups=groups)
+    torch.cuda.synchronize()
+    return err.cpu().numpy()
+
+
+@pytest.mark.parametrize("C,d,N,K", [(1, 1, 1, 1), (3, 5, 7, 2), (5, 33, 70, 4), (7, 64, 64, 3),
+                                     (11, 147, 129, 4), (4, 1000, 65, 2), (64, 576, 512, 4),
+                                     (2, 17, 300, 16)])
+def test_shared_input(gpu, oracle, C, d, N, K):
+    W = wlm.random_weights(C, d, C + d + N, "normal")
+    q = oracle.quantize_layer(W, 4, 32, K)
+    X = wlm.random_calibration(N, d, 7 + d)
+    e_or = oracle.output_error(X, 1, W, q["codes"], q["scales"], K)
+    e_gpu = gpu_err(X, W, q["codes"], q["scales"], K)
+    compare_err(e_gpu, e_or)
+
+
+@pytest.mark.parametrize("C,d,N,K", [(1, 9, 1, 1), (6, 9, 100, 8), (40, 9, 1024, 8), (3, 25, 77, 4),
+                                     (5, 300, 33, 16)])
+def test_per_channel_input(gpu, oracle, C, d, N, K):
+    W = wlm.random_weights(C, d, 3 * C + d, "laplace")
+    q = oracle.quantize_layer(W, 4, 64, K)
+    X = wlm.random_calibration(N, d, 11, groups=C)
+    e_or = oracle.output_error(X, C, W, q["codes"], q["scales"], K)
+    e_gpu = gpu_err(X, W, q["codes"], q["scales"], K, groups=C)
+    compare_err(e_gpu, e_or)
+
+
+def test_config1_layer(gpu, oracle):
+    wl = wlm.WORKLOADS["c1"]
+    W = wlm.make_weights(wl, 0)
+    X = wlm.make_calibration(wl, 0)
+    q = oracle.quantize_layer(W, 4, wl.G, wl.k_max)
+    worst = compare_err(gpu_err(X, W, q["codes"], q["scales"], wl.k_max),
+                        oracle.output_error(X, 1, W, q["codes"], q["scales"], wl.k_max))
+    assert worst < 1e-5
+
+
+def test_hot_columns_input(gpu, oracle):
+    """Inputs with a few large columns (the large-linear-layer workload's calibration recipe)."""
+    rng = np.random.default_rng(4)
+    X = rng.standard_normal((256, 512)).astype(np.float32)
+    X[:, rng.choice(512, 8, replace=False)] *= 10
+    W = (rng.standard_normal((24, 512)) * 0.02).astype(np.float32)
+    q = oracle.quantize_layer(W, 4, 256, 8)
+    compare_err(gpu_err(X, W, q["codes"], q["scales"], 8),
+                oracle.output_error(X, 1, W, q["codes"], q["scales"], 8))
+
+
+def test_nonfinite_weight_propagates(gpu, oracle):
+    W = wlm.random_weights(3, 20, 1, "normal")
+    W[1, 2] = np.nan
+    q = oracle.quantize_layer(W, 4, 16, 2)
+    X = wlm.random_calibration(10, 20, 2)
+    e = gpu_err(X, W, q["codes"], q["scales"], 2)
+    assert np.all(np.isnan(e[1])) and np.all(np.isfinite(e[[0, 2]]))

@@ -1,0 +1,91 @@
+"""End-to-end parity of the whole path on the single conv-shaped layer workload and sampled
+parity at full size on the ResNet-18-shaped and large-linear workloads."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2002_09049_gb300 import binding, pipeline, workloads as wlm
+from _parity import compare_err, compare_quantize
+
+pytestmark = pytest.mark.gpu
+
+
+def test_config1_end_to_end(gpu, oracle):
+    wl = wlm.WORKLOADS["c1"]
+    W = wlm.make_weights(wl, 0)
+    X = wlm.make_calibration(wl, 0)
+    spec = pipeline.LayerSpec(C=64, d=576, N=512, bits=4, G=wl.G, k_max=wl.k_max,
+                              budget_or_eps=wl.beta)
+    plan = pipeline.LayerPlan(spec, gpu)
+    Wd, Xd = torch.from_numpy(W).to(gpu), torch.from_numpy(X).to(gpu)
+    plan.run_device(Wd, Xd)
+    torch.cuda.synchronize()
+    gpu_q = dict(codes=plan.codes.cpu().numpy(), scales=plan.scales.cpu().numpy(),
+                 resid_sq=plan.resid_sq.cpu().numpy())
+    orc = oracle.quantize_layer(W, 4, wl.G, wl.k_max)
+    rep = compare_quantize(W, gpu_q, orc, 4, wl.G, wl.k_max, oracle=oracle)
+    err_or = oracle.output_error(X, 1, W, orc["codes"], orc["scales"], wl.k_max)
+    err_gpu = plan.err.cpu().numpy()
+    if rep["near_ties"] == 0:
+        compare_err(err_gpu, err_or)
+        # allocation on the GPU's own error table must equal the sequential loop on that table
+        n_or, used_or = oracle.allocate_budget(err_gpu, wl.k_max, wl.beta)
+        assert np.array_equal(plan.npoints.cpu().numpy(), n_or)
+        assert int(plan.points_used.item()) == used_or == int(np.floor(wl.beta * 64 + 0.5))
+        What = oracle.reconstruct(orc["codes"], orc["scales"], n_or)
+        assert np.array_equal(plan.W_hat.cpu().numpy(), What)
+
+
+def test_run_host_matches_device(gpu):
+    wl = wlm.WORKLOADS["c1"]
+    W = torch.from_numpy(wlm.make_weights(wl, 0)).pin_memory()
+    X = torch.from_numpy(wlm.make_calibration(wl, 0)).pin_memory()
+    spec = pipeline.LayerSpec(C=64, d=576, N=512, G=wl.G, k_max=wl.k_max, budget_or_eps=wl.beta)
+    plan = pipeline.LayerPlan(spec, gpu)
+    Wd, Xd = torch.empty_like(W, device=gpu), torch.empty_like(X, device=gpu)
+    h = plan.run_host(W, X, Wd, Xd)
+    torch.cuda.synchronize()
+    assert torch.equal(h["codes"], plan.codes.cpu()) and torch.equal(h["npoints"],
+                                                                     plan.npoints.cpu())
+
+
+def sample_channels(C, rng, edge=16, frac=0.02):
+    idx = set(range(min(edge, C))) | set(range(max(0, C - edge), C))
+    idx |= set(rng.choice(C, size=max(1, int(frac * C)), replace=False).tolist())
+    return sorted(idx)
+
+
+@pytest.mark.parametrize("key,layers", [("c2", [0, 9, 16, 20]), ("c5", [1]), ("c4", [0, 1, 49, 52]),
+                                        ("c3", [3, 40])])
+def test_full_size_sampled(gpu, oracle, key, layers):
+    """Full-size layers on the GPU in the bench's launch configuration; the oracle checks a
+    sample of channels (first/last 16 and 2 % at random) of codes, scales and output errors."""
+    wl = wlm.WORKLOADS[key]
+    rng = np.random.default_rng(0)
+    for li in layers:
+        layer = wl.layers[li]
+        W = wlm.make_weights(wl, li)
+        X = wlm.make_calibration(wl, li)
+        bits = wl.bits[-1]
+        spec = pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, groups=layer.groups,
+                                  bits=bits, G=wl.G, k_max=wl.k_max, budget_or_eps=wl.beta)
+        plan = pipeline.LayerPlan(spec, gpu)
+        plan.run_device(torch.from_numpy(W).to(gpu), torch.from_numpy(X).to(gpu))
+        torch.cuda.synchronize()
+        ch = sample_channels(layer.C, rng)
+        gq = dict(codes=plan.codes.cpu().numpy(), scales=plan.scales.cpu().numpy(),
+                  resid_sq=plan.resid_sq.cpu().numpy())
+        orc = {}
+        sub = W[ch]
+        o = oracle.quantize_layer(sub, bits, wl.G, wl.k_max, threads=8)
+        gsub = dict(codes=gq["codes"][:, ch], scales=gq["scales"][ch], resid_sq=gq["resid_sq"][ch])
+        rep = compare_quantize(sub, gsub, o, bits, wl.G, wl.k_max, oracle=oracle)
+        # output error of the sampled channels from the GPU's codes (same inputs on both sides)
+        Xs = X[ch] if layer.groups > 1 else X
+        e_or = oracle.output_error(Xs, len(ch) if layer.groups > 1 else 1, sub, gsub["codes"],
+                                   gsub["scales"], wl.k_max, threads=8)
+        compare_err(plan.err.cpu().numpy()[ch], e_or)
+        # allocation on the GPU's error table is exactly the sequential loop
+        n_or, used_or = oracle.allocate_budget(plan.err.cpu().numpy(), wl.k_max, wl.beta)
+        assert np.array_equal(plan.npoints.cpu().numpy(), n_or)
+        assert int(plan.points_used.item()) == used_or
