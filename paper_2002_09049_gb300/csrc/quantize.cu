@@ -224,7 +224,8 @@ quantize_direct_kernel(const float *__restrict__ W, int C, int d, int qmax, int 
                     }
                 }
             }
-            const int g = block_argmin(bestD, bestg, red);
+            int g = block_argmin(bestD, bestg, red);
+            if (g < 0 || g >= G) g = G - 1;   // unreachable: every D is finite
             s_best = __fmul_rn(grid.frac(g, G), smax);
         }
 

@@ -21,6 +21,13 @@ def _grid(m, qmax, G, grid_frac):
     return (f * smax).astype(np.float32)
 
 
+def _same_scale(a, b):
+    """Bit-identical fp32 scales; any two NaNs (a channel with a non-finite weight) match."""
+    if np.isnan(a) and np.isnan(b):
+        return True
+    return a.tobytes() == b.tobytes()
+
+
 def compare_quantize(W, gpu: dict, orc: dict, bits: int, G: int, k_max: int, grid_frac=None,
                      oracle=None, channels=None):
     """Returns a report dict; raises AssertionError on any non-near-tie mismatch.
@@ -39,13 +46,13 @@ def compare_quantize(W, gpu: dict, orc: dict, bits: int, G: int, k_max: int, gri
             if diverged:
                 diverged_steps += 1
                 continue
-            same_s = gpu["scales"][k, i].tobytes() == orc["scales"][k, i].tobytes()
+            same_s = _same_scale(gpu["scales"][k, i], orc["scales"][k, i])
             same_q = np.array_equal(gpu["codes"][i, k], orc["codes"][i, k])
             if same_s and same_q:
                 checked += 1
                 if "residuals" in gpu and gpu["residuals"] is not None:
-                    assert np.array_equal(gpu["residuals"][i, k], orc["residuals"][i, k]), \
-                        f"residual mismatch k={k} i={i}"
+                    assert np.array_equal(gpu["residuals"][i, k], orc["residuals"][i, k],
+                                          equal_nan=True), f"residual mismatch k={k} i={i}"
                 continue
             # mismatch: must be a near tie of this step's scale search
             assert oracle is not None, f"mismatch at k={k} step={i} and no oracle to judge it"
@@ -66,7 +73,7 @@ def compare_quantize(W, gpu: dict, orc: dict, bits: int, G: int, k_max: int, gri
             # steps before the first divergence (plus the initial norm)
             agree = 0
             for i in range(k_max):
-                if gpu["scales"][k, i].tobytes() == orc["scales"][k, i].tobytes() and \
+                if _same_scale(gpu["scales"][k, i], orc["scales"][k, i]) and \
                         np.array_equal(gpu["codes"][i, k], orc["codes"][i, k]):
                     agree += 1
                 else:
