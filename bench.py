@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", default=None,
+                    help="comma-separated layer indices to run (profiling a subset); default all")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
     return ap.parse_args()
@@ -169,7 +171,10 @@ def run_ours(args, world, rank, local):
     wl = wlm.WORKLOADS[args.config]
     bits = wl.bits[0]
     runs = []  # (spec, plan, W_dev, X_dev, W_host, X_host, layer)
+    keep = None if args.layers is None else {int(x) for x in args.layers.split(",")}
     for li, layer in enumerate(wl.layers):
+        if keep is not None and li not in keep:
+            continue
         W, X = layer_inputs(wl, li)
         spec = pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, groups=layer.groups,
                                   bits=bits, G=wl.G, k_max=wl.k_max, budget_or_eps=wl.beta)

@@ -33,6 +33,10 @@ mpq_status launch_output_error(const float *X, int N, int groups, const float *W
                                const int8_t *codes, const float *scales, int C, int d, int k_max,
                                float *err, cudaStream_t stream);
 
+mpq_status launch_output_error_tc(const float *X, int N, const float *W, const int8_t *codes,
+                                  const float *scales, int C, int d, int k_max, float *err,
+                                  cudaStream_t stream);
+
 mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
                                   int *npoints, int *points_used, cudaStream_t stream);
 

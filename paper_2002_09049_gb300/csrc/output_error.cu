@@ -11,6 +11,7 @@
 // Per-channel input (groups = C, depthwise): one CTA per channel, its k_max+1 residuals in shared
 // memory, threads over the calibration rows.
 #include <math.h>
+#include <stdlib.h>
 
 #include "mpq_internal.cuh"
 
@@ -184,6 +185,8 @@ mpq_status launch_output_error(const float *X, int N, int groups, const float *W
                                const int8_t *codes, const float *scales, int C, int d, int k_max,
                                float *err, cudaStream_t stream)
 {
+    if (groups == 1 && !getenv("MPQ_DEBUG_SIMT_OUTPUT_ERROR"))
+        return launch_output_error_tc(X, N, W, codes, scales, C, d, k_max, err, stream);
     if (groups == 1) {
         const long long V = (long long)C * (k_max + 1);
         const long long blocks = (V + BN - 1) / BN;
