@@ -4,7 +4,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/mpq.h"
+#include "mpq.h"
 
 namespace mpq {
 
