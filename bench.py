@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--streams", type=int, default=8,
+                    help="CUDA streams the independent layers are spread over")
     ap.add_argument("--layers", default=None,
                     help="comma-separated layer indices to run (profiling a subset); default all")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
@@ -169,20 +171,21 @@ def run_ours(args, world, rank, local):
     binding.load()
 
     wl = wlm.WORKLOADS[args.config]
-    bits = wl.bits[0]
-    runs = []  # (spec, plan, W_dev, X_dev, W_host, X_host, layer)
     keep = None if args.layers is None else {int(x) for x in args.layers.split(",")}
-    for li, layer in enumerate(wl.layers):
-        if keep is not None and li not in keep:
-            continue
+    idx = [li for li in range(len(wl.layers)) if keep is None or li in keep]
+    layers = [wl.layers[li] for li in idx]
+    specs, Ws, Xs, Whs, Xhs = [], [], [], [], []
+    for li, layer in zip(idx, layers):
         W, X = layer_inputs(wl, li)
-        spec = pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, groups=layer.groups,
-                                  bits=bits, G=wl.G, k_max=wl.k_max, budget_or_eps=wl.beta)
-        plan = pipeline.LayerPlan(spec, dev)
-        Wh = torch.from_numpy(W).pin_memory()
-        Xh = torch.from_numpy(X).pin_memory()
-        runs.append((spec, plan, Wh.to(dev), Xh.to(dev), Wh, Xh, layer))
-    units_per_step = sum(kernel_units(wl, r[6]) for r in runs) * len(wl.bits)
+        specs.append(pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, groups=layer.groups,
+                                        bits=wl.bits[0], G=wl.G, k_max=wl.k_max,
+                                        budget_or_eps=wl.beta))
+        Whs.append(torch.from_numpy(W).pin_memory())
+        Xhs.append(torch.from_numpy(X).pin_memory())
+        Ws.append(Whs[-1].to(dev))
+        Xs.append(Xhs[-1].to(dev))
+    net = pipeline.NetworkPlan(specs, dev, n_streams=args.streams)
+    units_per_step = sum(kernel_units(wl, l) for l in layers) * len(wl.bits)
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 512 MB > L2
     stream = torch.cuda.current_stream()
 
@@ -190,31 +193,20 @@ def run_ours(args, world, rank, local):
 
     def step(record=None):
         for b in wl.bits:
-            for spec, plan, Wd, Xd, _, _, layer in runs:
-                spec.bits = b
-                s = plan.spec
-                ev = record is not None
-                if ev:
-                    e = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
-                    e[0].record(stream)
-                binding.mpq_quantize_layer(Wd, s.bits, s.G, s.k_max, codes=plan.codes,
-                                           scales=plan.scales, resid_sq=plan.resid_sq)
-                if ev:
-                    e[1].record(stream)
-                binding.mpq_output_error(Xd, Wd, plan.codes, plan.scales, s.k_max,
-                                         groups=s.groups, err=plan.err)
-                if ev:
-                    e[2].record(stream)
-                binding.mpq_allocate_points(plan.err, s.k_max, s.mode, s.budget_or_eps,
-                                            npoints=plan.npoints, points_used=plan.points_used)
-                if ev:
-                    e[3].record(stream)
-                binding.mpq_reconstruct(plan.codes, plan.scales, plan.npoints, W_hat=plan.W_hat)
-                if ev:
-                    e[4].record(stream)
-                    record.append((layer, e))
+            for sp in specs:
+                sp.bits = b
+            cb = None
+            if record is not None:
+                evs = {}
 
-    launches_per_step = 4 * len(runs) * len(wl.bits)
+                def cb(i, st, ph, evs=evs):
+                    e = torch.cuda.Event(enable_timing=True)
+                    e.record(st)
+                    evs.setdefault(i, [None] * 5)[ph] = e
+                record.append(evs)
+            net.run_device(Ws, Xs, stream=stream, on_layer=cb)
+
+    launches_per_step = 4 * len(layers) * len(wl.bits)
 
     for _ in range(args.warmup):
         step()
@@ -248,16 +240,18 @@ def run_ours(args, world, rank, local):
         ms = float(t.item())
     value = units_per_step * world / (ms / 1e3)
 
-    # per-kernel-family device time from the events around each call
+    # per-kernel-family device time from the events around every call (on its own stream)
     fam_ms = {f: 0.0 for f in families}
-    fam_work = {"output_error": 0.0, "quantize": 0.0, "reconstruct": 0.0, "allocate": 0.0}
+    fam_work = {f: 0.0 for f in families}
     for rec in recs:
-        for layer, e in rec:
-            for i, f in enumerate(families):
-                fam_ms[f] += e[i].elapsed_time(e[i + 1])
-            fam_work["output_error"] += contraction_flops(wl, layer)
-            fam_work["quantize"] += kernel_units(wl, layer)
-            fam_work["reconstruct"] += layer.C * layer.d * (4 + 1 + 4 / wl.k_max)  # bytes, approx
+        for evs in rec:
+            for i, e in evs.items():
+                layer = layers[i]
+                for k, f in enumerate(families):
+                    fam_ms[f] += e[k].elapsed_time(e[k + 1])
+                fam_work["output_error"] += contraction_flops(wl, layer)
+                fam_work["quantize"] += kernel_units(wl, layer)
+                fam_work["reconstruct"] += layer.C * layer.d * (4 + 1 + 4 / wl.k_max)
     total_fam = sum(fam_ms.values())
     dominant = max(fam_ms, key=fam_ms.get)
 
@@ -269,18 +263,19 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": f"{args.config}: {wl.title}", "layers": len(wl.layers),
-                   "weights": wl.n_weights, "channels": wl.n_channels, "bits": list(wl.bits),
+        "config": {"workload": f"{args.config}: {wl.title}", "layers": len(layers),
+                   "weights": sum(l.C * l.d for l in layers),
+                   "channels": sum(l.C for l in layers), "bits": list(wl.bits),
                    "G": wl.G, "k_max": wl.k_max, "budget": wl.beta, "calib_rows": wl.n_calib,
                    "units_per_step": units_per_step, "l2": "flushed between steps (512 MB write)",
-                   "parallelism": f"replicas x{world}"},
+                   "streams": args.streams, "parallelism": f"replicas x{world}"},
         "roofline": roofline,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
     }
 
     if not args.no_e2e:
-        out["e2e"] = run_e2e(runs, wl, args, stream, world, units_per_step)
+        out["e2e"] = run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
     if world > 1:
@@ -324,18 +319,18 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
             "frac": ach / hbm, "traffic": traffic, "peak_source": peak_src}
 
 
-def run_e2e(runs, wl, args, stream, world, units_per_step):
-    """Same metric through the public per-layer call with host buffers: H2D of W and X from
-    pinned memory, the path, D2H of codes / scales / point counts -- all inside the timing."""
+def run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step):
+    """Same metric through the public network call with host buffers: per layer, H2D of W and X
+    from pinned memory, the path, D2H of codes / scales / point counts -- all inside the timing."""
     import torch
-    h2d = sum(r[4].numel() * 4 + r[5].numel() * 4 for r in runs) * len(wl.bits)
-    d2h = sum(r[1].d2h_bytes() for r in runs) * len(wl.bits)
+    h2d = sum(w.numel() * 4 + x.numel() * 4 for w, x in zip(Whs, Xhs)) * len(wl.bits)
+    d2h = sum(p.d2h_bytes() for p in net.plans) * len(wl.bits)
 
     def step():
         for b in wl.bits:
-            for spec, plan, Wd, Xd, Wh, Xh, _ in runs:
-                spec.bits = b
-                plan.run_host(Wh, Xh, Wd, Xd, stream=stream)
+            for sp in specs:
+                sp.bits = b
+            net.run_host(Whs, Xhs, Ws, Xs, stream=stream)
 
     for _ in range(max(1, args.warmup)):
         step()

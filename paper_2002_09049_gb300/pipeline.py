@@ -44,18 +44,26 @@ class LayerPlan:
         self._host = None
 
     # -- device-resident inputs ---------------------------------------------------------------
-    def run_device(self, W, X, stream=None, grid_frac=None):
+    def run_device(self, W, X, stream=None, grid_frac=None, timing=None):
+        """Enqueue the four calls on ``stream``.  timing(phase), if given, is called before the
+        first call (phase 0) and after call k (phase k = 1..4), e.g. to record CUDA events."""
         s = self.spec
+        tick = timing or (lambda ph: None)
+        tick(0)
         binding.mpq_quantize_layer(W, s.bits, s.G, s.k_max, grid_frac=grid_frac, codes=self.codes,
                                    scales=self.scales, resid_sq=self.resid_sq, stream=stream)
+        tick(1)
         binding.mpq_output_error(X, W, self.codes, self.scales, s.k_max, groups=s.groups,
                                  err=self.err, stream=stream)
+        tick(2)
         binding.mpq_allocate_points(self.err, s.k_max, s.mode, s.budget_or_eps,
                                     npoints=self.npoints, points_used=self.points_used,
                                     stream=stream)
+        tick(3)
         if self.W_hat is not None:
             binding.mpq_reconstruct(self.codes, self.scales, self.npoints, W_hat=self.W_hat,
                                     stream=stream)
+        tick(4)
         return self
 
     # -- host inputs / outputs (end to end) ----------------------------------------------------
@@ -91,3 +99,58 @@ class LayerPlan:
     def d2h_bytes(self) -> int:
         s = self.spec
         return s.k_max * s.C * s.d + 4 * s.C * s.k_max + 4 * s.C + 4
+
+
+class NetworkPlan:
+    """Every layer of a network through the path, layers spread over a pool of CUDA streams.
+
+    Layers are independent (each has its own weights, calibration inputs and outputs), so their
+    four-call chains run concurrently: small layers that cannot fill the GPU on their own overlap
+    with the large ones.  Layers are issued largest first; the pool is forked from and joined back
+    to the caller's stream, so the call as a whole is ordered like any single launch on it.
+    """
+
+    def __init__(self, specs, device, n_streams: int = 8, with_reconstruct: bool = True):
+        self.device = torch.device(device)
+        self.plans = [LayerPlan(s, self.device, with_reconstruct) for s in specs]
+        work = [s.C * s.d * s.G * s.k_max + s.C * s.d * s.N for s in specs]
+        self.order = sorted(range(len(specs)), key=lambda i: -work[i])
+        self.streams = [torch.cuda.Stream(self.device) for _ in range(max(1, n_streams))]
+
+    def _fork(self, main):
+        start = torch.cuda.Event()
+        start.record(main)
+        for s in self.streams:
+            s.wait_event(start)
+
+    def _join(self, main):
+        for s in self.streams:
+            e = torch.cuda.Event()
+            e.record(s)
+            main.wait_event(e)
+
+    def run_device(self, Ws, Xs, stream=None, on_layer=None):
+        """Ws[i], Xs[i]: device inputs of layer i.  on_layer(i, stream, phase), if given, is
+        called around layer i's calls as LayerPlan.run_device's timing hook (phases 0..4)."""
+        main = stream or torch.cuda.current_stream(self.device)
+        self._fork(main)
+        for n, i in enumerate(self.order):
+            st = self.streams[n % len(self.streams)]
+            hook = None if on_layer is None else (lambda ph, st=st, i=i: on_layer(i, st, ph))
+            self.plans[i].run_device(Ws[i], Xs[i], stream=st, timing=hook)
+        self._join(main)
+        return self
+
+    def run_host(self, W_hosts, X_hosts, W_devs, X_devs, stream=None):
+        """End to end: per layer, H2D of W and X from pinned memory, the path, D2H of codes,
+        scales, point counts; each layer on its own stream so copies overlap other layers'
+        kernels.  The caller synchronizes ``stream`` before reading the host outputs."""
+        main = stream or torch.cuda.current_stream(self.device)
+        self._fork(main)
+        outs = [None] * len(self.plans)
+        for n, i in enumerate(self.order):
+            st = self.streams[n % len(self.streams)]
+            outs[i] = self.plans[i].run_host(W_hosts[i], X_hosts[i], W_devs[i], X_devs[i],
+                                             stream=st)
+        self._join(main)
+        return outs

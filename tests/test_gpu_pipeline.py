@@ -89,3 +89,23 @@ def test_full_size_sampled(gpu, oracle, key, layers):
         n_or, used_or = oracle.allocate_budget(plan.err.cpu().numpy(), wl.k_max, wl.beta)
         assert np.array_equal(plan.npoints.cpu().numpy(), n_or)
         assert int(plan.points_used.item()) == used_or
+
+
+def test_network_plan_streams_match_single_stream(gpu):
+    """Layers spread over 8 streams give bit-identical outputs to one stream (layers are
+    independent; every kernel is deterministic)."""
+    wl = wlm.WORKLOADS["c2"]
+    idx = [0, 1, 5, 7, 12, 16, 20]
+    specs, Ws, Xs = [], [], []
+    for li in idx:
+        layer = wl.layers[li]
+        specs.append(pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, bits=4, G=wl.G,
+                                        k_max=wl.k_max, budget_or_eps=wl.beta))
+        Ws.append(torch.from_numpy(wlm.make_weights(wl, li)).to(gpu))
+        Xs.append(torch.from_numpy(wlm.make_calibration(wl, li)).to(gpu))
+    many = pipeline.NetworkPlan(specs, gpu, n_streams=8).run_device(Ws, Xs)
+    one = pipeline.NetworkPlan(specs, gpu, n_streams=1).run_device(Ws, Xs)
+    torch.cuda.synchronize()
+    for a, b in zip(many.plans, one.plans):
+        for name in ("codes", "scales", "resid_sq", "err", "npoints", "points_used", "W_hat"):
+            assert torch.equal(getattr(a, name), getattr(b, name)), name
