@@ -150,6 +150,18 @@ def kernel_units(wl, layer):
     return layer.C * layer.d * wl.G * wl.k_max
 
 
+def quantize_bytes(wl, layer):
+    """Algorithmic HBM bytes of one mpq_quantize_layer call: read W once, write k_max code planes,
+    the scales and the residual norms."""
+    return layer.C * (layer.d * (4 + wl.k_max) + 4 * wl.k_max + 4 * (wl.k_max + 1))
+
+
+def reconstruct_bytes(wl, layer):
+    """Algorithmic HBM bytes of one mpq_reconstruct call at the budget's average point count:
+    n_avg code bytes + one fp32 write per weight (scales and counts are negligible)."""
+    return layer.C * layer.d * (wl.beta + 4)
+
+
 def contraction_flops(wl, layer):
     """Algorithmic flops of Eq. 11 for one layer: 2 * N * d * C * (k_max + 1)."""
     return 2 * wl.n_calib * layer.d * layer.C * (wl.k_max + 1)
@@ -250,8 +262,9 @@ def run_ours(args, world, rank, local):
                 for k, f in enumerate(families):
                     fam_ms[f] += e[k].elapsed_time(e[k + 1])
                 fam_work["output_error"] += contraction_flops(wl, layer)
-                fam_work["quantize"] += kernel_units(wl, layer)
-                fam_work["reconstruct"] += layer.C * layer.d * (4 + 1 + 4 / wl.k_max)
+                fam_work["quantize"] += quantize_bytes(wl, layer)
+                fam_work["reconstruct"] += reconstruct_bytes(wl, layer)
+                fam_work["allocate"] += 4 * layer.C * (wl.k_max + 1) * 9 + 8 * layer.C
     total_fam = sum(fam_ms.values())
     dominant = max(fam_ms, key=fam_ms.get)
 
@@ -284,7 +297,16 @@ def run_ours(args, world, rank, local):
     return out if rank == 0 else None
 
 
+TF32_PER_BF16 = 1.1 / 2.25   # nominal dense tf32 / bf16 tensor rates of the part
+
+
 def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
+    """Roofline entry of the kernel family with the largest measured time.
+
+    output_error: tensor-pipe bound; achieved = algorithmic flops 2*N*d*C*(k_max+1) (the three
+      tf32 split passes are not counted) / measured time; peak = measured bf16 dense burst peak x
+      the nominal tf32/bf16 ratio.
+    quantize / reconstruct / allocate: HBM roofline; achieved = algorithmic bytes / time."""
     traffic = None
     tfile = os.path.join(PROFILES, "roofline_traffic.json")
     if os.path.exists(tfile):
@@ -292,31 +314,25 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
             tr = json.load(f)
         ent = tr.get(args.config, {}).get(dominant)
         if ent and ent.get("source_sha") == src_hash(KERNEL_SOURCES[dominant]):
-            traffic = ent.get("dram_bytes_per_step")
+            traffic = ent.get("dram_bytes_per_launch")
     t_s = fam_ms[dominant] / 1e3
+    launches = args.steps * len(wl.bits) * fam_work.get("_layers", 1)
     if dominant == "output_error":
-        # fp32 CUDA-core contraction: peak = 2 flops x 128 FFMA lanes x SMs x max SM clock
-        import torch
-        sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
-        peak = 2 * 128 * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        peak = peaks["bf16_tflops"] * TF32_PER_BF16
         ach = fam_work[dominant] / t_s / 1e12
-        return {"kernel": "output_error (Eq. 11 contraction, fp32 FFMA)", "bound": "alu",
-                "achieved": ach, "peak": peak, "unit": "TFLOP/s", "frac": ach / peak,
-                "traffic": traffic, "peak_source": f"derived: 2*128*{sms} SMs*max SM clock "
-                                                   f"({peak_src} clock)"}
-    if dominant == "quantize":
-        import torch
-        sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
-        ops_per_unit = 8  # minimal fp32/int ops per (element, candidate) of the direct search
-        peak = 128 * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
-        ach = fam_work[dominant] * ops_per_unit / t_s / 1e12
-        return {"kernel": "quantize (Eq. 9 scale search)", "bound": "alu", "achieved": ach,
-                "peak": peak, "unit": "Tops/s", "frac": ach / peak, "traffic": traffic,
-                "peak_source": f"derived: 128 lanes*{sms} SMs*max SM clock ({peak_src} clock)"}
+        return {"kernel": "output_error_tc_kernel (Eq. 11, tcgen05 kind::tf32, 3-pass split)",
+                "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                "frac": ach / peak, "traffic": traffic,
+                "peak_source": f"{peak_src} bf16 dense burst x nominal tf32/bf16 ratio "
+                               f"{TF32_PER_BF16:.3f}"}
     hbm = peaks["hbm_gbs"]
     ach = fam_work.get(dominant, 0.0) / t_s / 1e9
-    return {"kernel": dominant, "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
-            "frac": ach / hbm, "traffic": traffic, "peak_source": peak_src}
+    names = {"quantize": "quantize_event_kernel (Eq. 7-9, all k_max steps)",
+             "reconstruct": "reconstruct_vec4_kernel (Eq. 4)",
+             "allocate": "allocate_budget_kernel (Algorithm 2)"}
+    return {"kernel": names.get(dominant, dominant), "bound": "hbm", "achieved": ach, "peak": hbm,
+            "unit": "GB/s", "frac": ach / hbm, "traffic": traffic,
+            "peak_source": f"{peak_src} HBM copy"}
 
 
 def run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step):

@@ -90,6 +90,27 @@ __device__ float block_max(float v, Reduce &sh)
     return m;
 }
 
+// Block-wide max of non-negative floats and sum of doubles in one pass (fixed tree).
+__device__ void block_max_sum(float &m, double &v, Reduce &sh)
+{
+    m = warp_max(m);
+    v = warp_sum(v);
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    __syncthreads();
+    if (lane == 0) {
+        sh.f[w] = m;
+        sh.dd[w] = v;
+    }
+    __syncthreads();
+    m = sh.f[0];
+    v = 0.0;
+#pragma unroll
+    for (int i = 0; i < QWARPS; ++i) {
+        m = fmaxf(m, sh.f[i]);
+        v += sh.dd[i];
+    }
+}
+
 // Block-wide sums, fixed reduction tree (deterministic).
 __device__ double block_sum(double v, Reduce &sh)
 {
@@ -232,14 +253,18 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
 
     int bad = 0;
     float part = 0.0f;
+    float am = 0.0f;
     for (int j = tid; j < d; j += QBLOCK) {
         float v = w[j];
         sr[j] = v;
         bad |= !isfinite(v);
         part = fmaf(v, v, part);
+        am = fmaxf(am, fabsf(v));
     }
     bad = __syncthreads_or(bad);
-    double r2 = block_sum((double)part, red);
+    float m = am;                 // max |r| of the current residual (exact)
+    double r2 = (double)part;
+    block_max_sum(m, r2, red);
     if (resid_sq && tid == 0) resid_sq[(size_t)k * (k_max + 1)] = bad ? NAN : (float)r2;
 
     for (int i = 0; i < k_max; ++i) {
@@ -257,11 +282,7 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
             continue;
         }
 
-        float am = 0.0f;
-        for (int j = tid; j < d; j += QBLOCK) am = fmaxf(am, fabsf(sr[j]));
-        const float m = block_max(am, red);
-
-        float s_best = 0.0f;
+        float s_best = 0.0f, inv_best = 0.0f;
         if (m > 0.0f) {
             const float smax = __fdiv_rn(m, qmaxf);
             int e;
@@ -294,9 +315,10 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
                 for (int j = tid; j < d; j += QBLOCK) {
                     const float a = fabsf(sr[j]);
                     if (a == 0.0f) continue;
-                    const long long R = fixed_point(a, S);
                     const int c_hi = code_fast(a, s0, i0, qmaxf);
+                    if (c_hi == 0) continue;   // code 0 at every scale: no contribution
                     const int c_lo = code_fast(a, sG, iG, qmaxf);
+                    const long long R = fixed_point(a, S);
                     Pb += R * (long long)c_lo;
                     Nb += (long long)c_lo * c_lo;
                     const unsigned int Rlo = (unsigned int)R;
@@ -315,7 +337,21 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
                             }
                             T = lo;
                         } else {
-                            T = (int)fminf(fmaxf(floorf(ag * s_hinv[L]), 1.0f), (float)(G - 1));
+                            // s_g = (g+1)/G * smax up to two fp32 roundings and x is a*G/(smax*h)
+                            // up to 2^-22, so unless x is within 2^-20 x of an integer, level L
+                            // is held exactly for g + 1 < x: T = floor(x) with no further check.
+                            const float x = ag * s_hinv[L];
+                            const float fx = floorf(x);
+                            const float tolx = MPQ_FAST_REL * x;
+                            T = (int)fminf(fmaxf(fx, 1.0f), (float)(G - 1));
+                            if (x - fx > tolx && fx + 1.0f - x > tolx && fx >= 1.0f &&
+                                fx <= (float)(G - 1)) {
+                                const unsigned int old = atomicAdd(&hPw[2 * T], Rlo);
+                                const unsigned int carry = (old + Rlo < old) ? 1u : 0u;
+                                if (Rhi + carry) atomicAdd(&hPw[2 * T + 1], Rhi + carry);
+                                atomicAdd(&hN[T], 2 * L - 1);
+                                continue;
+                            }
                         }
                         const bool up = (T < G - 1) && level_held(a, stab[T], sinv[T], L);
                         const bool down = !up && (T > 1) && !level_held(a, stab[T - 1], sinv[T - 1], L);
@@ -397,15 +433,18 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
             int g = block_argmin(bestD, bestg, red);
             if (g < 0 || g >= G) g = G - 1;   // unreachable: every D is finite
             s_best = stab[g];
+            inv_best = sinv[g];
         }
 
-        // residual update (Eq. 7) and code emission
+        // residual update (Eq. 7) and code emission; also the next step's max |r|
         part = 0.0f;
+        am = 0.0f;
         for (int j = tid; j < d; j += QBLOCK) {
             float v = sr[j];
             int q = 0;
             if (s_best > 0.0f) {
-                const int c = code_mag(fabsf(v), s_best, qmaxf);
+                const int c = (inv_best > 0.0f) ? code_fast(fabsf(v), s_best, inv_best, qmaxf)
+                                                : code_mag(fabsf(v), s_best, qmaxf);
                 q = (v < 0.0f) ? -c : c;
                 v = __fmaf_rn(-s_best, (float)q, v);
             }
@@ -413,9 +452,12 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
             sr[j] = v;
             if (ri) ri[j] = v;
             part = fmaf(v, v, part);
+            am = fmaxf(am, fabsf(v));
         }
         if (tid == 0) scales[(size_t)k * k_max + i] = s_best;
-        r2 = block_sum((double)part, red);   // also orders the sr[] writes before the next step
+        m = am;
+        r2 = (double)part;
+        block_max_sum(m, r2, red);   // also orders the sr[] writes before the next step
         if (resid_sq && tid == 0) resid_sq[(size_t)k * (k_max + 1) + i + 1] = (float)r2;
     }
 }
