@@ -32,7 +32,7 @@ METRIC = "weight-elements x scale-candidates x points / s"
 UNIT = "elem*cand*pt/s"
 PROFILES = os.path.join(ROOT, "profiles")
 KERNEL_SOURCES = {
-    "output_error": "paper_2002_09049_gb300/csrc/output_error.cu",
+    "output_error": "paper_2002_09049_gb300/csrc/output_error_tc.cu",
     "quantize": "paper_2002_09049_gb300/csrc/quantize.cu",
     "allocate": "paper_2002_09049_gb300/csrc/allocate.cu",
     "reconstruct": "paper_2002_09049_gb300/csrc/reconstruct.cu",

@@ -1,27 +1,34 @@
 // Greedy multipoint construction (Sec. 3.2, Eq. 6-9, Algorithm 1) for every channel of a layer.
 //
-// One CTA owns one channel for all k_max steps: the residual row r (fp32) stays in shared memory
-// from the first load of w to the last update, so global memory sees one read of w and one write
-// of each step's codes (and of the optional residual / norm outputs).
+// A group of WPC warps (1, 2, 4 or 8; chosen per layer from C, d and shared memory) owns one
+// channel for all k_max steps: the residual row r (fp32) stays in shared memory from the first
+// load of w to the last update, so global memory sees one read of w and one write of each step's
+// codes (and of the optional residual / norm outputs).  Short channels (depthwise 3x3, d = 9) get
+// a single warp and synchronise with warp primitives only; long channels of layers with few
+// channels get up to 8 warps and named barriers.
 //
 // Scale search (Eq. 9).  For a candidate scale s with codes c_j = min(Qmax, rint(|r_j| / s)),
 //   E(s) = ||r - s q||^2 = ||r||^2 - 2 s P + s^2 N,   P = sum_j |r_j| c_j,   N = sum_j c_j^2,
 // so only D(s) = s (s N - 2 P) decides the argmin.  N is an exact integer and P is accumulated
 // exactly in 64-bit fixed point (|r_j| scaled by 2^S, S chosen per step from max|r| so the sum
-// cannot overflow; exact for every element whose code can be nonzero on the grid).  D is then
-// formed once per candidate in double: the decision carries ~1e-16 relative error, independent
-// of d and of summation order, hence deterministic.
+// cannot overflow; exact for every element whose code can be nonzero on the grid).  Every D is
+// first evaluated in fp32 together with a rigorous bound on its rounding error; only the
+// candidates whose interval can hold the minimum are re-evaluated in double, and the lowest index
+// among the exact minima wins.  The result is the argmin of the exact D values: deterministic and
+// independent of d and of the summation order, with the narrow fp64 pipe touched a few times per
+// step.
 //
 // Event form.  The candidate scales increase with g, so every element's code c_j(g) is a
 // non-increasing step function of g (the fp32 quotient, rint and the clamp are all monotone).
 // For each level L, {g : c_j(g) >= L} is a prefix [0, T_{j,L}); hence
 //   P_g = sum_{(j,L)} R_j [g < T_{j,L}],   N_g = sum_{(j,L)} (2L - 1) [g < T_{j,L}].
 // Levels held at the largest scale (L <= c_j(G-1)) count for every g and are summed directly;
-// every other level the element crosses adds (R_j, 2L-1) to a histogram bin T_{j,L}, found by a
-// binary search on the scale table followed by an exact check with the same correctly rounded
-// division and rint as the definition.  A suffix sum over the bins gives P_g and N_g for all g.
-// Work per element and step is O(Qmax) instead of O(G).  (If a candidate scale underflows to 0
-// the monotonicity argument fails; such steps evaluate every candidate directly.)
+// every other level the element crosses adds (R_j, 2L-1) to a histogram bin T_{j,L}.  T is found
+// in closed form on the linear grid (exact unless the estimate falls within 2^-20 of a grid point,
+// where the exact rule settles it) or by bisection on a caller's grid, then checked with the same
+// correctly rounded division and rint as the definition.  A suffix sum over the bins gives P_g and
+// N_g for all g.  Work per element and step is O(Qmax) instead of O(G).  (If a candidate scale
+// underflows to 0 the monotonicity argument fails; such steps evaluate every candidate directly.)
 #include <float.h>
 #include <limits.h>
 #include <math.h>
@@ -31,9 +38,8 @@
 namespace mpq {
 namespace {
 
-constexpr int QBLOCK = 256;
-constexpr int QWARPS = QBLOCK / 32;
-constexpr int MPQ_QMAX_LIMIT = (1 << (MPQ_MAX_BITS - 1)) - 1;
+constexpr int QTHREADS = 256;                                   // 8 warps per CTA
+constexpr int QMAX_LIMIT = (1 << (MPQ_MAX_BITS - 1)) - 1;
 
 template <bool CUSTOM>
 struct Grid;
@@ -53,6 +59,44 @@ struct Grid<true> {
     __device__ __forceinline__ float frac(int g0, int) const { return gf.f[g0]; }
 };
 
+// Per-group scratch for cross-warp reductions.
+struct Scratch {
+    float f[8];
+    float v[8];
+    unsigned long long key[8];
+    long long a[8];
+    long long b[8];
+    int g[8];
+    int flag[8];
+};
+
+// Shared memory: a CTA-wide table of the grid fractions f_g and fl(1/f_g) (2G words), then per
+// channel group (all 4-byte words): WPC private copies (one per warp, so warps never contend on
+// the same bin) of hLo[G+1], hHi[G+1] (64-bit P bins as two words) and hN[G+1], then r[d].
+// With the lattice form (below) each group also holds nb lattice buckets first: 64-bit R sums
+// (2 words each) and 32-bit counts.  Group regions are kept 8-byte aligned.
+__host__ __device__ constexpr size_t lattice_words(int nb)
+{
+    return ((size_t)3 * nb + 1) & ~(size_t)1;
+}
+
+__host__ __device__ constexpr size_t group_words(int G, int d, int wpc, int nb)
+{
+    return lattice_words(nb) + (((size_t)3 * (G + 1) * wpc + (size_t)d + 1) & ~(size_t)1);
+}
+
+template <int WPC>
+__device__ __forceinline__ void gsync(int grp)
+{
+    if (WPC == 1) {
+        __syncwarp();
+    } else if (WPC == 8) {
+        __syncthreads();
+    } else {
+        asm volatile("bar.sync %0, %1;" ::"r"(grp + 1), "r"(WPC * 32) : "memory");
+    }
+}
+
 __device__ __forceinline__ float warp_max(float v)
 {
 #pragma unroll
@@ -68,104 +112,121 @@ __device__ __forceinline__ T warp_sum(T v)
     return v;
 }
 
-struct Reduce {
-    float f[QWARPS];
-    double dd[QWARPS];
-    long long ll[QWARPS];
-    int g[QWARPS];
-    int flag;
-};
-
-// Block-wide max of non-negative floats (exact).
-__device__ float block_max(float v, Reduce &sh)
+__device__ __forceinline__ float warp_min(float v)
 {
-    v = warp_max(v);
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) sh.f[w] = v;
-    __syncthreads();
-    float m = sh.f[0];
 #pragma unroll
-    for (int i = 1; i < QWARPS; ++i) m = fmaxf(m, sh.f[i]);
-    return m;
+    for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
 }
 
-// Block-wide max of non-negative floats and sum of doubles in one pass (fixed tree).
-__device__ void block_max_sum(float &m, double &v, Reduce &sh)
+// Group-wide max (floats >= 0), fp32 sum (fixed tree) and OR, in one exchange.
+template <int WPC>
+__device__ __forceinline__ void group_max_sum_or(float &m, float &v, int &flag, Scratch &sc,
+                                                 int gw, int lane, int grp)
 {
     m = warp_max(m);
     v = warp_sum(v);
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) {
-        sh.f[w] = m;
-        sh.dd[w] = v;
-    }
-    __syncthreads();
-    m = sh.f[0];
-    v = 0.0;
+    flag = __any_sync(0xffffffffu, flag) ? 1 : 0;
+    if (WPC > 1) {
+        gsync<WPC>(grp);
+        if (lane == 0) {
+            sc.f[gw] = m;
+            sc.v[gw] = v;
+            sc.flag[gw] = flag;
+        }
+        gsync<WPC>(grp);
+        m = sc.f[0];
+        v = 0.0f;
+        flag = 0;
 #pragma unroll
-    for (int i = 0; i < QWARPS; ++i) {
-        m = fmaxf(m, sh.f[i]);
-        v += sh.dd[i];
-    }
-}
-
-// Block-wide sums, fixed reduction tree (deterministic).
-__device__ double block_sum(double v, Reduce &sh)
-{
-    v = warp_sum(v);
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) sh.dd[w] = v;
-    __syncthreads();
-    double s = 0.0;
-#pragma unroll
-    for (int i = 0; i < QWARPS; ++i) s += sh.dd[i];
-    return s;
-}
-
-__device__ long long block_sum_ll(long long v, Reduce &sh)
-{
-    v = warp_sum(v);
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) sh.ll[w] = v;
-    __syncthreads();
-    long long s = 0;
-#pragma unroll
-    for (int i = 0; i < QWARPS; ++i) s += sh.ll[i];
-    return s;
-}
-
-// Block-wide lexicographic min of (D, g): smallest D, lowest g among equal D.
-__device__ int block_argmin(double D, int g, Reduce &sh)
-{
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        double D2 = __shfl_xor_sync(0xffffffffu, D, o);
-        int g2 = __shfl_xor_sync(0xffffffffu, g, o);
-        if (D2 < D || (D2 == D && g2 < g)) {
-            D = D2;
-            g = g2;
+        for (int i = 0; i < WPC; ++i) {
+            m = fmaxf(m, sc.f[i]);
+            v += sc.v[i];
+            flag |= sc.flag[i];
         }
     }
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) {
-        sh.dd[w] = D;
-        sh.g[w] = g;
-    }
-    __syncthreads();
-    D = sh.dd[0];
-    g = sh.g[0];
-#pragma unroll
-    for (int i = 1; i < QWARPS; ++i)
-        if (sh.dd[i] < D || (sh.dd[i] == D && sh.g[i] < g)) {
-            D = sh.dd[i];
-            g = sh.g[i];
+}
+
+template <int WPC>
+__device__ __forceinline__ void group_sum2(long long &x, long long &y, Scratch &sc, int gw,
+                                           int lane, int grp)
+{
+    x = warp_sum(x);
+    y = warp_sum(y);
+    gsync<WPC>(grp);   // also publishes this group's shared-memory updates
+    if (WPC > 1) {
+        if (lane == 0) {
+            sc.a[gw] = x;
+            sc.b[gw] = y;
         }
-    return g;
+        gsync<WPC>(grp);
+        x = 0;
+        y = 0;
+#pragma unroll
+        for (int i = 0; i < WPC; ++i) {
+            x += sc.a[i];
+            y += sc.b[i];
+        }
+    }
+}
+
+template <int WPC>
+__device__ __forceinline__ float group_min(float v, Scratch &sc, int gw, int lane, int grp)
+{
+    v = warp_min(v);
+    if (WPC > 1) {
+        gsync<WPC>(grp);
+        if (lane == 0) sc.f[gw] = v;
+        gsync<WPC>(grp);
+        v = sc.f[0];
+#pragma unroll
+        for (int i = 1; i < WPC; ++i) v = fminf(v, sc.f[i]);
+    }
+    return v;
+}
+
+// Order-preserving map of a double to unsigned 64-bit (total order, -0 < +0 is harmless here).
+__device__ __forceinline__ unsigned long long ordered_bits(double x)
+{
+    const unsigned long long b = (unsigned long long)__double_as_longlong(x);
+    return (b >> 63) ? ~b : (b | 0x8000000000000000ull);
+}
+
+__device__ __forceinline__ unsigned long long umin64(unsigned long long a, unsigned long long b)
+{
+    return a < b ? a : b;
+}
+
+// Group-wide lexicographic min of (D, g): smallest D, lowest g among equal D.  The double is
+// reduced as its order-preserving integer image (no fp64 compares), then the lowest g among the
+// lanes that hold that minimum.
+template <int WPC>
+__device__ __forceinline__ int group_argmin(double D, int g, Scratch &sc, int gw, int lane,
+                                            int grp)
+{
+    unsigned long long key = ordered_bits(D);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) key = umin64(key, __shfl_xor_sync(0xffffffffu, key, o));
+    if (WPC > 1) {
+        gsync<WPC>(grp);
+        if (lane == 0) sc.key[gw] = key;
+        gsync<WPC>(grp);
+        key = sc.key[0];
+#pragma unroll
+        for (int i = 1; i < WPC; ++i) key = umin64(key, sc.key[i]);
+    }
+    int cand = (ordered_bits(D) == key) ? g : INT_MAX;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cand = min(cand, __shfl_xor_sync(0xffffffffu, cand, o));
+    if (WPC > 1) {
+        gsync<WPC>(grp);
+        if (lane == 0) sc.g[gw] = cand;
+        gsync<WPC>(grp);
+        cand = sc.g[0];
+#pragma unroll
+        for (int i = 1; i < WPC; ++i) cand = min(cand, sc.g[i]);
+    }
+    return cand;
 }
 
 // Code magnitude of |r| at scale s > 0 (Eq. 8): nearest integer (ties to even) of the correctly
@@ -175,9 +236,9 @@ __device__ __forceinline__ int code_mag(float a, float s, float qmaxf)
     return (int)fminf(rintf(__fdiv_rn(a, s)), qmaxf);
 }
 
-// |r| as a 64-bit fixed-point integer R = |r| * 2^S, from the fp32 bits (no fp64 work).  Exact
-// whenever |r| * 2^S is an integer, i.e. for every element large enough to take a nonzero code;
-// smaller elements are truncated (their P contribution is zero anyway).
+// |r| as a 64-bit fixed-point integer R = |r| * 2^S, from the fp32 bits.  Exact whenever
+// |r| * 2^S is an integer, i.e. for every element large enough to take a nonzero code; smaller
+// elements are truncated (their P contribution is zero anyway).
 __device__ __forceinline__ long long fixed_point(float a, int S)
 {
     const uint32_t bits = __float_as_uint(a);
@@ -188,10 +249,16 @@ __device__ __forceinline__ long long fixed_point(float a, int S)
     return sh > -40 ? (M >> -sh) : 0;
 }
 
+// 2^k as a double, built from its bits (k within the normal range).
+__device__ __forceinline__ double pow2d(int k)
+{
+    return __longlong_as_double((long long)(1023 + k) << 52);
+}
+
 // Bound on |a * fl(1/s) - fl(a/s)| relative to the quotient, with margin: both roundings are
 // 2^-24 each, so a fast quotient further than this from a rounding boundary decides exactly as
 // the correctly rounded division would.
-#define MPQ_FAST_REL 9.5367431640625e-07f   /* 2^-20 */
+#define MPQ_FAST_REL 9.5367431640625e-07f /* 2^-20 */
 
 // rint(fl(a/s)) >= L, decided from q' = a * (1/s) unless q' is too close to L - 1/2.
 __device__ __forceinline__ bool level_held(float a, float s, float inv_s, int L)
@@ -224,58 +291,107 @@ __device__ __forceinline__ double decision(float s, long long Pfix, long long N,
     return __dmul_rn(sd, T);
 }
 
-template <bool CUSTOM>
-__global__ void __launch_bounds__(QBLOCK, 4)
-quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G,
-                      const Grid<CUSTOM> grid, int k_max, int8_t *__restrict__ codes,
-                      float *__restrict__ scales, float *__restrict__ resid_sq,
-                      float *__restrict__ residuals, int hbits)
+__device__ __forceinline__ void kahan_add(float &sum, float &comp, float x)
 {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    // Event bins.  P bins are 64-bit values kept as two 32-bit words (32-bit shared atomics are
-    // native; 64-bit ones are several times slower under contention): the low word takes an
-    // atomic add whose returned old value shows every wrap-around exactly, and the high word
-    // takes R >> 32 plus that carry.  After the events hP holds the combined 64-bit sums.
-    long long *hP = reinterpret_cast<long long *>(smem_raw);    // [G + 1] P bins (lo | hi words)
-    int *hN = reinterpret_cast<int *>(hP + (G + 1));             // [G + 1] event bins of N
-    float *stab = reinterpret_cast<float *>(hN + (G + 1));       // [G] candidate scales
-    float *sinv = stab + G;                                       // [G] fl(1 / scale)
-    float *sr = sinv + G;                                         // [d] residual
-    __shared__ Reduce red;
-    __shared__ float s_hinv[MPQ_QMAX_LIMIT + 1];   // 1 / (L - 1/2): threshold estimates only
+    const float y = __fsub_rn(x, comp);
+    const float t = __fadd_rn(sum, y);
+    comp = __fsub_rn(__fsub_rn(t, sum), y);
+    sum = t;
+}
 
-    const int tid = threadIdx.x;
-    const int k = blockIdx.x;
+__device__ __forceinline__ void add_event(unsigned int *hLo, unsigned int *hHi, int *hN, int T,
+                                          unsigned int Rlo, unsigned int Rhi, int L)
+{
+    const unsigned int old = atomicAdd(&hLo[T], Rlo);
+    const unsigned int carry = (old + Rlo < old) ? 1u : 0u;   // exact wrap-around of the low word
+    if (Rhi + carry) atomicAdd(&hHi[T], Rhi + carry);
+    atomicAdd(&hN[T], 2 * L - 1);
+}
+
+__device__ __forceinline__ long long bin64(const unsigned int *hLo, const unsigned int *hHi, int t)
+{
+    return (long long)(((unsigned long long)hHi[t] << 32) | hLo[t]);
+}
+
+// Int64 -> fp32 without the fp64 pipe: two exact 32-bit halves, three roundings in total.
+__device__ __forceinline__ float i64_to_f32(long long x)
+{
+    const float hi = (float)(int)(x >> 32);
+    const float lo = (float)(unsigned int)x;
+    return __fmaf_rn(hi, 4294967296.0f, lo);
+}
+
+template <int WPC, bool CUSTOM, bool LAT>
+__global__ void __launch_bounds__(QTHREADS, 4)
+quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, const Grid<CUSTOM> grid,
+                int k_max, int8_t *__restrict__ codes, float *__restrict__ scales,
+                float *__restrict__ resid_sq, float *__restrict__ residuals, int hbits)
+{
+    const int nb = LAT ? 2 * G * qmax + 1 : 0;   // lattice buckets: floor(2u) in [0, 2 G Qmax]
+    constexpr int NT = WPC * 32;
+    constexpr int GPC = 8 / WPC;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    __shared__ Scratch scratch[GPC];
+    __shared__ float s_hinv[QMAX_LIMIT + 1];   // 1 / (L - 1/2): threshold estimates only
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int grp = warp / WPC, gw = warp % WPC, gt = gw * 32 + lane;
+    const int k = blockIdx.x * GPC + grp;
     const float qmaxf = (float)qmax;
-    for (int L = tid; L <= qmax; L += QBLOCK) s_hinv[L] = 1.0f / ((float)L - 0.5f);
+    float *fgrid = reinterpret_cast<float *>(smem_raw);   // [G] f_g
+    float *finv = fgrid + G;                              // [G] fl(1 / f_g)
+    for (int L = threadIdx.x; L <= qmax; L += QTHREADS) s_hinv[L] = 1.0f / ((float)L - 0.5f);
+    for (int g = threadIdx.x; g < G; g += QTHREADS) {
+        const float f = grid.frac(g, G);
+        fgrid[g] = f;
+        finv[g] = __frcp_rn(f);
+    }
+    __syncthreads();
+    if (k >= C) return;   // whole group idle (group-uniform)
+
+    unsigned int *gl =
+        reinterpret_cast<unsigned int *>(finv + G) + (size_t)grp * group_words(G, d, WPC, nb);
+    unsigned long long *latR = reinterpret_cast<unsigned long long *>(gl);   // [nb]
+    unsigned int *latC = gl + 2 * (size_t)nb;                                 // [nb]
+    unsigned int *gbase = gl + lattice_words(nb);
+    // this warp's private bins; copy 0 receives the merged suffix sums
+    unsigned int *hLo = gbase + (size_t)gw * 3 * (G + 1);
+    unsigned int *hHi = hLo + (G + 1);
+    int *hN = reinterpret_cast<int *>(hHi + (G + 1));
+    unsigned int *mLo = gbase;
+    unsigned int *mHi = mLo + (G + 1);
+    int *mN = reinterpret_cast<int *>(mHi + (G + 1));
+    float *sr = reinterpret_cast<float *>(gbase + (size_t)3 * (G + 1) * WPC);
+    Scratch &sc = scratch[grp];
+
     const size_t plane = (size_t)C * d;
     const float *w = W + (size_t)k * d;
+    const float pscale = ldexpf(1.0f, hbits - 62);   // P * 2^-S / 2^e for the fp32 screen
 
     int bad = 0;
-    float part = 0.0f;
-    float am = 0.0f;
-    for (int j = tid; j < d; j += QBLOCK) {
-        float v = w[j];
+    float ssum = 0.0f, scomp = 0.0f, am = 0.0f;
+    for (int j = gt; j < d; j += NT) {
+        const float v = w[j];
         sr[j] = v;
         bad |= !isfinite(v);
-        part = fmaf(v, v, part);
+        kahan_add(ssum, scomp, v * v);
         am = fmaxf(am, fabsf(v));
     }
-    bad = __syncthreads_or(bad);
-    float m = am;                 // max |r| of the current residual (exact)
-    double r2 = (double)part;
-    block_max_sum(m, r2, red);
-    if (resid_sq && tid == 0) resid_sq[(size_t)k * (k_max + 1)] = bad ? NAN : (float)r2;
+    float m = am;
+    float r2 = ssum;
+    group_max_sum_or<WPC>(m, r2, bad, sc, gw, lane, grp);
+    if (WPC == 1) __syncwarp();
+    if (resid_sq && gt == 0) resid_sq[(size_t)k * (k_max + 1)] = bad ? NAN : r2;
 
     for (int i = 0; i < k_max; ++i) {
         int8_t *qi = codes + (size_t)i * plane + (size_t)k * d;
         float *ri = residuals ? residuals + (size_t)i * plane + (size_t)k * d : nullptr;
         if (bad) {
-            for (int j = tid; j < d; j += QBLOCK) {
+            for (int j = gt; j < d; j += NT) {
                 qi[j] = 0;
                 if (ri) ri[j] = sr[j];
             }
-            if (tid == 0) {
+            if (gt == 0) {
                 scales[(size_t)k * k_max + i] = NAN;
                 if (resid_sq) resid_sq[(size_t)k * (k_max + 1) + i + 1] = NAN;
             }
@@ -284,37 +400,57 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
 
         float s_best = 0.0f, inv_best = 0.0f;
         if (m > 0.0f) {
+            // candidate scales s_g = fl(f_g * smax) exactly as defined; fl(1/f_g) * fl(1/smax)
+            // is within 2^-22 of 1/s_g, which the fast decisions' 2^-20 margin absorbs
             const float smax = __fdiv_rn(m, qmaxf);
+            const float ism = __frcp_rn(smax);
             int e;
             frexpf(m, &e);                      // m < 2^e
             const int S = 62 - e - hbits;       // sum_j R_j c_j < 2^62
-            const double down = ldexp(1.0, -S);
-            int zero_scale = 0;
-            for (int g = tid; g < G; g += QBLOCK) {
-                const float s = __fmul_rn(grid.frac(g, G), smax);
-                stab[g] = s;
-                sinv[g] = (s > 0.0f) ? __frcp_rn(s) : 0.0f;
-                zero_scale |= (s == 0.0f);
-            }
-            for (int t = tid; t <= G; t += QBLOCK) {
-                hP[t] = 0;
+            const double down = pow2d(-S);
+            const float smax_e = ldexpf(smax, -e);   // smax / 2^e for the fp32 screen
+            for (int t = lane; t <= G; t += 32) {   // each warp clears its own copy
+                hLo[t] = 0u;
+                hHi[t] = 0u;
                 hN[t] = 0;
             }
-            zero_scale = __syncthreads_or(zero_scale);
+            if (LAT)
+                for (int t = gt; t < nb; t += NT) {
+                    latR[t] = 0ull;
+                    latC[t] = 0u;
+                }
+            gsync<WPC>(grp);
+            const bool zero_scale = __fmul_rn(fgrid[0], smax) == 0.0f;   // s_g increases with g
 
             double bestD = DBL_MAX;
             int bestg = INT_MAX;
             if (!zero_scale) {
                 // ---- events: one per (element, level crossed inside the grid)
-                const float s0 = stab[0], sG = stab[G - 1];
-                const float i0 = sinv[0], iG = sinv[G - 1];
-                const float g_per_a = __fdiv_rn((float)G, smax);   // default grid: s_g ~ (g+1)/G*smax
-                unsigned int *hPw = reinterpret_cast<unsigned int *>(hP);   // [2*(G+1)] lo, hi
+                const float s0 = __fmul_rn(fgrid[0], smax), sG = __fmul_rn(fgrid[G - 1], smax);
+                const float i0 = finv[0] * ism, iG = finv[G - 1] * ism;
+                const float g_per_a = __fdiv_rn((float)G, smax);   // linear grid: s_g ~ (g+1)/G*smax
                 long long Pb = 0;
                 long long Nb = 0;
-                for (int j = tid; j < d; j += QBLOCK) {
+                for (int j = gt; j < d; j += NT) {
                     const float a = fabsf(sr[j]);
                     if (a == 0.0f) continue;
+                    if (LAT) {
+                        // Linear grid: level L is held at g iff u >= (g+1)(L - 1/2), u = aG/smax,
+                        // i.e. iff floor(2u) >= (g+1)(2L-1), an integer.  Unless 2u lies within
+                        // 2^-20 (relative) of an integer, one bucket update records the element
+                        // for every (g, L) exactly; near a lattice point the per-level events
+                        // below settle each threshold with the exact rule.
+                        const float u2 = 2.0f * (a * g_per_a);
+                        if (fabsf(u2 - rintf(u2)) > MPQ_FAST_REL * u2) {
+                            const int b = (int)floorf(u2);
+                            if (b >= 1) {
+                                const int bb = b < nb - 1 ? b : nb - 1;
+                                atomicAdd(&latR[bb], (unsigned long long)fixed_point(a, S));
+                                atomicAdd(&latC[bb], 1u);
+                            }
+                            continue;
+                        }
+                    }
                     const int c_hi = code_fast(a, s0, i0, qmaxf);
                     if (c_hi == 0) continue;   // code 0 at every scale: no contribution
                     const int c_lo = code_fast(a, sG, iG, qmaxf);
@@ -329,11 +465,11 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
                         // then settle with the exact rule (level_held is monotone in g)
                         int T;
                         if (CUSTOM) {
-                            const float s_est = a * s_hinv[L];
+                            const float f_est = a * s_hinv[L] * ism;
                             int lo = 1, hi = G - 1;
                             while (lo < hi) {
                                 const int mid = (lo + hi) >> 1;
-                                if (stab[mid] < s_est) lo = mid + 1; else hi = mid;
+                                if (fgrid[mid] < f_est) lo = mid + 1; else hi = mid;
                             }
                             T = lo;
                         } else {
@@ -346,73 +482,148 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
                             T = (int)fminf(fmaxf(fx, 1.0f), (float)(G - 1));
                             if (x - fx > tolx && fx + 1.0f - x > tolx && fx >= 1.0f &&
                                 fx <= (float)(G - 1)) {
-                                const unsigned int old = atomicAdd(&hPw[2 * T], Rlo);
-                                const unsigned int carry = (old + Rlo < old) ? 1u : 0u;
-                                if (Rhi + carry) atomicAdd(&hPw[2 * T + 1], Rhi + carry);
-                                atomicAdd(&hN[T], 2 * L - 1);
+                                add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
                                 continue;
                             }
                         }
-                        const bool up = (T < G - 1) && level_held(a, stab[T], sinv[T], L);
-                        const bool down = !up && (T > 1) && !level_held(a, stab[T - 1], sinv[T - 1], L);
+#define MPQ_HELD(t) level_held(a, __fmul_rn(fgrid[t], smax), finv[t] * ism, L)
+                        const bool up = (T < G - 1) && MPQ_HELD(T);
+                        const bool dn = !up && (T > 1) && !MPQ_HELD(T - 1);
                         if (up) {
                             ++T;
-                            while (T < G - 1 && level_held(a, stab[T], sinv[T], L)) ++T;
-                        } else if (down) {
+                            while (T < G - 1 && MPQ_HELD(T)) ++T;
+                        } else if (dn) {
                             --T;
-                            while (T > 1 && !level_held(a, stab[T - 1], sinv[T - 1], L)) --T;
+                            while (T > 1 && !MPQ_HELD(T - 1)) --T;
                         }
-                        const unsigned int old = atomicAdd(&hPw[2 * T], Rlo);
-                        const unsigned int carry = (old + Rlo < old) ? 1u : 0u;
-                        if (Rhi + carry) atomicAdd(&hPw[2 * T + 1], Rhi + carry);
-                        atomicAdd(&hN[T], 2 * L - 1);
+#undef MPQ_HELD
+                        add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
                     }
                 }
-                const long long Pbase = block_sum_ll(Pb, red);
-                const long long Nbase = block_sum_ll(Nb, red);   // also orders the bin updates
-                // ---- suffix sums over the bins (warp 0), in place: bin t <- sum_{u >= t}, so
-                // that P_g = Pbase + hP[g + 1].  Each lane owns bins (b0, b1].
-                if (tid < 32) {
+                group_sum2<WPC>(Pb, Nb, sc, gw, lane, grp);   // publishes the bins too
+                const long long Pbase = Pb, Nbase = Nb;
+                // ---- suffix sums over the bins (warp 0 of the group), in place: bin t <- sum
+                // of bins u >= t, so that P_g = Pbase + bin(g + 1).  Each lane owns (b0, b1].
+                if (gw == 0) {
                     const int per = (G + 31) / 32;
-                    const int b0 = min(G, tid * per), b1 = min(G, b0 + per);
-                    long long sp = 0;
-                    long long sn = 0;
+                    const int b0 = min(G, lane * per), b1 = min(G, b0 + per);
+                    long long sp = 0, sn = 0;
                     for (int t = b0 + 1; t <= b1; ++t) {
-                        sp += hP[t];
-                        sn += hN[t];
+                        // merge the warps' private copies into copy 0
+                        long long p = bin64(mLo, mHi, t);
+                        int n = mN[t];
+#pragma unroll
+                        for (int c = 1; c < WPC; ++c) {
+                            const unsigned int *cLo = mLo + (size_t)c * 3 * (G + 1);
+                            p += bin64(cLo, cLo + (G + 1), t);
+                            n += reinterpret_cast<const int *>(cLo + 2 * (G + 1))[t];
+                        }
+                        mLo[t] = (unsigned int)p;
+                        mHi[t] = (unsigned int)((unsigned long long)p >> 32);
+                        mN[t] = n;
+                        sp += p;
+                        sn += n;
                     }
-                    // inclusive scan toward lower lanes: lane l gets the totals of lanes >= l
-                    long long xp = sp, xn = sn;
+                    long long xp = sp, xn = sn;   // inclusive scan toward lower lanes
 #pragma unroll
                     for (int o = 1; o < 32; o <<= 1) {
                         const long long yp = __shfl_down_sync(0xffffffffu, xp, o);
                         const long long yn = __shfl_down_sync(0xffffffffu, xn, o);
-                        if (tid + o < 32) {
+                        if (lane + o < 32) {
                             xp += yp;
                             xn += yn;
                         }
                     }
                     long long rp = xp - sp, rn = xn - sn;   // bins beyond b1
                     for (int t = b1; t > b0; --t) {
-                        rp += hP[t];
-                        rn += hN[t];
-                        hP[t] = rp;
-                        hN[t] = (int)rn;
+                        rp += bin64(mLo, mHi, t);
+                        rn += mN[t];
+                        mLo[t] = (unsigned int)rp;
+                        mHi[t] = (unsigned int)((unsigned long long)rp >> 32);
+                        mN[t] = (int)rn;
                     }
                 }
-                __syncthreads();
-                for (int g = tid; g < G; g += QBLOCK) {
-                    const double D = decision(stab[g], Pbase + hP[g + 1],
-                                              Nbase + (long long)hN[g + 1], down);
-                    if (D < bestD) {
-                        bestD = D;
-                        bestg = g;
+                if (LAT && gw == (WPC > 1 ? 1 : 0)) {
+                    // suffix sums over the lattice buckets, in place: bucket t <- sum_{u >= t}
+                    const int per = (nb + 31) / 32;
+                    const int b0 = min(nb, lane * per), b1 = min(nb, b0 + per);
+                    unsigned long long sp = 0;
+                    unsigned int sn = 0;
+                    for (int t = b0; t < b1; ++t) {
+                        sp += latR[t];
+                        sn += latC[t];
+                    }
+                    unsigned long long xp = sp;
+                    unsigned int xn = sn;
+#pragma unroll
+                    for (int o = 1; o < 32; o <<= 1) {
+                        const unsigned long long yp = __shfl_down_sync(0xffffffffu, xp, o);
+                        const unsigned int yn = __shfl_down_sync(0xffffffffu, xn, o);
+                        if (lane + o < 32) {
+                            xp += yp;
+                            xn += yn;
+                        }
+                    }
+                    unsigned long long rp = xp - sp;
+                    unsigned int rn = xn - sn;
+                    for (int t = b1 - 1; t >= b0; --t) {
+                        rp += latR[t];
+                        rn += latC[t];
+                        latR[t] = rp;
+                        latC[t] = rn;
+                    }
+                }
+                gsync<WPC>(grp);
+                if (LAT) {
+                    // fold the lattice into the merged bins: bin(g + 1) += sum_L bucket((g+1)(2L-1))
+                    for (int g = gt; g < G; g += NT) {
+                        long long p = bin64(mLo, mHi, g + 1);
+                        long long n = mN[g + 1];
+                        for (int L = 1; L <= qmax; ++L) {
+                            const int b = (g + 1) * (2 * L - 1);
+                            p += (long long)latR[b];
+                            n += (long long)(2 * L - 1) * latC[b];
+                        }
+                        mLo[g + 1] = (unsigned int)p;
+                        mHi[g + 1] = (unsigned int)((unsigned long long)p >> 32);
+                        mN[g + 1] = (int)n;
+                    }
+                    gsync<WPC>(grp);
+                }
+                // ---- fp32 screen of D / 2^2e = s'(s'N - 2P') with s' = s / 2^e and
+                // P' = P 2^-S / 2^e (both O(1) by construction): keep every candidate whose error
+                // interval can contain the minimum, then decide among those in double.  The
+                // inputs carry at most ~8 roundings of 2^-24, the bound allows 2^-20.
+                float upper = FLT_MAX;
+                for (int g = gt; g < G; g += NT) {
+                    const float sh = fgrid[g] * smax_e;
+                    const float Nf = (float)(int)(Nbase + mN[g + 1]);
+                    const float Pf = i64_to_f32(Pbase + bin64(mLo, mHi, g + 1)) * pscale;
+                    const float D32 = sh * (sh * Nf - 2.0f * Pf);
+                    const float err = sh * (sh * Nf + 2.0f * Pf) * MPQ_FAST_REL;
+                    upper = fminf(upper, D32 + err);
+                }
+                upper = group_min<WPC>(upper, sc, gw, lane, grp);
+                for (int g = gt; g < G; g += NT) {
+                    const float sh = fgrid[g] * smax_e;
+                    const long long Pg = Pbase + bin64(mLo, mHi, g + 1);
+                    const long long Ng = Nbase + mN[g + 1];
+                    const float Nf = (float)(int)Ng;
+                    const float Pf = i64_to_f32(Pg) * pscale;
+                    const float D32 = sh * (sh * Nf - 2.0f * Pf);
+                    const float err = sh * (sh * Nf + 2.0f * Pf) * MPQ_FAST_REL;
+                    if (D32 - err <= upper) {
+                        const double D = decision(__fmul_rn(fgrid[g], smax), Pg, Ng, down);
+                        if (D < bestD) {
+                            bestD = D;
+                            bestg = g;
+                        }
                     }
                 }
             } else {
                 // ---- direct evaluation (a candidate scale underflowed to 0)
-                for (int g = tid; g < G; g += QBLOCK) {
-                    const float s = stab[g];
+                for (int g = gt; g < G; g += NT) {
+                    const float s = __fmul_rn(fgrid[g], smax);
                     double D = 0.0;  // s == 0: all codes 0, E = ||r||^2
                     if (s > 0.0f) {
                         long long P = 0, N = 0;
@@ -430,16 +641,17 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
                     }
                 }
             }
-            int g = block_argmin(bestD, bestg, red);
+            int g = group_argmin<WPC>(bestD, bestg, sc, gw, lane, grp);
             if (g < 0 || g >= G) g = G - 1;   // unreachable: every D is finite
-            s_best = stab[g];
-            inv_best = sinv[g];
+            s_best = __fmul_rn(fgrid[g], smax);
+            inv_best = zero_scale ? 0.0f : finv[g] * ism;
         }
 
         // residual update (Eq. 7) and code emission; also the next step's max |r|
-        part = 0.0f;
+        ssum = 0.0f;
+        scomp = 0.0f;
         am = 0.0f;
-        for (int j = tid; j < d; j += QBLOCK) {
+        for (int j = gt; j < d; j += NT) {
             float v = sr[j];
             int q = 0;
             if (s_best > 0.0f) {
@@ -451,14 +663,16 @@ quantize_event_kernel(const float *__restrict__ W, int C, int d, int qmax, int G
             qi[j] = (int8_t)q;
             sr[j] = v;
             if (ri) ri[j] = v;
-            part = fmaf(v, v, part);
+            kahan_add(ssum, scomp, v * v);
             am = fmaxf(am, fabsf(v));
         }
-        if (tid == 0) scales[(size_t)k * k_max + i] = s_best;
+        if (gt == 0) scales[(size_t)k * k_max + i] = s_best;
         m = am;
-        r2 = (double)part;
-        block_max_sum(m, r2, red);   // also orders the sr[] writes before the next step
-        if (resid_sq && tid == 0) resid_sq[(size_t)k * (k_max + 1) + i + 1] = (float)r2;
+        r2 = ssum;
+        int none = 0;
+        group_max_sum_or<WPC>(m, r2, none, sc, gw, lane, grp);   // orders the sr[] writes too
+        if (WPC == 1) __syncwarp();
+        if (resid_sq && gt == 0) resid_sq[(size_t)k * (k_max + 1) + i + 1] = r2;
     }
 }
 
@@ -469,41 +683,96 @@ int ceil_log2(long long x)
     return b;
 }
 
+template <int WPC, bool CUSTOM, bool LAT>
+mpq_status launch_wpc(const float *W, int C, int d, int qmax, int G, const Grid<CUSTOM> &grid,
+                      int k_max, int8_t *codes, float *scales, float *resid_sq, float *residuals,
+                      int hbits, size_t smem, cudaStream_t stream)
+{
+    constexpr int GPC = 8 / WPC;
+    cudaError_t e = cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) {
+        quantize_kernel<WPC, CUSTOM, LAT><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
+            W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, hbits);
+        e = cudaGetLastError();
+    }
+    return cuda_status(e, "quantize kernel launch");
+}
+
+template <int WPC, bool CUSTOM>
+mpq_status launch_lat(bool lat, const float *W, int C, int d, int qmax, int G,
+                      const Grid<CUSTOM> &grid, int k_max, int8_t *codes, float *scales,
+                      float *resid_sq, float *residuals, int hbits, size_t smem,
+                      cudaStream_t stream)
+{
+    if (lat && !CUSTOM)
+        return launch_wpc<WPC, CUSTOM, !CUSTOM>(W, C, d, qmax, G, grid, k_max, codes, scales,
+                                                resid_sq, residuals, hbits, smem, stream);
+    return launch_wpc<WPC, CUSTOM, false>(W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq,
+                                          residuals, hbits, smem, stream);
+}
+
+template <bool CUSTOM>
+mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid<CUSTOM> &grid,
+                       int k_max, int8_t *codes, float *scales, float *resid_sq, float *residuals,
+                       cudaStream_t stream)
+{
+    const int hbits = ceil_log2((long long)d * qmax) + 1;
+    // lattice form on the linear grid when its buckets fit (48 KB)
+    const bool lat = !CUSTOM && (long long)2 * G * qmax + 1 <= 4096;
+    const int nb = lat ? 2 * G * qmax + 1 : 0;
+    const size_t per_group = group_words(G, d, 1, nb) * 4;
+    const long long smem_cap = max_smem_optin();
+    // Warps per channel: enough channels in flight to fill the GPU, at least ~2 elements per
+    // lane, and enough warps per SM for the shared memory the channels need.
+    const long long warps_gpu = (long long)sm_count() * 32;
+    int wpc_c = 1;
+    while (wpc_c < 8 && (long long)C * wpc_c < warps_gpu) wpc_c *= 2;
+    int wpc_e = 1;
+    while (wpc_e < 8 && wpc_e * 64 <= d) wpc_e *= 2;
+    const long long groups_per_sm = (long long)(227 * 1024) / (long long)(per_group + 256);
+    int wpc_s = 1;
+    while (wpc_s < 8 && groups_per_sm * wpc_s < 32) wpc_s *= 2;
+    int wpc = wpc_c < wpc_e ? wpc_c : wpc_e;
+    if (wpc < wpc_s) wpc = wpc_s;
+    for (; wpc <= 8; wpc *= 2) {
+        const size_t smem =
+            (size_t)(8 / wpc) * group_words(G, d, wpc, nb) * 4 + (size_t)2 * G * sizeof(float);
+        if ((long long)smem <= smem_cap) {
+            switch (wpc) {
+            case 1:
+                return launch_lat<1, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
+                                             resid_sq, residuals, hbits, smem, stream);
+            case 2:
+                return launch_lat<2, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
+                                             resid_sq, residuals, hbits, smem, stream);
+            case 4:
+                return launch_lat<4, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
+                                             resid_sq, residuals, hbits, smem, stream);
+            default:
+                return launch_lat<8, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
+                                             resid_sq, residuals, hbits, smem, stream);
+            }
+        }
+    }
+    set_error("d = %d, G = %d need %zu bytes of shared memory per channel", d, G, per_group);
+    return MPQ_ERR_UNSUPPORTED;
+}
+
 }  // namespace
 
 mpq_status launch_quantize(const float *W, int C, int d, int qmax, int G, const GridFrac *grid,
                            int k_max, int8_t *codes, float *scales, float *resid_sq,
                            float *residuals, cudaStream_t stream)
 {
-    const size_t smem = (size_t)(G + 1) * (sizeof(long long) + sizeof(int)) +
-                        (size_t)2 * G * sizeof(float) + (size_t)d * sizeof(float);
-    if ((long long)smem > max_smem_optin()) {
-        set_error("d = %d, G = %d need %zu bytes of shared memory", d, G, smem);
-        return MPQ_ERR_UNSUPPORTED;
-    }
-    const int hbits = ceil_log2((long long)d * qmax) + 1;
-
-    cudaError_t e;
     if (grid) {
         Grid<true> g;
         g.gf = *grid;
-        e = cudaFuncSetAttribute(quantize_event_kernel<true>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e == cudaSuccess) {
-            quantize_event_kernel<true><<<C, QBLOCK, smem, stream>>>(
-                W, C, d, qmax, G, g, k_max, codes, scales, resid_sq, residuals, hbits);
-            e = cudaGetLastError();
-        }
-    } else {
-        e = cudaFuncSetAttribute(quantize_event_kernel<false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e == cudaSuccess) {
-            quantize_event_kernel<false><<<C, QBLOCK, smem, stream>>>(
-                W, C, d, qmax, G, Grid<false>(), k_max, codes, scales, resid_sq, residuals, hbits);
-            e = cudaGetLastError();
-        }
+        return launch_grid<true>(W, C, d, qmax, G, g, k_max, codes, scales, resid_sq, residuals,
+                                 stream);
     }
-    return cuda_status(e, "quantize kernel launch");
+    return launch_grid<false>(W, C, d, qmax, G, Grid<false>(), k_max, codes, scales, resid_sq,
+                              residuals, stream);
 }
 
 }  // namespace mpq
