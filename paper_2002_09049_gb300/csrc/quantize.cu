@@ -64,6 +64,8 @@ struct Scratch {
     float f[8];
     float v[8];
     unsigned long long key[8];
+    unsigned long long sp[8];
+    long long sn[8];
     long long a[8];
     long long b[8];
     int g[8];
@@ -227,6 +229,64 @@ __device__ __forceinline__ int group_argmin(double D, int g, Scratch &sc, int gw
         for (int i = 1; i < WPC; ++i) cand = min(cand, sc.g[i]);
     }
     return cand;
+}
+
+// In-place suffix sums over items t in [t0, t1) by the whole group: item t <- sum of items
+// u >= t, for a 64-bit and a 32-bit quantity.  Each thread owns a contiguous block; block totals
+// are combined with a shuffle scan inside each warp and scratch across warps.
+template <int WPC, typename Load, typename Store>
+__device__ __forceinline__ void group_suffix_scan(int t0, int t1, Load load, Store store,
+                                                  Scratch &sc, int gw, int lane, int grp)
+{
+    constexpr int NT = WPC * 32;
+    const int gt = gw * 32 + lane;
+    const int n = t1 - t0;
+    const int per = (n + NT - 1) / NT;
+    const int b0 = t0 + min(n, gt * per), b1 = t0 + min(n, gt * per + per);
+    unsigned long long sp = 0;
+    long long sn = 0;
+    for (int t = b0; t < b1; ++t) {
+        unsigned long long p;
+        long long q;
+        load(t, p, q);
+        sp += p;
+        sn += q;
+    }
+    unsigned long long xp = sp;   // inclusive scan toward lower lanes
+    long long xn = sn;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long yp = __shfl_down_sync(0xffffffffu, xp, o);
+        const long long yn = __shfl_down_sync(0xffffffffu, xn, o);
+        if (lane + o < 32) {
+            xp += yp;
+            xn += yn;
+        }
+    }
+    unsigned long long rp = xp - sp;   // blocks of higher lanes in this warp
+    long long rn = xn - sn;
+    if (WPC > 1) {
+        gsync<WPC>(grp);
+        if (lane == 0) {
+            sc.sp[gw] = xp;   // warp total
+            sc.sn[gw] = xn;
+        }
+        gsync<WPC>(grp);
+#pragma unroll
+        for (int w = 0; w < WPC; ++w)
+            if (w > gw) {
+                rp += sc.sp[w];
+                rn += sc.sn[w];
+            }
+    }
+    for (int t = b1 - 1; t >= b0; --t) {
+        unsigned long long p;
+        long long q;
+        load(t, p, q);
+        rp += p;
+        rn += q;
+        store(t, rp, rn);
+    }
 }
 
 // Code magnitude of |r| at scale s > 0 (Eq. 8): nearest integer (ties to even) of the correctly
@@ -502,76 +562,45 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 }
                 group_sum2<WPC>(Pb, Nb, sc, gw, lane, grp);   // publishes the bins too
                 const long long Pbase = Pb, Nbase = Nb;
-                // ---- suffix sums over the bins (warp 0 of the group), in place: bin t <- sum
-                // of bins u >= t, so that P_g = Pbase + bin(g + 1).  Each lane owns (b0, b1].
-                if (gw == 0) {
-                    const int per = (G + 31) / 32;
-                    const int b0 = min(G, lane * per), b1 = min(G, b0 + per);
-                    long long sp = 0, sn = 0;
-                    for (int t = b0 + 1; t <= b1; ++t) {
-                        // merge the warps' private copies into copy 0
-                        long long p = bin64(mLo, mHi, t);
-                        int n = mN[t];
+                // ---- suffix sums over the event bins (the warps' private copies merged into
+                // copy 0; warp 0), in place: bin t <- sum of bins u >= t, so P_g = Pbase +
+                // bin(g + 1); and over the lattice buckets (warp 1 concurrently, or the whole
+                // group afterwards when the lattice is large)
+                auto bins_load = [&](int t, unsigned long long &p, long long &q) {
+                    long long pp = bin64(mLo, mHi, t);
+                    long long nn = mN[t];
 #pragma unroll
-                        for (int c = 1; c < WPC; ++c) {
-                            const unsigned int *cLo = mLo + (size_t)c * 3 * (G + 1);
-                            p += bin64(cLo, cLo + (G + 1), t);
-                            n += reinterpret_cast<const int *>(cLo + 2 * (G + 1))[t];
-                        }
-                        mLo[t] = (unsigned int)p;
-                        mHi[t] = (unsigned int)((unsigned long long)p >> 32);
-                        mN[t] = n;
-                        sp += p;
-                        sn += n;
+                    for (int c = 1; c < WPC; ++c) {
+                        const unsigned int *cLo = mLo + (size_t)c * 3 * (G + 1);
+                        pp += bin64(cLo, cLo + (G + 1), t);
+                        nn += reinterpret_cast<const int *>(cLo + 2 * (G + 1))[t];
                     }
-                    long long xp = sp, xn = sn;   // inclusive scan toward lower lanes
-#pragma unroll
-                    for (int o = 1; o < 32; o <<= 1) {
-                        const long long yp = __shfl_down_sync(0xffffffffu, xp, o);
-                        const long long yn = __shfl_down_sync(0xffffffffu, xn, o);
-                        if (lane + o < 32) {
-                            xp += yp;
-                            xn += yn;
-                        }
-                    }
-                    long long rp = xp - sp, rn = xn - sn;   // bins beyond b1
-                    for (int t = b1; t > b0; --t) {
-                        rp += bin64(mLo, mHi, t);
-                        rn += mN[t];
-                        mLo[t] = (unsigned int)rp;
-                        mHi[t] = (unsigned int)((unsigned long long)rp >> 32);
-                        mN[t] = (int)rn;
-                    }
-                }
-                if (LAT && gw == (WPC > 1 ? 1 : 0)) {
-                    // suffix sums over the lattice buckets, in place: bucket t <- sum_{u >= t}
-                    const int per = (nb + 31) / 32;
-                    const int b0 = min(nb, lane * per), b1 = min(nb, b0 + per);
-                    unsigned long long sp = 0;
-                    unsigned int sn = 0;
-                    for (int t = b0; t < b1; ++t) {
-                        sp += latR[t];
-                        sn += latC[t];
-                    }
-                    unsigned long long xp = sp;
-                    unsigned int xn = sn;
-#pragma unroll
-                    for (int o = 1; o < 32; o <<= 1) {
-                        const unsigned long long yp = __shfl_down_sync(0xffffffffu, xp, o);
-                        const unsigned int yn = __shfl_down_sync(0xffffffffu, xn, o);
-                        if (lane + o < 32) {
-                            xp += yp;
-                            xn += yn;
-                        }
-                    }
-                    unsigned long long rp = xp - sp;
-                    unsigned int rn = xn - sn;
-                    for (int t = b1 - 1; t >= b0; --t) {
-                        rp += latR[t];
-                        rn += latC[t];
-                        latR[t] = rp;
-                        latC[t] = rn;
-                    }
+                    p = (unsigned long long)pp;
+                    q = nn;
+                };
+                auto bins_store = [&](int t, unsigned long long p, long long q) {
+                    mLo[t] = (unsigned int)p;
+                    mHi[t] = (unsigned int)(p >> 32);
+                    mN[t] = (int)q;
+                };
+                auto lat_load = [&](int t, unsigned long long &p, long long &q) {
+                    p = latR[t];
+                    q = latC[t];
+                };
+                auto lat_store = [&](int t, unsigned long long p, long long q) {
+                    latR[t] = p;
+                    latC[t] = (unsigned int)q;
+                };
+                // large grids (G * WPC bins to merge, or a long lattice): the whole group scans
+                const bool big = (LAT && nb > 2048) || G * WPC > 1024;
+                if (big) {
+                    group_suffix_scan<WPC>(1, G + 1, bins_load, bins_store, sc, gw, lane, grp);
+                    if (LAT) group_suffix_scan<WPC>(0, nb, lat_load, lat_store, sc, gw, lane, grp);
+                } else {
+                    if (gw == 0)
+                        group_suffix_scan<1>(1, G + 1, bins_load, bins_store, sc, 0, lane, grp);
+                    if (LAT && gw == (WPC > 1 ? 1 : 0))
+                        group_suffix_scan<1>(0, nb, lat_load, lat_store, sc, 0, lane, grp);
                 }
                 gsync<WPC>(grp);
                 if (LAT) {
