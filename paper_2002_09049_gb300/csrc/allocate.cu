@@ -11,8 +11,8 @@
 // at or above every other head is taken next -- so both rules visit the pairs in the same order.
 // Each pair becomes one unique 64-bit key (~bits(p) in the high word, k*(k_max-1)+(n-2) in the
 // low word); an MSB-first radix select finds the extra-th smallest key T, and
-// n_k = 1 + #{n : key(k, n) <= T}.  Keys are recomputed from the error table on every pass, so
-// nothing but a 256-bin histogram in shared memory is needed.
+// n_k = 1 + #{n : key(k, n) <= T}.  The keys live in shared memory when they fit (they are
+// recomputed from the error table on every pass otherwise); no global scratch is used.
 #include <math.h>
 
 #include "mpq_internal.cuh"
@@ -46,79 +46,133 @@ __device__ __forceinline__ void channel_keys(const float *__restrict__ err, int 
     }
 }
 
+constexpr int KEY_CACHE = 12288;   // keys held in shared memory (96 KB) when they fit
+
+// Radix select of the rank-th smallest selectable key, MSB first, 8 bits per pass.  A pass whose
+// target bucket holds one key ends the search with that key (recorded as the bucket's witness).
 __global__ void __launch_bounds__(AB_THREADS)
 allocate_budget_kernel(const float *__restrict__ err, int C, int k_max, long long extra,
-                       int *__restrict__ npoints, int *__restrict__ points_used)
+                       int *__restrict__ npoints, int *__restrict__ points_used, bool cached)
 {
+    extern __shared__ unsigned long long skeys[];   // [C * (k_max - 1)] when cached
     __shared__ unsigned int hist[256];
-    __shared__ unsigned long long s_prefix;
+    __shared__ unsigned long long witness[256];
+    __shared__ unsigned long long s_prefix, s_T, s_total;
     __shared__ long long s_rem;
-    __shared__ unsigned long long s_total;
-    const int tid = threadIdx.x;
+    __shared__ int s_done, s_used;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int KM1 = k_max - 1;
 
-    // number of selectable keys (p > 0)
-    if (tid == 0) s_total = 0;
+    if (tid == 0) {
+        s_total = 0;
+        s_used = 0;
+        s_done = 0;
+        s_prefix = 0;
+    }
     __syncthreads();
     unsigned long long mine = 0;
     for (int k = tid; k < C; k += AB_THREADS)
-        channel_keys(err, k, k_max, [&](int, unsigned long long key) { mine += key != NO_KEY; });
+        channel_keys(err, k, k_max, [&](int n, unsigned long long key) {
+            if (cached) skeys[(size_t)k * KM1 + (n - 2)] = key;
+            mine += key != NO_KEY;
+        });
     atomicAdd(&s_total, mine);
     __syncthreads();
     const long long total = (long long)s_total;
     const long long take = extra < total ? extra : total;
 
-    unsigned long long T = 0;  // threshold key; selected = keys <= T (when take > 0)
-    if (take == 0) {
-        T = 0;
-    } else if (take == total) {
-        T = NO_KEY - 1;
-    } else {
-        if (tid == 0) {
-            s_prefix = 0;
-            s_rem = take;  // 1-based rank of the key we look for
+    // visit every selectable key
+    auto for_keys = [&](auto f) {
+        if (cached) {
+            const long long nk = (long long)C * KM1;
+            for (long long i = tid; i < nk; i += AB_THREADS) {
+                const unsigned long long key = skeys[i];
+                if (key != NO_KEY) f(key);
+            }
+        } else {
+            for (int k = tid; k < C; k += AB_THREADS)
+                channel_keys(err, k, k_max, [&](int, unsigned long long key) {
+                    if (key != NO_KEY) f(key);
+                });
         }
+    };
+
+    unsigned long long T = 0;   // selected = keys <= T (when take > 0)
+    if (take > 0 && take == total) {
+        T = NO_KEY - 1;
+    } else if (take > 0) {
+        if (tid == 0) s_rem = take;   // 1-based rank of the key we look for
         for (int shift = 56; shift >= 0; shift -= 8) {
             for (int b = tid; b < 256; b += AB_THREADS) hist[b] = 0;
             __syncthreads();
             const unsigned long long prefix = s_prefix;
             const int hs = shift + 8;
-            for (int k = tid; k < C; k += AB_THREADS)
-                channel_keys(err, k, k_max, [&](int, unsigned long long key) {
-                    if (key == NO_KEY) return;
-                    if (hs < 64 && ((key ^ prefix) >> hs) != 0) return;
-                    atomicAdd(&hist[(key >> shift) & 255u], 1u);
-                });
+            for_keys([&](unsigned long long key) {
+                if (hs < 64 && ((key ^ prefix) >> hs) != 0) return;
+                const unsigned b = (unsigned)(key >> shift) & 255u;
+                atomicAdd(&hist[b], 1u);
+                witness[b] = key;   // meaningful only when the bucket ends with one key
+            });
             __syncthreads();
-            if (tid == 0) {
-                long long rem = s_rem, cum = 0;
-                int b = 0;
-                for (; b < 256; ++b) {
-                    if (cum + (long long)hist[b] >= rem) break;
-                    cum += hist[b];
+            if (warp == 0) {
+                // warp-parallel search for the bucket that holds the rem-th key
+                const long long rem = s_rem;
+                unsigned int loc = 0;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) loc += hist[lane * 8 + i];
+                unsigned long long incl = loc;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const unsigned long long y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += y;
                 }
-                s_rem = rem - cum;
-                s_prefix = prefix | ((unsigned long long)b << shift);
+                const unsigned long long excl = incl - loc;
+                const unsigned hit = __ballot_sync(0xffffffffu,
+                                                   (long long)excl < rem && rem <= (long long)incl);
+                const int src = __ffs(hit) - 1;
+                if (lane == src) {
+                    long long cum = (long long)excl;
+                    int b = lane * 8;
+                    for (; b < lane * 8 + 7; ++b) {
+                        if (cum + (long long)hist[b] >= rem) break;
+                        cum += hist[b];
+                    }
+                    s_rem = rem - cum;
+                    s_prefix = prefix | ((unsigned long long)b << shift);
+                    if (hist[b] == 1) {
+                        s_T = witness[b];
+                        s_done = 1;
+                    }
+                }
             }
             __syncthreads();
+            if (s_done) break;
         }
-        T = s_prefix;
+        T = s_done ? s_T : s_prefix;
     }
 
     // n_k = 1 + number of selected keys of channel k (a prefix n = 2..n_k, since p is monotone)
     int used = 0;
     for (int k = tid; k < C; k += AB_THREADS) {
         int n_k = 1;
-        channel_keys(err, k, k_max, [&](int, unsigned long long key) {
-            if (take > 0 && key != NO_KEY && key <= T) ++n_k;
-        });
+        if (take > 0) {
+            if (cached) {
+                for (int n = 0; n < KM1; ++n) {
+                    const unsigned long long key = skeys[(size_t)k * KM1 + n];
+                    if (key != NO_KEY && key <= T) ++n_k;
+                }
+            } else {
+                channel_keys(err, k, k_max, [&](int, unsigned long long key) {
+                    if (key != NO_KEY && key <= T) ++n_k;
+                });
+            }
+        }
         npoints[k] = n_k;
         used += n_k;
     }
     if (points_used) {
-        __shared__ int s_used;
-        if (tid == 0) s_used = 0;
-        __syncthreads();
-        atomicAdd(&s_used, used);
+        for (int o = 16; o > 0; o >>= 1) used += __shfl_xor_sync(0xffffffffu, used, o);
+        if (lane == 0) atomicAdd(&s_used, used);   // integer sum: order-free
         __syncthreads();
         if (tid == 0) *points_used = s_used;
     }
@@ -154,8 +208,17 @@ allocate_threshold_kernel(const float *__restrict__ err, int C, int k_max, doubl
 mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
                                   int *npoints, int *points_used, cudaStream_t stream)
 {
-    allocate_budget_kernel<<<1, AB_THREADS, 0, stream>>>(err, C, k_max, extra, npoints,
-                                                         points_used);
+    const long long nkeys = (long long)C * (k_max - 1);
+    const bool cached = nkeys <= KEY_CACHE;
+    const size_t smem = cached ? (size_t)nkeys * sizeof(unsigned long long) : 0;
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(allocate_budget_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
+    }
+    allocate_budget_kernel<<<1, AB_THREADS, smem, stream>>>(err, C, k_max, extra, npoints,
+                                                            points_used, cached);
     return cuda_status(cudaGetLastError(), "allocation kernel launch");
 }
 
