@@ -59,10 +59,8 @@ def parse():
 
 # ------------------------------------------------------------------------------------------------
 def dist_setup(args):
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return world, rank, local
+    from paper_2002_09049_gb300 import dist as dist_helpers
+    return dist_helpers.world_from_env()
 
 
 def host_cores():
@@ -170,6 +168,7 @@ def contraction_flops(wl, layer):
 def run_ours(args, world, rank, local):
     import torch
     from paper_2002_09049_gb300 import _build, binding, pipeline, workloads as wlm
+    from paper_2002_09049_gb300 import dist as dist_helpers
 
     dev = torch.device(f"cuda:{local}")
     torch.cuda.set_device(dev)
@@ -203,20 +202,11 @@ def run_ours(args, world, rank, local):
 
     families = ["quantize", "output_error", "allocate", "reconstruct"]
 
-    def step(record=None):
+    def step():
         for b in wl.bits:
             for sp in specs:
                 sp.bits = b
-            cb = None
-            if record is not None:
-                evs = {}
-
-                def cb(i, st, ph, evs=evs):
-                    e = torch.cuda.Event(enable_timing=True)
-                    e.record(st)
-                    evs.setdefault(i, [None] * 5)[ph] = e
-                record.append(evs)
-            net.run_device(Ws, Xs, stream=stream, on_layer=cb)
+            net.run_device(Ws, Xs, stream=stream)
 
     launches_per_step = 4 * len(layers) * len(wl.bits)
 
@@ -235,22 +225,32 @@ def run_ours(args, world, rank, local):
             flush.fill_(1.0)                    # evict L2 between steps (outside the timing)
             a = torch.cuda.Event(enable_timing=True)
             z = torch.cuda.Event(enable_timing=True)
-            rec = []
             a.record(stream)
-            step(rec)
+            step()
             z.record(stream)
-            recs.append(rec)
             torch.cuda.synchronize()
             step_ms.append(a.elapsed_time(z))
     torch.cuda.synchronize()
+    # Per-kernel durations for the roofline: the same steps once more with every layer on one
+    # stream and CUDA events around each call, so no launch shares the GPU with another layer's.
+    for _ in range(args.steps):
+        flush.fill_(1.0)
+        rec = []
+        for b in wl.bits:
+            for sp in specs:
+                sp.bits = b
+            evs = {}
+            for i in net.order:
+                evs[i] = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+                net.plans[i].run_device(Ws[i], Xs[i], stream=stream,
+                                        timing=lambda ph, e=evs[i]: e[ph].record(stream))
+            rec.append(evs)
+        torch.cuda.synchronize()
+        recs.append(rec)
     if world > 1:
         torch.distributed.barrier()
-    ms = float(np.mean(step_ms))
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    value = units_per_step * world / (ms / 1e3)
+    ms = dist_helpers.max_over_ranks(float(np.mean(step_ms)), device=dev)
+    value = dist_helpers.aggregate_throughput(units_per_step, ms, world)
 
     # per-kernel-family device time from the events around every call (on its own stream)
     fam_ms = {f: 0.0 for f in families}
@@ -271,6 +271,9 @@ def run_ours(args, world, rank, local):
     roofline = dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args)
     roofline["share"] = fam_ms[dominant] / total_fam if total_fam else None
     roofline["family_ms_per_step"] = {f: fam_ms[f] / args.steps for f in families}
+    roofline["timing"] = ("CUDA events around every call in a single-stream pass of the same "
+                          "steps inside bench.py (value itself is timed with layers on "
+                          f"{args.streams} streams)")
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -316,7 +319,6 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
         if ent and ent.get("source_sha") == src_hash(KERNEL_SOURCES[dominant]):
             traffic = ent.get("dram_bytes_per_launch")
     t_s = fam_ms[dominant] / 1e3
-    launches = args.steps * len(wl.bits) * fam_work.get("_layers", 1)
     if dominant == "output_error":
         peak = peaks["bf16_tflops"] * TF32_PER_BF16
         ach = fam_work[dominant] / t_s / 1e12
