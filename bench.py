@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--graph", type=int, default=1,
+                    help="replay the multi-stream step as a captured CUDA graph (1) or launch it (0)")
     ap.add_argument("--streams", type=int, default=8,
                     help="CUDA streams the independent layers are spread over")
     ap.add_argument("--layers", default=None,
@@ -202,7 +204,19 @@ def run_ours(args, world, rank, local):
 
     families = ["quantize", "output_error", "allocate", "reconstruct"]
 
+    graphs = []
+    if args.graph:
+        # one captured graph per bit width (the bit width is a launch argument)
+        for b in wl.bits:
+            for sp in specs:
+                sp.bits = b
+            graphs.append(pipeline.CapturedNetwork(net, Ws, Xs))
+
     def step():
+        if graphs:
+            for g in graphs:
+                g.replay()
+            return
         for b in wl.bits:
             for sp in specs:
                 sp.bits = b
@@ -284,7 +298,8 @@ def run_ours(args, world, rank, local):
                    "channels": sum(l.C for l in layers), "bits": list(wl.bits),
                    "G": wl.G, "k_max": wl.k_max, "budget": wl.beta, "calib_rows": wl.n_calib,
                    "units_per_step": units_per_step, "l2": "flushed between steps (512 MB write)",
-                   "streams": args.streams, "parallelism": f"replicas x{world}"},
+                   "streams": args.streams, "cuda_graph": bool(args.graph),
+                   "parallelism": f"replicas x{world}"},
         "roofline": roofline,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),

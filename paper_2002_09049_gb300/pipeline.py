@@ -154,3 +154,32 @@ class NetworkPlan:
                                              stream=st)
         self._join(main)
         return outs
+
+
+class CapturedNetwork:
+    """A NetworkPlan's multi-stream step captured once into a CUDA graph and replayed.
+
+    Capture records every launch of ``NetworkPlan.run_device`` (all layers, all streams, the fork and
+    join) for fixed input tensors; each ``replay`` re-executes all of that work on the GPU with one
+    host call.  Inputs are read from the captured tensors, so refresh their contents in place
+    (``copy_``) to quantize new weights of the same shapes.
+    """
+
+    def __init__(self, net: NetworkPlan, Ws, Xs, warmup: int = 1):
+        self.net = net
+        self.Ws, self.Xs = Ws, Xs
+        side = torch.cuda.Stream(net.device)
+        side.wait_stream(torch.cuda.current_stream(net.device))
+        with torch.cuda.stream(side):          # warm up outside capture (attributes, modules)
+            for _ in range(warmup):
+                net.run_device(Ws, Xs, stream=side)
+        torch.cuda.current_stream(net.device).wait_stream(side)
+        torch.cuda.synchronize(net.device)
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph, stream=side):
+            net.run_device(Ws, Xs, stream=side)
+        torch.cuda.synchronize(net.device)
+
+    def replay(self):
+        self.graph.replay()
+        return self.net

@@ -109,3 +109,30 @@ def test_network_plan_streams_match_single_stream(gpu):
     for a, b in zip(many.plans, one.plans):
         for name in ("codes", "scales", "resid_sq", "err", "npoints", "points_used", "W_hat"):
             assert torch.equal(getattr(a, name), getattr(b, name)), name
+
+
+def test_captured_graph_matches_launches(gpu):
+    """A CUDA-graph replay of the multi-stream step gives bit-identical outputs to launching it."""
+    wl = wlm.WORKLOADS["c2"]
+    idx = [0, 5, 16, 20]
+    specs, Ws, Xs = [], [], []
+    for li in idx:
+        layer = wl.layers[li]
+        specs.append(pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, bits=4, G=wl.G,
+                                        k_max=wl.k_max, budget_or_eps=wl.beta))
+        Ws.append(torch.from_numpy(wlm.make_weights(wl, li)).to(gpu))
+        Xs.append(torch.from_numpy(wlm.make_calibration(wl, li)).to(gpu))
+    ref = pipeline.NetworkPlan(specs, gpu, n_streams=4).run_device(Ws, Xs)
+    torch.cuda.synchronize()
+    ref_out = [{n: getattr(p, n).clone() for n in ("codes", "scales", "err", "npoints", "W_hat")}
+               for p in ref.plans]
+    net = pipeline.NetworkPlan(specs, gpu, n_streams=4)
+    cap = pipeline.CapturedNetwork(net, Ws, Xs)
+    for p in net.plans:                 # poison the outputs: the replay must rewrite them all
+        for n in ("codes", "scales", "err", "npoints", "W_hat"):
+            getattr(p, n).fill_(0)
+    cap.replay()
+    torch.cuda.synchronize()
+    for p, r in zip(net.plans, ref_out):
+        for n, v in r.items():
+            assert torch.equal(getattr(p, n), v), n
