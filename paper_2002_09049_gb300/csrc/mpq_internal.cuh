@@ -37,6 +37,12 @@ mpq_status launch_output_error_tc(const float *X, int N, const float *W, const i
                                   const float *scales, int C, int d, int k_max, float *err,
                                   cudaStream_t stream);
 
+// CTA-pair tensor-core kernel: needs d % 16 == 0 and 16-byte aligned X, W and codes.
+bool output_error_pair_ok(const float *X, const float *W, const int8_t *codes, int d);
+mpq_status launch_output_error_pair(const float *X, int N, const float *W, const int8_t *codes,
+                                    const float *scales, int C, int d, int k_max, float *err,
+                                    cudaStream_t stream);
+
 mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
                                   int *npoints, int *points_used, cudaStream_t stream);
 

@@ -97,8 +97,11 @@ mpq_status launch_output_error(const float *X, int N, int groups, const float *W
                                const int8_t *codes, const float *scales, int C, int d, int k_max,
                                float *err, cudaStream_t stream)
 {
-    if (groups == 1)
+    if (groups == 1) {
+        if (output_error_pair_ok(X, W, codes, d))
+            return launch_output_error_pair(X, N, W, codes, scales, C, d, k_max, err, stream);
         return launch_output_error_tc(X, N, W, codes, scales, C, d, k_max, err, stream);
+    }
     switch (k_max + 1) {
 #define MPQ_CASE(n) \
     case n: return launch_grouped<n>(X, N, W, codes, scales, C, d, err, stream);

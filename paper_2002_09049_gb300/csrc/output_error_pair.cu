@@ -1,0 +1,474 @@
+// Output error (Sec. 3.3, Eq. 11) as a CTA-pair tcgen05 contraction:
+//   err[k][n] = (1/N) sum_t (x_t . r_{k,n+1})^2,  n = 0..k_max.
+//
+// Y = R X^T with R the C*(k_max+1) residual vectors and X the N calibration rows (length d);
+// err is the row-wise mean of Y^2.  Two CTAs on neighbouring SMs (cluster ranks 2p, 2p+1) form one
+// UMMA of M = 256 residual vectors by N = 256 calibration rows: each CTA holds 128 vectors (whole
+// channels: floor(128/(k_max+1)) of them) as its half of A and 128 calibration rows as its half of
+// B, and receives its 128 vectors x all 256 rows in its own tensor memory.  Per flop, this halves
+// the operand bytes each SM's tensor core reads and the residual vectors each SM regenerates,
+// compared with one CTA computing 256 vectors x 128 rows alone.
+//
+// Precision is that of the single-CTA kernel: each operand is split exactly into a tf32 hi part and
+// an fp32 lo part and Y = hi*hi + hi*lo + lo*hi on kind::tf32; the accumulator restarts every 128
+// elements of d and the epilogue folds each segment into fp32 running sums in tensor memory
+// (columns [0, 256) segment, [256, 512) running sums), since the tensor core's accumulation
+// truncates.
+//
+// Input: one thread per CTA streams each K chunk's X rows, W rows and codes into a ring of raw
+// shared-memory slots with TMA tile copies (rows past N and channels past C read as zeros).  Eight
+// producer warps split X into the B tiles and regenerate the residuals r_{n+1} = r_n - s_n q_n
+// (Eq. 7) from W, codes and scales into the A tiles (128-byte swizzled, K-major); residuals never
+// exist in global memory.  Both CTAs' producers report a full stage to the even CTA, whose MMA
+// thread issues the pair MMAs and signals both CTAs (multicast commits) when a stage or a segment
+// is consumed.  Four epilogue warps per CTA drain the segments; a segment is restarted only once
+// both CTAs' epilogues have released it.
+//
+// Row tiles (256 rows) are split over the pairs of a cluster of up to 8 CTAs; ranks 0 and 1 add
+// their peers' partial sums from distributed shared memory in rank order.  Every wait is bounded;
+// on a timeout the outputs read NaN.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+#include <string.h>
+
+#include "mpq_internal.cuh"
+#include "sm100.cuh"
+#include "tf32_operands.cuh"
+
+namespace mpq {
+namespace {
+
+using namespace sm100;
+
+constexpr int P_VEC = 128;                      // residual vectors per CTA (TMEM lanes)
+constexpr int P_ROWS = 128;                     // calibration rows per CTA
+constexpr int P_N = 2 * P_ROWS;                 // rows per pair row tile (UMMA N)
+constexpr int P_KC = 32;                        // fp32 per K chunk = one 128-byte swizzle row
+constexpr int P_KC4 = P_KC / 4;
+constexpr int P_SEG = 4;                        // chunks per accumulation segment (128 elements)
+constexpr int P_STAGES = 2;                     // operand stages
+constexpr int P_TILE = 128 * P_KC * 4;          // 16 KB: one 128-row operand tile
+constexpr int P_OFF_A_HI = 0;
+constexpr int P_OFF_A_LO = P_TILE;
+constexpr int P_OFF_B_HI = 2 * P_TILE;
+constexpr int P_OFF_B_LO = 3 * P_TILE;
+constexpr int P_STAGE_BYTES = 4 * P_TILE;       // 64 KB
+constexpr int P_PROD_WARPS = 8;
+constexpr int P_PROD_THREADS = P_PROD_WARPS * 32;
+constexpr int P_EPI_WARP0 = P_PROD_WARPS;       // warps 8..11: warp % 4 selects TMEM lanes
+constexpr int P_MMA_WARP = P_EPI_WARP0 + 4;
+constexpr int P_TMA_WARP = P_MMA_WARP + 1;
+constexpr int P_THREADS = (P_TMA_WARP + 1) * 32;   // 448
+constexpr uint32_t P_TMEM_COLS = 512;
+constexpr uint32_t P_RUN_COL = 256;
+constexpr int P_MAX_RAW = 3;
+constexpr long long P_WAIT = 1LL << 31;         // SM clocks (~1 s)
+constexpr int P_SMEM_LIMIT = 232448;            // opt-in shared memory per CTA on sm_100 parts
+
+struct PairCtrl {
+    uint64_t full[P_STAGES];      // even CTA: both CTAs' producer warps
+    uint64_t empty[P_STAGES];     // both CTAs: pair MMA commit
+    uint64_t raw_full[P_MAX_RAW];
+    uint64_t raw_empty[P_MAX_RAW];
+    uint64_t segfull;             // both CTAs: pair MMA commit
+    uint64_t segempty;            // even CTA: both CTAs' epilogue warps
+    uint64_t done;                // even CTA
+    uint32_t tmem_base;
+    int abort;
+    double part[P_VEC];
+};
+constexpr int P_CTRL_BYTES = (sizeof(PairCtrl) + 1023) / 1024 * 1024;
+constexpr int P_BASE_SMEM = 1024 /* alignment slack */ + P_CTRL_BYTES + P_STAGES * P_STAGE_BYTES;
+
+// Per-KP1 geometry and the raw slot layout, in the order the tile copies write it:
+// X chunk [128 rows][32] fp32, W chunk [CH][32] fp32, codes [K][CH][32] int8.
+template <int KP1>
+struct PGeo {
+    static constexpr int K = KP1 - 1;
+    static constexpr int KQ = K > 0 ? K : 1;
+    static constexpr int CH = P_VEC / KP1;
+    static constexpr int ITEMS2 = (CH * (P_KC / 2) + P_PROD_THREADS - 1) / P_PROD_THREADS;
+    static constexpr int X_ITEMS = P_ROWS * P_KC4 / P_PROD_THREADS;
+    static constexpr int RAW_W = P_ROWS * P_KC * 4;
+    static constexpr int RAW_Q = (RAW_W + CH * P_KC * 4 + 127) / 128 * 128;
+    static constexpr uint32_t RAW_TX = P_ROWS * P_KC * 4 + CH * P_KC * 4 + K * CH * P_KC;
+    static constexpr int RAW_BYTES = (RAW_Q + KQ * CH * P_KC + 1023) / 1024 * 1024;
+    static constexpr int RAW_FIT = (P_SMEM_LIMIT - P_BASE_SMEM) / RAW_BYTES;
+    static constexpr int RAW_STAGES = RAW_FIT < P_MAX_RAW ? RAW_FIT : P_MAX_RAW;
+    static constexpr int SMEM = P_BASE_SMEM + RAW_STAGES * RAW_BYTES;
+    static_assert(RAW_STAGES >= 2, "raw ring needs two slots");
+    static_assert(X_ITEMS * P_PROD_THREADS == P_ROWS * P_KC4, "X items");
+};
+
+// Raw slot -> operand stage `sb`: X rows -> B tiles; for every (channel, element pair) item the
+// residuals r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7) -> A tiles.
+template <int KP1>
+__device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt, int nch,
+                                             const float (&sc)[PGeo<KP1>::ITEMS2][PGeo<KP1>::KQ])
+{
+    using G = PGeo<KP1>;
+    constexpr int K = KP1 - 1;
+#pragma unroll
+    for (int i = 0; i < G::X_ITEMS; ++i) {
+        const int q = pt + i * P_PROD_THREADS;
+        float4 hi, lo;
+        split4(ld_shared_v4(slot + (uint32_t)q * 16u), hi, lo);
+        const uint32_t off = sw128_offset(q / P_KC4, q % P_KC4);
+        st_shared_v4(sb + P_OFF_B_HI + off, hi);
+        st_shared_v4(sb + P_OFF_B_LO + off, lo);
+    }
+#pragma unroll
+    for (int i = 0; i < G::ITEMS2; ++i) {
+        const int p = pt + i * P_PROD_THREADS;
+        if (p < nch * (P_KC / 2)) {
+            const int ch = p / (P_KC / 2), e2 = p % (P_KC / 2);
+            float2 r = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
+            uint32_t qb[G::KQ];
+#pragma unroll
+            for (int n = 0; n < K; ++n)
+                qb[n] = ld_shared_u16(slot + G::RAW_Q + (uint32_t)((n * G::CH + ch) * P_KC + e2 * 2)) ^
+                        0x8080u;
+            const uint32_t cofs = (uint32_t)(e2 & 1) * 8u;
+#pragma unroll
+            for (int n = 0; n < KP1; ++n) {
+                float2 hi, lo;
+                split2(r, hi, lo);
+                const uint32_t off = sw128_offset(ch * KP1 + n, e2 >> 1) + cofs;
+                st_shared_v2(sb + P_OFF_A_HI + off, hi);
+                st_shared_v2(sb + P_OFF_A_LO + off, lo);
+                if (n < K) {
+                    const float sn = sc[i][n];
+                    r.x = __fmaf_rn(-sn, code_from_biased(qb[n], 0), r.x);
+                    r.y = __fmaf_rn(-sn, code_from_biased(qb[n], 1), r.y);
+                }
+            }
+        }
+    }
+}
+
+template <int KP1>
+__global__ void __launch_bounds__(P_THREADS, 1)
+output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d,
+                         float *__restrict__ err, int split,
+                         const __grid_constant__ CUtensorMap tmX,
+                         const __grid_constant__ CUtensorMap tmW,
+                         const __grid_constant__ CUtensorMap tmQ)
+{
+    using G = PGeo<KP1>;
+    constexpr int R = G::RAW_STAGES;
+    extern __shared__ unsigned char smem_raw[];
+    const uint32_t raw_u32 = smem_u32(smem_raw);
+    const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
+    PairCtrl &ctl = *reinterpret_cast<PairCtrl *>(smem_raw + pad);
+    const uint32_t stages_u32 = raw_u32 + pad + P_CTRL_BYTES;
+    const uint32_t ring_u32 = stages_u32 + P_STAGES * P_STAGE_BYTES;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t crank = cluster_ctarank();
+    const int half = (int)(crank & 1u);              // 0: even CTA (issues the MMAs), 1: its peer
+    const uint32_t leader = crank & ~1u;
+    const uint16_t pair_mask = (uint16_t)(3u << leader);
+    const int pr = (int)(crank >> 1);                // pair index in the cluster: row-tile phase
+    const int pair_tile = blockIdx.x / (2 * split);
+    const int k0 = (pair_tile * 2 + half) * G::CH;   // first channel of this CTA
+    const int nch = max(0, min(G::CH, C - k0));
+    const int nvec = nch * KP1;
+    const int n_rt = (N + P_N - 1) / P_N;
+    const int my_rt = (n_rt - pr + split - 1) / split;
+    const int n_kc = (d + P_KC - 1) / P_KC;
+    const int nseg = (n_kc + P_SEG - 1) / P_SEG;
+    const int total = my_rt * n_kc;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < P_STAGES; ++s) {
+            mbar_init(&ctl.full[s], 2 * P_PROD_WARPS);
+            mbar_init(&ctl.empty[s], 1);
+        }
+        for (int r = 0; r < P_MAX_RAW; ++r) {
+            mbar_init(&ctl.raw_full[r], 1);
+            mbar_init(&ctl.raw_empty[r], P_PROD_WARPS);
+        }
+        mbar_init(&ctl.segfull, 1);
+        mbar_init(&ctl.segempty, 2 * 4);
+        mbar_init(&ctl.done, 1);
+        ctl.abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == P_MMA_WARP) {
+        tmem_alloc_pair(&ctl.tmem_base, P_TMEM_COLS);
+        tc_fence_before();
+    }
+    cluster_sync();                     // barriers of both CTAs initialised, TMEM allocated
+    tc_fence_after();
+    const uint32_t tmem = ctl.tmem_base;
+    volatile int *abort_flag = &ctl.abort;
+
+    if (warp < P_PROD_WARPS) {
+        // ---------------------------------------------------------------- producers
+        const int pt = threadIdx.x;
+        float sc[G::ITEMS2][G::KQ];     // scales of this thread's items, the same for every chunk
+#pragma unroll
+        for (int i = 0; i < G::ITEMS2; ++i) {
+            const int p = pt + i * P_PROD_THREADS;
+            const int k = k0 + p / (P_KC / 2);
+#pragma unroll
+            for (int n = 0; n < G::KQ; ++n)
+                sc[i][n] = (n < KP1 - 1 && p < nch * (P_KC / 2))
+                               ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
+        }
+        for (int it = 0; it < total; ++it) {
+            const int s = it % P_STAGES, slot = it % R;
+            const uint32_t ph = (uint32_t)(it / P_STAGES) & 1u;
+            const bool ok = mbar_wait(&ctl.raw_full[slot], (uint32_t)(it / R) & 1u, P_WAIT) &&
+                            mbar_wait_cluster(&ctl.empty[s], ph ^ 1u, P_WAIT);
+            if (!ok) *abort_flag = 1;
+            if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
+            pair_consume<KP1>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + s * P_STAGE_BYTES, pt,
+                              nch, sc);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive_cluster(&ctl.full[s], leader);
+                mbar_arrive(&ctl.raw_empty[slot]);
+            }
+        }
+    } else if (warp < P_MMA_WARP) {
+        // ---------------------------------------------------------------- epilogue
+        const int ew = warp - P_EPI_WARP0;
+        const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16);
+        double acc = 0.0;
+        int g = 0;
+        bool stop = false;
+        for (int lt = 0; lt < my_rt && !stop; ++lt) {
+            for (int sg = 0; sg < nseg; ++sg, ++g) {
+                const bool ok = mbar_wait_cluster(&ctl.segfull, (uint32_t)g & 1u, P_WAIT);
+                if (!ok) *abort_flag = 1;
+                stop = __any_sync(0xffffffffu, !ok || *abort_flag);   // warp-uniform
+                if (stop) break;
+                tc_fence_after();
+                const bool first = (sg == 0), last = (sg == nseg - 1);
+#pragma unroll 1
+                for (int cb = 0; cb < P_N / 32; ++cb) {
+                    const uint32_t col = (uint32_t)(cb * 32);
+                    float v[32];
+                    tmem_ld_32x32b_x32(lane_base + col, v);
+                    if (!first) {
+                        float r[32];
+                        tmem_ld_32x32b_x32(lane_base + P_RUN_COL + col, r);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __fadd_rn(v[i], r[i]);
+                    }
+                    if (last) {
+                        float p = 0.0f;
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) p = fmaf(v[i], v[i], p);
+                        acc += (double)p;
+                    } else {
+                        tmem_st_32x32b_x32(lane_base + P_RUN_COL + col, v);
+                    }
+                }
+                if (!last) tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(&ctl.segempty, leader);
+            }
+        }
+        ctl.part[ew * 32 + lane] = *abort_flag ? (double)NAN : acc;
+    } else if (warp == P_MMA_WARP) {
+        // ---------------------------------------------------------------- MMA issuer (even CTA)
+        if (half == 0 && lane == 0) {
+            constexpr uint32_t idesc = idesc_tf32(2 * P_VEC, P_N);
+            int g = 0;
+            for (int lt = 0; lt < my_rt && !*abort_flag; ++lt) {
+                for (int kc = 0; kc < n_kc; ++kc) {
+                    const bool seg_start = (kc % P_SEG) == 0;
+                    if (seg_start) {
+                        // both CTAs' epilogues must have drained the previous segment
+                        if (!mbar_wait_cluster(&ctl.segempty, ((uint32_t)g & 1u) ^ 1u, P_WAIT))
+                            *abort_flag = 1;
+                        if (*abort_flag) break;
+                        tc_fence_after();
+                    }
+                    const int it = lt * n_kc + kc;
+                    const int s = it % P_STAGES;
+                    const uint32_t ph = (uint32_t)(it / P_STAGES) & 1u;
+                    if (!mbar_wait_cluster(&ctl.full[s], ph, P_WAIT)) *abort_flag = 1;
+                    if (*abort_flag) break;
+                    tc_fence_after();
+                    const uint32_t sb = stages_u32 + s * P_STAGE_BYTES;
+                    const uint64_t ah = smem_desc_sw128(sb + P_OFF_A_HI);
+                    const uint64_t al = smem_desc_sw128(sb + P_OFF_A_LO);
+                    const uint64_t bh = smem_desc_sw128(sb + P_OFF_B_HI);
+                    const uint64_t bl = smem_desc_sw128(sb + P_OFF_B_LO);
+#pragma unroll
+                    for (int kk = 0; kk < P_KC / 8; ++kk) {
+                        const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
+                        mma_tf32_pair(tmem, al + o, bh + o, idesc, (seg_start && kk == 0) ? 0u : 1u);
+                        mma_tf32_pair(tmem, ah + o, bl + o, idesc, 1u);
+                        mma_tf32_pair(tmem, ah + o, bh + o, idesc, 1u);
+                    }
+                    mma_commit_pair(&ctl.empty[s], pair_mask);
+                    if ((kc % P_SEG) == P_SEG - 1 || kc == n_kc - 1) {
+                        mma_commit_pair(&ctl.segfull, pair_mask);
+                        ++g;
+                    }
+                }
+            }
+            // drain: every MMA issued above completes before TMEM is released
+            mma_commit_pair(&ctl.done, (uint16_t)(1u << leader));
+            mbar_wait_cluster(&ctl.done, 0, P_WAIT);
+        }
+        __syncwarp();
+    } else {
+        // ---------------------------------------------------------------- raw tile copies
+        if (lane == 0) {
+            prefetch_tensormap(&tmX);
+            prefetch_tensormap(&tmW);
+            prefetch_tensormap(&tmQ);
+            int issued = 0;
+            for (int f = 0; f < total; ++f) {
+                const int slot = f % R;
+                if (f >= R &&
+                    !mbar_wait(&ctl.raw_empty[slot], (uint32_t)(f / R - 1) & 1u, P_WAIT))
+                    *abort_flag = 1;
+                if (*abort_flag) break;
+                const uint32_t dst = ring_u32 + slot * G::RAW_BYTES;
+                const int x = (f % n_kc) * P_KC;
+                const int row0 = (pr + (f / n_kc) * split) * P_N + half * P_ROWS;
+                mbar_arrive_expect_tx(&ctl.raw_full[slot], G::RAW_TX);
+                tma_load_2d(dst, &tmX, x, row0, &ctl.raw_full[slot]);
+                tma_load_2d(dst + G::RAW_W, &tmW, x, k0, &ctl.raw_full[slot]);
+                tma_load_3d(dst + G::RAW_Q, &tmQ, x, k0, 0, &ctl.raw_full[slot]);
+                issued = f + 1;
+            }
+            // no copy may land after the CTA is gone: wait for the last copies of every slot
+            for (int f = issued - R > 0 ? issued - R : 0; f < issued; ++f)
+                mbar_wait(&ctl.raw_full[f % R], (uint32_t)(f / R) & 1u, P_WAIT);
+        }
+        __syncwarp();
+    }
+
+    // ---------------------------------------------------------------- cluster reduction
+    cluster_sync();
+    if (crank < 2 && warp >= P_EPI_WARP0 && warp < P_MMA_WARP) {
+        const int m = (warp - P_EPI_WARP0) * 32 + lane;
+        if (m < nvec) {
+            double s = 0.0;
+            for (int j = 0; j < split; ++j) s += ld_dsmem_f64(&ctl.part[m], crank + 2u * (uint32_t)j);
+            err[(size_t)k0 * KP1 + m] = (float)(s / (double)N);
+        }
+    }
+    cluster_sync();
+    if (warp == P_MMA_WARP) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, P_TMEM_COLS);
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 pair_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+        return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+    }();
+    return fn;
+}
+
+// Tile map over a row-major tensor (dims[0] contiguous, byte strides for dims 1..), zero fill.
+bool pair_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *base,
+              const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box)
+{
+    PFN_cuTensorMapEncodeTiled_v12000 enc = pair_map_encoder();
+    if (!enc) return false;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, type, (cuuint32_t)rank, const_cast<void *>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int KP1>
+mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *codes,
+                       const float *scales, int C, int d, float *err, cudaStream_t stream)
+{
+    using G = PGeo<KP1>;
+    const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
+    const int n_rt = (N + P_N - 1) / P_N;
+    const int sms = sm_count();
+    int split = 1;
+    while (split < 4 && split * 2 <= n_rt && (long long)n_pairs * 2 * split < 2LL * sms)
+        split *= 2;
+
+    CUtensorMap tmX, tmW, tmQ;
+    memset(&tmX, 0, sizeof(tmX));
+    memset(&tmW, 0, sizeof(tmW));
+    memset(&tmQ, 0, sizeof(tmQ));
+    const cuuint64_t dx[2] = {(cuuint64_t)d, (cuuint64_t)N}, sx[1] = {(cuuint64_t)d * 4};
+    const cuuint32_t bx[2] = {P_KC, P_ROWS};
+    const cuuint64_t dw[2] = {(cuuint64_t)d, (cuuint64_t)C}, sw[1] = {(cuuint64_t)d * 4};
+    const cuuint32_t bw[2] = {P_KC, (cuuint32_t)G::CH};
+    const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)C, (cuuint64_t)G::K};
+    const cuuint64_t sq[2] = {(cuuint64_t)d, (cuuint64_t)C * d};
+    const cuuint32_t bq[3] = {P_KC, (cuuint32_t)G::CH, (cuuint32_t)G::K};
+    if (!pair_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, X, dx, sx, bx) ||
+        !pair_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw) ||
+        !pair_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq)) {
+        set_error("output error: tensor map encoding failed");
+        return MPQ_ERR_CUDA;
+    }
+    if ((long long)G::SMEM > max_smem_optin()) {
+        set_error("pair output error needs %d bytes of shared memory", G::SMEM);
+        return MPQ_ERR_UNSUPPORTED;
+    }
+    cudaError_t e = cudaFuncSetAttribute(output_error_pair_kernel<KP1>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM);
+    if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
+
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(n_pairs * 2 * split), 1, 1);
+    cfg.blockDim = dim3(P_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = (size_t)G::SMEM;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)(2 * split);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1>, scales, C, N, d, err, split, tmX,
+                           tmW, tmQ);
+    return cuda_status(e, "pair output-error kernel launch");
+}
+
+}  // namespace
+
+bool output_error_pair_ok(const float *X, const float *W, const int8_t *codes, int d)
+{
+    return (d % 16 == 0) && ((uintptr_t)X % 16 == 0) && ((uintptr_t)W % 16 == 0) &&
+           ((uintptr_t)codes % 16 == 0);
+}
+
+mpq_status launch_output_error_pair(const float *X, int N, const float *W, const int8_t *codes,
+                                    const float *scales, int C, int d, int k_max, float *err,
+                                    cudaStream_t stream)
+{
+    switch (k_max + 1) {
+#define MPQ_CASE(n) \
+    case n: return launch_pair<n>(X, N, W, codes, scales, C, d, err, stream);
+        MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7) MPQ_CASE(8)
+        MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14) MPQ_CASE(15)
+        MPQ_CASE(16) MPQ_CASE(17)
+#undef MPQ_CASE
+    }
+    set_error("k_max = %d unsupported", k_max);
+    return MPQ_ERR_UNSUPPORTED;
+}
+
+}  // namespace mpq

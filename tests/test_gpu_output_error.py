@@ -18,7 +18,12 @@ def gpu_err(X, W, codes, scales, k_max, groups=1, dev="cuda:0"):
 
 @pytest.mark.parametrize("C,d,N,K", [(1, 1, 1, 1), (3, 5, 7, 2), (5, 33, 70, 4), (7, 64, 64, 3),
                                      (11, 147, 129, 4), (4, 1000, 65, 2), (64, 576, 512, 4),
-                                     (2, 17, 300, 16)])
+                                     (2, 17, 300, 16),
+                                     # d % 16 == 0 (CTA-pair kernel): several pair tiles with a
+                                     # part-filled last pair, an empty odd CTA, ragged row tiles
+                                     # split over a cluster, k_max + 1 from 2 to 17
+                                     (130, 256, 600, 4), (30, 128, 1000, 1), (9, 32, 300, 16),
+                                     (50, 512, 1100, 6), (3, 48, 20, 8)])
 def test_shared_input(gpu, oracle, C, d, N, K):
     W = wlm.random_weights(C, d, C + d + N, "normal")
     q = oracle.quantize_layer(W, 4, 32, K)
