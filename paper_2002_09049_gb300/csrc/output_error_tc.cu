@@ -1,12 +1,14 @@
-// Output error (Sec. 3.3, Eq. 11) on the 5th-generation tensor cores:
+// Output error (Sec. 3.3, Eq. 11) on the 5th-generation tensor cores, single-CTA form:
 //   err[k][n] = (1/N) sum_t (x_t . r_{k,n+1})^2,  n = 0..k_max.
+// It serves the shapes the CTA-pair kernel's TMA tile copies cannot address (rows whose byte
+// length is not a multiple of 16, or unaligned buffers); producers read global memory directly.
 //
 // As a contraction: Y = R X^T with R the C*(k_max+1) residual vectors (rows) and X the N
 // calibration rows, both of length d; err is the row-wise mean of Y^2.  Mapping:
 //   * A operand = residual vectors, 256 per CTA as two M = 128 halves (TMEM lanes = vectors),
 //     whole channels per CTA (floor(256/(k_max+1)) channels);
 //   * B operand = 128 calibration rows per row tile (UMMA N = 128);
-//   * K = d in chunks of 16 fp32 (one 64-byte swizzle row).
+//   * K = d in chunks of 32 fp32 (one 128-byte swizzle row).
 // fp32-grade products with tcgen05 kind::tf32: each operand x is split exactly into
 // hi = x with the 13 low mantissa bits cleared (a tf32 value) and lo = x - hi, and
 // Y = hi*hi + hi*lo + lo*hi (the dropped lo*lo term is ~2^-22 relative).
@@ -18,29 +20,18 @@
 // running sum kept in tensor memory with round-to-nearest fp32 additions.  TMEM columns:
 // [0, 256) segment accumulators of the two halves, [256, 512) running sums.
 //
-// Warp roles (448 threads): warps 0-7 produce operand stages in shared memory (X rows and the
+// Warp roles (416 threads): warps 0-7 produce operand stages in shared memory (X rows and the
 // residuals, which are regenerated from W, codes and scales by the recursion of Eq. 7 and never
-// exist in global memory); warps 8-11 fold segments into the running sums and square-sum the
-// finished row tiles; warp 12 owns TMEM and one of its threads issues the MMAs; one thread of
-// warp 13 streams the raw input tiles.
-//
-// Producer input.  When d % 16 == 0 and the rows are aligned, each chunk's X rows, W rows and codes
-// arrive as three TMA tile copies in a ring of RAW_STAGES shared-memory slots, several chunks ahead
-// of the producers (rows past N and channels past C read as zeros).  The residual recursion is
-// spread over all producer threads as (channel, element pair) items; codes become floats exactly
-// through the fp32 exponent bias (2^23 + (q + 128) - (2^23 + 128)).  Otherwise the producers
-// prefetch the next chunk into registers with guarded loads.
+// exist in global memory), prefetching the next stage's global data into registers with guarded
+// loads while the current one is consumed; warps 8-11 fold segments into the running sums and
+// square-sum the finished row tiles; warp 12 owns TMEM and one of its threads issues the MMAs.
+// Each warp reports a stage with one arrival, and stops only on a warp-uniform decision.
 //
 // Row tiles are split over the CTAs of a thread-block cluster; rank 0 adds the partial sums of
 // its peers from distributed shared memory in rank order, so every result is written once, in a
 // fixed order, with no global scratch and no atomics.  Every wait is bounded; on a timeout the
 // CTA unwinds and its outputs read NaN.
-#include <cuda.h>
-#include <cudaTypedefs.h>
 #include <math.h>
-#include <string.h>
-
-#include <mutex>
 
 #include "mpq_internal.cuh"
 #include "sm100.cuh"
@@ -55,35 +46,29 @@ constexpr int TC_M = 128;                       // vectors per accumulator (TMEM
 constexpr int TC_HALVES = 2;                    // accumulators per CTA
 constexpr int TC_VEC = TC_M * TC_HALVES;        // 256 vectors per CTA
 constexpr int TC_ROWS = 128;                    // calibration rows per row tile (UMMA N)
-constexpr int TC_KC = 16;                       // fp32 per K chunk = one 64-byte swizzle row
-constexpr int KC4 = TC_KC / 4;                  // float4 per chunk row
-constexpr int SEG_CHUNKS = 8;                   // accumulator restart period: 128 elements of d
-constexpr int TC_STAGES = 3;                    // operand stages
-constexpr int A_TILE = TC_M * TC_KC * 4;        // 8 KB
-constexpr int B_TILE = TC_ROWS * TC_KC * 4;     // 8 KB
+constexpr int TC_KC = 32;                       // fp32 per K chunk = one 128-byte row
+constexpr int SEG_CHUNKS = 4;                   // accumulator restart period (chunks)
+constexpr int TC_STAGES = 2;
+constexpr int A_TILE = TC_M * TC_KC * 4;        // 16 KB
+constexpr int B_TILE = TC_ROWS * TC_KC * 4;     // 16 KB
 constexpr int OFF_A_HI = 0;                     // + h * A_TILE
 constexpr int OFF_A_LO = TC_HALVES * A_TILE;    // + h * A_TILE
 constexpr int OFF_B_HI = 2 * TC_HALVES * A_TILE;
 constexpr int OFF_B_LO = OFF_B_HI + B_TILE;
-constexpr int STAGE_BYTES = OFF_B_LO + B_TILE;  // 48 KB
+constexpr int STAGE_BYTES = OFF_B_LO + B_TILE;  // 96 KB
 constexpr int PRODUCER_WARPS = 8;
 constexpr int PRODUCER_THREADS = PRODUCER_WARPS * 32;
 constexpr int X_PER_THREAD = TC_ROWS * TC_KC / 4 / PRODUCER_THREADS;   // float4 per thread
 constexpr int EPI_WARP0 = PRODUCER_WARPS;       // warps 8..11: warp % 4 selects TMEM lanes
 constexpr int MMA_WARP = EPI_WARP0 + 4;
-constexpr int TMA_WARP = MMA_WARP + 1;
-constexpr int TC_THREADS = (TMA_WARP + 1) * 32; // 448
+constexpr int TC_THREADS = (MMA_WARP + 1) * 32; // 416
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t RUN_COL = 256;               // running sums start here
 constexpr long long WAIT_BUDGET = 1LL << 31;    // SM clocks (~1 s)
 
-constexpr int MAX_RAW = 4;                      // raw TMA slots at most
-
 struct Ctrl {
     uint64_t full[TC_STAGES];
     uint64_t empty[TC_STAGES];
-    uint64_t raw_full[MAX_RAW];
-    uint64_t raw_empty[MAX_RAW];
     uint64_t segfull;
     uint64_t segempty;
     uint64_t done;
@@ -92,30 +77,7 @@ struct Ctrl {
     double part[TC_VEC];
 };
 constexpr int CTRL_BYTES = (sizeof(Ctrl) + 1023) / 1024 * 1024;
-constexpr int SMEM_LIMIT = 232448;              // opt-in shared memory per CTA on sm_100 parts
-constexpr int BASE_SMEM = 1024 /* alignment slack */ + CTRL_BYTES + TC_STAGES * STAGE_BYTES;
-
-// Per-KP1 geometry: channels per CTA, float4 (channel, column) items per producer thread for the
-// register-prefetch path, (channel, element pair) items per thread for the TMA path, and the
-// layout of one raw TMA slot, which is the order the tile copies write: X chunk [128 rows][16]
-// fp32, W chunk [CH][16] fp32, codes [K][CH][16] int8, each part 128-byte aligned.
-template <int KP1>
-struct Geo {
-    static constexpr int K = KP1 - 1;
-    static constexpr int KQ = K > 0 ? K : 1;
-    static constexpr int CH = TC_VEC / KP1;
-    static constexpr int PAIRS = (CH * KC4 + PRODUCER_THREADS - 1) / PRODUCER_THREADS;
-    static constexpr int ITEMS2 = (CH * (TC_KC / 2) + PRODUCER_THREADS - 1) / PRODUCER_THREADS;
-    static constexpr int RAW_W = TC_ROWS * TC_KC * 4;
-    static constexpr int RAW_Q = (RAW_W + CH * TC_KC * 4 + 127) / 128 * 128;
-    static constexpr uint32_t RAW_TX = TC_ROWS * TC_KC * 4 + CH * TC_KC * 4 + K * CH * TC_KC;
-    static constexpr int RAW_BYTES = (RAW_Q + KQ * CH * TC_KC + 1023) / 1024 * 1024;
-    static constexpr int RAW_FIT = (SMEM_LIMIT - BASE_SMEM) / RAW_BYTES;
-    static constexpr int RAW_STAGES = RAW_FIT < MAX_RAW ? RAW_FIT : MAX_RAW;
-    static constexpr int SMEM_SYNC = BASE_SMEM;
-    static constexpr int SMEM_TMA = BASE_SMEM + RAW_STAGES * RAW_BYTES;
-    static_assert(RAW_STAGES >= 2, "raw ring needs two slots");
-};
+constexpr int TC_SMEM = 1024 /* alignment slack */ + CTRL_BYTES + TC_STAGES * STAGE_BYTES;
 
 __device__ __forceinline__ float4 load4_guarded(const float *__restrict__ p, int j, int d,
                                                 bool vec_ok)
@@ -149,11 +111,13 @@ __device__ __forceinline__ float code_byte(uint32_t w, int b)
 // Global data one producer thread needs for one stage.
 template <int KP1>
 struct Prefetch {
-    static constexpr int PAIRS = Geo<KP1>::PAIRS;
+    static constexpr int K = KP1 - 1;
+    static constexpr int CH = TC_VEC / KP1;                                // channels per CTA
+    static constexpr int PAIRS = (CH * 8 + PRODUCER_THREADS - 1) / PRODUCER_THREADS;
     float4 x[X_PER_THREAD];
     float4 w[PAIRS];
-    uint32_t q[PAIRS][Geo<KP1>::KQ];
-    float s[PAIRS][Geo<KP1>::KQ];
+    uint32_t q[PAIRS][K > 0 ? K : 1];
+    float s[PAIRS][K > 0 ? K : 1];
 };
 
 template <int KP1>
@@ -169,7 +133,7 @@ __device__ __forceinline__ void prefetch(Prefetch<KP1> &pf, int pt, int rt, int 
 #pragma unroll
     for (int i = 0; i < X_PER_THREAD; ++i) {
         const int q = pt + i * PRODUCER_THREADS;
-        const int row = q / KC4, c = q % KC4;
+        const int row = q >> 3, c = q & 7;
         const int t = rt * TC_ROWS + row;
         pf.x[i] = (t < N) ? load4_guarded(X + (size_t)t * d, jc + c * 4, d, vec_ok)
                           : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -177,8 +141,8 @@ __device__ __forceinline__ void prefetch(Prefetch<KP1> &pf, int pt, int rt, int 
 #pragma unroll
     for (int i = 0; i < Prefetch<KP1>::PAIRS; ++i) {
         const int p = pt + i * PRODUCER_THREADS;
-        if (p < nch * KC4) {
-            const int ch = p / KC4, c = p % KC4;
+        if (p < nch * 8) {
+            const int ch = p >> 3, c = p & 7;
             const int k = k0 + ch;
             const int j = jc + c * 4;
             pf.w[i] = load4_guarded(W + (size_t)k * d, j, d, vec_ok);
@@ -198,18 +162,18 @@ __device__ __forceinline__ void store_stage(const Prefetch<KP1> &pf, int pt, uin
 #pragma unroll
     for (int i = 0; i < X_PER_THREAD; ++i) {
         const int q = pt + i * PRODUCER_THREADS;
-        const int row = q / KC4, c = q % KC4;
+        const int row = q >> 3, c = q & 7;
         float4 hi, lo;
         split4(pf.x[i], hi, lo);
-        const uint32_t off = sw64_offset(row, c);
+        const uint32_t off = sw128_offset(row, c);
         st_shared_v4(sb + OFF_B_HI + off, hi);
         st_shared_v4(sb + OFF_B_LO + off, lo);
     }
 #pragma unroll
     for (int i = 0; i < Prefetch<KP1>::PAIRS; ++i) {
         const int p = pt + i * PRODUCER_THREADS;
-        if (p < nch * KC4) {
-            const int ch = p / KC4, c = p % KC4;
+        if (p < nch * 8) {
+            const int ch = p >> 3, c = p & 7;
             float4 r = pf.w[i];
 #pragma unroll
             for (int n = 0; n < KP1; ++n) {
@@ -217,7 +181,7 @@ __device__ __forceinline__ void store_stage(const Prefetch<KP1> &pf, int pt, uin
                 const int h = m >> 7, row = m & 127;
                 float4 hi, lo;
                 split4(r, hi, lo);
-                const uint32_t off = sw64_offset(row, c);
+                const uint32_t off = sw128_offset(row, c);
                 st_shared_v4(sb + OFF_A_HI + h * A_TILE + off, hi);
                 st_shared_v4(sb + OFF_A_LO + h * A_TILE + off, lo);
                 if (n < K) {
@@ -233,71 +197,17 @@ __device__ __forceinline__ void store_stage(const Prefetch<KP1> &pf, int pt, uin
     }
 }
 
-// Splits the raw slot into operand stage `sb`: X rows -> B tiles; for every (channel, element
-// pair) item the residuals r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7) -> A tiles.
 template <int KP1>
-__device__ __forceinline__ void consume_raw(uint32_t slot, uint32_t sb, int pt, int nch,
-                                            const float (&sc)[Geo<KP1>::ITEMS2][Geo<KP1>::KQ])
-{
-    using G = Geo<KP1>;
-    constexpr int K = KP1 - 1;
-#pragma unroll
-    for (int i = 0; i < X_PER_THREAD; ++i) {
-        const int q = pt + i * PRODUCER_THREADS;
-        float4 hi, lo;
-        split4(ld_shared_v4(slot + (uint32_t)q * 16u), hi, lo);
-        const uint32_t off = sw64_offset(q / KC4, q % KC4);
-        st_shared_v4(sb + OFF_B_HI + off, hi);
-        st_shared_v4(sb + OFF_B_LO + off, lo);
-    }
-#pragma unroll
-    for (int i = 0; i < G::ITEMS2; ++i) {
-        const int p = pt + i * PRODUCER_THREADS;
-        if (p < nch * (TC_KC / 2)) {
-            const int ch = p / (TC_KC / 2), e2 = p % (TC_KC / 2);
-            float2 r = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * TC_KC + e2 * 2) * 4u);
-            uint32_t qb[G::KQ];
-#pragma unroll
-            for (int n = 0; n < K; ++n)
-                qb[n] = ld_shared_u16(slot + G::RAW_Q + (uint32_t)((n * G::CH + ch) * TC_KC + e2 * 2)) ^
-                        0x8080u;
-            const uint32_t cofs = (uint32_t)(e2 & 1) * 8u;
-#pragma unroll
-            for (int n = 0; n < KP1; ++n) {
-                const int m = ch * KP1 + n;
-                const int h = m >> 7, row = m & 127;
-                float2 hi, lo;
-                split2(r, hi, lo);
-                const uint32_t off = sw64_offset(row, e2 >> 1) + cofs;
-                st_shared_v2(sb + OFF_A_HI + h * A_TILE + off, hi);
-                st_shared_v2(sb + OFF_A_LO + h * A_TILE + off, lo);
-                if (n < K) {
-                    const float sn = sc[i][n];
-                    r.x = __fmaf_rn(-sn, code_from_biased(qb[n], 0), r.x);
-                    r.y = __fmaf_rn(-sn, code_from_biased(qb[n], 1), r.y);
-                }
-            }
-        }
-    }
-}
-
-// TMA selects the input path: tile copies through the raw ring (tmX, tmW, tmQ describe X [N][d],
-// W [C][d] and codes [K][C][d]) or register prefetch with guarded loads (the maps are unused).
-template <int KP1, bool TMA>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restrict__ W,
                        const int8_t *__restrict__ codes, const float *__restrict__ scales, int C,
-                       int d, float *__restrict__ err, int split,
-                       const __grid_constant__ CUtensorMap tmX,
-                       const __grid_constant__ CUtensorMap tmW,
-                       const __grid_constant__ CUtensorMap tmQ)
+                       int d, float *__restrict__ err, int split, bool vec_ok)
 {
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
     Ctrl &ctl = *reinterpret_cast<Ctrl *>(smem_raw + pad);
     const uint32_t stages_u32 = raw_u32 + pad + CTRL_BYTES;
-    const uint32_t ring_u32 = stages_u32 + TC_STAGES * STAGE_BYTES;   // raw TMA slots
 
     constexpr int CH = TC_VEC / KP1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -318,10 +228,6 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
             mbar_init(&ctl.full[s], PRODUCER_WARPS);
             mbar_init(&ctl.empty[s], 1);
         }
-        for (int r = 0; r < MAX_RAW; ++r) {
-            mbar_init(&ctl.raw_full[r], 1);
-            mbar_init(&ctl.raw_empty[r], PRODUCER_WARPS);
-        }
         mbar_init(&ctl.segfull, 1);
         mbar_init(&ctl.segempty, 4);
         mbar_init(&ctl.done, 1);
@@ -341,55 +247,23 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
         // ---------------------------------------------------------------- producers
         const int pt = threadIdx.x;
         Prefetch<KP1> pf;
-        if constexpr (TMA) {
-            using G = Geo<KP1>;
-            constexpr int R = G::RAW_STAGES;
-            // scales of this thread's items are the same for every chunk
-            float sc[G::ITEMS2][G::KQ];
-#pragma unroll
-            for (int i = 0; i < G::ITEMS2; ++i) {
-                const int p = pt + i * PRODUCER_THREADS;
-                const int k = k0 + p / (TC_KC / 2);
-#pragma unroll
-                for (int n = 0; n < G::KQ; ++n)
-                    sc[i][n] = (n < KP1 - 1 && p < nch * (TC_KC / 2))
-                                   ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
-            }
-            for (int it = 0; it < total; ++it) {
-                const int s = it % TC_STAGES, slot = it % R;
-                const uint32_t ph = (uint32_t)(it / TC_STAGES) & 1u;
-                const bool ok = mbar_wait(&ctl.raw_full[slot], (uint32_t)(it / R) & 1u, WAIT_BUDGET) &&
-                                mbar_wait(&ctl.empty[s], ph ^ 1u, WAIT_BUDGET);
-                if (!ok) *abort_flag = 1;
-                if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-                consume_raw<KP1>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + s * STAGE_BYTES, pt,
-                                 nch, sc);
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    mbar_arrive(&ctl.full[s]);
-                    mbar_arrive(&ctl.raw_empty[slot]);
-                }
-            }
-        } else {
-            if (total > 0)
-                prefetch<KP1>(pf, pt, crank, 0, X, N, W, codes, scales, k0, nch, d, plane, false);
-            for (int it = 0; it < total; ++it) {
-                const int s = it % TC_STAGES;
-                const uint32_t ph = (uint32_t)(it / TC_STAGES) & 1u;
-                const bool ok = mbar_wait(&ctl.empty[s], ph ^ 1u, WAIT_BUDGET);
-                if (!ok) *abort_flag = 1;
-                if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-                store_stage<KP1>(pf, pt, stages_u32 + s * STAGE_BYTES, nch);
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&ctl.full[s]);
-                const int nx = it + 1;
-                if (nx < total) {
-                    const int lt = nx / n_kc, kc = nx % n_kc;
-                    prefetch<KP1>(pf, pt, crank + lt * split, kc, X, N, W, codes, scales, k0, nch,
-                                  d, plane, false);
-                }
+        if (total > 0)
+            prefetch<KP1>(pf, pt, crank, 0, X, N, W, codes, scales, k0, nch, d, plane, vec_ok);
+        for (int it = 0; it < total; ++it) {
+            const int s = it % TC_STAGES;
+            const uint32_t ph = (uint32_t)(it / TC_STAGES) & 1u;
+            const bool ok = mbar_wait(&ctl.empty[s], ph ^ 1u, WAIT_BUDGET);
+            if (!ok) *abort_flag = 1;
+            if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
+            store_stage<KP1>(pf, pt, stages_u32 + s * STAGE_BYTES, nch);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl.full[s]);
+            const int nx = it + 1;
+            if (nx < total) {
+                const int lt = nx / n_kc, kc = nx % n_kc;
+                prefetch<KP1>(pf, pt, crank + lt * split, kc, X, N, W, codes, scales, k0, nch,
+                              d, plane, vec_ok);
             }
         }
     } else if (warp < MMA_WARP) {
@@ -440,7 +314,7 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
         const bool ok = !*abort_flag;
         ctl.part[m0] = ok ? acc[0] : (double)NAN;
         ctl.part[TC_M + m0] = ok ? acc[1] : (double)NAN;
-    } else if (warp == MMA_WARP) {
+    } else {
         // ---------------------------------------------------------------- MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_tf32(TC_M, TC_ROWS);
@@ -462,12 +336,12 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
                     if (*abort_flag) break;
                     tc_fence_after();
                     const uint32_t sb = stages_u32 + s * STAGE_BYTES;
-                    const uint64_t bh = smem_desc_sw64(sb + OFF_B_HI);
-                    const uint64_t bl = smem_desc_sw64(sb + OFF_B_LO);
+                    const uint64_t bh = smem_desc_sw128(sb + OFF_B_HI);
+                    const uint64_t bl = smem_desc_sw128(sb + OFF_B_LO);
 #pragma unroll
                     for (int h = 0; h < TC_HALVES; ++h) {
-                        const uint64_t ah = smem_desc_sw64(sb + OFF_A_HI + h * A_TILE);
-                        const uint64_t al = smem_desc_sw64(sb + OFF_A_LO + h * A_TILE);
+                        const uint64_t ah = smem_desc_sw128(sb + OFF_A_HI + h * A_TILE);
+                        const uint64_t al = smem_desc_sw128(sb + OFF_A_LO + h * A_TILE);
                         const uint32_t dt = tmem + (uint32_t)(h * TC_ROWS);
 #pragma unroll
                         for (int kk = 0; kk < TC_KC / 8; ++kk) {
@@ -487,35 +361,6 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
             // drain: every MMA issued above completes before TMEM is released
             mma_commit(&ctl.done);
             mbar_wait(&ctl.done, 0, WAIT_BUDGET);
-        }
-        __syncwarp();
-    } else if constexpr (TMA) {
-        // ---------------------------------------------------------------- raw tile copies
-        if (lane == 0) {
-            using G = Geo<KP1>;
-            constexpr int R = G::RAW_STAGES;
-            prefetch_tensormap(&tmX);
-            prefetch_tensormap(&tmW);
-            prefetch_tensormap(&tmQ);
-            int issued = 0;
-            for (int f = 0; f < total; ++f) {
-                const int slot = f % R;
-                if (f >= R &&
-                    !mbar_wait(&ctl.raw_empty[slot], (uint32_t)(f / R - 1) & 1u, WAIT_BUDGET))
-                    *abort_flag = 1;
-                if (*abort_flag) break;
-                const uint32_t dst = ring_u32 + slot * G::RAW_BYTES;
-                const int x = (f % n_kc) * TC_KC;
-                const int rt = crank + (f / n_kc) * split;
-                mbar_arrive_expect_tx(&ctl.raw_full[slot], G::RAW_TX);
-                tma_load_2d(dst, &tmX, x, rt * TC_ROWS, &ctl.raw_full[slot]);
-                tma_load_2d(dst + G::RAW_W, &tmW, x, k0, &ctl.raw_full[slot]);
-                tma_load_3d(dst + G::RAW_Q, &tmQ, x, k0, 0, &ctl.raw_full[slot]);
-                issued = f + 1;
-            }
-            // no copy may land after the CTA is gone: wait for the last copies of every slot
-            for (int f = issued - R > 0 ? issued - R : 0; f < issued; ++f)
-                mbar_wait(&ctl.raw_full[f % R], (uint32_t)(f / R) & 1u, WAIT_BUDGET);
         }
         __syncwarp();
     }
@@ -541,41 +386,10 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
     }
 }
 
-// cuTensorMapEncodeTiled from the driver, looked up once.
-PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
-{
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                             &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    });
-    return fn;
-}
-
-// Tile map over a row-major tensor: dims[0] is the contiguous extent, strides in bytes for dims
-// 1.. ; box = {TC_KC, rows(, planes)}; zero fill outside.
-bool encode_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *base,
-                const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box)
-{
-    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
-    if (!enc) return false;
-    const cuuint32_t estr[3] = {1, 1, 1};
-    return enc(m, type, (cuuint32_t)rank, const_cast<void *>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int KP1>
 mpq_status launch_tc(const float *X, int N, const float *W, const int8_t *codes,
                      const float *scales, int C, int d, float *err, cudaStream_t stream)
 {
-    using G = Geo<KP1>;
     const int ch_per_tile = TC_VEC / KP1;
     const int n_tiles = (C + ch_per_tile - 1) / ch_per_tile;
     const int n_row_tiles = (N + TC_ROWS - 1) / TC_ROWS;
@@ -583,39 +397,17 @@ mpq_status launch_tc(const float *X, int N, const float *W, const int8_t *codes,
     const int sms = sm_count();
     while (split < 8 && split * 2 <= n_row_tiles && (long long)n_tiles * split < 2LL * sms)
         split *= 2;
+    const bool vec_ok = (d % 4 == 0) && ((uintptr_t)X % 16 == 0) && ((uintptr_t)W % 16 == 0) &&
+                        ((uintptr_t)codes % 4 == 0);
 
-    // TMA input path: 16-byte aligned rows for X, W and the int8 codes
-    CUtensorMap tmX, tmW, tmQ;
-    memset(&tmX, 0, sizeof(tmX));
-    memset(&tmW, 0, sizeof(tmW));
-    memset(&tmQ, 0, sizeof(tmQ));
-    bool tma = (d % 16 == 0) && ((uintptr_t)X % 16 == 0) && ((uintptr_t)W % 16 == 0) &&
-               ((uintptr_t)codes % 16 == 0);
-    if (tma) {
-        const cuuint64_t dx[2] = {(cuuint64_t)d, (cuuint64_t)N}, sx[1] = {(cuuint64_t)d * 4};
-        const cuuint32_t bx[2] = {TC_KC, TC_ROWS};
-        const cuuint64_t dw[2] = {(cuuint64_t)d, (cuuint64_t)C}, sw[1] = {(cuuint64_t)d * 4};
-        const cuuint32_t bw[2] = {TC_KC, (cuuint32_t)G::CH};
-        const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)C, (cuuint64_t)G::K};
-        const cuuint64_t sq[2] = {(cuuint64_t)d, (cuuint64_t)C * d};
-        const cuuint32_t bq[3] = {TC_KC, (cuuint32_t)G::CH, (cuuint32_t)G::K};
-        tma = encode_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, X, dx, sx, bx) &&
-              encode_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw) &&
-              encode_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq);
-    }
-    const int smem = tma ? G::SMEM_TMA : G::SMEM_SYNC;
-    if ((long long)smem > max_smem_optin()) {
-        set_error("tensor-core output error needs %d bytes of shared memory", smem);
-        return MPQ_ERR_UNSUPPORTED;
-    }
-    auto kernel = tma ? output_error_tc_kernel<KP1, true> : output_error_tc_kernel<KP1, false>;
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(output_error_tc_kernel<KP1>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
 
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(n_tiles * split), 1, 1);
     cfg.blockDim = dim3(TC_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.dynamicSmemBytes = TC_SMEM;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -624,7 +416,8 @@ mpq_status launch_tc(const float *X, int N, const float *W, const int8_t *codes,
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kernel, X, N, W, codes, scales, C, d, err, split, tmX, tmW, tmQ);
+    e = cudaLaunchKernelEx(&cfg, output_error_tc_kernel<KP1>, X, N, W, codes, scales, C, d, err,
+                           split, vec_ok);
     return cuda_status(e, "tensor-core output-error kernel launch");
 }
 
@@ -634,6 +427,10 @@ mpq_status launch_output_error_tc(const float *X, int N, const float *W, const i
                                   const float *scales, int C, int d, int k_max, float *err,
                                   cudaStream_t stream)
 {
+    if ((long long)TC_SMEM > max_smem_optin()) {
+        set_error("tensor-core output error needs %d bytes of shared memory", TC_SMEM);
+        return MPQ_ERR_UNSUPPORTED;
+    }
     switch (k_max + 1) {
 #define MPQ_CASE(n) \
     case n: return launch_tc<n>(X, N, W, codes, scales, C, d, err, stream);

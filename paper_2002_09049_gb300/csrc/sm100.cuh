@@ -240,18 +240,6 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
     return d;
 }
 
-// Same for the 64-byte swizzle layout (8-row x 64-byte atoms, atoms stacked every 512 bytes).
-__device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t saddr)
-{
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr & 0x3FFFF) >> 4);          // start address
-    d |= (uint64_t)1 << 16;                           // leading byte offset (unused for swizzled K-major)
-    d |= (uint64_t)(512 >> 4) << 32;                  // stride byte offset: next 8-row atom
-    d |= (uint64_t)1 << 46;                           // descriptor version (tcgen05)
-    d |= (uint64_t)4 << 61;                           // swizzle: 64B
-    return d;
-}
-
 // Instruction descriptor, kind::tf32: fp32 accumulate, A and B tf32, both K-major.
 __host__ __device__ constexpr uint32_t idesc_tf32(int M, int N)
 {

@@ -36,15 +36,8 @@ __device__ __forceinline__ float code_from_biased(uint32_t biased, int b)
                      8388736.0f);
 }
 
-// Byte offset of 16-byte chunk `chunk` (0..3) of row `row` of a K-major tile with 64-byte rows in
-// the 64-byte swizzle layout: 8-row atoms of 512 bytes, chunk XOR bits 1-2 of the row.
-__device__ __forceinline__ uint32_t sw64_offset(int row, int chunk)
-{
-    return (uint32_t)((row >> 3) * 512 + (row & 7) * 64 + ((chunk ^ ((row >> 1) & 3)) << 4));
-}
-
-// Same for 128-byte rows in the 128-byte swizzle layout: 8-row atoms of 1024 bytes, chunk (0..7)
-// XOR the row within the atom.
+// Byte offset of 16-byte chunk `chunk` (0..7) of row `row` of a K-major tile with 128-byte rows in
+// the 128-byte swizzle layout: 8-row atoms of 1024 bytes, chunk XOR the row within the atom.
 __device__ __forceinline__ uint32_t sw128_offset(int row, int chunk)
 {
     return (uint32_t)((row >> 3) * 1024 + (row & 7) * 128 + ((chunk ^ (row & 7)) << 4));
