@@ -32,7 +32,11 @@ METRIC = "weight-elements x scale-candidates x points / s"
 UNIT = "elem*cand*pt/s"
 PROFILES = os.path.join(ROOT, "profiles")
 KERNEL_SOURCES = {
-    "output_error": "paper_2002_09049_gb300/csrc/output_error_tc.cu",
+    "output_error": ("paper_2002_09049_gb300/csrc/output_error.cu",
+                     "paper_2002_09049_gb300/csrc/output_error_pair.cu",
+                     "paper_2002_09049_gb300/csrc/output_error_tc.cu",
+                     "paper_2002_09049_gb300/csrc/sm100.cuh",
+                     "paper_2002_09049_gb300/csrc/tf32_operands.cuh"),
     "quantize": "paper_2002_09049_gb300/csrc/quantize.cu",
     "allocate": "paper_2002_09049_gb300/csrc/allocate.cu",
     "reconstruct": "paper_2002_09049_gb300/csrc/reconstruct.cu",
@@ -73,8 +77,12 @@ def host_cores():
 
 
 def src_hash(rel):
-    with open(os.path.join(ROOT, rel), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """First 16 hex digits of the sha256 of a source file (or of several, concatenated)."""
+    h = hashlib.sha256()
+    for r in ([rel] if isinstance(rel, str) else rel):
+        with open(os.path.join(ROOT, r), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def measured_peaks():
@@ -337,7 +345,8 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
     if dominant == "output_error":
         peak = peaks["bf16_tflops"] * TF32_PER_BF16
         ach = fam_work[dominant] / t_s / 1e12
-        return {"kernel": "output_error_tc_kernel (Eq. 11, tcgen05 kind::tf32, 3-pass split)",
+        return {"kernel": "output_error_pair_kernel (Eq. 11, tcgen05 cta_group::2 kind::tf32, "
+                          "3-pass split; output_error_tc_kernel for rows not 16-byte multiples)",
                 "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
                 "frac": ach / peak, "traffic": traffic,
                 "peak_source": f"{peak_src} bf16 dense burst x nominal tf32/bf16 ratio "

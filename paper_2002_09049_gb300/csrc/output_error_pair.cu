@@ -32,6 +32,8 @@
 #include <math.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "mpq_internal.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
@@ -89,7 +91,7 @@ struct PGeo {
     static constexpr int KQ = K > 0 ? K : 1;
     static constexpr int CH = P_VEC / KP1;
     static constexpr int ITEMS2 = (CH * (P_KC / 2) + P_PROD_THREADS - 1) / P_PROD_THREADS;
-    static constexpr int X_ITEMS = P_ROWS * P_KC4 / P_PROD_THREADS;
+    static constexpr int X_ITEMS = (P_ROWS * P_KC4 + P_PROD_THREADS - 1) / P_PROD_THREADS;
     static constexpr int RAW_W = P_ROWS * P_KC * 4;
     static constexpr int RAW_Q = (RAW_W + CH * P_KC * 4 + 127) / 128 * 128;
     static constexpr uint32_t RAW_TX = P_ROWS * P_KC * 4 + CH * P_KC * 4 + K * CH * P_KC;
@@ -98,7 +100,6 @@ struct PGeo {
     static constexpr int RAW_STAGES = RAW_FIT < P_MAX_RAW ? RAW_FIT : P_MAX_RAW;
     static constexpr int SMEM = P_BASE_SMEM + RAW_STAGES * RAW_BYTES;
     static_assert(RAW_STAGES >= 2, "raw ring needs two slots");
-    static_assert(X_ITEMS * P_PROD_THREADS == P_ROWS * P_KC4, "X items");
 };
 
 // Raw slot -> operand stage `sb`: X rows -> B tiles; for every (channel, element pair) item the
@@ -112,6 +113,7 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
         const int q = pt + i * P_PROD_THREADS;
+        if (G::X_ITEMS * P_PROD_THREADS != P_ROWS * P_KC4 && q >= P_ROWS * P_KC4) break;
         float4 hi, lo;
         split4(ld_shared_v4(slot + (uint32_t)q * 16u), hi, lo);
         const uint32_t off = sw128_offset(q / P_KC4, q % P_KC4);
@@ -400,10 +402,6 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     using G = PGeo<KP1>;
     const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
     const int n_rt = (N + P_N - 1) / P_N;
-    const int sms = sm_count();
-    int split = 1;
-    while (split < 4 && split * 2 <= n_rt && (long long)n_pairs * 2 * split < 2LL * sms)
-        split *= 2;
 
     CUtensorMap tmX, tmW, tmQ;
     memset(&tmX, 0, sizeof(tmX));
@@ -431,17 +429,44 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
 
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(n_pairs * 2 * split), 1, 1);
     cfg.blockDim = dim3(P_THREADS, 1, 1);
     cfg.dynamicSmemBytes = (size_t)G::SMEM;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = (unsigned)(2 * split);
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+
+    // Row tiles split over `split` pairs per cluster (clusters of 2 * split CTAs).  Larger clusters
+    // fit fewer at a time on the GPU (SMs are grouped), so pick the split with the least
+    // (waves of resident clusters) x (row tiles per CTA), ties to the smaller cluster.
+    // resident clusters per cluster size, queried once per process (one device per process)
+    static std::atomic<int> resident[3] = {{0}, {0}, {0}};
+    int split = 1;
+    long long best = -1;
+    for (int sp = 1, i = 0; sp <= 4 && sp <= n_rt; sp *= 2, ++i) {
+        attr[0].val.clusterDim.x = (unsigned)(2 * sp);
+        cfg.gridDim = dim3((unsigned)(n_pairs * 2 * sp), 1, 1);
+        int active = resident[i].load(std::memory_order_relaxed);
+        if (active == 0) {
+            if (cudaOccupancyMaxActiveClusters(&active, output_error_pair_kernel<KP1>, &cfg) !=
+                cudaSuccess)
+                active = -1;
+            (void)cudaGetLastError();
+            resident[i].store(active, std::memory_order_relaxed);
+        }
+        if (active < 1) continue;
+        const long long waves = (n_pairs + active - 1) / active;
+        const long long cost = waves * ((n_rt + sp - 1) / sp);
+        if (best < 0 || cost < best) {
+            best = cost;
+            split = sp;
+        }
+    }
+    attr[0].val.clusterDim.x = (unsigned)(2 * split);
+    cfg.gridDim = dim3((unsigned)(n_pairs * 2 * split), 1, 1);
     e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1>, scales, C, N, d, err, split, tmX,
                            tmW, tmQ);
     return cuda_status(e, "pair output-error kernel launch");

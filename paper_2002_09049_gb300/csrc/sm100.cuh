@@ -77,15 +77,17 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity
     return true;
 }
 
-// Arrives (release, cluster scope) on the barrier at the same shared-memory offset as `bar` in
-// the CTA of cluster rank `rank` (possibly this one).
+// Arrives on the barrier at the same shared-memory offset as `bar` in the CTA of cluster rank
+// `rank` (possibly this one), with the default (CTA-scope) release.  Used as a signal only: what it
+// announces is ordered by the caller beforehand (a proxy fence after shared-memory writes that the
+// tensor cores read, or a completed tcgen05 load wait); a cluster-scope release here costs a
+// memory barrier per arrival.
 __device__ __forceinline__ void mbar_arrive_cluster(uint64_t *bar, uint32_t rank)
 {
     uint32_t remote;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)),
                  "r"(rank));
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote)
-                 : "memory");
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
 }
 
 __device__ __forceinline__ void fence_barrier_init()
