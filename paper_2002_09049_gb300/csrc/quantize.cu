@@ -73,18 +73,19 @@ struct Scratch {
 };
 
 // Shared memory: a CTA-wide table of the grid fractions f_g and fl(1/f_g) (2G words), then per
-// channel group (all 4-byte words): WPC private copies (one per warp, so warps never contend on
-// the same bin) of hLo[G+1], hHi[G+1] (64-bit P bins as two words) and hN[G+1], then r[d].
-// With the lattice form (below) each group also holds nb lattice buckets first: 64-bit R sums
-// (2 words each) and 32-bit counts.  Group regions are kept 8-byte aligned.
+// channel group (all 4-byte words): `copies` copies of hLo[G+1], hHi[G+1] (64-bit P bins as two
+// words) and hN[G+1], then r[d].  Without the lattice every warp has a private copy (so warps
+// never contend on a bin); with the lattice form (below) events are rare and the group shares one
+// copy, and the group also holds nb lattice buckets first: 64-bit R sums (2 words each) and
+// 32-bit counts.  Group regions are kept 8-byte aligned.
 __host__ __device__ constexpr size_t lattice_words(int nb)
 {
     return ((size_t)3 * nb + 1) & ~(size_t)1;
 }
 
-__host__ __device__ constexpr size_t group_words(int G, int d, int wpc, int nb)
+__host__ __device__ constexpr size_t group_words(int G, int d, int copies, int nb)
 {
-    return lattice_words(nb) + (((size_t)3 * (G + 1) * wpc + (size_t)d + 1) & ~(size_t)1);
+    return lattice_words(nb) + (((size_t)3 * (G + 1) * copies + (size_t)d + 1) & ~(size_t)1);
 }
 
 template <int WPC>
@@ -359,12 +360,20 @@ __device__ __forceinline__ void kahan_add(float &sum, float &comp, float x)
     sum = t;
 }
 
+// Exact 64-bit shared-memory accumulation from two 32-bit atomics: the low word's returned old
+// value shows whether it wrapped, and the carry goes into the high word with the high half.
+__device__ __forceinline__ void add64(unsigned int *lo_word, unsigned int *hi_word,
+                                      unsigned int Rlo, unsigned int Rhi)
+{
+    const unsigned int old = atomicAdd(lo_word, Rlo);
+    const unsigned int carry = (old + Rlo < old) ? 1u : 0u;
+    if (Rhi + carry) atomicAdd(hi_word, Rhi + carry);
+}
+
 __device__ __forceinline__ void add_event(unsigned int *hLo, unsigned int *hHi, int *hN, int T,
                                           unsigned int Rlo, unsigned int Rhi, int L)
 {
-    const unsigned int old = atomicAdd(&hLo[T], Rlo);
-    const unsigned int carry = (old + Rlo < old) ? 1u : 0u;   // exact wrap-around of the low word
-    if (Rhi + carry) atomicAdd(&hHi[T], Rhi + carry);
+    add64(&hLo[T], &hHi[T], Rlo, Rhi);
     atomicAdd(&hN[T], 2 * L - 1);
 }
 
@@ -389,6 +398,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
 {
     const int nb = LAT ? 2 * G * qmax + 1 : 0;   // lattice buckets: floor(2u) in [0, 2 G Qmax]
     constexpr int NT = WPC * 32;
+    constexpr int COPIES = LAT ? 1 : WPC;         // event bin copies per group
     constexpr int GPC = 8 / WPC;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ Scratch scratch[GPC];
@@ -410,18 +420,18 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
     if (k >= C) return;   // whole group idle (group-uniform)
 
     unsigned int *gl =
-        reinterpret_cast<unsigned int *>(finv + G) + (size_t)grp * group_words(G, d, WPC, nb);
+        reinterpret_cast<unsigned int *>(finv + G) + (size_t)grp * group_words(G, d, COPIES, nb);
     unsigned long long *latR = reinterpret_cast<unsigned long long *>(gl);   // [nb]
     unsigned int *latC = gl + 2 * (size_t)nb;                                 // [nb]
     unsigned int *gbase = gl + lattice_words(nb);
     // this warp's private bins; copy 0 receives the merged suffix sums
-    unsigned int *hLo = gbase + (size_t)gw * 3 * (G + 1);
+    unsigned int *hLo = gbase + (size_t)(COPIES > 1 ? gw : 0) * 3 * (G + 1);
     unsigned int *hHi = hLo + (G + 1);
     int *hN = reinterpret_cast<int *>(hHi + (G + 1));
     unsigned int *mLo = gbase;
     unsigned int *mHi = mLo + (G + 1);
     int *mN = reinterpret_cast<int *>(mHi + (G + 1));
-    float *sr = reinterpret_cast<float *>(gbase + (size_t)3 * (G + 1) * WPC);
+    float *sr = reinterpret_cast<float *>(gbase + (size_t)3 * (G + 1) * COPIES);
     Scratch &sc = scratch[grp];
 
     const size_t plane = (size_t)C * d;
@@ -469,8 +479,8 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             const int S = 62 - e - hbits;       // sum_j R_j c_j < 2^62
             const double down = pow2d(-S);
             const float smax_e = ldexpf(smax, -e);   // smax / 2^e for the fp32 screen
-            for (int t = lane; t <= G; t += 32) {   // each warp clears its own copy
-                hLo[t] = 0u;
+            for (int t = COPIES > 1 ? lane : gt; t <= G; t += COPIES > 1 ? 32 : NT) {
+                hLo[t] = 0u;   // each warp clears its own copy, or the group the shared one
                 hHi[t] = 0u;
                 hN[t] = 0;
             }
@@ -491,28 +501,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 const float g_per_a = __fdiv_rn((float)G, smax);   // linear grid: s_g ~ (g+1)/G*smax
                 long long Pb = 0;
                 long long Nb = 0;
-                for (int j = gt; j < d; j += NT) {
-                    const float a = fabsf(sr[j]);
-                    if (a == 0.0f) continue;
-                    if (LAT) {
-                        // Linear grid: level L is held at g iff u >= (g+1)(L - 1/2), u = aG/smax,
-                        // i.e. iff floor(2u) >= (g+1)(2L-1), an integer.  Unless 2u lies within
-                        // 2^-20 (relative) of an integer, one bucket update records the element
-                        // for every (g, L) exactly; near a lattice point the per-level events
-                        // below settle each threshold with the exact rule.
-                        const float u2 = 2.0f * (a * g_per_a);
-                        if (fabsf(u2 - rintf(u2)) > MPQ_FAST_REL * u2) {
-                            const int b = (int)floorf(u2);
-                            if (b >= 1) {
-                                const int bb = b < nb - 1 ? b : nb - 1;
-                                atomicAdd(&latR[bb], (unsigned long long)fixed_point(a, S));
-                                atomicAdd(&latC[bb], 1u);
-                            }
-                            continue;
-                        }
-                    }
+                // every level an element crosses inside the grid, one event each
+                auto events = [&](const float a) {
                     const int c_hi = code_fast(a, s0, i0, qmaxf);
-                    if (c_hi == 0) continue;   // code 0 at every scale: no contribution
+                    if (c_hi == 0) return;   // code 0 at every scale: no contribution
                     const int c_lo = code_fast(a, sG, iG, qmaxf);
                     const long long R = fixed_point(a, S);
                     Pb += R * (long long)c_lo;
@@ -559,10 +551,50 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
 #undef MPQ_HELD
                         add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
                     }
+                };
+                if (LAT) {
+                    // Linear grid: level L is held at g iff u >= (g+1)(L - 1/2), u = aG/smax, i.e.
+                    // iff floor(2u) >= (g+1)(2L-1), an integer.  Unless 2u lies within 2^-20
+                    // (relative) of an integer, one bucket update records the element for every
+                    // (g, L) exactly; near a lattice point the per-level events settle each
+                    // threshold with the exact rule.  Two elements per pass, for overlap.
+                    constexpr int U = 2;
+                    for (int j0 = gt; j0 < d; j0 += U * NT) {
+                        float av[U], u2[U];
+#pragma unroll
+                        for (int u = 0; u < U; ++u) {
+                            const int j = j0 + u * NT;
+                            av[u] = j < d ? fabsf(sr[j]) : 0.0f;
+                            u2[u] = 2.0f * (av[u] * g_per_a);
+                        }
+#pragma unroll
+                        for (int u = 0; u < U; ++u) {
+                            if (av[u] == 0.0f) continue;
+                            if (fabsf(u2[u] - rintf(u2[u])) > MPQ_FAST_REL * u2[u]) {
+                                const int b = (int)floorf(u2[u]);
+                                if (b >= 1) {
+                                    const int bb = b < nb - 1 ? b : nb - 1;
+                                    // two 32-bit atomics: measurably cheaper than one 64-bit
+                                    const unsigned long long R =
+                                        (unsigned long long)fixed_point(av[u], S);
+                                    unsigned int *Rw = reinterpret_cast<unsigned int *>(&latR[bb]);
+                                    add64(&Rw[0], &Rw[1], (unsigned int)R, (unsigned int)(R >> 32));
+                                    atomicAdd(&latC[bb], 1u);
+                                }
+                            } else {
+                                events(av[u]);
+                            }
+                        }
+                    }
+                } else {
+                    for (int j = gt; j < d; j += NT) {
+                        const float a = fabsf(sr[j]);
+                        if (a != 0.0f) events(a);
+                    }
                 }
                 group_sum2<WPC>(Pb, Nb, sc, gw, lane, grp);   // publishes the bins too
                 const long long Pbase = Pb, Nbase = Nb;
-                // ---- suffix sums over the event bins (the warps' private copies merged into
+                // ---- suffix sums over the event bins (private copies, if any, merged into
                 // copy 0; warp 0), in place: bin t <- sum of bins u >= t, so P_g = Pbase +
                 // bin(g + 1); and over the lattice buckets (warp 1 concurrently, or the whole
                 // group afterwards when the lattice is large)
@@ -570,7 +602,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     long long pp = bin64(mLo, mHi, t);
                     long long nn = mN[t];
 #pragma unroll
-                    for (int c = 1; c < WPC; ++c) {
+                    for (int c = 1; c < COPIES; ++c) {
                         const unsigned int *cLo = mLo + (size_t)c * 3 * (G + 1);
                         pp += bin64(cLo, cLo + (G + 1), t);
                         nn += reinterpret_cast<const int *>(cLo + 2 * (G + 1))[t];
@@ -591,8 +623,8 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     latR[t] = p;
                     latC[t] = (unsigned int)q;
                 };
-                // large grids (G * WPC bins to merge, or a long lattice): the whole group scans
-                const bool big = (LAT && nb > 2048) || G * WPC > 1024;
+                // large grids (G * COPIES bins to merge, or a long lattice): the whole group scans
+                const bool big = (LAT && nb > 2048) || G * COPIES > 1024;
                 if (big) {
                     group_suffix_scan<WPC>(1, G + 1, bins_load, bins_store, sc, gw, lane, grp);
                     if (LAT) group_suffix_scan<WPC>(0, nb, lat_load, lat_store, sc, gw, lane, grp);
@@ -765,8 +797,8 @@ mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid
     int wpc = wpc_c < wpc_e ? wpc_c : wpc_e;
     if (wpc < wpc_s) wpc = wpc_s;
     for (; wpc <= 8; wpc *= 2) {
-        const size_t smem =
-            (size_t)(8 / wpc) * group_words(G, d, wpc, nb) * 4 + (size_t)2 * G * sizeof(float);
+        const size_t smem = (size_t)(8 / wpc) * group_words(G, d, lat ? 1 : wpc, nb) * 4 +
+                            (size_t)2 * G * sizeof(float);
         if ((long long)smem <= smem_cap) {
             switch (wpc) {
             case 1:
