@@ -164,6 +164,22 @@ def quantize_bytes(wl, layer):
     return layer.C * (layer.d * (4 + wl.k_max) + 4 * wl.k_max + 4 * (wl.k_max + 1))
 
 
+# Greedy search (lattice form), algorithmic lane operations.  Per element-step: |r|, u2 = 2a*G/smax
+# (2), lattice-distance test (5), bucket index (3), 64-bit fixed point (6), three atomics (3) = 20;
+# residual update and code emission: code (6), sign (1), fma (1), two stores (2), compensated square
+# sum (4), max (1) = 15.  Per channel-step: clear, suffix scan and bucket reads of the
+# 2*G*Qmax + 1 buckets (7 per bucket), fold (4 per (g, L)), fp32 screen and argmin (12 per g).
+GREEDY_OPS_PER_ELEMENT_STEP = 35
+ALU_LANES_PER_SM = 128   # fp32 / int32 lanes per SM (4 SMSPs x 32)
+
+
+def quantize_ops(wl, layer, bits):
+    qmax = (1 << (bits - 1)) - 1
+    nb = 2 * wl.G * qmax + 1
+    per_channel_step = 7 * nb + 4 * wl.G * qmax + 12 * wl.G
+    return layer.C * wl.k_max * (GREEDY_OPS_PER_ELEMENT_STEP * layer.d + per_channel_step)
+
+
 def reconstruct_bytes(wl, layer):
     """Algorithmic HBM bytes of one mpq_reconstruct call at the budget's average point count:
     n_avg code bytes + one fp32 write per weight (scales and counts are negligible)."""
@@ -284,13 +300,14 @@ def run_ours(args, world, rank, local):
                 for k, f in enumerate(families):
                     fam_ms[f] += e[k].elapsed_time(e[k + 1])
                 fam_work["output_error"] += contraction_flops(wl, layer)
-                fam_work["quantize"] += quantize_bytes(wl, layer)
+                fam_work["quantize"] += quantize_ops(wl, layer, wl.bits[0])
                 fam_work["reconstruct"] += reconstruct_bytes(wl, layer)
                 fam_work["allocate"] += 4 * layer.C * (wl.k_max + 1) * 9 + 8 * layer.C
     total_fam = sum(fam_ms.values())
     dominant = max(fam_ms, key=fam_ms.get)
 
-    roofline = dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args)
+    roofline = dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args,
+                                 sm_count=torch.cuda.get_device_properties(dev).multi_processor_count)
     roofline["share"] = fam_ms[dominant] / total_fam if total_fam else None
     roofline["family_ms_per_step"] = {f: fam_ms[f] / args.steps for f in families}
     roofline["timing"] = ("CUDA events around every call in a single-stream pass of the same "
@@ -326,13 +343,15 @@ def run_ours(args, world, rank, local):
 TF32_PER_BF16 = 1.1 / 2.25   # nominal dense tf32 / bf16 tensor rates of the part
 
 
-def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
+def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_count=152):
     """Roofline entry of the kernel family with the largest measured time.
 
     output_error: tensor-pipe bound; achieved = algorithmic flops 2*N*d*C*(k_max+1) (the three
       tf32 split passes are not counted) / measured time; peak = measured bf16 dense burst peak x
       the nominal tf32/bf16 ratio.
-    quantize / reconstruct / allocate: HBM roofline; achieved = algorithmic bytes / time."""
+    quantize: ALU bound; achieved = algorithmic lane operations (quantize_ops) / time; peak = SMs x
+      128 lanes x the maximum SM clock.
+    reconstruct / allocate: HBM roofline; achieved = algorithmic bytes / time."""
     traffic = None
     tfile = os.path.join(PROFILES, "roofline_traffic.json")
     if os.path.exists(tfile):
@@ -351,10 +370,19 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args):
                 "frac": ach / peak, "traffic": traffic,
                 "peak_source": f"{peak_src} bf16 dense burst x nominal tf32/bf16 ratio "
                                f"{TF32_PER_BF16:.3f}"}
+    if dominant == "quantize":
+        mhz = peaks.get("sm_max_mhz", 2070.0)
+        peak = sm_count * ALU_LANES_PER_SM * mhz * 1e6 / 1e12
+        ach = fam_work[dominant] / t_s / 1e12
+        return {"kernel": "quantize_kernel (Eq. 7-9 lattice form, all k_max steps)", "bound": "alu",
+                "achieved": ach, "peak": peak, "unit": "Tlane-op/s", "frac": ach / peak,
+                "traffic": traffic,
+                "peak_source": f"{sm_count} SMs x {ALU_LANES_PER_SM} lanes x {mhz:.0f} MHz "
+                               f"(algorithmic ops: {GREEDY_OPS_PER_ELEMENT_STEP} per element-step "
+                               "+ per channel-step scan, fold and screen)"}
     hbm = peaks["hbm_gbs"]
     ach = fam_work.get(dominant, 0.0) / t_s / 1e9
-    names = {"quantize": "quantize_event_kernel (Eq. 7-9, all k_max steps)",
-             "reconstruct": "reconstruct_vec4_kernel (Eq. 4)",
+    names = {"reconstruct": "reconstruct_vec4_kernel (Eq. 4)",
              "allocate": "allocate_budget_kernel (Algorithm 2)"}
     return {"kernel": names.get(dominant, dominant), "bound": "hbm", "achieved": ach, "peak": hbm,
             "unit": "GB/s", "frac": ach / hbm, "traffic": traffic,
