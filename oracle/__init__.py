@@ -60,6 +60,12 @@ def _load():
         lib.mpqo_allocate_threshold.restype = L
         lib.mpqo_reconstruct.argtypes = [P, P, P, I, I, I, P]
         lib.mpqo_reconstruct.restype = None
+        lib.mpqo_clip_candidates.argtypes = [P, I, I, I, I, P]
+        lib.mpqo_clip_candidates.restype = None
+        lib.mpqo_clip_errors.argtypes = [P, I, I, P, I, I, I, I, P, P, I, I, P]
+        lib.mpqo_clip_errors.restype = None
+        lib.mpqo_clip_select.argtypes = [P, I, I, I, P]
+        lib.mpqo_clip_select.restype = None
         _lib = lib
     return _lib
 
@@ -177,6 +183,51 @@ def reconstruct(codes, scales, npoints):
     W_hat = np.zeros((C, d), np.float32)
     lib.mpqo_reconstruct(_p(codes), _p(scales), _p(npoints), C, d, k_max, _p(W_hat))
     return W_hat
+
+
+CLIP_PER_CHANNEL = 0
+CLIP_PER_LAYER = 1
+
+
+def clip_candidates(W, n_cand: int, mode: int):
+    """Eq. 12's candidate clipping factors K_c = (c+1)/n_cand * max|w| (per channel or per layer)."""
+    lib = _load()
+    W = _c(W, np.float32)
+    C, d = W.shape
+    clip = np.zeros((C, n_cand), np.float32)
+    lib.mpqo_clip_candidates(_p(W), C, d, n_cand, mode, _p(clip))
+    return clip
+
+
+def clip_errors(X, groups: int, W, bits: int, clip, channels=None, threads: int = 1):
+    """Eq. 12's objective: output error (Eq. 11 form) of every candidate clipping factor, in double."""
+    lib = _load()
+    W = _c(W, np.float32)
+    C, d = W.shape
+    X = _c(X, np.float32)
+    N = X.shape[-2]
+    clip = _c(clip, np.float32)
+    n_cand = clip.shape[1]
+    err = np.zeros((C, n_cand), np.float64)
+    c0, c1 = channels if channels is not None else (0, C)
+
+    def run(rng):
+        work = np.empty(d, np.float32)
+        lib.mpqo_clip_errors(_p(X), N, groups, _p(W), C, d, bits, n_cand, _p(clip), _p(err),
+                             rng[0], rng[1], _p(work))
+
+    _parallel(run, [(a + c0, b + c0) for a, b in _ranges(c1 - c0, threads)], threads)
+    return err
+
+
+def clip_select(err32, mode: int):
+    """Eq. 12's argmin on an fp32 error table: per channel, or per layer (sum over channels)."""
+    lib = _load()
+    err32 = _c(err32, np.float32)
+    C, n_cand = err32.shape
+    best = np.zeros(C, np.int32)
+    lib.mpqo_clip_select(_p(err32), C, n_cand, mode, _p(best))
+    return best
 
 
 def _parallel(fn, ranges, threads):

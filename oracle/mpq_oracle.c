@@ -307,3 +307,100 @@ void mpqo_reconstruct(const int8_t *codes, const float *scales, const int *npoin
         }
     }
 }
+
+/* ---- Eq. 12: output-error-driven clipping factor ------------------------------------------------
+ * The clipping factor K of the quantization set K x [-1 : eps_b : 1] (Eq. 1, B = 0) is chosen among
+ * nc candidates by the output error of Eq. 11 instead of the weight error.  Readings (also in
+ * the design doc): the candidates are K_c = f_c * m with f_c = (c+1)/nc in fp32, c = 0..nc-1 (nc = 20 is
+ * the experiments' uniform grid [0.05 : 0.05 : 1] x max|w|); m = max_j |w_kj| per channel
+ * (mode 0) or the maximum over the whole layer (mode 1, one K for every channel); the set's
+ * elements are s q with s = K / Qmax (fp32 division) and codes q = [w / s]_Q as in Eq. 8; the
+ * residual is fmaf(-s, q, w); a non-finite weight makes m -- and so every K of that channel, or of
+ * the layer in mode 1 -- NaN. */
+
+/* Candidate clipping factors clip[k][c] of channels 0..C-1. */
+void mpqo_clip_candidates(const float *W, int C, int d, int nc, int mode, float *clip)
+{
+    float layer_m = 0.0f;
+    for (int k = 0; k < C; ++k) {
+        const float *w = W + (long)k * d;
+        float m = 0.0f;
+        if (!all_finite(w, d)) {
+            m = NAN;
+        } else {
+            for (int j = 0; j < d; ++j)
+                if (fabsf(w[j]) > m) m = fabsf(w[j]);
+        }
+        if (mode == 0) {
+            for (int c = 0; c < nc; ++c) clip[(long)k * nc + c] = ((float)(c + 1) / (float)nc) * m;
+        }
+        if (isnan(m) || isnan(layer_m)) layer_m = NAN;
+        else if (m > layer_m) layer_m = m;
+    }
+    if (mode == 1)
+        for (int k = 0; k < C; ++k)
+            for (int c = 0; c < nc; ++c)
+                clip[(long)k * nc + c] = ((float)(c + 1) / (float)nc) * layer_m;
+}
+
+/* The objective of Eq. 12 for every candidate of channels [c0, c1):
+ * err[k][c] = (1/N) sum_t (x_t . r_{k,c})^2, r_{k,c} = fmaf(-s, [w_k / s]_Q, w_k), s = K_{k,c} / Qmax,
+ * dot products and the mean in double.  groups as in mpqo_output_error.  work: d floats. */
+void mpqo_clip_errors(const float *X, int N, int groups, const float *W, int C, int d, int bits,
+                      int nc, const float *clip, double *err, int c0, int c1, float *work)
+{
+    const int qmax = qmax_of(bits);
+    for (int k = c0; k < c1; ++k) {
+        const float *Xk = (groups == 1) ? X : X + (long)k * N * d;
+        const float *w = W + (long)k * d;
+        for (int c = 0; c < nc; ++c) {
+            const float s = clip[(long)k * nc + c] / (float)qmax;
+            for (int j = 0; j < d; ++j)
+                work[j] = fmaf(-s, (float)nearest_code(w[j], s, qmax), w[j]);
+            double acc = 0.0;
+            for (int t = 0; t < N; ++t) {
+                const float *x = Xk + (long)t * d;
+                double y = 0.0;
+                for (int j = 0; j < d; ++j) y += (double)x[j] * (double)work[j];
+                acc += y * y;
+            }
+            err[(long)k * nc + c] = acc / (double)N;
+        }
+    }
+}
+
+/* The argmin of Eq. 12 on an error table of fp32 values (as the device computes them):
+ * mode 0, per channel: the lowest c with the smallest err[k][c];
+ * mode 1, per layer: the lowest c with the smallest sum_k err[k][c] (double, k ascending), the same
+ * c for every channel.  NaN never wins; no finite candidate gives -1. */
+void mpqo_clip_select(const float *err, int C, int nc, int mode, int *best)
+{
+    if (mode == 0) {
+        for (int k = 0; k < C; ++k) {
+            int b = -1;
+            float bv = 0.0f;
+            for (int c = 0; c < nc; ++c) {
+                const float v = err[(long)k * nc + c];
+                if (isnan(v)) continue;
+                if (b < 0 || v < bv) {
+                    b = c;
+                    bv = v;
+                }
+            }
+            best[k] = b;
+        }
+        return;
+    }
+    int b = -1;
+    double bv = 0.0;
+    for (int c = 0; c < nc; ++c) {
+        double e = 0.0;
+        for (int k = 0; k < C; ++k) e += (double)err[(long)k * nc + c];
+        if (isnan(e)) continue;
+        if (b < 0 || e < bv) {
+            b = c;
+            bv = e;
+        }
+    }
+    for (int k = 0; k < C; ++k) best[k] = b;
+}

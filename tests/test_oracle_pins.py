@@ -309,3 +309,106 @@ def test_table1_overhead_closed_forms():
                       adds=3 * (d - 1) * Nb + 64)
     one = overhead.multipoint_cost(d, Nb, 1)
     assert one["memory_bits"] - naive["memory_bits"] == 32 and one["adds"] == naive["adds"]
+
+
+# ---- Eq. 12: output-error-driven clipping factor -------------------------------------------------
+
+def test_clip_hand_example(oracle):
+    """Candidates, errors and both argmins of a 2-channel example worked by hand (exact dyadics),
+    including a tie between two candidates (lowest index wins)."""
+    g = json.load(open(os.path.join(GOLDEN, "clip_hand_example.json")))
+    W = np.array(g["W"], np.float32)
+    for mode in (oracle.CLIP_PER_CHANNEL, oracle.CLIP_PER_LAYER):
+        clip = oracle.clip_candidates(W, g["n_cand"], mode)
+        assert np.array_equal(clip, np.tile(np.float32([0.25, 0.5, 0.75, 1.0]), (2, 1)))
+    clip = oracle.clip_candidates(W, g["n_cand"], oracle.CLIP_PER_CHANNEL)
+    for xs in ("X1", "X2"):
+        X = np.array(g[xs], np.float32)
+        e = oracle.clip_errors(X, 1, W, g["bits"], clip)
+        assert np.array_equal(e, np.array(g["err_" + xs]))
+        e32 = e.astype(np.float32)
+        assert list(oracle.clip_select(e32, oracle.CLIP_PER_CHANNEL)) == g["best_per_channel_" + xs]
+        assert list(oracle.clip_select(e32, oracle.CLIP_PER_LAYER)) == g["best_per_layer_" + xs]
+
+
+def test_clip_candidates_grid_and_modes(oracle):
+    rng = np.random.default_rng(31)
+    W = (rng.standard_normal((5, 40)) * rng.uniform(0.1, 3.0, (5, 1))).astype(np.float32)
+    per_ch = oracle.clip_candidates(W, 20, oracle.CLIP_PER_CHANNEL)
+    per_l = oracle.clip_candidates(W, 20, oracle.CLIP_PER_LAYER)
+    m = np.abs(W).max(axis=1)
+    assert np.array_equal(per_ch[:, -1], m)                  # f = 1: K = max|w| exactly
+    f = (np.arange(1, 21, dtype=np.float32) / np.float32(20)).astype(np.float32)
+    assert np.array_equal(per_ch, (f[None, :] * m[:, None]).astype(np.float32))
+    assert np.array_equal(per_l, np.tile((f * np.float32(m.max())).astype(np.float32), (5, 1)))
+
+
+def test_clip_scale_equivariance(oracle):
+    """W -> 2^k W scales every K by 2^k, every output error by 4^k, and keeps both argmins."""
+    rng = np.random.default_rng(32)
+    W = rng.standard_normal((6, 33)).astype(np.float32)
+    X = rng.standard_normal((17, 33)).astype(np.float32)
+    for mode in (oracle.CLIP_PER_CHANNEL, oracle.CLIP_PER_LAYER):
+        c0 = oracle.clip_candidates(W, 20, mode)
+        e0 = oracle.clip_errors(X, 1, W, 4, c0)
+        for k in (-3, 5):
+            W2 = np.ldexp(W, k).astype(np.float32)
+            c2 = oracle.clip_candidates(W2, 20, mode)
+            assert np.array_equal(c2, np.ldexp(c0, k).astype(np.float32))
+            e2 = oracle.clip_errors(X, 1, W2, 4, c2)
+            assert np.allclose(e2, e0 * 4.0 ** k, rtol=1e-12, atol=0)
+            assert np.array_equal(oracle.clip_select(e2.astype(np.float32), mode),
+                                  oracle.clip_select(e0.astype(np.float32), mode))
+
+
+def test_clip_top_candidate_is_greedy_top_scale(oracle):
+    """With X = sqrt(N) I, the error of K = max|w| is the weight error of the greedy search's largest
+    scale (same set, same codes): the two oracle functions agree."""
+    rng = np.random.default_rng(33)
+    d = 24
+    W = rng.standard_normal((4, d)).astype(np.float32)
+    X = (np.eye(d) * np.sqrt(d)).astype(np.float32)    # N = d rows: mean_t (x_t . r)^2 = ||r||^2
+    clip = oracle.clip_candidates(W, 20, oracle.CLIP_PER_CHANNEL)
+    e = oracle.clip_errors(X, 1, W, 3, clip)
+    for k in range(4):
+        ce, sg = oracle.candidate_errors(W[k], 3, 16)
+        assert sg[-1] == np.float32(clip[k, -1] / np.float32(3))   # the same scale m / Qmax
+        assert np.isclose(e[k, -1], ce[-1], rtol=1e-6, atol=0)
+
+
+def test_clip_select_brute_force(oracle):
+    """Both argmins against brute force on tie-heavy integer tables with NaNs."""
+    rng = np.random.default_rng(34)
+    for _ in range(200):
+        C, nc = int(rng.integers(1, 6)), int(rng.integers(1, 7))
+        t = rng.integers(0, 4, (C, nc)).astype(np.float32)
+        t[rng.random((C, nc)) < 0.15] = np.nan
+        got = oracle.clip_select(t, oracle.CLIP_PER_CHANNEL)
+        for k in range(C):
+            fin = [c for c in range(nc) if not np.isnan(t[k, c])]
+            want = min(fin, key=lambda c: (t[k, c], c)) if fin else -1
+            assert got[k] == want
+        got = oracle.clip_select(t, oracle.CLIP_PER_LAYER)
+        sums = [float(np.sum(t[:, c].astype(np.float64))) for c in range(nc)]
+        fin = [c for c in range(nc) if not np.isnan(sums[c])]
+        want = min(fin, key=lambda c: (sums[c], c)) if fin else -1
+        assert list(got) == [want] * C
+
+
+def test_clip_single_channel_layer_and_nonfinite(oracle):
+    rng = np.random.default_rng(35)
+    w = rng.standard_normal((1, 50)).astype(np.float32)
+    X = rng.standard_normal((9, 50)).astype(np.float32)
+    a = oracle.clip_candidates(w, 20, oracle.CLIP_PER_CHANNEL)
+    b = oracle.clip_candidates(w, 20, oracle.CLIP_PER_LAYER)
+    assert np.array_equal(a, b)
+    W = rng.standard_normal((3, 50)).astype(np.float32)
+    W[1, 7] = np.inf
+    c0 = oracle.clip_candidates(W, 20, oracle.CLIP_PER_CHANNEL)
+    assert np.all(np.isnan(c0[1])) and np.all(np.isfinite(c0[[0, 2]]))
+    e = oracle.clip_errors(X, 1, W, 4, c0).astype(np.float32)
+    assert list(oracle.clip_select(e, oracle.CLIP_PER_CHANNEL))[1] == -1
+    c1 = oracle.clip_candidates(W, 20, oracle.CLIP_PER_LAYER)
+    assert np.all(np.isnan(c1))
+    e1 = oracle.clip_errors(X, 1, W, 4, c1).astype(np.float32)
+    assert list(oracle.clip_select(e1, oracle.CLIP_PER_LAYER)) == [-1, -1, -1]
