@@ -57,6 +57,11 @@ typedef enum {
 #define MPQ_ALLOC_BUDGET 0
 #define MPQ_ALLOC_THRESHOLD 1
 
+/* Clipping-factor sets of mpq_clip_search: one K per channel, or one K for the whole layer. */
+#define MPQ_CLIP_PER_CHANNEL 0
+#define MPQ_CLIP_PER_LAYER 1
+#define MPQ_MAX_CLIP_CANDIDATES 32
+
 /*
  * mpq_quantize_layer -- greedy multipoint construction (Sec. 3.2, Eq. 6-9, Algorithm 1) for every
  * channel of one layer, run to k_max points.
@@ -137,6 +142,34 @@ mpq_status mpq_allocate_points(const float *err, int C, int k_max, int mode, dou
  */
 mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C,
                            int d, int k_max, float *W_hat, void *stream);
+
+/*
+ * mpq_clip_search -- output-error-driven clipping factor (Sec. 3.3, Eq. 12; candidate grid of
+ * App. B): the clipping factor K of the quantization set K x [-1 : eps_b : 1] (Eq. 1, B = 0) that
+ * minimises the output error of the quantized weights, chosen among n_cand candidates
+ *   K_c = f_c * m,  f_c = (c+1)/n_cand (fp32 division), c = 0..n_cand-1
+ * (n_cand = 20 is the experiments' grid [0.05 : 0.05 : 1] x max|w|), with m = max_j |w_kj| of
+ * channel k (MPQ_CLIP_PER_CHANNEL) or of the whole layer (MPQ_CLIP_PER_LAYER, one K for every
+ * channel).  The quantized channel is s q with s = K / Qmax (fp32 division) and
+ * q_j = clamp(rint(w_j / s), -Qmax, Qmax) as in Eq. 8; its output error is
+ *   err[k][c] = (1/N) sum_t (x_t . r_{k,c})^2,  r_{k,c} = fmaf(-s, q, w_k)   (Eq. 11's form).
+ * best[k] = the lowest c with the smallest err[k][c] (per channel), or the lowest c with the
+ * smallest sum_k err[k][c] summed in double over the channels in order (per layer, the same c for
+ * every channel).  A non-finite weight makes that channel's K (per layer: every K) NaN, its errors
+ * NaN, and NaN never wins; best is -1 where no candidate is finite.
+ *
+ *   X, N, groups  calibration inputs as for mpq_output_error.
+ *   W, C, d       [C][d] fp32 weights; 1 <= d <= MPQ_MAX_DIM.
+ *   bits          b in [MPQ_MIN_BITS, MPQ_MAX_BITS].
+ *   n_cand        1..MPQ_MAX_CLIP_CANDIDATES.
+ *   mode          MPQ_CLIP_PER_CHANNEL or MPQ_CLIP_PER_LAYER.
+ *   clip          out [C][n_cand] fp32: K_c of each channel (also used as working storage).
+ *   err           out [C][n_cand] fp32.
+ *   best          out [C] int32; the chosen factor of channel k is clip[k][best[k]].
+ */
+mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, int C, int d,
+                           int bits, int n_cand, int mode, float *clip, float *err, int *best,
+                           void *stream);
 
 /* Name of a status code (static string). */
 const char *mpq_status_string(mpq_status s);

@@ -6,6 +6,7 @@ on first use.  There is no CPU fallback: calling an entry point without the comp
 raises.
 """
 from . import overhead, workloads  # noqa: F401
-from .binding import (MPQ_ALLOC_BUDGET, MPQ_ALLOC_THRESHOLD, MPQError,  # noqa: F401
-                      mpq_allocate_points, mpq_output_error, mpq_quantize_layer, mpq_reconstruct,
-                      mpq_status_string, mpq_version)
+from .binding import (MPQ_ALLOC_BUDGET, MPQ_ALLOC_THRESHOLD, MPQ_CLIP_PER_CHANNEL,  # noqa: F401
+                      MPQ_CLIP_PER_LAYER, MPQError, mpq_allocate_points, mpq_clip_search,
+                      mpq_output_error, mpq_quantize_layer, mpq_reconstruct, mpq_status_string,
+                      mpq_version)

@@ -16,6 +16,8 @@ from . import _build
 
 MPQ_ALLOC_BUDGET = 0
 MPQ_ALLOC_THRESHOLD = 1
+MPQ_CLIP_PER_CHANNEL = 0
+MPQ_CLIP_PER_LAYER = 1
 
 MPQ_STATUS = {0: "MPQ_OK", 1: "MPQ_ERR_INVALID_ARG", 2: "MPQ_ERR_NONFINITE",
               3: "MPQ_ERR_UNSUPPORTED", 4: "MPQ_ERR_CUDA", 5: "MPQ_ERR_TIMEOUT",
@@ -28,6 +30,7 @@ SIGNATURES = {
     "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
     "mpq_reconstruct": ([_P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "mpq_clip_search": ([_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P], _I),
     "mpq_status_string": ([_I], ctypes.c_char_p),
     "mpq_last_error": ([], ctypes.c_char_p),
     "mpq_version": ([], _I),
@@ -150,6 +153,35 @@ def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None,
                                  k_max, _ptr(err), _stream(stream))
     _check(st, "mpq_output_error")
     return err
+
+
+def mpq_clip_search(X, W, bits: int, n_cand: int = 20, mode: int = None, groups: int = 1,
+                    clip=None, err=None, best=None, stream=None):
+    """Output-error-driven clipping factor (Eq. 12) among n_cand candidates (c+1)/n_cand x max|w|:
+    returns (clip [C][n_cand] fp32, err [C][n_cand] fp32, best [C] int32)."""
+    mode = MPQ_CLIP_PER_CHANNEL if mode is None else mode
+    _dev(W, "W", torch.float32)
+    C, d = W.shape
+    _dev(X, "X", torch.float32)
+    if groups == 1:
+        if X.dim() != 2 or X.shape[1] != d:
+            raise ValueError("X must be [N][d] for groups = 1")
+        N = X.shape[0]
+    else:
+        if X.dim() != 3 or X.shape[0] != C or X.shape[2] != d:
+            raise ValueError("X must be [C][N][d] for groups = C")
+        N = X.shape[1]
+    mk = lambda dt: torch.empty((C, n_cand), dtype=dt, device=W.device)
+    clip = clip if clip is not None else mk(torch.float32)
+    err = err if err is not None else mk(torch.float32)
+    best = best if best is not None else torch.empty((C,), dtype=torch.int32, device=W.device)
+    _dev(clip, "clip", torch.float32, (C, n_cand))
+    _dev(err, "err", torch.float32, (C, n_cand))
+    _dev(best, "best", torch.int32, (C,))
+    st = load().mpq_clip_search(_ptr(X), N, groups, _ptr(W), C, d, bits, n_cand, mode, _ptr(clip),
+                                _ptr(err), _ptr(best), _stream(stream))
+    _check(st, "mpq_clip_search")
+    return clip, err, best
 
 
 def mpq_allocate_points(err, k_max: int, mode: int = MPQ_ALLOC_BUDGET,

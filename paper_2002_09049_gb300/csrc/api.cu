@@ -133,6 +133,34 @@ extern "C" mpq_status mpq_output_error(const float *X, int N, int groups, const 
                                (cudaStream_t)stream);
 }
 
+extern "C" mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, int C,
+                                      int d, int bits, int n_cand, int mode, float *clip,
+                                      float *err, int *best, void *stream)
+{
+    g_msg[0] = 0;
+    mpq_status st = check_common(C, d, 1);
+    if (st != MPQ_OK) return st;
+    REQUIRE(d <= MPQ_MAX_DIM, MPQ_ERR_UNSUPPORTED, "d = %d exceeds MPQ_MAX_DIM = %d", d,
+            MPQ_MAX_DIM);
+    REQUIRE(bits >= MPQ_MIN_BITS && bits <= MPQ_MAX_BITS,
+            (bits > MPQ_MAX_BITS ? MPQ_ERR_UNSUPPORTED : MPQ_ERR_INVALID_ARG),
+            "bits = %d outside [%d, %d]", bits, MPQ_MIN_BITS, MPQ_MAX_BITS);
+    REQUIRE(n_cand >= 1, MPQ_ERR_INVALID_ARG, "n_cand = %d must be >= 1", n_cand);
+    REQUIRE(n_cand <= MPQ_MAX_CLIP_CANDIDATES, MPQ_ERR_UNSUPPORTED,
+            "n_cand = %d exceeds MPQ_MAX_CLIP_CANDIDATES = %d", n_cand, MPQ_MAX_CLIP_CANDIDATES);
+    REQUIRE(mode == MPQ_CLIP_PER_CHANNEL || mode == MPQ_CLIP_PER_LAYER, MPQ_ERR_INVALID_ARG,
+            "mode = %d is not MPQ_CLIP_PER_CHANNEL or MPQ_CLIP_PER_LAYER", mode);
+    REQUIRE(N >= 1, MPQ_ERR_INVALID_ARG, "N = %d must be >= 1", N);
+    REQUIRE(groups == 1 || groups == C, MPQ_ERR_INVALID_ARG, "groups = %d must be 1 or C = %d",
+            groups, C);
+    REQUIRE((long long)N * d <= (1LL << 40), MPQ_ERR_UNSUPPORTED, "N*d too large");
+    if (C == 0) return MPQ_OK;
+    REQUIRE(X && W && clip && err && best, MPQ_ERR_INVALID_ARG,
+            "X, W, clip, err and best must be non-NULL");
+    return launch_clip(X, N, groups, W, C, d, (1 << (bits - 1)) - 1, n_cand, mode, clip, err, best,
+                       (cudaStream_t)stream);
+}
+
 extern "C" mpq_status mpq_allocate_points(const float *err, int C, int k_max, int mode,
                                           double budget_or_eps, int *npoints, int *points_used,
                                           void *stream)

@@ -43,6 +43,12 @@ mpq_status launch_output_error_pair(const float *X, int N, const float *W, const
                                     const float *scales, int C, int d, int k_max, float *err,
                                     cudaStream_t stream);
 
+mpq_status launch_clip_pair(const float *X, int N, const float *W, const float *clip, int C, int d,
+                            int qmax, int n_cand, float *err, cudaStream_t stream);
+mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C, int d, int qmax,
+                       int n_cand, int mode, float *clip, float *err, int *best,
+                       cudaStream_t stream);
+
 mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
                                   int *npoints, int *points_used, cudaStream_t stream);
 

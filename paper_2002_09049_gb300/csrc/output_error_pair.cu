@@ -35,6 +35,7 @@
 #include <atomic>
 
 #include "mpq_internal.cuh"
+#include "rounding.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
 
@@ -79,15 +80,19 @@ struct PairCtrl {
     uint32_t tmem_base;
     int abort;
     double part[P_VEC];
+    float clip_s[P_VEC];          // clipping search: scale K / Qmax and fl(1 / scale) per row
+    float clip_inv[P_VEC];
 };
 constexpr int P_CTRL_BYTES = (sizeof(PairCtrl) + 1023) / 1024 * 1024;
 constexpr int P_BASE_SMEM = 1024 /* alignment slack */ + P_CTRL_BYTES + P_STAGES * P_STAGE_BYTES;
 
 // Per-KP1 geometry and the raw slot layout, in the order the tile copies write it:
-// X chunk [128 rows][32] fp32, W chunk [CH][32] fp32, codes [K][CH][32] int8.
-template <int KP1>
+// X chunk [128 rows][32] fp32, W chunk [CH][32] fp32, codes [K][CH][32] int8.  KP1 is the number of
+// residual vectors per channel: k_max + 1 greedy residuals, or (CLIP) one per candidate clipping
+// factor, which need no codes.
+template <int KP1, bool CLIP = false>
 struct PGeo {
-    static constexpr int K = KP1 - 1;
+    static constexpr int K = CLIP ? 0 : KP1 - 1;
     static constexpr int KQ = K > 0 ? K : 1;
     static constexpr int CH = P_VEC / KP1;
     static constexpr int ITEMS2 = (CH * (P_KC / 2) + P_PROD_THREADS - 1) / P_PROD_THREADS;
@@ -103,13 +108,15 @@ struct PGeo {
 };
 
 // Raw slot -> operand stage `sb`: X rows -> B tiles; for every (channel, element pair) item the
-// residuals r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7) -> A tiles.
-template <int KP1>
+// residuals -> A tiles: r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7), or (CLIP) r_c = w - s_c [w / s_c]_Q
+// for every candidate clipping factor (Eq. 12), with the scales and reciprocals of `ctl`.
+template <int KP1, bool CLIP>
 __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt, int nch,
-                                             const float (&sc)[PGeo<KP1>::ITEMS2][PGeo<KP1>::KQ])
+                                             const float (&sc)[PGeo<KP1, CLIP>::ITEMS2][PGeo<KP1, CLIP>::KQ],
+                                             const PairCtrl &ctl, float qmaxf)
 {
-    using G = PGeo<KP1>;
-    constexpr int K = KP1 - 1;
+    using G = PGeo<KP1, CLIP>;
+    constexpr int K = G::K;
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
         const int q = pt + i * P_PROD_THREADS;
@@ -123,7 +130,25 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
 #pragma unroll
     for (int i = 0; i < G::ITEMS2; ++i) {
         const int p = pt + i * P_PROD_THREADS;
-        if (p < nch * (P_KC / 2)) {
+        if (CLIP && p < nch * (P_KC / 2)) {
+            const int ch = p / (P_KC / 2), e2 = p % (P_KC / 2);
+            const float2 w = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
+            const uint32_t cofs = (uint32_t)(e2 & 1) * 8u;
+#pragma unroll 4
+            for (int c = 0; c < KP1; ++c) {
+                const float s = ctl.clip_s[ch * KP1 + c], inv = ctl.clip_inv[ch * KP1 + c];
+                // exact code of Eq. 8 (0 when the scale is 0 or NaN: the residual is then w or NaN)
+                const float qx = s > 0.0f ? copysignf((float)code_fast(fabsf(w.x), s, inv, qmaxf), w.x) : 0.0f;
+                const float qy = s > 0.0f ? copysignf((float)code_fast(fabsf(w.y), s, inv, qmaxf), w.y) : 0.0f;
+                float2 r, hi, lo;
+                r.x = __fmaf_rn(-s, qx, w.x);
+                r.y = __fmaf_rn(-s, qy, w.y);
+                split2(r, hi, lo);
+                const uint32_t off = sw128_offset(ch * KP1 + c, e2 >> 1) + cofs;
+                st_shared_v2(sb + P_OFF_A_HI + off, hi);
+                st_shared_v2(sb + P_OFF_A_LO + off, lo);
+            }
+        } else if (!CLIP && p < nch * (P_KC / 2)) {
             const int ch = p / (P_KC / 2), e2 = p % (P_KC / 2);
             float2 r = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
             uint32_t qb[G::KQ];
@@ -149,15 +174,17 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
     }
 }
 
-template <int KP1>
+// scales: [C][k_max] point scales, or (CLIP) [C][KP1] candidate clipping factors K; qmax: the
+// code range for CLIP.
+template <int KP1, bool CLIP>
 __global__ void __launch_bounds__(P_THREADS, 1)
-output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d,
+output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, int qmax,
                          float *__restrict__ err, int split,
                          const __grid_constant__ CUtensorMap tmX,
                          const __grid_constant__ CUtensorMap tmW,
                          const __grid_constant__ CUtensorMap tmQ)
 {
-    using G = PGeo<KP1>;
+    using G = PGeo<KP1, CLIP>;
     constexpr int R = G::RAW_STAGES;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
@@ -197,6 +224,14 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d,
         ctl.abort = 0;
         fence_barrier_init();
     }
+    const float qmaxf = (float)qmax;
+    if (CLIP) {
+        for (int i = threadIdx.x; i < nvec; i += P_THREADS) {
+            const float s = __fdiv_rn(__ldg(scales + (size_t)k0 * KP1 + i), qmaxf);
+            ctl.clip_s[i] = s;
+            ctl.clip_inv[i] = s > 0.0f ? __frcp_rn(s) : 0.0f;
+        }
+    }
     if (warp == P_MMA_WARP) {
         tmem_alloc_pair(&ctl.tmem_base, P_TMEM_COLS);
         tc_fence_before();
@@ -216,7 +251,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d,
             const int k = k0 + p / (P_KC / 2);
 #pragma unroll
             for (int n = 0; n < G::KQ; ++n)
-                sc[i][n] = (n < KP1 - 1 && p < nch * (P_KC / 2))
+                sc[i][n] = (!CLIP && n < KP1 - 1 && p < nch * (P_KC / 2))
                                ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
         }
         for (int it = 0; it < total; ++it) {
@@ -226,8 +261,8 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d,
                             mbar_wait_cluster(&ctl.empty[s], ph ^ 1u, P_WAIT);
             if (!ok) *abort_flag = 1;
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-            pair_consume<KP1>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + s * P_STAGE_BYTES, pt,
-                              nch, sc);
+            pair_consume<KP1, CLIP>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + s * P_STAGE_BYTES,
+                                    pt, nch, sc, ctl, qmaxf);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
@@ -341,7 +376,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d,
                 mbar_arrive_expect_tx(&ctl.raw_full[slot], G::RAW_TX);
                 tma_load_2d(dst, &tmX, x, row0, &ctl.raw_full[slot]);
                 tma_load_2d(dst + G::RAW_W, &tmW, x, k0, &ctl.raw_full[slot]);
-                tma_load_3d(dst + G::RAW_Q, &tmQ, x, k0, 0, &ctl.raw_full[slot]);
+                if (!CLIP) tma_load_3d(dst + G::RAW_Q, &tmQ, x, k0, 0, &ctl.raw_full[slot]);
                 issued = f + 1;
             }
             // no copy may land after the CTA is gone: wait for the last copies of every slot
@@ -395,11 +430,11 @@ bool pair_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *ba
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int KP1>
+template <int KP1, bool CLIP>
 mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *codes,
-                       const float *scales, int C, int d, float *err, cudaStream_t stream)
+                       const float *scales, int C, int d, int qmax, float *err, cudaStream_t stream)
 {
-    using G = PGeo<KP1>;
+    using G = PGeo<KP1, CLIP>;
     const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
     const int n_rt = (N + P_N - 1) / P_N;
 
@@ -416,7 +451,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     const cuuint32_t bq[3] = {P_KC, (cuuint32_t)G::CH, (cuuint32_t)G::K};
     if (!pair_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, X, dx, sx, bx) ||
         !pair_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw) ||
-        !pair_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq)) {
+        (!CLIP && !pair_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq))) {
         set_error("output error: tensor map encoding failed");
         return MPQ_ERR_CUDA;
     }
@@ -424,7 +459,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         set_error("pair output error needs %d bytes of shared memory", G::SMEM);
         return MPQ_ERR_UNSUPPORTED;
     }
-    cudaError_t e = cudaFuncSetAttribute(output_error_pair_kernel<KP1>,
+    cudaError_t e = cudaFuncSetAttribute(output_error_pair_kernel<KP1, CLIP>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
 
@@ -451,7 +486,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         cfg.gridDim = dim3((unsigned)(n_pairs * 2 * sp), 1, 1);
         int active = resident[i].load(std::memory_order_relaxed);
         if (active == 0) {
-            if (cudaOccupancyMaxActiveClusters(&active, output_error_pair_kernel<KP1>, &cfg) !=
+            if (cudaOccupancyMaxActiveClusters(&active, output_error_pair_kernel<KP1, CLIP>, &cfg) !=
                 cudaSuccess)
                 active = -1;
             (void)cudaGetLastError();
@@ -467,8 +502,8 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     }
     attr[0].val.clusterDim.x = (unsigned)(2 * split);
     cfg.gridDim = dim3((unsigned)(n_pairs * 2 * split), 1, 1);
-    e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1>, scales, C, N, d, err, split, tmX,
-                           tmW, tmQ);
+    e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax, err,
+                           split, tmX, tmW, tmQ);
     return cuda_status(e, "pair output-error kernel launch");
 }
 
@@ -486,13 +521,30 @@ mpq_status launch_output_error_pair(const float *X, int N, const float *W, const
 {
     switch (k_max + 1) {
 #define MPQ_CASE(n) \
-    case n: return launch_pair<n>(X, N, W, codes, scales, C, d, err, stream);
+    case n: return launch_pair<n, false>(X, N, W, codes, scales, C, d, 0, err, stream);
         MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7) MPQ_CASE(8)
         MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14) MPQ_CASE(15)
         MPQ_CASE(16) MPQ_CASE(17)
 #undef MPQ_CASE
     }
     set_error("k_max = %d unsupported", k_max);
+    return MPQ_ERR_UNSUPPORTED;
+}
+
+mpq_status launch_clip_pair(const float *X, int N, const float *W, const float *clip, int C, int d,
+                            int qmax, int n_cand, float *err, cudaStream_t stream)
+{
+    switch (n_cand) {
+#define MPQ_CASE(n) \
+    case n: return launch_pair<n, true>(X, N, W, nullptr, clip, C, d, qmax, err, stream);
+        MPQ_CASE(1) MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7)
+        MPQ_CASE(8) MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14)
+        MPQ_CASE(15) MPQ_CASE(16) MPQ_CASE(17) MPQ_CASE(18) MPQ_CASE(19) MPQ_CASE(20) MPQ_CASE(21)
+        MPQ_CASE(22) MPQ_CASE(23) MPQ_CASE(24) MPQ_CASE(25) MPQ_CASE(26) MPQ_CASE(27) MPQ_CASE(28)
+        MPQ_CASE(29) MPQ_CASE(30) MPQ_CASE(31) MPQ_CASE(32)
+#undef MPQ_CASE
+    }
+    set_error("n_cand = %d unsupported", n_cand);
     return MPQ_ERR_UNSUPPORTED;
 }
 

@@ -34,6 +34,7 @@
 #include <math.h>
 
 #include "mpq_internal.cuh"
+#include "rounding.cuh"
 
 namespace mpq {
 namespace {
@@ -290,13 +291,6 @@ __device__ __forceinline__ void group_suffix_scan(int t0, int t1, Load load, Sto
     }
 }
 
-// Code magnitude of |r| at scale s > 0 (Eq. 8): nearest integer (ties to even) of the correctly
-// rounded fp32 quotient, clipped to Qmax.
-__device__ __forceinline__ int code_mag(float a, float s, float qmaxf)
-{
-    return (int)fminf(rintf(__fdiv_rn(a, s)), qmaxf);
-}
-
 // |r| as a 64-bit fixed-point integer R = |r| * 2^S, from the fp32 bits.  Exact whenever
 // |r| * 2^S is an integer, i.e. for every element large enough to take a nonzero code; smaller
 // elements are truncated (their P contribution is zero anyway).
@@ -316,11 +310,6 @@ __device__ __forceinline__ double pow2d(int k)
     return __longlong_as_double((long long)(1023 + k) << 52);
 }
 
-// Bound on |a * fl(1/s) - fl(a/s)| relative to the quotient, with margin: both roundings are
-// 2^-24 each, so a fast quotient further than this from a rounding boundary decides exactly as
-// the correctly rounded division would.
-#define MPQ_FAST_REL 9.5367431640625e-07f /* 2^-20 */
-
 // rint(fl(a/s)) >= L, decided from q' = a * (1/s) unless q' is too close to L - 1/2.
 __device__ __forceinline__ bool level_held(float a, float s, float inv_s, int L)
 {
@@ -330,18 +319,6 @@ __device__ __forceinline__ bool level_held(float a, float s, float inv_s, int L)
     if (qf > h + tol) return true;
     if (qf < h - tol) return false;
     return rintf(__fdiv_rn(a, s)) >= (float)L;
-}
-
-// min(Qmax, rint(fl(a/s))), decided from q' = a * (1/s) unless q' is too close to a half-integer.
-__device__ __forceinline__ int code_fast(float a, float s, float inv_s, float qmaxf)
-{
-    const float qf = __fmul_rn(a, inv_s);
-    const float tol = MPQ_FAST_REL * (qf + 1.0f);
-    if (qf > qmaxf + 0.5f + tol) return (int)qmaxf;
-    const float fl = floorf(qf);
-    const float fr = qf - fl;   // exact
-    if (fabsf(fr - 0.5f) > tol) return (int)fminf(fr > 0.5f ? fl + 1.0f : fl, qmaxf);
-    return (int)fminf(rintf(__fdiv_rn(a, s)), qmaxf);
 }
 
 // Decision value D(s) = s (s N - 2 P) with P = Pfix * 2^-S, in double.

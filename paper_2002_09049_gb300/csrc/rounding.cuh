@@ -1,0 +1,33 @@
+// Exact codes of Eq. 8 for a symmetric b-bit set: c = min(Qmax, rint(fl(a / s))) for a = |r| >= 0 and
+// scale s > 0, with fl the correctly rounded fp32 division and rint ties-to-even -- and a fast path
+// that reaches the same integer from a multiply by a reciprocal whenever the quotient is not too
+// close to a rounding boundary.  Shared by the greedy search and the clipping-factor search.
+#pragma once
+
+namespace mpq {
+
+// Code magnitude of |r| at scale s > 0 (Eq. 8): nearest integer (ties to even) of the correctly
+// rounded fp32 quotient, clipped to Qmax.
+__device__ __forceinline__ int code_mag(float a, float s, float qmaxf)
+{
+    return (int)fminf(rintf(__fdiv_rn(a, s)), qmaxf);
+}
+
+// Bound on |a * fl(1/s) - fl(a/s)| relative to the quotient, with margin: both roundings are
+// 2^-24 each, so a fast quotient further than this from a rounding boundary decides exactly as
+// the correctly rounded division would.
+#define MPQ_FAST_REL 9.5367431640625e-07f /* 2^-20 */
+
+// min(Qmax, rint(fl(a/s))), decided from q' = a * (1/s) unless q' is too close to a half-integer.
+__device__ __forceinline__ int code_fast(float a, float s, float inv_s, float qmaxf)
+{
+    const float qf = __fmul_rn(a, inv_s);
+    const float tol = MPQ_FAST_REL * (qf + 1.0f);
+    if (qf > qmaxf + 0.5f + tol) return (int)qmaxf;
+    const float fl = floorf(qf);
+    const float fr = qf - fl;   // exact
+    if (fabsf(fr - 0.5f) > tol) return (int)fminf(fr > 0.5f ? fl + 1.0f : fl, qmaxf);
+    return (int)fminf(rintf(__fdiv_rn(a, s)), qmaxf);
+}
+
+}  // namespace mpq

@@ -29,7 +29,8 @@ def lib():
 
 def test_header_declares_the_boundary():
     names = declared_functions()
-    for n in ("mpq_quantize_layer", "mpq_output_error", "mpq_allocate_points", "mpq_reconstruct"):
+    for n in ("mpq_quantize_layer", "mpq_output_error", "mpq_allocate_points", "mpq_reconstruct",
+              "mpq_clip_search"):
         assert n in names
 
 
@@ -102,3 +103,22 @@ def test_allocate_requires_outputs(lib):
 def test_reconstruct_validation(lib):
     assert lib.mpq_reconstruct(FAKE, FAKE, None, 4, 16, 2, FAKE, None) == 1
     assert lib.mpq_reconstruct(FAKE, FAKE, FAKE, 4, 16, 0, FAKE, None) == 1
+
+
+@pytest.mark.parametrize("kwargs,status", [
+    (dict(N=0), 1), (dict(groups=3), 1), (dict(bits=1), 1), (dict(bits=9), 3), (dict(n_cand=0), 1),
+    (dict(n_cand=33), 3), (dict(mode=2), 1), (dict(d=0), 1), (dict(d=8193), 3), (dict(X=None), 1),
+    (dict(clip=None), 1), (dict(err=None), 1), (dict(best=None), 1),
+])
+def test_clip_search_validation(lib, kwargs, status):
+    a = dict(X=FAKE, N=8, groups=1, W=FAKE, C=4, d=16, bits=4, n_cand=20, mode=0, clip=FAKE,
+             err=FAKE, best=FAKE)
+    a.update(kwargs)
+    st = lib.mpq_clip_search(a["X"], a["N"], a["groups"], a["W"], a["C"], a["d"], a["bits"],
+                             a["n_cand"], a["mode"], a["clip"], a["err"], a["best"], None)
+    assert st == status
+    assert lib.mpq_last_error() != b""
+
+
+def test_clip_search_empty_layer(lib):
+    assert lib.mpq_clip_search(None, 8, 1, None, 0, 16, 4, 20, 1, None, None, None, None) == 0
