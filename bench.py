@@ -60,6 +60,11 @@ def parse():
                     help="comma-separated layer indices to run (profiling a subset); default all")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--op", default="quantize", choices=["quantize", "clip"],
+                    help="quantize: the multipoint path (Algorithm 1, Eq. 11, Algorithm 2, Eq. 4); "
+                         "clip: the output-error-driven clipping factor search (Eq. 12)")
+    ap.add_argument("--clip-candidates", type=int, default=20,
+                    help="clipping factor candidates (c+1)/n x max|w| for --op clip")
     return ap.parse_args()
 
 
@@ -511,11 +516,239 @@ def run_reference(args, world, rank):
                     "d2h_bytes_per_step": 0}}
 
 
+CLIP_METRIC = "weight-elements x clip-candidates / s"
+CLIP_UNIT = "elem*cand/s"
+
+
+def clip_oracle_step(wl, stride, threads, inputs, n_cand):
+    """The oracle's Eq. 12 search (per-channel candidates, errors, argmin) on the sampled channels."""
+    import oracle
+    units = 0
+    for li, layer in enumerate(wl.layers):
+        W, X = inputs[li]
+        groups = W.shape[0] if layer.groups > 1 else 1
+        clip = oracle.clip_candidates(W, n_cand, oracle.CLIP_PER_CHANNEL)
+        err = oracle.clip_errors(X, groups, W, wl.bits[0], clip, threads=threads)
+        oracle.clip_select(err.astype(np.float32), oracle.CLIP_PER_CHANNEL)
+        units += W.shape[0] * W.shape[1] * n_cand
+    return units
+
+
+def clip_oracle_stride(wl, target_s, n_cand):
+    est = sum(l.C * l.d * wl.n_calib * n_cand * 1.2e-9 for l in wl.layers)
+    return max(1, int(np.ceil(est / host_cores() / target_s)))
+
+
+def run_clip(args, world, rank, local):
+    """Eq. 12 over every layer of the workload: mpq_clip_search (per-channel candidates, output
+    errors on the tensor cores, argmin) with layers on a pool of streams."""
+    import torch
+    from paper_2002_09049_gb300 import _build, binding
+    from paper_2002_09049_gb300 import dist as dist_helpers
+    from paper_2002_09049_gb300 import workloads as wlm
+
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0 or world == 1:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    binding.load()
+    wl = wlm.WORKLOADS[args.config]
+    nc = args.clip_candidates
+    bits = wl.bits[0]
+    keep = None if args.layers is None else {int(x) for x in args.layers.split(",")}
+    idx = [li for li in range(len(wl.layers)) if keep is None or li in keep]
+    layers = [wl.layers[li] for li in idx]
+    Ws, Xs, Whs, Xhs, outs = [], [], [], [], []
+    for li, layer in zip(idx, layers):
+        W, X = layer_inputs(wl, li)
+        Whs.append(torch.from_numpy(W).pin_memory())
+        Xhs.append(torch.from_numpy(X).pin_memory())
+        Ws.append(Whs[-1].to(dev))
+        Xs.append(Xhs[-1].to(dev))
+        mk = lambda dt, shape: torch.empty(shape, dtype=dt, device=dev)
+        outs.append((mk(torch.float32, (layer.C, nc)), mk(torch.float32, (layer.C, nc)),
+                     mk(torch.int32, (layer.C,))))
+    order = sorted(range(len(layers)), key=lambda i: -layers[i].C * layers[i].d)
+    streams = [torch.cuda.Stream(dev) for _ in range(max(1, args.streams))]
+    main = torch.cuda.current_stream()
+    units_per_step = sum(l.C * l.d * nc for l in layers)
+    flops_per_step = sum(2.0 * wl.n_calib * l.d * l.C * nc for l in layers)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+
+    def call(i, st):
+        c, e, b = outs[i]
+        binding.mpq_clip_search(Xs[i], Ws[i], bits, nc, binding.MPQ_CLIP_PER_CHANNEL,
+                                groups=layers[i].groups, clip=c, err=e, best=b, stream=st)
+
+    def step():
+        ev = torch.cuda.Event()
+        ev.record(main)
+        for st in streams:
+            st.wait_event(ev)
+        for n, i in enumerate(order):
+            call(i, streams[n % len(streams)])
+        for st in streams:
+            e = torch.cuda.Event()
+            e.record(st)
+            main.wait_event(e)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    peaks, peak_src = measured_peaks()
+    step_ms = []
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            a = torch.cuda.Event(enable_timing=True)
+            z = torch.cuda.Event(enable_timing=True)
+            a.record(main)
+            step()
+            z.record(main)
+            torch.cuda.synchronize()
+            step_ms.append(a.elapsed_time(z))
+    # per-call durations on one stream for the roofline
+    one_ms = []
+    for _ in range(args.steps):
+        flush.fill_(1.0)
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(order) + 1)]
+        evs[0].record(main)
+        for n, i in enumerate(order):
+            call(i, main)
+            evs[n + 1].record(main)
+        torch.cuda.synchronize()
+        one_ms.append(evs[0].elapsed_time(evs[-1]))
+    if world > 1:
+        torch.distributed.barrier()
+    ms = dist_helpers.max_over_ranks(float(np.mean(step_ms)), device=dev)
+    value = dist_helpers.aggregate_throughput(units_per_step, ms, world)
+    t1 = float(np.mean(one_ms)) / 1e3
+    peak = peaks["bf16_tflops"] * TF32_PER_BF16
+    ach = flops_per_step / t1 / 1e12
+    roofline = {"kernel": "output_error_pair_kernel in clip mode (Eq. 12 residuals generated on chip, "
+                          "tcgen05 cta_group::2 kind::tf32, 3-pass split) + candidate and argmin kernels",
+                "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                "frac": ach / peak, "traffic": None,
+                "peak_source": f"{peak_src} bf16 dense burst x nominal tf32/bf16 ratio "
+                               f"{TF32_PER_BF16:.3f}",
+                "timing": "whole calls (candidates, errors, argmin) on one stream, CUDA events; "
+                          "achieved = algorithmic flops 2*N*d*C*n_cand / that time",
+                "single_stream_ms_per_step": t1 * 1e3}
+    out = {"metric": CLIP_METRIC, "value": value, "unit": CLIP_UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+           "data": "synthetic",
+           "config": {"workload": f"{args.config}: {wl.title}", "op": "clip (Eq. 12)",
+                      "layers": len(layers), "clip_candidates": nc, "sets": "per channel",
+                      "bits": bits, "calib_rows": wl.n_calib, "units_per_step": units_per_step,
+                      "l2": "flushed between steps (512 MB write)", "streams": args.streams,
+                      "parallelism": f"replicas x{world}"},
+           "roofline": roofline, "gpu_launches": 3 * len(layers) * args.steps,
+           "clocks": clk.summary()}
+    if not args.no_e2e:
+        def e2e_step():
+            ev = torch.cuda.Event()
+            ev.record(main)
+            for st in streams:
+                st.wait_event(ev)
+            host = []
+            for n, i in enumerate(order):
+                st = streams[n % len(streams)]
+                with torch.cuda.stream(st):
+                    Ws[i].copy_(Whs[i], non_blocking=True)
+                    Xs[i].copy_(Xhs[i], non_blocking=True)
+                    call(i, st)
+                    c, e, b = outs[i]
+                    host.append((c.to("cpu", non_blocking=True), e.to("cpu", non_blocking=True),
+                                 b.to("cpu", non_blocking=True)))
+            for st in streams:
+                e = torch.cuda.Event()
+                e.record(st)
+                main.wait_event(e)
+            return host
+        for _ in range(max(1, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize()
+        tms = []
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            e2e_step()
+            torch.cuda.synchronize()
+            tms.append((time.perf_counter() - t0) * 1e3)
+        e_ms = float(np.mean(tms))
+        out["e2e"] = {"value": units_per_step / (e_ms / 1e3), "unit": CLIP_UNIT, "ms_per_step": e_ms,
+                      "h2d_bytes_per_step": sum(w.numel() * 4 + x.numel() * 4
+                                                for w, x in zip(Whs, Xhs)),
+                      "d2h_bytes_per_step": sum(l.C * nc * 8 + l.C * 4 for l in layers)}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        stride = clip_oracle_stride(wl, args.cpu_seconds, nc)
+        inputs = sample_inputs(wl, stride)
+        t0 = time.perf_counter()
+        units = clip_oracle_step(wl, stride, host_cores(), inputs, nc)
+        dt = time.perf_counter() - t0
+        out["cpu_baseline"] = {"value": units / dt, "unit": CLIP_UNIT, "cores": host_cores(),
+                               "kind": "oracle", "seconds": dt,
+                               "sample": f"every {stride}th channel of every layer ({units:.3e} "
+                                         "units), oracle threads over channels"}
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    return out if rank == 0 else None
+
+
+def run_clip_reference(args, world, rank):
+    """The oracle's Eq. 12 search as the reference arm of --op clip, on the host cores."""
+    if rank != 0:
+        return None
+    import oracle
+    from paper_2002_09049_gb300 import workloads as wlm
+    oracle.build()
+    wl = wlm.WORKLOADS[args.config]
+    nc = args.clip_candidates
+    per_step = max(2.0, 150.0 / max(1, args.steps + args.warmup))
+    stride = clip_oracle_stride(wl, per_step, nc)
+    inputs = sample_inputs(wl, stride)
+    for _ in range(args.warmup):
+        clip_oracle_step(wl, stride, host_cores(), inputs, nc)
+    times, units = [], 0
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        units = clip_oracle_step(wl, stride, host_cores(), inputs, nc)
+        times.append(time.perf_counter() - t0)
+    s = float(np.mean(times))
+    value = units / s
+    return {"impl": "reference", "metric": CLIP_METRIC, "value": value, "unit": CLIP_UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": f"{args.config}: {wl.title}", "op": "clip (Eq. 12)",
+                       "clip_candidates": nc, "sets": "per channel"},
+            "cpu_baseline": {"value": value, "unit": CLIP_UNIT, "cores": host_cores(),
+                             "kind": "oracle",
+                             "sample": f"every {stride}th channel of every layer per step"},
+            "e2e": {"value": value, "unit": CLIP_UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
 def main():
     args = parse()
     world, rank, local = dist_setup(args)
     if args.impl == "reference":
-        out = run_reference(args, world, rank)
+        out = (run_clip_reference if args.op == "clip" else run_reference)(args, world, rank)
+    elif args.op == "clip":
+        out = run_clip(args, world, rank, local)
     else:
         out = run_ours(args, world, rank, local)
     if out is not None:

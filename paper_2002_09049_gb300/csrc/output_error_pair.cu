@@ -130,25 +130,7 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
 #pragma unroll
     for (int i = 0; i < G::ITEMS2; ++i) {
         const int p = pt + i * P_PROD_THREADS;
-        if (CLIP && p < nch * (P_KC / 2)) {
-            const int ch = p / (P_KC / 2), e2 = p % (P_KC / 2);
-            const float2 w = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
-            const uint32_t cofs = (uint32_t)(e2 & 1) * 8u;
-#pragma unroll 4
-            for (int c = 0; c < KP1; ++c) {
-                const float s = ctl.clip_s[ch * KP1 + c], inv = ctl.clip_inv[ch * KP1 + c];
-                // exact code of Eq. 8 (0 when the scale is 0 or NaN: the residual is then w or NaN)
-                const float qx = s > 0.0f ? copysignf((float)code_fast(fabsf(w.x), s, inv, qmaxf), w.x) : 0.0f;
-                const float qy = s > 0.0f ? copysignf((float)code_fast(fabsf(w.y), s, inv, qmaxf), w.y) : 0.0f;
-                float2 r, hi, lo;
-                r.x = __fmaf_rn(-s, qx, w.x);
-                r.y = __fmaf_rn(-s, qy, w.y);
-                split2(r, hi, lo);
-                const uint32_t off = sw128_offset(ch * KP1 + c, e2 >> 1) + cofs;
-                st_shared_v2(sb + P_OFF_A_HI + off, hi);
-                st_shared_v2(sb + P_OFF_A_LO + off, lo);
-            }
-        } else if (!CLIP && p < nch * (P_KC / 2)) {
+        if (!CLIP && p < nch * (P_KC / 2)) {
             const int ch = p / (P_KC / 2), e2 = p % (P_KC / 2);
             float2 r = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
             uint32_t qb[G::KQ];
@@ -169,6 +151,33 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
                     r.x = __fmaf_rn(-sn, code_from_biased(qb[n], 0), r.x);
                     r.y = __fmaf_rn(-sn, code_from_biased(qb[n], 1), r.y);
                 }
+            }
+        }
+    }
+    if constexpr (CLIP) {
+        // (candidate, channel, element pair) units over all producer threads, element pairs
+        // lane-contiguous: each warp store fills whole 128-byte rows.
+        const int rows = nch * KP1;                     // row = c * nch + ch
+        const int e2 = pt % (P_KC / 2);                  // the same for all of this thread's units
+        int row = pt / (P_KC / 2);
+        int c = nch > 0 ? row / nch : 0, ch = nch > 0 ? row - c * nch : 0;
+        for (; row < rows; row += P_PROD_THREADS / (P_KC / 2)) {
+            const float2 w = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
+            const float s = ctl.clip_s[ch * KP1 + c], inv = ctl.clip_inv[ch * KP1 + c];
+            // exact code of Eq. 8 (0 when the scale is 0 or NaN: the residual is then w or NaN)
+            const float qx = s > 0.0f ? copysignf((float)code_fast(fabsf(w.x), s, inv, qmaxf), w.x) : 0.0f;
+            const float qy = s > 0.0f ? copysignf((float)code_fast(fabsf(w.y), s, inv, qmaxf), w.y) : 0.0f;
+            float2 r, hi, lo;
+            r.x = __fmaf_rn(-s, qx, w.x);
+            r.y = __fmaf_rn(-s, qy, w.y);
+            split2(r, hi, lo);
+            const uint32_t off = sw128_offset(ch * KP1 + c, e2 >> 1) + (uint32_t)(e2 & 1) * 8u;
+            st_shared_v2(sb + P_OFF_A_HI + off, hi);
+            st_shared_v2(sb + P_OFF_A_LO + off, lo);
+            ch += P_PROD_THREADS / (P_KC / 2);           // next row: advance (c, ch) without dividing
+            while (ch >= nch) {
+                ch -= nch;
+                ++c;
             }
         }
     }

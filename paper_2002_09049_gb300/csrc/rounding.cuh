@@ -18,15 +18,13 @@ __device__ __forceinline__ int code_mag(float a, float s, float qmaxf)
 // the correctly rounded division would.
 #define MPQ_FAST_REL 9.5367431640625e-07f /* 2^-20 */
 
-// min(Qmax, rint(fl(a/s))), decided from q' = a * (1/s) unless q' is too close to a half-integer.
+// min(Qmax, rint(fl(a/s))), decided from q' = a * (1/s) unless q' is too close to a half-integer:
+// then q' and the exact quotient round to the same integer (no tie can lie between them).
 __device__ __forceinline__ int code_fast(float a, float s, float inv_s, float qmaxf)
 {
     const float qf = __fmul_rn(a, inv_s);
-    const float tol = MPQ_FAST_REL * (qf + 1.0f);
-    if (qf > qmaxf + 0.5f + tol) return (int)qmaxf;
-    const float fl = floorf(qf);
-    const float fr = qf - fl;   // exact
-    if (fabsf(fr - 0.5f) > tol) return (int)fminf(fr > 0.5f ? fl + 1.0f : fl, qmaxf);
+    const float rq = rintf(qf);
+    if (0.5f - fabsf(qf - rq) > MPQ_FAST_REL * (qf + 1.0f)) return (int)fminf(rq, qmaxf);
     return (int)fminf(rintf(__fdiv_rn(a, s)), qmaxf);
 }
 
