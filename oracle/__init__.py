@@ -66,6 +66,10 @@ def _load():
         lib.mpqo_clip_errors.restype = None
         lib.mpqo_clip_select.argtypes = [P, I, I, I, P]
         lib.mpqo_clip_select.restype = None
+        lib.mpqo_fixed_coeff.argtypes = [ctypes.c_float, I, P]
+        lib.mpqo_fixed_coeff.restype = ctypes.c_longlong
+        lib.mpqo_multipoint_linear.argtypes = [P, I, P, P, P, I, I, I, I, P, I, I]
+        lib.mpqo_multipoint_linear.restype = I
         _lib = lib
     return _lib
 
@@ -228,6 +232,38 @@ def clip_select(err32, mode: int):
     best = np.zeros(C, np.int32)
     lib.mpqo_clip_select(_p(err32), C, n_cand, mode, _p(best))
     return best
+
+
+def fixed_coeff(s: float, p: int):
+    """Eq. 13: A = rint(2^p s) as an int; None when it does not fit 32 bits."""
+    lib = _load()
+    ok = ctypes.c_int(1)
+    a = lib.mpqo_fixed_coeff(float(s), p, ctypes.byref(ok))
+    return int(a) if ok.value else None
+
+
+def multipoint_linear(X, codes, scales, npoints, p: int, channels=None, threads: int = 1):
+    """Sec. 3.4 steps 1-3: Y [C][T] int32 = sat32(floor(sum_i A_i (q_i . x_t) / 2^p)), exact."""
+    lib = _load()
+    X = _c(X, np.int8)
+    codes = _c(codes, np.int8)
+    scales = _c(scales, np.float32)
+    npoints = _c(npoints, np.int32)
+    T, d = X.shape
+    k_max, C, _ = codes.shape
+    Y = np.zeros((C, T), np.int32)
+    c0, c1 = channels if channels is not None else (0, C)
+    bad = []
+
+    def run(rng):
+        if lib.mpqo_multipoint_linear(_p(X), T, _p(codes), _p(scales), _p(npoints), C, d, k_max,
+                                      p, _p(Y), rng[0], rng[1]):
+            bad.append(rng)
+
+    _parallel(run, [(a + c0, b + c0) for a, b in _ranges(c1 - c0, threads)], threads)
+    if bad:
+        raise OverflowError("a coefficient 2^p * s does not fit 32 bits")
+    return Y
 
 
 def _parallel(fn, ranges, threads):

@@ -404,3 +404,60 @@ void mpqo_clip_select(const float *err, int C, int nc, int mode, int *best)
     }
     for (int k = 0; k < C; ++k) best[k] = b;
 }
+
+/* ---- Eq. 13 and Sec. 3.4: integer inference with multipoint weights -------------------------------
+ * A layer whose channel k holds n_k points (s_{k,i}, q_{k,i}) computes, for integer inputs x_t,
+ *   w~_k^T x_t = sum_i s_{k,i} (q_{k,i}^T x_t) ~ (sum_i A_{k,i} (q_{k,i}^T x_t)) / 2^p,
+ *   A_{k,i} = [2^p s_{k,i}]  (Eq. 13),
+ * in three steps: integer dot products (step 1), multiplication by the 32-bit coefficients and
+ * summation (step 2), and a shift by p bits (step 3).  Readings (also in the design doc): the codes q are
+ * the integers of the symmetric set, so the coefficient of q is s = a / Qmax and A = rint(2^p s)
+ * (ties to even); "shifting p bits" is an arithmetic right shift, i.e. floor division by 2^p; the
+ * products and sums are exact (64-bit); the result saturates to the 32-bit range; n_k = npoints[k]
+ * clamped to [0, k_max]; a coefficient that does not fit 32 bits is an error. */
+
+/* A = rint(2^p s); *ok = 0 when it does not fit a 32-bit integer (or s is not finite). */
+long long mpqo_fixed_coeff(float s, int p, int *ok)
+{
+    double v = nearbyint(ldexp((double)s, p));
+    if (!(fabs(v) < 2147483648.0)) {
+        *ok = 0;
+        return 0;
+    }
+    return (long long)v;
+}
+
+/* Y[k][t] for channels [c0, c1), X [T][d] int8, Y [C][T] int32.  Returns 0, or 1 if a coefficient
+ * did not fit 32 bits (Y is then unspecified). */
+int mpqo_multipoint_linear(const int8_t *X, int T, const int8_t *codes, const float *scales,
+                           const int *npoints, int C, int d, int k_max, int p, int32_t *Y, int c0,
+                           int c1)
+{
+    long plane = (long)C * d;
+    for (int k = c0; k < c1; ++k) {
+        int n = npoints[k];
+        if (n < 0) n = 0;
+        if (n > k_max) n = k_max;
+        long long A[64];
+        for (int i = 0; i < n; ++i) {
+            int ok = 1;
+            A[i] = mpqo_fixed_coeff(scales[(long)k * k_max + i], p, &ok);
+            if (!ok) return 1;
+        }
+        for (int t = 0; t < T; ++t) {
+            const int8_t *x = X + (long)t * d;
+            long long sum = 0;
+            for (int i = 0; i < n; ++i) {
+                const int8_t *q = codes + (long)i * plane + (long)k * d;
+                long long acc = 0;                                  /* step 1 */
+                for (int j = 0; j < d; ++j) acc += (long long)q[j] * (long long)x[j];
+                sum += A[i] * acc;                                  /* step 2 */
+            }
+            long long y = sum >= 0 ? (sum >> p) : -((-sum + ((1LL << p) - 1)) >> p);  /* step 3: floor */
+            if (y > 2147483647LL) y = 2147483647LL;
+            if (y < -2147483648LL) y = -2147483648LL;
+            Y[(long)k * T + t] = (int32_t)y;
+        }
+    }
+    return 0;
+}

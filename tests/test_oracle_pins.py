@@ -412,3 +412,73 @@ def test_clip_single_channel_layer_and_nonfinite(oracle):
     assert np.all(np.isnan(c1))
     e1 = oracle.clip_errors(X, 1, W, 4, c1).astype(np.float32)
     assert list(oracle.clip_select(e1, oracle.CLIP_PER_LAYER)) == [-1, -1, -1]
+
+
+# ---- Eq. 13 / Sec. 3.4: integer inference with multipoint weights ---------------------------------
+
+def test_integer_inference_hand_example(oracle):
+    g = json.load(open(os.path.join(GOLDEN, "integer_inference_hand_example.json")))
+    codes = np.array(g["codes"], np.int8)
+    scales = np.array(g["scales"], np.float32)
+    for k in range(2):
+        for i in range(2):
+            assert oracle.fixed_coeff(scales[k, i], g["p"]) == g["A"][k][i]
+    Y = oracle.multipoint_linear(np.array(g["X"], np.int8), codes, scales,
+                                 np.array(g["npoints"], np.int32), g["p"])
+    assert Y.tolist() == g["Y"]
+
+
+def test_integer_inference_exact_rational(oracle):
+    """Scales that are multiples of 2^-p: the result is floor(sum_i s_i (q_i . x)) exactly, checked
+    with Python's rational arithmetic."""
+    rng = np.random.default_rng(41)
+    for p in (0, 3, 12):
+        k_max, C, d, T = 3, 5, 17, 6
+        codes = rng.integers(-7, 8, (k_max, C, d)).astype(np.int8)
+        A = rng.integers(-2000, 2000, (C, k_max))
+        scales = (A / 2.0 ** p).astype(np.float32)
+        assert np.array_equal(scales.astype(np.float64) * 2.0 ** p, A)
+        npts = rng.integers(0, k_max + 1, C).astype(np.int32)
+        X = rng.integers(-128, 128, (T, d)).astype(np.int8)
+        Y = oracle.multipoint_linear(X, codes, scales, npts, p)
+        for k in range(C):
+            for t in range(T):
+                v = sum(Fraction(int(A[k, i]), 2 ** p) *
+                        int(np.dot(codes[i, k].astype(np.int64), X[t].astype(np.int64)))
+                        for i in range(npts[k]))
+                assert Y[k, t] == (v.numerator // v.denominator)
+
+
+def test_integer_inference_tracks_reconstruction(oracle):
+    """Against Eq. 4: Y is w~^T x up to the coefficient rounding (|A/2^p - s| <= 2^-(p+1) per point
+    and dot product), the floor, and the fp32 rounding of the reconstructed weights."""
+    rng = np.random.default_rng(42)
+    W = rng.standard_normal((12, 96)).astype(np.float32) * 0.05
+    q = oracle.quantize_layer(W, 4, 32, 4)
+    npts = rng.integers(1, 5, 12).astype(np.int32)
+    W_hat = oracle.reconstruct(q["codes"], q["scales"], npts)
+    X = rng.integers(-128, 128, (20, 96)).astype(np.int8)
+    for p in (8, 16, 20):
+        Y = oracle.multipoint_linear(X, q["codes"], q["scales"], npts, p).astype(np.float64)
+        ref = W_hat.astype(np.float64) @ X.T.astype(np.float64)
+        for k in range(12):
+            acc = np.abs(q["codes"][:npts[k], k].astype(np.int64) @ X.T.astype(np.int64))
+            sq = np.abs(q["scales"][k, :npts[k], None].astype(np.float64) *
+                        q["codes"][:npts[k], k].astype(np.float64))
+            bound = (0.5 * acc.sum(axis=0) / 2.0 ** p + 1 +
+                     npts[k] * 2.0 ** -23 * np.abs(X.astype(np.float64)) @ sq.sum(axis=0))
+            assert np.all(np.abs(Y[k] - ref[k]) <= bound)
+
+
+def test_integer_inference_edges(oracle):
+    codes = np.full((2, 1, 4), 127, np.int8)
+    X = np.full((1, 4), 127, np.int8)
+    big = np.array([[40000.0, 40000.0]], np.float32)        # 2 * 40000 * 64516 > 2^31: saturates
+    assert oracle.multipoint_linear(X, codes, big, np.array([2], np.int32), 0)[0, 0] == 2 ** 31 - 1
+    assert oracle.multipoint_linear(X, codes, -big, np.array([2], np.int32), 0)[0, 0] == -2 ** 31
+    with pytest.raises(OverflowError):                        # 2^p s does not fit 32 bits
+        oracle.multipoint_linear(X, codes, big, np.array([1], np.int32), 16)
+    s = np.array([[0.5, 0.25]], np.float32)
+    assert oracle.multipoint_linear(X, codes, s, np.array([0], np.int32), 4)[0, 0] == 0
+    y2 = oracle.multipoint_linear(X, codes, s, np.array([2], np.int32), 4)
+    assert np.array_equal(oracle.multipoint_linear(X, codes, s, np.array([9], np.int32), 4), y2)
