@@ -171,6 +171,57 @@ mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, in
                            int bits, int n_cand, int mode, float *clip, float *err, int *best,
                            void *stream);
 
+/*
+ * Integer inference with multipoint weights (Sec. 3.4, Eq. 13).  For integer inputs x_t (int8),
+ * channel k with n_k points (s_{k,i}, q_{k,i}) computes
+ *   Y[k][t] = sat32( floor( sum_{i<n_k} A_{k,i} (q_{k,i} . x_t) / 2^p ) ),  A_{k,i} = rint(2^p s_{k,i})
+ * (ties to even): integer dot products (step 1), multiplication by the 32-bit coefficients and
+ * summation (step 2), and the shift by p bits (step 3; an arithmetic right shift, i.e. floor), with
+ * exact 64-bit products and sums and saturation to the int32 range.  n_k = npoints[k] clamped to
+ * [0, k_max]; a channel with no point outputs 0.  The q are the integer codes of mpq_quantize_layer,
+ * so the coefficient of q is s = a / Qmax.
+ *
+ * Deployment is split as in the paper: the coefficients and a packed copy of the used points are
+ * made once, offline (mpq_pack_layout on the host, then mpq_pack_points), and
+ * mpq_multipoint_linear runs per input batch.
+ */
+typedef struct {
+    int C, d, k_max, bits, p;
+    int d_pad;           /* d rounded up to a multiple of 64 */
+    int rows;            /* packed code rows, a multiple of 128 */
+    int tiles;           /* rows / 128 */
+    size_t off_coef, off_chan, off_point, off_tile, off_codes;   /* byte offsets in the buffer */
+    size_t bytes;        /* size of the device buffer to allocate */
+} mpq_packed_layout;
+
+/*
+ * mpq_pack_layout -- HOST only: the layout of a packed layer for the given point counts.
+ *   npoints  HOST [C] int32 (e.g. copied back from mpq_allocate_points).
+ *   bits     the codes' width (their magnitude is at most 2^(bits-1) - 1).
+ *   p        coefficient precision, 0..30.
+ *   layout   out.
+ */
+mpq_status mpq_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
+                           mpq_packed_layout *layout);
+
+/*
+ * mpq_pack_points -- fill a packed layer: coefficients A = rint(2^p s) of the used points and their
+ * codes (as bf16, exact).  Synchronous: returns after the device has finished with the host array.
+ *   codes [k_max][C][d] int8 and scales [C][k_max] fp32 on the device (from mpq_quantize_layer);
+ *   npoints HOST [C], the same as given to mpq_pack_layout;
+ *   packed  device buffer of layout->bytes bytes, written here.
+ * MPQ_ERR_UNSUPPORTED if a coefficient does not fit 32 bits.
+ */
+mpq_status mpq_pack_points(const int8_t *codes, const float *scales, const int *npoints,
+                           const mpq_packed_layout *layout, void *packed, void *stream);
+
+/*
+ * mpq_multipoint_linear -- Y [C][T] int32 (channel-major: one channel's T outputs are contiguous)
+ * for X [T][d] int8 inputs (row-major), from a packed layer.  T >= 1.
+ */
+mpq_status mpq_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout *layout,
+                                 const void *packed, int32_t *Y, void *stream);
+
 /* Name of a status code (static string). */
 const char *mpq_status_string(mpq_status s);
 

@@ -7,6 +7,7 @@ raises.
 """
 from . import overhead, workloads  # noqa: F401
 from .binding import (MPQ_ALLOC_BUDGET, MPQ_ALLOC_THRESHOLD, MPQ_CLIP_PER_CHANNEL,  # noqa: F401
-                      MPQ_CLIP_PER_LAYER, MPQError, mpq_allocate_points, mpq_clip_search,
-                      mpq_output_error, mpq_quantize_layer, mpq_reconstruct, mpq_status_string,
+                      MPQ_CLIP_PER_LAYER, MPQError, PackedLayout, mpq_allocate_points,
+                      mpq_clip_search, mpq_multipoint_linear, mpq_output_error, mpq_pack_layout,
+                      mpq_pack_points, mpq_quantize_layer, mpq_reconstruct, mpq_status_string,
                       mpq_version)

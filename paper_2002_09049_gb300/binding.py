@@ -25,12 +25,27 @@ MPQ_STATUS = {0: "MPQ_OK", 1: "MPQ_ERR_INVALID_ARG", 2: "MPQ_ERR_NONFINITE",
 
 # name -> (argtypes, restype), in the order of include/mpq.h
 _P, _I, _D = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+class PackedLayout(ctypes.Structure):
+    """mpq_packed_layout of include/mpq.h: the layout of a packed multipoint layer (Sec. 3.4)."""
+    _fields_ = [("C", ctypes.c_int), ("d", ctypes.c_int), ("k_max", ctypes.c_int),
+                ("bits", ctypes.c_int), ("p", ctypes.c_int), ("d_pad", ctypes.c_int),
+                ("rows", ctypes.c_int), ("tiles", ctypes.c_int),
+                ("off_coef", ctypes.c_size_t), ("off_chan", ctypes.c_size_t),
+                ("off_point", ctypes.c_size_t), ("off_tile", ctypes.c_size_t),
+                ("off_codes", ctypes.c_size_t), ("bytes", ctypes.c_size_t)]
+
+
+_L = ctypes.POINTER(PackedLayout)
+
 SIGNATURES = {
     "mpq_quantize_layer": ([_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P], _I),
     "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
     "mpq_reconstruct": ([_P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_clip_search": ([_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P], _I),
+    "mpq_pack_layout": ([_P, _I, _I, _I, _I, _I, _L], _I),
+    "mpq_pack_points": ([_P, _P, _P, _L, _P, _P], _I),
+    "mpq_multipoint_linear": ([_P, _I, _L, _P, _P, _P], _I),
     "mpq_status_string": ([_I], ctypes.c_char_p),
     "mpq_last_error": ([], ctypes.c_char_p),
     "mpq_version": ([], _I),
@@ -182,6 +197,55 @@ def mpq_clip_search(X, W, bits: int, n_cand: int = 20, mode: int = None, groups:
                                 _ptr(err), _ptr(best), _stream(stream))
     _check(st, "mpq_clip_search")
     return clip, err, best
+
+
+def _host_int32(a):
+    import numpy as np
+    if isinstance(a, torch.Tensor):
+        a = a.detach().cpu().numpy()
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def mpq_pack_layout(npoints, d: int, k_max: int, bits: int, p: int) -> PackedLayout:
+    """Host-side layout of a packed multipoint layer (Sec. 3.4) for the point counts npoints [C]."""
+    n = _host_int32(npoints)
+    lay = PackedLayout()
+    st = load().mpq_pack_layout(n.ctypes.data, int(n.size), d, k_max, bits, p, ctypes.byref(lay))
+    _check(st, "mpq_pack_layout")
+    return lay
+
+
+def mpq_pack_points(codes, scales, npoints, layout: PackedLayout, packed=None, stream=None):
+    """Coefficients rint(2^p s) and bf16 codes of the used points (offline, synchronous).
+    Returns the packed device buffer (uint8 [layout.bytes])."""
+    _dev(codes, "codes", torch.int8, (layout.k_max, layout.C, layout.d))
+    _dev(scales, "scales", torch.float32, (layout.C, layout.k_max))
+    n = _host_int32(npoints)
+    if n.size != layout.C:
+        raise ValueError("npoints must have C entries")
+    packed = packed if packed is not None else torch.empty((max(1, layout.bytes),), dtype=torch.uint8,
+                                                           device=codes.device)
+    _dev(packed, "packed", torch.uint8)
+    if packed.numel() < layout.bytes:
+        raise ValueError("packed buffer smaller than layout.bytes")
+    st = load().mpq_pack_points(_ptr(codes), _ptr(scales), n.ctypes.data, ctypes.byref(layout),
+                                _ptr(packed), _stream(stream))
+    _check(st, "mpq_pack_points")
+    return packed
+
+
+def mpq_multipoint_linear(X, layout: PackedLayout, packed, Y=None, stream=None):
+    """Integer inference (Eq. 13): Y [C][T] int32 for X [T][d] int8."""
+    _dev(X, "X", torch.int8)
+    if X.dim() != 2 or X.shape[1] != layout.d:
+        raise ValueError("X must be [T][d]")
+    T = X.shape[0]
+    Y = Y if Y is not None else torch.empty((layout.C, T), dtype=torch.int32, device=X.device)
+    _dev(Y, "Y", torch.int32, (layout.C, T))
+    st = load().mpq_multipoint_linear(_ptr(X), T, ctypes.byref(layout), _ptr(packed), _ptr(Y),
+                                      _stream(stream))
+    _check(st, "mpq_multipoint_linear")
+    return Y
 
 
 def mpq_allocate_points(err, k_max: int, mode: int = MPQ_ALLOC_BUDGET,

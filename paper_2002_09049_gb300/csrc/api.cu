@@ -161,6 +161,51 @@ extern "C" mpq_status mpq_clip_search(const float *X, int N, int groups, const f
                        (cudaStream_t)stream);
 }
 
+extern "C" mpq_status mpq_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
+                                      mpq_packed_layout *layout)
+{
+    g_msg[0] = 0;
+    mpq_status st = check_common(C, d, k_max);
+    if (st != MPQ_OK) return st;
+    REQUIRE(d <= MPQ_MAX_DIM, MPQ_ERR_UNSUPPORTED, "d = %d exceeds MPQ_MAX_DIM = %d", d,
+            MPQ_MAX_DIM);
+    REQUIRE(bits >= MPQ_MIN_BITS && bits <= MPQ_MAX_BITS,
+            (bits > MPQ_MAX_BITS ? MPQ_ERR_UNSUPPORTED : MPQ_ERR_INVALID_ARG),
+            "bits = %d outside [%d, %d]", bits, MPQ_MIN_BITS, MPQ_MAX_BITS);
+    REQUIRE(p >= 0 && p <= 30, MPQ_ERR_INVALID_ARG, "p = %d outside [0, 30]", p);
+    REQUIRE(layout, MPQ_ERR_INVALID_ARG, "layout must be non-NULL");
+    REQUIRE(C == 0 || npoints, MPQ_ERR_INVALID_ARG, "npoints must be non-NULL");
+    return make_pack_layout(npoints, C, d, k_max, bits, p, layout);
+}
+
+extern "C" mpq_status mpq_pack_points(const int8_t *codes, const float *scales, const int *npoints,
+                                      const mpq_packed_layout *layout, void *packed, void *stream)
+{
+    g_msg[0] = 0;
+    REQUIRE(layout, MPQ_ERR_INVALID_ARG, "layout must be non-NULL");
+    mpq_status st = check_common(layout->C, layout->d, layout->k_max);
+    if (st != MPQ_OK) return st;
+    if (layout->C == 0) return MPQ_OK;
+    REQUIRE(codes && scales && npoints && packed, MPQ_ERR_INVALID_ARG,
+            "codes, scales, npoints and packed must be non-NULL");
+    return launch_pack(codes, scales, npoints, layout, packed, (cudaStream_t)stream);
+}
+
+extern "C" mpq_status mpq_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout *layout,
+                                            const void *packed, int32_t *Y, void *stream)
+{
+    g_msg[0] = 0;
+    REQUIRE(layout, MPQ_ERR_INVALID_ARG, "layout must be non-NULL");
+    mpq_status st = check_common(layout->C, layout->d, layout->k_max);
+    if (st != MPQ_OK) return st;
+    REQUIRE(T >= 1, MPQ_ERR_INVALID_ARG, "T = %d must be >= 1", T);
+    REQUIRE((long long)T * layout->d <= (1LL << 40) && (long long)T * layout->C <= (1LL << 40),
+            MPQ_ERR_UNSUPPORTED, "T too large");
+    if (layout->C == 0) return MPQ_OK;
+    REQUIRE(X && packed && Y, MPQ_ERR_INVALID_ARG, "X, packed and Y must be non-NULL");
+    return launch_multipoint_linear(X, T, layout, packed, Y, (cudaStream_t)stream);
+}
+
 extern "C" mpq_status mpq_allocate_points(const float *err, int C, int k_max, int mode,
                                           double budget_or_eps, int *npoints, int *points_used,
                                           void *stream)

@@ -49,6 +49,13 @@ mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C,
                        int n_cand, int mode, float *clip, float *err, int *best,
                        cudaStream_t stream);
 
+mpq_status make_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
+                            mpq_packed_layout *L);
+mpq_status launch_pack(const int8_t *codes, const float *scales, const int *npoints,
+                       const mpq_packed_layout *L, void *packed, cudaStream_t stream);
+mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout *L,
+                                    const void *packed, int32_t *Y, cudaStream_t stream);
+
 mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
                                   int *npoints, int *points_used, cudaStream_t stream);
 

@@ -1,0 +1,485 @@
+// Integer inference with multipoint weights (Sec. 3.4, Eq. 13):
+//   Y[k][t] = sat32( floor( sum_{i<n_k} A_{k,i} (q_{k,i} . x_t) / 2^p ) ),  A_{k,i} = rint(2^p s_{k,i}),
+// in the paper's three steps: integer dot products of every point's codes with the integer input
+// (step 1), multiplication by the 32-bit coefficients and summation (step 2), and the shift by p
+// (step 3).
+//
+// Packing (offline, mpq_pack_points).  Each channel's n_k code rows become consecutive rows of one
+// operand: channels are grouped by R = the power of two >= n_k (a channel with no point gets one
+// zero row), and every 128-row tile holds 128/R channels of one group, so a channel's rows are R
+// aligned TMEM lanes of one warp.  Rows past n_k and empty slots are zero with coefficient 0.  The
+// codes are stored as bf16 (every int8 value is exact), rows padded to a multiple of 64 elements.
+//
+// Step 1 on the tensor cores.  tcgen05.mma kind::f16 with bf16 operands: the codes (TMA straight
+// into 128-byte-swizzled K-major tiles) against the input rows (int8 by TMA into a raw ring, turned
+// into bf16 exactly by eight producer warps through the fp32 exponent bias).  Products are exact
+// and every partial sum is an integer of magnitude below 2^24 when d * Qmax * 128 < 2^24, so the
+// fp32 accumulator holds the exact dot products (checked on the host; other layers take the
+// integer kernel below).  Tile: 128 packed rows x 256 inputs, K chunks of 64, 3 stages.
+// Steps 2 and 3 in the epilogue: each lane turns its accumulator into an integer, multiplies by its
+// row's coefficient in 64 bits, the R lanes of a channel add with warp shuffles, and the first lane
+// shifts (arithmetic: floor), saturates and writes 32 consecutive outputs.  Every wait is bounded.
+//
+// Rows that TMA cannot address (d not a multiple of 16, unaligned input) and layers beyond the
+// exactness bound use a CUDA-core kernel with the same integer arithmetic.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+#include <string.h>
+
+#include <vector>
+
+#include "mpq_internal.cuh"
+#include "sm100.cuh"
+#include "tf32_operands.cuh"
+
+namespace mpq {
+namespace {
+
+using namespace sm100;
+
+constexpr int L_M = 128;                        // packed rows per tile (TMEM lanes)
+constexpr int L_N = 256;                        // inputs per tile (UMMA N)
+constexpr int L_KC = 64;                        // bf16 per K chunk = one 128-byte swizzle row
+constexpr int L_STAGES = 3;
+constexpr int L_A_BYTES = L_M * L_KC * 2;       // 16 KB codes tile
+constexpr int L_B_BYTES = L_N * L_KC * 2;       // 32 KB input tile (bf16)
+constexpr int L_RAW_BYTES = L_N * L_KC;         // 16 KB input tile (int8, as loaded)
+constexpr int L_OFF_B = L_A_BYTES;
+constexpr int L_OFF_RAW = L_A_BYTES + L_B_BYTES;
+constexpr int L_STAGE_BYTES = L_A_BYTES + L_B_BYTES + L_RAW_BYTES;   // 64 KB
+constexpr int L_PROD_WARPS = 8;
+constexpr int L_PROD_THREADS = L_PROD_WARPS * 32;
+constexpr int L_EPI_WARP0 = L_PROD_WARPS;       // warps 8..11: warp % 4 selects TMEM lanes
+constexpr int L_MMA_WARP = L_EPI_WARP0 + 4;
+constexpr int L_TMA_WARP = L_MMA_WARP + 1;
+constexpr int L_THREADS = (L_TMA_WARP + 1) * 32;   // 448
+constexpr uint32_t L_TMEM_COLS = 256;
+constexpr long long L_WAIT = 1LL << 31;
+
+struct LinCtrl {
+    uint64_t loaded[L_STAGES];    // TMA bytes of a stage have landed
+    uint64_t full[L_STAGES];      // producers converted the input tile
+    uint64_t empty[L_STAGES];     // MMAs on the stage completed
+    uint64_t done;                // every MMA completed
+    uint32_t tmem_base;
+    int abort;
+    int coef[L_M];                // this tile's row coefficients A
+};
+constexpr int L_CTRL_BYTES = (sizeof(LinCtrl) + 1023) / 1024 * 1024;
+constexpr int L_SMEM = 1024 + L_CTRL_BYTES + L_STAGES * L_STAGE_BYTES;
+
+// Row r of a packed buffer: (channel, point) or channel -1 / point -1 for padding.
+struct PackView {
+    int *coef;
+    int *chan;
+    int *point;
+    int *tile_R;
+    __nv_bfloat16 *codes;
+    int *flag;
+};
+
+PackView view(const mpq_packed_layout *L, void *packed)
+{
+    unsigned char *b = static_cast<unsigned char *>(packed);
+    PackView v;
+    v.coef = reinterpret_cast<int *>(b + L->off_coef);
+    v.chan = reinterpret_cast<int *>(b + L->off_chan);
+    v.point = reinterpret_cast<int *>(b + L->off_point);
+    v.tile_R = reinterpret_cast<int *>(b + L->off_tile);
+    v.codes = reinterpret_cast<__nv_bfloat16 *>(b + L->off_codes);
+    v.flag = reinterpret_cast<int *>(b);   // header word 0: coefficient overflow
+    return v;
+}
+
+// A = rint(2^p s) (ties to even) and the bf16 codes of every packed row.
+__global__ void pack_kernel(const int8_t *__restrict__ codes, const float *__restrict__ scales,
+                            int C, int d, int d_pad, int k_max, int p, int rows, PackView v)
+{
+    const int r = blockIdx.x;
+    const int k = v.chan[r], i = v.point[r];
+    const bool live = k >= 0 && i >= 0;
+    if (threadIdx.x == 0) {
+        int a = 0;
+        if (live) {
+            const double x = nearbyint(ldexp((double)scales[(size_t)k * k_max + i], p));
+            if (fabs(x) < 2147483648.0) a = (int)x;
+            else atomicExch(v.flag, 1);
+        }
+        v.coef[r] = a;
+    }
+    const int8_t *q = live ? codes + (size_t)i * C * d + (size_t)k * d : nullptr;
+    for (int j = threadIdx.x; j < d_pad; j += blockDim.x)
+        v.codes[(size_t)r * d_pad + j] = __float2bfloat16_rn(live && j < d ? (float)q[j] : 0.0f);
+}
+
+// Two int8 -> two bf16 packed in a word (exact: |v| <= 128 has at most 8 significant bits).
+__device__ __forceinline__ uint32_t bf16x2_from_biased(uint32_t biased, int b0)
+{
+    const uint32_t lo = __float_as_uint(code_from_biased(biased, b0));
+    const uint32_t hi = __float_as_uint(code_from_biased(biased, b0 + 1));
+    return __byte_perm(lo, hi, 0x7632u);
+}
+
+__global__ void __launch_bounds__(L_THREADS, 1)
+multipoint_linear_kernel(int T, int n_kc, int p, const int *__restrict__ coef,
+                         const int *__restrict__ chan, const int *__restrict__ tile_R,
+                         int32_t *__restrict__ Y, const __grid_constant__ CUtensorMap tmA,
+                         const __grid_constant__ CUtensorMap tmX)
+{
+    extern __shared__ unsigned char smem_raw[];
+    const uint32_t raw_u32 = smem_u32(smem_raw);
+    const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
+    LinCtrl &ctl = *reinterpret_cast<LinCtrl *>(smem_raw + pad);
+    const uint32_t stages_u32 = raw_u32 + pad + L_CTRL_BYTES;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tile = blockIdx.x, n0 = blockIdx.y * L_N;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < L_STAGES; ++s) {
+            mbar_init(&ctl.loaded[s], 1);
+            mbar_init(&ctl.full[s], L_PROD_WARPS);
+            mbar_init(&ctl.empty[s], 1);
+        }
+        mbar_init(&ctl.done, 1);
+        ctl.abort = 0;
+        fence_barrier_init();
+    }
+    for (int r = threadIdx.x; r < L_M; r += L_THREADS) ctl.coef[r] = coef[(size_t)tile * L_M + r];
+    if (warp == L_MMA_WARP) {
+        tmem_alloc(&ctl.tmem_base, L_TMEM_COLS);
+        tc_fence_before();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = ctl.tmem_base;
+    volatile int *abort_flag = &ctl.abort;
+
+    if (warp < L_PROD_WARPS) {
+        // ---------------------------------------------------------------- producers: int8 -> bf16
+        for (int kc = 0; kc < n_kc; ++kc) {
+            const int s = kc % L_STAGES;
+            const uint32_t ph = (uint32_t)(kc / L_STAGES) & 1u;
+            const bool ok = mbar_wait(&ctl.loaded[s], ph, L_WAIT);
+            if (!ok) *abort_flag = 1;
+            if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
+            const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
+            // 16 input bytes (one input row, 16 K elements) per item, 4 items per thread
+#pragma unroll
+            for (int it = 0; it < L_N * (L_KC / 16) / L_PROD_THREADS; ++it) {
+                const int q = threadIdx.x + it * L_PROD_THREADS;
+                const int row = q >> 2, c16 = q & 3;
+                const float4 raw = ld_shared_v4(sb + L_OFF_RAW + (uint32_t)q * 16u);
+                const uint32_t w[4] = {__float_as_uint(raw.x) ^ 0x80808080u,
+                                       __float_as_uint(raw.y) ^ 0x80808080u,
+                                       __float_as_uint(raw.z) ^ 0x80808080u,
+                                       __float_as_uint(raw.w) ^ 0x80808080u};
+                float4 o0, o1;
+                o0.x = __uint_as_float(bf16x2_from_biased(w[0], 0));
+                o0.y = __uint_as_float(bf16x2_from_biased(w[0], 2));
+                o0.z = __uint_as_float(bf16x2_from_biased(w[1], 0));
+                o0.w = __uint_as_float(bf16x2_from_biased(w[1], 2));
+                o1.x = __uint_as_float(bf16x2_from_biased(w[2], 0));
+                o1.y = __uint_as_float(bf16x2_from_biased(w[2], 2));
+                o1.z = __uint_as_float(bf16x2_from_biased(w[3], 0));
+                o1.w = __uint_as_float(bf16x2_from_biased(w[3], 2));
+                st_shared_v4(sb + L_OFF_B + sw128_offset(row, 2 * c16), o0);
+                st_shared_v4(sb + L_OFF_B + sw128_offset(row, 2 * c16 + 1), o1);
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl.full[s]);
+        }
+    } else if (warp < L_MMA_WARP) {
+        // ---------------------------------------------------------------- epilogue
+        const int ew = warp - L_EPI_WARP0;
+        const bool ok = mbar_wait(&ctl.done, 0, L_WAIT);
+        if (!ok) *abort_flag = 1;
+        const bool good = !__any_sync(0xffffffffu, !ok || *abort_flag);
+        tc_fence_after();
+        const int R = tile_R[tile];
+        const int r = ew * 32 + lane;
+        const int k = chan[(size_t)tile * L_M + r];
+        const long long a = ctl.coef[r];
+        const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16);
+        if (good) {
+#pragma unroll 1
+            for (int cb = 0; cb < L_N / 32; ++cb) {
+                float v[32];
+                tmem_ld_32x32b_x32(lane_base + (uint32_t)(cb * 32), v);
+                long long sum[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) sum[j] = a * (long long)__float2int_rz(v[j]);
+                for (int o = 1; o < R; o <<= 1) {   // the channel's R lanes (R-aligned)
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) sum[j] += __shfl_xor_sync(0xffffffffu, sum[j], o);
+                }
+                if ((lane & (R - 1)) == 0 && k >= 0) {
+                    const int t0 = n0 + cb * 32;
+                    int32_t *y = Y + (size_t)k * T + t0;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        long long z = sum[j] >> p;   // arithmetic shift: floor division by 2^p
+                        z = z > 2147483647LL ? 2147483647LL : (z < -2147483648LL ? -2147483648LL : z);
+                        if (t0 + j < T) y[j] = (int32_t)z;
+                    }
+                }
+            }
+        }
+    } else if (warp == L_MMA_WARP) {
+        // ---------------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(L_M, L_N);
+            for (int kc = 0; kc < n_kc; ++kc) {
+                const int s = kc % L_STAGES;
+                const uint32_t ph = (uint32_t)(kc / L_STAGES) & 1u;
+                if (!mbar_wait(&ctl.full[s], ph, L_WAIT)) *abort_flag = 1;
+                if (*abort_flag) break;
+                tc_fence_after();
+                const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
+                const uint64_t ad = smem_desc_sw128(sb);
+                const uint64_t bd = smem_desc_sw128(sb + L_OFF_B);
+#pragma unroll
+                for (int kk = 0; kk < L_KC / 16; ++kk) {
+                    const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
+                    mma_bf16(tmem, ad + o, bd + o, idesc, (kc > 0 || kk > 0) ? 1u : 0u);
+                }
+                mma_commit(&ctl.empty[s]);
+            }
+            mma_commit(&ctl.done);
+        }
+        __syncwarp();
+    } else {
+        // ---------------------------------------------------------------- TMA: codes and inputs
+        if (lane == 0) {
+            prefetch_tensormap(&tmA);
+            prefetch_tensormap(&tmX);
+            int issued = 0;
+            for (int kc = 0; kc < n_kc; ++kc) {
+                const int s = kc % L_STAGES;
+                if (kc >= L_STAGES &&
+                    !mbar_wait(&ctl.empty[s], (uint32_t)(kc / L_STAGES - 1) & 1u, L_WAIT))
+                    *abort_flag = 1;
+                if (*abort_flag) break;
+                const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
+                mbar_arrive_expect_tx(&ctl.loaded[s], L_A_BYTES + L_RAW_BYTES);
+                tma_load_2d(sb, &tmA, kc * L_KC, tile * L_M, &ctl.loaded[s]);
+                tma_load_2d(sb + L_OFF_RAW, &tmX, kc * L_KC, n0, &ctl.loaded[s]);
+                issued = kc + 1;
+            }
+            // no copy may land after the CTA is gone
+            for (int kc = issued - L_STAGES > 0 ? issued - L_STAGES : 0; kc < issued; ++kc)
+                mbar_wait(&ctl.loaded[kc % L_STAGES], (uint32_t)(kc / L_STAGES) & 1u, L_WAIT);
+        }
+        __syncwarp();
+    }
+
+    __syncthreads();
+    if (warp == L_MMA_WARP) {
+        // every MMA has completed: the epilogue waited for `done` (or the wait timed out)
+        if (lane == 0 && *abort_flag) mbar_wait(&ctl.done, 0, L_WAIT);
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, L_TMEM_COLS);
+    }
+}
+
+// The same integer arithmetic on CUDA cores: one thread per (channel, input).
+__global__ void multipoint_linear_simt(const int8_t *__restrict__ X, int T, int d, int d_pad, int rows,
+                                       int p, const int *__restrict__ coef,
+                                       const int *__restrict__ chan,
+                                       const __nv_bfloat16 *__restrict__ codes,
+                                       const int *__restrict__ tile_R, int32_t *__restrict__ Y)
+{
+    const size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x;
+    const int slot_row = (int)(idx / T), t = (int)(idx % T);   // slot_row: first row of a channel
+    if (slot_row >= rows) return;
+    const int R = tile_R[slot_row / L_M];
+    if (slot_row % R != 0) return;
+    const int k = chan[slot_row];
+    if (k < 0) return;
+    const int8_t *x = X + (size_t)t * d;
+    long long sum = 0;
+    for (int i = 0; i < R; ++i) {
+        const int r = slot_row + i;
+        const __nv_bfloat16 *q = codes + (size_t)r * d_pad;
+        long long acc = 0;
+        for (int j = 0; j < d; ++j) acc += (long long)__bfloat162float(q[j]) * (long long)x[j];
+        sum += (long long)coef[r] * acc;
+    }
+    long long z = sum >> p;
+    z = z > 2147483647LL ? 2147483647LL : (z < -2147483648LL ? -2147483648LL : z);
+    Y[(size_t)k * T + t] = (int32_t)z;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 lin_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+        return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+    }();
+    return fn;
+}
+
+int pow2_at_least(int n)
+{
+    int r = 1;
+    while (r < n) r <<= 1;
+    return r;
+}
+
+}  // namespace
+
+mpq_status make_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
+                            mpq_packed_layout *L)
+{
+    memset(L, 0, sizeof(*L));
+    L->C = C;
+    L->d = d;
+    L->k_max = k_max;
+    L->bits = bits;
+    L->p = p;
+    L->d_pad = (d + L_KC - 1) / L_KC * L_KC;
+    long long tiles = 0;
+    for (int R = 1; R <= MPQ_MAX_POINTS; R <<= 1) {
+        long long n = 0;
+        for (int k = 0; k < C; ++k) {
+            int nk = npoints[k] < 0 ? 0 : (npoints[k] > k_max ? k_max : npoints[k]);
+            if (pow2_at_least(nk < 1 ? 1 : nk) == R) ++n;
+        }
+        tiles += (n + (L_M / R) - 1) / (L_M / R);
+    }
+    if (tiles * L_M > (1LL << 30)) {
+        set_error("packed layer too large");
+        return MPQ_ERR_UNSUPPORTED;
+    }
+    L->tiles = (int)tiles;
+    L->rows = (int)(tiles * L_M);
+    size_t off = 64;
+    L->off_coef = off;
+    off += (size_t)L->rows * 4;
+    L->off_chan = off;
+    off += (size_t)L->rows * 4;
+    L->off_point = off;
+    off += (size_t)L->rows * 4;
+    L->off_tile = off;
+    off += (size_t)L->tiles * 4;
+    off = (off + 1023) / 1024 * 1024;
+    L->off_codes = off;
+    off += (size_t)L->rows * L->d_pad * 2;
+    L->bytes = off;
+    return MPQ_OK;
+}
+
+mpq_status launch_pack(const int8_t *codes, const float *scales, const int *npoints,
+                       const mpq_packed_layout *L, void *packed, cudaStream_t stream)
+{
+    const int C = L->C, rows = L->rows;
+    std::vector<int> chan((size_t)rows, -1), point((size_t)rows, -1), tR((size_t)L->tiles, 1);
+    int t = 0;
+    for (int R = 1; R <= MPQ_MAX_POINTS; R <<= 1) {
+        int slot = 0, per = L_M / R;
+        for (int k = 0; k < C; ++k) {
+            int nk = npoints[k] < 0 ? 0 : (npoints[k] > L->k_max ? L->k_max : npoints[k]);
+            if (pow2_at_least(nk < 1 ? 1 : nk) != R) continue;
+            if (slot == per) {
+                slot = 0;
+                ++t;
+            }
+            tR[(size_t)t] = R;
+            for (int i = 0; i < R; ++i) {
+                const size_t r = (size_t)t * L_M + (size_t)slot * R + i;
+                chan[r] = (i == 0 || i < nk) ? k : -1;   // the first row carries the channel
+                point[r] = i < nk ? i : -1;
+            }
+            ++slot;
+        }
+        if (slot > 0) ++t;
+    }
+    if (t != L->tiles) {
+        set_error("npoints differ from the ones the layout was made for");
+        return MPQ_ERR_INVALID_ARG;
+    }
+    PackView v = view(L, packed);
+    cudaError_t e = cudaMemsetAsync(packed, 0, 64, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(v.chan, chan.data(), (size_t)rows * 4, cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(v.point, point.data(), (size_t)rows * 4, cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(v.tile_R, tR.data(), (size_t)L->tiles * 4, cudaMemcpyHostToDevice,
+                            stream);
+    if (e != cudaSuccess) return cuda_status(e, "packing copies");
+    if (rows > 0) {
+        pack_kernel<<<rows, 256, 0, stream>>>(codes, scales, C, L->d, L->d_pad, L->k_max, L->p, rows,
+                                              v);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_status(e, "pack kernel launch");
+    }
+    int flag = 0;
+    e = cudaMemcpyAsync(&flag, v.flag, sizeof(int), cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);   // host arrays above must outlive the copies
+    if (e != cudaSuccess) return cuda_status(e, "packing");
+    if (flag) {
+        set_error("a coefficient rint(2^p * s) does not fit 32 bits (p = %d)", L->p);
+        return MPQ_ERR_UNSUPPORTED;
+    }
+    return MPQ_OK;
+}
+
+mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout *L,
+                                    const void *packed, int32_t *Y, cudaStream_t stream)
+{
+    PackView v = view(L, const_cast<void *>(packed));
+    const int d = L->d, qmax = (1 << (L->bits - 1)) - 1;
+    const bool exact = (double)d * qmax * 128.0 < 16777216.0;
+    const bool tma = exact && d % 16 == 0 && (uintptr_t)X % 16 == 0 && L->rows > 0;
+    if (tma) {
+        PFN_cuTensorMapEncodeTiled_v12000 enc = lin_map_encoder();
+        CUtensorMap tmA, tmX;
+        memset(&tmA, 0, sizeof(tmA));
+        memset(&tmX, 0, sizeof(tmX));
+        const cuuint64_t da[2] = {(cuuint64_t)L->d_pad, (cuuint64_t)L->rows};
+        const cuuint64_t sa[1] = {(cuuint64_t)L->d_pad * 2};
+        const cuuint32_t ba[2] = {L_KC, L_M};
+        const cuuint64_t dx[2] = {(cuuint64_t)d, (cuuint64_t)T};
+        const cuuint64_t sx[1] = {(cuuint64_t)d};
+        const cuuint32_t bx[2] = {L_KC, L_N};
+        const cuuint32_t es[2] = {1, 1};
+        if (!enc ||
+            enc(&tmA, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, v.codes, da, sa, ba, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
+            enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t *>(X), dx, sx, bx, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
+            set_error("multipoint linear: tensor map encoding failed");
+            return MPQ_ERR_CUDA;
+        }
+        if ((long long)L_SMEM > max_smem_optin()) {
+            set_error("multipoint linear needs %d bytes of shared memory", L_SMEM);
+            return MPQ_ERR_UNSUPPORTED;
+        }
+        cudaError_t e = cudaFuncSetAttribute(multipoint_linear_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, L_SMEM);
+        if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
+        const dim3 grid((unsigned)L->tiles, (unsigned)((T + L_N - 1) / L_N));
+        multipoint_linear_kernel<<<grid, L_THREADS, L_SMEM, stream>>>(
+            T, L->d_pad / L_KC, L->p, v.coef, v.chan, v.tile_R, Y, tmA, tmX);
+        return cuda_status(cudaGetLastError(), "multipoint linear kernel launch");
+    }
+    const size_t n = (size_t)L->rows * T;
+    if (n == 0) return MPQ_OK;
+    multipoint_linear_simt<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(
+        X, T, d, L->d_pad, L->rows, L->p, v.coef, v.chan, v.codes, v.tile_R, Y);
+    return cuda_status(cudaGetLastError(), "multipoint linear (integer) kernel launch");
+}
+
+}  // namespace mpq

@@ -154,6 +154,18 @@ __device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a_desc, uint6
         : "memory");
 }
 
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 with bf16 A and B (fp32 accumulate), one thread.
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                         uint32_t idesc, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // CTA-pair MMA, issued by one thread of the pair's even CTA: A is M = 256 rows, 128 in each CTA's
 // shared memory at the descriptor's offset; B is N rows, N/2 in each CTA; D lands in each CTA's
 // tensor memory (its own 128 rows x N columns) at d_tmem.
@@ -322,6 +334,16 @@ __device__ __forceinline__ uint32_t ld_shared_u16(uint32_t addr)
     uint16_t v;
     asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(addr) : "memory");
     return v;
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulate, A and B bf16, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N)
+{
+    return (1u << 4)                      // D format: f32
+           | (1u << 7)                    // A format: bf16
+           | (1u << 10)                   // B format: bf16
+           | ((uint32_t)(N >> 3) << 17)   // N / 8
+           | ((uint32_t)(M >> 4) << 24);  // M / 16
 }
 
 // ---- clusters --------------------------------------------------------------------------------

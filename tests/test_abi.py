@@ -122,3 +122,38 @@ def test_clip_search_validation(lib, kwargs, status):
 
 def test_clip_search_empty_layer(lib):
     assert lib.mpq_clip_search(None, 8, 1, None, 0, 16, 4, 20, 1, None, None, None, None) == 0
+
+
+def test_pack_layout_groups_channels(lib):
+    """Host-only layout: channels grouped by the power of two >= n_k (n_k = 0 takes one row), 128/R
+    channels per 128-row tile, rows padded to 64 elements, byte offsets in order."""
+    assert ctypes.sizeof(binding.PackedLayout) == 8 * 4 + 6 * 8
+    npts = [1] * 200 + [2] * 70 + [3] * 5 + [0] * 3 + [16]
+    lay = binding.mpq_pack_layout(npts, 100, 16, 4, 12)
+    tiles = -(-203 // 128) + -(-70 // 64) + -(-5 // 32) + 1   # R = 1, 2, 4, 16
+    assert (lay.C, lay.d, lay.d_pad, lay.tiles, lay.rows) == (279, 100, 128, tiles, 128 * tiles)
+    assert lay.off_coef < lay.off_chan < lay.off_point < lay.off_tile < lay.off_codes < lay.bytes
+    assert lay.off_codes % 1024 == 0
+    assert lay.bytes == lay.off_codes + lay.rows * lay.d_pad * 2
+
+
+@pytest.mark.parametrize("kwargs,status", [
+    (dict(p=31), 1), (dict(p=-1), 1), (dict(bits=1), 1), (dict(bits=9), 3), (dict(k_max=17), 3),
+    (dict(d=0), 1), (dict(npoints=None), 1), (dict(layout=None), 1),
+])
+def test_pack_layout_validation(lib, kwargs, status):
+    n = (ctypes.c_int * 3)(1, 2, 3)
+    lay = binding.PackedLayout()
+    a = dict(npoints=n, C=3, d=32, k_max=4, bits=4, p=12, layout=ctypes.byref(lay))
+    a.update(kwargs)
+    assert lib.mpq_pack_layout(a["npoints"], a["C"], a["d"], a["k_max"], a["bits"], a["p"],
+                               a["layout"]) == status
+
+
+def test_pack_and_linear_validation(lib):
+    lay = binding.mpq_pack_layout([1, 2], 32, 4, 4, 12)
+    assert lib.mpq_pack_points(None, FAKE, FAKE, ctypes.byref(lay), FAKE, None) == 1
+    assert lib.mpq_pack_points(FAKE, FAKE, FAKE, None, FAKE, None) == 1
+    assert lib.mpq_multipoint_linear(FAKE, 0, ctypes.byref(lay), FAKE, FAKE, None) == 1
+    assert lib.mpq_multipoint_linear(None, 4, ctypes.byref(lay), FAKE, FAKE, None) == 1
+    assert lib.mpq_multipoint_linear(FAKE, 4, None, FAKE, FAKE, None) == 1
