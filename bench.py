@@ -60,9 +60,11 @@ def parse():
                     help="comma-separated layer indices to run (profiling a subset); default all")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
-    ap.add_argument("--op", default="quantize", choices=["quantize", "clip"],
+    ap.add_argument("--op", default="quantize", choices=["quantize", "clip", "infer"],
                     help="quantize: the multipoint path (Algorithm 1, Eq. 11, Algorithm 2, Eq. 4); "
-                         "clip: the output-error-driven clipping factor search (Eq. 12)")
+                         "clip: the output-error-driven clipping factor search (Eq. 12); "
+                         "infer: integer inference with the packed multipoint weights (Eq. 13)")
+    ap.add_argument("--coef-bits", type=int, default=16, help="p of Eq. 13 for --op infer")
     ap.add_argument("--clip-candidates", type=int, default=20,
                     help="clipping factor candidates (c+1)/n x max|w| for --op clip")
     return ap.parse_args()
@@ -708,6 +710,190 @@ def run_clip(args, world, rank, local):
     return out if rank == 0 else None
 
 
+INFER_METRIC = "multipoint integer MACs / s"
+INFER_UNIT = "MAC/s"
+
+
+def infer_layers(args, wl, dev):
+    """Per layer: quantize, output error and budget allocation on the device (not timed), the
+    packed layer, and int8 inputs (T = the workload's calibration rows)."""
+    import torch
+    from paper_2002_09049_gb300 import binding
+    keep = None if args.layers is None else {int(x) for x in args.layers.split(",")}
+    out = []
+    for li, layer in enumerate(wl.layers):
+        if keep is not None and li not in keep:
+            continue
+        W, X = layer_inputs(wl, li)
+        Wd, Xd = torch.from_numpy(W).to(dev), torch.from_numpy(X).to(dev)
+        codes, scales, _, _ = binding.mpq_quantize_layer(Wd, wl.bits[0], wl.G, wl.k_max)
+        err = binding.mpq_output_error(Xd, Wd, codes, scales, wl.k_max,
+                                       groups=layer.C if layer.groups > 1 else 1)
+        npts, _ = binding.mpq_allocate_points(err, wl.k_max, binding.MPQ_ALLOC_BUDGET, wl.beta)
+        n_host = npts.cpu().numpy()
+        lay = binding.mpq_pack_layout(n_host, layer.d, wl.k_max, wl.bits[0], args.coef_bits)
+        packed = binding.mpq_pack_points(codes, scales, n_host, lay)
+        Xq = np.random.default_rng(900000 + li).integers(-128, 128, (wl.n_calib, layer.d))
+        Xh = torch.from_numpy(Xq.astype(np.int8)).pin_memory()
+        out.append(dict(layer=layer, lay=lay, packed=packed, Xh=Xh, X=Xh.to(dev),
+                        Y=torch.empty((layer.C, wl.n_calib), dtype=torch.int32, device=dev),
+                        macs=int(n_host.sum()) * layer.d * wl.n_calib,
+                        codes=codes.cpu().numpy(), scales=scales.cpu().numpy(), n=n_host, Xq=Xq))
+    return out
+
+
+def run_infer(args, world, rank, local):
+    """Eq. 13 over every layer: mpq_multipoint_linear on the packed layers, layers on streams."""
+    import torch
+    from paper_2002_09049_gb300 import _build, binding
+    from paper_2002_09049_gb300 import dist as dist_helpers
+    from paper_2002_09049_gb300 import workloads as wlm
+
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0 or world == 1:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    binding.load()
+    wl = wlm.WORKLOADS[args.config]
+    L = infer_layers(args, wl, dev)
+    order = sorted(range(len(L)), key=lambda i: -L[i]["macs"])
+    streams = [torch.cuda.Stream(dev) for _ in range(max(1, args.streams))]
+    main = torch.cuda.current_stream()
+    macs = sum(x["macs"] for x in L)
+    mma_macs = sum(x["lay"].rows * x["layer"].d * wl.n_calib for x in L)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+
+    def call(i, st):
+        x = L[i]
+        binding.mpq_multipoint_linear(x["X"], x["lay"], x["packed"], Y=x["Y"], stream=st)
+
+    def step():
+        ev = torch.cuda.Event()
+        ev.record(main)
+        for st in streams:
+            st.wait_event(ev)
+        for n, i in enumerate(order):
+            call(i, streams[n % len(streams)])
+        for st in streams:
+            e = torch.cuda.Event()
+            e.record(st)
+            main.wait_event(e)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    peaks, peak_src = measured_peaks()
+    step_ms = []
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            a = torch.cuda.Event(enable_timing=True)
+            z = torch.cuda.Event(enable_timing=True)
+            a.record(main)
+            step()
+            z.record(main)
+            torch.cuda.synchronize()
+            step_ms.append(a.elapsed_time(z))
+    one_ms = []
+    for _ in range(args.steps):
+        flush.fill_(1.0)
+        a = torch.cuda.Event(enable_timing=True)
+        z = torch.cuda.Event(enable_timing=True)
+        a.record(main)
+        for i in order:
+            call(i, main)
+        z.record(main)
+        torch.cuda.synchronize()
+        one_ms.append(a.elapsed_time(z))
+    if world > 1:
+        torch.distributed.barrier()
+    ms = dist_helpers.max_over_ranks(float(np.mean(step_ms)), device=dev)
+    value = dist_helpers.aggregate_throughput(macs, ms, world)
+    t1 = float(np.mean(one_ms)) / 1e3
+    peak = peaks["bf16_tflops"]
+    ach = 2.0 * macs / t1 / 1e12
+    roofline = {"kernel": "multipoint_linear_kernel (Eq. 13 step 1 on tcgen05 kind::f16 bf16, "
+                          "steps 2-3 in the epilogue)",
+                "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                "frac": ach / peak, "traffic": None,
+                "peak_source": f"{peak_src} bf16 dense burst",
+                "timing": "all layers on one stream, CUDA events; achieved = 2 x the multipoint "
+                          "MACs (used points only) / that time",
+                "packed_row_macs_per_used_mac": mma_macs / macs,
+                "single_stream_ms_per_step": t1 * 1e3}
+    out = {"metric": INFER_METRIC, "value": value, "unit": INFER_UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int8 x int4",
+           "data": "synthetic",
+           "config": {"workload": f"{args.config}: {wl.title}", "op": "infer (Eq. 13)",
+                      "layers": len(L), "inputs_per_layer": wl.n_calib, "p": args.coef_bits,
+                      "points": f"budget {wl.beta} per channel (Algorithm 2)",
+                      "macs_per_step": macs, "l2": "flushed between steps (512 MB write)",
+                      "streams": args.streams, "parallelism": f"replicas x{world}"},
+           "roofline": roofline, "gpu_launches": len(L) * args.steps, "clocks": clk.summary()}
+    if not args.no_e2e:
+        def e2e_step():
+            ev = torch.cuda.Event()
+            ev.record(main)
+            for st in streams:
+                st.wait_event(ev)
+            host = []
+            for n, i in enumerate(order):
+                st = streams[n % len(streams)]
+                with torch.cuda.stream(st):
+                    L[i]["X"].copy_(L[i]["Xh"], non_blocking=True)
+                    call(i, st)
+                    host.append(L[i]["Y"].to("cpu", non_blocking=True))
+            for st in streams:
+                e = torch.cuda.Event()
+                e.record(st)
+                main.wait_event(e)
+        for _ in range(max(1, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize()
+        tms = []
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            e2e_step()
+            torch.cuda.synchronize()
+            tms.append((time.perf_counter() - t0) * 1e3)
+        e_ms = float(np.mean(tms))
+        out["e2e"] = {"value": macs / (e_ms / 1e3), "unit": INFER_UNIT, "ms_per_step": e_ms,
+                      "h2d_bytes_per_step": sum(x["Xh"].numel() for x in L),
+                      "d2h_bytes_per_step": sum(x["Y"].numel() * 4 for x in L)}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        t0 = time.perf_counter()
+        units = 0
+        for x in L:   # a channel sample of every layer, bounded to about --cpu-seconds
+            C = x["layer"].C
+            per_ch = x["macs"] / max(1, C) * 1.5e-9
+            nc = max(1, min(C, int(args.cpu_seconds / len(L) / max(per_ch, 1e-12)) * host_cores()))
+            oracle.multipoint_linear(x["Xq"].astype(np.int8), x["codes"], x["scales"], x["n"],
+                                     args.coef_bits, channels=(0, nc), threads=host_cores())
+            units += int(x["n"][:nc].sum()) * x["layer"].d * wl.n_calib
+        dt = time.perf_counter() - t0
+        out["cpu_baseline"] = {"value": units / dt, "unit": INFER_UNIT, "cores": host_cores(),
+                               "kind": "oracle", "seconds": dt,
+                               "sample": f"the first channels of every layer ({units:.3e} MACs), "
+                                         "oracle threads over channels"}
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    return out if rank == 0 else None
+
+
 def run_clip_reference(args, world, rank):
     """The oracle's Eq. 12 search as the reference arm of --op clip, on the host cores."""
     if rank != 0:
@@ -746,9 +932,16 @@ def main():
     args = parse()
     world, rank, local = dist_setup(args)
     if args.impl == "reference":
-        out = (run_clip_reference if args.op == "clip" else run_reference)(args, world, rank)
+        if args.op == "infer":
+            out = {"impl": "reference", "op": "infer",
+                   "unavailable": "the integer inference path needs the device-quantized layers; "
+                                  "its oracle is timed as cpu_baseline of --op infer"}
+        else:
+            out = (run_clip_reference if args.op == "clip" else run_reference)(args, world, rank)
     elif args.op == "clip":
         out = run_clip(args, world, rank, local)
+    elif args.op == "infer":
+        out = run_infer(args, world, rank, local)
     else:
         out = run_ours(args, world, rank, local)
     if out is not None:
