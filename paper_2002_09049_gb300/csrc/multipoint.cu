@@ -15,7 +15,10 @@
 // into bf16 exactly by eight producer warps through the fp32 exponent bias).  Products are exact
 // and every partial sum is an integer of magnitude below 2^24 when d * Qmax * 128 < 2^24, so the
 // fp32 accumulator holds the exact dot products (checked on the host; other layers take the
-// integer kernel below).  Tile: 128 packed rows x 256 inputs, K chunks of 64, 3 stages.
+// integer kernel below).  A CTA takes RT 128-row tiles against 256 inputs (RT accumulators of 256
+// TMEM columns): two on large layers, so each converted input tile feeds both, one on small layers
+// for more CTAs; K chunks of 64.  The inputs vary fastest in the grid, so the CTAs that share a row
+// tile run together and read its codes from L2.
 // Steps 2 and 3 in the epilogue: each lane turns its accumulator into an integer, multiplies by its
 // row's coefficient in 64 bits, the R lanes of a channel add with warp shuffles, and the first lane
 // shifts (arithmetic: floor), saturates and writes 32 consecutive outputs.  Every wait is bounded.
@@ -42,33 +45,40 @@ using namespace sm100;
 constexpr int L_M = 128;                        // packed rows per tile (TMEM lanes)
 constexpr int L_N = 256;                        // inputs per tile (UMMA N)
 constexpr int L_KC = 64;                        // bf16 per K chunk = one 128-byte swizzle row
-constexpr int L_STAGES = 3;
 constexpr int L_A_BYTES = L_M * L_KC * 2;       // 16 KB codes tile
 constexpr int L_B_BYTES = L_N * L_KC * 2;       // 32 KB input tile (bf16)
 constexpr int L_RAW_BYTES = L_N * L_KC;         // 16 KB input tile (int8, as loaded)
-constexpr int L_OFF_B = L_A_BYTES;
-constexpr int L_OFF_RAW = L_A_BYTES + L_B_BYTES;
-constexpr int L_STAGE_BYTES = L_A_BYTES + L_B_BYTES + L_RAW_BYTES;   // 64 KB
+constexpr int L_MAX_RT = 2;
+
+// Stage layout for RT row tiles per CTA: RT codes tiles, the bf16 input tile, the raw input tile.
+template <int RT>
+struct LGeo {
+    static constexpr int STAGES = RT == 1 ? 3 : 2;
+    static constexpr int OFF_B = RT * L_A_BYTES;
+    static constexpr int OFF_RAW = OFF_B + L_B_BYTES;
+    static constexpr int STAGE_BYTES = OFF_RAW + L_RAW_BYTES;   // 64 or 80 KB
+    static constexpr uint32_t TMEM_COLS = RT * L_N;
+};
 constexpr int L_PROD_WARPS = 8;
 constexpr int L_PROD_THREADS = L_PROD_WARPS * 32;
 constexpr int L_EPI_WARP0 = L_PROD_WARPS;       // warps 8..11: warp % 4 selects TMEM lanes
 constexpr int L_MMA_WARP = L_EPI_WARP0 + 4;
 constexpr int L_TMA_WARP = L_MMA_WARP + 1;
 constexpr int L_THREADS = (L_TMA_WARP + 1) * 32;   // 448
-constexpr uint32_t L_TMEM_COLS = 256;
 constexpr long long L_WAIT = 1LL << 31;
 
 struct LinCtrl {
-    uint64_t loaded[L_STAGES];    // TMA bytes of a stage have landed
-    uint64_t full[L_STAGES];      // producers converted the input tile
-    uint64_t empty[L_STAGES];     // MMAs on the stage completed
+    uint64_t loaded[3];           // TMA bytes of a stage have landed
+    uint64_t full[3];             // producers converted the input tile
+    uint64_t empty[3];            // MMAs on the stage completed
     uint64_t done;                // every MMA completed
     uint32_t tmem_base;
     int abort;
-    int coef[L_M];                // this tile's row coefficients A
+    int coef[L_MAX_RT][L_M];      // the row coefficients A of this CTA's tiles
 };
 constexpr int L_CTRL_BYTES = (sizeof(LinCtrl) + 1023) / 1024 * 1024;
-constexpr int L_SMEM = 1024 + L_CTRL_BYTES + L_STAGES * L_STAGE_BYTES;
+template <int RT>
+constexpr int lin_smem() { return 1024 + L_CTRL_BYTES + LGeo<RT>::STAGES * LGeo<RT>::STAGE_BYTES; }
 
 // Row r of a packed buffer: (channel, point) or channel -1 / point -1 for padding.
 struct PackView {
@@ -122,12 +132,20 @@ __device__ __forceinline__ uint32_t bf16x2_from_biased(uint32_t biased, int b0)
     return __byte_perm(lo, hi, 0x7632u);
 }
 
+template <int RT>
 __global__ void __launch_bounds__(L_THREADS, 1)
-multipoint_linear_kernel(int T, int n_kc, int p, const int *__restrict__ coef,
+multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restrict__ coef,
                          const int *__restrict__ chan, const int *__restrict__ tile_R,
                          int32_t *__restrict__ Y, const __grid_constant__ CUtensorMap tmA,
                          const __grid_constant__ CUtensorMap tmX)
 {
+    using G = LGeo<RT>;
+    constexpr int L_STAGES = G::STAGES;
+    constexpr int L_STAGE_BYTES = G::STAGE_BYTES;
+    constexpr int L_OFF_B = G::OFF_B;
+    constexpr int L_OFF_RAW = G::OFF_RAW;
+    constexpr uint32_t L_TMEM_COLS = G::TMEM_COLS;
+    constexpr int L_RT = RT;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
@@ -135,7 +153,9 @@ multipoint_linear_kernel(int T, int n_kc, int p, const int *__restrict__ coef,
     const uint32_t stages_u32 = raw_u32 + pad + L_CTRL_BYTES;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tile = blockIdx.x, n0 = blockIdx.y * L_N;
+    // inputs vary fastest: the CTAs sharing a row tile run together and read its codes from L2
+    const int tile0 = blockIdx.y * L_RT, n0 = blockIdx.x * L_N;
+    const int nt = min(L_RT, tiles - tile0);        // row tiles of this CTA (the last may hold one)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < L_STAGES; ++s) {
@@ -147,7 +167,8 @@ multipoint_linear_kernel(int T, int n_kc, int p, const int *__restrict__ coef,
         ctl.abort = 0;
         fence_barrier_init();
     }
-    for (int r = threadIdx.x; r < L_M; r += L_THREADS) ctl.coef[r] = coef[(size_t)tile * L_M + r];
+    for (int r = threadIdx.x; r < L_RT * L_M; r += L_THREADS)
+        ctl.coef[r / L_M][r % L_M] = r / L_M < nt ? coef[(size_t)tile0 * L_M + r] : 0;
     if (warp == L_MMA_WARP) {
         tmem_alloc(&ctl.tmem_base, L_TMEM_COLS);
         tc_fence_before();
@@ -199,12 +220,12 @@ multipoint_linear_kernel(int T, int n_kc, int p, const int *__restrict__ coef,
         if (!ok) *abort_flag = 1;
         const bool good = !__any_sync(0xffffffffu, !ok || *abort_flag);
         tc_fence_after();
-        const int R = tile_R[tile];
-        const int r = ew * 32 + lane;
-        const int k = chan[(size_t)tile * L_M + r];
-        const long long a = ctl.coef[r];
-        const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16);
-        if (good) {
+        for (int u = 0; u < nt && good; ++u) {
+            const int R = tile_R[tile0 + u];
+            const int r = ew * 32 + lane;
+            const int k = chan[(size_t)(tile0 + u) * L_M + r];
+            const long long a = ctl.coef[u][r];
+            const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16) + (uint32_t)(u * L_N);
 #pragma unroll 1
             for (int cb = 0; cb < L_N / 32; ++cb) {
                 float v[32];
@@ -239,12 +260,15 @@ multipoint_linear_kernel(int T, int n_kc, int p, const int *__restrict__ coef,
                 if (*abort_flag) break;
                 tc_fence_after();
                 const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
-                const uint64_t ad = smem_desc_sw128(sb);
                 const uint64_t bd = smem_desc_sw128(sb + L_OFF_B);
+                for (int u = 0; u < nt; ++u) {
+                    const uint64_t ad = smem_desc_sw128(sb + u * L_A_BYTES);
 #pragma unroll
-                for (int kk = 0; kk < L_KC / 16; ++kk) {
-                    const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
-                    mma_bf16(tmem, ad + o, bd + o, idesc, (kc > 0 || kk > 0) ? 1u : 0u);
+                    for (int kk = 0; kk < L_KC / 16; ++kk) {
+                        const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
+                        mma_bf16(tmem + (uint32_t)(u * L_N), ad + o, bd + o, idesc,
+                                 (kc > 0 || kk > 0) ? 1u : 0u);
+                    }
                 }
                 mma_commit(&ctl.empty[s]);
             }
@@ -264,8 +288,10 @@ multipoint_linear_kernel(int T, int n_kc, int p, const int *__restrict__ coef,
                     *abort_flag = 1;
                 if (*abort_flag) break;
                 const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
-                mbar_arrive_expect_tx(&ctl.loaded[s], L_A_BYTES + L_RAW_BYTES);
-                tma_load_2d(sb, &tmA, kc * L_KC, tile * L_M, &ctl.loaded[s]);
+                mbar_arrive_expect_tx(&ctl.loaded[s], (uint32_t)(nt * L_A_BYTES + L_RAW_BYTES));
+                for (int u = 0; u < nt; ++u)
+                    tma_load_2d(sb + u * L_A_BYTES, &tmA, kc * L_KC, (tile0 + u) * L_M,
+                                &ctl.loaded[s]);
                 tma_load_2d(sb + L_OFF_RAW, &tmX, kc * L_KC, n0, &ctl.loaded[s]);
                 issued = kc + 1;
             }
@@ -463,16 +489,21 @@ mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_lay
             set_error("multipoint linear: tensor map encoding failed");
             return MPQ_ERR_CUDA;
         }
-        if ((long long)L_SMEM > max_smem_optin()) {
-            set_error("multipoint linear needs %d bytes of shared memory", L_SMEM);
+        // two row tiles per CTA when that still gives at least two waves of CTAs
+        const long long tt = (T + L_N - 1) / L_N;
+        const bool two = (long long)((L->tiles + 1) / 2) * tt >= 2LL * sm_count();
+        const int smem = two ? lin_smem<2>() : lin_smem<1>();
+        if ((long long)smem > max_smem_optin()) {
+            set_error("multipoint linear needs %d bytes of shared memory", smem);
             return MPQ_ERR_UNSUPPORTED;
         }
-        cudaError_t e = cudaFuncSetAttribute(multipoint_linear_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, L_SMEM);
+        auto kernel = two ? multipoint_linear_kernel<2> : multipoint_linear_kernel<1>;
+        cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
-        const dim3 grid((unsigned)L->tiles, (unsigned)((T + L_N - 1) / L_N));
-        multipoint_linear_kernel<<<grid, L_THREADS, L_SMEM, stream>>>(
-            T, L->d_pad / L_KC, L->p, v.coef, v.chan, v.tile_R, Y, tmA, tmX);
+        const int rt = two ? 2 : 1;
+        const dim3 grid((unsigned)tt, (unsigned)((L->tiles + rt - 1) / rt));
+        kernel<<<grid, L_THREADS, smem, stream>>>(T, L->tiles, L->d_pad / L_KC, L->p, v.coef,
+                                                  v.chan, v.tile_R, Y, tmA, tmX);
         return cuda_status(cudaGetLastError(), "multipoint linear kernel launch");
     }
     const size_t n = (size_t)L->rows * T;
