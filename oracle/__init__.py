@@ -58,7 +58,9 @@ def _load():
         lib.mpqo_allocate_budget.restype = L
         lib.mpqo_allocate_threshold.argtypes = [P, I, I, D, P]
         lib.mpqo_allocate_threshold.restype = L
-        lib.mpqo_reconstruct.argtypes = [P, P, P, I, I, I, P]
+        lib.mpqo_reconstruct.argtypes = [P, P, P, P, I, I, I, P]
+        lib.mpqo_center.argtypes = [P, I, I, I, P, P]
+        lib.mpqo_center.restype = None
         lib.mpqo_reconstruct.restype = None
         lib.mpqo_clip_candidates.argtypes = [P, I, I, I, I, P]
         lib.mpqo_clip_candidates.restype = None
@@ -68,7 +70,7 @@ def _load():
         lib.mpqo_clip_select.restype = None
         lib.mpqo_fixed_coeff.argtypes = [ctypes.c_float, I, P]
         lib.mpqo_fixed_coeff.restype = ctypes.c_longlong
-        lib.mpqo_multipoint_linear.argtypes = [P, I, P, P, P, I, I, I, I, P, I, I]
+        lib.mpqo_multipoint_linear.argtypes = [P, I, P, P, P, P, I, I, I, I, P, I, I]
         lib.mpqo_multipoint_linear.restype = I
         _lib = lib
     return _lib
@@ -177,16 +179,34 @@ def allocate_threshold(err32, k_max: int, eps: float):
     return n, int(used)
 
 
-def reconstruct(codes, scales, npoints):
-    """Eq. 4: w~_k = sum_{i<=n_k} s_{k,i} q_{k,i} (fmaf chain from 0)."""
+def reconstruct(codes, scales, npoints, center=None):
+    """Eq. 4: w~_k = B_k + sum_{i<=n_k} s_{k,i} q_{k,i} (fmaf chain from the centre B_k, or 0)."""
     lib = _load()
     codes = _c(codes, np.int8)
     scales = _c(scales, np.float32)
     npoints = _c(npoints, np.int32)
     k_max, C, d = codes.shape
+    cen = None if center is None else _c(center, np.float32)
     W_hat = np.zeros((C, d), np.float32)
-    lib.mpqo_reconstruct(_p(codes), _p(scales), _p(npoints), C, d, k_max, _p(W_hat))
+    lib.mpqo_reconstruct(_p(codes), _p(scales), _p(npoints), None if cen is None else _p(cen),
+                         C, d, k_max, _p(W_hat))
     return W_hat
+
+
+CENTER_PER_CHANNEL = 0
+CENTER_PER_LAYER = 1
+
+
+def center(W, mode: int):
+    """Eq. 1 with B != 0: the centre B per channel (mode 0) or per layer (mode 1) = the midpoint of
+    the weights' range in fp32, and the centred weights W - B (fp32)."""
+    lib = _load()
+    W = _c(W, np.float32)
+    C, d = W.shape
+    B = np.zeros(C, np.float32)
+    Wc = np.zeros((C, d), np.float32)
+    lib.mpqo_center(_p(W), C, d, mode, _p(B), _p(Wc))
+    return B, Wc
 
 
 CLIP_PER_CHANNEL = 0
@@ -242,9 +262,12 @@ def fixed_coeff(s: float, p: int):
     return int(a) if ok.value else None
 
 
-def multipoint_linear(X, codes, scales, npoints, p: int, channels=None, threads: int = 1):
-    """Sec. 3.4 steps 1-3: Y [C][T] int32 = sat32(floor(sum_i A_i (q_i . x_t) / 2^p)), exact."""
+def multipoint_linear(X, codes, scales, npoints, p: int, channels=None, threads: int = 1,
+                      center=None):
+    """Sec. 3.4 steps 1-3: Y [C][T] int32 = sat32(floor(sum_i A_i (q_i . x_t) / 2^p)), exact; with
+    a centre B (asymmetric set), A_B (sum_j x_tj) joins the sum, A_B = rint(2^p B)."""
     lib = _load()
+    cen = None if center is None else _c(center, np.float32)
     X = _c(X, np.int8)
     codes = _c(codes, np.int8)
     scales = _c(scales, np.float32)
@@ -256,8 +279,9 @@ def multipoint_linear(X, codes, scales, npoints, p: int, channels=None, threads:
     bad = []
 
     def run(rng):
-        if lib.mpqo_multipoint_linear(_p(X), T, _p(codes), _p(scales), _p(npoints), C, d, k_max,
-                                      p, _p(Y), rng[0], rng[1]):
+        if lib.mpqo_multipoint_linear(_p(X), T, _p(codes), _p(scales), _p(npoints),
+                                      None if cen is None else _p(cen), C, d, k_max, p, _p(Y),
+                                      rng[0], rng[1]):
             bad.append(rng)
 
     _parallel(run, [(a + c0, b + c0) for a, b in _ranges(c1 - c0, threads)], threads)

@@ -290,8 +290,8 @@ long mpqo_allocate_threshold(const float *err, int C, int k_max, double eps, int
 
 /* Eq. 4: w~_k = sum_{i=1..n_k} s_{k,i} q_{k,i}, accumulated as acc = fmaf(s_i, q_i, acc) from
  * acc = 0 in the order i = 1, 2, ...  n_k is clamped to [0, k_max]. */
-void mpqo_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C, int d,
-                      int k_max, float *W_hat)
+void mpqo_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
+                      const float *center, int C, int d, int k_max, float *W_hat)
 {
     long plane = (long)C * d;
     for (int k = 0; k < C; ++k) {
@@ -299,13 +299,55 @@ void mpqo_reconstruct(const int8_t *codes, const float *scales, const int *npoin
         if (n < 0) n = 0;
         if (n > k_max) n = k_max;
         for (int j = 0; j < d; ++j) {
-            float acc = 0.0f;
+            float acc = center ? center[k] : 0.0f;   /* the set's centre B (Eq. 1), 0 if symmetric */
             for (int i = 0; i < n; ++i)
                 acc = fmaf(scales[(long)k * k_max + i], (float)codes[(long)i * plane + (long)k * d + j],
                            acc);
             W_hat[(long)k * d + j] = acc;
         }
     }
+}
+
+/* ---- Eq. 1 with B != 0: asymmetric sets ---------------------------------------------------------
+ * The quantization set K x [-1 : eps_b : 1] + B has the centre B.  Per channel (mode 0) every
+ * channel has its own B; per layer (mode 1) one B serves all the layer's channels.  Readings (also
+ * in the design doc): B is the midpoint of the weights' range, (max w + min w) / 2 rounded once to fp32,
+ * so that K = (max w - min w) / 2 covers every weight without clipping (the per-channel
+ * experiments clip nothing); the multipoint approximation takes B once and approximates the
+ * centred weights w - B (one fp32 subtraction) with the greedy points, so that
+ * w~ = B + sum_i s_i q_i; a non-finite weight makes B NaN for its channel (per layer: for all). */
+void mpqo_center(const float *W, int C, int d, int mode, float *center, float *Wc)
+{
+    double lo = 0.0, hi = 0.0;
+    int bad = 0, seen = 0;
+    for (int k = 0; k < C; ++k) {
+        const float *w = W + (long)k * d;
+        double klo = 0.0, khi = 0.0;
+        int kbad = !all_finite(w, d);
+        for (int j = 0; j < d; ++j) {
+            double v = (double)w[j];
+            if (j == 0 || v < klo) klo = v;
+            if (j == 0 || v > khi) khi = v;
+        }
+        if (mode == 0) {
+            /* (hi + lo) / 2 is exact in double for two fp32 values of a weight range; one rounding */
+            center[k] = kbad ? NAN : (d > 0 ? (float)((khi + klo) * 0.5) : 0.0f);
+        } else if (d > 0) {
+            if (!seen || klo < lo) lo = klo;
+            if (!seen || khi > hi) hi = khi;
+            seen = 1;
+        }
+        bad |= kbad;
+    }
+    if (mode == 1) {
+        float b = bad ? NAN : (float)((hi + lo) * 0.5);
+        for (int k = 0; k < C; ++k) center[k] = b;
+    }
+    for (int k = 0; k < C; ++k)
+        for (int j = 0; j < d; ++j) {
+            float v = W[(long)k * d + j] - center[k];   /* one fp32 subtraction */
+            Wc[(long)k * d + j] = v;
+        }
 }
 
 /* ---- Eq. 12: output-error-driven clipping factor ------------------------------------------------
@@ -427,11 +469,13 @@ long long mpqo_fixed_coeff(float s, int p, int *ok)
     return (long long)v;
 }
 
-/* Y[k][t] for channels [c0, c1), X [T][d] int8, Y [C][T] int32.  Returns 0, or 1 if a coefficient
- * did not fit 32 bits (Y is then unspecified). */
+/* Y[k][t] for channels [c0, c1), X [T][d] int8, Y [C][T] int32.  With a centre B_k (asymmetric set,
+ * Eq. 1; center may be NULL), w~ = B_k 1 + sum_i s_i q_i and the centre adds A_B (sum_j x_j) with
+ * A_B = rint(2^p B_k) to the sum before the shift.  Returns 0, or 1 if a coefficient did not fit 32
+ * bits (Y is then unspecified). */
 int mpqo_multipoint_linear(const int8_t *X, int T, const int8_t *codes, const float *scales,
-                           const int *npoints, int C, int d, int k_max, int p, int32_t *Y, int c0,
-                           int c1)
+                           const int *npoints, const float *center, int C, int d, int k_max, int p,
+                           int32_t *Y, int c0, int c1)
 {
     long plane = (long)C * d;
     for (int k = c0; k < c1; ++k) {
@@ -444,9 +488,20 @@ int mpqo_multipoint_linear(const int8_t *X, int T, const int8_t *codes, const fl
             A[i] = mpqo_fixed_coeff(scales[(long)k * k_max + i], p, &ok);
             if (!ok) return 1;
         }
+        long long AB = 0;
+        if (center) {
+            int ok = 1;
+            AB = mpqo_fixed_coeff(center[k], p, &ok);
+            if (!ok) return 1;
+        }
         for (int t = 0; t < T; ++t) {
             const int8_t *x = X + (long)t * d;
             long long sum = 0;
+            if (center) {
+                long long xs = 0;
+                for (int j = 0; j < d; ++j) xs += (long long)x[j];
+                sum += AB * xs;                                     /* the centre's term */
+            }
             for (int i = 0; i < n; ++i) {
                 const int8_t *q = codes + (long)i * plane + (long)k * d;
                 long long acc = 0;                                  /* step 1 */

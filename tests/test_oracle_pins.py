@@ -482,3 +482,122 @@ def test_integer_inference_edges(oracle):
     assert oracle.multipoint_linear(X, codes, s, np.array([0], np.int32), 4)[0, 0] == 0
     y2 = oracle.multipoint_linear(X, codes, s, np.array([2], np.int32), 4)
     assert np.array_equal(oracle.multipoint_linear(X, codes, s, np.array([9], np.int32), 4), y2)
+
+
+# ---- Eq. 1 with B != 0: asymmetric (centred) sets ---------------------------------------------------
+
+def _round_f32(v: Fraction) -> np.float32:
+    """Correct rounding of an exact rational to fp32 (nearest, ties to even), by comparing with the
+    two fp32 neighbours exactly."""
+    f = np.float32(float(v))
+    lo, hi = (np.nextafter(f, np.float32(-np.inf)), f) if Fraction(float(f)) > v else \
+        (f, np.nextafter(f, np.float32(np.inf)))
+    dl, dh = v - Fraction(float(lo)), Fraction(float(hi)) - v
+    if dl != dh:
+        return lo if dl < dh else hi
+    return lo if (lo.view(np.uint32) & 1) == 0 else hi
+
+
+def test_center_hand_example(oracle):
+    g = json.load(open(os.path.join(GOLDEN, "center_hand_example.json")))
+    W = np.array(g["W"], np.float32)
+    for mode, key in ((oracle.CENTER_PER_CHANNEL, "per_channel"), (oracle.CENTER_PER_LAYER, "per_layer")):
+        B, Wc = oracle.center(W, mode)
+        assert B.tolist() == g[key]["B"] and Wc.tolist() == g[key]["Wc"]
+    pt = g["points"]
+    codes, scales = np.array(pt["codes"], np.int8), np.array(pt["scales"], np.float32)
+    B = np.array(g["per_channel"]["B"], np.float32)
+    npts = np.array(pt["npoints"], np.int32)
+    assert oracle.reconstruct(codes, scales, npts, center=B).tolist() == pt["W_hat"]
+    it = g["integer"]
+    assert [oracle.fixed_coeff(b, it["p"]) for b in B] == it["A_B"]
+    Y = oracle.multipoint_linear(np.array(it["X"], np.int8), codes, scales, npts, it["p"], center=B)
+    assert Y.tolist() == it["Y"]
+
+
+def test_center_is_the_rounded_midrange(oracle):
+    """B = (max + min) / 2 correctly rounded to fp32 and W - B correctly rounded, against exact
+    rational arithmetic, for ranges of very different magnitudes and offsets."""
+    rng = np.random.default_rng(51)
+    W = np.concatenate([rng.standard_normal((4, 33)) * 0.02 + 0.3,
+                        rng.uniform(-1e-3, 5.0, (3, 33)),
+                        rng.standard_normal((3, 33)) * 1e4 - 2.0]).astype(np.float32)
+    B, Wc = oracle.center(W, oracle.CENTER_PER_CHANNEL)
+    for k in range(W.shape[0]):
+        mid = (Fraction(float(W[k].max())) + Fraction(float(W[k].min()))) / 2
+        assert B[k] == _round_f32(mid)
+        for j in range(0, 33, 4):
+            assert Wc[k, j] == _round_f32(Fraction(float(W[k, j])) - Fraction(float(B[k])))
+    Bl, Wl = oracle.center(W, oracle.CENTER_PER_LAYER)
+    assert np.all(Bl == _round_f32((Fraction(float(W.max())) + Fraction(float(W.min()))) / 2))
+    # per layer equals per channel on the layer flattened to one channel
+    B1, W1 = oracle.center(W.reshape(1, -1), oracle.CENTER_PER_CHANNEL)
+    assert np.all(Bl == B1[0]) and np.array_equal(Wl.reshape(1, -1), W1)
+
+
+def test_center_symmetric_range_is_the_symmetric_method(oracle):
+    """A channel with max = -min has B = 0: centring changes nothing, so the greedy points and the
+    reconstruction equal the symmetric method's."""
+    rng = np.random.default_rng(52)
+    W = rng.standard_normal((6, 40)).astype(np.float32)
+    W[:, 0] = np.abs(W).max(axis=1)
+    W[:, 1] = -W[:, 0]
+    B, Wc = oracle.center(W, oracle.CENTER_PER_CHANNEL)
+    assert np.all(B == 0) and np.array_equal(Wc, W)
+    q0, q1 = oracle.quantize_layer(W, 4, 32, 3), oracle.quantize_layer(Wc, 4, 32, 3)
+    assert np.array_equal(q0["codes"], q1["codes"]) and np.array_equal(q0["scales"], q1["scales"])
+    n = np.full(6, 2, np.int32)
+    assert np.array_equal(oracle.reconstruct(q0["codes"], q0["scales"], n),
+                          oracle.reconstruct(q1["codes"], q1["scales"], n, center=B))
+
+
+def test_center_affine_lattice_is_exact(oracle):
+    """w = B0 + s0 q with q covering -Qmax..Qmax (dyadic B0, s0): the centre is B0, the centred
+    weights are s0 q, one greedy point on the full-range grid scale reproduces w exactly."""
+    rng = np.random.default_rng(53)
+    for bits in (3, 4):
+        qm = 2 ** (bits - 1) - 1
+        q = rng.integers(-qm, qm + 1, (5, 24))
+        q[:, 0], q[:, 1] = qm, -qm
+        B0 = np.array([0.75, -3.5, 1024.0, 0.0078125, -0.5], np.float32)
+        s0 = np.array([0.125, 0.5, 2.0, 2.0 ** -12, 0.25], np.float32)
+        W = (B0[:, None] + s0[:, None] * q).astype(np.float32)
+        B, Wc = oracle.center(W, oracle.CENTER_PER_CHANNEL)
+        assert np.array_equal(B, B0) and np.array_equal(Wc, (s0[:, None] * q).astype(np.float32))
+        out = oracle.quantize_layer(Wc, bits, 4, 1)
+        What = oracle.reconstruct(out["codes"], out["scales"], np.ones(5, np.int32), center=B)
+        assert np.array_equal(What, W)
+
+
+def test_center_nonfinite(oracle):
+    W = np.random.default_rng(54).standard_normal((3, 10)).astype(np.float32)
+    W[1, 4] = np.nan
+    B, _ = oracle.center(W, oracle.CENTER_PER_CHANNEL)
+    assert np.isnan(B[1]) and np.all(np.isfinite(B[[0, 2]]))
+    Bl, _ = oracle.center(W, oracle.CENTER_PER_LAYER)
+    assert np.all(np.isnan(Bl))
+
+
+def test_integer_inference_with_center_exact(oracle):
+    """Dyadic scales and centres: Y = floor(B sum(x) + sum_i s_i (q_i . x)) exactly (rational
+    arithmetic); with no points, Y = floor(B sum(x))."""
+    rng = np.random.default_rng(55)
+    for p in (0, 5, 14):
+        k_max, C, d, T = 3, 6, 19, 5
+        codes = rng.integers(-7, 8, (k_max, C, d)).astype(np.int8)
+        A = rng.integers(-3000, 3000, (C, k_max))
+        AB = rng.integers(-5000, 5000, C)
+        scales = (A / 2.0 ** p).astype(np.float32)
+        B = (AB / 2.0 ** p).astype(np.float32)
+        npts = rng.integers(0, k_max + 1, C).astype(np.int32)
+        npts[0] = 0
+        X = rng.integers(-128, 128, (T, d)).astype(np.int8)
+        Y = oracle.multipoint_linear(X, codes, scales, npts, p, center=B)
+        for k in range(C):
+            for t in range(T):
+                xs = int(X[t].astype(np.int64).sum())
+                v = Fraction(int(AB[k]), 2 ** p) * xs + sum(
+                    Fraction(int(A[k, i]), 2 ** p) *
+                    int(np.dot(codes[i, k].astype(np.int64), X[t].astype(np.int64)))
+                    for i in range(npts[k]))
+                assert Y[k, t] == (v.numerator // v.denominator)
