@@ -41,7 +41,11 @@ KERNEL_SOURCES = {
                  "paper_2002_09049_gb300/csrc/rounding.cuh"),
     "allocate": "paper_2002_09049_gb300/csrc/allocate.cu",
     "reconstruct": "paper_2002_09049_gb300/csrc/reconstruct.cu",
+    "center": "paper_2002_09049_gb300/csrc/center.cu",
 }
+
+
+CENTER_MODES = {"none": -1, "channel": 0, "layer": 1}
 
 
 def parse():
@@ -68,6 +72,9 @@ def parse():
     ap.add_argument("--coef-bits", type=int, default=16, help="p of Eq. 13 for --op infer")
     ap.add_argument("--clip-candidates", type=int, default=20,
                     help="clipping factor candidates (c+1)/n x max|w| for --op clip")
+    ap.add_argument("--center", default="none", choices=list(CENTER_MODES),
+                    help="asymmetric sets (Eq. 1, B != 0) for --op quantize / infer: one centre per "
+                         "channel or per layer, the points approximating the centred weights")
     return ap.parse_args()
 
 
@@ -224,7 +231,7 @@ def run_ours(args, world, rank, local):
         W, X = layer_inputs(wl, li)
         specs.append(pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, groups=layer.groups,
                                         bits=wl.bits[0], G=wl.G, k_max=wl.k_max,
-                                        budget_or_eps=wl.beta))
+                                        budget_or_eps=wl.beta, center=CENTER_MODES[args.center]))
         Whs.append(torch.from_numpy(W).pin_memory())
         Xhs.append(torch.from_numpy(X).pin_memory())
         Ws.append(Whs[-1].to(dev))
@@ -234,7 +241,7 @@ def run_ours(args, world, rank, local):
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 512 MB > L2
     stream = torch.cuda.current_stream()
 
-    families = ["quantize", "output_error", "allocate", "reconstruct"]
+    families = ["center", "quantize", "output_error", "allocate", "reconstruct"]
 
     graphs = []
     if args.graph:
@@ -254,7 +261,8 @@ def run_ours(args, world, rank, local):
                 sp.bits = b
             net.run_device(Ws, Xs, stream=stream)
 
-    launches_per_step = 4 * len(layers) * len(wl.bits)
+    center_launches = {"none": 0, "channel": 1, "layer": 3}[args.center]
+    launches_per_step = (4 + center_launches) * len(layers) * len(wl.bits)
 
     for _ in range(args.warmup):
         step()
@@ -287,7 +295,7 @@ def run_ours(args, world, rank, local):
                 sp.bits = b
             evs = {}
             for i in net.order:
-                evs[i] = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+                evs[i] = [torch.cuda.Event(enable_timing=True) for _ in range(len(families) + 1)]
                 net.plans[i].run_device(Ws[i], Xs[i], stream=stream,
                                         timing=lambda ph, e=evs[i]: e[ph].record(stream))
             rec.append(evs)
@@ -311,6 +319,7 @@ def run_ours(args, world, rank, local):
                 fam_work["quantize"] += quantize_ops(wl, layer, wl.bits[0])
                 fam_work["reconstruct"] += reconstruct_bytes(wl, layer)
                 fam_work["allocate"] += 4 * layer.C * (wl.k_max + 1) * 9 + 8 * layer.C
+                fam_work["center"] += 8 * layer.C * layer.d + 4 * layer.C
     total_fam = sum(fam_ms.values())
     dominant = max(fam_ms, key=fam_ms.get)
 
@@ -332,7 +341,7 @@ def run_ours(args, world, rank, local):
                    "G": wl.G, "k_max": wl.k_max, "budget": wl.beta, "calib_rows": wl.n_calib,
                    "units_per_step": units_per_step, "l2": "flushed between steps (512 MB write)",
                    "streams": args.streams, "cuda_graph": bool(args.graph),
-                   "parallelism": f"replicas x{world}"},
+                   "center": args.center, "parallelism": f"replicas x{world}"},
         "roofline": roofline,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
@@ -341,7 +350,7 @@ def run_ours(args, world, rank, local):
     if not args.no_e2e:
         out["e2e"] = run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
+        out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds, CENTER_MODES[args.center])
     if world > 1:
         torch.distributed.barrier()
         torch.distributed.destroy_process_group()
@@ -359,7 +368,7 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_
       the nominal tf32/bf16 ratio.
     quantize: ALU bound; achieved = algorithmic lane operations (quantize_ops) / time; peak = SMs x
       128 lanes x the maximum SM clock.
-    reconstruct / allocate: HBM roofline; achieved = algorithmic bytes / time."""
+    reconstruct / allocate / center: HBM roofline; achieved = algorithmic bytes / time."""
     traffic = None
     tfile = os.path.join(PROFILES, "roofline_traffic.json")
     if os.path.exists(tfile):
@@ -391,7 +400,8 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_
     hbm = peaks["hbm_gbs"]
     ach = fam_work.get(dominant, 0.0) / t_s / 1e9
     names = {"reconstruct": "reconstruct_vec4_kernel (Eq. 4)",
-             "allocate": "allocate_budget_kernel (Algorithm 2)"}
+             "allocate": "allocate_budget_kernel (Algorithm 2)",
+             "center": "center_channel_kernel (Eq. 1 centre, centred weights)"}
     return {"kernel": names.get(dominant, dominant), "bound": "hbm", "achieved": ach, "peak": hbm,
             "unit": "GB/s", "frac": ach / hbm, "traffic": traffic,
             "peak_source": f"{peak_src} HBM copy"}
@@ -441,20 +451,24 @@ def oracle_sample(wl, target_s):
     return stride
 
 
-def run_oracle_step(wl, stride, threads, inputs):
-    """The oracle over the sampled channels of every layer: Algorithm 1, Eq. 11, Algorithm 2
-    (budget, per layer, on the sample), Eq. 4.  Returns the metric units processed."""
+def run_oracle_step(wl, stride, threads, inputs, center=-1):
+    """The oracle over the sampled channels of every layer: centring (asymmetric sets), Algorithm
+    1, Eq. 11, Algorithm 2 (budget, per layer, on the sample), Eq. 4.  Returns the metric units
+    processed."""
     import oracle
     units = 0
     for b in wl.bits:
         for li, layer in enumerate(wl.layers):
             W, X = inputs[li]
+            B = None
+            if center >= 0:
+                B, W = oracle.center(W, center)
             q = oracle.quantize_layer(W, b, wl.G, wl.k_max, want_residuals=False, threads=threads)
             groups = W.shape[0] if layer.groups > 1 else 1
             err = oracle.output_error(X, groups, W, q["codes"], q["scales"], wl.k_max,
                                       threads=threads)
             n, _ = oracle.allocate_budget(err.astype(np.float32), wl.k_max, wl.beta)
-            oracle.reconstruct(q["codes"], q["scales"], n)
+            oracle.reconstruct(q["codes"], q["scales"], n, center=B)
             units += W.shape[0] * layer.d * wl.G * wl.k_max
     return units
 
@@ -471,14 +485,14 @@ def sample_inputs(wl, stride):
     return inputs
 
 
-def cpu_baseline(wl, target_s):
+def cpu_baseline(wl, target_s, center=-1):
     import oracle
     oracle.build()
     stride = oracle_sample(wl, target_s)
     threads = host_cores()
     inputs = sample_inputs(wl, stride)
     t0 = time.perf_counter()
-    units = run_oracle_step(wl, stride, threads, inputs)
+    units = run_oracle_step(wl, stride, threads, inputs, center)
     dt = time.perf_counter() - t0
     return {"value": units / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
             "seconds": dt,
@@ -498,12 +512,13 @@ def run_reference(args, world, rank):
     stride = oracle_sample(wl, per_step)
     threads = host_cores()
     inputs = sample_inputs(wl, stride)
+    cen = CENTER_MODES[args.center]
     for _ in range(args.warmup):
-        run_oracle_step(wl, stride, threads, inputs)
+        run_oracle_step(wl, stride, threads, inputs, cen)
     times, units = [], 0
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        units = run_oracle_step(wl, stride, threads, inputs)
+        units = run_oracle_step(wl, stride, threads, inputs, cen)
         times.append(time.perf_counter() - t0)
     s = float(np.mean(times))
     value = units / s
@@ -512,7 +527,7 @@ def run_reference(args, world, rank):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
             "config": {"workload": f"{args.config}: {wl.title}", "bits": list(wl.bits), "G": wl.G,
-                       "k_max": wl.k_max, "budget": wl.beta},
+                       "k_max": wl.k_max, "budget": wl.beta, "center": args.center},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
                              "sample": f"every {stride}th channel of every layer per step"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -727,19 +742,24 @@ def infer_layers(args, wl, dev):
             continue
         W, X = layer_inputs(wl, li)
         Wd, Xd = torch.from_numpy(W).to(dev), torch.from_numpy(X).to(dev)
+        B = None
+        if CENTER_MODES[args.center] >= 0:
+            B, Wd = binding.mpq_center_weights(Wd, CENTER_MODES[args.center])
         codes, scales, _, _ = binding.mpq_quantize_layer(Wd, wl.bits[0], wl.G, wl.k_max)
         err = binding.mpq_output_error(Xd, Wd, codes, scales, wl.k_max,
                                        groups=layer.C if layer.groups > 1 else 1)
         npts, _ = binding.mpq_allocate_points(err, wl.k_max, binding.MPQ_ALLOC_BUDGET, wl.beta)
         n_host = npts.cpu().numpy()
-        lay = binding.mpq_pack_layout(n_host, layer.d, wl.k_max, wl.bits[0], args.coef_bits)
-        packed = binding.mpq_pack_points(codes, scales, n_host, lay)
+        lay = binding.mpq_pack_layout(n_host, layer.d, wl.k_max, wl.bits[0], args.coef_bits,
+                                      centered=B is not None)
+        packed = binding.mpq_pack_points(codes, scales, n_host, lay, center=B)
         Xq = np.random.default_rng(900000 + li).integers(-128, 128, (wl.n_calib, layer.d))
         Xh = torch.from_numpy(Xq.astype(np.int8)).pin_memory()
         out.append(dict(layer=layer, lay=lay, packed=packed, Xh=Xh, X=Xh.to(dev),
                         Y=torch.empty((layer.C, wl.n_calib), dtype=torch.int32, device=dev),
                         macs=int(n_host.sum()) * layer.d * wl.n_calib,
-                        codes=codes.cpu().numpy(), scales=scales.cpu().numpy(), n=n_host, Xq=Xq))
+                        codes=codes.cpu().numpy(), scales=scales.cpu().numpy(), n=n_host, Xq=Xq,
+                        center=None if B is None else B.cpu().numpy()))
     return out
 
 
@@ -837,6 +857,7 @@ def run_infer(args, world, rank, local):
            "config": {"workload": f"{args.config}: {wl.title}", "op": "infer (Eq. 13)",
                       "layers": len(L), "inputs_per_layer": wl.n_calib, "p": args.coef_bits,
                       "points": f"budget {wl.beta} per channel (Algorithm 2)",
+                      "center": args.center,
                       "macs_per_step": macs, "l2": "flushed between steps (512 MB write)",
                       "streams": args.streams, "parallelism": f"replicas x{world}"},
            "roofline": roofline, "gpu_launches": len(L) * args.steps, "clocks": clk.summary()}
@@ -882,7 +903,8 @@ def run_infer(args, world, rank, local):
             per_ch = x["macs"] / max(1, C) * 1.5e-9
             nc = max(1, min(C, int(args.cpu_seconds / len(L) / max(per_ch, 1e-12)) * host_cores()))
             oracle.multipoint_linear(x["Xq"].astype(np.int8), x["codes"], x["scales"], x["n"],
-                                     args.coef_bits, channels=(0, nc), threads=host_cores())
+                                     args.coef_bits, channels=(0, nc), threads=host_cores(),
+                                     center=x["center"])
             units += int(x["n"][:nc].sum()) * x["layer"].d * wl.n_calib
         dt = time.perf_counter() - t0
         out["cpu_baseline"] = {"value": units / dt, "unit": INFER_UNIT, "cores": host_cores(),

@@ -57,6 +57,10 @@ typedef enum {
 #define MPQ_ALLOC_BUDGET 0
 #define MPQ_ALLOC_THRESHOLD 1
 
+/* Centres of mpq_center_weights: one B per channel, or one B for the whole layer. */
+#define MPQ_CENTER_PER_CHANNEL 0
+#define MPQ_CENTER_PER_LAYER 1
+
 /* Clipping-factor sets of mpq_clip_search: one K per channel, or one K for the whole layer. */
 #define MPQ_CLIP_PER_CHANNEL 0
 #define MPQ_CLIP_PER_LAYER 1
@@ -132,16 +136,39 @@ mpq_status mpq_allocate_points(const float *err, int C, int k_max, int mode, dou
                                int *npoints, int *points_used, void *stream);
 
 /*
- * mpq_reconstruct -- multipoint weights (Eq. 4): W_hat[k][j] = sum_{i=1..n_k} s_{k,i} q_{k,i,j},
- * accumulated as acc = fmaf(s_{k,i}, q_{k,i,j}, acc) from acc = 0 in the order i = 1, 2, ...
+ * mpq_reconstruct -- multipoint weights (Eq. 4): W_hat[k][j] = B_k + sum_{i=1..n_k} s_{k,i} q_{k,i,j},
+ * accumulated as acc = fmaf(s_{k,i}, q_{k,i,j}, acc) from acc = B_k (the centre of an asymmetric
+ * set, from mpq_center_weights; 0 when center is NULL) in the order i = 1, 2, ...
  * n_k = npoints[k] clamped to [0, k_max] (npoints lives on the device and is not checked on the
  * host).
  *
  *   codes [k_max][C][d] int8, scales [C][k_max] fp32, npoints [C] int32.
+ *   center [C] fp32 or NULL.
  *   W_hat out [C][d] fp32.
  */
-mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C,
-                           int d, int k_max, float *W_hat, void *stream);
+mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
+                           const float *center, int C, int d, int k_max, float *W_hat,
+                           void *stream);
+
+/*
+ * mpq_center_weights -- asymmetric quantization sets (Eq. 1 with B != 0; per-channel and per-layer
+ * settings of Sec. 3.1 and App. B).  The set K x [-1 : eps_b : 1] + B has the centre
+ *   B = (max w + min w) / 2, rounded once to fp32,
+ * over the channel's weights (MPQ_CENTER_PER_CHANNEL) or over the whole layer
+ * (MPQ_CENTER_PER_LAYER, one B for every channel), so that K = (max w - min w) / 2 covers every
+ * weight.  The multipoint approximation takes B once and approximates the centred weights with
+ * the greedy points: Wc = fl(w - B) (one fp32 subtraction) is the W to give mpq_quantize_layer,
+ * mpq_output_error and mpq_clip_search, and center is the B to give mpq_reconstruct and
+ * mpq_pack_points, so that w~ = B + sum_i s_i q_i.  A non-finite weight makes B NaN for its
+ * channel (per layer: for every channel), and so that channel's Wc.
+ *
+ *   W, C, d   [C][d] fp32 weights; d >= 1.
+ *   mode      MPQ_CENTER_PER_CHANNEL or MPQ_CENTER_PER_LAYER.
+ *   center    out [C] fp32.
+ *   Wc        out [C][d] fp32 (per layer, its first C values also serve as working storage).
+ */
+mpq_status mpq_center_weights(const float *W, int C, int d, int mode, float *center, float *Wc,
+                              void *stream);
 
 /*
  * mpq_clip_search -- output-error-driven clipping factor (Sec. 3.3, Eq. 12; candidate grid of
@@ -178,8 +205,10 @@ mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, in
  * (ties to even): integer dot products (step 1), multiplication by the 32-bit coefficients and
  * summation (step 2), and the shift by p bits (step 3; an arithmetic right shift, i.e. floor), with
  * exact 64-bit products and sums and saturation to the int32 range.  n_k = npoints[k] clamped to
- * [0, k_max]; a channel with no point outputs 0.  The q are the integer codes of mpq_quantize_layer,
- * so the coefficient of q is s = a / Qmax.
+ * [0, k_max]; a channel with no point outputs 0 (with a centre, its A_B term alone).  The q are the
+ * integer codes of mpq_quantize_layer, so the coefficient of q is s = a / Qmax.  With asymmetric
+ * sets (a centre B_k per channel, from mpq_center_weights), w~ = B_k 1 + sum_i s_i q_i and the sum
+ * before the shift also holds A_{B,k} (sum_j x_tj), A_{B,k} = rint(2^p B_k).
  *
  * Deployment is split as in the paper: the coefficients and a packed copy of the used points are
  * made once, offline (mpq_pack_layout on the host, then mpq_pack_points), and
@@ -187,10 +216,11 @@ mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, in
  */
 typedef struct {
     int C, d, k_max, bits, p;
+    int centered;        /* 1: the layer has centres B_k (asymmetric sets) */
     int d_pad;           /* d rounded up to a multiple of 64 */
     int rows;            /* packed code rows, a multiple of 128 */
     int tiles;           /* rows / 128 */
-    size_t off_coef, off_chan, off_point, off_tile, off_codes;   /* byte offsets in the buffer */
+    size_t off_coef, off_chan, off_point, off_tile, off_center, off_codes;   /* byte offsets */
     size_t bytes;        /* size of the device buffer to allocate */
 } mpq_packed_layout;
 
@@ -199,21 +229,25 @@ typedef struct {
  *   npoints  HOST [C] int32 (e.g. copied back from mpq_allocate_points).
  *   bits     the codes' width (their magnitude is at most 2^(bits-1) - 1).
  *   p        coefficient precision, 0..30.
+ *   centered 1 if the layer has centres (mpq_pack_points then takes them), else 0.
  *   layout   out.
  */
 mpq_status mpq_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
-                           mpq_packed_layout *layout);
+                           int centered, mpq_packed_layout *layout);
 
 /*
  * mpq_pack_points -- fill a packed layer: coefficients A = rint(2^p s) of the used points and their
- * codes (as bf16, exact).  Synchronous: returns after the device has finished with the host array.
+ * codes (as bf16, exact), and A_B = rint(2^p B) of the centres.  Synchronous: returns after the
+ * device has finished with the host arrays.
  *   codes [k_max][C][d] int8 and scales [C][k_max] fp32 on the device (from mpq_quantize_layer);
+ *   center  [C] fp32 on the device (from mpq_center_weights) if layout->centered, else NULL;
  *   npoints HOST [C], the same as given to mpq_pack_layout;
  *   packed  device buffer of layout->bytes bytes, written here.
- * MPQ_ERR_UNSUPPORTED if a coefficient does not fit 32 bits.
+ * MPQ_ERR_UNSUPPORTED if a coefficient (or a centre's) does not fit 32 bits, NaN included.
  */
-mpq_status mpq_pack_points(const int8_t *codes, const float *scales, const int *npoints,
-                           const mpq_packed_layout *layout, void *packed, void *stream);
+mpq_status mpq_pack_points(const int8_t *codes, const float *scales, const float *center,
+                           const int *npoints, const mpq_packed_layout *layout, void *packed,
+                           void *stream);
 
 /*
  * mpq_multipoint_linear -- Y [C][T] int32 (channel-major: one channel's T outputs are contiguous)

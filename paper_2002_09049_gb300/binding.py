@@ -16,6 +16,8 @@ from . import _build
 
 MPQ_ALLOC_BUDGET = 0
 MPQ_ALLOC_THRESHOLD = 1
+MPQ_CENTER_PER_CHANNEL = 0
+MPQ_CENTER_PER_LAYER = 1
 MPQ_CLIP_PER_CHANNEL = 0
 MPQ_CLIP_PER_LAYER = 1
 
@@ -28,11 +30,12 @@ _P, _I, _D = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
 class PackedLayout(ctypes.Structure):
     """mpq_packed_layout of include/mpq.h: the layout of a packed multipoint layer (Sec. 3.4)."""
     _fields_ = [("C", ctypes.c_int), ("d", ctypes.c_int), ("k_max", ctypes.c_int),
-                ("bits", ctypes.c_int), ("p", ctypes.c_int), ("d_pad", ctypes.c_int),
-                ("rows", ctypes.c_int), ("tiles", ctypes.c_int),
+                ("bits", ctypes.c_int), ("p", ctypes.c_int), ("centered", ctypes.c_int),
+                ("d_pad", ctypes.c_int), ("rows", ctypes.c_int), ("tiles", ctypes.c_int),
                 ("off_coef", ctypes.c_size_t), ("off_chan", ctypes.c_size_t),
                 ("off_point", ctypes.c_size_t), ("off_tile", ctypes.c_size_t),
-                ("off_codes", ctypes.c_size_t), ("bytes", ctypes.c_size_t)]
+                ("off_center", ctypes.c_size_t), ("off_codes", ctypes.c_size_t),
+                ("bytes", ctypes.c_size_t)]
 
 
 _L = ctypes.POINTER(PackedLayout)
@@ -41,10 +44,11 @@ SIGNATURES = {
     "mpq_quantize_layer": ([_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P], _I),
     "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
-    "mpq_reconstruct": ([_P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "mpq_reconstruct": ([_P, _P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "mpq_center_weights": ([_P, _I, _I, _I, _P, _P, _P], _I),
     "mpq_clip_search": ([_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P], _I),
-    "mpq_pack_layout": ([_P, _I, _I, _I, _I, _I, _L], _I),
-    "mpq_pack_points": ([_P, _P, _P, _L, _P, _P], _I),
+    "mpq_pack_layout": ([_P, _I, _I, _I, _I, _I, _I, _L], _I),
+    "mpq_pack_points": ([_P, _P, _P, _P, _L, _P, _P], _I),
     "mpq_multipoint_linear": ([_P, _I, _L, _P, _P, _P], _I),
     "mpq_status_string": ([_I], ctypes.c_char_p),
     "mpq_last_error": ([], ctypes.c_char_p),
@@ -206,20 +210,27 @@ def _host_int32(a):
     return np.ascontiguousarray(a, dtype=np.int32)
 
 
-def mpq_pack_layout(npoints, d: int, k_max: int, bits: int, p: int) -> PackedLayout:
-    """Host-side layout of a packed multipoint layer (Sec. 3.4) for the point counts npoints [C]."""
+def mpq_pack_layout(npoints, d: int, k_max: int, bits: int, p: int,
+                    centered: bool = False) -> PackedLayout:
+    """Host-side layout of a packed multipoint layer (Sec. 3.4) for the point counts npoints [C]
+    (centered: the layer has centres B_k of asymmetric sets)."""
     n = _host_int32(npoints)
     lay = PackedLayout()
-    st = load().mpq_pack_layout(n.ctypes.data, int(n.size), d, k_max, bits, p, ctypes.byref(lay))
+    st = load().mpq_pack_layout(n.ctypes.data, int(n.size), d, k_max, bits, p, int(bool(centered)),
+                                ctypes.byref(lay))
     _check(st, "mpq_pack_layout")
     return lay
 
 
-def mpq_pack_points(codes, scales, npoints, layout: PackedLayout, packed=None, stream=None):
-    """Coefficients rint(2^p s) and bf16 codes of the used points (offline, synchronous).
-    Returns the packed device buffer (uint8 [layout.bytes])."""
+def mpq_pack_points(codes, scales, npoints, layout: PackedLayout, packed=None, stream=None,
+                    center=None):
+    """Coefficients rint(2^p s) and bf16 codes of the used points, and rint(2^p B) of the centres
+    when the layout is centered (offline, synchronous).  Returns the packed device buffer
+    (uint8 [layout.bytes])."""
     _dev(codes, "codes", torch.int8, (layout.k_max, layout.C, layout.d))
     _dev(scales, "scales", torch.float32, (layout.C, layout.k_max))
+    if center is not None:
+        _dev(center, "center", torch.float32, (layout.C,))
     n = _host_int32(npoints)
     if n.size != layout.C:
         raise ValueError("npoints must have C entries")
@@ -228,8 +239,8 @@ def mpq_pack_points(codes, scales, npoints, layout: PackedLayout, packed=None, s
     _dev(packed, "packed", torch.uint8)
     if packed.numel() < layout.bytes:
         raise ValueError("packed buffer smaller than layout.bytes")
-    st = load().mpq_pack_points(_ptr(codes), _ptr(scales), n.ctypes.data, ctypes.byref(layout),
-                                _ptr(packed), _stream(stream))
+    st = load().mpq_pack_points(_ptr(codes), _ptr(scales), _ptr(center), n.ctypes.data,
+                                ctypes.byref(layout), _ptr(packed), _stream(stream))
     _check(st, "mpq_pack_points")
     return packed
 
@@ -269,19 +280,37 @@ def mpq_allocate_points(err, k_max: int, mode: int = MPQ_ALLOC_BUDGET,
     return npoints, points_used
 
 
-def mpq_reconstruct(codes, scales, npoints, W_hat=None, stream=None):
-    """Multipoint weights (Eq. 4): W_hat [C][d] fp32."""
+def mpq_reconstruct(codes, scales, npoints, W_hat=None, stream=None, center=None):
+    """Multipoint weights (Eq. 4): W_hat [C][d] fp32, from the centres B [C] of asymmetric sets
+    when given."""
     _dev(codes, "codes", torch.int8)
     k_max, C, d = codes.shape
     _dev(scales, "scales", torch.float32, (C, k_max))
     _dev(npoints, "npoints", torch.int32, (C,))
+    if center is not None:
+        _dev(center, "center", torch.float32, (C,))
     W_hat = W_hat if W_hat is not None else torch.empty((C, d), dtype=torch.float32,
                                                         device=codes.device)
     _dev(W_hat, "W_hat", torch.float32, (C, d))
-    st = load().mpq_reconstruct(_ptr(codes), _ptr(scales), _ptr(npoints), C, d, k_max,
-                                _ptr(W_hat), _stream(stream))
+    st = load().mpq_reconstruct(_ptr(codes), _ptr(scales), _ptr(npoints), _ptr(center), C, d,
+                                k_max, _ptr(W_hat), _stream(stream))
     _check(st, "mpq_reconstruct")
     return W_hat
+
+
+def mpq_center_weights(W, mode: int = MPQ_CENTER_PER_CHANNEL, center=None, Wc=None, stream=None):
+    """Asymmetric sets (Eq. 1, B != 0): the centres B = the fp32 midpoint of the weights' range per
+    channel or per layer, and the centred weights Wc = W - B.  Returns (center [C], Wc [C][d])."""
+    _dev(W, "W", torch.float32)
+    C, d = W.shape
+    center = center if center is not None else torch.empty((C,), dtype=torch.float32,
+                                                           device=W.device)
+    Wc = Wc if Wc is not None else torch.empty((C, d), dtype=torch.float32, device=W.device)
+    _dev(center, "center", torch.float32, (C,))
+    _dev(Wc, "Wc", torch.float32, (C, d))
+    st = load().mpq_center_weights(_ptr(W), C, d, mode, _ptr(center), _ptr(Wc), _stream(stream))
+    _check(st, "mpq_center_weights")
+    return center, Wc
 
 
 def mpq_status_string(status: int) -> str:

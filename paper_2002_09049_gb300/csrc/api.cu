@@ -162,7 +162,7 @@ extern "C" mpq_status mpq_clip_search(const float *X, int N, int groups, const f
 }
 
 extern "C" mpq_status mpq_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
-                                      mpq_packed_layout *layout)
+                                      int centered, mpq_packed_layout *layout)
 {
     g_msg[0] = 0;
     mpq_status st = check_common(C, d, k_max);
@@ -175,20 +175,26 @@ extern "C" mpq_status mpq_pack_layout(const int *npoints, int C, int d, int k_ma
     REQUIRE(p >= 0 && p <= 30, MPQ_ERR_INVALID_ARG, "p = %d outside [0, 30]", p);
     REQUIRE(layout, MPQ_ERR_INVALID_ARG, "layout must be non-NULL");
     REQUIRE(C == 0 || npoints, MPQ_ERR_INVALID_ARG, "npoints must be non-NULL");
-    return make_pack_layout(npoints, C, d, k_max, bits, p, layout);
+    REQUIRE(centered == 0 || centered == 1, MPQ_ERR_INVALID_ARG, "centered = %d must be 0 or 1",
+            centered);
+    return make_pack_layout(npoints, C, d, k_max, bits, p, centered, layout);
 }
 
-extern "C" mpq_status mpq_pack_points(const int8_t *codes, const float *scales, const int *npoints,
+extern "C" mpq_status mpq_pack_points(const int8_t *codes, const float *scales,
+                                      const float *center, const int *npoints,
                                       const mpq_packed_layout *layout, void *packed, void *stream)
 {
     g_msg[0] = 0;
     REQUIRE(layout, MPQ_ERR_INVALID_ARG, "layout must be non-NULL");
     mpq_status st = check_common(layout->C, layout->d, layout->k_max);
     if (st != MPQ_OK) return st;
+    REQUIRE((center != nullptr) == (layout->centered == 1), MPQ_ERR_INVALID_ARG,
+            "center must be given exactly when the layout is centered (centered = %d)",
+            layout->centered);
     if (layout->C == 0) return MPQ_OK;
     REQUIRE(codes && scales && npoints && packed, MPQ_ERR_INVALID_ARG,
             "codes, scales, npoints and packed must be non-NULL");
-    return launch_pack(codes, scales, npoints, layout, packed, (cudaStream_t)stream);
+    return launch_pack(codes, scales, center, npoints, layout, packed, (cudaStream_t)stream);
 }
 
 extern "C" mpq_status mpq_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout *layout,
@@ -241,7 +247,8 @@ extern "C" mpq_status mpq_allocate_points(const float *err, int C, int k_max, in
 }
 
 extern "C" mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
-                                      int C, int d, int k_max, float *W_hat, void *stream)
+                                      const float *center, int C, int d, int k_max, float *W_hat,
+                                      void *stream)
 {
     g_msg[0] = 0;
     mpq_status st = check_common(C, d, k_max);
@@ -249,7 +256,21 @@ extern "C" mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, 
     if (C == 0) return MPQ_OK;
     REQUIRE(codes && scales && npoints && W_hat, MPQ_ERR_INVALID_ARG,
             "codes, scales, npoints and W_hat must be non-NULL");
-    return launch_reconstruct(codes, scales, npoints, C, d, k_max, W_hat, (cudaStream_t)stream);
+    return launch_reconstruct(codes, scales, npoints, center, C, d, k_max, W_hat,
+                              (cudaStream_t)stream);
+}
+
+extern "C" mpq_status mpq_center_weights(const float *W, int C, int d, int mode, float *center,
+                                         float *Wc, void *stream)
+{
+    g_msg[0] = 0;
+    mpq_status st = check_common(C, d, 1);
+    if (st != MPQ_OK) return st;
+    REQUIRE(mode == MPQ_CENTER_PER_CHANNEL || mode == MPQ_CENTER_PER_LAYER, MPQ_ERR_INVALID_ARG,
+            "mode = %d is not MPQ_CENTER_PER_CHANNEL or MPQ_CENTER_PER_LAYER", mode);
+    if (C == 0) return MPQ_OK;
+    REQUIRE(W && center && Wc, MPQ_ERR_INVALID_ARG, "W, center and Wc must be non-NULL");
+    return launch_center(W, C, d, mode, center, Wc, (cudaStream_t)stream);
 }
 
 extern "C" const char *mpq_status_string(mpq_status s)
@@ -268,4 +289,4 @@ extern "C" const char *mpq_status_string(mpq_status s)
 
 extern "C" const char *mpq_last_error(void) { return g_msg; }
 
-extern "C" int mpq_version(void) { return 100; }
+extern "C" int mpq_version(void) { return 200; }

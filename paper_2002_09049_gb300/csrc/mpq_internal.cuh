@@ -50,9 +50,10 @@ mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C,
                        cudaStream_t stream);
 
 mpq_status make_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
-                            mpq_packed_layout *L);
-mpq_status launch_pack(const int8_t *codes, const float *scales, const int *npoints,
-                       const mpq_packed_layout *L, void *packed, cudaStream_t stream);
+                            int centered, mpq_packed_layout *L);
+mpq_status launch_pack(const int8_t *codes, const float *scales, const float *center,
+                       const int *npoints, const mpq_packed_layout *L, void *packed,
+                       cudaStream_t stream);
 mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout *L,
                                     const void *packed, int32_t *Y, cudaStream_t stream);
 
@@ -62,7 +63,10 @@ mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long 
 mpq_status launch_allocate_threshold(const float *err, int C, int k_max, double eps,
                                      int *npoints, int *points_used, cudaStream_t stream);
 
-mpq_status launch_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C,
-                              int d, int k_max, float *W_hat, cudaStream_t stream);
+mpq_status launch_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
+                              const float *center, int C, int d, int k_max, float *W_hat,
+                              cudaStream_t stream);
+mpq_status launch_center(const float *W, int C, int d, int mode, float *center, float *Wc,
+                         cudaStream_t stream);
 
 }  // namespace mpq

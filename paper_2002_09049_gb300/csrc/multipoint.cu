@@ -22,6 +22,9 @@
 // Steps 2 and 3 in the epilogue: each lane turns its accumulator into an integer, multiplies by its
 // row's coefficient in 64 bits, the R lanes of a channel add with warp shuffles, and the first lane
 // shifts (arithmetic: floor), saturates and writes 32 consecutive outputs.  Every wait is bounded.
+// Asymmetric sets (a centre B_k, Eq. 1): the producers also sum each input row's int8 values while
+// they convert it, and the first lane adds A_B,k (sum_j x_tj), A_B,k = rint(2^p B_k), before the
+// shift.
 //
 // Rows that TMA cannot address (d not a multiple of 16, unaligned input) and layers beyond the
 // exactness bound use a CUDA-core kernel with the same integer arithmetic.
@@ -72,9 +75,11 @@ struct LinCtrl {
     uint64_t full[3];             // producers converted the input tile
     uint64_t empty[3];            // MMAs on the stage completed
     uint64_t done;                // every MMA completed
+    uint64_t xs_ready;            // producers stored the input-row sums
     uint32_t tmem_base;
     int abort;
     int coef[L_MAX_RT][L_M];      // the row coefficients A of this CTA's tiles
+    int xsum[L_N];                // sum_j x_tj of this CTA's inputs (centred layers)
 };
 constexpr int L_CTRL_BYTES = (sizeof(LinCtrl) + 1023) / 1024 * 1024;
 template <int RT>
@@ -86,6 +91,7 @@ struct PackView {
     int *chan;
     int *point;
     int *tile_R;
+    int *center;                  // A_B of each channel, or null
     __nv_bfloat16 *codes;
     int *flag;
 };
@@ -98,9 +104,26 @@ PackView view(const mpq_packed_layout *L, void *packed)
     v.chan = reinterpret_cast<int *>(b + L->off_chan);
     v.point = reinterpret_cast<int *>(b + L->off_point);
     v.tile_R = reinterpret_cast<int *>(b + L->off_tile);
+    v.center = L->centered ? reinterpret_cast<int *>(b + L->off_center) : nullptr;
     v.codes = reinterpret_cast<__nv_bfloat16 *>(b + L->off_codes);
     v.flag = reinterpret_cast<int *>(b);   // header word 0: coefficient overflow
     return v;
+}
+
+// rint(2^p v) (ties to even) as a 32-bit coefficient; sets *flag when it does not fit (NaN included).
+__device__ __forceinline__ int fixed_coeff(float v, int p, int *flag)
+{
+    const double x = nearbyint(ldexp((double)v, p));
+    if (fabs(x) < 2147483648.0) return (int)x;
+    atomicExch(flag, 1);
+    return 0;
+}
+
+// A_B = rint(2^p B_k) of every channel.
+__global__ void pack_center_kernel(const float *__restrict__ center, int C, int p, PackView v)
+{
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    if (k < C) v.center[k] = fixed_coeff(center[k], p, v.flag);
 }
 
 // A = rint(2^p s) (ties to even) and the bf16 codes of every packed row.
@@ -110,15 +133,7 @@ __global__ void pack_kernel(const int8_t *__restrict__ codes, const float *__res
     const int r = blockIdx.x;
     const int k = v.chan[r], i = v.point[r];
     const bool live = k >= 0 && i >= 0;
-    if (threadIdx.x == 0) {
-        int a = 0;
-        if (live) {
-            const double x = nearbyint(ldexp((double)scales[(size_t)k * k_max + i], p));
-            if (fabs(x) < 2147483648.0) a = (int)x;
-            else atomicExch(v.flag, 1);
-        }
-        v.coef[r] = a;
-    }
+    if (threadIdx.x == 0) v.coef[r] = live ? fixed_coeff(scales[(size_t)k * k_max + i], p, v.flag) : 0;
     const int8_t *q = live ? codes + (size_t)i * C * d + (size_t)k * d : nullptr;
     for (int j = threadIdx.x; j < d_pad; j += blockDim.x)
         v.codes[(size_t)r * d_pad + j] = __float2bfloat16_rn(live && j < d ? (float)q[j] : 0.0f);
@@ -136,6 +151,7 @@ template <int RT>
 __global__ void __launch_bounds__(L_THREADS, 1)
 multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restrict__ coef,
                          const int *__restrict__ chan, const int *__restrict__ tile_R,
+                         const int *__restrict__ center_coef,
                          int32_t *__restrict__ Y, const __grid_constant__ CUtensorMap tmA,
                          const __grid_constant__ CUtensorMap tmX)
 {
@@ -164,6 +180,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             mbar_init(&ctl.empty[s], 1);
         }
         mbar_init(&ctl.done, 1);
+        mbar_init(&ctl.xs_ready, L_PROD_WARPS);
         ctl.abort = 0;
         fence_barrier_init();
     }
@@ -178,8 +195,13 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
     const uint32_t tmem = ctl.tmem_base;
     volatile int *abort_flag = &ctl.abort;
 
+    const bool centered = center_coef != nullptr;
     if (warp < L_PROD_WARPS) {
         // ---------------------------------------------------------------- producers: int8 -> bf16
+        constexpr int ITEMS = L_N * (L_KC / 16) / L_PROD_THREADS;
+        int xs[ITEMS];   // this thread's 16-byte share of each input row's sum
+#pragma unroll
+        for (int it = 0; it < ITEMS; ++it) xs[it] = 0;
         for (int kc = 0; kc < n_kc; ++kc) {
             const int s = kc % L_STAGES;
             const uint32_t ph = (uint32_t)(kc / L_STAGES) & 1u;
@@ -189,10 +211,16 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
             // 16 input bytes (one input row, 16 K elements) per item, 4 items per thread
 #pragma unroll
-            for (int it = 0; it < L_N * (L_KC / 16) / L_PROD_THREADS; ++it) {
+            for (int it = 0; it < ITEMS; ++it) {
                 const int q = threadIdx.x + it * L_PROD_THREADS;
                 const int row = q >> 2, c16 = q & 3;
                 const float4 raw = ld_shared_v4(sb + L_OFF_RAW + (uint32_t)q * 16u);
+                if (centered) {   // signed bytes summed exactly (|sum| <= 128 d)
+                    xs[it] = __dp4a(__float_as_int(raw.x), 0x01010101, xs[it]);
+                    xs[it] = __dp4a(__float_as_int(raw.y), 0x01010101, xs[it]);
+                    xs[it] = __dp4a(__float_as_int(raw.z), 0x01010101, xs[it]);
+                    xs[it] = __dp4a(__float_as_int(raw.w), 0x01010101, xs[it]);
+                }
                 const uint32_t w[4] = {__float_as_uint(raw.x) ^ 0x80808080u,
                                        __float_as_uint(raw.y) ^ 0x80808080u,
                                        __float_as_uint(raw.z) ^ 0x80808080u,
@@ -213,10 +241,23 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             __syncwarp();
             if (lane == 0) mbar_arrive(&ctl.full[s]);
         }
+        if (centered) {
+            // the 4 threads of an input row (lanes 4m..4m+3) hold its 4 column shares
+#pragma unroll
+            for (int it = 0; it < ITEMS; ++it) {
+                int v = xs[it];
+                v += __shfl_xor_sync(0xffffffffu, v, 1);
+                v += __shfl_xor_sync(0xffffffffu, v, 2);
+                if ((threadIdx.x & 3) == 0) ctl.xsum[(threadIdx.x + it * L_PROD_THREADS) >> 2] = v;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl.xs_ready);   // also after an abort: no wait is left open
+        }
     } else if (warp < L_MMA_WARP) {
         // ---------------------------------------------------------------- epilogue
         const int ew = warp - L_EPI_WARP0;
-        const bool ok = mbar_wait(&ctl.done, 0, L_WAIT);
+        bool ok = mbar_wait(&ctl.done, 0, L_WAIT);
+        if (ok && centered) ok = mbar_wait(&ctl.xs_ready, 0, L_WAIT);
         if (!ok) *abort_flag = 1;
         const bool good = !__any_sync(0xffffffffu, !ok || *abort_flag);
         tc_fence_after();
@@ -225,6 +266,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             const int r = ew * 32 + lane;
             const int k = chan[(size_t)(tile0 + u) * L_M + r];
             const long long a = ctl.coef[u][r];
+            const long long ab = centered && k >= 0 ? (long long)center_coef[k] : 0;
             const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16) + (uint32_t)(u * L_N);
 #pragma unroll 1
             for (int cb = 0; cb < L_N / 32; ++cb) {
@@ -242,7 +284,8 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                     int32_t *y = Y + (size_t)k * T + t0;
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
-                        long long z = sum[j] >> p;   // arithmetic shift: floor division by 2^p
+                        const long long tot = sum[j] + ab * (long long)ctl.xsum[cb * 32 + j];
+                        long long z = tot >> p;   // arithmetic shift: floor division by 2^p
                         z = z > 2147483647LL ? 2147483647LL : (z < -2147483648LL ? -2147483648LL : z);
                         if (t0 + j < T) y[j] = (int32_t)z;
                     }
@@ -317,7 +360,8 @@ __global__ void multipoint_linear_simt(const int8_t *__restrict__ X, int T, int 
                                        int p, const int *__restrict__ coef,
                                        const int *__restrict__ chan,
                                        const __nv_bfloat16 *__restrict__ codes,
-                                       const int *__restrict__ tile_R, int32_t *__restrict__ Y)
+                                       const int *__restrict__ tile_R,
+                                       const int *__restrict__ center_coef, int32_t *__restrict__ Y)
 {
     const size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x;
     const int slot_row = (int)(idx / T), t = (int)(idx % T);   // slot_row: first row of a channel
@@ -334,6 +378,11 @@ __global__ void multipoint_linear_simt(const int8_t *__restrict__ X, int T, int 
         long long acc = 0;
         for (int j = 0; j < d; ++j) acc += (long long)__bfloat162float(q[j]) * (long long)x[j];
         sum += (long long)coef[r] * acc;
+    }
+    if (center_coef) {
+        long long xs = 0;
+        for (int j = 0; j < d; ++j) xs += x[j];
+        sum += (long long)center_coef[k] * xs;
     }
     long long z = sum >> p;
     z = z > 2147483647LL ? 2147483647LL : (z < -2147483648LL ? -2147483648LL : z);
@@ -364,7 +413,7 @@ int pow2_at_least(int n)
 }  // namespace
 
 mpq_status make_pack_layout(const int *npoints, int C, int d, int k_max, int bits, int p,
-                            mpq_packed_layout *L)
+                            int centered, mpq_packed_layout *L)
 {
     memset(L, 0, sizeof(*L));
     L->C = C;
@@ -372,6 +421,7 @@ mpq_status make_pack_layout(const int *npoints, int C, int d, int k_max, int bit
     L->k_max = k_max;
     L->bits = bits;
     L->p = p;
+    L->centered = centered;
     L->d_pad = (d + L_KC - 1) / L_KC * L_KC;
     long long tiles = 0;
     for (int R = 1; R <= MPQ_MAX_POINTS; R <<= 1) {
@@ -397,6 +447,8 @@ mpq_status make_pack_layout(const int *npoints, int C, int d, int k_max, int bit
     off += (size_t)L->rows * 4;
     L->off_tile = off;
     off += (size_t)L->tiles * 4;
+    L->off_center = off;
+    off += centered ? (size_t)C * 4 : 0;
     off = (off + 1023) / 1024 * 1024;
     L->off_codes = off;
     off += (size_t)L->rows * L->d_pad * 2;
@@ -404,8 +456,9 @@ mpq_status make_pack_layout(const int *npoints, int C, int d, int k_max, int bit
     return MPQ_OK;
 }
 
-mpq_status launch_pack(const int8_t *codes, const float *scales, const int *npoints,
-                       const mpq_packed_layout *L, void *packed, cudaStream_t stream)
+mpq_status launch_pack(const int8_t *codes, const float *scales, const float *center,
+                       const int *npoints, const mpq_packed_layout *L, void *packed,
+                       cudaStream_t stream)
 {
     const int C = L->C, rows = L->rows;
     std::vector<int> chan((size_t)rows, -1), point((size_t)rows, -1), tR((size_t)L->tiles, 1);
@@ -449,12 +502,17 @@ mpq_status launch_pack(const int8_t *codes, const float *scales, const int *npoi
         e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_status(e, "pack kernel launch");
     }
+    if (L->centered) {
+        pack_center_kernel<<<(C + 255) / 256, 256, 0, stream>>>(center, C, L->p, v);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_status(e, "pack center kernel launch");
+    }
     int flag = 0;
     e = cudaMemcpyAsync(&flag, v.flag, sizeof(int), cudaMemcpyDeviceToHost, stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(stream);   // host arrays above must outlive the copies
     if (e != cudaSuccess) return cuda_status(e, "packing");
     if (flag) {
-        set_error("a coefficient rint(2^p * s) does not fit 32 bits (p = %d)", L->p);
+        set_error("a coefficient rint(2^p * s) or rint(2^p * B) does not fit 32 bits (p = %d)", L->p);
         return MPQ_ERR_UNSUPPORTED;
     }
     return MPQ_OK;
@@ -503,13 +561,13 @@ mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_lay
         const int rt = two ? 2 : 1;
         const dim3 grid((unsigned)tt, (unsigned)((L->tiles + rt - 1) / rt));
         kernel<<<grid, L_THREADS, smem, stream>>>(T, L->tiles, L->d_pad / L_KC, L->p, v.coef,
-                                                  v.chan, v.tile_R, Y, tmA, tmX);
+                                                  v.chan, v.tile_R, v.center, Y, tmA, tmX);
         return cuda_status(cudaGetLastError(), "multipoint linear kernel launch");
     }
     const size_t n = (size_t)L->rows * T;
     if (n == 0) return MPQ_OK;
     multipoint_linear_simt<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(
-        X, T, d, L->d_pad, L->rows, L->p, v.coef, v.chan, v.codes, v.tile_R, Y);
+        X, T, d, L->d_pad, L->rows, L->p, v.coef, v.chan, v.codes, v.tile_R, v.center, Y);
     return cuda_status(cudaGetLastError(), "multipoint linear (integer) kernel launch");
 }
 

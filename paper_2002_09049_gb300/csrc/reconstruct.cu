@@ -1,5 +1,6 @@
-// Multipoint weights (Eq. 4): W_hat[k][j] = sum_{i=1..n_k} s_{k,i} q_{k,i,j}, accumulated as
-// acc = fmaf(s_{k,i}, q_{k,i,j}, acc) from 0 in the order i = 1, 2, ...; n_k clamped to [0, k_max].
+// Multipoint weights (Eq. 4): W_hat[k][j] = B_k + sum_{i=1..n_k} s_{k,i} q_{k,i,j}, accumulated as
+// acc = fmaf(s_{k,i}, q_{k,i,j}, acc) from the set's centre B_k (Eq. 1; 0 for symmetric sets) in
+// the order i = 1, 2, ...; n_k clamped to [0, k_max].
 // Memory-bound: each element reads n_k code bytes and writes one fp32; four elements per thread
 // when d allows 16-byte stores.
 #include "mpq_internal.cuh"
@@ -11,8 +12,8 @@ constexpr int RC_THREADS = 256;
 
 __global__ void __launch_bounds__(RC_THREADS)
 reconstruct_kernel(const int8_t *__restrict__ codes, const float *__restrict__ scales,
-                   const int *__restrict__ npoints, int C, int d, int k_max,
-                   float *__restrict__ W_hat)
+                   const int *__restrict__ npoints, const float *__restrict__ center, int C, int d,
+                   int k_max, float *__restrict__ W_hat)
 {
     const size_t plane = (size_t)C * d;
     const size_t total = plane;
@@ -21,7 +22,7 @@ reconstruct_kernel(const int8_t *__restrict__ codes, const float *__restrict__ s
         const int k = (int)(idx / d);
         int n = npoints[k];
         n = n < 0 ? 0 : (n > k_max ? k_max : n);
-        float acc = 0.0f;
+        float acc = center ? center[k] : 0.0f;
         for (int i = 0; i < n; ++i)
             acc = __fmaf_rn(scales[(size_t)k * k_max + i], (float)codes[(size_t)i * plane + idx], acc);
         W_hat[idx] = acc;
@@ -32,8 +33,8 @@ reconstruct_kernel(const int8_t *__restrict__ codes, const float *__restrict__ s
 // stores).
 __global__ void __launch_bounds__(RC_THREADS)
 reconstruct_vec4_kernel(const int8_t *__restrict__ codes, const float *__restrict__ scales,
-                        const int *__restrict__ npoints, int C, int d, int k_max,
-                        float *__restrict__ W_hat)
+                        const int *__restrict__ npoints, const float *__restrict__ center, int C,
+                        int d, int k_max, float *__restrict__ W_hat)
 {
     const size_t plane = (size_t)C * d;
     const size_t total4 = plane / 4;
@@ -43,7 +44,8 @@ reconstruct_vec4_kernel(const int8_t *__restrict__ codes, const float *__restric
         const int k = (int)(idx / d);
         int n = npoints[k];
         n = n < 0 ? 0 : (n > k_max ? k_max : n);
-        float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
+        const float b = center ? center[k] : 0.0f;
+        float a0 = b, a1 = b, a2 = b, a3 = b;
         for (int i = 0; i < n; ++i) {
             const float s = scales[(size_t)k * k_max + i];
             const char4 c = *reinterpret_cast<const char4 *>(codes + (size_t)i * plane + idx);
@@ -58,8 +60,9 @@ reconstruct_vec4_kernel(const int8_t *__restrict__ codes, const float *__restric
 
 }  // namespace
 
-mpq_status launch_reconstruct(const int8_t *codes, const float *scales, const int *npoints, int C,
-                              int d, int k_max, float *W_hat, cudaStream_t stream)
+mpq_status launch_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
+                              const float *center, int C, int d, int k_max, float *W_hat,
+                              cudaStream_t stream)
 {
     const size_t total = (size_t)C * d;
     const bool vec = (d % 4 == 0) && ((uintptr_t)codes % 4 == 0) && ((uintptr_t)W_hat % 16 == 0);
@@ -68,11 +71,11 @@ mpq_status launch_reconstruct(const int8_t *codes, const float *scales, const in
     const size_t cap = (size_t)sm_count() * 8;
     if (blocks > cap) blocks = cap;
     if (vec)
-        reconstruct_vec4_kernel<<<(unsigned)blocks, RC_THREADS, 0, stream>>>(codes, scales, npoints,
-                                                                              C, d, k_max, W_hat);
+        reconstruct_vec4_kernel<<<(unsigned)blocks, RC_THREADS, 0, stream>>>(
+            codes, scales, npoints, center, C, d, k_max, W_hat);
     else
-        reconstruct_kernel<<<(unsigned)blocks, RC_THREADS, 0, stream>>>(codes, scales, npoints, C,
-                                                                         d, k_max, W_hat);
+        reconstruct_kernel<<<(unsigned)blocks, RC_THREADS, 0, stream>>>(
+            codes, scales, npoints, center, C, d, k_max, W_hat);
     return cuda_status(cudaGetLastError(), "reconstruct kernel launch");
 }
 

@@ -1,5 +1,6 @@
 """One layer through the whole hot path: greedy points (Algorithm 1), output error (Eq. 11),
-point allocation (Algorithm 2), multipoint weights (Eq. 4).
+point allocation (Algorithm 2), multipoint weights (Eq. 4); with asymmetric sets (Eq. 1, B != 0)
+the weights are centred first and the points approximate the centred weights.
 
 ``LayerPlan`` owns the device output buffers of one layer so that repeated runs allocate nothing;
 ``run_device`` enqueues the four C-ABI calls on one stream; ``run_host`` is the end-to-end call
@@ -26,6 +27,7 @@ class LayerSpec:
     k_max: int = 4
     mode: int = binding.MPQ_ALLOC_BUDGET
     budget_or_eps: float = 1.5
+    center: int = -1        # -1 symmetric sets, else MPQ_CENTER_PER_CHANNEL / _PER_LAYER
 
 
 class LayerPlan:
@@ -41,29 +43,39 @@ class LayerPlan:
         self.points_used = torch.empty((1,), dtype=torch.int32, device=dev)
         self.W_hat = torch.empty((s.C, s.d), dtype=torch.float32, device=dev) \
             if with_reconstruct else None
+        self.center = self.Wc = None
+        if s.center >= 0:
+            self.center = torch.empty((s.C,), dtype=torch.float32, device=dev)
+            self.Wc = torch.empty((s.C, s.d), dtype=torch.float32, device=dev)
         self._host = None
 
     # -- device-resident inputs ---------------------------------------------------------------
     def run_device(self, W, X, stream=None, grid_frac=None, timing=None):
-        """Enqueue the four calls on ``stream``.  timing(phase), if given, is called before the
-        first call (phase 0) and after call k (phase k = 1..4), e.g. to record CUDA events."""
+        """Enqueue the four calls (five with centring) on ``stream``.  timing(phase), if given, is
+        called before the first call (phase 0) and after the centring (1, also when there is
+        none), the greedy points (2), the output error (3), the allocation (4) and the
+        reconstruction (5), e.g. to record CUDA events."""
         s = self.spec
         tick = timing or (lambda ph: None)
         tick(0)
+        if self.center is not None:
+            binding.mpq_center_weights(W, s.center, center=self.center, Wc=self.Wc, stream=stream)
+            W = self.Wc
+        tick(1)
         binding.mpq_quantize_layer(W, s.bits, s.G, s.k_max, grid_frac=grid_frac, codes=self.codes,
                                    scales=self.scales, resid_sq=self.resid_sq, stream=stream)
-        tick(1)
+        tick(2)
         binding.mpq_output_error(X, W, self.codes, self.scales, s.k_max, groups=s.groups,
                                  err=self.err, stream=stream)
-        tick(2)
+        tick(3)
         binding.mpq_allocate_points(self.err, s.k_max, s.mode, s.budget_or_eps,
                                     npoints=self.npoints, points_used=self.points_used,
                                     stream=stream)
-        tick(3)
+        tick(4)
         if self.W_hat is not None:
             binding.mpq_reconstruct(self.codes, self.scales, self.npoints, W_hat=self.W_hat,
-                                    stream=stream)
-        tick(4)
+                                    stream=stream, center=self.center)
+        tick(5)
         return self
 
     # -- host inputs / outputs (end to end) ----------------------------------------------------
@@ -76,6 +88,8 @@ class LayerPlan:
                               scales=mk((s.C, s.k_max), torch.float32),
                               npoints=mk((s.C,), torch.int32),
                               points_used=mk((1,), torch.int32))
+            if self.center is not None:
+                self._host["center"] = mk((s.C,), torch.float32)
         return self._host
 
     def run_host(self, W_host, X_host, W_dev, X_dev, stream=None):
@@ -91,6 +105,8 @@ class LayerPlan:
             h["scales"].copy_(self.scales, non_blocking=True)
             h["npoints"].copy_(self.npoints, non_blocking=True)
             h["points_used"].copy_(self.points_used, non_blocking=True)
+            if self.center is not None:
+                h["center"].copy_(self.center, non_blocking=True)
         return h
 
     def h2d_bytes(self, W, X) -> int:
@@ -98,7 +114,8 @@ class LayerPlan:
 
     def d2h_bytes(self) -> int:
         s = self.spec
-        return s.k_max * s.C * s.d + 4 * s.C * s.k_max + 4 * s.C + 4
+        return s.k_max * s.C * s.d + 4 * s.C * s.k_max + 4 * s.C + 4 + \
+            (4 * s.C if self.center is not None else 0)
 
 
 class NetworkPlan:
@@ -131,7 +148,7 @@ class NetworkPlan:
 
     def run_device(self, Ws, Xs, stream=None, on_layer=None):
         """Ws[i], Xs[i]: device inputs of layer i.  on_layer(i, stream, phase), if given, is
-        called around layer i's calls as LayerPlan.run_device's timing hook (phases 0..4)."""
+        called around layer i's calls as LayerPlan.run_device's timing hook (phases 0..5)."""
         main = stream or torch.cuda.current_stream(self.device)
         self._fork(main)
         for n, i in enumerate(self.order):

@@ -30,7 +30,8 @@ def lib():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for n in ("mpq_quantize_layer", "mpq_output_error", "mpq_allocate_points", "mpq_reconstruct",
-              "mpq_clip_search"):
+              "mpq_clip_search", "mpq_center_weights", "mpq_pack_layout", "mpq_pack_points",
+              "mpq_multipoint_linear"):
         assert n in names
 
 
@@ -76,7 +77,8 @@ def test_quantize_rejects_bad_grid(lib, grid):
 def test_empty_layer_is_a_no_op(lib):
     assert lib.mpq_quantize_layer(None, 0, 16, 4, 8, None, 2, None, None, None, None, None) == 0
     assert lib.mpq_output_error(None, 5, 1, None, None, None, 0, 16, 2, None, None) == 0
-    assert lib.mpq_reconstruct(None, None, None, 0, 16, 2, None, None) == 0
+    assert lib.mpq_reconstruct(None, None, None, None, 0, 16, 2, None, None) == 0
+    assert lib.mpq_center_weights(None, 0, 16, 0, None, None, None) == 0
 
 
 @pytest.mark.parametrize("args,status", [
@@ -101,8 +103,20 @@ def test_allocate_requires_outputs(lib):
 
 
 def test_reconstruct_validation(lib):
-    assert lib.mpq_reconstruct(FAKE, FAKE, None, 4, 16, 2, FAKE, None) == 1
-    assert lib.mpq_reconstruct(FAKE, FAKE, FAKE, 4, 16, 0, FAKE, None) == 1
+    assert lib.mpq_reconstruct(FAKE, FAKE, None, None, 4, 16, 2, FAKE, None) == 1
+    assert lib.mpq_reconstruct(FAKE, FAKE, FAKE, FAKE, 4, 16, 0, FAKE, None) == 1
+
+
+@pytest.mark.parametrize("kwargs,status", [
+    (dict(mode=2), 1), (dict(mode=-1), 1), (dict(d=0), 1), (dict(C=-1), 1), (dict(W=None), 1),
+    (dict(center=None), 1), (dict(Wc=None), 1),
+])
+def test_center_validation(lib, kwargs, status):
+    a = dict(W=FAKE, C=4, d=16, mode=1, center=FAKE, Wc=FAKE)
+    a.update(kwargs)
+    assert lib.mpq_center_weights(a["W"], a["C"], a["d"], a["mode"], a["center"], a["Wc"],
+                                  None) == status
+    assert lib.mpq_last_error() != b""
 
 
 @pytest.mark.parametrize("kwargs,status", [
@@ -127,33 +141,41 @@ def test_clip_search_empty_layer(lib):
 def test_pack_layout_groups_channels(lib):
     """Host-only layout: channels grouped by the power of two >= n_k (n_k = 0 takes one row), 128/R
     channels per 128-row tile, rows padded to 64 elements, byte offsets in order."""
-    assert ctypes.sizeof(binding.PackedLayout) == 8 * 4 + 6 * 8
+    assert ctypes.sizeof(binding.PackedLayout) == 10 * 4 + 7 * 8   # 9 ints + padding, 7 size_t
     npts = [1] * 200 + [2] * 70 + [3] * 5 + [0] * 3 + [16]
     lay = binding.mpq_pack_layout(npts, 100, 16, 4, 12)
     tiles = -(-203 // 128) + -(-70 // 64) + -(-5 // 32) + 1   # R = 1, 2, 4, 16
     assert (lay.C, lay.d, lay.d_pad, lay.tiles, lay.rows) == (279, 100, 128, tiles, 128 * tiles)
-    assert lay.off_coef < lay.off_chan < lay.off_point < lay.off_tile < lay.off_codes < lay.bytes
+    assert lay.centered == 0
+    assert lay.off_coef < lay.off_chan < lay.off_point < lay.off_tile <= lay.off_center
+    assert lay.off_center < lay.off_codes < lay.bytes
     assert lay.off_codes % 1024 == 0
     assert lay.bytes == lay.off_codes + lay.rows * lay.d_pad * 2
+    cen = binding.mpq_pack_layout(npts, 100, 16, 4, 12, centered=True)
+    assert cen.centered == 1 and cen.off_center == lay.off_center
+    assert cen.off_codes >= cen.off_center + 279 * 4 and cen.off_codes % 1024 == 0
 
 
 @pytest.mark.parametrize("kwargs,status", [
     (dict(p=31), 1), (dict(p=-1), 1), (dict(bits=1), 1), (dict(bits=9), 3), (dict(k_max=17), 3),
-    (dict(d=0), 1), (dict(npoints=None), 1), (dict(layout=None), 1),
+    (dict(d=0), 1), (dict(npoints=None), 1), (dict(layout=None), 1), (dict(centered=2), 1),
 ])
 def test_pack_layout_validation(lib, kwargs, status):
     n = (ctypes.c_int * 3)(1, 2, 3)
     lay = binding.PackedLayout()
-    a = dict(npoints=n, C=3, d=32, k_max=4, bits=4, p=12, layout=ctypes.byref(lay))
+    a = dict(npoints=n, C=3, d=32, k_max=4, bits=4, p=12, centered=0, layout=ctypes.byref(lay))
     a.update(kwargs)
     assert lib.mpq_pack_layout(a["npoints"], a["C"], a["d"], a["k_max"], a["bits"], a["p"],
-                               a["layout"]) == status
+                               a["centered"], a["layout"]) == status
 
 
 def test_pack_and_linear_validation(lib):
     lay = binding.mpq_pack_layout([1, 2], 32, 4, 4, 12)
-    assert lib.mpq_pack_points(None, FAKE, FAKE, ctypes.byref(lay), FAKE, None) == 1
-    assert lib.mpq_pack_points(FAKE, FAKE, FAKE, None, FAKE, None) == 1
+    assert lib.mpq_pack_points(None, FAKE, None, FAKE, ctypes.byref(lay), FAKE, None) == 1
+    assert lib.mpq_pack_points(FAKE, FAKE, None, FAKE, None, FAKE, None) == 1
+    assert lib.mpq_pack_points(FAKE, FAKE, FAKE, FAKE, ctypes.byref(lay), FAKE, None) == 1  # not centred
+    cen = binding.mpq_pack_layout([1, 2], 32, 4, 4, 12, centered=True)
+    assert lib.mpq_pack_points(FAKE, FAKE, None, FAKE, ctypes.byref(cen), FAKE, None) == 1
     assert lib.mpq_multipoint_linear(FAKE, 0, ctypes.byref(lay), FAKE, FAKE, None) == 1
     assert lib.mpq_multipoint_linear(None, 4, ctypes.byref(lay), FAKE, FAKE, None) == 1
     assert lib.mpq_multipoint_linear(FAKE, 4, None, FAKE, FAKE, None) == 1
