@@ -59,7 +59,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--graph", type=int, default=1,
                     help="replay the multi-stream step as a captured CUDA graph (1) or launch it (0)")
-    ap.add_argument("--streams", type=int, default=8,
+    ap.add_argument("--streams", type=int, default=12,
                     help="CUDA streams the independent layers are spread over")
     ap.add_argument("--layers", default=None,
                     help="comma-separated layer indices to run (profiling a subset); default all")

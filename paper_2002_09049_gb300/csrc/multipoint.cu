@@ -80,6 +80,8 @@ struct LinCtrl {
     int abort;
     int coef[L_MAX_RT][L_M];      // the row coefficients A of this CTA's tiles
     int xsum[L_N];                // sum_j x_tj of this CTA's inputs (centred layers)
+    int out[4][32][33];           // per epilogue warp: 32 channels x 32 outputs, for the stores
+    int kch[4][32];               // per epilogue warp: the channel of each lane's row (-1: none)
 };
 constexpr int L_CTRL_BYTES = (sizeof(LinCtrl) + 1023) / 1024 * 1024;
 template <int RT>
@@ -268,6 +270,9 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             const long long a = ctl.coef[u][r];
             const long long ab = centered && k >= 0 ? (long long)center_coef[k] : 0;
             const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16) + (uint32_t)(u * L_N);
+            // the rows this warp writes: one per channel (its first lane), -1 for none
+            ctl.kch[ew][lane] = (lane & (R - 1)) == 0 ? k : -1;
+            __syncwarp();
 #pragma unroll 1
             for (int cb = 0; cb < L_N / 32; ++cb) {
                 float v[32];
@@ -279,16 +284,37 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
 #pragma unroll
                     for (int j = 0; j < 32; ++j) sum[j] += __shfl_xor_sync(0xffffffffu, sum[j], o);
                 }
-                if ((lane & (R - 1)) == 0 && k >= 0) {
-                    const int t0 = n0 + cb * 32;
-                    int32_t *y = Y + (size_t)k * T + t0;
+                if (centered) {   // the row sums first: no shared-memory store comes before them
+                    int xs[32];
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const long long tot = sum[j] + ab * (long long)ctl.xsum[cb * 32 + j];
-                        long long z = tot >> p;   // arithmetic shift: floor division by 2^p
-                        z = z > 2147483647LL ? 2147483647LL : (z < -2147483648LL ? -2147483648LL : z);
-                        if (t0 + j < T) y[j] = (int32_t)z;
-                    }
+                    for (int j = 0; j < 32; ++j) xs[j] = ctl.xsum[cb * 32 + j];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) sum[j] += ab * (long long)xs[j];
+                }
+                int zr[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    long long z = sum[j] >> p;   // arithmetic shift: floor division by 2^p
+                    z = z > 2147483647LL ? 2147483647LL : (z < -2147483648LL ? -2147483648LL : z);
+                    zr[j] = (int)z;
+                }
+#pragma unroll
+                for (int j = 0; j < 32; ++j) ctl.out[ew][lane][j] = zr[j];
+                __syncwarp();
+                // one channel's 32 consecutive outputs per store: 128 contiguous bytes; every
+                // shared-memory read is issued before the first store
+                int kv[32], ov[32];
+#pragma unroll
+                for (int L = 0; L < 32; ++L) {
+                    kv[L] = ctl.kch[ew][L];
+                    ov[L] = ctl.out[ew][L][lane];
+                }
+                __syncwarp();
+                const int t = n0 + cb * 32 + lane;
+                if (t < T) {
+#pragma unroll
+                    for (int L = 0; L < 32; ++L)
+                        if (kv[L] >= 0) Y[(size_t)kv[L] * T + t] = ov[L];
                 }
             }
         }
