@@ -18,7 +18,10 @@
 // integer kernel below).  A CTA takes RT 128-row tiles against 256 inputs (RT accumulators of 256
 // TMEM columns): two on large layers, so each converted input tile feeds both, one on small layers
 // for more CTAs; K chunks of 64.  The inputs vary fastest in the grid, so the CTAs that share a row
-// tile run together and read its codes from L2.
+// tile run together and read its codes from L2.  Codes tiles, raw input tiles and bf16 input tiles
+// have rings of their own, so each kind of load runs as far ahead as its latency needs: a raw tile
+// is handed back as soon as the producers have read it, the others when the MMAs reading them
+// complete.
 // Steps 2 and 3 in the epilogue: each lane turns its accumulator into an integer, multiplies by its
 // row's coefficient in 64 bits, the R lanes of a channel add with warp shuffles, and the first lane
 // shifts (arithmetic: floor), saturates and writes 32 consecutive outputs.  Every wait is bounded.
@@ -53,39 +56,50 @@ constexpr int L_B_BYTES = L_N * L_KC * 2;       // 32 KB input tile (bf16)
 constexpr int L_RAW_BYTES = L_N * L_KC;         // 16 KB input tile (int8, as loaded)
 constexpr int L_MAX_RT = 2;
 
-// Stage layout for RT row tiles per CTA: RT codes tiles, the bf16 input tile, the raw input tile.
+// Three rings, each as deep as its own latency needs: codes tiles (TMA, freed by the MMAs), raw
+// int8 input tiles (TMA, freed as soon as the producers have read them) and bf16 input tiles
+// (written by the producers, freed by the MMAs).  208 KB for RT = 1 and RT = 2.
+constexpr int L_MAX_SLOTS = 4;
 template <int RT>
 struct LGeo {
-    static constexpr int STAGES = RT == 1 ? 3 : 2;
-    static constexpr int OFF_B = RT * L_A_BYTES;
-    static constexpr int OFF_RAW = OFF_B + L_B_BYTES;
-    static constexpr int STAGE_BYTES = OFF_RAW + L_RAW_BYTES;   // 64 or 80 KB
+    static constexpr int A_SLOTS = RT == 1 ? 4 : 3;
+    static constexpr int A_SLOT = RT * L_A_BYTES;
+    static constexpr int B_SLOTS = RT == 1 ? 3 : 2;
+    static constexpr int R_SLOTS = 3;
+    static constexpr int OFF_B = A_SLOTS * A_SLOT;
+    static constexpr int OFF_RAW = OFF_B + B_SLOTS * L_B_BYTES;
+    static constexpr int BYTES = OFF_RAW + R_SLOTS * L_RAW_BYTES;
     static constexpr uint32_t TMEM_COLS = RT * L_N;
 };
 constexpr int L_PROD_WARPS = 8;
 constexpr int L_PROD_THREADS = L_PROD_WARPS * 32;
 constexpr int L_EPI_WARP0 = L_PROD_WARPS;       // warps 8..11: warp % 4 selects TMEM lanes
 constexpr int L_MMA_WARP = L_EPI_WARP0 + 4;
-constexpr int L_TMA_WARP = L_MMA_WARP + 1;
-constexpr int L_THREADS = (L_TMA_WARP + 1) * 32;   // 448
+constexpr int L_TMA_A_WARP = L_MMA_WARP + 1;    // codes tiles
+constexpr int L_TMA_X_WARP = L_TMA_A_WARP + 1;  // raw input tiles
+constexpr int L_THREADS = (L_TMA_X_WARP + 1) * 32;   // 480
 constexpr long long L_WAIT = 1LL << 31;
 
 struct LinCtrl {
-    uint64_t loaded[3];           // TMA bytes of a stage have landed
-    uint64_t full[3];             // producers converted the input tile
-    uint64_t empty[3];            // MMAs on the stage completed
-    uint64_t done;                // every MMA completed
-    uint64_t xs_ready;            // producers stored the input-row sums
+    uint64_t a_full[L_MAX_SLOTS];     // a codes slot has landed
+    uint64_t a_empty[L_MAX_SLOTS];    // the MMAs reading a codes slot completed
+    uint64_t b_full[L_MAX_SLOTS];     // producers wrote a bf16 input slot
+    uint64_t b_empty[L_MAX_SLOTS];    // the MMAs reading a bf16 input slot completed
+    uint64_t r_full[L_MAX_SLOTS];     // a raw input slot has landed
+    uint64_t r_empty[L_MAX_SLOTS];    // producers read a raw input slot
+    uint64_t done;                    // every MMA completed
+    uint64_t xs_ready;                // producers stored the input-row sums
     uint32_t tmem_base;
     int abort;
-    int coef[L_MAX_RT][L_M];      // the row coefficients A of this CTA's tiles
-    int xsum[L_N];                // sum_j x_tj of this CTA's inputs (centred layers)
-    int out[4][32][33];           // per epilogue warp: 32 channels x 32 outputs, for the stores
-    int kch[4][32];               // per epilogue warp: the channel of each lane's row (-1: none)
+    int coef[L_MAX_RT][L_M];          // the row coefficients A of this CTA's tiles
+    int xsum[L_N];                    // sum_j x_tj of this CTA's inputs (centred layers)
+    int kch[4][32];                   // per epilogue warp: the channel of each lane's row (-1: none)
 };
 constexpr int L_CTRL_BYTES = (sizeof(LinCtrl) + 1023) / 1024 * 1024;
 template <int RT>
-constexpr int lin_smem() { return 1024 + L_CTRL_BYTES + LGeo<RT>::STAGES * LGeo<RT>::STAGE_BYTES; }
+constexpr int lin_smem() { return 1024 + L_CTRL_BYTES + LGeo<RT>::BYTES; }
+// the epilogue's staging (4 warps x 32 x 33 ints) reuses the bf16 input ring once every MMA is done
+static_assert(4 * 32 * 33 * 4 <= 2 * L_B_BYTES, "epilogue staging fits the bf16 ring");
 
 // Row r of a packed buffer: (channel, point) or channel -1 / point -1 for padding.
 struct PackView {
@@ -158,38 +172,41 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                          const __grid_constant__ CUtensorMap tmX)
 {
     using G = LGeo<RT>;
-    constexpr int L_STAGES = G::STAGES;
-    constexpr int L_STAGE_BYTES = G::STAGE_BYTES;
-    constexpr int L_OFF_B = G::OFF_B;
-    constexpr int L_OFF_RAW = G::OFF_RAW;
-    constexpr uint32_t L_TMEM_COLS = G::TMEM_COLS;
-    constexpr int L_RT = RT;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
     LinCtrl &ctl = *reinterpret_cast<LinCtrl *>(smem_raw + pad);
-    const uint32_t stages_u32 = raw_u32 + pad + L_CTRL_BYTES;
+    unsigned char *ring = smem_raw + pad + L_CTRL_BYTES;
+    const uint32_t ring_u32 = raw_u32 + pad + L_CTRL_BYTES;
+    const uint32_t a_u32 = ring_u32, b_u32 = ring_u32 + G::OFF_B, x_u32 = ring_u32 + G::OFF_RAW;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // inputs vary fastest: the CTAs sharing a row tile run together and read its codes from L2
-    const int tile0 = blockIdx.y * L_RT, n0 = blockIdx.x * L_N;
-    const int nt = min(L_RT, tiles - tile0);        // row tiles of this CTA (the last may hold one)
+    const int tile0 = blockIdx.y * RT, n0 = blockIdx.x * L_N;
+    const int nt = min(RT, tiles - tile0);          // row tiles of this CTA (the last may hold one)
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < L_STAGES; ++s) {
-            mbar_init(&ctl.loaded[s], 1);
-            mbar_init(&ctl.full[s], L_PROD_WARPS);
-            mbar_init(&ctl.empty[s], 1);
+        for (int i = 0; i < G::A_SLOTS; ++i) {
+            mbar_init(&ctl.a_full[i], 1);
+            mbar_init(&ctl.a_empty[i], 1);
+        }
+        for (int i = 0; i < G::B_SLOTS; ++i) {
+            mbar_init(&ctl.b_full[i], L_PROD_WARPS);
+            mbar_init(&ctl.b_empty[i], 1);
+        }
+        for (int i = 0; i < G::R_SLOTS; ++i) {
+            mbar_init(&ctl.r_full[i], 1);
+            mbar_init(&ctl.r_empty[i], L_PROD_WARPS);
         }
         mbar_init(&ctl.done, 1);
         mbar_init(&ctl.xs_ready, L_PROD_WARPS);
         ctl.abort = 0;
         fence_barrier_init();
     }
-    for (int r = threadIdx.x; r < L_RT * L_M; r += L_THREADS)
+    for (int r = threadIdx.x; r < RT * L_M; r += L_THREADS)
         ctl.coef[r / L_M][r % L_M] = r / L_M < nt ? coef[(size_t)tile0 * L_M + r] : 0;
     if (warp == L_MMA_WARP) {
-        tmem_alloc(&ctl.tmem_base, L_TMEM_COLS);
+        tmem_alloc(&ctl.tmem_base, G::TMEM_COLS);
         tc_fence_before();
     }
     __syncthreads();
@@ -205,28 +222,36 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
 #pragma unroll
         for (int it = 0; it < ITEMS; ++it) xs[it] = 0;
         for (int kc = 0; kc < n_kc; ++kc) {
-            const int s = kc % L_STAGES;
-            const uint32_t ph = (uint32_t)(kc / L_STAGES) & 1u;
-            const bool ok = mbar_wait(&ctl.loaded[s], ph, L_WAIT);
+            const int rs = kc % G::R_SLOTS, bs = kc % G::B_SLOTS;
+            bool ok = mbar_wait(&ctl.r_full[rs], (uint32_t)(kc / G::R_SLOTS) & 1u, L_WAIT);
+            if (ok && kc >= G::B_SLOTS)
+                ok = mbar_wait(&ctl.b_empty[bs], (uint32_t)(kc / G::B_SLOTS - 1) & 1u, L_WAIT);
             if (!ok) *abort_flag = 1;
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-            const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
-            // 16 input bytes (one input row, 16 K elements) per item, 4 items per thread
+            // 16 input bytes (one input row, 16 K elements) per item, 4 items per thread: all
+            // reads first, then the raw slot goes back to the TMA thread
+            float4 raw[ITEMS];
+#pragma unroll
+            for (int it = 0; it < ITEMS; ++it)
+                raw[it] = ld_shared_v4(x_u32 + rs * L_RAW_BYTES +
+                                       (uint32_t)(threadIdx.x + it * L_PROD_THREADS) * 16u);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl.r_empty[rs]);
+            const uint32_t bb = b_u32 + bs * L_B_BYTES;
 #pragma unroll
             for (int it = 0; it < ITEMS; ++it) {
                 const int q = threadIdx.x + it * L_PROD_THREADS;
                 const int row = q >> 2, c16 = q & 3;
-                const float4 raw = ld_shared_v4(sb + L_OFF_RAW + (uint32_t)q * 16u);
                 if (centered) {   // signed bytes summed exactly (|sum| <= 128 d)
-                    xs[it] = __dp4a(__float_as_int(raw.x), 0x01010101, xs[it]);
-                    xs[it] = __dp4a(__float_as_int(raw.y), 0x01010101, xs[it]);
-                    xs[it] = __dp4a(__float_as_int(raw.z), 0x01010101, xs[it]);
-                    xs[it] = __dp4a(__float_as_int(raw.w), 0x01010101, xs[it]);
+                    xs[it] = __dp4a(__float_as_int(raw[it].x), 0x01010101, xs[it]);
+                    xs[it] = __dp4a(__float_as_int(raw[it].y), 0x01010101, xs[it]);
+                    xs[it] = __dp4a(__float_as_int(raw[it].z), 0x01010101, xs[it]);
+                    xs[it] = __dp4a(__float_as_int(raw[it].w), 0x01010101, xs[it]);
                 }
-                const uint32_t w[4] = {__float_as_uint(raw.x) ^ 0x80808080u,
-                                       __float_as_uint(raw.y) ^ 0x80808080u,
-                                       __float_as_uint(raw.z) ^ 0x80808080u,
-                                       __float_as_uint(raw.w) ^ 0x80808080u};
+                const uint32_t w[4] = {__float_as_uint(raw[it].x) ^ 0x80808080u,
+                                       __float_as_uint(raw[it].y) ^ 0x80808080u,
+                                       __float_as_uint(raw[it].z) ^ 0x80808080u,
+                                       __float_as_uint(raw[it].w) ^ 0x80808080u};
                 float4 o0, o1;
                 o0.x = __uint_as_float(bf16x2_from_biased(w[0], 0));
                 o0.y = __uint_as_float(bf16x2_from_biased(w[0], 2));
@@ -236,12 +261,12 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                 o1.y = __uint_as_float(bf16x2_from_biased(w[2], 2));
                 o1.z = __uint_as_float(bf16x2_from_biased(w[3], 0));
                 o1.w = __uint_as_float(bf16x2_from_biased(w[3], 2));
-                st_shared_v4(sb + L_OFF_B + sw128_offset(row, 2 * c16), o0);
-                st_shared_v4(sb + L_OFF_B + sw128_offset(row, 2 * c16 + 1), o1);
+                st_shared_v4(bb + sw128_offset(row, 2 * c16), o0);
+                st_shared_v4(bb + sw128_offset(row, 2 * c16 + 1), o1);
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&ctl.full[s]);
+            if (lane == 0) mbar_arrive(&ctl.b_full[bs]);
         }
         if (centered) {
             // the 4 threads of an input row (lanes 4m..4m+3) hold its 4 column shares
@@ -263,6 +288,8 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
         if (!ok) *abort_flag = 1;
         const bool good = !__any_sync(0xffffffffu, !ok || *abort_flag);
         tc_fence_after();
+        // staging for the stores: the bf16 input ring, idle once every MMA has completed
+        int (*out)[33] = reinterpret_cast<int (*)[33]>(ring + G::OFF_B) + ew * 32;
         for (int u = 0; u < nt && good; ++u) {
             const int R = tile_R[tile0 + u];
             const int r = ew * 32 + lane;
@@ -299,7 +326,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                     zr[j] = (int)z;
                 }
 #pragma unroll
-                for (int j = 0; j < 32; ++j) ctl.out[ew][lane][j] = zr[j];
+                for (int j = 0; j < 32; ++j) out[lane][j] = zr[j];
                 __syncwarp();
                 // one channel's 32 consecutive outputs per store: 128 contiguous bytes; every
                 // shared-memory read is issued before the first store
@@ -307,7 +334,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
 #pragma unroll
                 for (int L = 0; L < 32; ++L) {
                     kv[L] = ctl.kch[ew][L];
-                    ov[L] = ctl.out[ew][L][lane];
+                    ov[L] = out[L][lane];
                 }
                 __syncwarp();
                 const int t = n0 + cb * 32 + lane;
@@ -323,15 +350,15 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(L_M, L_N);
             for (int kc = 0; kc < n_kc; ++kc) {
-                const int s = kc % L_STAGES;
-                const uint32_t ph = (uint32_t)(kc / L_STAGES) & 1u;
-                if (!mbar_wait(&ctl.full[s], ph, L_WAIT)) *abort_flag = 1;
+                const int as = kc % G::A_SLOTS, bs = kc % G::B_SLOTS;
+                bool ok = mbar_wait(&ctl.a_full[as], (uint32_t)(kc / G::A_SLOTS) & 1u, L_WAIT);
+                if (ok) ok = mbar_wait(&ctl.b_full[bs], (uint32_t)(kc / G::B_SLOTS) & 1u, L_WAIT);
+                if (!ok) *abort_flag = 1;
                 if (*abort_flag) break;
                 tc_fence_after();
-                const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
-                const uint64_t bd = smem_desc_sw128(sb + L_OFF_B);
+                const uint64_t bd = smem_desc_sw128(b_u32 + bs * L_B_BYTES);
                 for (int u = 0; u < nt; ++u) {
-                    const uint64_t ad = smem_desc_sw128(sb + u * L_A_BYTES);
+                    const uint64_t ad = smem_desc_sw128(a_u32 + as * G::A_SLOT + u * L_A_BYTES);
 #pragma unroll
                     for (int kk = 0; kk < L_KC / 16; ++kk) {
                         const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
@@ -339,34 +366,51 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                                  (kc > 0 || kk > 0) ? 1u : 0u);
                     }
                 }
-                mma_commit(&ctl.empty[s]);
+                mma_commit(&ctl.a_empty[as]);
+                mma_commit(&ctl.b_empty[bs]);
             }
             mma_commit(&ctl.done);
         }
         __syncwarp();
-    } else {
-        // ---------------------------------------------------------------- TMA: codes and inputs
+    } else if (warp == L_TMA_A_WARP) {
+        // ---------------------------------------------------------------- TMA: codes tiles
         if (lane == 0) {
             prefetch_tensormap(&tmA);
-            prefetch_tensormap(&tmX);
             int issued = 0;
             for (int kc = 0; kc < n_kc; ++kc) {
-                const int s = kc % L_STAGES;
-                if (kc >= L_STAGES &&
-                    !mbar_wait(&ctl.empty[s], (uint32_t)(kc / L_STAGES - 1) & 1u, L_WAIT))
+                const int as = kc % G::A_SLOTS;
+                if (kc >= G::A_SLOTS &&
+                    !mbar_wait(&ctl.a_empty[as], (uint32_t)(kc / G::A_SLOTS - 1) & 1u, L_WAIT))
                     *abort_flag = 1;
                 if (*abort_flag) break;
-                const uint32_t sb = stages_u32 + s * L_STAGE_BYTES;
-                mbar_arrive_expect_tx(&ctl.loaded[s], (uint32_t)(nt * L_A_BYTES + L_RAW_BYTES));
+                mbar_arrive_expect_tx(&ctl.a_full[as], (uint32_t)(nt * L_A_BYTES));
                 for (int u = 0; u < nt; ++u)
-                    tma_load_2d(sb + u * L_A_BYTES, &tmA, kc * L_KC, (tile0 + u) * L_M,
-                                &ctl.loaded[s]);
-                tma_load_2d(sb + L_OFF_RAW, &tmX, kc * L_KC, n0, &ctl.loaded[s]);
+                    tma_load_2d(a_u32 + as * G::A_SLOT + u * L_A_BYTES, &tmA, kc * L_KC,
+                                (tile0 + u) * L_M, &ctl.a_full[as]);
                 issued = kc + 1;
             }
             // no copy may land after the CTA is gone
-            for (int kc = issued - L_STAGES > 0 ? issued - L_STAGES : 0; kc < issued; ++kc)
-                mbar_wait(&ctl.loaded[kc % L_STAGES], (uint32_t)(kc / L_STAGES) & 1u, L_WAIT);
+            for (int kc = issued - G::A_SLOTS > 0 ? issued - G::A_SLOTS : 0; kc < issued; ++kc)
+                mbar_wait(&ctl.a_full[kc % G::A_SLOTS], (uint32_t)(kc / G::A_SLOTS) & 1u, L_WAIT);
+        }
+        __syncwarp();
+    } else {
+        // ---------------------------------------------------------------- TMA: raw input tiles
+        if (lane == 0) {
+            prefetch_tensormap(&tmX);
+            int issued = 0;
+            for (int kc = 0; kc < n_kc; ++kc) {
+                const int rs = kc % G::R_SLOTS;
+                if (kc >= G::R_SLOTS &&
+                    !mbar_wait(&ctl.r_empty[rs], (uint32_t)(kc / G::R_SLOTS - 1) & 1u, L_WAIT))
+                    *abort_flag = 1;
+                if (*abort_flag) break;
+                mbar_arrive_expect_tx(&ctl.r_full[rs], (uint32_t)L_RAW_BYTES);
+                tma_load_2d(x_u32 + rs * L_RAW_BYTES, &tmX, kc * L_KC, n0, &ctl.r_full[rs]);
+                issued = kc + 1;
+            }
+            for (int kc = issued - G::R_SLOTS > 0 ? issued - G::R_SLOTS : 0; kc < issued; ++kc)
+                mbar_wait(&ctl.r_full[kc % G::R_SLOTS], (uint32_t)(kc / G::R_SLOTS) & 1u, L_WAIT);
         }
         __syncwarp();
     }
@@ -377,7 +421,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
         if (lane == 0 && *abort_flag) mbar_wait(&ctl.done, 0, L_WAIT);
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem, L_TMEM_COLS);
+        tmem_dealloc(tmem, G::TMEM_COLS);
     }
 }
 
