@@ -117,12 +117,17 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
 {
     using G = PGeo<KP1, CLIP>;
     constexpr int K = G::K;
+    static_assert(G::X_ITEMS * P_PROD_THREADS == P_ROWS * P_KC4, "X items cover the chunk");
+    // every shared-memory read of a group before its stores (the accessors are ordered), so the
+    // reads' latencies overlap instead of adding up
+    float4 xr[G::X_ITEMS];
+#pragma unroll
+    for (int i = 0; i < G::X_ITEMS; ++i) xr[i] = ld_shared_v4(slot + (uint32_t)(pt + i * P_PROD_THREADS) * 16u);
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
         const int q = pt + i * P_PROD_THREADS;
-        if (G::X_ITEMS * P_PROD_THREADS != P_ROWS * P_KC4 && q >= P_ROWS * P_KC4) break;
         float4 hi, lo;
-        split4(ld_shared_v4(slot + (uint32_t)q * 16u), hi, lo);
+        split4(xr[i], hi, lo);
         const uint32_t off = sw128_offset(q / P_KC4, q % P_KC4);
         st_shared_v4(sb + P_OFF_B_HI + off, hi);
         st_shared_v4(sb + P_OFF_B_LO + off, lo);
@@ -157,28 +162,44 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
     if constexpr (CLIP) {
         // (candidate, channel, element pair) units over all producer threads, element pairs
         // lane-contiguous: each warp store fills whole 128-byte rows.
+        constexpr int STEP = P_PROD_THREADS / (P_KC / 2);   // rows between a thread's units
+        constexpr int UNITS = P_VEC / STEP;                 // at most 8 units per thread
         const int rows = nch * KP1;                     // row = c * nch + ch
         const int e2 = pt % (P_KC / 2);                  // the same for all of this thread's units
-        int row = pt / (P_KC / 2);
-        int c = nch > 0 ? row / nch : 0, ch = nch > 0 ? row - c * nch : 0;
-        for (; row < rows; row += P_PROD_THREADS / (P_KC / 2)) {
-            const float2 w = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
-            const float s = ctl.clip_s[ch * KP1 + c], inv = ctl.clip_inv[ch * KP1 + c];
-            // exact code of Eq. 8 (0 when the scale is 0 or NaN: the residual is then w or NaN)
-            const float qx = s > 0.0f ? copysignf((float)code_fast(fabsf(w.x), s, inv, qmaxf), w.x) : 0.0f;
-            const float qy = s > 0.0f ? copysignf((float)code_fast(fabsf(w.y), s, inv, qmaxf), w.y) : 0.0f;
-            float2 r, hi, lo;
-            r.x = __fmaf_rn(-s, qx, w.x);
-            r.y = __fmaf_rn(-s, qy, w.y);
-            split2(r, hi, lo);
-            const uint32_t off = sw128_offset(ch * KP1 + c, e2 >> 1) + (uint32_t)(e2 & 1) * 8u;
-            st_shared_v2(sb + P_OFF_A_HI + off, hi);
-            st_shared_v2(sb + P_OFF_A_LO + off, lo);
-            ch += P_PROD_THREADS / (P_KC / 2);           // next row: advance (c, ch) without dividing
-            while (ch >= nch) {
+        const int row0 = pt / (P_KC / 2);
+        int c = nch > 0 ? row0 / nch : 0, ch = nch > 0 ? row0 - c * nch : 0;
+        // all reads first (weights, scales, reciprocals of every unit), then the residuals
+        float2 w[UNITS];
+        float sv[UNITS], iv[UNITS];
+        int arow[UNITS];
+#pragma unroll
+        for (int u = 0; u < UNITS; ++u) {
+            arow[u] = ch * KP1 + c;
+            if (row0 + u * STEP < rows) {
+                w[u] = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
+                sv[u] = ctl.clip_s[arow[u]];
+                iv[u] = ctl.clip_inv[arow[u]];
+            }
+            ch += STEP;                                  // next row: advance (c, ch) without dividing
+            while (ch >= nch && nch > 0) {
                 ch -= nch;
                 ++c;
             }
+        }
+#pragma unroll
+        for (int u = 0; u < UNITS; ++u) {
+            if (row0 + u * STEP >= rows) break;
+            const float s = sv[u], inv = iv[u];
+            // exact code of Eq. 8 (0 when the scale is 0 or NaN: the residual is then w or NaN)
+            const float qx = s > 0.0f ? copysignf((float)code_fast(fabsf(w[u].x), s, inv, qmaxf), w[u].x) : 0.0f;
+            const float qy = s > 0.0f ? copysignf((float)code_fast(fabsf(w[u].y), s, inv, qmaxf), w[u].y) : 0.0f;
+            float2 r, hi, lo;
+            r.x = __fmaf_rn(-s, qx, w[u].x);
+            r.y = __fmaf_rn(-s, qy, w[u].y);
+            split2(r, hi, lo);
+            const uint32_t off = sw128_offset(arow[u], e2 >> 1) + (uint32_t)(e2 & 1) * 8u;
+            st_shared_v2(sb + P_OFF_A_HI + off, hi);
+            st_shared_v2(sb + P_OFF_A_LO + off, lo);
         }
     }
 }
