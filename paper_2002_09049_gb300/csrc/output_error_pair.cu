@@ -21,8 +21,8 @@
 // (Eq. 7) from W, codes and scales into the A tiles (128-byte swizzled, K-major); residuals never
 // exist in global memory.  Both CTAs' producers report a full stage to the even CTA, whose MMA
 // thread issues the pair MMAs and signals both CTAs (multicast commits) when a stage or a segment
-// is consumed.  Four epilogue warps per CTA drain the segments; a segment is restarted only once
-// both CTAs' epilogues have released it.
+// is consumed.  Eight epilogue warps per CTA (one per TMEM lane quarter and column half) drain the
+// segments; a segment is restarted only once both CTAs' epilogues have released it.
 //
 // Row tiles (256 rows) are split over the pairs of a cluster of up to 8 CTAs; ranks 0 and 1 add
 // their peers' partial sums from distributed shared memory in rank order.  Every wait is bounded;
@@ -59,10 +59,11 @@ constexpr int P_OFF_B_LO = 3 * P_TILE;
 constexpr int P_STAGE_BYTES = 4 * P_TILE;       // 64 KB
 constexpr int P_PROD_WARPS = 8;
 constexpr int P_PROD_THREADS = P_PROD_WARPS * 32;
-constexpr int P_EPI_WARP0 = P_PROD_WARPS;       // warps 8..11: warp % 4 selects TMEM lanes
-constexpr int P_MMA_WARP = P_EPI_WARP0 + 4;
+constexpr int P_EPI_WARPS = 8;                  // two per TMEM lane quarter, one per column half
+constexpr int P_EPI_WARP0 = P_PROD_WARPS;       // warps 8..15: warp % 4 selects TMEM lanes
+constexpr int P_MMA_WARP = P_EPI_WARP0 + P_EPI_WARPS;
 constexpr int P_TMA_WARP = P_MMA_WARP + 1;
-constexpr int P_THREADS = (P_TMA_WARP + 1) * 32;   // 448
+constexpr int P_THREADS = (P_TMA_WARP + 1) * 32;   // 576
 constexpr uint32_t P_TMEM_COLS = 512;
 constexpr uint32_t P_RUN_COL = 256;
 constexpr int P_MAX_RAW = 3;
@@ -75,11 +76,11 @@ struct PairCtrl {
     uint64_t raw_full[P_MAX_RAW];
     uint64_t raw_empty[P_MAX_RAW];
     uint64_t segfull;             // both CTAs: pair MMA commit
-    uint64_t segempty;            // even CTA: both CTAs' epilogue warps
+    uint64_t segempty;            // even CTA: both CTAs' epilogue warps (16 arrivals)
     uint64_t done;                // even CTA
     uint32_t tmem_base;
     int abort;
-    double part[P_VEC];
+    double part[2][P_VEC];        // per column half: sum over the rows' y^2
     float clip_s[P_VEC];          // clipping search: scale K / Qmax and fl(1 / scale) per row
     float clip_inv[P_VEC];
 };
@@ -249,7 +250,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             mbar_init(&ctl.raw_empty[r], P_PROD_WARPS);
         }
         mbar_init(&ctl.segfull, 1);
-        mbar_init(&ctl.segempty, 2 * 4);
+        mbar_init(&ctl.segempty, 2 * P_EPI_WARPS);
         mbar_init(&ctl.done, 1);
         ctl.abort = 0;
         fence_barrier_init();
@@ -302,8 +303,9 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         }
     } else if (warp < P_MMA_WARP) {
         // ---------------------------------------------------------------- epilogue
-        const int ew = warp - P_EPI_WARP0;
-        const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16);
+        // lane quarter q (the TMEM lanes this warp may access) and column half h
+        const int ew = warp - P_EPI_WARP0, q = ew & 3, h = ew >> 2;
+        const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(h * (P_N / 2));
         double acc = 0.0;
         int g = 0;
         bool stop = false;
@@ -316,13 +318,14 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 tc_fence_after();
                 const bool first = (sg == 0), last = (sg == nseg - 1);
 #pragma unroll 1
-                for (int cb = 0; cb < P_N / 32; ++cb) {
+                for (int cb = 0; cb < P_N / 64; ++cb) {
                     const uint32_t col = (uint32_t)(cb * 32);
                     float v[32];
-                    tmem_ld_32x32b_x32(lane_base + col, v);
-                    if (!first) {
+                    if (first) {
+                        tmem_ld_32x32b_x32(lane_base + col, v);
+                    } else {   // segment and running sums loaded together
                         float r[32];
-                        tmem_ld_32x32b_x32(lane_base + P_RUN_COL + col, r);
+                        tmem_ld2_32x32b_x32(lane_base + col, lane_base + P_RUN_COL + col, v, r);
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] = __fadd_rn(v[i], r[i]);
                     }
@@ -341,7 +344,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 if (lane == 0) mbar_arrive_cluster(&ctl.segempty, leader);
             }
         }
-        ctl.part[ew * 32 + lane] = *abort_flag ? (double)NAN : acc;
+        ctl.part[h][q * 32 + lane] = *abort_flag ? (double)NAN : acc;
     } else if (warp == P_MMA_WARP) {
         // ---------------------------------------------------------------- MMA issuer (even CTA)
         if (half == 0 && lane == 0) {
@@ -418,11 +421,14 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
 
     // ---------------------------------------------------------------- cluster reduction
     cluster_sync();
-    if (crank < 2 && warp >= P_EPI_WARP0 && warp < P_MMA_WARP) {
+    if (crank < 2 && warp >= P_EPI_WARP0 && warp < P_EPI_WARP0 + 4) {
         const int m = (warp - P_EPI_WARP0) * 32 + lane;
         if (m < nvec) {
             double s = 0.0;
-            for (int j = 0; j < split; ++j) s += ld_dsmem_f64(&ctl.part[m], crank + 2u * (uint32_t)j);
+            for (int j = 0; j < split; ++j) {
+                s += ld_dsmem_f64(&ctl.part[0][m], crank + 2u * (uint32_t)j);
+                s += ld_dsmem_f64(&ctl.part[1][m], crank + 2u * (uint32_t)j);
+            }
             err[(size_t)k0 * KP1 + m] = (float)(s / (double)N);
         }
     }
