@@ -617,9 +617,12 @@ mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_lay
             set_error("multipoint linear: tensor map encoding failed");
             return MPQ_ERR_CUDA;
         }
-        // two row tiles per CTA when that still gives at least two waves of CTAs
-        const long long tt = (T + L_N - 1) / L_N;
-        const bool two = (long long)((L->tiles + 1) / 2) * tt >= 2LL * sm_count();
+        // two row tiles per CTA when that takes fewer waves of CTAs: such a CTA runs its K loop
+        // near the tensor rate but takes ~1.4x as long as a one-tile CTA (measured)
+        const long long tt = (T + L_N - 1) / L_N, sms = sm_count();
+        const long long w1 = ((long long)L->tiles * tt + sms - 1) / sms;
+        const long long w2 = ((long long)((L->tiles + 1) / 2) * tt + sms - 1) / sms;
+        const bool two = 7 * w2 < 5 * w1;
         const int smem = two ? lin_smem<2>() : lin_smem<1>();
         if ((long long)smem > max_smem_optin()) {
             set_error("multipoint linear needs %d bytes of shared memory", smem);
