@@ -92,14 +92,15 @@ __global__ void clip_layer_kernel(int C, int n_cand, float *__restrict__ clip)
 }
 
 // One CTA per (channel, chunk of CL_CHUNK candidates): residuals r_c = fmaf(-s_c, q_c, w) in
-// shared memory, threads over the calibration rows, fp32 dot products, squares summed in double.
+// shared memory, threads over the calibration rows, fp32 dot products, squares summed in fp32
+// (16-row partial sums, a compensated sum per thread, a tree over the threads).
 __global__ void __launch_bounds__(CL_THREADS)
 clip_errors_kernel(const float *__restrict__ X, int N, int groups, const float *__restrict__ W,
                    int C, int d, int qmax, int n_cand, const float *__restrict__ clip,
                    float *__restrict__ err)
 {
     extern __shared__ __align__(16) float R[];   // [CL_CHUNK][d]
-    __shared__ double red[CL_THREADS / 32][CL_CHUNK];
+    __shared__ float red[CL_THREADS / 32][CL_CHUNK];
     const int k = blockIdx.x, c0 = blockIdx.y * CL_CHUNK;
     const int nc = min(CL_CHUNK, n_cand - c0);
     const float qmaxf = (float)qmax;
@@ -113,9 +114,16 @@ clip_errors_kernel(const float *__restrict__ X, int N, int groups, const float *
     }
     __syncthreads();
     const float *Xk = groups == 1 ? X : X + (size_t)k * N * d;
-    double acc[CL_CHUNK];
+    // all in fp32 (fp64 throughput is a small fraction of fp32's on this part): squares summed over
+    // at most 16 rows of a thread, folded into a compensated sum, then a tree over the threads
+    float acc[CL_CHUNK], comp[CL_CHUNK], part[CL_CHUNK];
 #pragma unroll
-    for (int c = 0; c < CL_CHUNK; ++c) acc[c] = 0.0;
+    for (int c = 0; c < CL_CHUNK; ++c) {
+        acc[c] = 0.0f;
+        comp[c] = 0.0f;
+        part[c] = 0.0f;
+    }
+    int rows = 0;
     for (int t = threadIdx.x; t < N; t += CL_THREADS) {
         const float *x = Xk + (size_t)t * d;
         float y[CL_CHUNK];
@@ -128,20 +136,31 @@ clip_errors_kernel(const float *__restrict__ X, int N, int groups, const float *
                 if (c < nc) y[c] = fmaf(xv, R[c * d + j], y[c]);
         }
 #pragma unroll
-        for (int c = 0; c < CL_CHUNK; ++c) acc[c] += (double)y[c] * (double)y[c];
+        for (int c = 0; c < CL_CHUNK; ++c) part[c] = fmaf(y[c], y[c], part[c]);
+        if (++rows == 16) {
+#pragma unroll
+            for (int c = 0; c < CL_CHUNK; ++c) {
+                kahan_add(acc[c], comp[c], part[c]);
+                part[c] = 0.0f;
+            }
+            rows = 0;
+        }
     }
     const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5;
 #pragma unroll
     for (int c = 0; c < CL_CHUNK; ++c) {
-        double v = acc[c];
+        kahan_add(acc[c], comp[c], part[c]);
+        float v = acc[c];
         for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
         if (lane == 0) red[wp][c] = v;
     }
     __syncthreads();
     if (threadIdx.x < nc) {
-        double s = 0.0;
-        for (int i = 0; i < CL_THREADS / 32; ++i) s += red[i][threadIdx.x];
-        err[(size_t)k * n_cand + c0 + threadIdx.x] = (float)(s / (double)N);
+        float v[CL_THREADS / 32];
+        for (int i = 0; i < CL_THREADS / 32; ++i) v[i] = red[i][threadIdx.x];
+        for (int w = CL_THREADS / 64; w > 0; w >>= 1)   // tree over the warps
+            for (int i = 0; i < w; ++i) v[i] += v[i + w];
+        err[(size_t)k * n_cand + c0 + threadIdx.x] = mean_of_sum(v[0], N);
     }
 }
 

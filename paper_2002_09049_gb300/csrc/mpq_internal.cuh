@@ -8,6 +8,22 @@
 
 namespace mpq {
 
+// acc + comp += v, compensated (Kahan): the rounding error of each addition is carried in comp.
+__device__ __forceinline__ void kahan_add(float &acc, float &comp, float v)
+{
+    const float y = __fsub_rn(v, comp);
+    const float t = __fadd_rn(acc, y);
+    comp = __fsub_rn(__fsub_rn(t, acc), y);
+    acc = t;
+}
+
+// sum / N rounded once to fp32 (N exactly representable below 2^24, else in double).
+__device__ __forceinline__ float mean_of_sum(float sum, int N)
+{
+    return N < (1 << 24) ? __fdiv_rn(sum, (float)N) : (float)((double)sum / (double)N);
+}
+
+
 // Records a formatted failure message for mpq_last_error() on the calling thread.
 void set_error(const char *fmt, ...);
 

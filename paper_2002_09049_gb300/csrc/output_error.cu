@@ -3,10 +3,11 @@
 // with the residuals r_{k,n+1} regenerated on chip from W, codes and scales by the recursion of
 // Eq. 7 (never materialised in global memory).
 //
-// Shared input (groups = 1) is a dense contraction and runs on the tensor cores
+// Shared input (groups = 1) is a dense contraction and runs on the tensor cores: the CTA-pair kernel
+// (output_error_pair.cu) when rows are 16-byte multiples, else the single-CTA one
 // (output_error_tc.cu).  Per-channel input (groups = C, depthwise convolution, d = 9): one CTA per
-// channel, its k_max+1 residuals in shared memory, threads over the calibration rows; each
-// channel's own X block is read once, so this path is bound by HBM.
+// channel, its k_max+1 residuals in shared memory, the channel's own rows of X staged through
+// shared memory with coalesced reads (each read once), threads over the rows.
 #include <math.h>
 
 #include "mpq_internal.cuh"
@@ -16,14 +17,16 @@ namespace {
 
 constexpr int GR_THREADS = 256;
 
+constexpr int GR_X_FLOATS = 4096;                 // 16 KB of calibration rows staged at a time
+
 template <int KP1>
 __global__ void __launch_bounds__(GR_THREADS)
 output_error_grouped_kernel(const float *__restrict__ X, int N, const float *__restrict__ W,
                             const int8_t *__restrict__ codes, const float *__restrict__ scales,
                             int C, int d, float *__restrict__ err)
 {
-    extern __shared__ __align__(16) float Rsh[];   // [KP1][d]
-    __shared__ double red[GR_THREADS / 32][KP1];
+    extern __shared__ __align__(16) float Rsh[];   // [KP1][d], then rows of X [GR_X_FLOATS]
+    __shared__ float red[GR_THREADS / 32][KP1];
     const int k = blockIdx.x;
     const int tid = threadIdx.x;
     const int k_max = KP1 - 1;
@@ -40,34 +43,64 @@ output_error_grouped_kernel(const float *__restrict__ X, int N, const float *__r
     __syncthreads();
 
     const float *Xk = X + (size_t)k * N * d;
-    double acc[KP1];
+    float *Xsh = Rsh + ((KP1 * d + 3) & ~3);
+    const int chunk = GR_X_FLOATS / d;               // rows per staged chunk (d <= GR_X_FLOATS)
+    // All in fp32 (the part's fp64 rate is a small fraction of its fp32 rate, and fp64 work per
+    // row, or fp64 warp reductions, bound the kernel): squares summed over at most ERR_FOLD rows of
+    // a thread, folded into a compensated (Kahan) sum, then a tree over the threads and one
+    // division -- relative error below (ERR_FOLD + 2 + 8 + 1) * 2^-24 in all.
+    constexpr int ERR_FOLD = 16;
+    float acc[KP1], comp[KP1], part[KP1];
 #pragma unroll
-    for (int n = 0; n < KP1; ++n) acc[n] = 0.0;
-    for (int t = tid; t < N; t += GR_THREADS) {
-        float y[KP1];
+    for (int n = 0; n < KP1; ++n) {
+        acc[n] = 0.0f;
+        comp[n] = 0.0f;
+        part[n] = 0.0f;
+    }
+    int rows = 0;
+    for (int t0 = 0; t0 < N; t0 += chunk) {
+        // the channel's next rows of X, read with consecutive threads on consecutive words
+        const int nr = min(chunk, N - t0);
+        __syncthreads();   // the previous chunk is no longer read
+        for (int i = tid; i < nr * d; i += GR_THREADS) Xsh[i] = Xk[(size_t)t0 * d + i];
+        __syncthreads();
+        for (int t = tid; t < nr; t += GR_THREADS) {
+            float y[KP1];
 #pragma unroll
-        for (int n = 0; n < KP1; ++n) y[n] = 0.0f;
-        const float *x = Xk + (size_t)t * d;
-        for (int j = 0; j < d; ++j) {
-            const float xv = x[j];
+            for (int n = 0; n < KP1; ++n) y[n] = 0.0f;
+            const float *x = Xsh + t * d;
+            for (int j = 0; j < d; ++j) {
+                const float xv = x[j];
 #pragma unroll
-            for (int n = 0; n < KP1; ++n) y[n] = fmaf(xv, Rsh[n * d + j], y[n]);
+                for (int n = 0; n < KP1; ++n) y[n] = fmaf(xv, Rsh[n * d + j], y[n]);
+            }
+#pragma unroll
+            for (int n = 0; n < KP1; ++n) part[n] = fmaf(y[n], y[n], part[n]);
+            if (++rows == ERR_FOLD) {
+#pragma unroll
+                for (int n = 0; n < KP1; ++n) {
+                    kahan_add(acc[n], comp[n], part[n]);
+                    part[n] = 0.0f;
+                }
+                rows = 0;
+            }
         }
-#pragma unroll
-        for (int n = 0; n < KP1; ++n) acc[n] += (double)y[n] * (double)y[n];
     }
     const int lane = tid & 31, wp = tid >> 5;
 #pragma unroll
     for (int n = 0; n < KP1; ++n) {
-        double v = acc[n];
+        kahan_add(acc[n], comp[n], part[n]);
+        float v = acc[n];
         for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
         if (lane == 0) red[wp][n] = v;
     }
     __syncthreads();
     if (tid < KP1) {
-        double s = 0.0;
-        for (int i = 0; i < GR_THREADS / 32; ++i) s += red[i][tid];
-        err[(size_t)k * KP1 + tid] = (float)(s / (double)N);
+        float v[GR_THREADS / 32];
+        for (int i = 0; i < GR_THREADS / 32; ++i) v[i] = red[i][tid];
+        for (int w = GR_THREADS / 64; w > 0; w >>= 1)   // tree over the warps
+            for (int i = 0; i < w; ++i) v[i] += v[i + w];
+        err[(size_t)k * KP1 + tid] = mean_of_sum(v[0], N);
     }
 }
 
@@ -75,8 +108,8 @@ template <int KP1>
 mpq_status launch_grouped(const float *X, int N, const float *W, const int8_t *codes,
                           const float *scales, int C, int d, float *err, cudaStream_t stream)
 {
-    const size_t smem = (size_t)KP1 * d * sizeof(float);
-    if ((long long)smem > max_smem_optin()) {
+    const size_t smem = ((size_t)(KP1 * d + 3) / 4 * 4 + GR_X_FLOATS) * sizeof(float);
+    if (d > GR_X_FLOATS || (long long)smem > max_smem_optin()) {
         set_error("groups = C with d = %d and k_max = %d needs %zu bytes of shared memory", d,
                   KP1 - 1, smem);
         return MPQ_ERR_UNSUPPORTED;
