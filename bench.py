@@ -413,12 +413,25 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_
 
 def run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step):
     """Same metric through the public network call with host buffers: per layer, H2D of W and X
-    from pinned memory, the path, D2H of codes / scales / point counts -- all inside the timing."""
+    from pinned memory, the path, D2H of codes / scales / point counts -- all inside the timing.
+    The step is NetworkPlan.run_host, captured into a CUDA graph like the device step (one graph
+    per bit width; --graph 0 launches it call by call)."""
     import torch
+    from paper_2002_09049_gb300 import pipeline
     h2d = sum(w.numel() * 4 + x.numel() * 4 for w, x in zip(Whs, Xhs)) * len(wl.bits)
     d2h = sum(p.d2h_bytes() for p in net.plans) * len(wl.bits)
+    graphs = []
+    if args.graph:
+        for b in wl.bits:
+            for sp in specs:
+                sp.bits = b
+            graphs.append(pipeline.CapturedNetwork(net, Ws, Xs, host=(Whs, Xhs)))
 
     def step():
+        if graphs:
+            for g in graphs:
+                g.replay()
+            return
         for b in wl.bits:
             for sp in specs:
                 sp.bits = b

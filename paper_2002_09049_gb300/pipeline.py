@@ -133,6 +133,10 @@ class NetworkPlan:
         work = [s.C * s.d * s.G * s.k_max + s.C * s.d * s.N for s in specs]
         self.order = sorted(range(len(specs)), key=lambda i: -work[i])
         self.streams = [torch.cuda.Stream(self.device) for _ in range(max(1, n_streams))]
+        # host <-> device copies of run_host: one stream each way, so that no layer's input copy
+        # waits in a compute stream's queue behind another layer's kernels
+        self.copy_in = torch.cuda.Stream(self.device)
+        self.copy_out = torch.cuda.Stream(self.device)
 
     def _fork(self, main):
         start = torch.cuda.Event()
@@ -160,16 +164,45 @@ class NetworkPlan:
 
     def run_host(self, W_hosts, X_hosts, W_devs, X_devs, stream=None):
         """End to end: per layer, H2D of W and X from pinned memory, the path, D2H of codes,
-        scales, point counts; each layer on its own stream so copies overlap other layers'
-        kernels.  The caller synchronizes ``stream`` before reading the host outputs."""
+        scales, point counts.  Input copies run back to back on one stream (largest layer
+        first), each layer's kernels start on its compute stream as soon as its inputs have
+        landed, and its outputs go back on one D2H stream once its kernels are done -- copies in
+        both directions overlap other layers' kernels.  The caller synchronizes ``stream`` before
+        reading the host outputs."""
         main = stream or torch.cuda.current_stream(self.device)
         self._fork(main)
+        for s in (self.copy_in, self.copy_out):
+            s.wait_stream(main)
         outs = [None] * len(self.plans)
+        landed = {}
+        for i in self.order:
+            with torch.cuda.stream(self.copy_in):
+                W_devs[i].copy_(W_hosts[i], non_blocking=True)
+                X_devs[i].copy_(X_hosts[i], non_blocking=True)
+                landed[i] = torch.cuda.Event()
+                landed[i].record(self.copy_in)
         for n, i in enumerate(self.order):
             st = self.streams[n % len(self.streams)]
-            outs[i] = self.plans[i].run_host(W_hosts[i], X_hosts[i], W_devs[i], X_devs[i],
-                                             stream=st)
+            st.wait_event(landed[i])
+            self.plans[i].run_device(W_devs[i], X_devs[i], stream=st)
+            done = torch.cuda.Event()
+            done.record(st)
+            self.copy_out.wait_event(done)
+            h = self.plans[i].host_buffers()
+            p = self.plans[i]
+            with torch.cuda.stream(self.copy_out):
+                h["codes"].copy_(p.codes, non_blocking=True)
+                h["scales"].copy_(p.scales, non_blocking=True)
+                h["npoints"].copy_(p.npoints, non_blocking=True)
+                h["points_used"].copy_(p.points_used, non_blocking=True)
+                if p.center is not None:
+                    h["center"].copy_(p.center, non_blocking=True)
+            outs[i] = h
         self._join(main)
+        for s in (self.copy_in, self.copy_out):
+            e = torch.cuda.Event()
+            e.record(s)
+            main.wait_event(e)
         return outs
 
 
@@ -179,24 +212,39 @@ class CapturedNetwork:
     Capture records every launch of ``NetworkPlan.run_device`` (all layers, all streams, the fork and
     join) for fixed input tensors; each ``replay`` re-executes all of that work on the GPU with one
     host call.  Inputs are read from the captured tensors, so refresh their contents in place
-    (``copy_``) to quantize new weights of the same shapes.
+    (``copy_``) to quantize new weights of the same shapes.  With ``host = (W_hosts, X_hosts)``
+    (pinned) the captured step is ``NetworkPlan.run_host`` instead: every replay copies those host
+    tensors in, runs the path and copies codes, scales and point counts out to the plans' pinned
+    ``host_buffers()`` -- the end-to-end step for one host call.
     """
 
-    def __init__(self, net: NetworkPlan, Ws, Xs, warmup: int = 1):
+    def __init__(self, net: NetworkPlan, Ws, Xs, warmup: int = 1, host=None):
         self.net = net
         self.Ws, self.Xs = Ws, Xs
+        self.host = host
+
+        def step(st):
+            if host is None:
+                net.run_device(Ws, Xs, stream=st)
+            else:
+                net.run_host(host[0], host[1], Ws, Xs, stream=st)
+
         side = torch.cuda.Stream(net.device)
         side.wait_stream(torch.cuda.current_stream(net.device))
         with torch.cuda.stream(side):          # warm up outside capture (attributes, modules)
             for _ in range(warmup):
-                net.run_device(Ws, Xs, stream=side)
+                step(side)
         torch.cuda.current_stream(net.device).wait_stream(side)
         torch.cuda.synchronize(net.device)
         self.graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(self.graph, stream=side):
-            net.run_device(Ws, Xs, stream=side)
+            step(side)
         torch.cuda.synchronize(net.device)
 
     def replay(self):
         self.graph.replay()
         return self.net
+
+    def host_outputs(self):
+        """The pinned host outputs the end-to-end replays write (per layer)."""
+        return [p.host_buffers() for p in self.net.plans]

@@ -136,3 +136,63 @@ def test_captured_graph_matches_launches(gpu):
     for p, r in zip(net.plans, ref_out):
         for n, v in r.items():
             assert torch.equal(getattr(p, n), v), n
+
+
+@pytest.mark.parametrize("center", [-1, 0])
+def test_network_run_host_matches_device(gpu, center):
+    """The end-to-end network call (inputs copied in on one stream, outputs copied out on another,
+    kernels on the compute streams in between) returns exactly what the device-resident call
+    computes, on every repetition."""
+    wl = wlm.WORKLOADS["c2"]
+    idx = [0, 3, 9, 16, 20]
+    specs, Whs, Xhs = [], [], []
+    for li in idx:
+        layer = wl.layers[li]
+        specs.append(pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, bits=4, G=wl.G,
+                                        k_max=wl.k_max, budget_or_eps=wl.beta, center=center))
+        Whs.append(torch.from_numpy(wlm.make_weights(wl, li)).pin_memory())
+        Xhs.append(torch.from_numpy(wlm.make_calibration(wl, li)).pin_memory())
+    ref = pipeline.NetworkPlan(specs, gpu, n_streams=3).run_device(
+        [w.to(gpu) for w in Whs], [x.to(gpu) for x in Xhs])
+    torch.cuda.synchronize()
+    net = pipeline.NetworkPlan(specs, gpu, n_streams=3)
+    Wds = [torch.empty_like(w, device=gpu) for w in Whs]
+    Xds = [torch.empty_like(x, device=gpu) for x in Xhs]
+    for _ in range(2):
+        outs = net.run_host(Whs, Xhs, Wds, Xds)
+        torch.cuda.synchronize()
+        for h, p in zip(outs, ref.plans):
+            assert torch.equal(h["codes"], p.codes.cpu()) and torch.equal(h["scales"], p.scales.cpu())
+            assert torch.equal(h["npoints"], p.npoints.cpu())
+            assert int(h["points_used"].item()) == int(p.points_used.item())
+            if center >= 0:
+                assert torch.equal(h["center"], p.center.cpu())
+
+
+def test_captured_end_to_end_matches_device(gpu):
+    """The captured end-to-end step (copies in, path, copies out) writes the same host outputs as
+    the device-resident call, and a replay after new host inputs picks them up."""
+    wl = wlm.WORKLOADS["c2"]
+    idx = [1, 9, 16]
+    specs, Whs, Xhs = [], [], []
+    for li in idx:
+        layer = wl.layers[li]
+        specs.append(pipeline.LayerSpec(C=layer.C, d=layer.d, N=wl.n_calib, bits=4, G=wl.G,
+                                        k_max=wl.k_max, budget_or_eps=wl.beta))
+        Whs.append(torch.from_numpy(wlm.make_weights(wl, li)).pin_memory())
+        Xhs.append(torch.from_numpy(wlm.make_calibration(wl, li)).pin_memory())
+    net = pipeline.NetworkPlan(specs, gpu, n_streams=2)
+    Wds = [torch.empty_like(w, device=gpu) for w in Whs]
+    Xds = [torch.empty_like(x, device=gpu) for x in Xhs]
+    cap = pipeline.CapturedNetwork(net, Wds, Xds, host=(Whs, Xhs))
+    for scale in (1.0, 0.5):
+        for w in Whs:
+            w.mul_(scale)
+        cap.replay()
+        torch.cuda.synchronize()
+        ref = pipeline.NetworkPlan(specs, gpu, n_streams=1).run_device(
+            [w.to(gpu) for w in Whs], [x.to(gpu) for x in Xhs])
+        torch.cuda.synchronize()
+        for h, p in zip(cap.host_outputs(), ref.plans):
+            assert torch.equal(h["codes"], p.codes.cpu()) and torch.equal(h["scales"], p.scales.cpu())
+            assert torch.equal(h["npoints"], p.npoints.cpu())
