@@ -879,24 +879,57 @@ def run_infer(args, world, rank, local):
                       "streams": args.streams, "parallelism": f"replicas x{world}"},
            "roofline": roofline, "gpu_launches": len(L) * args.steps, "clocks": clk.summary()}
     if not args.no_e2e:
-        def e2e_step():
+        # inputs in on one copy stream (largest layer first), each layer's kernel as soon as its
+        # inputs have landed, outputs out on a second copy stream into pinned buffers; captured
+        # into a CUDA graph (one host call per step) unless --graph 0
+        Yh = [torch.empty(x["Y"].shape, dtype=torch.int32).pin_memory() for x in L]
+        copy_in, copy_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+
+        def e2e_launch(root):
             ev = torch.cuda.Event()
-            ev.record(main)
-            for st in streams:
+            ev.record(root)
+            for st in streams + [copy_in, copy_out]:
                 st.wait_event(ev)
-            host = []
+            landed = {}
+            for i in order:
+                with torch.cuda.stream(copy_in):
+                    L[i]["X"].copy_(L[i]["Xh"], non_blocking=True)
+                landed[i] = torch.cuda.Event()
+                landed[i].record(copy_in)
             for n, i in enumerate(order):
                 st = streams[n % len(streams)]
-                with torch.cuda.stream(st):
-                    L[i]["X"].copy_(L[i]["Xh"], non_blocking=True)
-                    call(i, st)
-                    host.append(L[i]["Y"].to("cpu", non_blocking=True))
-            for st in streams:
+                st.wait_event(landed[i])
+                call(i, st)
+                done = torch.cuda.Event()
+                done.record(st)
+                copy_out.wait_event(done)
+                with torch.cuda.stream(copy_out):
+                    Yh[i].copy_(L[i]["Y"], non_blocking=True)
+            for st in streams + [copy_in, copy_out]:
                 e = torch.cuda.Event()
                 e.record(st)
-                main.wait_event(e)
-        for _ in range(max(1, args.warmup)):
-            e2e_step()
+                root.wait_event(e)
+
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(main)
+        with torch.cuda.stream(side):
+            for _ in range(max(1, args.warmup)):
+                e2e_launch(side)
+        main.wait_stream(side)
+        torch.cuda.synchronize()
+        graph = None
+        if args.graph:
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=side):
+                e2e_launch(side)
+            torch.cuda.synchronize()
+
+        def e2e_step():
+            if graph is not None:
+                graph.replay()
+            else:
+                e2e_launch(main)
+        e2e_step()
         torch.cuda.synchronize()
         tms = []
         for _ in range(args.steps):
@@ -906,6 +939,9 @@ def run_infer(args, world, rank, local):
             e2e_step()
             torch.cuda.synchronize()
             tms.append((time.perf_counter() - t0) * 1e3)
+        for x, y in zip(L, Yh):   # the host outputs are the device results
+            if not torch.equal(y, x["Y"].cpu()):
+                raise RuntimeError("end-to-end outputs differ from the device results")
         e_ms = float(np.mean(tms))
         out["e2e"] = {"value": macs / (e_ms / 1e3), "unit": INFER_UNIT, "ms_per_step": e_ms,
                       "h2d_bytes_per_step": sum(x["Xh"].numel() for x in L),
