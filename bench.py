@@ -418,24 +418,26 @@ def run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step):
     per bit width; --graph 0 launches it call by call)."""
     import torch
     from paper_2002_09049_gb300 import pipeline
-    h2d = sum(w.numel() * 4 + x.numel() * 4 for w, x in zip(Whs, Xhs)) * len(wl.bits)
+    # the inputs are copied in once per step; every bit width's outputs are copied out
+    h2d = sum(w.numel() * 4 + x.numel() * 4 for w, x in zip(Whs, Xhs))
     d2h = sum(p.d2h_bytes() for p in net.plans) * len(wl.bits)
     graphs = []
     if args.graph:
-        for b in wl.bits:
+        for n, b in enumerate(wl.bits):
             for sp in specs:
                 sp.bits = b
-            graphs.append(pipeline.CapturedNetwork(net, Ws, Xs, host=(Whs, Xhs)))
+            graphs.append(pipeline.CapturedNetwork(net, Ws, Xs, host=(Whs, Xhs),
+                                                   copy_inputs=n == 0))
 
     def step():
         if graphs:
             for g in graphs:
                 g.replay()
             return
-        for b in wl.bits:
+        for n, b in enumerate(wl.bits):
             for sp in specs:
                 sp.bits = b
-            net.run_host(Whs, Xhs, Ws, Xs, stream=stream)
+            net.run_host(Whs, Xhs, Ws, Xs, stream=stream, copy_inputs=n == 0)
 
     for _ in range(max(1, args.warmup)):
         step()

@@ -162,13 +162,14 @@ class NetworkPlan:
         self._join(main)
         return self
 
-    def run_host(self, W_hosts, X_hosts, W_devs, X_devs, stream=None):
+    def run_host(self, W_hosts, X_hosts, W_devs, X_devs, stream=None, copy_inputs=True):
         """End to end: per layer, H2D of W and X from pinned memory, the path, D2H of codes,
         scales, point counts.  Input copies run back to back on one stream (largest layer
         first), each layer's kernels start on its compute stream as soon as its inputs have
         landed, and its outputs go back on one D2H stream once its kernels are done -- copies in
-        both directions overlap other layers' kernels.  The caller synchronizes ``stream`` before
-        reading the host outputs."""
+        both directions overlap other layers' kernels.  copy_inputs=False reuses the inputs an
+        earlier call copied in (e.g. a second bit width over the same weights).  The caller
+        synchronizes ``stream`` before reading the host outputs."""
         main = stream or torch.cuda.current_stream(self.device)
         self._fork(main)
         for s in (self.copy_in, self.copy_out):
@@ -177,8 +178,9 @@ class NetworkPlan:
         landed = {}
         for i in self.order:
             with torch.cuda.stream(self.copy_in):
-                W_devs[i].copy_(W_hosts[i], non_blocking=True)
-                X_devs[i].copy_(X_hosts[i], non_blocking=True)
+                if copy_inputs:
+                    W_devs[i].copy_(W_hosts[i], non_blocking=True)
+                    X_devs[i].copy_(X_hosts[i], non_blocking=True)
                 landed[i] = torch.cuda.Event()
                 landed[i].record(self.copy_in)
         for n, i in enumerate(self.order):
@@ -215,10 +217,12 @@ class CapturedNetwork:
     (``copy_``) to quantize new weights of the same shapes.  With ``host = (W_hosts, X_hosts)``
     (pinned) the captured step is ``NetworkPlan.run_host`` instead: every replay copies those host
     tensors in, runs the path and copies codes, scales and point counts out to the plans' pinned
-    ``host_buffers()`` -- the end-to-end step for one host call.
+    ``host_buffers()`` -- the end-to-end step for one host call (``copy_inputs=False``: the
+    inputs are already on the device, only the outputs are copied out).
     """
 
-    def __init__(self, net: NetworkPlan, Ws, Xs, warmup: int = 1, host=None):
+    def __init__(self, net: NetworkPlan, Ws, Xs, warmup: int = 1, host=None,
+                 copy_inputs: bool = True):
         self.net = net
         self.Ws, self.Xs = Ws, Xs
         self.host = host
@@ -227,7 +231,7 @@ class CapturedNetwork:
             if host is None:
                 net.run_device(Ws, Xs, stream=st)
             else:
-                net.run_host(host[0], host[1], Ws, Xs, stream=st)
+                net.run_host(host[0], host[1], Ws, Xs, stream=st, copy_inputs=copy_inputs)
 
         side = torch.cuda.Stream(net.device)
         side.wait_stream(torch.cuda.current_stream(net.device))
