@@ -33,6 +33,8 @@
 #include <limits.h>
 #include <math.h>
 
+#include <type_traits>
+
 #include "mpq_internal.cuh"
 #include "rounding.cuh"
 
@@ -78,15 +80,19 @@ struct Scratch {
 // words) and hN[G+1], then r[d].  Without the lattice every warp has a private copy (so warps
 // never contend on a bin); with the lattice form (below) events are rare and the group shares one
 // copy, and the group also holds nb lattice buckets first: 64-bit R sums (2 words each) and
-// 32-bit counts.  Group regions are kept 8-byte aligned.
-__host__ __device__ constexpr size_t lattice_words(int nb)
+// 32-bit counts.  Group regions are kept 8-byte aligned.  When it fits one more CTA per SM, the
+// lattice form on the linear grid leaves the table out (computing f_g where needed) and packs its
+// counts into 16 bits, two per word (a count never exceeds d <= 8192).
+__host__ __device__ constexpr size_t lattice_words(int nb, bool packed = false)
 {
-    return ((size_t)3 * nb + 1) & ~(size_t)1;
+    return packed ? ((size_t)2 * nb + (size_t)(nb + 1) / 2 + 1) & ~(size_t)1
+                  : ((size_t)3 * nb + 1) & ~(size_t)1;
 }
 
-__host__ __device__ constexpr size_t group_words(int G, int d, int copies, int nb)
+__host__ __device__ constexpr size_t group_words(int G, int d, int copies, int nb,
+                                                 bool packed = false)
 {
-    return lattice_words(nb) + (((size_t)3 * (G + 1) * copies + (size_t)d + 1) & ~(size_t)1);
+    return lattice_words(nb, packed) + (((size_t)3 * (G + 1) * copies + (size_t)d + 1) & ~(size_t)1);
 }
 
 template <int WPC>
@@ -367,7 +373,7 @@ __device__ __forceinline__ float i64_to_f32(long long x)
     return __fmaf_rn(hi, 4294967296.0f, lo);
 }
 
-template <int WPC, bool CUSTOM, bool LAT>
+template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
 __global__ void __launch_bounds__(QTHREADS, 4)
 quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, const Grid<CUSTOM> grid,
                 int k_max, int8_t *__restrict__ codes, float *__restrict__ scales,
@@ -385,22 +391,29 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
     const int grp = warp / WPC, gw = warp % WPC, gt = gw * 32 + lane;
     const int k = blockIdx.x * GPC + grp;
     const float qmaxf = (float)qmax;
-    float *fgrid = reinterpret_cast<float *>(smem_raw);   // [G] f_g
-    float *finv = fgrid + G;                              // [G] fl(1 / f_g)
+    // the grid fractions f_g and fl(1 / f_g): a table, or (linear grid, when the table's 2G words
+    // would cost a CTA per SM) computed where needed
+    static_assert(TABLE || !CUSTOM, "a caller's grid needs the table");
+    float *ftab = reinterpret_cast<float *>(smem_raw);   // [G] f_g, then [G] fl(1 / f_g)
     for (int L = threadIdx.x; L <= qmax; L += QTHREADS) s_hinv[L] = 1.0f / ((float)L - 0.5f);
-    for (int g = threadIdx.x; g < G; g += QTHREADS) {
-        const float f = grid.frac(g, G);
-        fgrid[g] = f;
-        finv[g] = __frcp_rn(f);
-    }
+    if (TABLE)
+        for (int g = threadIdx.x; g < G; g += QTHREADS) {
+            const float f = grid.frac(g, G);
+            ftab[g] = f;
+            ftab[G + g] = __frcp_rn(f);
+        }
+    auto fg = [&](int g) -> float { return TABLE ? ftab[g] : grid.frac(g, G); };
+    auto fi = [&](int g) -> float { return TABLE ? ftab[G + g] : __frcp_rn(grid.frac(g, G)); };
     __syncthreads();
     if (k >= C) return;   // whole group idle (group-uniform)
 
-    unsigned int *gl =
-        reinterpret_cast<unsigned int *>(finv + G) + (size_t)grp * group_words(G, d, COPIES, nb);
+    unsigned int *gl = reinterpret_cast<unsigned int *>(ftab + (TABLE ? 2 * G : 0)) +
+                       (size_t)grp * group_words(G, d, COPIES, nb, !TABLE);
     unsigned long long *latR = reinterpret_cast<unsigned long long *>(gl);   // [nb]
-    unsigned int *latC = gl + 2 * (size_t)nb;                                 // [nb]
-    unsigned int *gbase = gl + lattice_words(nb);
+    // bucket counts: 32-bit, or 16-bit two per word without the table
+    using Count = typename std::conditional<TABLE, unsigned int, unsigned short>::type;
+    Count *latC = reinterpret_cast<Count *>(gl + 2 * (size_t)nb);           // [nb]
+    unsigned int *gbase = gl + lattice_words(nb, !TABLE);
     // this warp's private bins; copy 0 receives the merged suffix sums
     unsigned int *hLo = gbase + (size_t)(COPIES > 1 ? gw : 0) * 3 * (G + 1);
     unsigned int *hHi = hLo + (G + 1);
@@ -464,17 +477,17 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             if (LAT)
                 for (int t = gt; t < nb; t += NT) {
                     latR[t] = 0ull;
-                    latC[t] = 0u;
+                    latC[t] = 0;
                 }
             gsync<WPC>(grp);
-            const bool zero_scale = __fmul_rn(fgrid[0], smax) == 0.0f;   // s_g increases with g
+            const bool zero_scale = __fmul_rn(fg(0), smax) == 0.0f;   // s_g increases with g
 
             double bestD = DBL_MAX;
             int bestg = INT_MAX;
             if (!zero_scale) {
                 // ---- events: one per (element, level crossed inside the grid)
-                const float s0 = __fmul_rn(fgrid[0], smax), sG = __fmul_rn(fgrid[G - 1], smax);
-                const float i0 = finv[0] * ism, iG = finv[G - 1] * ism;
+                const float s0 = __fmul_rn(fg(0), smax), sG = __fmul_rn(fg(G - 1), smax);
+                const float i0 = fi(0) * ism, iG = fi(G - 1) * ism;
                 const float g_per_a = __fdiv_rn((float)G, smax);   // linear grid: s_g ~ (g+1)/G*smax
                 long long Pb = 0;
                 long long Nb = 0;
@@ -498,7 +511,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                             int lo = 1, hi = G - 1;
                             while (lo < hi) {
                                 const int mid = (lo + hi) >> 1;
-                                if (fgrid[mid] < f_est) lo = mid + 1; else hi = mid;
+                                if (fg(mid) < f_est) lo = mid + 1; else hi = mid;
                             }
                             T = lo;
                         } else {
@@ -515,7 +528,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                                 continue;
                             }
                         }
-#define MPQ_HELD(t) level_held(a, __fmul_rn(fgrid[t], smax), finv[t] * ism, L)
+#define MPQ_HELD(t) level_held(a, __fmul_rn(fg(t), smax), fi(t) * ism, L)
                         const bool up = (T < G - 1) && MPQ_HELD(T);
                         const bool dn = !up && (T > 1) && !MPQ_HELD(T - 1);
                         if (up) {
@@ -556,7 +569,11 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                                         (unsigned long long)fixed_point(av[u], S);
                                     unsigned int *Rw = reinterpret_cast<unsigned int *>(&latR[bb]);
                                     add64(&Rw[0], &Rw[1], (unsigned int)R, (unsigned int)(R >> 32));
-                                    atomicAdd(&latC[bb], 1u);
+                                    if (TABLE)
+                                        atomicAdd(reinterpret_cast<unsigned int *>(latC) + bb, 1u);
+                                    else   // 16-bit count in its word (no carry: count <= d)
+                                        atomicAdd(reinterpret_cast<unsigned int *>(latC) + (bb >> 1),
+                                                  1u << ((bb & 1) * 16));
                                 }
                             } else {
                                 events(av[u]);
@@ -598,7 +615,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 };
                 auto lat_store = [&](int t, unsigned long long p, long long q) {
                     latR[t] = p;
-                    latC[t] = (unsigned int)q;
+                    latC[t] = (Count)q;
                 };
                 // large grids (G * COPIES bins to merge, or a long lattice): the whole group scans
                 const bool big = (LAT && nb > 2048) || G * COPIES > 1024;
@@ -634,7 +651,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 // inputs carry at most ~8 roundings of 2^-24, the bound allows 2^-20.
                 float upper = FLT_MAX;
                 for (int g = gt; g < G; g += NT) {
-                    const float sh = fgrid[g] * smax_e;
+                    const float sh = fg(g) * smax_e;
                     const float Nf = (float)(int)(Nbase + mN[g + 1]);
                     const float Pf = i64_to_f32(Pbase + bin64(mLo, mHi, g + 1)) * pscale;
                     const float D32 = sh * (sh * Nf - 2.0f * Pf);
@@ -643,7 +660,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 }
                 upper = group_min<WPC>(upper, sc, gw, lane, grp);
                 for (int g = gt; g < G; g += NT) {
-                    const float sh = fgrid[g] * smax_e;
+                    const float sh = fg(g) * smax_e;
                     const long long Pg = Pbase + bin64(mLo, mHi, g + 1);
                     const long long Ng = Nbase + mN[g + 1];
                     const float Nf = (float)(int)Ng;
@@ -651,7 +668,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     const float D32 = sh * (sh * Nf - 2.0f * Pf);
                     const float err = sh * (sh * Nf + 2.0f * Pf) * MPQ_FAST_REL;
                     if (D32 - err <= upper) {
-                        const double D = decision(__fmul_rn(fgrid[g], smax), Pg, Ng, down);
+                        const double D = decision(__fmul_rn(fg(g), smax), Pg, Ng, down);
                         if (D < bestD) {
                             bestD = D;
                             bestg = g;
@@ -661,7 +678,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             } else {
                 // ---- direct evaluation (a candidate scale underflowed to 0)
                 for (int g = gt; g < G; g += NT) {
-                    const float s = __fmul_rn(fgrid[g], smax);
+                    const float s = __fmul_rn(fg(g), smax);
                     double D = 0.0;  // s == 0: all codes 0, E = ||r||^2
                     if (s > 0.0f) {
                         long long P = 0, N = 0;
@@ -681,8 +698,8 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             }
             int g = group_argmin<WPC>(bestD, bestg, sc, gw, lane, grp);
             if (g < 0 || g >= G) g = G - 1;   // unreachable: every D is finite
-            s_best = __fmul_rn(fgrid[g], smax);
-            inv_best = zero_scale ? 0.0f : finv[g] * ism;
+            s_best = __fmul_rn(fg(g), smax);
+            inv_best = zero_scale ? 0.0f : fi(g) * ism;
         }
 
         // residual update (Eq. 7) and code emission; also the next step's max |r|
@@ -721,20 +738,34 @@ int ceil_log2(long long x)
     return b;
 }
 
-template <int WPC, bool CUSTOM, bool LAT>
+template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
 mpq_status launch_wpc(const float *W, int C, int d, int qmax, int G, const Grid<CUSTOM> &grid,
                       int k_max, int8_t *codes, float *scales, float *resid_sq, float *residuals,
                       int hbits, size_t smem, cudaStream_t stream)
 {
     constexpr int GPC = 8 / WPC;
-    cudaError_t e = cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT>,
+    cudaError_t e = cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e == cudaSuccess) {
-        quantize_kernel<WPC, CUSTOM, LAT><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
+        quantize_kernel<WPC, CUSTOM, LAT, TABLE><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
             W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, hbits);
         e = cudaGetLastError();
     }
     return cuda_status(e, "quantize kernel launch");
+}
+
+// CTAs of a quantize kernel that fit on one SM with `smem` bytes of dynamic shared memory.
+template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
+int quantize_ctas_per_sm(size_t smem)
+{
+    int n = 0;
+    if (cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
+                                                      QTHREADS, smem) != cudaSuccess)
+        n = 0;
+    (void)cudaGetLastError();
+    return n;
 }
 
 template <int WPC, bool CUSTOM>
@@ -743,11 +774,23 @@ mpq_status launch_lat(bool lat, const float *W, int C, int d, int qmax, int G,
                       float *resid_sq, float *residuals, int hbits, size_t smem,
                       cudaStream_t stream)
 {
-    if (lat && !CUSTOM)
-        return launch_wpc<WPC, CUSTOM, !CUSTOM>(W, C, d, qmax, G, grid, k_max, codes, scales,
+    if constexpr (!CUSTOM) {
+        if (lat) {
+            // the lattice form on the linear grid: no grid table and packed counts when that fits
+            // one more CTA on an SM (it costs some arithmetic per candidate otherwise)
+            const int nb = 2 * G * qmax + 1;
+            const size_t packed = (size_t)(8 / WPC) * group_words(G, d, 1, nb, true) * 4;
+            if (quantize_ctas_per_sm<WPC, false, true, false>(packed) >
+                quantize_ctas_per_sm<WPC, false, true, true>(smem))
+                return launch_wpc<WPC, false, true, false>(W, C, d, qmax, G, grid, k_max, codes,
+                                                           scales, resid_sq, residuals, hbits,
+                                                           packed, stream);
+            return launch_wpc<WPC, false, true, true>(W, C, d, qmax, G, grid, k_max, codes, scales,
+                                                      resid_sq, residuals, hbits, smem, stream);
+        }
+    }
+    return launch_wpc<WPC, CUSTOM, false, true>(W, C, d, qmax, G, grid, k_max, codes, scales,
                                                 resid_sq, residuals, hbits, smem, stream);
-    return launch_wpc<WPC, CUSTOM, false>(W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq,
-                                          residuals, hbits, smem, stream);
 }
 
 template <bool CUSTOM>
