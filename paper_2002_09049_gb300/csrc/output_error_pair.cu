@@ -17,7 +17,8 @@
 //
 // Input: one thread per CTA streams each K chunk's X rows, W rows and codes into a ring of raw
 // shared-memory slots with TMA tile copies (rows past N and channels past C read as zeros).  Eight
-// producer warps split X into the B tiles and regenerate the residuals r_{n+1} = r_n - s_n q_n
+// producer warps (twelve in the clipping search) split X into the B tiles and regenerate the
+// residuals r_{n+1} = r_n - s_n q_n
 // (Eq. 7) from W, codes and scales into the A tiles (128-byte swizzled, K-major); residuals never
 // exist in global memory.  Both CTAs' producers report a full stage to the even CTA, whose MMA
 // thread issues the pair MMAs and signals both CTAs (multicast commits) when a stage or a segment
@@ -57,13 +58,22 @@ constexpr int P_OFF_A_LO = P_TILE;
 constexpr int P_OFF_B_HI = 2 * P_TILE;
 constexpr int P_OFF_B_LO = 3 * P_TILE;
 constexpr int P_STAGE_BYTES = 4 * P_TILE;       // 64 KB
-constexpr int P_PROD_WARPS = 8;
-constexpr int P_PROD_THREADS = P_PROD_WARPS * 32;
 constexpr int P_EPI_WARPS = 8;                  // two per TMEM lane quarter, one per column half
-constexpr int P_EPI_WARP0 = P_PROD_WARPS;       // warps 8..15: warp % 4 selects TMEM lanes
-constexpr int P_MMA_WARP = P_EPI_WARP0 + P_EPI_WARPS;
-constexpr int P_TMA_WARP = P_MMA_WARP + 1;
-constexpr int P_THREADS = (P_TMA_WARP + 1) * 32;   // 576
+
+// Warp roles: producers first, then the epilogue warps (warp % 4 selects TMEM lanes, so the
+// producer count is a multiple of 4), the MMA warp and the TMA warp.  The clipping search's
+// producers regenerate a residual per candidate and bound that mode, so it gets 12 warps of them;
+// the greedy mode keeps 8 (more registers per thread).
+template <bool CLIP>
+struct PRoles {
+    static constexpr int PROD_WARPS = CLIP ? 12 : 8;
+    static constexpr int PROD_THREADS = PROD_WARPS * 32;
+    static constexpr int EPI_WARP0 = PROD_WARPS;
+    static constexpr int MMA_WARP = EPI_WARP0 + P_EPI_WARPS;
+    static constexpr int TMA_WARP = MMA_WARP + 1;
+    static constexpr int THREADS = (TMA_WARP + 1) * 32;   // 576 or 704
+    static_assert(PROD_WARPS % 4 == 0, "epilogue warps start at a TMEM lane quarter boundary");
+};
 constexpr uint32_t P_TMEM_COLS = 512;
 constexpr uint32_t P_RUN_COL = 256;
 constexpr int P_MAX_RAW = 3;
@@ -96,8 +106,9 @@ struct PGeo {
     static constexpr int K = CLIP ? 0 : KP1 - 1;
     static constexpr int KQ = K > 0 ? K : 1;
     static constexpr int CH = P_VEC / KP1;
-    static constexpr int ITEMS2 = (CH * (P_KC / 2) + P_PROD_THREADS - 1) / P_PROD_THREADS;
-    static constexpr int X_ITEMS = (P_ROWS * P_KC4 + P_PROD_THREADS - 1) / P_PROD_THREADS;
+    static constexpr int PT = PRoles<CLIP>::PROD_THREADS;
+    static constexpr int ITEMS2 = (CH * (P_KC / 2) + PT - 1) / PT;
+    static constexpr int X_ITEMS = (P_ROWS * P_KC4 + PT - 1) / PT;
     static constexpr int RAW_W = P_ROWS * P_KC * 4;
     static constexpr int RAW_Q = (RAW_W + CH * P_KC * 4 + 127) / 128 * 128;
     static constexpr uint32_t RAW_TX = P_ROWS * P_KC * 4 + CH * P_KC * 4 + K * CH * P_KC;
@@ -118,15 +129,19 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
 {
     using G = PGeo<KP1, CLIP>;
     constexpr int K = G::K;
-    static_assert(G::X_ITEMS * P_PROD_THREADS == P_ROWS * P_KC4, "X items cover the chunk");
     // every shared-memory read of a group before its stores (the accessors are ordered), so the
     // reads' latencies overlap instead of adding up
+    constexpr int XN = P_ROWS * P_KC4;                  // 16-byte X items per chunk
     float4 xr[G::X_ITEMS];
 #pragma unroll
-    for (int i = 0; i < G::X_ITEMS; ++i) xr[i] = ld_shared_v4(slot + (uint32_t)(pt + i * P_PROD_THREADS) * 16u);
+    for (int i = 0; i < G::X_ITEMS; ++i) {
+        const int q = pt + i * G::PT;
+        if (G::X_ITEMS * G::PT == XN || q < XN) xr[i] = ld_shared_v4(slot + (uint32_t)q * 16u);
+    }
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
-        const int q = pt + i * P_PROD_THREADS;
+        const int q = pt + i * G::PT;
+        if (G::X_ITEMS * G::PT != XN && q >= XN) break;
         float4 hi, lo;
         split4(xr[i], hi, lo);
         const uint32_t off = sw128_offset(q / P_KC4, q % P_KC4);
@@ -135,7 +150,7 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
     }
 #pragma unroll
     for (int i = 0; i < G::ITEMS2; ++i) {
-        const int p = pt + i * P_PROD_THREADS;
+        const int p = pt + i * G::PT;
         if (!CLIP && p < nch * (P_KC / 2)) {
             const int ch = p / (P_KC / 2), e2 = p % (P_KC / 2);
             float2 r = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
@@ -163,8 +178,8 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
     if constexpr (CLIP) {
         // (candidate, channel, element pair) units over all producer threads, element pairs
         // lane-contiguous: each warp store fills whole 128-byte rows.
-        constexpr int STEP = P_PROD_THREADS / (P_KC / 2);   // rows between a thread's units
-        constexpr int UNITS = P_VEC / STEP;                 // at most 8 units per thread
+        constexpr int STEP = G::PT / (P_KC / 2);   // rows between a thread's units
+        constexpr int UNITS = (P_VEC + STEP - 1) / STEP;    // most units of one thread
         const int rows = nch * KP1;                     // row = c * nch + ch
         const int e2 = pt % (P_KC / 2);                  // the same for all of this thread's units
         const int row0 = pt / (P_KC / 2);
@@ -208,7 +223,7 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
 // scales: [C][k_max] point scales, or (CLIP) [C][KP1] candidate clipping factors K; qmax: the
 // code range for CLIP.
 template <int KP1, bool CLIP>
-__global__ void __launch_bounds__(P_THREADS, 1)
+__global__ void __launch_bounds__(PRoles<CLIP>::THREADS, 1)
 output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, int qmax,
                          float *__restrict__ err, int split,
                          const __grid_constant__ CUtensorMap tmX,
@@ -216,6 +231,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                          const __grid_constant__ CUtensorMap tmQ)
 {
     using G = PGeo<KP1, CLIP>;
+    using PR = PRoles<CLIP>;
     constexpr int R = G::RAW_STAGES;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
@@ -242,12 +258,12 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < P_STAGES; ++s) {
-            mbar_init(&ctl.full[s], 2 * P_PROD_WARPS);
+            mbar_init(&ctl.full[s], 2 * PR::PROD_WARPS);
             mbar_init(&ctl.empty[s], 1);
         }
         for (int r = 0; r < P_MAX_RAW; ++r) {
             mbar_init(&ctl.raw_full[r], 1);
-            mbar_init(&ctl.raw_empty[r], P_PROD_WARPS);
+            mbar_init(&ctl.raw_empty[r], PR::PROD_WARPS);
         }
         mbar_init(&ctl.segfull, 1);
         mbar_init(&ctl.segempty, 2 * P_EPI_WARPS);
@@ -257,13 +273,13 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
     }
     const float qmaxf = (float)qmax;
     if (CLIP) {
-        for (int i = threadIdx.x; i < nvec; i += P_THREADS) {
+        for (int i = threadIdx.x; i < nvec; i += PR::THREADS) {
             const float s = __fdiv_rn(__ldg(scales + (size_t)k0 * KP1 + i), qmaxf);
             ctl.clip_s[i] = s;
             ctl.clip_inv[i] = s > 0.0f ? __frcp_rn(s) : 0.0f;
         }
     }
-    if (warp == P_MMA_WARP) {
+    if (warp == PR::MMA_WARP) {
         tmem_alloc_pair(&ctl.tmem_base, P_TMEM_COLS);
         tc_fence_before();
     }
@@ -272,13 +288,13 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
     const uint32_t tmem = ctl.tmem_base;
     volatile int *abort_flag = &ctl.abort;
 
-    if (warp < P_PROD_WARPS) {
+    if (warp < PR::PROD_WARPS) {
         // ---------------------------------------------------------------- producers
         const int pt = threadIdx.x;
         float sc[G::ITEMS2][G::KQ];     // scales of this thread's items, the same for every chunk
 #pragma unroll
         for (int i = 0; i < G::ITEMS2; ++i) {
-            const int p = pt + i * P_PROD_THREADS;
+            const int p = pt + i * PR::PROD_THREADS;
             const int k = k0 + p / (P_KC / 2);
 #pragma unroll
             for (int n = 0; n < G::KQ; ++n)
@@ -301,10 +317,10 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 mbar_arrive(&ctl.raw_empty[slot]);
             }
         }
-    } else if (warp < P_MMA_WARP) {
+    } else if (warp < PR::MMA_WARP) {
         // ---------------------------------------------------------------- epilogue
         // lane quarter q (the TMEM lanes this warp may access) and column half h
-        const int ew = warp - P_EPI_WARP0, q = ew & 3, h = ew >> 2;
+        const int ew = warp - PR::EPI_WARP0, q = ew & 3, h = ew >> 2;
         const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(h * (P_N / 2));
         double acc = 0.0;
         int g = 0;
@@ -345,7 +361,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             }
         }
         ctl.part[h][q * 32 + lane] = *abort_flag ? (double)NAN : acc;
-    } else if (warp == P_MMA_WARP) {
+    } else if (warp == PR::MMA_WARP) {
         // ---------------------------------------------------------------- MMA issuer (even CTA)
         if (half == 0 && lane == 0) {
             constexpr uint32_t idesc = idesc_tf32(2 * P_VEC, P_N);
@@ -421,8 +437,8 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
 
     // ---------------------------------------------------------------- cluster reduction
     cluster_sync();
-    if (crank < 2 && warp >= P_EPI_WARP0 && warp < P_EPI_WARP0 + 4) {
-        const int m = (warp - P_EPI_WARP0) * 32 + lane;
+    if (crank < 2 && warp >= PR::EPI_WARP0 && warp < PR::EPI_WARP0 + 4) {
+        const int m = (warp - PR::EPI_WARP0) * 32 + lane;
         if (m < nvec) {
             double s = 0.0;
             for (int j = 0; j < split; ++j) {
@@ -433,7 +449,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         }
     }
     cluster_sync();
-    if (warp == P_MMA_WARP) {
+    if (warp == PR::MMA_WARP) {
         tc_fence_after();
         tmem_dealloc_pair(tmem, P_TMEM_COLS);
     }
@@ -500,7 +516,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
 
     cudaLaunchConfig_t cfg = {};
-    cfg.blockDim = dim3(P_THREADS, 1, 1);
+    cfg.blockDim = dim3(PRoles<CLIP>::THREADS, 1, 1);
     cfg.dynamicSmemBytes = (size_t)G::SMEM;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
