@@ -17,7 +17,7 @@
 //
 // Input: one thread per CTA streams each K chunk's X rows, W rows and codes into a ring of raw
 // shared-memory slots with TMA tile copies (rows past N and channels past C read as zeros).  Eight
-// producer warps (twelve in the clipping search) split X into the B tiles and regenerate the
+// producer warps (sixteen in the clipping search) split X into the B tiles and regenerate the
 // residuals r_{n+1} = r_n - s_n q_n
 // (Eq. 7) from W, codes and scales into the A tiles (128-byte swizzled, K-major); residuals never
 // exist in global memory.  Both CTAs' producers report a full stage to the even CTA, whose MMA
@@ -62,16 +62,16 @@ constexpr int P_EPI_WARPS = 8;                  // two per TMEM lane quarter, on
 
 // Warp roles: producers first, then the epilogue warps (warp % 4 selects TMEM lanes, so the
 // producer count is a multiple of 4), the MMA warp and the TMA warp.  The clipping search's
-// producers regenerate a residual per candidate and bound that mode, so it gets 12 warps of them;
+// producers regenerate a residual per candidate and bound that mode, so it gets 16 warps of them;
 // the greedy mode keeps 8 (more registers per thread).
 template <bool CLIP>
 struct PRoles {
-    static constexpr int PROD_WARPS = CLIP ? 12 : 8;
+    static constexpr int PROD_WARPS = CLIP ? 16 : 8;
     static constexpr int PROD_THREADS = PROD_WARPS * 32;
     static constexpr int EPI_WARP0 = PROD_WARPS;
     static constexpr int MMA_WARP = EPI_WARP0 + P_EPI_WARPS;
     static constexpr int TMA_WARP = MMA_WARP + 1;
-    static constexpr int THREADS = (TMA_WARP + 1) * 32;   // 576 or 704
+    static constexpr int THREADS = (TMA_WARP + 1) * 32;   // 576 or 832
     static_assert(PROD_WARPS % 4 == 0, "epilogue warps start at a TMEM lane quarter boundary");
 };
 constexpr uint32_t P_TMEM_COLS = 512;
