@@ -15,6 +15,7 @@ all ranks / max-over-ranks time.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import os
@@ -245,16 +246,34 @@ def run_ours(args, world, rank, local):
 
     graphs = []
     if args.graph:
-        # one captured graph per bit width (the bit width is a launch argument)
-        for b in wl.bits:
-            for sp in specs:
-                sp.bits = b
-            graphs.append(pipeline.CapturedNetwork(net, Ws, Xs))
+        # one captured graph per bit width (the bit width is a launch argument); each bit width
+        # has its own plan (output buffers), so the graphs replay concurrently on their own streams
+        for n, b in enumerate(wl.bits):
+            if n == 0:
+                for sp in specs:
+                    sp.bits = b
+                plan_b = net
+            else:
+                plan_b = pipeline.NetworkPlan([dataclasses.replace(sp, bits=b) for sp in specs],
+                                              dev, n_streams=args.streams)
+            graphs.append(pipeline.CapturedNetwork(plan_b, Ws, Xs))
+    graph_streams = [torch.cuda.Stream(dev) for _ in graphs]
 
     def step():
+        if len(graphs) == 1:
+            graphs[0].replay()
+            return
         if graphs:
-            for g in graphs:
-                g.replay()
+            ev = torch.cuda.Event()
+            ev.record(stream)
+            for g, gs in zip(graphs, graph_streams):
+                gs.wait_event(ev)
+                with torch.cuda.stream(gs):
+                    g.replay()
+            for gs in graph_streams:
+                e = torch.cuda.Event()
+                e.record(gs)
+                stream.wait_event(e)
             return
         for b in wl.bits:
             for sp in specs:
