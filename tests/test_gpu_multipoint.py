@@ -34,6 +34,7 @@ def run(oracle, codes, scales, npts, X, bits, p):
     (64, 64, 513, 16, 4, 20, [16, 9, 1]),           # R = 16, three 256-input tiles (ragged)
     (1000, 1152, 100, 4, 4, 0, [1, 2]),             # p = 0
     (130, 96, 700, 6, 3, 24, None),                 # 3-bit codes, d not a multiple of 64
+    (20, 8192, 300, 2, 4, 16, None),                # the longest rows (8192 x 7 x 128 < 2^24)
 ])
 def test_tensor_path(gpu, oracle, C, d, T, k_max, bits, p, mix):
     W = wlm.random_weights(C, d, C + d, "laplace")

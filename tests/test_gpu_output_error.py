@@ -23,7 +23,8 @@ def gpu_err(X, W, codes, scales, k_max, groups=1, dev="cuda:0"):
                                      # part-filled last pair, an empty odd CTA, ragged row tiles
                                      # split over a cluster, k_max + 1 from 2 to 17
                                      (130, 256, 600, 4), (30, 128, 1000, 1), (9, 32, 300, 16),
-                                     (50, 512, 1100, 6), (3, 48, 20, 8)])
+                                     (50, 512, 1100, 6), (3, 48, 20, 8),
+                                     (3, 8192, 300, 4)])          # the longest rows taken
 def test_shared_input(gpu, oracle, C, d, N, K):
     W = wlm.random_weights(C, d, C + d + N, "normal")
     q = oracle.quantize_layer(W, 4, 32, K)

@@ -34,6 +34,21 @@ def test_shapes(gpu, oracle, C, d):
     assert rep["near_ties"] <= max(1, C * 4 // 50)
 
 
+def test_max_dim(gpu, oracle):
+    """The longest channel the library takes (d = 8192): residual, bins and lattice on chip."""
+    W = wlm.random_weights(3, 8192, 81, "normal")
+    rep = check(oracle, W, 4, 128, 4)
+    assert rep["near_ties"] <= 1
+
+
+def test_occupancy_variant_without_grid_table(gpu, oracle):
+    """d = 4096 with G = 256 (c5's shape): the launcher drops the grid table and packs the lattice
+    counts to fit one more CTA per SM; results as the definition."""
+    W = wlm.random_weights(24, 4096, 82, "normal")
+    rep = check(oracle, W, 4, 256, 8)
+    assert rep["near_ties"] <= 2
+
+
 @pytest.mark.parametrize("bits", [2, 3, 4, 5, 6, 7, 8])
 def test_bit_widths(gpu, oracle, bits):
     W = wlm.random_weights(16, 200, 50 + bits, "laplace")
