@@ -50,11 +50,13 @@ class LayerPlan:
         self._host = None
 
     # -- device-resident inputs ---------------------------------------------------------------
-    def run_device(self, W, X, stream=None, grid_frac=None, timing=None):
+    def run_device(self, W, X, stream=None, grid_frac=None, timing=None, x_ready=None):
         """Enqueue the four calls (five with centring) on ``stream``.  timing(phase), if given, is
         called before the first call (phase 0) and after the centring (1, also when there is
         none), the greedy points (2), the output error (3), the allocation (4) and the
-        reconstruction (5), e.g. to record CUDA events."""
+        reconstruction (5), e.g. to record CUDA events.  x_ready, if given, is a CUDA event the
+        stream waits on before the output error, the first call that reads X (its copy may still
+        be in flight while the greedy search runs)."""
         s = self.spec
         tick = timing or (lambda ph: None)
         tick(0)
@@ -65,6 +67,8 @@ class LayerPlan:
         binding.mpq_quantize_layer(W, s.bits, s.G, s.k_max, grid_frac=grid_frac, codes=self.codes,
                                    scales=self.scales, resid_sq=self.resid_sq, stream=stream)
         tick(2)
+        if x_ready is not None:
+            (stream or torch.cuda.current_stream()).wait_event(x_ready)
         binding.mpq_output_error(X, W, self.codes, self.scales, s.k_max, groups=s.groups,
                                  err=self.err, stream=stream)
         tick(3)
@@ -164,10 +168,12 @@ class NetworkPlan:
 
     def run_host(self, W_hosts, X_hosts, W_devs, X_devs, stream=None, copy_inputs=True):
         """End to end: per layer, H2D of W and X from pinned memory, the path, D2H of codes,
-        scales, point counts.  Input copies run back to back on one stream (largest layer
-        first), each layer's kernels start on its compute stream as soon as its inputs have
-        landed, and its outputs go back on one D2H stream once its kernels are done -- copies in
-        both directions overlap other layers' kernels.  copy_inputs=False reuses the inputs an
+        scales, point counts.  Input copies run back to back on one stream: every layer's W
+        first, then every layer's X (largest layer first in both).  A layer's greedy search
+        starts on its compute stream as soon as its W has landed and only its output error waits
+        for its X, so the greedy searches overlap the calibration inputs' copies.  Its outputs go
+        back on one D2H stream once its kernels are done -- copies in both directions overlap
+        other layers' kernels.  copy_inputs=False reuses the inputs an
         earlier call copied in (e.g. a second bit width over the same weights).  The caller
         synchronizes ``stream`` before reading the host outputs."""
         main = stream or torch.cuda.current_stream(self.device)
@@ -175,18 +181,18 @@ class NetworkPlan:
         for s in (self.copy_in, self.copy_out):
             s.wait_stream(main)
         outs = [None] * len(self.plans)
-        landed = {}
-        for i in self.order:
-            with torch.cuda.stream(self.copy_in):
-                if copy_inputs:
-                    W_devs[i].copy_(W_hosts[i], non_blocking=True)
-                    X_devs[i].copy_(X_hosts[i], non_blocking=True)
-                landed[i] = torch.cuda.Event()
-                landed[i].record(self.copy_in)
+        w_landed, x_landed = {}, {}
+        with torch.cuda.stream(self.copy_in):
+            for dst, src, landed in ((W_devs, W_hosts, w_landed), (X_devs, X_hosts, x_landed)):
+                for i in self.order:
+                    if copy_inputs:
+                        dst[i].copy_(src[i], non_blocking=True)
+                    landed[i] = torch.cuda.Event()
+                    landed[i].record(self.copy_in)
         for n, i in enumerate(self.order):
             st = self.streams[n % len(self.streams)]
-            st.wait_event(landed[i])
-            self.plans[i].run_device(W_devs[i], X_devs[i], stream=st)
+            st.wait_event(w_landed[i])
+            self.plans[i].run_device(W_devs[i], X_devs[i], stream=st, x_ready=x_landed[i])
             done = torch.cuda.Event()
             done.record(st)
             self.copy_out.wait_event(done)
