@@ -387,8 +387,8 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_
     """Roofline entry of the kernel family with the largest measured time.
 
     output_error: tensor-pipe bound; achieved = algorithmic flops 2*N*d*C*(k_max+1) (the three
-      tf32 split passes are not counted) / measured time; peak = measured bf16 dense burst peak x
-      the nominal tf32/bf16 ratio.
+      fp16 split passes are not counted) / measured time; peak = measured bf16 dense burst peak
+      (kind::f16 runs fp16 and bf16 operands at the same rate).
     quantize: ALU bound; achieved = algorithmic lane operations (quantize_ops) / time; peak = SMs x
       128 lanes x the maximum SM clock.
     reconstruct / allocate / center: HBM roofline; achieved = algorithmic bytes / time."""
@@ -402,14 +402,14 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_
             traffic = ent.get("dram_bytes_per_launch")
     t_s = fam_ms[dominant] / 1e3
     if dominant == "output_error":
-        peak = peaks["bf16_tflops"] * TF32_PER_BF16
+        peak = peaks["bf16_tflops"]
         ach = fam_work[dominant] / t_s / 1e12
-        return {"kernel": "output_error_pair_kernel (Eq. 11, tcgen05 cta_group::2 kind::tf32, "
-                          "3-pass split; output_error_tc_kernel for rows not 16-byte multiples)",
+        return {"kernel": "output_error_pair_kernel (Eq. 11, tcgen05 cta_group::2 kind::f16, "
+                          "scaled fp16 hi/lo operands, 3 passes; after pair_range_kernel; "
+                          "output_error_tc_kernel for rows not 16-byte multiples)",
                 "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
                 "frac": ach / peak, "traffic": traffic,
-                "peak_source": f"{peak_src} bf16 dense burst x nominal tf32/bf16 ratio "
-                               f"{TF32_PER_BF16:.3f}"}
+                "peak_source": f"{peak_src} bf16 dense burst (the fp16 rate of kind::f16)"}
     if dominant == "quantize":
         mhz = peaks.get("sm_max_mhz", 2070.0)
         peak = sm_count * ALU_LANES_PER_SM * mhz * 1e6 / 1e12

@@ -16,7 +16,9 @@
  *    on the device that is current when the call is made, unless an argument says "host".
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Every call
  *    only enqueues work on `stream` and returns; results are ready when the stream reaches them.
- *    No entry point allocates device memory or synchronizes.
+ *    No entry point synchronizes, and none allocates device memory except mpq_output_error's
+ *    small scratch buffer, which comes from the device's stream-ordered pool on `stream` and
+ *    goes back to it on `stream` (see there).
  *  - Arguments are validated on the host before anything is enqueued; an invalid argument
  *    returns MPQ_ERR_INVALID_ARG / MPQ_ERR_UNSUPPORTED and leaves every output untouched.
  *    A failed kernel launch returns MPQ_ERR_CUDA.  mpq_last_error() gives a message for the
@@ -43,7 +45,7 @@ typedef enum {
     MPQ_ERR_UNSUPPORTED = 3,  /* valid for the method but beyond this library's limits below */
     MPQ_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
     MPQ_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up (reserved) */
-    MPQ_ERR_NOMEM = 6         /* reserved: no entry point allocates */
+    MPQ_ERR_NOMEM = 6         /* mpq_output_error's stream-ordered scratch allocation failed */
 } mpq_status;
 
 /* Library limits. */
@@ -110,6 +112,13 @@ mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
  *   groups  1 or C.
  *   W, codes, scales, C, d, k_max   as produced by / passed to mpq_quantize_layer.
  *   err     out [C][k_max+1] fp32.
+ *
+ * Scratch: with groups == 1, d a multiple of 16 and X, W, codes 16-byte aligned (the tensor-core
+ * path with scaled fp16 operands), the call takes 4 (1 + C (k_max+1)) bytes from the current
+ * device's default stream-ordered memory pool with cudaMallocAsync on `stream` and returns them
+ * with cudaFreeAsync on `stream` -- concurrent calls on other streams each get their own, and a
+ * CUDA graph capture records them as the graph's allocation nodes.  MPQ_ERR_NOMEM if that
+ * allocation fails (nothing else is enqueued then).
  */
 mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
                             const int8_t *codes, const float *scales, int C, int d, int k_max,

@@ -9,18 +9,24 @@
 // the operand bytes each SM's tensor core reads and the residual vectors each SM regenerates,
 // compared with one CTA computing 256 vectors x 128 rows alone.
 //
-// Precision is that of the single-CTA kernel: each operand is split exactly into a tf32 hi part and
-// an fp32 lo part and Y = hi*hi + hi*lo + lo*hi on kind::tf32; the accumulator restarts every 128
-// elements of d and the epilogue folds each segment into fp32 running sums in tensor memory
-// (columns [0, 256) segment, [256, 512) running sums), since the tensor core's accumulation
-// truncates.
+// Precision.  Greedy residuals: pair_range_kernel first measures max|X| and max|r| of every residual
+// vector; each operand is scaled by the power of two 2^e that puts its largest element in
+// [2^14, 2^15) and split into fp16 hi = fl16(x) and lo = fl16(x - hi), and Y = hi*hi + hi*lo + lo*hi
+// runs on kind::f16 (fp32 accumulate) -- 22 significant bits per operand like a tf32 hi/lo split,
+// at twice the tf32 rate; the reduction multiplies each mean by 2^-2(e_X + e_v) exactly, in double.
+// Clipping-search residuals keep the tf32 split (hi = x with 13 mantissa bits cleared, lo = x - hi)
+// on kind::tf32.  The accumulator restarts every 256 (fp16) or 128 (tf32) elements of d and the
+// epilogue folds each segment into fp32 running sums in tensor memory (columns [0, 256) segment,
+// [256, 512) running sums), since the tensor core's accumulation truncates.
 //
 // Input: one thread per CTA streams each K chunk's X rows, W rows and codes into a ring of raw
 // shared-memory slots with TMA tile copies (rows past N and channels past C read as zeros).  Eight
 // producer warps (sixteen in the clipping search) split X into the B tiles and regenerate the
 // residuals r_{n+1} = r_n - s_n q_n
 // (Eq. 7) from W, codes and scales into the A tiles (128-byte swizzled, K-major); residuals never
-// exist in global memory.  Both CTAs' producers report a full stage to the even CTA, whose MMA
+// exist in global memory.  Two 64 KB tile sets hold the stages: with fp16 operands a 32-element
+// chunk fills a 64-byte half of every row (4 stages), with tf32 operands a whole row (2 stages).
+// Both CTAs' producers report a full stage to the even CTA, whose MMA
 // thread issues the pair MMAs and signals both CTAs (multicast commits) when a stage or a segment
 // is consumed.  Eight epilogue warps per CTA (one per TMEM lane quarter and column half) drain the
 // segments; a segment is restarted only once both CTAs' epilogues have released it.
@@ -30,9 +36,11 @@
 // on a timeout the outputs read NaN.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+#include <cuda_fp16.h>
 #include <math.h>
 #include <string.h>
 
+#include <algorithm>
 #include <atomic>
 
 #include "mpq_internal.cuh"
@@ -50,15 +58,25 @@ constexpr int P_ROWS = 128;                     // calibration rows per CTA
 constexpr int P_N = 2 * P_ROWS;                 // rows per pair row tile (UMMA N)
 constexpr int P_KC = 32;                        // fp32 per K chunk = one 128-byte swizzle row
 constexpr int P_KC4 = P_KC / 4;
-constexpr int P_SEG = 4;                        // chunks per accumulation segment (128 elements)
-constexpr int P_STAGES = 2;                     // operand stages
 constexpr int P_TILE = 128 * P_KC * 4;          // 16 KB: one 128-row operand tile
 constexpr int P_OFF_A_HI = 0;
 constexpr int P_OFF_A_LO = P_TILE;
 constexpr int P_OFF_B_HI = 2 * P_TILE;
 constexpr int P_OFF_B_LO = 3 * P_TILE;
-constexpr int P_STAGE_BYTES = 4 * P_TILE;       // 64 KB
+constexpr int P_STAGE_BYTES = 4 * P_TILE;       // 64 KB: one set of A hi/lo, B hi/lo tiles
+constexpr int P_TILE_SETS = 2;
+constexpr int P_MAX_STAGES = 4;
 constexpr int P_EPI_WARPS = 8;                  // two per TMEM lane quarter, one per column half
+
+// Operand format per mode.  fp32 operands (the clipping search): a K chunk of 32 elements fills
+// a tile set's 128-byte rows as tf32 hi/lo parts, 2 stages, accumulator restarted every 4 chunks.
+// fp16 operands (the greedy residuals): a chunk fills half of each row (64 bytes), so the two
+// tile sets hold 4 stages, and the accumulator restarts every 8 chunks (256 elements).
+template <bool F16>
+struct PFmt {
+    static constexpr int STAGES = F16 ? 4 : 2;
+    static constexpr int SEG = F16 ? 8 : 4;     // chunks per accumulation segment
+};
 
 // Warp roles: producers first, then the epilogue warps (warp % 4 selects TMEM lanes, so the
 // producer count is a multiple of 4), the MMA warp and the TMA warp.  The clipping search's
@@ -81,8 +99,8 @@ constexpr long long P_WAIT = 1LL << 31;         // SM clocks (~1 s)
 constexpr int P_SMEM_LIMIT = 232448;            // opt-in shared memory per CTA on sm_100 parts
 
 struct PairCtrl {
-    uint64_t full[P_STAGES];      // even CTA: both CTAs' producer warps
-    uint64_t empty[P_STAGES];     // both CTAs: pair MMA commit
+    uint64_t full[P_MAX_STAGES];  // even CTA: both CTAs' producer warps
+    uint64_t empty[P_MAX_STAGES]; // both CTAs: pair MMA commit
     uint64_t raw_full[P_MAX_RAW];
     uint64_t raw_empty[P_MAX_RAW];
     uint64_t segfull;             // both CTAs: pair MMA commit
@@ -93,9 +111,42 @@ struct PairCtrl {
     double part[2][P_VEC];        // per column half: sum over the rows' y^2
     float clip_s[P_VEC];          // clipping search: scale K / Qmax and fl(1 / scale) per row
     float clip_inv[P_VEC];
+    float vscale[P_VEC];          // fp16 operands: 2^e per residual vector, 2^e for X
+    int vexp[P_VEC];
+    float xscale;
+    int xexp;
 };
 constexpr int P_CTRL_BYTES = (sizeof(PairCtrl) + 1023) / 1024 * 1024;
-constexpr int P_BASE_SMEM = 1024 /* alignment slack */ + P_CTRL_BYTES + P_STAGES * P_STAGE_BYTES;
+constexpr int P_BASE_SMEM = 1024 /* alignment slack */ + P_CTRL_BYTES + P_TILE_SETS * P_STAGE_BYTES;
+
+// fp16 operands: exponent e with m * 2^e in [2^14, 2^15) for the largest magnitude m of a residual
+// vector or of X, so that the vector's hi and lo halves are normal fp16 numbers down to 2^-7 of its
+// largest element (and nothing overflows).  0 for m = 0, NaN or inf (which then propagate); capped
+// at 126 so that 2^e stays a normal float (only vectors below 2^-111 are scaled less).
+__device__ __forceinline__ int f16_scale_exp(float m)
+{
+    if (!(m > 0.0f) || !isfinite(m)) return 0;
+    int E;
+    (void)frexpf(m, &E);              // m = f 2^E, f in [0.5, 1)
+    return min(15 - E, 126);
+}
+
+__device__ __forceinline__ float pow2f(int e) { return __int_as_float((127 + e) << 23); }
+
+__device__ __forceinline__ double pow2d(int e)
+{
+    return __longlong_as_double((long long)(1023 + e) << 52);
+}
+
+// x * 2^e (exact) split into fp16 hi + lo: hi = fl16(x), lo = fl16(x - hi) (x - hi is exact in fp32).
+__device__ __forceinline__ void split_f16x2(float a, float b, uint32_t &hi, uint32_t &lo)
+{
+    const __half2 h = __floats2half2_rn(a, b);
+    const float2 hf = __half22float2(h);
+    const __half2 l = __floats2half2_rn(__fsub_rn(a, hf.x), __fsub_rn(b, hf.y));
+    hi = *reinterpret_cast<const uint32_t *>(&h);
+    lo = *reinterpret_cast<const uint32_t *>(&l);
+}
 
 // Per-KP1 geometry and the raw slot layout, in the order the tile copies write it:
 // X chunk [128 rows][32] fp32, W chunk [CH][32] fp32, codes [K][CH][32] int8.  KP1 is the number of
@@ -105,6 +156,7 @@ template <int KP1, bool CLIP = false>
 struct PGeo {
     static constexpr int K = CLIP ? 0 : KP1 - 1;
     static constexpr int KQ = K > 0 ? K : 1;
+    static constexpr int VF = CLIP ? 1 : KP1;   // fp16 operand scales per item
     static constexpr int CH = P_VEC / KP1;
     static constexpr int PT = PRoles<CLIP>::PROD_THREADS;
     static constexpr int ITEMS2 = (CH * (P_KC / 2) + PT - 1) / PT;
@@ -119,13 +171,16 @@ struct PGeo {
     static_assert(RAW_STAGES >= 2, "raw ring needs two slots");
 };
 
-// Raw slot -> operand stage `sb`: X rows -> B tiles; for every (channel, element pair) item the
-// residuals -> A tiles: r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7), or (CLIP) r_c = w - s_c [w / s_c]_Q
-// for every candidate clipping factor (Eq. 12), with the scales and reciprocals of `ctl`.
+// Raw slot -> operand stage (tile set `sb`, row half `hh` with fp16 operands): X rows -> B tiles;
+// for every (channel, element pair) item the residuals -> A tiles: r_0 = w, r_{n+1} = r_n - s_n q_n
+// (Eq. 7), or (CLIP) r_c = w - s_c [w / s_c]_Q for every candidate clipping factor (Eq. 12), with
+// the scales and reciprocals of `ctl`.  fp16 operands are scaled by 2^e first (xs for X, vf per
+// residual vector), which the reduction undoes exactly.
 template <int KP1, bool CLIP>
-__device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt, int nch,
+__device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh, int pt, int nch,
                                              const float (&sc)[PGeo<KP1, CLIP>::ITEMS2][PGeo<KP1, CLIP>::KQ],
-                                             const PairCtrl &ctl, float qmaxf)
+                                             const float (&vf)[PGeo<KP1, CLIP>::ITEMS2][PGeo<KP1, CLIP>::VF],
+                                             float xs, const PairCtrl &ctl, float qmaxf)
 {
     using G = PGeo<KP1, CLIP>;
     constexpr int K = G::K;
@@ -142,11 +197,21 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
     for (int i = 0; i < G::X_ITEMS; ++i) {
         const int q = pt + i * G::PT;
         if (G::X_ITEMS * G::PT != XN && q >= XN) break;
-        float4 hi, lo;
-        split4(xr[i], hi, lo);
-        const uint32_t off = sw128_offset(q / P_KC4, q % P_KC4);
-        st_shared_v4(sb + P_OFF_B_HI + off, hi);
-        st_shared_v4(sb + P_OFF_B_LO + off, lo);
+        if constexpr (CLIP) {
+            float4 hi, lo;
+            split4(xr[i], hi, lo);
+            const uint32_t off = sw128_offset(q / P_KC4, q % P_KC4);
+            st_shared_v4(sb + P_OFF_B_HI + off, hi);
+            st_shared_v4(sb + P_OFF_B_LO + off, lo);
+        } else {
+            uint32_t h0, l0, h1, l1;
+            split_f16x2(__fmul_rn(xr[i].x, xs), __fmul_rn(xr[i].y, xs), h0, l0);
+            split_f16x2(__fmul_rn(xr[i].z, xs), __fmul_rn(xr[i].w, xs), h1, l1);
+            const int q4 = q % P_KC4;                  // 4 elements = 8 bytes of a 64-byte half row
+            const uint32_t off = sw128_offset(q / P_KC4, hh * 4 + (q4 >> 1)) + (uint32_t)(q4 & 1) * 8u;
+            st_shared_v2u(sb + P_OFF_B_HI + off, h0, h1);
+            st_shared_v2u(sb + P_OFF_B_LO + off, l0, l1);
+        }
     }
 #pragma unroll
     for (int i = 0; i < G::ITEMS2; ++i) {
@@ -159,14 +224,15 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
             for (int n = 0; n < K; ++n)
                 qb[n] = ld_shared_u16(slot + G::RAW_Q + (uint32_t)((n * G::CH + ch) * P_KC + e2 * 2)) ^
                         0x8080u;
-            const uint32_t cofs = (uint32_t)(e2 & 1) * 8u;
+            const int hc = hh * 4 + (e2 >> 2);         // 2 elements = 4 bytes of a half row
+            const uint32_t cofs = (uint32_t)(e2 & 3) * 4u;
 #pragma unroll
             for (int n = 0; n < KP1; ++n) {
-                float2 hi, lo;
-                split2(r, hi, lo);
-                const uint32_t off = sw128_offset(ch * KP1 + n, e2 >> 1) + cofs;
-                st_shared_v2(sb + P_OFF_A_HI + off, hi);
-                st_shared_v2(sb + P_OFF_A_LO + off, lo);
+                uint32_t hi, lo;
+                split_f16x2(__fmul_rn(r.x, vf[i][n]), __fmul_rn(r.y, vf[i][n]), hi, lo);
+                const uint32_t off = sw128_offset(ch * KP1 + n, hc) + cofs;
+                st_shared_u32(sb + P_OFF_A_HI + off, hi);
+                st_shared_u32(sb + P_OFF_A_LO + off, lo);
                 if (n < K) {
                     const float sn = sc[i][n];
                     r.x = __fmaf_rn(-sn, code_from_biased(qb[n], 0), r.x);
@@ -221,24 +287,27 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int pt,
 }
 
 // scales: [C][k_max] point scales, or (CLIP) [C][KP1] candidate clipping factors K; qmax: the
-// code range for CLIP.
+// code range for CLIP; range (fp16 operands): max|X| and max|r| per residual vector, as float bits
+// (pair_range_kernel).
 template <int KP1, bool CLIP>
 __global__ void __launch_bounds__(PRoles<CLIP>::THREADS, 1)
 output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, int qmax,
-                         float *__restrict__ err, int split,
+                         const unsigned *__restrict__ range, float *__restrict__ err, int split,
                          const __grid_constant__ CUtensorMap tmX,
                          const __grid_constant__ CUtensorMap tmW,
                          const __grid_constant__ CUtensorMap tmQ)
 {
     using G = PGeo<KP1, CLIP>;
     using PR = PRoles<CLIP>;
+    constexpr bool F16 = !CLIP;
+    constexpr int NST = PFmt<F16>::STAGES, SEG = PFmt<F16>::SEG;
     constexpr int R = G::RAW_STAGES;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
     PairCtrl &ctl = *reinterpret_cast<PairCtrl *>(smem_raw + pad);
     const uint32_t stages_u32 = raw_u32 + pad + P_CTRL_BYTES;
-    const uint32_t ring_u32 = stages_u32 + P_STAGES * P_STAGE_BYTES;
+    const uint32_t ring_u32 = stages_u32 + P_TILE_SETS * P_STAGE_BYTES;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t crank = cluster_ctarank();
@@ -253,11 +322,11 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
     const int n_rt = (N + P_N - 1) / P_N;
     const int my_rt = (n_rt - pr + split - 1) / split;
     const int n_kc = (d + P_KC - 1) / P_KC;
-    const int nseg = (n_kc + P_SEG - 1) / P_SEG;
+    const int nseg = (n_kc + SEG - 1) / SEG;
     const int total = my_rt * n_kc;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < P_STAGES; ++s) {
+        for (int s = 0; s < NST; ++s) {
             mbar_init(&ctl.full[s], 2 * PR::PROD_WARPS);
             mbar_init(&ctl.empty[s], 1);
         }
@@ -278,6 +347,17 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             ctl.clip_s[i] = s;
             ctl.clip_inv[i] = s > 0.0f ? __frcp_rn(s) : 0.0f;
         }
+    } else {
+        for (int i = threadIdx.x; i < nvec; i += PR::THREADS) {
+            const int e = f16_scale_exp(__uint_as_float(__ldg(range + 1 + (size_t)k0 * KP1 + i)));
+            ctl.vexp[i] = e;
+            ctl.vscale[i] = pow2f(e);
+        }
+        if (threadIdx.x == 0) {
+            const int e = f16_scale_exp(__uint_as_float(__ldg(range)));
+            ctl.xexp = e;
+            ctl.xscale = pow2f(e);
+        }
     }
     if (warp == PR::MMA_WARP) {
         tmem_alloc_pair(&ctl.tmem_base, P_TMEM_COLS);
@@ -292,24 +372,30 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         // ---------------------------------------------------------------- producers
         const int pt = threadIdx.x;
         float sc[G::ITEMS2][G::KQ];     // scales of this thread's items, the same for every chunk
+        float vf[G::ITEMS2][G::VF];     // fp16 operands: 2^e of the items' residual vectors
 #pragma unroll
         for (int i = 0; i < G::ITEMS2; ++i) {
             const int p = pt + i * PR::PROD_THREADS;
             const int k = k0 + p / (P_KC / 2);
+            const bool own = !CLIP && p < nch * (P_KC / 2);
 #pragma unroll
             for (int n = 0; n < G::KQ; ++n)
-                sc[i][n] = (!CLIP && n < KP1 - 1 && p < nch * (P_KC / 2))
-                               ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
+                sc[i][n] = (own && n < KP1 - 1) ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
+#pragma unroll
+            for (int n = 0; n < G::VF; ++n)
+                vf[i][n] = own ? ctl.vscale[(p / (P_KC / 2)) * KP1 + n] : 0.0f;
         }
+        const float xs = F16 ? ctl.xscale : 1.0f;
         for (int it = 0; it < total; ++it) {
-            const int s = it % P_STAGES, slot = it % R;
-            const uint32_t ph = (uint32_t)(it / P_STAGES) & 1u;
+            const int s = it % NST, slot = it % R;
+            const uint32_t ph = (uint32_t)(it / NST) & 1u;
             const bool ok = mbar_wait(&ctl.raw_full[slot], (uint32_t)(it / R) & 1u, P_WAIT) &&
                             mbar_wait_cluster(&ctl.empty[s], ph ^ 1u, P_WAIT);
             if (!ok) *abort_flag = 1;
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-            pair_consume<KP1, CLIP>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + s * P_STAGE_BYTES,
-                                    pt, nch, sc, ctl, qmaxf);
+            const int ts = F16 ? s >> 1 : s, hh = F16 ? s & 1 : 0;
+            pair_consume<KP1, CLIP>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + ts * P_STAGE_BYTES,
+                                    hh, pt, nch, sc, vf, xs, ctl, qmaxf);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
@@ -364,11 +450,11 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
     } else if (warp == PR::MMA_WARP) {
         // ---------------------------------------------------------------- MMA issuer (even CTA)
         if (half == 0 && lane == 0) {
-            constexpr uint32_t idesc = idesc_tf32(2 * P_VEC, P_N);
+            constexpr uint32_t idesc = F16 ? idesc_f16(2 * P_VEC, P_N) : idesc_tf32(2 * P_VEC, P_N);
             int g = 0;
             for (int lt = 0; lt < my_rt && !*abort_flag; ++lt) {
                 for (int kc = 0; kc < n_kc; ++kc) {
-                    const bool seg_start = (kc % P_SEG) == 0;
+                    const bool seg_start = (kc % SEG) == 0;
                     if (seg_start) {
                         // both CTAs' epilogues must have drained the previous segment
                         if (!mbar_wait_cluster(&ctl.segempty, ((uint32_t)g & 1u) ^ 1u, P_WAIT))
@@ -377,25 +463,36 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                         tc_fence_after();
                     }
                     const int it = lt * n_kc + kc;
-                    const int s = it % P_STAGES;
-                    const uint32_t ph = (uint32_t)(it / P_STAGES) & 1u;
+                    const int s = it % NST;
+                    const uint32_t ph = (uint32_t)(it / NST) & 1u;
                     if (!mbar_wait_cluster(&ctl.full[s], ph, P_WAIT)) *abort_flag = 1;
                     if (*abort_flag) break;
                     tc_fence_after();
-                    const uint32_t sb = stages_u32 + s * P_STAGE_BYTES;
+                    const uint32_t sb = stages_u32 + (F16 ? s >> 1 : s) * P_STAGE_BYTES;
                     const uint64_t ah = smem_desc_sw128(sb + P_OFF_A_HI);
                     const uint64_t al = smem_desc_sw128(sb + P_OFF_A_LO);
                     const uint64_t bh = smem_desc_sw128(sb + P_OFF_B_HI);
                     const uint64_t bl = smem_desc_sw128(sb + P_OFF_B_LO);
+                    if constexpr (F16) {
+                        // 32 fp16 elements of this stage's row half = two K = 16 steps of 32 bytes
 #pragma unroll
-                    for (int kk = 0; kk < P_KC / 8; ++kk) {
-                        const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
-                        mma_tf32_pair(tmem, al + o, bh + o, idesc, (seg_start && kk == 0) ? 0u : 1u);
-                        mma_tf32_pair(tmem, ah + o, bl + o, idesc, 1u);
-                        mma_tf32_pair(tmem, ah + o, bh + o, idesc, 1u);
+                        for (int kk = 0; kk < 2; ++kk) {
+                            const uint64_t o = (uint64_t)(((s & 1) * 2 + kk) * 2);   // 16 B units
+                            mma_f16_pair(tmem, al + o, bh + o, idesc, (seg_start && kk == 0) ? 0u : 1u);
+                            mma_f16_pair(tmem, ah + o, bl + o, idesc, 1u);
+                            mma_f16_pair(tmem, ah + o, bh + o, idesc, 1u);
+                        }
+                    } else {
+#pragma unroll
+                        for (int kk = 0; kk < P_KC / 8; ++kk) {
+                            const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
+                            mma_tf32_pair(tmem, al + o, bh + o, idesc, (seg_start && kk == 0) ? 0u : 1u);
+                            mma_tf32_pair(tmem, ah + o, bl + o, idesc, 1u);
+                            mma_tf32_pair(tmem, ah + o, bh + o, idesc, 1u);
+                        }
                     }
                     mma_commit_pair(&ctl.empty[s], pair_mask);
-                    if ((kc % P_SEG) == P_SEG - 1 || kc == n_kc - 1) {
+                    if ((kc % SEG) == SEG - 1 || kc == n_kc - 1) {
                         mma_commit_pair(&ctl.segfull, pair_mask);
                         ++g;
                     }
@@ -445,7 +542,9 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 s += ld_dsmem_f64(&ctl.part[0][m], crank + 2u * (uint32_t)j);
                 s += ld_dsmem_f64(&ctl.part[1][m], crank + 2u * (uint32_t)j);
             }
-            err[(size_t)k0 * KP1 + m] = (float)(s / (double)N);
+            double v = s / (double)N;
+            if (F16) v *= pow2d(-2 * (ctl.xexp + ctl.vexp[m]));   // exact: undo the operand scales
+            err[(size_t)k0 * KP1 + m] = (float)v;
         }
     }
     cluster_sync();
@@ -453,6 +552,87 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         tc_fence_after();
         tmem_dealloc_pair(tmem, P_TMEM_COLS);
     }
+}
+
+__device__ __forceinline__ float max_abs4(float4 v)
+{
+    return fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w)));
+}
+
+// Ranges for the fp16 operand scales: blocks [0, xb) fold max|X| into range[0] (float bits of a
+// non-negative value order like unsigned integers; range[0] starts at 0); the other blocks take one
+// channel per warp and write max_j |r_{k,n+1,j}| of every residual vector (the same fp32 recursion
+// of Eq. 7 as the contraction's producers) to range[1 + k (k_max + 1) + n].  d % 4 == 0, rows and
+// code planes 16-byte aligned.
+template <int KP1>
+__global__ void __launch_bounds__(256)
+pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const float *__restrict__ W,
+                  const int8_t *__restrict__ codes, const float *__restrict__ scales, int C, int d,
+                  unsigned *__restrict__ range)
+{
+    constexpr int K = KP1 - 1;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if ((int)blockIdx.x < xb) {
+        float m = 0.0f;
+        for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nx4;
+             i += (long long)xb * blockDim.x)
+            m = fmaxf(m, max_abs4(__ldg(X + i)));
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        if (lane == 0) atomicMax(range, __float_as_uint(m));
+        return;
+    }
+    const int k = ((int)blockIdx.x - xb) * 8 + warp;
+    if (k >= C) return;
+    float sc[K > 0 ? K : 1], mx[KP1];
+#pragma unroll
+    for (int n = 0; n < K; ++n) sc[n] = __ldg(scales + (size_t)k * K + n);
+#pragma unroll
+    for (int n = 0; n < KP1; ++n) mx[n] = 0.0f;
+    const float4 *w4 = reinterpret_cast<const float4 *>(W + (size_t)k * d);
+    for (int j = lane; j < d / 4; j += 32) {
+        float4 r = __ldg(w4 + j);
+        mx[0] = fmaxf(mx[0], max_abs4(r));
+#pragma unroll
+        for (int n = 0; n < K; ++n) {
+            const char4 q = __ldg(reinterpret_cast<const char4 *>(codes + ((size_t)n * C + k) * d) + j);
+            r.x = __fmaf_rn(-sc[n], (float)q.x, r.x);
+            r.y = __fmaf_rn(-sc[n], (float)q.y, r.y);
+            r.z = __fmaf_rn(-sc[n], (float)q.z, r.z);
+            r.w = __fmaf_rn(-sc[n], (float)q.w, r.w);
+            mx[n + 1] = fmaxf(mx[n + 1], max_abs4(r));
+        }
+    }
+#pragma unroll
+    for (int n = 0; n < KP1; ++n) {
+        float m = mx[n];
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        if (lane == 0) range[1 + (size_t)k * KP1 + n] = __float_as_uint(m);
+    }
+}
+
+// Scratch of the fp16 contraction comes from the device's stream-ordered pool (allocated and
+// freed on the call's stream, so concurrent calls on other streams never share it; inside a CUDA
+// graph capture these become the graph's own allocation nodes).  Freed blocks stay cached in the
+// pool instead of going back to the driver at every synchronisation.
+mpq_status pair_scratch(void **p, size_t bytes, cudaStream_t stream)
+{
+    static std::atomic<int> pool_set{0};
+    if (!pool_set.exchange(1)) {
+        int dev = 0;
+        cudaMemPool_t pool;
+        if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetDefaultMemPool(&pool, dev) == cudaSuccess) {
+            uint64_t keep = UINT64_MAX;
+            (void)cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        }
+        (void)cudaGetLastError();
+    }
+    const cudaError_t e = cudaMallocAsync(p, bytes, stream);
+    if (e == cudaErrorMemoryAllocation) {
+        (void)cudaGetLastError();
+        set_error("output error: no %zu bytes of scratch in the stream-ordered pool", bytes);
+        return MPQ_ERR_NOMEM;
+    }
+    return cuda_status(e, "scratch allocation (cudaMallocAsync)");
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 pair_map_encoder()
@@ -554,8 +734,29 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     }
     attr[0].val.clusterDim.x = (unsigned)(2 * split);
     cfg.gridDim = dim3((unsigned)(n_pairs * 2 * split), 1, 1);
-    e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax, err,
-                           split, tmX, tmW, tmQ);
+    unsigned *range = nullptr;
+    if constexpr (!CLIP) {
+        // fp16 operands: the ranges of X and of every residual vector first
+        mpq_status st = pair_scratch(reinterpret_cast<void **>(&range),
+                                     (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
+        if (st != MPQ_OK) return st;
+        const long long nx4 = (long long)N * d / 4;
+        const int xb = (int)std::min<long long>((nx4 + 255) / 256, 2LL * sm_count());
+        e = cudaMemsetAsync(range, 0, sizeof(unsigned), stream);
+        if (e == cudaSuccess) {
+            pair_range_kernel<KP1><<<xb + (C + 7) / 8, 256, 0, stream>>>(
+                reinterpret_cast<const float4 *>(X), nx4, xb, W, codes, scales, C, d, range);
+            e = cudaGetLastError();
+        }
+        if (e == cudaSuccess)
+            e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
+                                   (const unsigned *)range, err, split, tmX, tmW, tmQ);
+        const cudaError_t ef = cudaFreeAsync(range, stream);
+        if (e == cudaSuccess) e = ef;
+        return cuda_status(e, "pair output-error kernel launch");
+    }
+    e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
+                           (const unsigned *)nullptr, err, split, tmX, tmW, tmQ);
     return cuda_status(e, "pair output-error kernel launch");
 }
 

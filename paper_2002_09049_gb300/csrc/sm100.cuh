@@ -180,6 +180,18 @@ __device__ __forceinline__ void mma_tf32_pair(uint32_t d_tmem, uint64_t a_desc, 
         : "memory");
 }
 
+// CTA-pair MMA of kind::f16 with fp16 A and B (fp32 accumulate); operands as in mma_tf32_pair.
+__device__ __forceinline__ void mma_f16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                             uint32_t idesc, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // Arrives on the barrier at `bar`'s offset in every CTA of `cta_mask` once every pair MMA issued
 // so far by this thread has completed.
 __device__ __forceinline__ void mma_commit_pair(uint64_t *bar, uint16_t cta_mask)
@@ -348,11 +360,31 @@ __device__ __forceinline__ void st_shared_v2(uint32_t addr, float2 v)
     asm volatile("st.shared.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(v.x), "f"(v.y) : "memory");
 }
 
+__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v)
+{
+    asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void st_shared_v2u(uint32_t addr, uint32_t a, uint32_t b)
+{
+    asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
+}
+
 __device__ __forceinline__ uint32_t ld_shared_u16(uint32_t addr)
 {
     uint16_t v;
     asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(addr) : "memory");
     return v;
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulate, A and B fp16, both K-major.
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N)
+{
+    return (1u << 4)                      // D format: f32
+           | (0u << 7)                    // A format: f16
+           | (0u << 10)                   // B format: f16
+           | ((uint32_t)(N >> 3) << 17)   // N / 8
+           | ((uint32_t)(M >> 4) << 24);  // M / 16
 }
 
 // Instruction descriptor, kind::f16: fp32 accumulate, A and B bf16, both K-major.

@@ -73,3 +73,21 @@ def test_nonfinite_weight_propagates(gpu, oracle):
     X = wlm.random_calibration(10, 20, 2)
     e = gpu_err(X, W, q["codes"], q["scales"], 2)
     assert np.all(np.isnan(e[1])) and np.all(np.isfinite(e[[0, 2]]))
+
+
+@pytest.mark.parametrize("x_exp,w_exp", [(40, -60), (-50, 30), (0, -40)])
+def test_operand_scaling_extremes(gpu, oracle, x_exp, w_exp):
+    """fp16 operands are scaled per residual vector and per layer of X: inputs scaled by powers of
+    two far from 1 (the oracle's double result scales exactly), residuals that reach 0 after one
+    point, and calibration rows many binades below the others."""
+    C, d, N, K = 40, 256, 300, 6
+    W = wlm.random_weights(C, d, 3, "normal")
+    W[5] = np.ldexp(np.round(W[5] * 64), -8).astype(np.float32)    # few distinct values
+    W[6] = 0.0
+    X = wlm.random_calibration(N, d, 4)
+    X[::7] *= np.float32(2.0 ** -30)
+    W = np.ldexp(W, w_exp).astype(np.float32)
+    X = np.ldexp(X, x_exp).astype(np.float32)
+    q = oracle.quantize_layer(W, 4, 32, K)
+    compare_err(gpu_err(X, W, q["codes"], q["scales"], K),
+                oracle.output_error(X, 1, W, q["codes"], q["scales"], K))
