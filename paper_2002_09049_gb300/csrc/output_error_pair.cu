@@ -171,6 +171,29 @@ struct PGeo {
     static_assert(RAW_STAGES >= 2, "raw ring needs two slots");
 };
 
+// fp16 operand stores fill 64-byte half rows, and the 128-byte swizzle puts a half row in banks
+// 0-15 or 16-31 by bit 2 of its row.  So that each warp store reaches both bank halves:
+// X item q (16 bytes of raw input) of a warp's 32 items goes to rows {r, r+1, r+4, r+5} of an 8-row
+// atom ...
+__device__ __forceinline__ int pair_x_item(int q)
+{
+    const int g = q >> 5, j = (q & 31) >> 3;
+    const int row = (g >> 1) * 8 + (g & 1) * 2 + (j & 1) + (j >> 1) * 4;
+    return row * P_KC4 + (q & 7);
+}
+
+// ... and the two channels of a warp's residual items (slots j = 2t, 2t+1) are D apart, with
+// D (k_max+1) = 4 (mod 8) where possible, so that their rows differ in bit 2.  A bijection of the
+// slots 0..nch-1 (the tail that does not fill a block of 2D slots is kept in place).
+template <int KP1>
+__device__ __forceinline__ int pair_channel(int j, int nch)
+{
+    constexpr int D = (KP1 & 1) ? 4 : ((KP1 & 3) == 2 ? 2 : 1);
+    if (j >= nch / (2 * D) * (2 * D)) return j;
+    const int w = j % (2 * D);
+    return j - w + (w >> 1) + (w & 1) * D;
+}
+
 // Raw slot -> operand stage (tile set `sb`, row half `hh` with fp16 operands): X rows -> B tiles;
 // for every (channel, element pair) item the residuals -> A tiles: r_0 = w, r_{n+1} = r_n - s_n q_n
 // (Eq. 7), or (CLIP) r_c = w - s_c [w / s_c]_Q for every candidate clipping factor (Eq. 12), with
@@ -178,6 +201,7 @@ struct PGeo {
 // residual vector), which the reduction undoes exactly.
 template <int KP1, bool CLIP>
 __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh, int pt, int nch,
+                                             const int (&chs)[PGeo<KP1, CLIP>::ITEMS2],
                                              const float (&sc)[PGeo<KP1, CLIP>::ITEMS2][PGeo<KP1, CLIP>::KQ],
                                              const float (&vf)[PGeo<KP1, CLIP>::ITEMS2][PGeo<KP1, CLIP>::VF],
                                              float xs, const PairCtrl &ctl, float qmaxf)
@@ -191,7 +215,8 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh,
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
         const int q = pt + i * G::PT;
-        if (G::X_ITEMS * G::PT == XN || q < XN) xr[i] = ld_shared_v4(slot + (uint32_t)q * 16u);
+        const int qi = CLIP ? q : pair_x_item(q);
+        if (G::X_ITEMS * G::PT == XN || q < XN) xr[i] = ld_shared_v4(slot + (uint32_t)qi * 16u);
     }
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
@@ -207,8 +232,8 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh,
             uint32_t h0, l0, h1, l1;
             split_f16x2(__fmul_rn(xr[i].x, xs), __fmul_rn(xr[i].y, xs), h0, l0);
             split_f16x2(__fmul_rn(xr[i].z, xs), __fmul_rn(xr[i].w, xs), h1, l1);
-            const int q4 = q % P_KC4;                  // 4 elements = 8 bytes of a 64-byte half row
-            const uint32_t off = sw128_offset(q / P_KC4, hh * 4 + (q4 >> 1)) + (uint32_t)(q4 & 1) * 8u;
+            const int qi = pair_x_item(q), q4 = qi % P_KC4;   // 4 elements = 8 bytes of a half row
+            const uint32_t off = sw128_offset(qi / P_KC4, hh * 4 + (q4 >> 1)) + (uint32_t)(q4 & 1) * 8u;
             st_shared_v2u(sb + P_OFF_B_HI + off, h0, h1);
             st_shared_v2u(sb + P_OFF_B_LO + off, l0, l1);
         }
@@ -217,7 +242,7 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh,
     for (int i = 0; i < G::ITEMS2; ++i) {
         const int p = pt + i * G::PT;
         if (!CLIP && p < nch * (P_KC / 2)) {
-            const int ch = p / (P_KC / 2), e2 = p % (P_KC / 2);
+            const int ch = chs[i], e2 = p % (P_KC / 2);
             float2 r = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
             uint32_t qb[G::KQ];
 #pragma unroll
@@ -373,17 +398,19 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         const int pt = threadIdx.x;
         float sc[G::ITEMS2][G::KQ];     // scales of this thread's items, the same for every chunk
         float vf[G::ITEMS2][G::VF];     // fp16 operands: 2^e of the items' residual vectors
+        int chs[G::ITEMS2];             // channel of each item
 #pragma unroll
         for (int i = 0; i < G::ITEMS2; ++i) {
             const int p = pt + i * PR::PROD_THREADS;
-            const int k = k0 + p / (P_KC / 2);
+            chs[i] = CLIP ? p / (P_KC / 2) : pair_channel<KP1>(p / (P_KC / 2), nch);
+            const int k = k0 + chs[i];
             const bool own = !CLIP && p < nch * (P_KC / 2);
 #pragma unroll
             for (int n = 0; n < G::KQ; ++n)
                 sc[i][n] = (own && n < KP1 - 1) ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
 #pragma unroll
             for (int n = 0; n < G::VF; ++n)
-                vf[i][n] = own ? ctl.vscale[(p / (P_KC / 2)) * KP1 + n] : 0.0f;
+                vf[i][n] = own ? ctl.vscale[chs[i] * KP1 + n] : 0.0f;
         }
         const float xs = F16 ? ctl.xscale : 1.0f;
         for (int it = 0; it < total; ++it) {
@@ -395,7 +422,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
             const int ts = F16 ? s >> 1 : s, hh = F16 ? s & 1 : 0;
             pair_consume<KP1, CLIP>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + ts * P_STAGE_BYTES,
-                                    hh, pt, nch, sc, vf, xs, ctl, qmaxf);
+                                    hh, pt, nch, chs, sc, vf, xs, ctl, qmaxf);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
