@@ -586,29 +586,53 @@ __device__ __forceinline__ float max_abs4(float4 v)
     return fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w)));
 }
 
-// Ranges for the fp16 operand scales: blocks [0, xb) fold max|X| into range[0] (float bits of a
-// non-negative value order like unsigned integers; range[0] starts at 0); the other blocks take one
-// channel per warp and write max_j |r_{k,n+1,j}| of every residual vector (the same fp32 recursion
-// of Eq. 7 as the contraction's producers) to range[1 + k (k_max + 1) + n].  d % 4 == 0, rows and
-// code planes 16-byte aligned.
+// Ranges for the fp16 operand scales, folded with atomicMax into a zeroed range[] (float bits of
+// non-negative values order like unsigned integers): blocks [0, xb) take max|X| into range[0], four
+// independent 16-byte loads in flight per thread; the other blocks give each channel `split`
+// warps, each over a 1/split share of the row, for max_j |r_{k,n+1,j}| of every residual vector
+// (the same fp32 recursion of Eq. 7 as the contraction's producers) into
+// range[1 + k (k_max + 1) + n].  d % 4 == 0, rows and code planes 16-byte aligned.
+template <int KP1>
+__device__ __forceinline__ void range_step(float4 r, const int8_t *__restrict__ codes, size_t plane,
+                                           size_t row, int j, const float (&sc)[KP1 > 1 ? KP1 - 1 : 1],
+                                           float (&mx)[KP1])
+{
+    mx[0] = fmaxf(mx[0], max_abs4(r));
+#pragma unroll
+    for (int n = 0; n < KP1 - 1; ++n) {
+        const char4 q = __ldg(reinterpret_cast<const char4 *>(codes + n * plane + row) + j);
+        r.x = __fmaf_rn(-sc[n], (float)q.x, r.x);
+        r.y = __fmaf_rn(-sc[n], (float)q.y, r.y);
+        r.z = __fmaf_rn(-sc[n], (float)q.z, r.z);
+        r.w = __fmaf_rn(-sc[n], (float)q.w, r.w);
+        mx[n + 1] = fmaxf(mx[n + 1], max_abs4(r));
+    }
+}
+
 template <int KP1>
 __global__ void __launch_bounds__(256)
 pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const float *__restrict__ W,
                   const int8_t *__restrict__ codes, const float *__restrict__ scales, int C, int d,
-                  unsigned *__restrict__ range)
+                  int split, unsigned *__restrict__ range)
 {
     constexpr int K = KP1 - 1;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     if ((int)blockIdx.x < xb) {
         float m = 0.0f;
-        for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nx4;
-             i += (long long)xb * blockDim.x)
-            m = fmaxf(m, max_abs4(__ldg(X + i)));
+        const long long stride = (long long)xb * blockDim.x;
+        long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+        for (; i + 3 * stride < nx4; i += 4 * stride) {
+            const float4 a = __ldg(X + i), b = __ldg(X + i + stride);
+            const float4 c = __ldg(X + i + 2 * stride), e = __ldg(X + i + 3 * stride);
+            m = fmaxf(m, fmaxf(fmaxf(max_abs4(a), max_abs4(b)), fmaxf(max_abs4(c), max_abs4(e))));
+        }
+        for (; i < nx4; i += stride) m = fmaxf(m, max_abs4(__ldg(X + i)));
         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
         if (lane == 0) atomicMax(range, __float_as_uint(m));
         return;
     }
-    const int k = ((int)blockIdx.x - xb) * 8 + warp;
+    const int gw = ((int)blockIdx.x - xb) * 8 + warp;
+    const int k = gw / split, part = gw - k * split;
     if (k >= C) return;
     float sc[K > 0 ? K : 1], mx[KP1];
 #pragma unroll
@@ -616,24 +640,20 @@ pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const flo
 #pragma unroll
     for (int n = 0; n < KP1; ++n) mx[n] = 0.0f;
     const float4 *w4 = reinterpret_cast<const float4 *>(W + (size_t)k * d);
-    for (int j = lane; j < d / 4; j += 32) {
-        float4 r = __ldg(w4 + j);
-        mx[0] = fmaxf(mx[0], max_abs4(r));
-#pragma unroll
-        for (int n = 0; n < K; ++n) {
-            const char4 q = __ldg(reinterpret_cast<const char4 *>(codes + ((size_t)n * C + k) * d) + j);
-            r.x = __fmaf_rn(-sc[n], (float)q.x, r.x);
-            r.y = __fmaf_rn(-sc[n], (float)q.y, r.y);
-            r.z = __fmaf_rn(-sc[n], (float)q.z, r.z);
-            r.w = __fmaf_rn(-sc[n], (float)q.w, r.w);
-            mx[n + 1] = fmaxf(mx[n + 1], max_abs4(r));
-        }
+    const size_t plane = (size_t)C * d, row = (size_t)k * d;
+    const int d4 = d / 4, step = 32 * split;
+    int j = part * 32 + lane;
+    for (; j + step < d4; j += 2 * step) {          // two rows' worth of loads in flight
+        const float4 a = __ldg(w4 + j), b = __ldg(w4 + j + step);
+        range_step<KP1>(a, codes, plane, row, j, sc, mx);
+        range_step<KP1>(b, codes, plane, row, j + step, sc, mx);
     }
+    if (j < d4) range_step<KP1>(__ldg(w4 + j), codes, plane, row, j, sc, mx);
 #pragma unroll
     for (int n = 0; n < KP1; ++n) {
         float m = mx[n];
         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-        if (lane == 0) range[1 + (size_t)k * KP1 + n] = __float_as_uint(m);
+        if (lane == 0) atomicMax(range + 1 + (size_t)k * KP1 + n, __float_as_uint(m));
     }
 }
 
@@ -768,11 +788,13 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
                                      (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
         if (st != MPQ_OK) return st;
         const long long nx4 = (long long)N * d / 4;
-        const int xb = (int)std::min<long long>((nx4 + 255) / 256, 2LL * sm_count());
-        e = cudaMemsetAsync(range, 0, sizeof(unsigned), stream);
+        const int xb = (int)std::min<long long>((nx4 + 1023) / 1024, 4LL * sm_count());
+        const int rsplit = std::min(8, std::max(1, (d / 4 + 255) / 256));   // >= 8 loads per lane
+        const long long cb = ((long long)C * rsplit + 7) / 8;
+        e = cudaMemsetAsync(range, 0, (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
         if (e == cudaSuccess) {
-            pair_range_kernel<KP1><<<xb + (C + 7) / 8, 256, 0, stream>>>(
-                reinterpret_cast<const float4 *>(X), nx4, xb, W, codes, scales, C, d, range);
+            pair_range_kernel<KP1><<<(unsigned)(xb + cb), 256, 0, stream>>>(
+                reinterpret_cast<const float4 *>(X), nx4, xb, W, codes, scales, C, d, rsplit, range);
             e = cudaGetLastError();
         }
         if (e == cudaSuccess)
