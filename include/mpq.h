@@ -124,6 +124,29 @@ mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
                             const int8_t *codes, const float *scales, int C, int d, int k_max,
                             float *err, void *stream);
 
+/* Words of mpq_output_error_noalloc's fixed scratch buffer (4 MiB). */
+#define MPQ_NOALLOC_RANGE_WORDS (1 << 20)
+
+/*
+ * mpq_output_error_noalloc -- mpq_output_error that allocates nothing.  The paper has no
+ * counterpart: it is an engineering variant of the Eq. 11 call for callers that must not touch
+ * a memory pool (a caller-managed memory budget, a process that disables stream-ordered pools).
+ *
+ * Same arguments, layouts, validation, results (bit for bit) and errors as mpq_output_error,
+ * except for the scratch: the tensor-core path's range table (1 + C (k_max+1) words) lives in one
+ * fixed device array of MPQ_NOALLOC_RANGE_WORDS words inside the library, allocated when the
+ * library's module is loaded.  Therefore:
+ *  - a call whose table would exceed MPQ_NOALLOC_RANGE_WORDS words is rejected with
+ *    MPQ_ERR_UNSUPPORTED before anything is enqueued;
+ *  - overlapping calls race: every call of this entry point uses the same buffer, so two calls
+ *    whose kernels can run at the same time (on different streams, in different threads, or in
+ *    CUDA graphs replayed concurrently) overwrite each other's ranges and return wrong errors.
+ *    Order them (one stream, or events between streams).  mpq_output_error has no such limit.
+ */
+mpq_status mpq_output_error_noalloc(const float *X, int N, int groups, const float *W,
+                                    const int8_t *codes, const float *scales, int C, int d,
+                                    int k_max, float *err, void *stream);
+
 /*
  * mpq_allocate_points -- per-channel point counts from the output-error table (Sec. 3.3,
  * Algorithm 2).

@@ -20,6 +20,7 @@ MPQ_CENTER_PER_CHANNEL = 0
 MPQ_CENTER_PER_LAYER = 1
 MPQ_CLIP_PER_CHANNEL = 0
 MPQ_CLIP_PER_LAYER = 1
+MPQ_NOALLOC_RANGE_WORDS = 1 << 20     # the fixed scratch of mpq_output_error_noalloc
 
 MPQ_STATUS = {0: "MPQ_OK", 1: "MPQ_ERR_INVALID_ARG", 2: "MPQ_ERR_NONFINITE",
               3: "MPQ_ERR_UNSUPPORTED", 4: "MPQ_ERR_CUDA", 5: "MPQ_ERR_TIMEOUT",
@@ -43,6 +44,7 @@ _L = ctypes.POINTER(PackedLayout)
 SIGNATURES = {
     "mpq_quantize_layer": ([_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P], _I),
     "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "mpq_output_error_noalloc": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
     "mpq_reconstruct": ([_P, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_center_weights": ([_P, _I, _I, _I, _P, _P, _P], _I),
@@ -150,7 +152,8 @@ def mpq_quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, codes=N
     return codes, scales, resid_sq, residuals
 
 
-def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None, stream=None):
+def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None, stream=None,
+                     _entry: str = "mpq_output_error"):
     """Output error (Eq. 11) for n = 0..k_max points: err [C][k_max+1] fp32."""
     _dev(W, "W", torch.float32)
     C, d = W.shape
@@ -168,10 +171,18 @@ def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None,
     err = err if err is not None else torch.empty((C, k_max + 1), dtype=torch.float32,
                                                   device=W.device)
     _dev(err, "err", torch.float32, (C, k_max + 1))
-    st = load().mpq_output_error(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales), C, d,
+    st = getattr(load(), _entry)(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales), C, d,
                                  k_max, _ptr(err), _stream(stream))
-    _check(st, "mpq_output_error")
+    _check(st, _entry)
     return err
+
+
+def mpq_output_error_noalloc(X, W, codes, scales, k_max: int, groups: int = 1, err=None,
+                             stream=None):
+    """mpq_output_error through the entry point that allocates nothing (one fixed scratch buffer
+    inside the library: calls must not overlap)."""
+    return mpq_output_error(X, W, codes, scales, k_max, groups, err, stream,
+                            _entry="mpq_output_error_noalloc")
 
 
 def mpq_clip_search(X, W, bits: int, n_cand: int = 20, mode: int = None, groups: int = 1,

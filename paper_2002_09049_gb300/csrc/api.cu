@@ -115,11 +115,10 @@ extern "C" mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits,
                            resid_sq, residuals, (cudaStream_t)stream);
 }
 
-extern "C" mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
-                                       const int8_t *codes, const float *scales, int C, int d,
-                                       int k_max, float *err, void *stream)
+static mpq_status check_output_error(const float *X, int N, int groups, const float *W,
+                                     const int8_t *codes, const float *scales, int C, int d,
+                                     int k_max, float *err)
 {
-    g_msg[0] = 0;
     mpq_status st = check_common(C, d, k_max);
     if (st != MPQ_OK) return st;
     REQUIRE(N >= 1, MPQ_ERR_INVALID_ARG, "N = %d must be >= 1", N);
@@ -129,8 +128,42 @@ extern "C" mpq_status mpq_output_error(const float *X, int N, int groups, const 
     if (C == 0) return MPQ_OK;
     REQUIRE(X && W && codes && scales && err, MPQ_ERR_INVALID_ARG,
             "X, W, codes, scales and err must be non-NULL");
+    return MPQ_OK;
+}
+
+extern "C" mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
+                                       const int8_t *codes, const float *scales, int C, int d,
+                                       int k_max, float *err, void *stream)
+{
+    g_msg[0] = 0;
+    const mpq_status st = check_output_error(X, N, groups, W, codes, scales, C, d, k_max, err);
+    if (st != MPQ_OK || C == 0) return st;
     return launch_output_error(X, N, groups, W, codes, scales, C, d, k_max, err,
                                (cudaStream_t)stream);
+}
+
+// The fixed scratch of mpq_output_error_noalloc: one array for every call of that entry point
+// (overlapping calls race on it, as its declaration states).
+static __device__ __align__(256) unsigned g_noalloc_range[MPQ_NOALLOC_RANGE_WORDS];
+
+extern "C" mpq_status mpq_output_error_noalloc(const float *X, int N, int groups, const float *W,
+                                               const int8_t *codes, const float *scales, int C,
+                                               int d, int k_max, float *err, void *stream)
+{
+    g_msg[0] = 0;
+    const mpq_status st = check_output_error(X, N, groups, W, codes, scales, C, d, k_max, err);
+    if (st != MPQ_OK || C == 0) return st;
+    const size_t words = output_error_scratch_words(X, groups, W, codes, C, d, k_max);
+    REQUIRE(words <= (size_t)MPQ_NOALLOC_RANGE_WORDS, MPQ_ERR_UNSUPPORTED,
+            "C = %d, k_max = %d need %zu scratch words; the fixed buffer holds %d", C, k_max, words,
+            MPQ_NOALLOC_RANGE_WORDS);
+    unsigned *range = nullptr;
+    if (words > 0) {
+        const cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&range), g_noalloc_range);
+        if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress (fixed scratch)");
+    }
+    return launch_output_error(X, N, groups, W, codes, scales, C, d, k_max, err,
+                               (cudaStream_t)stream, range);
 }
 
 extern "C" mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, int C,

@@ -126,13 +126,20 @@ mpq_status launch_grouped(const float *X, int N, const float *W, const int8_t *c
 
 }  // namespace
 
+size_t output_error_scratch_words(const float *X, int groups, const float *W,
+                                  const int8_t *codes, int C, int d, int k_max)
+{
+    return (groups == 1 && output_error_pair_ok(X, W, codes, d)) ? 1 + (size_t)C * (k_max + 1) : 0;
+}
+
 mpq_status launch_output_error(const float *X, int N, int groups, const float *W,
                                const int8_t *codes, const float *scales, int C, int d, int k_max,
-                               float *err, cudaStream_t stream)
+                               float *err, cudaStream_t stream, unsigned *range)
 {
     if (groups == 1) {
         if (output_error_pair_ok(X, W, codes, d))
-            return launch_output_error_pair(X, N, W, codes, scales, C, d, k_max, err, stream);
+            return launch_output_error_pair(X, N, W, codes, scales, C, d, k_max, err, stream,
+                                            range);
         return launch_output_error_tc(X, N, W, codes, scales, C, d, k_max, err, stream);
     }
     switch (k_max + 1) {

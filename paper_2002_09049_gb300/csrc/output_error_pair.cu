@@ -709,9 +709,11 @@ bool pair_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *ba
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// ext_range: caller-provided range scratch (fp16 operands), or NULL for the stream-ordered pool.
 template <int KP1, bool CLIP>
 mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *codes,
-                       const float *scales, int C, int d, int qmax, float *err, cudaStream_t stream)
+                       const float *scales, int C, int d, int qmax, float *err, cudaStream_t stream,
+                       unsigned *ext_range = nullptr)
 {
     using G = PGeo<KP1, CLIP>;
     const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
@@ -781,12 +783,14 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     }
     attr[0].val.clusterDim.x = (unsigned)(2 * split);
     cfg.gridDim = dim3((unsigned)(n_pairs * 2 * split), 1, 1);
-    unsigned *range = nullptr;
+    unsigned *range = ext_range;
     if constexpr (!CLIP) {
         // fp16 operands: the ranges of X and of every residual vector first
-        mpq_status st = pair_scratch(reinterpret_cast<void **>(&range),
-                                     (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
-        if (st != MPQ_OK) return st;
+        if (!ext_range) {
+            mpq_status st = pair_scratch(reinterpret_cast<void **>(&range),
+                                         (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
+            if (st != MPQ_OK) return st;
+        }
         const long long nx4 = (long long)N * d / 4;
         const int xb = (int)std::min<long long>((nx4 + 1023) / 1024, 4LL * sm_count());
         const int rsplit = std::min(8, std::max(1, (d / 4 + 255) / 256));   // >= 8 loads per lane
@@ -800,8 +804,10 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         if (e == cudaSuccess)
             e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
                                    (const unsigned *)range, err, split, tmX, tmW, tmQ);
-        const cudaError_t ef = cudaFreeAsync(range, stream);
-        if (e == cudaSuccess) e = ef;
+        if (!ext_range) {
+            const cudaError_t ef = cudaFreeAsync(range, stream);
+            if (e == cudaSuccess) e = ef;
+        }
         return cuda_status(e, "pair output-error kernel launch");
     }
     e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
@@ -819,11 +825,11 @@ bool output_error_pair_ok(const float *X, const float *W, const int8_t *codes, i
 
 mpq_status launch_output_error_pair(const float *X, int N, const float *W, const int8_t *codes,
                                     const float *scales, int C, int d, int k_max, float *err,
-                                    cudaStream_t stream)
+                                    cudaStream_t stream, unsigned *range)
 {
     switch (k_max + 1) {
 #define MPQ_CASE(n) \
-    case n: return launch_pair<n, false>(X, N, W, codes, scales, C, d, 0, err, stream);
+    case n: return launch_pair<n, false>(X, N, W, codes, scales, C, d, 0, err, stream, range);
         MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7) MPQ_CASE(8)
         MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14) MPQ_CASE(15)
         MPQ_CASE(16) MPQ_CASE(17)

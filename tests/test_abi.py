@@ -91,6 +91,18 @@ def test_output_error_validation(lib, args, status):
     assert lib.mpq_output_error(*args, None) == status
 
 
+def test_output_error_noalloc_validation(lib):
+    """The fixed-scratch entry point validates like mpq_output_error and rejects, on the host, a
+    range table larger than its buffer (16-byte aligned fake pointers and d % 16 == 0 select the
+    tensor-core path, whose table has 1 + C (k_max+1) words)."""
+    f = lib.mpq_output_error_noalloc
+    assert f(FAKE, 0, 1, FAKE, FAKE, FAKE, 4, 16, 2, FAKE, None) == 1                  # N = 0
+    assert f(None, 8, 1, FAKE, FAKE, FAKE, 4, 16, 2, FAKE, None) == 1                  # X NULL
+    assert f(FAKE, 8, 1, FAKE, FAKE, FAKE, 0, 16, 2, FAKE, None) == 0                  # C = 0
+    C = binding.MPQ_NOALLOC_RANGE_WORDS // 3 + 1                                       # 3C + 1 > words
+    assert f(FAKE, 8, 1, FAKE, FAKE, FAKE, C, 16, 2, FAKE, None) == 3
+
+
 @pytest.mark.parametrize("mode,val,status", [
     (2, 1.0, 1), (0, float("nan"), 2), (0, float("inf"), 2), (0, -0.5, 1), (1, float("nan"), 2),
 ])
