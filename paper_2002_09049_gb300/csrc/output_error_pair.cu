@@ -172,26 +172,32 @@ struct PGeo {
 };
 
 // fp16 operand stores fill 64-byte half rows, and the 128-byte swizzle puts a half row in banks
-// 0-15 or 16-31 by bit 2 of its row.  So that each warp store reaches both bank halves:
-// X item q (16 bytes of raw input) of a warp's 32 items goes to rows {r, r+1, r+4, r+5} of an 8-row
-// atom ...
+// 0-15 or 16-31 by bit 2 of its row.  A store wavefront serves 128 bytes: a half warp's 8-byte
+// stores, or a whole warp's 4-byte stores.  So that each of them reaches both bank halves:
+// X item q (8 bytes per operand half) of a warp's 32 items goes to rows r, r+4 (lanes 0-15) and
+// r+1, r+5 (lanes 16-31) of an 8-row atom ...
 __device__ __forceinline__ int pair_x_item(int q)
 {
     const int g = q >> 5, j = (q & 31) >> 3;
-    const int row = (g >> 1) * 8 + (g & 1) * 2 + (j & 1) + (j >> 1) * 4;
+    const int row = (g >> 1) * 8 + (g & 1) * 2 + (j >> 1) + (j & 1) * 4;
     return row * P_KC4 + (q & 7);
 }
 
-// ... and the two channels of a warp's residual items (slots j = 2t, 2t+1) are D apart, with
-// D (k_max+1) = 4 (mod 8) where possible, so that their rows differ in bit 2.  A bijection of the
-// slots 0..nch-1 (the tail that does not fill a block of 2D slots is kept in place).
+// ... and the two channels of a warp's residual items (slots j = 2t, 2t+1: lanes 0-15 and 16-31)
+// are D apart, with D (k_max+1) = 4 (mod 8) where possible, so that their rows differ in bit 2.
+// A bijection of the slots 0..nch-1: blocks of 2D slots pair channel i with i + D; a last partial
+// block of T slots pairs its first T - D channels so and keeps the rest in place.
 template <int KP1>
 __device__ __forceinline__ int pair_channel(int j, int nch)
 {
     constexpr int D = (KP1 & 1) ? 4 : ((KP1 & 3) == 2 ? 2 : 1);
-    if (j >= nch / (2 * D) * (2 * D)) return j;
-    const int w = j % (2 * D);
-    return j - w + (w >> 1) + (w & 1) * D;
+    const int F = nch / (2 * D) * (2 * D);
+    if (j < F) {
+        const int w = j % (2 * D);
+        return j - w + (w >> 1) + (w & 1) * D;
+    }
+    const int T = nch - F, m = T > D ? T - D : 0, s = j - F;
+    return s < 2 * m ? F + (s >> 1) + (s & 1) * D : F + m + (s - 2 * m);
 }
 
 // Raw slot -> operand stage (tile set `sb`, row half `hh` with fp16 operands): X rows -> B tiles;
