@@ -281,7 +281,10 @@ def run_ours(args, world, rank, local):
             net.run_device(Ws, Xs, stream=stream)
 
     center_launches = {"none": 0, "channel": 1, "layer": 3}[args.center]
-    launches_per_step = (4 + center_launches) * len(layers) * len(wl.bits)
+    # one kernel per call, plus the range pre-pass of every output error on the CTA-pair kernel
+    # (shared calibration input, rows a multiple of 16 elements; torch buffers are 16-byte aligned)
+    range_launches = sum(1 for l in layers if l.groups == 1 and l.d % 16 == 0)
+    launches_per_step = ((4 + center_launches) * len(layers) + range_launches) * len(wl.bits)
 
     for _ in range(args.warmup):
         step()
