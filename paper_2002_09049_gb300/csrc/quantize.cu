@@ -42,6 +42,7 @@ namespace mpq {
 namespace {
 
 constexpr int QTHREADS = 256;                                   // 8 warps per CTA
+constexpr int QDIRECT_MAX_D = 32;                               // direct candidate evaluation up to here
 constexpr int QMAX_LIMIT = (1 << (MPQ_MAX_BITS - 1)) - 1;
 
 template <bool CUSTOM>
@@ -426,6 +427,9 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
 
     const size_t plane = (size_t)C * d;
     const float *w = W + (size_t)k * d;
+    // rows this short take every candidate directly: G*d code evaluations per step cost less than
+    // the lattice's per-step clears, scans and fold over its 2 G Qmax + 1 buckets
+    const bool direct = d <= QDIRECT_MAX_D;
     const float pscale = ldexpf(1.0f, hbits - 62);   // P * 2^-S / 2^e for the fp32 screen
 
     int bad = 0;
@@ -469,17 +473,19 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             const int S = 62 - e - hbits;       // sum_j R_j c_j < 2^62
             const double down = pow2d(-S);
             const float smax_e = ldexpf(smax, -e);   // smax / 2^e for the fp32 screen
-            for (int t = COPIES > 1 ? lane : gt; t <= G; t += COPIES > 1 ? 32 : NT) {
-                hLo[t] = 0u;   // each warp clears its own copy, or the group the shared one
-                hHi[t] = 0u;
-                hN[t] = 0;
-            }
-            if (LAT)
-                for (int t = gt; t < nb; t += NT) {
-                    latR[t] = 0ull;
-                    latC[t] = 0;
+            if (!direct) {
+                for (int t = COPIES > 1 ? lane : gt; t <= G; t += COPIES > 1 ? 32 : NT) {
+                    hLo[t] = 0u;   // each warp clears its own copy, or the group the shared one
+                    hHi[t] = 0u;
+                    hN[t] = 0;
                 }
-            gsync<WPC>(grp);
+                if (LAT)
+                    for (int t = gt; t < nb; t += NT) {
+                        latR[t] = 0ull;
+                        latC[t] = 0;
+                    }
+                gsync<WPC>(grp);
+            }
             const bool zero_scale = __fmul_rn(fg(0), smax) == 0.0f;   // s_g increases with g
 
             double bestD = DBL_MAX;
@@ -542,7 +548,24 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                         add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
                     }
                 };
-                if (LAT) {
+                if (direct) {
+                    // Short rows: every candidate's P_g and N_g straight from the codes, exact
+                    // (the codes as the update emits them; P in the same fixed point), into the
+                    // merged bins the screen reads, with Pbase = Nbase = 0.
+                    for (int g = gt; g < G; g += NT) {
+                        const float sg = __fmul_rn(fg(g), smax), ig = fi(g) * ism;
+                        long long P = 0, N = 0;
+                        for (int j = 0; j < d; ++j) {
+                            const float a = fabsf(sr[j]);
+                            const int c = code_fast(a, sg, ig, qmaxf);
+                            P += fixed_point(a, S) * (long long)c;
+                            N += (long long)c * c;
+                        }
+                        mLo[g + 1] = (unsigned int)P;
+                        mHi[g + 1] = (unsigned int)((unsigned long long)P >> 32);
+                        mN[g + 1] = (int)N;
+                    }
+                } else if (LAT) {
                     // Linear grid: level L is held at g iff u >= (g+1)(L - 1/2), u = aG/smax, i.e.
                     // iff floor(2u) >= (g+1)(2L-1), an integer.  Unless 2u lies within 2^-20
                     // (relative) of an integer, one bucket update records the element for every
@@ -619,7 +642,9 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 };
                 // large grids (G * COPIES bins to merge, or a long lattice): the whole group scans
                 const bool big = (LAT && nb > 2048) || G * COPIES > 1024;
-                if (big) {
+                if (direct) {
+                    // the bins already hold P_g, N_g (group_sum2 above ordered their writes)
+                } else if (big) {
                     group_suffix_scan<WPC>(1, G + 1, bins_load, bins_store, sc, gw, lane, grp);
                     if (LAT) group_suffix_scan<WPC>(0, nb, lat_load, lat_store, sc, gw, lane, grp);
                 } else {
@@ -628,8 +653,8 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     if (LAT && gw == (WPC > 1 ? 1 : 0))
                         group_suffix_scan<1>(0, nb, lat_load, lat_store, sc, 0, lane, grp);
                 }
-                gsync<WPC>(grp);
-                if (LAT) {
+                if (!direct) gsync<WPC>(grp);
+                if (LAT && !direct) {
                     // fold the lattice into the merged bins: bin(g + 1) += sum_L bucket((g+1)(2L-1))
                     for (int g = gt; g < G; g += NT) {
                         long long p = bin64(mLo, mHi, g + 1);

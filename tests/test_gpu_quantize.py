@@ -34,6 +34,27 @@ def test_shapes(gpu, oracle, C, d):
     assert rep["near_ties"] <= max(1, C * 4 // 50)
 
 
+@pytest.mark.parametrize("C,d,bits,G,k_max,dist", [
+    (960, 9, 4, 64, 8, "laplace"),      # the MobileNetV2 set's largest depthwise layer
+    (50, 25, 3, 128, 6, "t"),
+    (20, 32, 8, 256, 4, "normal"),      # the longest direct row, 8-bit codes (Qmax = 127)
+    (30, 16, 2, 1024, 3, "normal"),     # the largest grid, b = 2
+    (40, 1, 4, 7, 16, "normal"),        # one weight per channel, 16 points
+])
+def test_short_rows_direct(gpu, oracle, C, d, bits, G, k_max, dist):
+    """Rows of at most 32 weights evaluate every candidate's P and N directly from the codes
+    instead of through the lattice; the chosen scales, codes and residuals stay the definition's."""
+    W = wlm.random_weights(C, d, 7 * C + d + G, dist)
+    rep = check(oracle, W, bits, G, k_max)
+    assert rep["near_ties"] <= max(1, C * k_max // 50)
+
+
+def test_short_rows_custom_grid(gpu, oracle):
+    W = wlm.random_weights(64, 9, 12, "laplace")
+    gf = np.sort(np.random.default_rng(2).uniform(0.02, 1.0, 33)).astype(np.float32)
+    check(oracle, W, 4, gf.size, 8, grid_frac=gf)
+
+
 def test_max_dim(gpu, oracle):
     """The longest channel the library takes (d = 8192): residual, bins and lattice on chip."""
     W = wlm.random_weights(3, 8192, 81, "normal")
