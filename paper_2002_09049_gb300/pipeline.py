@@ -171,9 +171,11 @@ class NetworkPlan:
         scales, point counts.  Input copies run back to back on one stream: every layer's W
         first, then every layer's X (largest layer first in both).  A layer's greedy search
         starts on its compute stream as soon as its W has landed and only its output error waits
-        for its X, so the greedy searches overlap the calibration inputs' copies.  Its outputs go
-        back on one D2H stream once its kernels are done -- copies in both directions overlap
-        other layers' kernels.  copy_inputs=False reuses the inputs an
+        for its X, so the greedy searches overlap the calibration inputs' copies.  Outputs go
+        back on one D2H stream: codes and scales as soon as the greedy search has made them
+        (overlapping the layer's own output error and allocation), point counts once the
+        allocation is done -- copies in both directions overlap kernels.  copy_inputs=False
+        reuses the inputs an
         earlier call copied in (e.g. a second bit width over the same weights).  The caller
         synchronizes ``stream`` before reading the host outputs."""
         main = stream or torch.cuda.current_stream(self.device)
@@ -192,15 +194,24 @@ class NetworkPlan:
         for n, i in enumerate(self.order):
             st = self.streams[n % len(self.streams)]
             st.wait_event(w_landed[i])
-            self.plans[i].run_device(W_devs[i], X_devs[i], stream=st, x_ready=x_landed[i])
+            p = self.plans[i]
+            h = p.host_buffers()
+
+            def points_out(phase, st=st, p=p, h=h):
+                if phase != 2:            # after the greedy search: codes and scales are final
+                    return
+                made = torch.cuda.Event()
+                made.record(st)
+                self.copy_out.wait_event(made)
+                with torch.cuda.stream(self.copy_out):
+                    h["codes"].copy_(p.codes, non_blocking=True)
+                    h["scales"].copy_(p.scales, non_blocking=True)
+
+            p.run_device(W_devs[i], X_devs[i], stream=st, x_ready=x_landed[i], timing=points_out)
             done = torch.cuda.Event()
             done.record(st)
             self.copy_out.wait_event(done)
-            h = self.plans[i].host_buffers()
-            p = self.plans[i]
             with torch.cuda.stream(self.copy_out):
-                h["codes"].copy_(p.codes, non_blocking=True)
-                h["scales"].copy_(p.scales, non_blocking=True)
                 h["npoints"].copy_(p.npoints, non_blocking=True)
                 h["points_used"].copy_(p.points_used, non_blocking=True)
                 if p.center is not None:
