@@ -91,3 +91,18 @@ def test_operand_scaling_extremes(gpu, oracle, x_exp, w_exp):
     q = oracle.quantize_layer(W, 4, 32, K)
     compare_err(gpu_err(X, W, q["codes"], q["scales"], K),
                 oracle.output_error(X, 1, W, q["codes"], q["scales"], K))
+
+
+def test_nonfinite_on_the_pair_path(gpu, oracle):
+    """Rows a multiple of 16 (scaled fp16 operands): the range pass skips NaN in its maxima, and
+    the NaN still propagates -- a NaN weight into its channel's errors only, a NaN calibration
+    input into every error."""
+    W = wlm.random_weights(40, 64, 5, "normal")
+    W[7, 3] = np.nan
+    q = oracle.quantize_layer(W, 4, 16, 3)
+    X = wlm.random_calibration(300, 64, 6)
+    e = gpu_err(X, W, q["codes"], q["scales"], 3)
+    assert np.all(np.isnan(e[7])) and np.all(np.isfinite(np.delete(e, 7, axis=0)))
+    compare_err(e, oracle.output_error(X, 1, W, q["codes"], q["scales"], 3))
+    X[100, 10] = np.nan
+    assert np.all(np.isnan(gpu_err(X, W, q["codes"], q["scales"], 3)))
