@@ -152,9 +152,7 @@ def mpq_quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, codes=N
     return codes, scales, resid_sq, residuals
 
 
-def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None, stream=None,
-                     _entry: str = "mpq_output_error"):
-    """Output error (Eq. 11) for n = 0..k_max points: err [C][k_max+1] fp32."""
+def _output_error(entry, X, W, codes, scales, k_max, groups, err, stream):
     _dev(W, "W", torch.float32)
     C, d = W.shape
     _dev(X, "X", torch.float32)
@@ -171,18 +169,23 @@ def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None,
     err = err if err is not None else torch.empty((C, k_max + 1), dtype=torch.float32,
                                                   device=W.device)
     _dev(err, "err", torch.float32, (C, k_max + 1))
-    st = getattr(load(), _entry)(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales), C, d,
-                                 k_max, _ptr(err), _stream(stream))
-    _check(st, _entry)
+    st = getattr(load(), entry)(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales), C, d,
+                                k_max, _ptr(err), _stream(stream))
+    _check(st, entry)
     return err
+
+
+def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None, stream=None):
+    """Output error (Eq. 11) for n = 0..k_max points: err [C][k_max+1] fp32."""
+    return _output_error("mpq_output_error", X, W, codes, scales, k_max, groups, err, stream)
 
 
 def mpq_output_error_noalloc(X, W, codes, scales, k_max: int, groups: int = 1, err=None,
                              stream=None):
     """mpq_output_error through the entry point that allocates nothing (one fixed scratch buffer
     inside the library: calls must not overlap)."""
-    return mpq_output_error(X, W, codes, scales, k_max, groups, err, stream,
-                            _entry="mpq_output_error_noalloc")
+    return _output_error("mpq_output_error_noalloc", X, W, codes, scales, k_max, groups, err,
+                         stream)
 
 
 def mpq_clip_search(X, W, bits: int, n_cand: int = 20, mode: int = None, groups: int = 1,
