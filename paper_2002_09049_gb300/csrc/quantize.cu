@@ -298,6 +298,60 @@ __device__ __forceinline__ void group_suffix_scan(int t0, int t1, Load load, Sto
     }
 }
 
+// The same suffix sum by `nw` warps of a group (sw = 0..nw-1, contiguous blocks in warp order),
+// which meet at named barrier `bar_id` (nw * 32 threads) to combine the warp totals in `sc`.
+template <typename Load, typename Store>
+__device__ __forceinline__ void warps_suffix_scan(int t0, int t1, Load load, Store store,
+                                                  Scratch &sc, int nw, int sw, int lane, int bar_id)
+{
+    const int nt = nw * 32, st = sw * 32 + lane;
+    const int n = t1 - t0;
+    const int per = (n + nt - 1) / nt;
+    const int b0 = t0 + min(n, st * per), b1 = t0 + min(n, st * per + per);
+    unsigned long long sp = 0;
+    long long sn = 0;
+    for (int t = b0; t < b1; ++t) {
+        unsigned long long p;
+        long long q;
+        load(t, p, q);
+        sp += p;
+        sn += q;
+    }
+    unsigned long long xp = sp;   // inclusive scan toward lower lanes
+    long long xn = sn;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long yp = __shfl_down_sync(0xffffffffu, xp, o);
+        const long long yn = __shfl_down_sync(0xffffffffu, xn, o);
+        if (lane + o < 32) {
+            xp += yp;
+            xn += yn;
+        }
+    }
+    unsigned long long rp = xp - sp;   // blocks of higher lanes in this warp
+    long long rn = xn - sn;
+    if (nw > 1) {
+        asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(nt) : "memory");
+        if (lane == 0) {
+            sc.sp[sw] = xp;   // warp total
+            sc.sn[sw] = xn;
+        }
+        asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(nt) : "memory");
+        for (int w = sw + 1; w < nw; ++w) {
+            rp += sc.sp[w];
+            rn += sc.sn[w];
+        }
+    }
+    for (int t = b1 - 1; t >= b0; --t) {
+        unsigned long long p;
+        long long q;
+        load(t, p, q);
+        rp += p;
+        rn += q;
+        store(t, rp, rn);
+    }
+}
+
 // |r| as a 64-bit fixed-point integer R = |r| * 2^S, from the fp32 bits.  Exact whenever
 // |r| * 2^S is an integer, i.e. for every element large enough to take a nonzero code; smaller
 // elements are truncated (their P contribution is zero anyway).
@@ -648,10 +702,15 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     group_suffix_scan<WPC>(1, G + 1, bins_load, bins_store, sc, gw, lane, grp);
                     if (LAT) group_suffix_scan<WPC>(0, nb, lat_load, lat_store, sc, gw, lane, grp);
                 } else {
+                    // warp 0 the bins; the lattice warp 0 after them (one warp), else the other
+                    // warps together (named barrier 8 + grp: gsync takes 0 or 1..4)
                     if (gw == 0)
                         group_suffix_scan<1>(1, G + 1, bins_load, bins_store, sc, 0, lane, grp);
-                    if (LAT && gw == (WPC > 1 ? 1 : 0))
+                    if (LAT && WPC == 1)
                         group_suffix_scan<1>(0, nb, lat_load, lat_store, sc, 0, lane, grp);
+                    if (LAT && WPC > 1 && gw >= 1)
+                        warps_suffix_scan(0, nb, lat_load, lat_store, sc, WPC - 1, gw - 1, lane,
+                                          8 + grp);
                 }
                 if (!direct) gsync<WPC>(grp);
                 if (LAT && !direct) {
