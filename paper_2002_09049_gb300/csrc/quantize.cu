@@ -694,23 +694,23 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     latR[t] = p;
                     latC[t] = (Count)q;
                 };
-                // large grids (G * COPIES bins to merge, or a long lattice): the whole group scans
-                const bool big = (LAT && nb > 2048) || G * COPIES > 1024;
+                // with the lattice: warp 0 scans the bins while the other warps scan the lattice
+                // together (named barrier 8 + grp: gsync takes 0 or 1..4), or one warp both;
+                // event-form grids with many bins to merge: the whole group
                 if (direct) {
                     // the bins already hold P_g, N_g (group_sum2 above ordered their writes)
-                } else if (big) {
-                    group_suffix_scan<WPC>(1, G + 1, bins_load, bins_store, sc, gw, lane, grp);
-                    if (LAT) group_suffix_scan<WPC>(0, nb, lat_load, lat_store, sc, gw, lane, grp);
-                } else {
-                    // warp 0 the bins; the lattice warp 0 after them (one warp), else the other
-                    // warps together (named barrier 8 + grp: gsync takes 0 or 1..4)
+                } else if (LAT) {
                     if (gw == 0)
                         group_suffix_scan<1>(1, G + 1, bins_load, bins_store, sc, 0, lane, grp);
-                    if (LAT && WPC == 1)
+                    if (WPC == 1)
                         group_suffix_scan<1>(0, nb, lat_load, lat_store, sc, 0, lane, grp);
-                    if (LAT && WPC > 1 && gw >= 1)
+                    else if (gw >= 1)
                         warps_suffix_scan(0, nb, lat_load, lat_store, sc, WPC - 1, gw - 1, lane,
                                           8 + grp);
+                } else if (G * COPIES > 1024) {
+                    group_suffix_scan<WPC>(1, G + 1, bins_load, bins_store, sc, gw, lane, grp);
+                } else if (gw == 0) {
+                    group_suffix_scan<1>(1, G + 1, bins_load, bins_store, sc, 0, lane, grp);
                 }
                 if (!direct) gsync<WPC>(grp);
                 if (LAT && !direct) {
