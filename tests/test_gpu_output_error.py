@@ -24,6 +24,9 @@ def gpu_err(X, W, codes, scales, k_max, groups=1, dev="cuda:0"):
                                      # split over a cluster, k_max + 1 from 2 to 17
                                      (130, 256, 600, 4), (30, 128, 1000, 1), (9, 32, 300, 16),
                                      (50, 512, 1100, 6), (3, 48, 20, 8),
+                                     # k_max + 1 = 8 and 16: no channel pairing separates the
+                                     # stores' bank halves there (layout unchanged, results too)
+                                     (40, 96, 300, 7), (17, 64, 260, 15),
                                      (3, 8192, 300, 4)])          # the longest rows taken
 def test_shared_input(gpu, oracle, C, d, N, K):
     W = wlm.random_weights(C, d, C + d + N, "normal")
