@@ -72,6 +72,10 @@ def _load():
         lib.mpqo_fixed_coeff.restype = ctypes.c_longlong
         lib.mpqo_multipoint_linear.argtypes = [P, I, P, P, P, P, I, I, I, I, P, I, I]
         lib.mpqo_multipoint_linear.restype = I
+        lib.mpqo_minimal_gap.argtypes = [P, I, P]
+        lib.mpqo_minimal_gap.restype = D
+        lib.mpqo_quantize_channel_adaptive.argtypes = [P, I, I, I, D, L, P, P, P, P, P, P, P, P, P]
+        lib.mpqo_quantize_channel_adaptive.restype = I
         _lib = lib
     return _lib
 
@@ -99,6 +103,47 @@ def candidate_errors(r, bits: int, G: int, grid_frac=None):
     s = np.empty(G, np.float32)
     lib.mpqo_candidate_errors(_p(r), r.size, bits, G, _p(gf), _p(E), _p(s))
     return E, s
+
+
+def minimal_gap(t) -> float:
+    """Definition 1: half the smallest difference between two distinct element magnitudes of t
+    (the pair condition read as |t_i| != |t_j|); inf with fewer than two distinct magnitudes."""
+    lib = _load()
+    t = _c(t, np.float32).ravel()
+    work = np.empty(max(1, t.size), np.float64)
+    return float(lib.mpqo_minimal_gap(_p(t), t.size, _p(work)))
+
+
+ETA = 2.0 ** -10   # the maximal grid step of the paper's experiments (Sec. 5)
+
+
+def quantize_adaptive(W, bits: int, k_max: int, eta: float = ETA, max_candidates: int = 10 ** 7):
+    """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) for every channel of W (C x d):
+    step i searches a = m * gamma, m = 1..floor(2 Qmax ||r_i|| / gamma), gamma = min(Delta_{r_i} /
+    Qmax, eta), as fp32 point scales s = a / Qmax.  A plain enumeration, for small channels: a
+    channel whose grid would exceed ``max_candidates`` raises ValueError.
+
+    Returns a dict with codes [k_max][C][d] int8, scales [C][k_max] fp32, resid_sq [C][k_max+1],
+    gamma [C][k_max] (the a-grid step of each step), ncand [C][k_max], best/second [C][k_max]."""
+    lib = _load()
+    W = _c(W, np.float32)
+    C, d = W.shape
+    out = dict(codes=np.zeros((k_max, C, d), np.int8), scales=np.zeros((C, k_max), np.float32),
+               resid_sq=np.zeros((C, k_max + 1), np.float64),
+               gamma=np.zeros((C, k_max), np.float64), ncand=np.zeros((C, k_max), np.int64),
+               best=np.zeros((C, k_max), np.float64), second=np.zeros((C, k_max), np.float64))
+    codes = np.zeros((k_max, d), np.int8)
+    r = np.empty(d, np.float32)
+    work = np.empty(d, np.float64)
+    for k in range(C):
+        st = lib.mpqo_quantize_channel_adaptive(
+            _p(W[k]), d, bits, k_max, float(eta), int(max_candidates), _p(codes),
+            _p(out["scales"][k]), _p(out["resid_sq"][k]), _p(out["gamma"][k]), _p(out["ncand"][k]),
+            _p(out["best"][k]), _p(out["second"][k]), _p(r), _p(work))
+        if st != 0:
+            raise ValueError(f"channel {k}: the adaptive grid exceeds {max_candidates} candidates")
+        out["codes"][:, k, :] = codes
+    return out
 
 
 def quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, channels=None,

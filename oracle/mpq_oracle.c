@@ -20,7 +20,8 @@
  *  - exact half-way ties of the nearest rounding (Eq. 2) go to the even integer (C nearbyintf);
  *  - r / a is one correctly rounded fp32 division (Eq. 8 writes a division);
  *  - the scale grid is G points s_g = f_g * (max|r| / Qmax), f_g = (g+1)/G in fp32 unless the caller
- *    gives its own increasing fractions in (0, 1] (replaces the adaptive grid of Eq. 10);
+ *    gives its own increasing fractions in (0, 1] (replaces the adaptive grid of Eq. 10, which
+ *    mpqo_quantize_channel_adaptive restates, with its own readings, for small channels);
  *  - the scale search keeps the FIRST (lowest g) minimiser;
  *  - a candidate whose fp32 scale underflows to 0 gives all-zero codes;
  *  - a residual that is exactly zero gives a "null point": scale 0, codes 0, residual unchanged;
@@ -33,6 +34,7 @@
 #include <math.h>
 #include <stdint.h>
 #include <stddef.h>
+#include <stdlib.h>
 
 /* Eq. 1 with b bits: the symmetric integer grid {-Qmax..Qmax}, Qmax = 2^(b-1) - 1. */
 static int qmax_of(int bits) { return (1 << (bits - 1)) - 1; }
@@ -172,6 +174,104 @@ void mpqo_quantize_channel(const float *w, int d, int bits, int G, const float *
             resid_sq[i + 1] = finite ? s2 : NAN;
         }
     }
+}
+
+/* ---- The adaptive grid of Eq. 10 (Definition 1) ---------------------------------------------- */
+
+static int cmp_double(const void *a, const void *b)
+{
+    const double x = *(const double *)a, y = *(const double *)b;
+    return (x > y) - (x < y);
+}
+
+/* Definition 1: the minimal gap of t, half the smallest difference between two of its element
+ * magnitudes.  Reading: the pair condition is |t_i| != |t_j| (as printed, t_i != t_j admits
+ * t_i = -t_j, whose gap would be 0).  Magnitudes sorted in double; INFINITY when t has fewer than
+ * two distinct magnitudes.  work: scratch of d doubles. */
+double mpqo_minimal_gap(const float *t, int d, double *work)
+{
+    for (int j = 0; j < d; ++j) work[j] = fabs((double)t[j]);
+    qsort(work, (size_t)d, sizeof(double), cmp_double);
+    double g = INFINITY;
+    for (int j = 1; j < d; ++j)
+        if (work[j] != work[j - 1]) {
+            const double x = (work[j] - work[j - 1]) / 2.0;
+            if (x < g) g = x;
+        }
+    return g;
+}
+
+/* Algorithm 1 with the grid of Eq. 10 for one channel w, run to k_max points.  Each step i:
+ * Delta = minimal gap of r_i (Definition 1), gamma = min(Delta / Qmax, eta) (gamma = eta when
+ * Delta is infinite), and the search over a in I = [0, 2 Qmax ||r_i||] with step gamma: the
+ * candidates a_m = m * gamma, m = 1..M, M = floor(2 Qmax ||r_i|| / gamma) (a = 0 leaves [r/a]
+ * undefined), each as the fp32 point scale s_m = fl(a_m / Qmax) (s q = a [r/a]_Q, Eq. 1).  The codes,
+ * the error (double, index order), the first minimiser and the update r <- fmaf(-s, q, r) are those
+ * of the fixed grid above.  A zero residual gives a null point (gamma = 0, no candidates).
+ * Writes codes [k_max][d], scales [k_max], resid_sq [k_max+1], gamma [k_max], ncand [k_max],
+ * best/second [k_max] (nullable).  Returns 0, or -1 as soon as a step's grid would exceed max_cand
+ * candidates (the steps before it are written; that step and later ones are not).
+ * r: scratch of d floats; work: scratch of d doubles. */
+int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, double eta,
+                                   long max_cand, int8_t *codes, float *scales, double *resid_sq,
+                                   double *gamma, long *ncand, double *best, double *second,
+                                   float *r, double *work)
+{
+    int qmax = qmax_of(bits);
+    for (int j = 0; j < d; ++j) r[j] = w[j];
+    int finite = all_finite(w, d);
+    double r2 = 0.0;
+    for (int j = 0; j < d; ++j) r2 += (double)r[j] * (double)r[j];
+    resid_sq[0] = finite ? r2 : NAN;
+
+    for (int i = 0; i < k_max; ++i) {
+        int8_t *qi = codes + (long)i * d;
+        double E1 = INFINITY, E2 = INFINITY, g = 0.0;
+        long M = 0;
+        float sbest = 0.0f;
+        if (!finite) {
+            for (int j = 0; j < d; ++j) qi[j] = 0;
+            scales[i] = NAN;
+            g = NAN;
+        } else if (r2 == 0.0) {
+            for (int j = 0; j < d; ++j) qi[j] = 0;   /* null point */
+            scales[i] = 0.0f;
+            E1 = E2 = 0.0;
+        } else {
+            const double delta = mpqo_minimal_gap(r, d, work);
+            g = delta / (double)qmax;
+            if (!(g < eta)) g = eta;
+            const double top = 2.0 * (double)qmax * sqrt(r2);
+            const double mf = floor(top / g);
+            if (mf > (double)max_cand) return -1;
+            M = (long)mf;
+            for (long m = 1; m <= M; ++m) {
+                const float sm = (float)(((double)m * g) / (double)qmax);
+                const double E = candidate_error(r, d, sm, qmax);
+                if (E < E1) {
+                    E2 = E1;
+                    E1 = E;
+                    sbest = sm;
+                } else if (E < E2) {
+                    E2 = E;
+                }
+            }
+            for (int j = 0; j < d; ++j) {
+                int q = nearest_code(r[j], sbest, qmax);
+                qi[j] = (int8_t)q;
+                r[j] = fmaf(-sbest, (float)q, r[j]);
+            }
+            scales[i] = sbest;
+        }
+        gamma[i] = g;
+        ncand[i] = M;
+        if (best) best[i] = E1;
+        if (second) second[i] = E2;
+        r2 = 0.0;
+        for (int j = 0; j < d; ++j) r2 += (double)r[j] * (double)r[j];
+        resid_sq[i + 1] = finite ? r2 : NAN;
+    }
+    return 0;
 }
 
 /* Algorithm 1 for channels [c0, c1) of a C x d layer (row-major W).  Output layouts match the

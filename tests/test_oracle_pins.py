@@ -601,3 +601,113 @@ def test_integer_inference_with_center_exact(oracle):
                     int(np.dot(codes[i, k].astype(np.int64), X[t].astype(np.int64)))
                     for i in range(npts[k]))
                 assert Y[k, t] == (v.numerator // v.denominator)
+
+
+# --- The adaptive grid of Eq. 10 (Definition 1) -------------------------------------------------
+
+def _gap_pairs(t):
+    """Definition 1 by its pairs: half the smallest ||t_i| - |t_j|| over pairs of distinct
+    magnitudes (the |t_i| != |t_j| reading), inf if there is no such pair."""
+    a = np.abs(np.asarray(t, np.float64))
+    best = np.inf
+    for i in range(a.size):
+        for j in range(a.size):
+            if a[i] != a[j]:
+                best = min(best, abs(a[i] - a[j]) / 2.0)
+    return best
+
+
+def test_adaptive_grid_hand_example(oracle):
+    """Definition 1 and Eq. 10 on examples worked by hand (tests/golden)."""
+    ex = json.load(open(os.path.join(GOLDEN, "adaptive_grid_hand_example.json")))
+    for case in ex["minimal_gap"]:
+        want = np.inf if case["delta"] == "inf" else case["delta"]
+        assert oracle.minimal_gap(np.asarray(case["t"], np.float32)) == want
+    g = ex["greedy"]
+    out = oracle.quantize_adaptive(np.asarray([g["w"]], np.float32), g["bits"], g["k_max"], g["eta"])
+    np.testing.assert_array_equal(out["scales"][0], np.asarray(g["scales"], np.float32))
+    np.testing.assert_array_equal(out["codes"][:, 0, :], np.asarray(g["codes"], np.int8))
+    np.testing.assert_array_equal(out["resid_sq"][0], np.asarray(g["resid_sq"]))
+    np.testing.assert_array_equal(out["gamma"][0], np.asarray(g["gamma"]))
+    np.testing.assert_array_equal(out["ncand"][0], np.asarray(g["ncand"]))
+
+
+def test_minimal_gap_against_pairs(oracle):
+    """The oracle's sorted-magnitude minimal gap equals Definition 1 evaluated pair by pair, on
+    vectors with repeated magnitudes, sign flips and zeros."""
+    rng = np.random.default_rng(17)
+    for trial in range(200):
+        d = int(rng.integers(1, 12))
+        t = np.round(rng.standard_normal(d) * 8) / 8          # repeats are common
+        t[rng.random(d) < 0.3] *= -1
+        t = t.astype(np.float32)
+        assert oracle.minimal_gap(t) == _gap_pairs(t)
+
+
+def _piecewise_grid_minimum(r, bits, eta):
+    """The smallest objective of Eq. 9 over the grid of Eq. 10, found without enumerating the grid:
+    between consecutive code-change points s = |r_j| / (L - 1/2) the codes are constant and the
+    objective is the quadratic ||r||^2 - 2 s P + s^2 N, so only the grid points nearest its
+    minimiser (and the interval ends) can win.  Those few points are evaluated by the definition.
+    Also returns the continuous minimum over all s > 0 (a lower bound for any grid)."""
+    qmax = (1 << (bits - 1)) - 1
+    r = np.asarray(r, np.float32)
+    a = np.abs(r.astype(np.float64))
+    delta = _gap_pairs(r)
+    gamma = eta if not np.isfinite(delta) else min(delta / qmax, eta)
+    R2 = float(np.sum(r.astype(np.float64) ** 2))
+    M = int(np.floor(2 * qmax * np.sqrt(R2) / gamma))
+
+    def scale(m):
+        return np.float32((m * gamma) / qmax)
+
+    def objective(s):
+        q = np.clip(np.rint(r / np.float32(s)), -qmax, qmax)
+        return float(np.sum((r.astype(np.float64) - np.float64(s) * q) ** 2))
+
+    cuts = sorted({float(x) / (L - 0.5) for x in a[a > 0] for L in range(1, qmax + 1)})
+    edges = [0.0] + cuts + [np.inf]
+    best, cont = np.inf, np.inf
+    for lo, hi in zip(edges[:-1], edges[1:]):
+        inside = (lo + hi) / 2 if np.isfinite(hi) else 2 * lo + 1
+        c = np.minimum(qmax, np.rint(a / inside))
+        N, P = float(np.sum(c * c)), float(np.sum(a * c))
+        target = P / N if N > 0 else inside
+        cont = min(cont, R2 - 2 * min(max(target, lo), hi if np.isfinite(hi) else target) * P +
+                   min(max(target, lo), hi if np.isfinite(hi) else target) ** 2 * N)
+        m_lo = max(1, int(np.floor(lo * qmax / gamma)))
+        m_hi = M if not np.isfinite(hi) else min(M, int(np.ceil(hi * qmax / gamma)))
+        if m_lo > m_hi:
+            continue
+        m_t = min(max(int(round(target * qmax / gamma)), m_lo), m_hi)
+        for m in {m_lo, m_lo + 1, m_t - 1, m_t, m_t + 1, m_hi - 1, m_hi}:
+            if 1 <= m <= M:
+                best = min(best, objective(scale(m)))
+    return best, cont
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_adaptive_step_against_piecewise_search(oracle, bits):
+    """The first greedy step over the grid of Eq. 10 reaches the smallest grid objective, found by
+    the piecewise-quadratic analysis above instead of enumeration, and never beats the continuous
+    optimum over all scales."""
+    rng = np.random.default_rng(100 + bits)
+    for trial in range(40):
+        d = int(rng.integers(1, 7))
+        w = (rng.standard_normal(d) * rng.choice([0.05, 1.0, 20.0])).astype(np.float32)
+        out = oracle.quantize_adaptive(w[None, :], bits, 1, max_candidates=10 ** 8)
+        grid_best, cont = _piecewise_grid_minimum(w, bits, oracle.ETA)
+        assert out["best"][0, 0] == pytest.approx(grid_best, rel=1e-12, abs=1e-300)
+        assert out["best"][0, 0] >= cont * (1 - 1e-9) - 1e-30
+
+
+def test_adaptive_grid_decay_theorem1(oracle):
+    """Theorem 1 under the grid of Eq. 10 (b = 2, eta = 2^-10): the residual energy never grows and
+    falls by orders of magnitude within a few points, down to the eta floor."""
+    W = wlm.random_weights(6, 12, 23, "normal")
+    out = oracle.quantize_adaptive(W, 2, 8, max_candidates=10 ** 8)
+    rs = out["resid_sq"]
+    assert np.all(rs[:, 1:] <= rs[:, :-1])
+    prev, nxt = rs[:, :-1], rs[:, 1:]
+    assert np.all(nxt[prev > 0] < 0.5 * prev[prev > 0])   # a fixed fraction removed per point
+    assert np.all(rs[:, 6] < 5e-4 * rs[:, 0])
