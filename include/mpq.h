@@ -118,8 +118,8 @@ mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
  * device's default stream-ordered memory pool with cudaMallocAsync on `stream` and returns them
  * with cudaFreeAsync on `stream` -- concurrent calls on other streams each get their own, and a
  * CUDA graph capture records them as the graph's allocation nodes.  MPQ_ERR_NOMEM if that
- * allocation fails (nothing else is enqueued then).  The first such call in a process raises
- * that pool's release threshold (cudaMemPoolAttrReleaseThreshold) to keep freed blocks cached in
+ * allocation fails (nothing else is enqueued then).  The first such call in a process made
+ * outside a stream capture raises that pool's release threshold (cudaMemPoolAttrReleaseThreshold) to keep freed blocks cached in
  * the pool instead of returning them to the driver at every synchronization; a process that
  * manages the default pool itself can call mpq_output_error_noalloc instead.
  */

@@ -666,11 +666,17 @@ pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const flo
 // Scratch of the fp16 contraction comes from the device's stream-ordered pool (allocated and
 // freed on the call's stream, so concurrent calls on other streams never share it; inside a CUDA
 // graph capture these become the graph's own allocation nodes).  Freed blocks stay cached in the
-// pool instead of going back to the driver at every synchronisation.
+// pool instead of going back to the driver at every synchronisation (set on the first call made
+// outside a stream capture, where a pool attribute may not be changed).
 mpq_status pair_scratch(void **p, size_t bytes, cudaStream_t stream)
 {
     static std::atomic<int> pool_set{0};
-    if (!pool_set.exchange(1)) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusActive;
+    if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) {
+        (void)cudaGetLastError();
+        cs = cudaStreamCaptureStatusActive;
+    }
+    if (cs == cudaStreamCaptureStatusNone && !pool_set.exchange(1)) {
         int dev = 0;
         cudaMemPool_t pool;
         if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetDefaultMemPool(&pool, dev) == cudaSuccess) {
