@@ -66,7 +66,7 @@ def parse():
                     help="comma-separated layer indices to run (profiling a subset); default all")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
-    ap.add_argument("--op", default="quantize", choices=["quantize", "clip", "infer"],
+    ap.add_argument("--op", default="quantize", choices=["quantize", "clip", "infer", "adaptive"],
                     help="quantize: the multipoint path (Algorithm 1, Eq. 11, Algorithm 2, Eq. 4); "
                          "clip: the output-error-driven clipping factor search (Eq. 12); "
                          "infer: integer inference with the packed multipoint weights (Eq. 13)")
@@ -997,6 +997,223 @@ def run_infer(args, world, rank, local):
     return out if rank == 0 else None
 
 
+FP64_NOMINAL_TFLOPS = 1.25   # the part's nominal dense FP64 rate (no measured FP64 peak exists)
+ADAPTIVE_CAP = 10 ** 7       # most candidates one adaptive-grid step may enumerate (a larger
+                             # step is refused; refused steps are counted in the config)
+ADAPTIVE_ORACLE_CAP = 10 ** 6   # the oracle sample's cap: bounds its time; it counts what it ran
+ADAPTIVE_METRIC = "weight-elements x adaptive-grid candidates x points / s"
+
+
+def adaptive_layers(wl):
+    from paper_2002_09049_gb300 import binding
+    idx = [li for li, l in enumerate(wl.layers) if l.d <= binding.MPQ_ADAPTIVE_MAX_DIM]
+    if not idx:
+        raise SystemExit("--op adaptive needs layers of at most 64 weights per channel "
+                         "(e.g. --config c4, the depthwise 3x3 convolutions)")
+    return idx
+
+
+def adaptive_oracle_step(wl, idx, per_layer, threads):
+    """The oracle's adaptive grid (Eq. 10) on the first `per_layer` channels of every short layer,
+    steps above ADAPTIVE_ORACLE_CAP candidates refused (not enumerated, not counted); returns the
+    element-candidate units it processed."""
+    import oracle
+    from concurrent.futures import ThreadPoolExecutor
+    jobs = [(li, c) for li in idx for c in range(min(per_layer, wl.layers[li].C))]
+    Ws = {li: layer_inputs(wl, li)[0] for li in idx}
+
+    def one(job):
+        li, c = job
+        o = oracle.quantize_adaptive(Ws[li][c:c + 1], wl.bits[0], wl.k_max,
+                                     max_candidates=ADAPTIVE_ORACLE_CAP, refuse="mark")
+        return int(np.maximum(o["ncand"], 0).sum()) * wl.layers[li].d
+
+    with ThreadPoolExecutor(max_workers=threads) as ex:
+        return sum(ex.map(one, jobs))
+
+
+def run_adaptive(args, world, rank, local):
+    """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) on every short layer of the
+    workload (c4: the 17 depthwise layers, 9 weights per channel): mpq_quantize_layer_adaptive per
+    layer on a pool of streams; value = element-candidate evaluations (d x grid size, summed over
+    channels and points) per second."""
+    import torch
+    from paper_2002_09049_gb300 import _build, binding
+    from paper_2002_09049_gb300 import dist as dist_helpers
+    from paper_2002_09049_gb300 import workloads as wlm
+
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0 or world == 1:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    binding.load()
+    wl = wlm.WORKLOADS[args.config]
+    idx = adaptive_layers(wl)
+    layers = [wl.layers[li] for li in idx]
+    bits, k_max = wl.bits[0], wl.k_max
+    Whs = [torch.from_numpy(layer_inputs(wl, li)[0]).pin_memory() for li in idx]
+    Ws = [w.to(dev) for w in Whs]
+    mk = lambda dt, shape: torch.empty(shape, dtype=dt, device=dev)
+    outs = [(mk(torch.int8, (k_max, l.C, l.d)), mk(torch.float32, (l.C, k_max)),
+             mk(torch.float32, (l.C, k_max + 1)), mk(torch.int64, (l.C, k_max))) for l in layers]
+    hosts = [(torch.empty(o[0].shape, dtype=torch.int8, pin_memory=True),
+              torch.empty(o[1].shape, dtype=torch.float32, pin_memory=True)) for o in outs]
+    order = sorted(range(len(layers)), key=lambda i: -layers[i].C)
+    streams = [torch.cuda.Stream(dev) for _ in range(max(1, args.streams))]
+    main = torch.cuda.current_stream()
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+
+    def call(i, st):
+        c, s_, r, n = outs[i]
+        binding.mpq_quantize_layer_adaptive(Ws[i], bits, k_max, max_cand=ADAPTIVE_CAP, codes=c,
+                                            scales=s_, resid_sq=r, ncand=n, stream=st)
+
+    def step(host=False):
+        ev = torch.cuda.Event()
+        ev.record(main)
+        for st in streams:
+            st.wait_event(ev)
+        for n, i in enumerate(order):
+            st = streams[n % len(streams)]
+            if host:
+                with torch.cuda.stream(st):
+                    Ws[i].copy_(Whs[i], non_blocking=True)
+            call(i, st)
+            if host:
+                with torch.cuda.stream(st):
+                    hosts[i][0].copy_(outs[i][0], non_blocking=True)
+                    hosts[i][1].copy_(outs[i][1], non_blocking=True)
+        for st in streams:
+            e = torch.cuda.Event()
+            e.record(st)
+            main.wait_event(e)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    ncand = [int(o[3].sum().item()) for o in outs]
+    refused = sum(int((o[3] < 0).sum().item()) for o in outs)
+    units_per_step = sum(max(0, n) * l.d for n, l in zip(ncand, layers))
+    step_ms = []
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            a = torch.cuda.Event(enable_timing=True)
+            z = torch.cuda.Event(enable_timing=True)
+            a.record(main)
+            step()
+            z.record(main)
+            torch.cuda.synchronize()
+            step_ms.append(a.elapsed_time(z))
+    one_ms = []
+    for _ in range(args.steps):
+        flush.fill_(1.0)
+        a = torch.cuda.Event(enable_timing=True)
+        z = torch.cuda.Event(enable_timing=True)
+        a.record(main)
+        for i in order:
+            call(i, main)
+        z.record(main)
+        torch.cuda.synchronize()
+        one_ms.append(a.elapsed_time(z))
+    if world > 1:
+        torch.distributed.barrier()
+    ms = dist_helpers.max_over_ranks(float(np.mean(step_ms)), device=dev)
+    value = dist_helpers.aggregate_throughput(units_per_step, ms, world)
+    t1 = float(np.mean(one_ms)) / 1e3
+    ach = 4.0 * units_per_step / t1 / 1e12
+    roofline = {"kernel": "adaptive_kernel (Algorithm 1 over the grid of Eq. 10, objective in "
+                          "double)", "bound": "alu", "achieved": ach, "peak": FP64_NOMINAL_TFLOPS,
+                "unit": "TFLOP/s (fp64)", "frac": ach / FP64_NOMINAL_TFLOPS, "traffic": None,
+                "peak_source": "nominal dense FP64 rate of the part (no measured FP64 peak)",
+                "timing": "every layer on one stream, CUDA events; achieved = 4 fp64 operations "
+                          "(multiply, subtract, square, add) per element and candidate / that time",
+                "single_stream_ms_per_step": t1 * 1e3}
+    out = {"metric": ADAPTIVE_METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic",
+           "config": {"workload": f"{args.config}: {wl.title}, layers of <= 64 weights per channel",
+                      "op": "adaptive grid (Def. 1 + Eq. 10)", "layers": len(layers),
+                      "channels": sum(l.C for l in layers), "bits": bits, "k_max": k_max,
+                      "eta": 2.0 ** -10, "max_cand": ADAPTIVE_CAP, "refused_steps": refused,
+                      "units_per_step": units_per_step,
+                      "l2": "flushed between steps (512 MB write)", "streams": args.streams,
+                      "parallelism": f"replicas x{world}"},
+           "roofline": roofline, "gpu_launches": len(layers) * args.steps,
+           "clocks": clk.summary()}
+    if not args.no_e2e:
+        step(host=True)
+        torch.cuda.synchronize()
+        times = []
+        for _ in range(args.steps):
+            a = torch.cuda.Event(enable_timing=True)
+            z = torch.cuda.Event(enable_timing=True)
+            a.record(main)
+            step(host=True)
+            z.record(main)
+            z.synchronize()
+            times.append(a.elapsed_time(z))
+        e_ms = float(np.mean(times))
+        out["e2e"] = {"value": units_per_step / (e_ms / 1e3), "unit": UNIT, "ms_per_step": e_ms,
+                      "h2d_bytes_per_step": int(sum(w.numel() * 4 for w in Whs)),
+                      "d2h_bytes_per_step": int(sum(h[0].numel() + 4 * h[1].numel()
+                                                    for h in hosts))}
+    if not args.no_cpu_baseline and rank == 0:
+        import oracle
+        oracle.build()
+        per_layer = 2
+        t0 = time.perf_counter()
+        units = adaptive_oracle_step(wl, idx, per_layer, host_cores())
+        dt = time.perf_counter() - t0
+        out["cpu_baseline"] = {"value": units / dt, "unit": UNIT, "cores": host_cores(),
+                               "kind": "oracle", "seconds": dt,
+                               "sample": f"the first {per_layer} channels of every short layer "
+                                         f"(steps above {ADAPTIVE_ORACLE_CAP} candidates refused), "
+                                         "oracle threads over channels"}
+    return out
+
+
+def run_adaptive_reference(args, world, rank):
+    """The oracle's adaptive grid as the reference arm of --op adaptive, on the host cores."""
+    if rank != 0:
+        return None
+    import oracle
+    from paper_2002_09049_gb300 import workloads as wlm
+    oracle.build()
+    wl = wlm.WORKLOADS[args.config]
+    idx = adaptive_layers(wl)
+    per_layer = 2
+    for _ in range(args.warmup):
+        adaptive_oracle_step(wl, idx, 1, host_cores())
+    times, units = [], 0
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        units = adaptive_oracle_step(wl, idx, per_layer, host_cores())
+        times.append(time.perf_counter() - t0)
+    v = units / float(np.mean(times))
+    return {"impl": "reference", "metric": ADAPTIVE_METRIC, "value": v, "unit": UNIT, "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(times)),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": f"{args.config}: {wl.title}, layers of <= 64 weights per channel",
+                       "op": "adaptive grid (Def. 1 + Eq. 10)", "bits": wl.bits[0],
+                       "k_max": wl.k_max},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+                             "sample": f"the first {per_layer} channels of every short layer per "
+                                       f"step (steps above {ADAPTIVE_ORACLE_CAP} candidates "
+                                       "refused)"},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
 def run_clip_reference(args, world, rank):
     """The oracle's Eq. 12 search as the reference arm of --op clip, on the host cores."""
     if rank != 0:
@@ -1040,11 +1257,14 @@ def main():
                    "unavailable": "the integer inference path needs the device-quantized layers; "
                                   "its oracle is timed as cpu_baseline of --op infer"}
         else:
-            out = (run_clip_reference if args.op == "clip" else run_reference)(args, world, rank)
+            out = {"clip": run_clip_reference,
+                   "adaptive": run_adaptive_reference}.get(args.op, run_reference)(args, world, rank)
     elif args.op == "clip":
         out = run_clip(args, world, rank, local)
     elif args.op == "infer":
         out = run_infer(args, world, rank, local)
+    elif args.op == "adaptive":
+        out = run_adaptive(args, world, rank, local)
     else:
         out = run_ours(args, world, rank, local)
     if out is not None:

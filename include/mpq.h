@@ -127,6 +127,36 @@ mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
                             const int8_t *codes, const float *scales, int C, int d, int k_max,
                             float *err, void *stream);
 
+/* Longest channel of mpq_quantize_layer_adaptive. */
+#define MPQ_ADAPTIVE_MAX_DIM 64
+
+/*
+ * mpq_quantize_layer_adaptive -- Algorithm 1 with the adaptive grid of Eq. 10 (Sec. 3.2,
+ * Definition 1) instead of a fixed grid, for short channels (e.g. depthwise 3x3 filters).
+ * Step i of channel k, with r = r_{k,i} (r_1 = w_k):
+ *   Delta = the minimal gap of r (Definition 1): half the smallest difference between two distinct
+ *     element magnitudes |r_j| (the printed pair condition t_i != t_j read as |t_i| != |t_j|);
+ *   gamma = min(Delta / Qmax, eta), or eta when r has fewer than two distinct magnitudes;
+ *   grid search of a over I = [0, 2 Qmax ||r||] with step gamma (Eq. 10): a_m = m gamma for
+ *     m = 1..M, M = floor(2 Qmax ||r|| / gamma) (double), as fp32 point scales s_m = fl(a_m / Qmax);
+ *   codes, objective (double, index order), first minimiser and update as mpq_quantize_layer.
+ * A zero residual gives a null point (scale 0, codes 0); so does a grid without candidates.
+ *
+ *   W          [C][d] fp32; 1 <= d <= MPQ_ADAPTIVE_MAX_DIM.
+ *   bits, k_max, codes, scales, resid_sq   as for mpq_quantize_layer (resid_sq nullable).
+ *   eta        the largest grid step (the paper's experiments: 2^-10); finite, > 0.
+ *   max_cand   the most candidates one step may enumerate (>= 1).  A step whose grid is larger
+ *              is refused on the device: its scale and every later scale of that channel read NaN,
+ *              their codes 0, and ncand holds -1 for it (0 for the later steps).
+ *   ncand      out [C][k_max] int64, nullable: M of every step (0 for a null point).
+ * Each step enumerates its whole grid (d M code evaluations); the grid grows as the minimal gap
+ * shrinks, so long channels (hundreds of weights) are out of reach: MPQ_ERR_UNSUPPORTED.
+ */
+mpq_status mpq_quantize_layer_adaptive(const float *W, int C, int d, int bits, int k_max,
+                                       double eta, long long max_cand, int8_t *codes,
+                                       float *scales, float *resid_sq, long long *ncand,
+                                       void *stream);
+
 /* Words of mpq_output_error_noalloc's fixed scratch buffer (4 MiB). */
 #define MPQ_NOALLOC_RANGE_WORDS (1 << 20)
 

@@ -117,11 +117,13 @@ def minimal_gap(t) -> float:
 ETA = 2.0 ** -10   # the maximal grid step of the paper's experiments (Sec. 5)
 
 
-def quantize_adaptive(W, bits: int, k_max: int, eta: float = ETA, max_candidates: int = 10 ** 7):
+def quantize_adaptive(W, bits: int, k_max: int, eta: float = ETA, max_candidates: int = 10 ** 7,
+                      refuse: str = "raise"):
     """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) for every channel of W (C x d):
     step i searches a = m * gamma, m = 1..floor(2 Qmax ||r_i|| / gamma), gamma = min(Delta_{r_i} /
-    Qmax, eta), as fp32 point scales s = a / Qmax.  A plain enumeration, for small channels: a
-    channel whose grid would exceed ``max_candidates`` raises ValueError.
+    Qmax, eta), as fp32 point scales s = a / Qmax.  A plain enumeration, for small channels: a step
+    whose grid would exceed ``max_candidates`` is refused -- ValueError, or with refuse="mark" its
+    scale and the later ones NaN, codes 0, ncand -1 for it and 0 after.
 
     Returns a dict with codes [k_max][C][d] int8, scales [C][k_max] fp32, resid_sq [C][k_max+1],
     gamma [C][k_max] (the a-grid step of each step), ncand [C][k_max], best/second [C][k_max]."""
@@ -140,7 +142,7 @@ def quantize_adaptive(W, bits: int, k_max: int, eta: float = ETA, max_candidates
             _p(W[k]), d, bits, k_max, float(eta), int(max_candidates), _p(codes),
             _p(out["scales"][k]), _p(out["resid_sq"][k]), _p(out["gamma"][k]), _p(out["ncand"][k]),
             _p(out["best"][k]), _p(out["second"][k]), _p(r), _p(work))
-        if st != 0:
+        if st != 0 and refuse == "raise":
             raise ValueError(f"channel {k}: the adaptive grid exceeds {max_candidates} candidates")
         out["codes"][:, k, :] = codes
     return out

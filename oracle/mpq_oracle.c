@@ -209,9 +209,9 @@ double mpqo_minimal_gap(const float *t, int d, double *work)
  * the error (double, index order), the first minimiser and the update r <- fmaf(-s, q, r) are those
  * of the fixed grid above.  A zero residual gives a null point (gamma = 0, no candidates).
  * Writes codes [k_max][d], scales [k_max], resid_sq [k_max+1], gamma [k_max], ncand [k_max],
- * best/second [k_max] (nullable).  Returns 0, or -1 as soon as a step's grid would exceed max_cand
- * candidates (the steps before it are written; that step and later ones are not).
- * r: scratch of d floats; work: scratch of d doubles. */
+ * best/second [k_max] (nullable).  A step whose grid would exceed max_cand candidates is refused:
+ * its scale and every later one NaN, codes 0, squared norms NaN, ncand -1 for it and 0 after;
+ * returns -1 then, else 0.  r: scratch of d floats; work: scratch of d doubles. */
 int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, double eta,
                                    long max_cand, int8_t *codes, float *scales, double *resid_sq,
                                    double *gamma, long *ncand, double *best, double *second,
@@ -224,12 +224,13 @@ int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, d
     for (int j = 0; j < d; ++j) r2 += (double)r[j] * (double)r[j];
     resid_sq[0] = finite ? r2 : NAN;
 
+    int refused = 0;
     for (int i = 0; i < k_max; ++i) {
         int8_t *qi = codes + (long)i * d;
         double E1 = INFINITY, E2 = INFINITY, g = 0.0;
         long M = 0;
         float sbest = 0.0f;
-        if (!finite) {
+        if (!finite || refused) {
             for (int j = 0; j < d; ++j) qi[j] = 0;
             scales[i] = NAN;
             g = NAN;
@@ -243,7 +244,17 @@ int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, d
             if (!(g < eta)) g = eta;
             const double top = 2.0 * (double)qmax * sqrt(r2);
             const double mf = floor(top / g);
-            if (mf > (double)max_cand) return -1;
+            if (mf > (double)max_cand) {
+                refused = 1;
+                for (int j = 0; j < d; ++j) qi[j] = 0;
+                scales[i] = NAN;
+                gamma[i] = g;
+                ncand[i] = -1;
+                if (best) best[i] = NAN;
+                if (second) second[i] = NAN;
+                resid_sq[i + 1] = NAN;
+                continue;
+            }
             M = (long)mf;
             for (long m = 1; m <= M; ++m) {
                 const float sm = (float)(((double)m * g) / (double)qmax);
@@ -269,9 +280,9 @@ int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, d
         if (second) second[i] = E2;
         r2 = 0.0;
         for (int j = 0; j < d; ++j) r2 += (double)r[j] * (double)r[j];
-        resid_sq[i + 1] = finite ? r2 : NAN;
+        resid_sq[i + 1] = (finite && !refused) ? r2 : NAN;
     }
-    return 0;
+    return refused ? -1 : 0;
 }
 
 /* Algorithm 1 for channels [c0, c1) of a C x d layer (row-major W).  Output layouts match the

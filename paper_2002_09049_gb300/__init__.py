@@ -10,5 +10,6 @@ from .binding import (MPQ_ALLOC_BUDGET, MPQ_ALLOC_THRESHOLD, MPQ_CENTER_PER_CHAN
                       MPQ_CENTER_PER_LAYER, MPQ_CLIP_PER_CHANNEL, MPQ_CLIP_PER_LAYER, MPQError,
                       PackedLayout, mpq_allocate_points, mpq_center_weights, mpq_clip_search,
                       mpq_multipoint_linear, mpq_output_error, mpq_output_error_noalloc,
-                      mpq_pack_layout, mpq_pack_points, mpq_quantize_layer, mpq_reconstruct,
+                      mpq_pack_layout, mpq_pack_points, mpq_quantize_layer,
+                      mpq_quantize_layer_adaptive, mpq_reconstruct,
                       mpq_status_string, mpq_version)

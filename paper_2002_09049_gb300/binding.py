@@ -21,6 +21,7 @@ MPQ_CENTER_PER_LAYER = 1
 MPQ_CLIP_PER_CHANNEL = 0
 MPQ_CLIP_PER_LAYER = 1
 MPQ_NOALLOC_RANGE_WORDS = 1 << 20     # the fixed scratch of mpq_output_error_noalloc
+MPQ_ADAPTIVE_MAX_DIM = 64             # the longest channel of mpq_quantize_layer_adaptive
 
 MPQ_STATUS = {0: "MPQ_OK", 1: "MPQ_ERR_INVALID_ARG", 2: "MPQ_ERR_NONFINITE",
               3: "MPQ_ERR_UNSUPPORTED", 4: "MPQ_ERR_CUDA", 5: "MPQ_ERR_TIMEOUT",
@@ -43,6 +44,8 @@ _L = ctypes.POINTER(PackedLayout)
 
 SIGNATURES = {
     "mpq_quantize_layer": ([_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P], _I),
+    "mpq_quantize_layer_adaptive": ([_P, _I, _I, _I, _I, _D, ctypes.c_longlong, _P, _P, _P, _P,
+                                     _P], _I),
     "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_output_error_noalloc": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
@@ -150,6 +153,35 @@ def mpq_quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, codes=N
                                    _ptr(resid_sq), _ptr(residuals), _stream(stream))
     _check(st, "mpq_quantize_layer")
     return codes, scales, resid_sq, residuals
+
+
+ETA = 2.0 ** -10   # the largest grid step of the paper's experiments
+
+
+def mpq_quantize_layer_adaptive(W, bits: int, k_max: int, eta: float = ETA,
+                                max_cand: int = 10 ** 7, codes=None, scales=None, resid_sq=None,
+                                ncand=None, stream=None):
+    """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) for short channels
+    (d <= MPQ_ADAPTIVE_MAX_DIM).  Returns (codes [k_max][C][d] int8, scales [C][k_max] fp32,
+    resid_sq [C][k_max+1] fp32, ncand [C][k_max] int64: each step's grid size, -1 if refused)."""
+    _dev(W, "W", torch.float32)
+    C, d = W.shape
+    dev = W.device
+    codes = codes if codes is not None else torch.empty((k_max, C, d), dtype=torch.int8, device=dev)
+    scales = scales if scales is not None else torch.empty((C, k_max), dtype=torch.float32,
+                                                           device=dev)
+    resid_sq = resid_sq if resid_sq is not None else torch.empty((C, k_max + 1),
+                                                                 dtype=torch.float32, device=dev)
+    ncand = ncand if ncand is not None else torch.empty((C, k_max), dtype=torch.int64, device=dev)
+    _dev(codes, "codes", torch.int8, (k_max, C, d))
+    _dev(scales, "scales", torch.float32, (C, k_max))
+    _dev(resid_sq, "resid_sq", torch.float32, (C, k_max + 1))
+    _dev(ncand, "ncand", torch.int64, (C, k_max))
+    st = load().mpq_quantize_layer_adaptive(_ptr(W), C, d, bits, k_max, float(eta), int(max_cand),
+                                            _ptr(codes), _ptr(scales), _ptr(resid_sq),
+                                            _ptr(ncand), _stream(stream))
+    _check(st, "mpq_quantize_layer_adaptive")
+    return codes, scales, resid_sq, ncand
 
 
 def _output_error(entry, X, W, codes, scales, k_max, groups, err, stream):

@@ -87,6 +87,10 @@ mpq_status launch_allocate_threshold(const float *err, int C, int k_max, double 
 mpq_status launch_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
                               const float *center, int C, int d, int k_max, float *W_hat,
                               cudaStream_t stream);
+mpq_status launch_adaptive(const float *W, int C, int d, int qmax, int k_max, double eta,
+                           long long max_cand, int8_t *codes, float *scales, float *resid_sq,
+                           long long *ncand, cudaStream_t stream);
+
 mpq_status launch_center(const float *W, int C, int d, int mode, float *center, float *Wc,
                          cudaStream_t stream);
 

@@ -103,6 +103,19 @@ def test_output_error_noalloc_validation(lib):
     assert f(FAKE, 8, 1, FAKE, FAKE, FAKE, C, 16, 2, FAKE, None) == 3
 
 
+@pytest.mark.parametrize("d,bits,eta,cap,status", [
+    (65, 4, 2.0 ** -10, 100, 3),          # longer than MPQ_ADAPTIVE_MAX_DIM
+    (9, 9, 2.0 ** -10, 100, 3),           # bits above the limit
+    (9, 1, 2.0 ** -10, 100, 1),
+    (9, 4, 0.0, 100, 1),                  # eta must be > 0
+    (9, 4, float("nan"), 100, 2),
+    (9, 4, 2.0 ** -10, 0, 1),             # max_cand >= 1
+])
+def test_quantize_adaptive_validation(lib, d, bits, eta, cap, status):
+    assert lib.mpq_quantize_layer_adaptive(FAKE, 4, d, bits, 3, eta, cap, FAKE, FAKE, None, None,
+                                           None) == status
+
+
 @pytest.mark.parametrize("mode,val,status", [
     (2, 1.0, 1), (0, float("nan"), 2), (0, float("inf"), 2), (0, -0.5, 1), (1, float("nan"), 2),
 ])
