@@ -711,3 +711,18 @@ def test_adaptive_grid_decay_theorem1(oracle):
     prev, nxt = rs[:, :-1], rs[:, 1:]
     assert np.all(nxt[prev > 0] < 0.5 * prev[prev > 0])   # a fixed fraction removed per point
     assert np.all(rs[:, 6] < 5e-4 * rs[:, 0])
+
+
+def test_adaptive_refusal_marking(oracle):
+    """A step whose grid exceeds the cap is refused: ValueError by default; with refuse="mark" its
+    scale and the later ones NaN, codes 0, ncand -1 then 0, while the steps before it are kept."""
+    w = np.asarray([[1.0, 0.5]], np.float32)             # grids of 2289 and 724 candidates
+    with pytest.raises(ValueError):
+        oracle.quantize_adaptive(w, 2, 3, max_candidates=1000)
+    o = oracle.quantize_adaptive(w, 2, 3, max_candidates=1000, refuse="mark")
+    np.testing.assert_array_equal(o["ncand"][0], [-1, 0, 0])
+    assert np.all(np.isnan(o["scales"][0])) and np.all(o["codes"] == 0)
+    assert o["resid_sq"][0, 0] == 1.25 and np.all(np.isnan(o["resid_sq"][0, 1:]))
+    o = oracle.quantize_adaptive(w, 2, 3, max_candidates=2289, refuse="mark")
+    np.testing.assert_array_equal(o["ncand"][0], [2289, 724, 0])
+    np.testing.assert_array_equal(o["scales"][0], np.asarray([0.75, 0.25, 0.0], np.float32))
