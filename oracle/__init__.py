@@ -74,7 +74,7 @@ def _load():
         lib.mpqo_multipoint_linear.restype = I
         lib.mpqo_minimal_gap.argtypes = [P, I, P]
         lib.mpqo_minimal_gap.restype = D
-        lib.mpqo_quantize_channel_adaptive.argtypes = [P, I, I, I, D, L, P, P, P, P, P, P, P, P, P]
+        lib.mpqo_quantize_channel_adaptive.argtypes = [P, I, I, I, D, L, P, P, P, P, P, P, P, P, P, I]
         lib.mpqo_quantize_channel_adaptive.restype = I
         _lib = lib
     return _lib
@@ -118,12 +118,15 @@ ETA = 2.0 ** -10   # the maximal grid step of the paper's experiments (Sec. 5)
 
 
 def quantize_adaptive(W, bits: int, k_max: int, eta: float = ETA, max_candidates: int = 10 ** 7,
-                      refuse: str = "raise"):
+                      refuse: str = "raise", piecewise: bool = False):
     """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) for every channel of W (C x d):
     step i searches a = m * gamma, m = 1..floor(2 Qmax ||r_i|| / gamma), gamma = min(Delta_{r_i} /
     Qmax, eta), as fp32 point scales s = a / Qmax.  A plain enumeration, for small channels: a step
     whose grid would exceed ``max_candidates`` is refused -- ValueError, or with refuse="mark" its
-    scale and the later ones NaN, codes 0, ncand -1 for it and 0 after.
+    scale and the later ones NaN, codes 0, ncand -1 for it and 0 after.  piecewise=True takes the
+    same decisions without enumerating the grid (code-change points by binary search, the
+    objective's quadratic form to bound where its minimum can be, the definition to settle it),
+    for grids too large to enumerate; ``second`` is NaN then.
 
     Returns a dict with codes [k_max][C][d] int8, scales [C][k_max] fp32, resid_sq [C][k_max+1],
     gamma [C][k_max] (the a-grid step of each step), ncand [C][k_max], best/second [C][k_max]."""
@@ -141,7 +144,9 @@ def quantize_adaptive(W, bits: int, k_max: int, eta: float = ETA, max_candidates
         st = lib.mpqo_quantize_channel_adaptive(
             _p(W[k]), d, bits, k_max, float(eta), int(max_candidates), _p(codes),
             _p(out["scales"][k]), _p(out["resid_sq"][k]), _p(out["gamma"][k]), _p(out["ncand"][k]),
-            _p(out["best"][k]), _p(out["second"][k]), _p(r), _p(work))
+            _p(out["best"][k]), _p(out["second"][k]), _p(r), _p(work), int(bool(piecewise)))
+        if st < -1:
+            raise RuntimeError(f"channel {k}: the piecewise search failed ({st})")
         if st != 0 and refuse == "raise":
             raise ValueError(f"channel {k}: the adaptive grid exceeds {max_candidates} candidates")
         out["codes"][:, k, :] = codes

@@ -201,6 +201,175 @@ double mpqo_minimal_gap(const float *t, int d, double *work)
     return g;
 }
 
+/* ---- The same grid search without enumerating the grid (long channels) ---------------------- */
+
+static float adaptive_scale(long m, double gamma, int qmax)
+{
+    return (float)(((double)m * gamma) / (double)qmax);
+}
+
+/* Code magnitude of |r| = a at scale s, as nearest_code computes it (the rounding is symmetric). */
+static int code_mag_at(float a, float s, int qmax)
+{
+    if (s == 0.0f) return 0;
+    float t = nearbyintf(a / s);
+    if (t > (float)qmax) t = (float)qmax;
+    return (int)t;
+}
+
+struct ad_event {
+    long m;      /* first grid index with the code below L */
+    int j, L;
+};
+
+struct ad_piece {
+    long ma, mb;     /* grid indices with the same codes */
+    double P, N;     /* sum a_j c_j and sum c_j^2 there */
+};
+
+static int cmp_event(const void *x, const void *y)
+{
+    const struct ad_event *a = (const struct ad_event *)x, *b = (const struct ad_event *)y;
+    return (a->m > b->m) - (a->m < b->m);
+}
+
+/* first m in [lo, hi] with s_m >= target (hi + 1 if none) */
+static long first_scale_at_least(long lo, long hi, double target, double gamma, int qmax)
+{
+    long a = lo, b = hi + 1;
+    while (a < b) {
+        const long mid = a + (b - a) / 2;
+        if ((double)adaptive_scale(mid, gamma, qmax) >= target) b = mid; else a = mid + 1;
+    }
+    return a;
+}
+
+/* The quadratic form of the objective and a bound on its distance from the definition's sum
+ * (d double roundings of terms no larger than R2 + 2 s P + s^2 N, d <= 8192 < 2^13). */
+static double quad(double R2, double P, double N, double s) { return R2 - 2.0 * s * P + s * s * N; }
+static double quad_tol(double R2, double P, double N, double s)
+{
+    return 0x1p-36 * (R2 + 2.0 * s * P + s * s * N);
+}
+
+/* One step of the grid search of Eq. 10 taking the same decision as the enumeration (the first m
+ * with the smallest objective), without enumerating the grid:
+ *  - each element's code magnitude is a non-increasing step function of m (s_m and the correctly
+ *    rounded division are monotone): its change points come from binary searches, and between
+ *    them (pieces) the codes are constant and the objective is, up to rounding, the convex
+ *    quadratic R2 - 2 s P + s^2 N of the fp32 scale s_m, smallest next to s = P / N;
+ *  - pass 1 bounds the smallest objective from above with the grid points around each piece's
+ *    minimiser; pass 2 evaluates by the definition, in m order, every grid point whose quadratic
+ *    lower bound reaches that bound (the first of each run of equal scales).
+ * ev: scratch of d Qmax events; pc: scratch of d Qmax + 1 pieces; c: scratch of d ints.
+ * Returns the chosen m (0 when M = 0) and its objective in *E; -1 if more than max_eval points
+ * would need the definition (never seen; a guard). */
+static long adaptive_step_piecewise(const float *r, int d, int qmax, double gamma, long M,
+                                    long max_eval, struct ad_event *ev, struct ad_piece *pc,
+                                    int *c, double *E)
+{
+    *E = INFINITY;
+    if (M <= 0) return 0;
+    double R2 = 0.0;
+    for (int j = 0; j < d; ++j) R2 += (double)r[j] * (double)r[j];
+    long ne = 0;
+    double P = 0.0, N = 0.0;
+    const float s1 = adaptive_scale(1, gamma, qmax);
+    for (int j = 0; j < d; ++j) {
+        const float a = fabsf(r[j]);
+        c[j] = code_mag_at(a, s1, qmax);
+        P += (double)a * (double)c[j];
+        N += (double)c[j] * (double)c[j];
+        for (int L = c[j]; L >= 1; --L) {
+            long lo = 2, hi = M + 1;         /* first m in [2, M] with code < L, or M + 1 */
+            while (lo < hi) {
+                const long mid = lo + (hi - lo) / 2;
+                if (code_mag_at(a, adaptive_scale(mid, gamma, qmax), qmax) < L) hi = mid;
+                else lo = mid + 1;
+            }
+            if (lo <= M) {
+                ev[ne].m = lo;
+                ev[ne].j = j;
+                ev[ne].L = L;
+                ++ne;
+            }
+        }
+    }
+    qsort(ev, (size_t)ne, sizeof(struct ad_event), cmp_event);
+    /* pass 1: the pieces, and an upper bound of the smallest objective */
+    long np = 0, e = 0, ma = 1;
+    double upper = INFINITY;
+    while (ma <= M) {
+        const long mb = (e < ne) ? ev[e].m - 1 : M;
+        if (mb >= ma) {
+            pc[np].ma = ma;
+            pc[np].mb = mb;
+            pc[np].P = P;
+            pc[np].N = N;
+            ++np;
+            long pick[3];
+            int k = 0;
+            pick[k++] = ma;
+            if (N > 0.0) {
+                const long g = first_scale_at_least(ma, mb, P / N, gamma, qmax);
+                if (g <= mb) pick[k++] = g;
+                if (g - 1 >= ma) pick[k++] = g - 1;
+            }
+            for (int t = 0; t < k; ++t) {
+                const double sd = (double)adaptive_scale(pick[t], gamma, qmax);
+                const double u = quad(R2, P, N, sd) + quad_tol(R2, P, N, sd);
+                if (u < upper) upper = u;
+            }
+        }
+        const long next = mb + 1;
+        while (e < ne && ev[e].m == next) {
+            P -= (double)fabsf(r[ev[e].j]);
+            N -= (double)(2 * ev[e].L - 1);
+            ++e;
+        }
+        ma = next;
+    }
+    /* pass 2: every grid point whose objective may reach the smallest, by the definition */
+    long bestm = 0, evals = 0;
+    double bestE = INFINITY;
+    for (long t = 0; t < np; ++t) {
+        const struct ad_piece *q = &pc[t];
+        long lo = q->ma, hi = q->mb;
+        if (q->N > 0.0) {
+            /* N (s - P/N)^2 + R2 - P^2/N - tol <= upper, tol taken at the piece's largest scale */
+            const double smax = (double)adaptive_scale(q->mb, gamma, qmax);
+            const double tol = quad_tol(R2, q->P, q->N, smax);
+            const double floor_q = R2 - q->P * q->P / q->N;
+            const double room = (upper + 2.0 * tol - floor_q) / q->N;
+            if (room < 0.0) continue;
+            const double half = sqrt(room) * (1.0 + 0x1p-30) + 0x1p-60;
+            const double tgt = q->P / q->N;
+            lo = first_scale_at_least(q->ma, q->mb, tgt - half, gamma, qmax);
+            hi = first_scale_at_least(q->ma, q->mb, tgt + half, gamma, qmax);   /* exclusive */
+            if (hi <= q->mb) ++hi;   /* the first scale past the window too */
+            hi -= 1;
+            if (lo > hi) continue;
+        } else {
+            if (R2 - quad_tol(R2, 0.0, 0.0, 0.0) > upper) continue;
+            hi = lo;              /* constant objective: the first index only */
+        }
+        float prev = -1.0f;
+        for (long m = lo; m <= hi; ++m) {
+            const float sm = adaptive_scale(m, gamma, qmax);
+            if (sm == prev) continue;      /* same scale, same objective: the earlier m wins */
+            prev = sm;
+            if (++evals > max_eval) return -1;
+            const double Em = candidate_error(r, d, sm, qmax);
+            if (Em < bestE || (Em == bestE && m < bestm)) {
+                bestE = Em;
+                bestm = m;
+            }
+        }
+    }
+    *E = bestE;
+    return bestm;
+}
+
 /* Algorithm 1 with the grid of Eq. 10 for one channel w, run to k_max points.  Each step i:
  * Delta = minimal gap of r_i (Definition 1), gamma = min(Delta / Qmax, eta) (gamma = eta when
  * Delta is infinite), and the search over a in I = [0, 2 Qmax ||r_i||] with step gamma: the
@@ -211,13 +380,30 @@ double mpqo_minimal_gap(const float *t, int d, double *work)
  * Writes codes [k_max][d], scales [k_max], resid_sq [k_max+1], gamma [k_max], ncand [k_max],
  * best/second [k_max] (nullable).  A step whose grid would exceed max_cand candidates is refused:
  * its scale and every later one NaN, codes 0, squared norms NaN, ncand -1 for it and 0 after;
- * returns -1 then, else 0.  r: scratch of d floats; work: scratch of d doubles. */
+ * returns -1 then, else 0.  piecewise = 0 enumerates every grid point; 1 takes the same decisions
+ * through adaptive_step_piecewise (best holds the chosen objective, second is NaN), for grids too
+ * large to enumerate (-2 if its guard trips).  r: scratch of d floats; work: scratch of d doubles. */
 int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, double eta,
                                    long max_cand, int8_t *codes, float *scales, double *resid_sq,
                                    double *gamma, long *ncand, double *best, double *second,
-                                   float *r, double *work)
+                                   float *r, double *work, int piecewise)
 {
     int qmax = qmax_of(bits);
+    struct ad_event *ev = NULL;
+    struct ad_piece *pc = NULL;
+    int *cw = NULL;
+    if (piecewise) {
+        ev = (struct ad_event *)malloc(sizeof(struct ad_event) * ((size_t)d * qmax + 1));
+        pc = (struct ad_piece *)malloc(sizeof(struct ad_piece) * ((size_t)d * qmax + 1));
+        cw = (int *)malloc(sizeof(int) * (size_t)d);
+        if (!ev || !pc || !cw) {
+            free(ev);
+            free(pc);
+            free(cw);
+            return -3;
+        }
+    }
+    int status = 0;
     for (int j = 0; j < d; ++j) r[j] = w[j];
     int finite = all_finite(w, d);
     double r2 = 0.0;
@@ -256,15 +442,28 @@ int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, d
                 continue;
             }
             M = (long)mf;
-            for (long m = 1; m <= M; ++m) {
-                const float sm = (float)(((double)m * g) / (double)qmax);
-                const double E = candidate_error(r, d, sm, qmax);
-                if (E < E1) {
-                    E2 = E1;
-                    E1 = E;
-                    sbest = sm;
-                } else if (E < E2) {
-                    E2 = E;
+            if (piecewise) {
+                double Ebest;
+                const long mb = adaptive_step_piecewise(r, d, qmax, g, M, 100000000L, ev, pc, cw,
+                                                        &Ebest);
+                if (mb < 0) {
+                    status = -2;
+                    break;
+                }
+                sbest = mb > 0 ? adaptive_scale(mb, g, qmax) : 0.0f;
+                E1 = Ebest;
+                E2 = NAN;
+            } else {
+                for (long m = 1; m <= M; ++m) {
+                    const float sm = adaptive_scale(m, g, qmax);
+                    const double E = candidate_error(r, d, sm, qmax);
+                    if (E < E1) {
+                        E2 = E1;
+                        E1 = E;
+                        sbest = sm;
+                    } else if (E < E2) {
+                        E2 = E;
+                    }
                 }
             }
             for (int j = 0; j < d; ++j) {
@@ -282,6 +481,10 @@ int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, d
         for (int j = 0; j < d; ++j) r2 += (double)r[j] * (double)r[j];
         resid_sq[i + 1] = (finite && !refused) ? r2 : NAN;
     }
+    free(ev);
+    free(pc);
+    free(cw);
+    if (status) return status;
     return refused ? -1 : 0;
 }
 

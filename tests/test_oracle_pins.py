@@ -726,3 +726,30 @@ def test_adaptive_refusal_marking(oracle):
     o = oracle.quantize_adaptive(w, 2, 3, max_candidates=2289, refuse="mark")
     np.testing.assert_array_equal(o["ncand"][0], [2289, 724, 0])
     np.testing.assert_array_equal(o["scales"][0], np.asarray([0.75, 0.25, 0.0], np.float32))
+
+
+def test_adaptive_piecewise_equals_enumeration(oracle):
+    """The piecewise search of the grid of Eq. 10 (code-change points by binary search, the
+    objective's quadratic form to bound where its minimum can be, the definition to settle it)
+    takes every decision of the enumeration: random short channels of every kind, and grids fine
+    enough that neighbouring points share an fp32 scale."""
+    rng = np.random.default_rng(31)
+    cases = []
+    for _ in range(150):
+        d = int(rng.integers(1, 10))
+        w = [rng.standard_normal(d), np.round(rng.standard_normal(d) * 4) / 4,
+             rng.standard_normal(d) * 1e-6, rng.laplace(size=d) * 30][int(rng.integers(0, 4))]
+        cases.append((w, int(rng.choice([2, 3, 4, 6, 8])), float(rng.choice([2.0 ** -10, 1e-3, 1.0])),
+                      int(rng.integers(1, 4))))
+    for _ in range(3):                                   # scales repeat near the top of the grid
+        cases.append((rng.standard_normal(2) * 0.6, 2, 2.0 ** -24, 1))
+    for w, bits, eta, k_max in cases:
+        w = np.asarray(w, np.float32)[None, :]
+        a = oracle.quantize_adaptive(w, bits, k_max, eta, max_candidates=6 * 10 ** 7, refuse="mark")
+        b = oracle.quantize_adaptive(w, bits, k_max, eta, max_candidates=6 * 10 ** 7, refuse="mark",
+                                     piecewise=True)
+        np.testing.assert_array_equal(a["codes"], b["codes"])
+        np.testing.assert_array_equal(a["scales"], b["scales"])
+        np.testing.assert_array_equal(a["resid_sq"], b["resid_sq"])
+        np.testing.assert_array_equal(a["ncand"], b["ncand"])
+        np.testing.assert_array_equal(a["best"], b["best"])
