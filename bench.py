@@ -54,7 +54,8 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--config", default="c2", choices=["c1", "c2", "c3", "c4", "c5"])
+    ap.add_argument("--config", default="c5", choices=["c1", "c2", "c3", "c4", "c5"],
+                    help="workload; c5 (the two large linear layers) is the largest")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -207,6 +208,19 @@ def contraction_flops(wl, layer):
     return 2 * wl.n_calib * layer.d * layer.C * (wl.k_max + 1)
 
 
+def output_error_bytes(wl, layer):
+    """Algorithmic HBM bytes of one mpq_output_error call: read X, W, the k_max code planes and the
+    scales once, write the error table."""
+    x = layer.C * wl.n_calib * layer.d if layer.groups > 1 else wl.n_calib * layer.d
+    return 4 * x + layer.C * (layer.d * (4 + wl.k_max) + 4 * wl.k_max + 4 * (wl.k_max + 1))
+
+
+def allocate_bytes(wl, layer):
+    """Algorithmic HBM bytes of one mpq_allocate_points call: read the error table, write the
+    point counts."""
+    return 4 * layer.C * (wl.k_max + 1) + 4 * layer.C + 4
+
+
 def run_ours(args, world, rank, local):
     import torch
     from paper_2002_09049_gb300 import _build, binding, pipeline, workloads as wlm
@@ -330,7 +344,8 @@ def run_ours(args, world, rank, local):
 
     # per-kernel-family device time from the events around every call (on its own stream)
     fam_ms = {f: 0.0 for f in families}
-    fam_work = {f: 0.0 for f in families}
+    fam_work = {f: 0.0 for f in families}     # flops (output error), lane-ops (quantize), bytes
+    fam_bytes = {f: 0.0 for f in families}    # algorithmic HBM bytes of every family
     for rec in recs:
         for evs in rec:
             for i, e in evs.items():
@@ -340,22 +355,40 @@ def run_ours(args, world, rank, local):
                 fam_work["output_error"] += contraction_flops(wl, layer)
                 fam_work["quantize"] += quantize_ops(wl, layer, wl.bits[0])
                 fam_work["reconstruct"] += reconstruct_bytes(wl, layer)
-                fam_work["allocate"] += 4 * layer.C * (wl.k_max + 1) * 9 + 8 * layer.C
+                fam_work["allocate"] += allocate_bytes(wl, layer)
                 fam_work["center"] += 8 * layer.C * layer.d + 4 * layer.C
+                fam_bytes["output_error"] += output_error_bytes(wl, layer)
+                fam_bytes["quantize"] += quantize_bytes(wl, layer)
+                fam_bytes["reconstruct"] += reconstruct_bytes(wl, layer)
+                fam_bytes["allocate"] += allocate_bytes(wl, layer)
+                fam_bytes["center"] += 8 * layer.C * layer.d + 4 * layer.C
     if args.center == "none":   # no centring call: its (empty) interval is not a kernel family
         families = [f for f in families if f != "center"]
-        fam_ms.pop("center")
-        fam_work.pop("center")
+        for t in (fam_ms, fam_work, fam_bytes):
+            t.pop("center")
     total_fam = sum(fam_ms.values())
     dominant = max(fam_ms, key=fam_ms.get)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
 
     roofline = dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args,
-                                 sm_count=torch.cuda.get_device_properties(dev).multi_processor_count)
+                                 sm_count=sms)
     roofline["share"] = fam_ms[dominant] / total_fam if total_fam else None
     roofline["family_ms_per_step"] = {f: fam_ms[f] / args.steps for f in families}
     roofline["timing"] = ("CUDA events around every call in a single-stream pass of the same "
                           "steps inside bench.py (value itself is timed with layers on "
                           f"{args.streams} streams)")
+    # every family against HBM (algorithmic bytes / its single-stream time), the greedy search
+    # also against its ALU lane rate, the contraction against the tensor peak
+    hbm = peaks["hbm_gbs"]
+    fam_hbm = {}
+    for f in families:
+        t_s = fam_ms[f] / 1e3
+        ach = fam_bytes[f] / t_s / 1e9 if t_s > 0 else None
+        fam_hbm[f] = {"achieved": ach, "frac": ach / hbm if ach else None,
+                      "bytes_per_step": fam_bytes[f] / args.steps,
+                      "ms_per_step": fam_ms[f] / args.steps}
+    roofline_greedy = greedy_roofline(fam_ms, fam_work, fam_bytes, peaks, peak_src, wl, args, sms)
+    step_bytes = sum(fam_bytes.values()) / args.steps
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -369,6 +402,12 @@ def run_ours(args, world, rank, local):
                    "streams": args.streams, "cuda_graph": bool(args.graph),
                    "center": args.center, "parallelism": f"replicas x{world}"},
         "roofline": roofline,
+        "roofline_greedy": roofline_greedy,
+        "hbm": {"achieved": step_bytes / (ms / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
+                "frac": step_bytes / (ms / 1e3) / 1e9 / hbm, "bytes_per_step": step_bytes,
+                "what": "algorithmic HBM bytes of the whole step (every call reads its inputs and "
+                        "writes its outputs once) / ms_per_step",
+                "families": fam_hbm},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
     }
@@ -376,7 +415,11 @@ def run_ours(args, world, rank, local):
     if not args.no_e2e:
         out["e2e"] = run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds, CENTER_MODES[args.center])
+        gpu_out = gpu_sample_outputs(net, specs, Ws, Xs, wl, stream, oracle_sample(
+            wl, args.cpu_seconds))
+        out["cpu_baseline"], orc_out = cpu_baseline(wl, args.cpu_seconds,
+                                                    CENTER_MODES[args.center])
+        out["parity"] = parity_report(wl, gpu_out, orc_out, CENTER_MODES[args.center])
     if world > 1:
         torch.distributed.barrier()
         torch.distributed.destroy_process_group()
@@ -431,6 +474,38 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_
     return {"kernel": names.get(dominant, dominant), "bound": "hbm", "achieved": ach, "peak": hbm,
             "unit": "GB/s", "frac": ach / hbm, "traffic": traffic,
             "peak_source": f"{peak_src} HBM copy"}
+
+
+def greedy_roofline(fam_ms, fam_work, fam_bytes, peaks, peak_src, wl, args, sm_count):
+    """The greedy search (mpq_quantize_layer) against HBM: algorithmic bytes (read W once, write
+    the k_max code planes, the scales and the residual norms) / its single-stream time, with its
+    lane-operation rate against the ALU peak beside it (the kernel is bound by instruction issue,
+    not by HBM)."""
+    hbm = peaks["hbm_gbs"]
+    t_s = fam_ms["quantize"] / 1e3
+    ach = fam_bytes["quantize"] / t_s / 1e9
+    traffic = None
+    tfile = os.path.join(PROFILES, "roofline_traffic.json")
+    if os.path.exists(tfile):
+        with open(tfile) as f:
+            ent = json.load(f).get(args.config, {}).get("quantize")
+        if ent and ent.get("source_sha") == src_hash(KERNEL_SOURCES["quantize"]):
+            traffic = ent.get("dram_bytes_per_launch")
+    mhz = peaks.get("sm_max_mhz", 2070.0)
+    alu_peak = sm_count * ALU_LANES_PER_SM * mhz * 1e6 / 1e12
+    alu = fam_work["quantize"] / t_s / 1e12
+    n_launch = len(wl.layers) * len(wl.bits)
+    return {"kernel": "quantize_kernel (Eq. 7-9, lattice form, all k_max steps in one launch)",
+            "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+            "traffic": traffic, "peak_source": f"{peak_src} HBM copy",
+            "bytes_per_launch": fam_bytes["quantize"] / args.steps / n_launch,
+            "ms_per_step": fam_ms["quantize"] / args.steps,
+            "alu": {"achieved": alu, "peak": alu_peak, "unit": "Tlane-op/s",
+                    "frac": alu / alu_peak,
+                    "peak_source": f"{sm_count} SMs x {ALU_LANES_PER_SM} lanes x {mhz:.0f} MHz; "
+                                   f"{GREEDY_OPS_PER_ELEMENT_STEP} algorithmic lane operations "
+                                   "per element-step + the per channel-step scan, fold and "
+                                   "screen"}}
 
 
 def run_e2e(net, specs, Whs, Xhs, Ws, Xs, wl, args, stream, units_per_step):
@@ -495,10 +570,11 @@ def oracle_sample(wl, target_s):
     return stride
 
 
-def run_oracle_step(wl, stride, threads, inputs, center=-1):
+def run_oracle_step(wl, stride, threads, inputs, center=-1, collect=None):
     """The oracle over the sampled channels of every layer: centring (asymmetric sets), Algorithm
     1, Eq. 11, Algorithm 2 (budget, per layer, on the sample), Eq. 4.  Returns the metric units
-    processed."""
+    processed; with a dict ``collect``, also keeps each (bits, layer)'s codes, scales, error table
+    and near-tie record there."""
     import oracle
     units = 0
     for b in wl.bits:
@@ -514,6 +590,9 @@ def run_oracle_step(wl, stride, threads, inputs, center=-1):
             n, _ = oracle.allocate_budget(err.astype(np.float32), wl.k_max, wl.beta)
             oracle.reconstruct(q["codes"], q["scales"], n, center=B)
             units += W.shape[0] * layer.d * wl.G * wl.k_max
+            if collect is not None:
+                collect[(b, li)] = dict(W=W, codes=q["codes"], scales=q["scales"], err=err,
+                                        best=q["best"], second=q["second"])
     return units
 
 
@@ -530,18 +609,119 @@ def sample_inputs(wl, stride):
 
 
 def cpu_baseline(wl, target_s, center=-1):
+    """The oracle timed on the sampled channels; returns (cpu_baseline record, the oracle's
+    outputs per (bits, layer) for the parity report)."""
     import oracle
     oracle.build()
     stride = oracle_sample(wl, target_s)
     threads = host_cores()
     inputs = sample_inputs(wl, stride)
+    collect = {}
     t0 = time.perf_counter()
-    units = run_oracle_step(wl, stride, threads, inputs, center)
+    units = run_oracle_step(wl, stride, threads, inputs, center, collect=collect)
     dt = time.perf_counter() - t0
-    return {"value": units / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
-            "seconds": dt,
-            "sample": f"every {stride}th channel of every layer of the same workload "
-                      f"({units:.3e} units), oracle threads over channels"}
+    return ({"value": units / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+             "seconds": dt,
+             "sample": f"every {stride}th channel of every layer of the same workload "
+                       f"({units:.3e} units), oracle threads over channels"}, collect)
+
+
+def gpu_sample_outputs(net, specs, Ws, Xs, wl, stream, stride):
+    """Runs every bit width once more (one stream) and keeps the GPU's results for the parity
+    report: codes, scales and reconstructions of the sampled channels (every stride-th), the whole
+    error table and point counts of every layer (the allocation is checked on the full table)."""
+    import torch
+    out = {}
+    for b in wl.bits:
+        for sp in specs:
+            sp.bits = b
+        net.run_device(Ws, Xs, stream=stream)
+        torch.cuda.synchronize()
+        for li, p in enumerate(net.plans):
+            sel = torch.arange(0, p.spec.C, stride, device=p.codes.device)
+            out[(b, li)] = dict(codes=p.codes.index_select(1, sel).cpu().numpy(),
+                                scales=p.scales.index_select(0, sel).cpu().numpy(),
+                                err=p.err.cpu().numpy(), npoints=p.npoints.cpu().numpy(),
+                                points_used=int(p.points_used.item()),
+                                W_hat=p.W_hat.index_select(0, sel).cpu().numpy(),
+                                center=None if p.center is None else
+                                p.center.index_select(0, sel).cpu().numpy(), stride=stride)
+    return out
+
+
+NEAR_TIE_RTOL = 1e-6     # oracle top-two candidate errors this close (relative) are a near tie
+VALUE_RTOL = 1e-5        # fp32 values (output errors) against the oracle's double results
+
+
+def parity_report(wl, gpu, orc, center=-1):
+    """GPU results against the oracle on the sampled channels, counted the way the parity bar
+    states them: codes and scales bit-exact per greedy step except at a near tie (the oracle's
+    error at the GPU's scale within 1e-6 relative of its best; the channel's later steps are then
+    excluded), output errors within 1e-5 relative (channels that never diverged), point counts
+    bit-exact against the oracle's allocation of the GPU's whole error table (Algorithm 2 as a
+    sequential loop), reconstructions (Eq. 4) bit-exact."""
+    import oracle
+    rep = dict(channels=0, steps_compared=0, mismatch_steps=0, near_tie_mismatches=0,
+               other_mismatches=0, diverged_steps_excluded=0, oracle_near_ties=0, err_values=0,
+               err_max_rel=0.0, npoints_compared=0, npoints_mismatches=0,
+               points_used_mismatches=0, reconstruct_mismatch_channels=0)
+    K = wl.k_max
+    for (b, li), o in orc.items():
+        g = gpu[(b, li)]
+        C_s = o["codes"].shape[1]
+        rep["channels"] += C_s
+        o_best, o_second = o["best"], o["second"]
+        rep["oracle_near_ties"] += int(np.sum((o_second - o_best) <= NEAR_TIE_RTOL * o_second))
+        for c in range(C_s):
+            diverged = None
+            for i in range(K):
+                same = (g["scales"][c, i].tobytes() == o["scales"][c, i].tobytes() and
+                        np.array_equal(g["codes"][i, c], o["codes"][i, c]))
+                if same:
+                    rep["steps_compared"] += 1
+                    continue
+                rep["mismatch_steps"] += 1
+                if g["scales"][c, i].tobytes() == o["scales"][c, i].tobytes():
+                    rep["other_mismatches"] += 1      # same scale, other codes: never a tie
+                    rep["diverged_steps_excluded"] += K - 1 - i
+                    diverged = i
+                    break
+                r = o["W"][c] if i == 0 else oracle.quantize_layer(
+                    o["W"][c:c + 1], b, wl.G, i)["residuals"][i - 1, 0]
+                E, s = oracle.candidate_errors(r, b, wl.G)
+                hit = np.nonzero(s == g["scales"][c, i])[0]
+                if hit.size and E[hit[0]] <= E.min() * (1 + NEAR_TIE_RTOL):
+                    rep["near_tie_mismatches"] += 1
+                else:
+                    rep["other_mismatches"] += 1
+                rep["diverged_steps_excluded"] += K - 1 - i
+                diverged = i
+                break
+            if diverged is None:
+                ge = g["err"][c * g["stride"]].astype(np.float64)
+                oe = o["err"][c]
+                f = np.isfinite(oe)
+                if f.any():
+                    rel = np.abs(ge[f] - oe[f]) / np.maximum(np.abs(oe[f]), 1e-300)
+                    rep["err_max_rel"] = max(rep["err_max_rel"], float(rel.max()))
+                    rep["err_values"] += int(f.sum())
+        n_or, used_or = oracle.allocate_budget(g["err"], K, wl.beta)
+        rep["npoints_compared"] += n_or.size
+        rep["npoints_mismatches"] += int(np.sum(n_or != g["npoints"]))
+        rep["points_used_mismatches"] += int(used_or != g["points_used"])
+        sel_n = g["npoints"][::g["stride"]]
+        W_or = oracle.reconstruct(g["codes"], g["scales"], sel_n, center=g["center"])
+        rep["reconstruct_mismatch_channels"] += int(np.sum(
+            np.any(W_or.view(np.uint32) != g["W_hat"].view(np.uint32), axis=1)))
+    rep["err_rtol"] = VALUE_RTOL
+    rep["near_tie_rtol"] = NEAR_TIE_RTOL
+    rep["status"] = "pass" if (rep["other_mismatches"] == 0 and rep["npoints_mismatches"] == 0 and
+                               rep["points_used_mismatches"] == 0 and
+                               rep["reconstruct_mismatch_channels"] == 0 and
+                               rep["err_max_rel"] <= VALUE_RTOL) else "fail"
+    rep["sample"] = (f"every {next(iter(gpu.values()))['stride']}th channel of every layer "
+                     "(the cpu_baseline sample); point counts on every channel")
+    return rep
 
 
 def run_reference(args, world, rank):

@@ -162,19 +162,25 @@ mpq_status mpq_quantize_layer_adaptive(const float *W, int C, int d, int bits, i
 
 /*
  * mpq_output_error_noalloc -- mpq_output_error that allocates nothing.  The paper has no
- * counterpart: it is an engineering variant of the Eq. 11 call for callers that must not touch
- * a memory pool (a caller-managed memory budget, a process that disables stream-ordered pools).
+ * counterpart: it is an engineering variant of the Eq. 11 call for callers that cannot allocate
+ * device memory while they run -- a process whose memory is budgeted up front by its owner, a
+ * framework whose allocator owns the stream-ordered pool, or a pool that is switched off.
  *
  * Same arguments, layouts, validation, results (bit for bit) and errors as mpq_output_error,
  * except for the scratch: the tensor-core path's range table (1 + C (k_max+1) words) lives in one
- * fixed device array of MPQ_NOALLOC_RANGE_WORDS words inside the library, allocated when the
- * library's module is loaded.  Therefore:
+ * fixed device array of MPQ_NOALLOC_RANGE_WORDS words (4 MiB) inside the library, which every
+ * device that loads the library's module keeps until the process exits.  The call zeroes the
+ * part of the table it uses before filling it.  Therefore:
  *  - a call whose table would exceed MPQ_NOALLOC_RANGE_WORDS words is rejected with
  *    MPQ_ERR_UNSUPPORTED before anything is enqueued;
- *  - overlapping calls race: every call of this entry point uses the same buffer, so two calls
- *    whose kernels can run at the same time (on different streams, in different threads, or in
- *    CUDA graphs replayed concurrently) overwrite each other's ranges and return wrong errors.
- *    Order them (one stream, or events between streams).  mpq_output_error has no such limit.
+ *  - the first call on a device (made with that device current) looks up the array's device
+ *    address (cudaGetSymbolAddress) and keeps it; under CUDA's default lazy module loading that
+ *    lookup is also what loads the module, and so the array, on that device.  Make this first
+ *    call before any stream capture begins;
+ *  - overlapping calls race: every call of this entry point uses the same array, so two calls
+ *    whose kernels can run at the same time (on different streams or from different threads)
+ *    overwrite each other's ranges and return wrong errors.  Order them (one stream, or events
+ *    between streams).  mpq_output_error has no such limit.
  */
 mpq_status mpq_output_error_noalloc(const float *X, int N, int groups, const float *W,
                                     const int8_t *codes, const float *scales, int C, int d,

@@ -16,7 +16,7 @@
  * is written here as s_i q_i with integer codes q_i in {-Qmax..Qmax}, Qmax = 2^(b-1)-1 and
  * s_i = a_i / Qmax (Eq. 1, symmetric set, B = 0).
  *
- * Readings where the paper is silent (each one is also listed in the design doc):
+ * Readings where the paper is silent, ambiguous or garbled:
  *  - exact half-way ties of the nearest rounding (Eq. 2) go to the even integer (C nearbyintf);
  *  - r / a is one correctly rounded fp32 division (Eq. 8 writes a division);
  *  - the scale grid is G points s_g = f_g * (max|r| / Qmax), f_g = (g+1)/G in fp32 unless the caller
@@ -624,8 +624,8 @@ void mpqo_reconstruct(const int8_t *codes, const float *scales, const int *npoin
 
 /* ---- Eq. 1 with B != 0: asymmetric sets ---------------------------------------------------------
  * The quantization set K x [-1 : eps_b : 1] + B has the centre B.  Per channel (mode 0) every
- * channel has its own B; per layer (mode 1) one B serves all the layer's channels.  Readings (also
- * in the design doc): B is the midpoint of the weights' range, (max w + min w) / 2 rounded once to fp32,
+ * channel has its own B; per layer (mode 1) one B serves all the layer's channels.  Readings (the
+ * paper gives no formula for B): B is the midpoint of the weights' range, (max w + min w) / 2 rounded once to fp32,
  * so that K = (max w - min w) / 2 covers every weight without clipping (the per-channel
  * experiments clip nothing); the multipoint approximation takes B once and approximates the
  * centred weights w - B (one fp32 subtraction) with the greedy points, so that
@@ -666,8 +666,8 @@ void mpqo_center(const float *W, int C, int d, int mode, float *center, float *W
 
 /* ---- Eq. 12: output-error-driven clipping factor ------------------------------------------------
  * The clipping factor K of the quantization set K x [-1 : eps_b : 1] (Eq. 1, B = 0) is chosen among
- * nc candidates by the output error of Eq. 11 instead of the weight error.  Readings (also in
- * the design doc): the candidates are K_c = f_c * m with f_c = (c+1)/nc in fp32, c = 0..nc-1 (nc = 20 is
+ * nc candidates by the output error of Eq. 11 instead of the weight error.  Readings (App. B gives
+ * only the grid): the candidates are K_c = f_c * m with f_c = (c+1)/nc in fp32, c = 0..nc-1 (nc = 20 is
  * the experiments' uniform grid [0.05 : 0.05 : 1] x max|w|); m = max_j |w_kj| per channel
  * (mode 0) or the maximum over the whole layer (mode 1, one K for every channel); the set's
  * elements are s q with s = K / Qmax (fp32 division) and codes q = [w / s]_Q as in Eq. 8; the
@@ -766,7 +766,7 @@ void mpqo_clip_select(const float *err, int C, int nc, int mode, int *best)
  *   w~_k^T x_t = sum_i s_{k,i} (q_{k,i}^T x_t) ~ (sum_i A_{k,i} (q_{k,i}^T x_t)) / 2^p,
  *   A_{k,i} = [2^p s_{k,i}]  (Eq. 13),
  * in three steps: integer dot products (step 1), multiplication by the 32-bit coefficients and
- * summation (step 2), and a shift by p bits (step 3).  Readings (also in the design doc): the codes q are
+ * summation (step 2), and a shift by p bits (step 3).  Readings of Sec. 3.4: the codes q are
  * the integers of the symmetric set, so the coefficient of q is s = a / Qmax and A = rint(2^p s)
  * (ties to even); "shifting p bits" is an arithmetic right shift, i.e. floor division by 2^p; the
  * products and sums are exact (64-bit); the result saturates to the 32-bit range; n_k = npoints[k]

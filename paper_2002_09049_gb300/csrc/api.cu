@@ -5,6 +5,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
+
 #include "mpq_internal.cuh"
 
 namespace mpq {
@@ -26,7 +28,7 @@ mpq_status cuda_status(cudaError_t e, const char *what)
     return MPQ_ERR_CUDA;
 }
 
-static const int kMaxDevices = 64;
+const int kMaxDevices = 64;
 
 int sm_count()
 {
@@ -166,8 +168,30 @@ extern "C" mpq_status mpq_output_error(const float *X, int N, int groups, const 
 }
 
 // The fixed scratch of mpq_output_error_noalloc: one array for every call of that entry point
-// (overlapping calls race on it, as its declaration states).
+// (overlapping calls race on it, as its declaration states).  Host code cannot use the symbol
+// itself as a device address: its address on each device is resolved once, with that device
+// current, by the first call made there, and kept.
 static __device__ __align__(256) unsigned g_noalloc_range[MPQ_NOALLOC_RANGE_WORDS];
+static unsigned *g_noalloc_addr[kMaxDevices];
+static std::mutex g_noalloc_mu;
+
+static mpq_status noalloc_scratch(unsigned **out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_status(e, "cudaGetDevice");
+    REQUIRE(dev >= 0 && dev < kMaxDevices, MPQ_ERR_UNSUPPORTED, "device %d beyond %d devices", dev,
+            kMaxDevices);
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_range);
+        if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress (fixed scratch)");
+        g_noalloc_addr[dev] = static_cast<unsigned *>(p);
+    }
+    *out = g_noalloc_addr[dev];
+    return MPQ_OK;
+}
 
 extern "C" mpq_status mpq_output_error_noalloc(const float *X, int N, int groups, const float *W,
                                                const int8_t *codes, const float *scales, int C,
@@ -182,8 +206,8 @@ extern "C" mpq_status mpq_output_error_noalloc(const float *X, int N, int groups
             MPQ_NOALLOC_RANGE_WORDS);
     unsigned *range = nullptr;
     if (words > 0) {
-        const cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&range), g_noalloc_range);
-        if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress (fixed scratch)");
+        const mpq_status sa = noalloc_scratch(&range);
+        if (sa != MPQ_OK) return sa;
     }
     return launch_output_error(X, N, groups, W, codes, scales, C, d, k_max, err,
                                (cudaStream_t)stream, range);
