@@ -44,7 +44,7 @@ typedef enum {
     MPQ_ERR_NONFINITE = 2,    /* a host-side numeric parameter is NaN/Inf */
     MPQ_ERR_UNSUPPORTED = 3,  /* valid for the method but beyond this library's limits below */
     MPQ_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
-    MPQ_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up (reserved) */
+    MPQ_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up (mpq_device_status) */
     MPQ_ERR_NOMEM = 6         /* mpq_output_error's stream-ordered scratch allocation failed */
 } mpq_status;
 
@@ -326,6 +326,45 @@ mpq_status mpq_pack_points(const int8_t *codes, const float *scales, const float
  */
 mpq_status mpq_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout *layout,
                                  const void *packed, int32_t *Y, void *stream);
+
+/*
+ * Bounded device-side waits.  The tensor-core kernels (mpq_output_error and its _noalloc variant,
+ * mpq_clip_search, mpq_multipoint_linear) hand work between their warps through shared-memory
+ * barriers, and every wait on one is bounded by a clock budget.  A kernel whose wait gives up
+ * stops issuing work, waits for the copies and MMAs it has already issued to finish, releases its
+ * tensor memory and returns, with NaN in its output errors (its inference outputs unspecified);
+ * it records which kernel it was in a word kept per device.  A NaN error can therefore mean a
+ * non-finite input or a timeout: mpq_device_status tells them apart.
+ */
+#define MPQ_TIMEOUT_OUTPUT_ERROR 0x1u   /* mpq_output_error / mpq_output_error_noalloc */
+#define MPQ_TIMEOUT_CLIP 0x2u           /* mpq_clip_search */
+#define MPQ_TIMEOUT_INFERENCE 0x4u      /* mpq_multipoint_linear */
+#define MPQ_TIMEOUT_DRAIN 0x100u        /* a wait for the kernel's own copies or MMAs also gave up */
+
+/*
+ * mpq_device_status -- synchronizes `stream`, then takes the current device's timeout word
+ * (reads and clears it in one atomic exchange on the device): MPQ_OK if no bounded wait gave up
+ * since the last call, else MPQ_ERR_TIMEOUT with the MPQ_TIMEOUT_* bits in *flags (nullable; 0 on
+ * MPQ_OK).  It covers the kernels that have finished when the exchange runs: synchronize the
+ * other streams first to include their calls.  Synchronous.
+ */
+mpq_status mpq_device_status(void *stream, unsigned *flags);
+
+/*
+ * mpq_set_wait_limit -- the clock budget of every bounded wait of the kernels launched after
+ * this call (process-wide), in SM clocks; clocks <= 0 restores the default of 2^31 (about one
+ * second at the maximum SM clock).  A budget far below a kernel's normal waits makes healthy
+ * launches give up: it is meant for tests.
+ */
+mpq_status mpq_set_wait_limit(long long clocks);
+
+/*
+ * mpq_test_withhold_copies -- TEST HOOK, process-wide: while on (1), the tile-copy thread of the
+ * output-error contraction (mpq_output_error's tensor-core path) issues no copies, so that every
+ * wait of that kernel runs out with nothing in flight and the call reports MPQ_TIMEOUT_OUTPUT_ERROR
+ * through mpq_device_status.  Off (0) by default; never on outside tests of the timeout path.
+ */
+mpq_status mpq_test_withhold_copies(int on);
 
 /* Name of a status code (static string). */
 const char *mpq_status_string(mpq_status s);

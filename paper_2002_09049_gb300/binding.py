@@ -22,6 +22,10 @@ MPQ_CLIP_PER_CHANNEL = 0
 MPQ_CLIP_PER_LAYER = 1
 MPQ_NOALLOC_RANGE_WORDS = 1 << 20     # the fixed scratch of mpq_output_error_noalloc
 MPQ_ADAPTIVE_MAX_DIM = 64             # the longest channel of mpq_quantize_layer_adaptive
+MPQ_TIMEOUT_OUTPUT_ERROR = 0x1        # timeout bits of mpq_device_status
+MPQ_TIMEOUT_CLIP = 0x2
+MPQ_TIMEOUT_INFERENCE = 0x4
+MPQ_TIMEOUT_DRAIN = 0x100
 
 MPQ_STATUS = {0: "MPQ_OK", 1: "MPQ_ERR_INVALID_ARG", 2: "MPQ_ERR_NONFINITE",
               3: "MPQ_ERR_UNSUPPORTED", 4: "MPQ_ERR_CUDA", 5: "MPQ_ERR_TIMEOUT",
@@ -55,6 +59,9 @@ SIGNATURES = {
     "mpq_pack_layout": ([_P, _I, _I, _I, _I, _I, _I, _L], _I),
     "mpq_pack_points": ([_P, _P, _P, _P, _L, _P, _P], _I),
     "mpq_multipoint_linear": ([_P, _I, _L, _P, _P, _P], _I),
+    "mpq_device_status": ([_P, _P], _I),
+    "mpq_set_wait_limit": ([ctypes.c_longlong], _I),
+    "mpq_test_withhold_copies": ([_I], _I),
     "mpq_status_string": ([_I], ctypes.c_char_p),
     "mpq_last_error": ([], ctypes.c_char_p),
     "mpq_version": ([], _I),
@@ -365,3 +372,23 @@ def mpq_status_string(status: int) -> str:
 
 def mpq_version() -> int:
     return load().mpq_version()
+
+
+def mpq_device_status(stream=None):
+    """Synchronizes the stream and takes the current device's timeout word: 0 if no bounded wait
+    of a tensor-core kernel gave up since the last call, else the MPQ_TIMEOUT_* bits."""
+    flags = ctypes.c_uint(0)
+    st = load().mpq_device_status(_stream(stream), ctypes.byref(flags))
+    if st not in (0, 5):
+        _check(st, "mpq_device_status")
+    return int(flags.value)
+
+
+def mpq_set_wait_limit(clocks: int):
+    """Clock budget of every bounded device wait of later launches (<= 0: the default)."""
+    _check(load().mpq_set_wait_limit(int(clocks)), "mpq_set_wait_limit")
+
+
+def mpq_test_withhold_copies(on: bool):
+    """Test hook: the output-error contraction's copy thread issues no copies while on."""
+    _check(load().mpq_test_withhold_copies(1 if on else 0), "mpq_test_withhold_copies")

@@ -8,6 +8,9 @@
 
 namespace mpq {
 
+// Devices whose per-device state (cached attributes, resolved symbol addresses) is kept.
+constexpr int kMaxDevices = 64;
+
 // acc + comp += v, compensated (Kahan): the rounding error of each addition is carried in comp.
 __device__ __forceinline__ void kahan_add(float &acc, float &comp, float v)
 {

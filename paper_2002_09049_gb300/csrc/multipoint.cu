@@ -42,6 +42,7 @@
 #include "mpq_internal.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
+#include "waits.cuh"
 
 namespace mpq {
 namespace {
@@ -78,7 +79,6 @@ constexpr int L_MMA_WARP = L_EPI_WARP0 + 4;
 constexpr int L_TMA_A_WARP = L_MMA_WARP + 1;    // codes tiles
 constexpr int L_TMA_X_WARP = L_TMA_A_WARP + 1;  // raw input tiles
 constexpr int L_THREADS = (L_TMA_X_WARP + 1) * 32;   // 480
-constexpr long long L_WAIT = 1LL << 31;
 
 struct LinCtrl {
     uint64_t a_full[L_MAX_SLOTS];     // a codes slot has landed
@@ -168,7 +168,8 @@ __global__ void __launch_bounds__(L_THREADS, 1)
 multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restrict__ coef,
                          const int *__restrict__ chan, const int *__restrict__ tile_R,
                          const int *__restrict__ center_coef,
-                         int32_t *__restrict__ Y, const __grid_constant__ CUtensorMap tmA,
+                         int32_t *__restrict__ Y, const WaitCtl wc,
+                         const __grid_constant__ CUtensorMap tmA,
                          const __grid_constant__ CUtensorMap tmX)
 {
     using G = LGeo<RT>;
@@ -223,10 +224,13 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
         for (int it = 0; it < ITEMS; ++it) xs[it] = 0;
         for (int kc = 0; kc < n_kc; ++kc) {
             const int rs = kc % G::R_SLOTS, bs = kc % G::B_SLOTS;
-            bool ok = mbar_wait(&ctl.r_full[rs], (uint32_t)(kc / G::R_SLOTS) & 1u, L_WAIT);
+            bool ok = mbar_wait(&ctl.r_full[rs], (uint32_t)(kc / G::R_SLOTS) & 1u, wc.budget);
             if (ok && kc >= G::B_SLOTS)
-                ok = mbar_wait(&ctl.b_empty[bs], (uint32_t)(kc / G::B_SLOTS - 1) & 1u, L_WAIT);
-            if (!ok) *abort_flag = 1;
+                ok = mbar_wait(&ctl.b_empty[bs], (uint32_t)(kc / G::B_SLOTS - 1) & 1u, wc.budget);
+            if (!ok) {
+                *abort_flag = 1;
+                note_timeout(wc, MPQ_TIMEOUT_INFERENCE);
+            }
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
             // 16 input bytes (one input row, 16 K elements) per item, 4 items per thread: all
             // reads first, then the raw slot goes back to the TMA thread
@@ -283,9 +287,12 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
     } else if (warp < L_MMA_WARP) {
         // ---------------------------------------------------------------- epilogue
         const int ew = warp - L_EPI_WARP0;
-        bool ok = mbar_wait(&ctl.done, 0, L_WAIT);
-        if (ok && centered) ok = mbar_wait(&ctl.xs_ready, 0, L_WAIT);
-        if (!ok) *abort_flag = 1;
+        bool ok = mbar_wait(&ctl.done, 0, wc.budget);
+        if (ok && centered) ok = mbar_wait(&ctl.xs_ready, 0, wc.budget);
+        if (!ok) {
+            *abort_flag = 1;
+            note_timeout(wc, MPQ_TIMEOUT_INFERENCE);
+        }
         const bool good = !__any_sync(0xffffffffu, !ok || *abort_flag);
         tc_fence_after();
         // staging for the stores: the bf16 input ring, idle once every MMA has completed
@@ -351,9 +358,12 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             constexpr uint32_t idesc = idesc_bf16(L_M, L_N);
             for (int kc = 0; kc < n_kc; ++kc) {
                 const int as = kc % G::A_SLOTS, bs = kc % G::B_SLOTS;
-                bool ok = mbar_wait(&ctl.a_full[as], (uint32_t)(kc / G::A_SLOTS) & 1u, L_WAIT);
-                if (ok) ok = mbar_wait(&ctl.b_full[bs], (uint32_t)(kc / G::B_SLOTS) & 1u, L_WAIT);
-                if (!ok) *abort_flag = 1;
+                bool ok = mbar_wait(&ctl.a_full[as], (uint32_t)(kc / G::A_SLOTS) & 1u, wc.budget);
+                if (ok) ok = mbar_wait(&ctl.b_full[bs], (uint32_t)(kc / G::B_SLOTS) & 1u, wc.budget);
+                if (!ok) {
+                    *abort_flag = 1;
+                    note_timeout(wc, MPQ_TIMEOUT_INFERENCE);
+                }
                 if (*abort_flag) break;
                 tc_fence_after();
                 const uint64_t bd = smem_desc_sw128(b_u32 + bs * L_B_BYTES);
@@ -380,8 +390,10 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             for (int kc = 0; kc < n_kc; ++kc) {
                 const int as = kc % G::A_SLOTS;
                 if (kc >= G::A_SLOTS &&
-                    !mbar_wait(&ctl.a_empty[as], (uint32_t)(kc / G::A_SLOTS - 1) & 1u, L_WAIT))
+                    !mbar_wait(&ctl.a_empty[as], (uint32_t)(kc / G::A_SLOTS - 1) & 1u, wc.budget)) {
                     *abort_flag = 1;
+                    note_timeout(wc, MPQ_TIMEOUT_INFERENCE);
+                }
                 if (*abort_flag) break;
                 mbar_arrive_expect_tx(&ctl.a_full[as], (uint32_t)(nt * L_A_BYTES));
                 for (int u = 0; u < nt; ++u)
@@ -391,7 +403,8 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             }
             // no copy may land after the CTA is gone
             for (int kc = issued - G::A_SLOTS > 0 ? issued - G::A_SLOTS : 0; kc < issued; ++kc)
-                mbar_wait(&ctl.a_full[kc % G::A_SLOTS], (uint32_t)(kc / G::A_SLOTS) & 1u, L_WAIT);
+                drain_wait(&ctl.a_full[kc % G::A_SLOTS], (uint32_t)(kc / G::A_SLOTS) & 1u, wc,
+                           MPQ_TIMEOUT_INFERENCE);
         }
         __syncwarp();
     } else {
@@ -402,15 +415,18 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             for (int kc = 0; kc < n_kc; ++kc) {
                 const int rs = kc % G::R_SLOTS;
                 if (kc >= G::R_SLOTS &&
-                    !mbar_wait(&ctl.r_empty[rs], (uint32_t)(kc / G::R_SLOTS - 1) & 1u, L_WAIT))
+                    !mbar_wait(&ctl.r_empty[rs], (uint32_t)(kc / G::R_SLOTS - 1) & 1u, wc.budget)) {
                     *abort_flag = 1;
+                    note_timeout(wc, MPQ_TIMEOUT_INFERENCE);
+                }
                 if (*abort_flag) break;
                 mbar_arrive_expect_tx(&ctl.r_full[rs], (uint32_t)L_RAW_BYTES);
                 tma_load_2d(x_u32 + rs * L_RAW_BYTES, &tmX, kc * L_KC, n0, &ctl.r_full[rs]);
                 issued = kc + 1;
             }
             for (int kc = issued - G::R_SLOTS > 0 ? issued - G::R_SLOTS : 0; kc < issued; ++kc)
-                mbar_wait(&ctl.r_full[kc % G::R_SLOTS], (uint32_t)(kc / G::R_SLOTS) & 1u, L_WAIT);
+                drain_wait(&ctl.r_full[kc % G::R_SLOTS], (uint32_t)(kc / G::R_SLOTS) & 1u, wc,
+                           MPQ_TIMEOUT_INFERENCE);
         }
         __syncwarp();
     }
@@ -418,7 +434,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
     __syncthreads();
     if (warp == L_MMA_WARP) {
         // every MMA has completed: the epilogue waited for `done` (or the wait timed out)
-        if (lane == 0 && *abort_flag) mbar_wait(&ctl.done, 0, L_WAIT);
+        if (lane == 0 && *abort_flag) drain_wait(&ctl.done, 0, wc, MPQ_TIMEOUT_INFERENCE);
         __syncwarp();
         tc_fence_after();
         tmem_dealloc(tmem, G::TMEM_COLS);
@@ -633,8 +649,11 @@ mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_lay
         if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
         const int rt = two ? 2 : 1;
         const dim3 grid((unsigned)tt, (unsigned)((L->tiles + rt - 1) / rt));
+        WaitCtl wc;
+        const mpq_status wst = wait_ctl(&wc);
+        if (wst != MPQ_OK) return wst;
         kernel<<<grid, L_THREADS, smem, stream>>>(T, L->tiles, L->d_pad / L_KC, L->p, v.coef,
-                                                  v.chan, v.tile_R, v.center, Y, tmA, tmX);
+                                                  v.chan, v.tile_R, v.center, Y, wc, tmA, tmX);
         return cuda_status(cudaGetLastError(), "multipoint linear kernel launch");
     }
     const size_t n = (size_t)L->rows * T;

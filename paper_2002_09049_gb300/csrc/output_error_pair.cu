@@ -33,7 +33,8 @@
 //
 // Row tiles (256 rows) are split over the pairs of a cluster of up to 8 CTAs; ranks 0 and 1 add
 // their peers' partial sums from distributed shared memory in rank order.  Every wait is bounded;
-// on a timeout the outputs read NaN.
+// on a timeout the kernel records MPQ_TIMEOUT_OUTPUT_ERROR (or _CLIP), unwinds and the outputs
+// read NaN.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
@@ -47,6 +48,7 @@
 #include "rounding.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
+#include "waits.cuh"
 
 namespace mpq {
 namespace {
@@ -95,7 +97,6 @@ struct PRoles {
 constexpr uint32_t P_TMEM_COLS = 512;
 constexpr uint32_t P_RUN_COL = 256;
 constexpr int P_MAX_RAW = 3;
-constexpr long long P_WAIT = 1LL << 31;         // SM clocks (~1 s)
 constexpr int P_SMEM_LIMIT = 232448;            // opt-in shared memory per CTA on sm_100 parts
 
 struct PairCtrl {
@@ -324,13 +325,14 @@ template <int KP1, bool CLIP>
 __global__ void __launch_bounds__(PRoles<CLIP>::THREADS, 1)
 output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, int qmax,
                          const unsigned *__restrict__ range, float *__restrict__ err, int split,
-                         const __grid_constant__ CUtensorMap tmX,
+                         const WaitCtl wc, const __grid_constant__ CUtensorMap tmX,
                          const __grid_constant__ CUtensorMap tmW,
                          const __grid_constant__ CUtensorMap tmQ)
 {
     using G = PGeo<KP1, CLIP>;
     using PR = PRoles<CLIP>;
     constexpr bool F16 = !CLIP;
+    constexpr unsigned KBIT = CLIP ? MPQ_TIMEOUT_CLIP : MPQ_TIMEOUT_OUTPUT_ERROR;
     constexpr int NST = PFmt<F16>::STAGES, SEG = PFmt<F16>::SEG;
     constexpr int R = G::RAW_STAGES;
     extern __shared__ unsigned char smem_raw[];
@@ -422,9 +424,12 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         for (int it = 0; it < total; ++it) {
             const int s = it % NST, slot = it % R;
             const uint32_t ph = (uint32_t)(it / NST) & 1u;
-            const bool ok = mbar_wait(&ctl.raw_full[slot], (uint32_t)(it / R) & 1u, P_WAIT) &&
-                            mbar_wait_cluster(&ctl.empty[s], ph ^ 1u, P_WAIT);
-            if (!ok) *abort_flag = 1;
+            const bool ok = mbar_wait(&ctl.raw_full[slot], (uint32_t)(it / R) & 1u, wc.budget) &&
+                            mbar_wait_cluster(&ctl.empty[s], ph ^ 1u, wc.budget);
+            if (!ok) {
+                *abort_flag = 1;
+                note_timeout(wc, KBIT);
+            }
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
             const int ts = F16 ? s >> 1 : s, hh = F16 ? s & 1 : 0;
             pair_consume<KP1, CLIP>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + ts * P_STAGE_BYTES,
@@ -446,8 +451,11 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         bool stop = false;
         for (int lt = 0; lt < my_rt && !stop; ++lt) {
             for (int sg = 0; sg < nseg; ++sg, ++g) {
-                const bool ok = mbar_wait_cluster(&ctl.segfull, (uint32_t)g & 1u, P_WAIT);
-                if (!ok) *abort_flag = 1;
+                const bool ok = mbar_wait_cluster(&ctl.segfull, (uint32_t)g & 1u, wc.budget);
+                if (!ok) {
+                    *abort_flag = 1;
+                    note_timeout(wc, KBIT);
+                }
                 stop = __any_sync(0xffffffffu, !ok || *abort_flag);   // warp-uniform
                 if (stop) break;
                 tc_fence_after();
@@ -490,15 +498,20 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                     const bool seg_start = (kc % SEG) == 0;
                     if (seg_start) {
                         // both CTAs' epilogues must have drained the previous segment
-                        if (!mbar_wait_cluster(&ctl.segempty, ((uint32_t)g & 1u) ^ 1u, P_WAIT))
+                        if (!mbar_wait_cluster(&ctl.segempty, ((uint32_t)g & 1u) ^ 1u, wc.budget)) {
                             *abort_flag = 1;
+                            note_timeout(wc, KBIT);
+                        }
                         if (*abort_flag) break;
                         tc_fence_after();
                     }
                     const int it = lt * n_kc + kc;
                     const int s = it % NST;
                     const uint32_t ph = (uint32_t)(it / NST) & 1u;
-                    if (!mbar_wait_cluster(&ctl.full[s], ph, P_WAIT)) *abort_flag = 1;
+                    if (!mbar_wait_cluster(&ctl.full[s], ph, wc.budget)) {
+                        *abort_flag = 1;
+                        note_timeout(wc, KBIT);
+                    }
                     if (*abort_flag) break;
                     tc_fence_after();
                     const uint32_t sb = stages_u32 + (F16 ? s >> 1 : s) * P_STAGE_BYTES;
@@ -533,7 +546,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             }
             // drain: every MMA issued above completes before TMEM is released
             mma_commit_pair(&ctl.done, (uint16_t)(1u << leader));
-            mbar_wait_cluster(&ctl.done, 0, P_WAIT);
+            drain_wait_cluster(&ctl.done, 0, wc, KBIT);
         }
         __syncwarp();
     } else {
@@ -543,11 +556,13 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             prefetch_tensormap(&tmW);
             prefetch_tensormap(&tmQ);
             int issued = 0;
-            for (int f = 0; f < total; ++f) {
+            for (int f = 0; f < ((!CLIP && wc.withhold) ? 0 : total); ++f) {
                 const int slot = f % R;
                 if (f >= R &&
-                    !mbar_wait(&ctl.raw_empty[slot], (uint32_t)(f / R - 1) & 1u, P_WAIT))
+                    !mbar_wait(&ctl.raw_empty[slot], (uint32_t)(f / R - 1) & 1u, wc.budget)) {
                     *abort_flag = 1;
+                    note_timeout(wc, KBIT);
+                }
                 if (*abort_flag) break;
                 const uint32_t dst = ring_u32 + slot * G::RAW_BYTES;
                 const int x = (f % n_kc) * P_KC;
@@ -560,7 +575,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             }
             // no copy may land after the CTA is gone: wait for the last copies of every slot
             for (int f = issued - R > 0 ? issued - R : 0; f < issued; ++f)
-                mbar_wait(&ctl.raw_full[f % R], (uint32_t)(f / R) & 1u, P_WAIT);
+                drain_wait(&ctl.raw_full[f % R], (uint32_t)(f / R) & 1u, wc, KBIT);
         }
         __syncwarp();
     }
@@ -795,6 +810,9 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     }
     attr[0].val.clusterDim.x = (unsigned)(2 * split);
     cfg.gridDim = dim3((unsigned)(n_pairs * 2 * split), 1, 1);
+    WaitCtl wc;
+    mpq_status wst = wait_ctl(&wc);
+    if (wst != MPQ_OK) return wst;
     unsigned *range = ext_range;
     if constexpr (!CLIP) {
         // fp16 operands: the ranges of X and of every residual vector first
@@ -815,7 +833,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         }
         if (e == cudaSuccess)
             e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
-                                   (const unsigned *)range, err, split, tmX, tmW, tmQ);
+                                   (const unsigned *)range, err, split, wc, tmX, tmW, tmQ);
         if (!ext_range) {
             const cudaError_t ef = cudaFreeAsync(range, stream);
             if (e == cudaSuccess) e = ef;
@@ -823,7 +841,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         return cuda_status(e, "pair output-error kernel launch");
     }
     e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
-                           (const unsigned *)nullptr, err, split, tmX, tmW, tmQ);
+                           (const unsigned *)nullptr, err, split, wc, tmX, tmW, tmQ);
     return cuda_status(e, "pair output-error kernel launch");
 }
 

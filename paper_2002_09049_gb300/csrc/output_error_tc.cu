@@ -36,6 +36,7 @@
 #include "mpq_internal.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
+#include "waits.cuh"
 
 namespace mpq {
 namespace {
@@ -64,7 +65,6 @@ constexpr int MMA_WARP = EPI_WARP0 + 4;
 constexpr int TC_THREADS = (MMA_WARP + 1) * 32; // 416
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t RUN_COL = 256;               // running sums start here
-constexpr long long WAIT_BUDGET = 1LL << 31;    // SM clocks (~1 s)
 
 struct Ctrl {
     uint64_t full[TC_STAGES];
@@ -201,7 +201,7 @@ template <int KP1>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restrict__ W,
                        const int8_t *__restrict__ codes, const float *__restrict__ scales, int C,
-                       int d, float *__restrict__ err, int split, bool vec_ok)
+                       int d, float *__restrict__ err, int split, bool vec_ok, const WaitCtl wc)
 {
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
@@ -252,8 +252,11 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
         for (int it = 0; it < total; ++it) {
             const int s = it % TC_STAGES;
             const uint32_t ph = (uint32_t)(it / TC_STAGES) & 1u;
-            const bool ok = mbar_wait(&ctl.empty[s], ph ^ 1u, WAIT_BUDGET);
-            if (!ok) *abort_flag = 1;
+            const bool ok = mbar_wait(&ctl.empty[s], ph ^ 1u, wc.budget);
+            if (!ok) {
+                *abort_flag = 1;
+                note_timeout(wc, MPQ_TIMEOUT_OUTPUT_ERROR);
+            }
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
             store_stage<KP1>(pf, pt, stages_u32 + s * STAGE_BYTES, nch);
             fence_proxy_async_smem();
@@ -275,8 +278,11 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
         bool stop = false;
         for (int lt = 0; lt < my_rt && !stop; ++lt) {
             for (int sg = 0; sg < nseg; ++sg, ++g) {
-                const bool ok = mbar_wait(&ctl.segfull, (uint32_t)g & 1u, WAIT_BUDGET);
-                if (!ok) *abort_flag = 1;
+                const bool ok = mbar_wait(&ctl.segfull, (uint32_t)g & 1u, wc.budget);
+                if (!ok) {
+                    *abort_flag = 1;
+                    note_timeout(wc, MPQ_TIMEOUT_OUTPUT_ERROR);
+                }
                 stop = __any_sync(0xffffffffu, !ok || *abort_flag);   // warp-uniform
                 if (stop) break;
                 tc_fence_after();
@@ -324,15 +330,20 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
                     const bool seg_start = (kc % SEG_CHUNKS) == 0;
                     if (seg_start) {
                         // the epilogue must have drained the previous segment
-                        if (!mbar_wait(&ctl.segempty, ((uint32_t)g & 1u) ^ 1u, WAIT_BUDGET))
+                        if (!mbar_wait(&ctl.segempty, ((uint32_t)g & 1u) ^ 1u, wc.budget)) {
                             *abort_flag = 1;
+                            note_timeout(wc, MPQ_TIMEOUT_OUTPUT_ERROR);
+                        }
                         if (*abort_flag) break;
                         tc_fence_after();
                     }
                     const int it = lt * n_kc + kc;
                     const int s = it % TC_STAGES;
                     const uint32_t ph = (uint32_t)(it / TC_STAGES) & 1u;
-                    if (!mbar_wait(&ctl.full[s], ph, WAIT_BUDGET)) *abort_flag = 1;
+                    if (!mbar_wait(&ctl.full[s], ph, wc.budget)) {
+                        *abort_flag = 1;
+                        note_timeout(wc, MPQ_TIMEOUT_OUTPUT_ERROR);
+                    }
                     if (*abort_flag) break;
                     tc_fence_after();
                     const uint32_t sb = stages_u32 + s * STAGE_BYTES;
@@ -360,7 +371,7 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
             }
             // drain: every MMA issued above completes before TMEM is released
             mma_commit(&ctl.done);
-            mbar_wait(&ctl.done, 0, WAIT_BUDGET);
+            drain_wait(&ctl.done, 0, wc, MPQ_TIMEOUT_OUTPUT_ERROR);
         }
         __syncwarp();
     }
@@ -416,8 +427,11 @@ mpq_status launch_tc(const float *X, int N, const float *W, const int8_t *codes,
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    WaitCtl wc;
+    const mpq_status wst = wait_ctl(&wc);
+    if (wst != MPQ_OK) return wst;
     e = cudaLaunchKernelEx(&cfg, output_error_tc_kernel<KP1>, X, N, W, codes, scales, C, d, err,
-                           split, vec_ok);
+                           split, vec_ok, wc);
     return cuda_status(e, "tensor-core output-error kernel launch");
 }
 
