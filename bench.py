@@ -1177,26 +1177,39 @@ def run_infer(args, world, rank, local):
     return out if rank == 0 else None
 
 
-FP64_NOMINAL_TFLOPS = 1.25   # the part's nominal dense FP64 rate (no measured FP64 peak exists)
-ADAPTIVE_CAP = 10 ** 7       # most candidates one adaptive-grid step may enumerate (a larger
-                             # step is refused; refused steps are counted in the config)
-ADAPTIVE_ORACLE_CAP = 10 ** 6   # the oracle sample's cap: bounds its time; it counts what it ran
-ADAPTIVE_METRIC = "weight-elements x adaptive-grid candidates x points / s"
+ADAPTIVE_CAP = 10 ** 15      # no refusal: the search does not enumerate the grid
+ADAPTIVE_METRIC = "weight-elements x points / s (adaptive grid of Eq. 10)"
+ADAPTIVE_UNIT = "elem*pt/s"
+ADAPTIVE_BUDGET_S = 20.0     # timed GPU work of one --op adaptive run, at most
+# Algorithmic lane operations of the adaptive search, per code-level threshold (every element
+# has Qmax of them a step): finding it (two correctly rounded divisions, rint, compare: 25),
+# sorting it (4 radix passes of 2 loads, a match, a popc, a store: 48), its piece's running sums
+# and fp32 lower bound (30); per element-step: the magnitude sort for Definition 1 (48), its gap
+# (6), the update and code store (11).
+ADAPTIVE_OPS_PER_THRESHOLD = 103
+ADAPTIVE_OPS_PER_ELEMENT = 65
 
 
 def adaptive_layers(wl):
     from paper_2002_09049_gb300 import binding
-    idx = [li for li, l in enumerate(wl.layers) if l.d <= binding.MPQ_ADAPTIVE_MAX_DIM]
+    qmax = (1 << (wl.bits[0] - 1)) - 1
+    idx = [li for li, l in enumerate(wl.layers)
+           if l.d * qmax <= binding.MPQ_ADAPTIVE_MAX_THRESHOLDS]
     if not idx:
-        raise SystemExit("--op adaptive needs layers of at most 64 weights per channel "
-                         "(e.g. --config c4, the depthwise 3x3 convolutions)")
+        raise SystemExit("--op adaptive: no layer with d * Qmax <= MPQ_ADAPTIVE_MAX_THRESHOLDS")
     return idx
 
 
+def adaptive_ops(wl, layer):
+    qmax = (1 << (wl.bits[0] - 1)) - 1
+    return layer.C * layer.d * wl.k_max * (ADAPTIVE_OPS_PER_THRESHOLD * qmax +
+                                           ADAPTIVE_OPS_PER_ELEMENT)
+
+
 def adaptive_oracle_step(wl, idx, per_layer, threads):
-    """The oracle's adaptive grid (Eq. 10) on the first `per_layer` channels of every short layer,
-    steps above ADAPTIVE_ORACLE_CAP candidates refused (not enumerated, not counted); returns the
-    element-candidate units it processed."""
+    """The oracle's adaptive grid (Eq. 10; its piecewise search, the definition's decisions
+    without enumerating) on the first `per_layer` channels of every layer; returns the
+    element-steps (C d k_max) it processed."""
     import oracle
     from concurrent.futures import ThreadPoolExecutor
     jobs = [(li, c) for li in idx for c in range(min(per_layer, wl.layers[li].C))]
@@ -1204,19 +1217,19 @@ def adaptive_oracle_step(wl, idx, per_layer, threads):
 
     def one(job):
         li, c = job
-        o = oracle.quantize_adaptive(Ws[li][c:c + 1], wl.bits[0], wl.k_max,
-                                     max_candidates=ADAPTIVE_ORACLE_CAP, refuse="mark")
-        return int(np.maximum(o["ncand"], 0).sum()) * wl.layers[li].d
+        oracle.quantize_adaptive(Ws[li][c:c + 1], wl.bits[0], wl.k_max,
+                                 max_candidates=ADAPTIVE_CAP, refuse="mark", piecewise=True)
+        return wl.layers[li].d * wl.k_max
 
     with ThreadPoolExecutor(max_workers=threads) as ex:
         return sum(ex.map(one, jobs))
 
 
 def run_adaptive(args, world, rank, local):
-    """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) on every short layer of the
-    workload (c4: the 17 depthwise layers, 9 weights per channel): mpq_quantize_layer_adaptive per
-    layer on a pool of streams; value = element-candidate evaluations (d x grid size, summed over
-    channels and points) per second."""
+    """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) on every layer of the workload:
+    mpq_quantize_layer_adaptive per layer on a pool of streams; value = weight-element-steps
+    (C d k_max summed over layers) per second.  One single-stream pass is timed first and the
+    number of timed steps is cut to fit ADAPTIVE_BUDGET_S."""
     import torch
     from paper_2002_09049_gb300 import _build, binding
     from paper_2002_09049_gb300 import dist as dist_helpers
@@ -1234,6 +1247,9 @@ def run_adaptive(args, world, rank, local):
     binding.load()
     wl = wlm.WORKLOADS[args.config]
     idx = adaptive_layers(wl)
+    if args.layers is not None:
+        keep = {int(x) for x in args.layers.split(",")}
+        idx = [li for li in idx if li in keep]
     layers = [wl.layers[li] for li in idx]
     bits, k_max = wl.bits[0], wl.k_max
     Whs = [torch.from_numpy(layer_inputs(wl, li)[0]).pin_memory() for li in idx]
@@ -1243,11 +1259,10 @@ def run_adaptive(args, world, rank, local):
              mk(torch.float32, (l.C, k_max + 1)), mk(torch.int64, (l.C, k_max))) for l in layers]
     hosts = [(torch.empty(o[0].shape, dtype=torch.int8, pin_memory=True),
               torch.empty(o[1].shape, dtype=torch.float32, pin_memory=True)) for o in outs]
-    order = sorted(range(len(layers)), key=lambda i: -layers[i].C)
+    order = sorted(range(len(layers)), key=lambda i: -layers[i].C * layers[i].d)
     streams = [torch.cuda.Stream(dev) for _ in range(max(1, args.streams))]
     main = torch.cuda.current_stream()
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
-
     def call(i, st):
         c, s_, r, n = outs[i]
         binding.mpq_quantize_layer_adaptive(Ws[i], bits, k_max, max_cand=ADAPTIVE_CAP, codes=c,
@@ -1273,18 +1288,33 @@ def run_adaptive(args, world, rank, local):
             e.record(st)
             main.wait_event(e)
 
-    for _ in range(args.warmup):
+    def one_stream():
+        a = torch.cuda.Event(enable_timing=True)
+        z = torch.cuda.Event(enable_timing=True)
+        flush.fill_(1.0)
+        a.record(main)
+        for i in order:
+            call(i, main)
+        z.record(main)
+        torch.cuda.synchronize()
+        return a.elapsed_time(z)
+
+    first_ms = one_stream()                     # also the first warm-up pass
+    steps = max(1, min(args.steps, int(ADAPTIVE_BUDGET_S * 1e3 / max(first_ms, 1e-3) / 2)))
+    warm = max(1, min(args.warmup, steps))
+    for _ in range(warm):
         step()
     torch.cuda.synchronize()
-    ncand = [int(o[3].sum().item()) for o in outs]
-    refused = sum(int((o[3] < 0).sum().item()) for o in outs)
-    units_per_step = sum(max(0, n) * l.d for n, l in zip(ncand, layers))
+    ncand = [o[3].cpu().numpy() for o in outs]
+    grid_points = int(sum(np.maximum(n, 0).sum() for n in ncand))
+    refused = int(sum((n < 0).sum() for n in ncand))
+    units_per_step = sum(l.C * l.d * k_max for l in layers)
     step_ms = []
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
-        for _ in range(args.steps):
+        for _ in range(steps):
             flush.fill_(1.0)
             a = torch.cuda.Event(enable_timing=True)
             z = torch.cuda.Event(enable_timing=True)
@@ -1293,48 +1323,46 @@ def run_adaptive(args, world, rank, local):
             z.record(main)
             torch.cuda.synchronize()
             step_ms.append(a.elapsed_time(z))
-    one_ms = []
-    for _ in range(args.steps):
-        flush.fill_(1.0)
-        a = torch.cuda.Event(enable_timing=True)
-        z = torch.cuda.Event(enable_timing=True)
-        a.record(main)
-        for i in order:
-            call(i, main)
-        z.record(main)
-        torch.cuda.synchronize()
-        one_ms.append(a.elapsed_time(z))
+    one_ms = [one_stream() for _ in range(steps)]
     if world > 1:
         torch.distributed.barrier()
     ms = dist_helpers.max_over_ranks(float(np.mean(step_ms)), device=dev)
     value = dist_helpers.aggregate_throughput(units_per_step, ms, world)
     t1 = float(np.mean(one_ms)) / 1e3
-    ach = 4.0 * units_per_step / t1 / 1e12
-    roofline = {"kernel": "adaptive_kernel (Algorithm 1 over the grid of Eq. 10, objective in "
-                          "double)", "bound": "alu", "achieved": ach, "peak": FP64_NOMINAL_TFLOPS,
-                "unit": "TFLOP/s (fp64)", "frac": ach / FP64_NOMINAL_TFLOPS, "traffic": None,
-                "peak_source": "nominal dense FP64 rate of the part (no measured FP64 peak)",
-                "timing": "every layer on one stream, CUDA events; achieved = 4 fp64 operations "
-                          "(multiply, subtract, square, add) per element and candidate / that time",
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peaks, _ = measured_peaks()
+    mhz = peaks.get("sm_max_mhz", 2070.0)
+    alu_peak = sms * ALU_LANES_PER_SM * mhz * 1e6 / 1e12
+    ach = sum(adaptive_ops(wl, l) for l in layers) / t1 / 1e12
+    roofline = {"kernel": "adaptive_kernel (Algorithm 1 over the grid of Eq. 10: code-level "
+                          "thresholds sorted, piecewise quadratic screened in fp32, settled in "
+                          "double)", "bound": "alu", "achieved": ach, "peak": alu_peak,
+                "unit": "Tlane-op/s", "frac": ach / alu_peak, "traffic": None,
+                "peak_source": f"{sms} SMs x {ALU_LANES_PER_SM} lanes x {mhz:.0f} MHz; "
+                               f"{ADAPTIVE_OPS_PER_THRESHOLD} lane operations per code-level "
+                               f"threshold (Qmax per element-step) + {ADAPTIVE_OPS_PER_ELEMENT} "
+                               "per element-step",
+                "timing": "every layer on one stream, CUDA events",
                 "single_stream_ms_per_step": t1 * 1e3}
-    out = {"metric": ADAPTIVE_METRIC, "value": value, "unit": UNIT, "n_gpus": world,
-           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
-           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+    out = {"metric": ADAPTIVE_METRIC, "value": value, "unit": ADAPTIVE_UNIT, "n_gpus": world,
+           "steps": steps, "warmup": warm, "ms_per_step": ms,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
            "data": "synthetic",
-           "config": {"workload": f"{args.config}: {wl.title}, layers of <= 64 weights per channel",
+           "config": {"workload": f"{args.config}: {wl.title}",
                       "op": "adaptive grid (Def. 1 + Eq. 10)", "layers": len(layers),
                       "channels": sum(l.C for l in layers), "bits": bits, "k_max": k_max,
-                      "eta": 2.0 ** -10, "max_cand": ADAPTIVE_CAP, "refused_steps": refused,
-                      "units_per_step": units_per_step,
+                      "eta": 2.0 ** -10, "grid_points_per_step": grid_points,
+                      "refused_steps": refused, "units_per_step": units_per_step,
+                      "first_pass_ms": first_ms,
                       "l2": "flushed between steps (512 MB write)", "streams": args.streams,
                       "parallelism": f"replicas x{world}"},
-           "roofline": roofline, "gpu_launches": len(layers) * args.steps,
+           "roofline": roofline, "gpu_launches": len(layers) * steps,
            "clocks": clk.summary()}
     if not args.no_e2e:
         step(host=True)
         torch.cuda.synchronize()
         times = []
-        for _ in range(args.steps):
+        for _ in range(steps):
             a = torch.cuda.Event(enable_timing=True)
             z = torch.cuda.Event(enable_timing=True)
             a.record(main)
@@ -1343,7 +1371,8 @@ def run_adaptive(args, world, rank, local):
             z.synchronize()
             times.append(a.elapsed_time(z))
         e_ms = float(np.mean(times))
-        out["e2e"] = {"value": units_per_step / (e_ms / 1e3), "unit": UNIT, "ms_per_step": e_ms,
+        out["e2e"] = {"value": units_per_step / (e_ms / 1e3), "unit": ADAPTIVE_UNIT,
+                      "ms_per_step": e_ms,
                       "h2d_bytes_per_step": int(sum(w.numel() * 4 for w in Whs)),
                       "d2h_bytes_per_step": int(sum(h[0].numel() + 4 * h[1].numel()
                                                     for h in hosts))}
@@ -1354,11 +1383,10 @@ def run_adaptive(args, world, rank, local):
         t0 = time.perf_counter()
         units = adaptive_oracle_step(wl, idx, per_layer, host_cores())
         dt = time.perf_counter() - t0
-        out["cpu_baseline"] = {"value": units / dt, "unit": UNIT, "cores": host_cores(),
+        out["cpu_baseline"] = {"value": units / dt, "unit": ADAPTIVE_UNIT, "cores": host_cores(),
                                "kind": "oracle", "seconds": dt,
-                               "sample": f"the first {per_layer} channels of every short layer "
-                                         f"(steps above {ADAPTIVE_ORACLE_CAP} candidates refused), "
-                                         "oracle threads over channels"}
+                               "sample": f"the first {per_layer} channels of every layer (the "
+                                         "oracle's piecewise search), threads over channels"}
     return out
 
 
@@ -1380,18 +1408,19 @@ def run_adaptive_reference(args, world, rank):
         units = adaptive_oracle_step(wl, idx, per_layer, host_cores())
         times.append(time.perf_counter() - t0)
     v = units / float(np.mean(times))
-    return {"impl": "reference", "metric": ADAPTIVE_METRIC, "value": v, "unit": UNIT, "n_gpus": 1,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(times)),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic",
-            "config": {"workload": f"{args.config}: {wl.title}, layers of <= 64 weights per channel",
+    return {"impl": "reference", "metric": ADAPTIVE_METRIC, "value": v, "unit": ADAPTIVE_UNIT,
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * float(np.mean(times)), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"{args.config}: {wl.title}",
                        "op": "adaptive grid (Def. 1 + Eq. 10)", "bits": wl.bits[0],
                        "k_max": wl.k_max},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
-                             "sample": f"the first {per_layer} channels of every short layer per "
-                                       f"step (steps above {ADAPTIVE_ORACLE_CAP} candidates "
-                                       "refused)"},
-            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+            "cpu_baseline": {"value": v, "unit": ADAPTIVE_UNIT, "cores": host_cores(),
+                             "kind": "oracle",
+                             "sample": f"the first {per_layer} channels of every layer per step "
+                                       "(the oracle's piecewise search)"},
+            "e2e": {"value": v, "unit": ADAPTIVE_UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
 
 
 def run_clip_reference(args, world, rank):

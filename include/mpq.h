@@ -16,9 +16,9 @@
  *    on the device that is current when the call is made, unless an argument says "host".
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Every call
  *    only enqueues work on `stream` and returns; results are ready when the stream reaches them.
- *    No entry point synchronizes, and none allocates device memory except mpq_output_error's
- *    small scratch buffer, which comes from the device's stream-ordered pool on `stream` and
- *    goes back to it on `stream` (see there).
+ *    No entry point synchronizes, and none allocates device memory except the scratch of
+ *    mpq_output_error and mpq_quantize_layer_adaptive, which comes from the device's
+ *    stream-ordered pool on `stream` and goes back to it on `stream` (see there).
  *  - Arguments are validated on the host before anything is enqueued; an invalid argument
  *    returns MPQ_ERR_INVALID_ARG / MPQ_ERR_UNSUPPORTED and leaves every output untouched.
  *    A failed kernel launch returns MPQ_ERR_CUDA.  mpq_last_error() gives a message for the
@@ -127,30 +127,35 @@ mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
                             const int8_t *codes, const float *scales, int C, int d, int k_max,
                             float *err, void *stream);
 
-/* Longest channel of mpq_quantize_layer_adaptive. */
-#define MPQ_ADAPTIVE_MAX_DIM 64
+/* Most code-level thresholds (d * Qmax) one step of mpq_quantize_layer_adaptive sorts. */
+#define MPQ_ADAPTIVE_MAX_THRESHOLDS 65536
 
 /*
  * mpq_quantize_layer_adaptive -- Algorithm 1 with the adaptive grid of Eq. 10 (Sec. 3.2,
- * Definition 1) instead of a fixed grid, for short channels (e.g. depthwise 3x3 filters).
- * Step i of channel k, with r = r_{k,i} (r_1 = w_k):
+ * Definition 1) instead of a fixed grid.  Step i of channel k, with r = r_{k,i} (r_1 = w_k):
  *   Delta = the minimal gap of r (Definition 1): half the smallest difference between two distinct
  *     element magnitudes |r_j| (the printed pair condition t_i != t_j read as |t_i| != |t_j|);
  *   gamma = min(Delta / Qmax, eta), or eta when r has fewer than two distinct magnitudes;
  *   grid search of a over I = [0, 2 Qmax ||r||] with step gamma (Eq. 10): a_m = m gamma for
- *     m = 1..M, M = floor(2 Qmax ||r|| / gamma) (double), as fp32 point scales s_m = fl(a_m / Qmax);
- *   codes, objective (double, index order), first minimiser and update as mpq_quantize_layer.
+ *     m = 1..M, M = floor(2 Qmax ||r|| / gamma) (double, ||r||^2 summed in index order), as fp32
+ *     point scales s_m = fl(a_m / Qmax);
+ *   codes as mpq_quantize_layer; the chosen m minimises ||r - s_m q||^2 (the first m on ties);
+ *   r <- fmaf(-s, q, r).
  * A zero residual gives a null point (scale 0, codes 0); so does a grid without candidates.
+ * The grid is not enumerated: the thresholds where each element's code changes are sorted and the
+ * objective, a quadratic in s between them, is minimised exactly; the work per step is
+ * O(d Qmax log(d Qmax)) whatever M is (Definition 1 makes M 1e8..1e10 on real channels).
  *
- *   W          [C][d] fp32; 1 <= d <= MPQ_ADAPTIVE_MAX_DIM.
+ *   W          [C][d] fp32; 1 <= d <= MPQ_MAX_DIM and d * Qmax <= MPQ_ADAPTIVE_MAX_THRESHOLDS.
  *   bits, k_max, codes, scales, resid_sq   as for mpq_quantize_layer (resid_sq nullable).
  *   eta        the largest grid step (the paper's experiments: 2^-10); finite, > 0.
- *   max_cand   the most candidates one step may enumerate (>= 1).  A step whose grid is larger
- *              is refused on the device: its scale and every later scale of that channel read NaN,
- *              their codes 0, and ncand holds -1 for it (0 for the later steps).
+ *   max_cand   the largest grid a step may have (>= 1).  A step whose grid is larger is refused on
+ *              the device: its scale and every later scale of that channel read NaN, their codes
+ *              0, and ncand holds -1 for it (0 for the later steps).
  *   ncand      out [C][k_max] int64, nullable: M of every step (0 for a null point).
- * Each step enumerates its whole grid (d M code evaluations); the grid grows as the minimal gap
- * shrinks, so long channels (hundreds of weights) are out of reach: MPQ_ERR_UNSUPPORTED.
+ * Scratch: the threshold lists, 16 d Qmax bytes per resident CTA (at most 2 per SM), come from the
+ * current device's stream-ordered pool on `stream` (as for mpq_output_error; MPQ_ERR_NOMEM if it
+ * has no room).
  */
 mpq_status mpq_quantize_layer_adaptive(const float *W, int C, int d, int bits, int k_max,
                                        double eta, long long max_cand, int8_t *codes,

@@ -74,8 +74,11 @@ def _load():
         lib.mpqo_multipoint_linear.restype = I
         lib.mpqo_minimal_gap.argtypes = [P, I, P]
         lib.mpqo_minimal_gap.restype = D
-        lib.mpqo_quantize_channel_adaptive.argtypes = [P, I, I, I, D, L, P, P, P, P, P, P, P, P, P, I]
+        lib.mpqo_quantize_channel_adaptive.argtypes = [P, I, I, I, D, L, P, P, P, P, P, P, P, P, P, I,
+                                                       P]
         lib.mpqo_quantize_channel_adaptive.restype = I
+        lib.mpqo_objective.argtypes = [P, I, I, ctypes.c_float, P]
+        lib.mpqo_objective.restype = D
         _lib = lib
     return _lib
 
@@ -129,28 +132,42 @@ def quantize_adaptive(W, bits: int, k_max: int, eta: float = ETA, max_candidates
     for grids too large to enumerate; ``second`` is NaN then.
 
     Returns a dict with codes [k_max][C][d] int8, scales [C][k_max] fp32, resid_sq [C][k_max+1],
-    gamma [C][k_max] (the a-grid step of each step), ncand [C][k_max], best/second [C][k_max]."""
+    gamma [C][k_max] (the a-grid step of each step), ncand [C][k_max], best/second [C][k_max],
+    rin [k_max][C][d] (the residual each step starts from)."""
     lib = _load()
     W = _c(W, np.float32)
     C, d = W.shape
     out = dict(codes=np.zeros((k_max, C, d), np.int8), scales=np.zeros((C, k_max), np.float32),
                resid_sq=np.zeros((C, k_max + 1), np.float64),
                gamma=np.zeros((C, k_max), np.float64), ncand=np.zeros((C, k_max), np.int64),
-               best=np.zeros((C, k_max), np.float64), second=np.zeros((C, k_max), np.float64))
+               best=np.zeros((C, k_max), np.float64), second=np.zeros((C, k_max), np.float64),
+               rin=np.zeros((k_max, C, d), np.float32))
     codes = np.zeros((k_max, d), np.int8)
+    rin = np.zeros((k_max, d), np.float32)
     r = np.empty(d, np.float32)
     work = np.empty(d, np.float64)
     for k in range(C):
         st = lib.mpqo_quantize_channel_adaptive(
             _p(W[k]), d, bits, k_max, float(eta), int(max_candidates), _p(codes),
             _p(out["scales"][k]), _p(out["resid_sq"][k]), _p(out["gamma"][k]), _p(out["ncand"][k]),
-            _p(out["best"][k]), _p(out["second"][k]), _p(r), _p(work), int(bool(piecewise)))
+            _p(out["best"][k]), _p(out["second"][k]), _p(r), _p(work), int(bool(piecewise)),
+            _p(rin))
         if st < -1:
             raise RuntimeError(f"channel {k}: the piecewise search failed ({st})")
         if st != 0 and refuse == "raise":
             raise ValueError(f"channel {k}: the adaptive grid exceeds {max_candidates} candidates")
         out["codes"][:, k, :] = codes
+        out["rin"][:, k, :] = rin
     return out
+
+
+def objective(r, bits: int, s: float):
+    """Eq. 9 at one fp32 scale by its definition: (||r - s [r/s]_Q||^2 in double, the codes)."""
+    lib = _load()
+    r = _c(r, np.float32).ravel()
+    q = np.zeros(r.size, np.int8)
+    E = lib.mpqo_objective(_p(r), r.size, bits, ctypes.c_float(np.float32(s)), _p(q))
+    return float(E), q
 
 
 def quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, channels=None,

@@ -370,6 +370,16 @@ static long adaptive_step_piecewise(const float *r, int d, int qmax, double gamm
     return bestm;
 }
 
+/* The objective of Eq. 9 at one scale s, by its definition (double, index order), and the codes
+ * q = [r/s]_Q it takes (Eq. 8; nullable).  Used to judge a scale another implementation chose. */
+double mpqo_objective(const float *r, int d, int bits, float s, int8_t *codes)
+{
+    const int qmax = qmax_of(bits);
+    if (codes)
+        for (int j = 0; j < d; ++j) codes[j] = (int8_t)nearest_code(r[j], s, qmax);
+    return candidate_error(r, d, s, qmax);
+}
+
 /* Algorithm 1 with the grid of Eq. 10 for one channel w, run to k_max points.  Each step i:
  * Delta = minimal gap of r_i (Definition 1), gamma = min(Delta / Qmax, eta) (gamma = eta when
  * Delta is infinite), and the search over a in I = [0, 2 Qmax ||r_i||] with step gamma: the
@@ -382,11 +392,12 @@ static long adaptive_step_piecewise(const float *r, int d, int qmax, double gamm
  * its scale and every later one NaN, codes 0, squared norms NaN, ncand -1 for it and 0 after;
  * returns -1 then, else 0.  piecewise = 0 enumerates every grid point; 1 takes the same decisions
  * through adaptive_step_piecewise (best holds the chosen objective, second is NaN), for grids too
- * large to enumerate (-2 if its guard trips).  r: scratch of d floats; work: scratch of d doubles. */
+ * large to enumerate (-2 if its guard trips).  r: scratch of d floats; work: scratch of d doubles;
+ * rin (nullable): [k_max][d], the residual each step starts from. */
 int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, double eta,
                                    long max_cand, int8_t *codes, float *scales, double *resid_sq,
                                    double *gamma, long *ncand, double *best, double *second,
-                                   float *r, double *work, int piecewise)
+                                   float *r, double *work, int piecewise, float *rin)
 {
     int qmax = qmax_of(bits);
     struct ad_event *ev = NULL;
@@ -413,6 +424,8 @@ int mpqo_quantize_channel_adaptive(const float *w, int d, int bits, int k_max, d
     int refused = 0;
     for (int i = 0; i < k_max; ++i) {
         int8_t *qi = codes + (long)i * d;
+        if (rin)
+            for (int j = 0; j < d; ++j) rin[(long)i * d + j] = r[j];
         double E1 = INFINITY, E2 = INFINITY, g = 0.0;
         long M = 0;
         float sbest = 0.0f;

@@ -21,7 +21,7 @@ MPQ_CENTER_PER_LAYER = 1
 MPQ_CLIP_PER_CHANNEL = 0
 MPQ_CLIP_PER_LAYER = 1
 MPQ_NOALLOC_RANGE_WORDS = 1 << 20     # the fixed scratch of mpq_output_error_noalloc
-MPQ_ADAPTIVE_MAX_DIM = 64             # the longest channel of mpq_quantize_layer_adaptive
+MPQ_ADAPTIVE_MAX_THRESHOLDS = 1 << 16  # most d * Qmax of mpq_quantize_layer_adaptive
 MPQ_TIMEOUT_OUTPUT_ERROR = 0x1        # timeout bits of mpq_device_status
 MPQ_TIMEOUT_CLIP = 0x2
 MPQ_TIMEOUT_INFERENCE = 0x4
@@ -168,8 +168,8 @@ ETA = 2.0 ** -10   # the largest grid step of the paper's experiments
 def mpq_quantize_layer_adaptive(W, bits: int, k_max: int, eta: float = ETA,
                                 max_cand: int = 10 ** 7, codes=None, scales=None, resid_sq=None,
                                 ncand=None, stream=None):
-    """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1) for short channels
-    (d <= MPQ_ADAPTIVE_MAX_DIM).  Returns (codes [k_max][C][d] int8, scales [C][k_max] fp32,
+    """Algorithm 1 with the adaptive grid of Eq. 10 (Definition 1), d * Qmax <=
+    MPQ_ADAPTIVE_MAX_THRESHOLDS.  Returns (codes [k_max][C][d] int8, scales [C][k_max] fp32,
     resid_sq [C][k_max+1] fp32, ncand [C][k_max] int64: each step's grid size, -1 if refused)."""
     _dev(W, "W", torch.float32)
     C, d = W.shape

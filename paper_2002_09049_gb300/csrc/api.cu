@@ -143,15 +143,17 @@ extern "C" mpq_status mpq_quantize_layer_adaptive(const float *W, int C, int d, 
     g_msg[0] = 0;
     mpq_status st = check_common(C, d, k_max);
     if (st != MPQ_OK) return st;
-    REQUIRE(d <= MPQ_ADAPTIVE_MAX_DIM, MPQ_ERR_UNSUPPORTED,
-            "d = %d exceeds MPQ_ADAPTIVE_MAX_DIM = %d (the adaptive grid is enumerated)", d,
-            MPQ_ADAPTIVE_MAX_DIM);
+    REQUIRE(d <= MPQ_MAX_DIM, MPQ_ERR_UNSUPPORTED, "d = %d exceeds MPQ_MAX_DIM = %d", d,
+            MPQ_MAX_DIM);
     REQUIRE(bits >= MPQ_MIN_BITS && bits <= MPQ_MAX_BITS,
             (bits > MPQ_MAX_BITS ? MPQ_ERR_UNSUPPORTED : MPQ_ERR_INVALID_ARG),
             "bits = %d outside [%d, %d]", bits, MPQ_MIN_BITS, MPQ_MAX_BITS);
     REQUIRE(isfinite(eta), MPQ_ERR_NONFINITE, "eta is not finite");
     REQUIRE(eta > 0.0, MPQ_ERR_INVALID_ARG, "eta = %g must be > 0", eta);
     REQUIRE(max_cand >= 1, MPQ_ERR_INVALID_ARG, "max_cand = %lld must be >= 1", max_cand);
+    REQUIRE((long long)d * ((1 << (bits - 1)) - 1) <= MPQ_ADAPTIVE_MAX_THRESHOLDS,
+            MPQ_ERR_UNSUPPORTED, "d * Qmax = %lld exceeds MPQ_ADAPTIVE_MAX_THRESHOLDS = %d",
+            (long long)d * ((1 << (bits - 1)) - 1), MPQ_ADAPTIVE_MAX_THRESHOLDS);
     if (C == 0) return MPQ_OK;
     REQUIRE(W && codes && scales, MPQ_ERR_INVALID_ARG, "W, codes and scales must be non-NULL");
     return launch_adaptive(W, C, d, (1 << (bits - 1)) - 1, k_max, eta, max_cand, codes, scales,

@@ -33,6 +33,10 @@ void set_error(const char *fmt, ...);
 // Maps a CUDA error to MPQ_ERR_CUDA (recording its text), cudaSuccess to MPQ_OK.
 mpq_status cuda_status(cudaError_t e, const char *what);
 
+// `bytes` of device scratch from the current device's default stream-ordered pool, allocated on
+// `stream` (free it with cudaFreeAsync on the same stream).  MPQ_ERR_NOMEM if the pool has no room.
+mpq_status pool_scratch(void **p, size_t bytes, cudaStream_t stream);
+
 // Multiprocessor count of the current device (cached per device).
 int sm_count();
 

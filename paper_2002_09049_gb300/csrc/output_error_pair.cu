@@ -678,37 +678,6 @@ pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const flo
     }
 }
 
-// Scratch of the fp16 contraction comes from the device's stream-ordered pool (allocated and
-// freed on the call's stream, so concurrent calls on other streams never share it; inside a CUDA
-// graph capture these become the graph's own allocation nodes).  Freed blocks stay cached in the
-// pool instead of going back to the driver at every synchronisation (set on the first call made
-// outside a stream capture, where a pool attribute may not be changed).
-mpq_status pair_scratch(void **p, size_t bytes, cudaStream_t stream)
-{
-    static std::atomic<int> pool_set{0};
-    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusActive;
-    if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) {
-        (void)cudaGetLastError();
-        cs = cudaStreamCaptureStatusActive;
-    }
-    if (cs == cudaStreamCaptureStatusNone && !pool_set.exchange(1)) {
-        int dev = 0;
-        cudaMemPool_t pool;
-        if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetDefaultMemPool(&pool, dev) == cudaSuccess) {
-            uint64_t keep = UINT64_MAX;
-            (void)cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
-        }
-        (void)cudaGetLastError();
-    }
-    const cudaError_t e = cudaMallocAsync(p, bytes, stream);
-    if (e == cudaErrorMemoryAllocation) {
-        (void)cudaGetLastError();
-        set_error("output error: no %zu bytes of scratch in the stream-ordered pool", bytes);
-        return MPQ_ERR_NOMEM;
-    }
-    return cuda_status(e, "scratch allocation (cudaMallocAsync)");
-}
-
 PFN_cuTensorMapEncodeTiled_v12000 pair_map_encoder()
 {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
@@ -817,7 +786,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     if constexpr (!CLIP) {
         // fp16 operands: the ranges of X and of every residual vector first
         if (!ext_range) {
-            mpq_status st = pair_scratch(reinterpret_cast<void **>(&range),
+            mpq_status st = pool_scratch(reinterpret_cast<void **>(&range),
                                          (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
             if (st != MPQ_OK) return st;
         }
@@ -846,6 +815,37 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
 }
 
 }  // namespace
+
+// Scratch (the fp16 contraction's range table, the adaptive grid's event lists) comes from the device's stream-ordered pool (allocated and
+// freed on the call's stream, so concurrent calls on other streams never share it; inside a CUDA
+// graph capture these become the graph's own allocation nodes).  Freed blocks stay cached in the
+// pool instead of going back to the driver at every synchronisation (set on the first call made
+// outside a stream capture, where a pool attribute may not be changed).
+mpq_status pool_scratch(void **p, size_t bytes, cudaStream_t stream)
+{
+    static std::atomic<int> pool_set{0};
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusActive;
+    if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) {
+        (void)cudaGetLastError();
+        cs = cudaStreamCaptureStatusActive;
+    }
+    if (cs == cudaStreamCaptureStatusNone && !pool_set.exchange(1)) {
+        int dev = 0;
+        cudaMemPool_t pool;
+        if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetDefaultMemPool(&pool, dev) == cudaSuccess) {
+            uint64_t keep = UINT64_MAX;
+            (void)cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        }
+        (void)cudaGetLastError();
+    }
+    const cudaError_t e = cudaMallocAsync(p, bytes, stream);
+    if (e == cudaErrorMemoryAllocation) {
+        (void)cudaGetLastError();
+        set_error("no %zu bytes of scratch in the stream-ordered pool", bytes);
+        return MPQ_ERR_NOMEM;
+    }
+    return cuda_status(e, "scratch allocation (cudaMallocAsync)");
+}
 
 bool output_error_pair_ok(const float *X, const float *W, const int8_t *codes, int d)
 {

@@ -104,7 +104,8 @@ def test_output_error_noalloc_validation(lib):
 
 
 @pytest.mark.parametrize("d,bits,eta,cap,status", [
-    (65, 4, 2.0 ** -10, 100, 3),          # longer than MPQ_ADAPTIVE_MAX_DIM
+    (8193, 4, 2.0 ** -10, 100, 3),        # longer than MPQ_MAX_DIM
+    (1024, 8, 2.0 ** -10, 100, 3),        # d * Qmax above MPQ_ADAPTIVE_MAX_THRESHOLDS
     (9, 9, 2.0 ** -10, 100, 3),           # bits above the limit
     (9, 1, 2.0 ** -10, 100, 1),
     (9, 4, 0.0, 100, 1),                  # eta must be > 0

@@ -753,3 +753,25 @@ def test_adaptive_piecewise_equals_enumeration(oracle):
         np.testing.assert_array_equal(a["resid_sq"], b["resid_sq"])
         np.testing.assert_array_equal(a["ncand"], b["ncand"])
         np.testing.assert_array_equal(a["best"], b["best"])
+
+
+@pytest.mark.parametrize("bits,d,seed", [(2, 4, 1), (3, 3, 2), (4, 3, 3)])
+def test_objective_is_the_best_code_vector(oracle, bits, d, seed):
+    """Eq. 9 at one scale (oracle.objective): its value is the smallest ||r - s q||^2 over every
+    code vector q in {-Qmax..Qmax}^d (exhaustive, exact rationals), and its codes attain it; an
+    r exactly on the lattice s Z gives 0 and those integers."""
+    qmax = 2 ** (bits - 1) - 1
+    rng = np.random.default_rng(seed)
+    for _ in range(20):
+        r = rng.standard_normal(d).astype(np.float32)
+        s = np.float32(abs(rng.standard_normal()) * 0.7 + 0.05)
+        E, q = oracle.objective(r, bits, s)
+        best = min(sum((Fraction(float(x)) - Fraction(float(s)) * c) ** 2 for x, c in zip(r, qq))
+                   for qq in itertools.product(range(-qmax, qmax + 1), repeat=d))
+        got = sum((Fraction(float(x)) - Fraction(float(s)) * int(c)) ** 2 for x, c in zip(r, q))
+        assert got == best
+        assert abs(E - float(best)) <= 1e-12 * max(1.0, float(best))
+    s = np.float32(0.375)
+    ints = np.array([3, -1, 0, 2][:d], np.int64).clip(-qmax, qmax)
+    E, q = oracle.objective((ints * s).astype(np.float32), bits, s)
+    assert E == 0.0 and np.array_equal(q, ints)
