@@ -81,28 +81,28 @@ __device__ __forceinline__ float ad_threshold(float a, int L)
     return s;
 }
 
-// Smallest m in [lo, M] with s_m >= x (ge) or s_m > x (!ge); M + 1 if none.  s_m is
-// non-decreasing in m; the start x Qmax / gamma is within 2^-22 (relative) of the answer, which
-// is then bracketed and bisected on exact s_m values (at most ~40 of them for M < 2^40).
-__device__ long long ad_first_m(double x, bool ge, long long lo, long long M, double gamma, int qmax)
+// Smallest m in [lo, M] with s_m >= f (an fp32 value); M + 1 if none.  s_m = fl32(y_m) is
+// non-decreasing in m and reaches f once y_m passes the midpoint between f's predecessor and f,
+// which y_m = m gamma / Qmax (1 + O(2^-52)) crosses within a couple of indices of
+// midpoint * Qmax / gamma: the answer is bracketed there by two exact s_m and bisected (about
+// five exact scales in all); a failed bracket falls back to bisecting [lo, M].
+__device__ long long ad_first_m_ge(float f, long long lo, long long M, double gamma, int qmax)
 {
-    auto ok = [&](long long m) {
-        const double s = (double)ad_scale(m, gamma, qmax);
-        return ge ? s >= x : s > x;
-    };
+    auto ok = [&](long long m) { return ad_scale(m, gamma, qmax) >= f; };
     if (lo > M) return M + 1;
     if (ok(lo)) return lo;
     if (!ok(M)) return M + 1;
-    // ok(lo) false, ok(M) true: bracket (a, b] around the estimate
-    const double est = __dmul_rn(x, __ddiv_rn((double)qmax, gamma));
-    long long a = lo, b = M;
+    long long a = lo, b = M;   // ok(a) false, ok(b) true
+    const double h = 0.5 * ((double)nextafterf(f, 0.0f) + (double)f);   // exact
+    const double est = __dmul_rn(h, __ddiv_rn((double)qmax, gamma));
     if (est > (double)lo && est < (double)M) {
-        const long long w = (long long)(est * 0x1p-21) + 4;
         const long long c = (long long)est;
-        const long long a2 = c - w > lo ? c - w : lo;
-        const long long b2 = c + w < M ? c + w : M;
-        if (!ok(a2)) a = a2;
-        if (ok(b2)) b = b2;
+        const long long a2 = c - 2 > lo ? c - 2 : lo;
+        const long long b2 = c + 3 < M ? c + 3 : M;
+        if (!ok(a2) && ok(b2)) {
+            a = a2;
+            b = b2;
+        }
     }
     for (int it = 0; it < 80 && b - a > 1; ++it) {
         const long long mid = a + (b - a) / 2;
@@ -111,6 +111,14 @@ __device__ long long ad_first_m(double x, bool ge, long long lo, long long M, do
     return b;
 }
 
+// the smallest fp32 value >= x, and the one after the fp32 value x
+__device__ __forceinline__ float ad_ceil_f(double x)
+{
+    float f = __double2float_rn(x);
+    if ((double)f < x) f = nextafterf(f, INFINITY);
+    return f;
+}
+__device__ __forceinline__ float ad_next_f(float x) { return nextafterf(x, INFINITY); }
 
 // ---- CTA-wide building blocks (all AT threads call them) -------------------------------------
 struct ASort {
@@ -241,8 +249,18 @@ __device__ __forceinline__ double ad_decision(float s, long long Pfix, long long
     return __dmul_rn(sd, __fma_rn(sd, (double)N, -2.0 * ((double)Pfix * down)));
 }
 
+constexpr int A_LIST = 512;   // candidate pieces settled by the whole CTA
+
+struct APiece {
+    float lo, hi;
+    long long P, N;
+};
+
 struct AShared {
     ASort sort;
+    APiece list[A_LIST];
+    int nlist;
+    int finite;
     double r2;                  // ||r||^2, double, index order
     double gamma;
     long long M, mpos;
@@ -294,9 +312,9 @@ __device__ bool ad_settle_piece(float lo, float hi, long long Pfix, long long N,
                                 double gamma, int qmax, long long mpos, long long M, double &D,
                                 float &s)
 {
-    const long long m1 = ad_first_m((double)lo, false, mpos, M, gamma, qmax);
+    const long long m1 = ad_first_m_ge(ad_next_f(lo), mpos, M, gamma, qmax);
     if (m1 > M) return false;
-    const long long m2 = ad_first_m((double)hi, false, m1, M, gamma, qmax) - 1;
+    const long long m2 = ad_first_m_ge(ad_next_f(hi), m1, M, gamma, qmax) - 1;
     if (m1 > m2) return false;
     if (N == 0) {   // every code 0: D = 0 on the whole piece, its smallest scale first
         D = 0.0;
@@ -304,7 +322,7 @@ __device__ bool ad_settle_piece(float lo, float hi, long long Pfix, long long N,
         return true;
     }
     const double sbar = __ddiv_rn((double)Pfix * down, (double)N);
-    long long mb = ad_first_m(sbar, true, m1, m2, gamma, qmax);
+    long long mb = ad_first_m_ge(ad_ceil_f(sbar), m1, m2, gamma, qmax);
     if (mb > m2) mb = m2;
     const long long ma = mb > m1 ? mb - 1 : m1;
     const float sa = ad_scale(ma, gamma, qmax), sb = ad_scale(mb, gamma, qmax);
@@ -334,6 +352,23 @@ __device__ __forceinline__ float ad_piece_lb(float lo, float hi, float Pn, float
 }
 
 
+// sum_j x_j in double, in index order, one rounding per addition (the definition's ||r||^2 once
+// the exact squares are in x); the loads run ahead of the dependent additions
+__device__ __forceinline__ double ad_serial_sum(const double *__restrict__ x, int d)
+{
+    double s = 0.0;
+    int j = 0;
+    for (; j + 8 <= d; j += 8) {
+        double v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = x[j + u];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) s = __dadd_rn(s, v[u]);
+    }
+    for (; j < d; ++j) s = __dadd_rn(s, x[j]);
+    return s;
+}
+
 __global__ void __launch_bounds__(AT, A_CTAS_PER_SM)
 adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, double eta,
                 long long max_cand, int hbits, int8_t *__restrict__ codes,
@@ -345,21 +380,26 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
     const int t = threadIdx.x, lane = t & 31, w = t >> 5;
     uint2 *bufA = scratch + (size_t)blockIdx.x * 2 * cap;
     uint2 *bufB = bufA + cap;
+    double *sq = reinterpret_cast<double *>(bufB);   // r_j^2 for the serial sum (cap >= d)
     const size_t plane = (size_t)C * d;
 
     for (int k = blockIdx.x; k < C; k += gridDim.x) {
-        for (int j = t; j < d; j += AT) r[j] = W[(size_t)k * d + j];
+        if (t == 0) sh.finite = 1;
+        __syncthreads();
+        int fin = 1;
+        for (int j = t; j < d; j += AT) {
+            const float v = W[(size_t)k * d + j];
+            r[j] = v;
+            sq[j] = __dmul_rn((double)v, (double)v);   // exact: 24-bit times 24-bit
+            fin &= isfinite(v);
+        }
+        if (!fin) atomicAnd(&sh.finite, 0);
         __syncthreads();
         if (t == 0) {
-            double r2 = 0.0;
-            int finite = 1;
-            for (int j = 0; j < d; ++j) {
-                finite &= isfinite(r[j]);
-                r2 = __dadd_rn(r2, __dmul_rn((double)r[j], (double)r[j]));
-            }
+            const double r2 = ad_serial_sum(sq, d);
             sh.r2 = r2;
-            sh.state = finite ? 0 : 2;
-            if (resid_sq) resid_sq[(size_t)k * (k_max + 1)] = finite ? (float)r2 : NAN;
+            sh.state = sh.finite ? 0 : 2;
+            if (resid_sq) resid_sq[(size_t)k * (k_max + 1)] = sh.finite ? (float)r2 : NAN;
         }
         __syncthreads();
         bool dead = sh.state == 2;
@@ -375,6 +415,7 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                     sh.lbkey = ~0ull;
                     sh.dkey = ~0ull;
                     sh.skey = ~0u;
+                    sh.nlist = 0;
                 }
                 __syncthreads();
                 unsigned am = 0u;
@@ -417,7 +458,7 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                             sh.M = M;
                             sh.state = 1;
                             if (M > 0) {
-                                const long long mp = ad_first_m(0.0, false, 1, M, g, qmax);
+                                const long long mp = ad_first_m_ge(ad_next_f(0.0f), 1, M, g, qmax);
                                 sh.mpos = mp;
                                 sh.U = mp > 1 ? 0.0 : INFINITY;
                                 if (mp <= M) {
@@ -569,15 +610,33 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                             const float lb = ad_piece_lb(lo, hi, (float)P * pscale, (float)N, e);
                             double D;
                             float sv;
-                            if (lb <= Uf &&
-                                ad_settle_piece(lo, hi, P, N, down, gamma, qmax, mpos, M, D, sv) &&
-                                (!have || D < bD || (D == bD && sv < bS))) {
-                                bD = D;
-                                bS = sv;
-                                have = true;
+                            if (lb <= Uf) {
+                                const int slot = atomicAdd(&sh.nlist, 1);
+                                if (slot < A_LIST) {
+                                    sh.list[slot] = APiece{lo, hi, P, N};
+                                } else if (ad_settle_piece(lo, hi, P, N, down, gamma, qmax, mpos, M,
+                                                           D, sv) &&
+                                           (!have || D < bD || (D == bD && sv < bS))) {
+                                    bD = D;   // beyond the list: settled by its own thread
+                                    bS = sv;
+                                    have = true;
+                                }
                             }
                         }
                         advance(x, cp, cn);
+                    }
+                }
+                __syncthreads();
+                // the queued pieces, spread over the CTA (neighbouring pieces share a thread above)
+                for (int x = t; x < min(sh.nlist, A_LIST); x += AT) {
+                    const APiece pc = sh.list[x];
+                    double D;
+                    float sv;
+                    if (ad_settle_piece(pc.lo, pc.hi, pc.P, pc.N, down, gamma, qmax, mpos, M, D, sv) &&
+                        (!have || D < bD || (D == bD && sv < bS))) {
+                        bD = D;
+                        bS = sv;
+                        have = true;
                     }
                 }
                 const unsigned long long dk = have ? ad_ordered(bD) : ~0ull;
@@ -593,14 +652,15 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                 int q = ad_code_mag(fabsf(v), sbest, qmax);
                 q = v < 0.0f ? -q : q;
                 qi[j] = (int8_t)q;
-                r[j] = __fmaf_rn(-sbest, (float)q, v);
+                const float nv = __fmaf_rn(-sbest, (float)q, v);
+                r[j] = nv;
+                sq[j] = __dmul_rn((double)nv, (double)nv);
             }
             __syncthreads();
             if (t == 0) {
                 scales[(size_t)k * k_max + i] = sbest;
                 if (ncand) ncand[(size_t)k * k_max + i] = sh.M;
-                double r2 = 0.0;
-                for (int j = 0; j < d; ++j) r2 = __dadd_rn(r2, __dmul_rn((double)r[j], (double)r[j]));
+                const double r2 = ad_serial_sum(sq, d);
                 sh.r2 = r2;
                 if (resid_sq) resid_sq[(size_t)k * (k_max + 1) + i + 1] = (float)r2;
             }
