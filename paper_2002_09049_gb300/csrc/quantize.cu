@@ -63,8 +63,12 @@ struct Grid<true> {
     __device__ __forceinline__ float frac(int g0, int) const { return gf.f[g0]; }
 };
 
-// Per-group scratch for cross-warp reductions.
+constexpr int QNEAR = 128;   // lattice-adjacent elements a group queues per step
+
+// Per-group scratch for cross-warp reductions, and the queue of lattice-adjacent elements.
 struct Scratch {
+    float nearq[QNEAR];
+    int nq;
     float f[8];
     float v[8];
     unsigned long long key[8];
@@ -76,24 +80,21 @@ struct Scratch {
     int flag[8];
 };
 
-// Shared memory: a CTA-wide table of the grid fractions f_g and fl(1/f_g) (2G words), then per
+// Shared memory: a CTA-wide table of the grid fractions f_g and fl(1/f_g) (2G words; left out on
+// the linear grid when that fits one more CTA per SM, f_g then computed where needed), then per
 // channel group (all 4-byte words): `copies` copies of hLo[G+1], hHi[G+1] (64-bit P bins as two
 // words) and hN[G+1], then r[d].  Without the lattice every warp has a private copy (so warps
 // never contend on a bin); with the lattice form (below) events are rare and the group shares one
-// copy, and the group also holds nb lattice buckets first: 64-bit R sums (2 words each) and
-// 32-bit counts.  Group regions are kept 8-byte aligned.  When it fits one more CTA per SM, the
-// lattice form on the linear grid leaves the table out (computing f_g where needed) and packs its
-// counts into 16 bits, two per word (a count never exceeds d <= 8192).
-__host__ __device__ constexpr size_t lattice_words(int nb, bool packed = false)
-{
-    return packed ? ((size_t)2 * nb + (size_t)(nb + 1) / 2 + 1) & ~(size_t)1
-                  : ((size_t)3 * nb + 1) & ~(size_t)1;
-}
+// copy, and the group also holds nb lattice buckets first, two words each: the low 32 bits of the
+// bucket's fixed-point R sum, and its high bits plus the bucket's element count shifted to bit
+// cnt_bit (the launcher checks that neither field can overflow).  (Two separate word arrays, low
+// words on all 32 banks, measured no faster.)  Group regions stay 8-byte
+// aligned.
+__host__ __device__ constexpr size_t lattice_words(int nb) { return (size_t)2 * nb; }
 
-__host__ __device__ constexpr size_t group_words(int G, int d, int copies, int nb,
-                                                 bool packed = false)
+__host__ __device__ constexpr size_t group_words(int G, int d, int copies, int nb)
 {
-    return lattice_words(nb, packed) + (((size_t)3 * (G + 1) * copies + (size_t)d + 1) & ~(size_t)1);
+    return lattice_words(nb) + (((size_t)3 * (G + 1) * copies + (size_t)d + 1) & ~(size_t)1);
 }
 
 template <int WPC>
@@ -432,7 +433,8 @@ template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
 __global__ void __launch_bounds__(QTHREADS, 4)
 quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, const Grid<CUSTOM> grid,
                 int k_max, int8_t *__restrict__ codes, float *__restrict__ scales,
-                float *__restrict__ resid_sq, float *__restrict__ residuals, int hbits)
+                float *__restrict__ resid_sq, float *__restrict__ residuals, int hbits,
+                int lat_bits, int cnt_bit)
 {
     const int nb = LAT ? 2 * G * qmax + 1 : 0;   // lattice buckets: floor(2u) in [0, 2 G Qmax]
     constexpr int NT = WPC * 32;
@@ -463,12 +465,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
     if (k >= C) return;   // whole group idle (group-uniform)
 
     unsigned int *gl = reinterpret_cast<unsigned int *>(ftab + (TABLE ? 2 * G : 0)) +
-                       (size_t)grp * group_words(G, d, COPIES, nb, !TABLE);
-    unsigned long long *latR = reinterpret_cast<unsigned long long *>(gl);   // [nb]
-    // bucket counts: 32-bit, or 16-bit two per word without the table
-    using Count = typename std::conditional<TABLE, unsigned int, unsigned short>::type;
-    Count *latC = reinterpret_cast<Count *>(gl + 2 * (size_t)nb);           // [nb]
-    unsigned int *gbase = gl + lattice_words(nb, !TABLE);
+                       (size_t)grp * group_words(G, d, COPIES, nb);
+    unsigned int *lat = gl;                         // [nb][2]: R low word, R high | count
+    const unsigned cnt_one = 1u << cnt_bit, hmask = cnt_one - 1u;
+    unsigned int *gbase = gl + lattice_words(nb);
     // this warp's private bins; copy 0 receives the merged suffix sums
     unsigned int *hLo = gbase + (size_t)(COPIES > 1 ? gw : 0) * 3 * (G + 1);
     unsigned int *hHi = hLo + (G + 1);
@@ -481,10 +481,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
 
     const size_t plane = (size_t)C * d;
     const float *w = W + (size_t)k * d;
+    const bool short_share = d <= 64 * NT;
     // rows this short take every candidate directly: G*d code evaluations per step cost less than
     // the lattice's per-step clears, scans and fold over its 2 G Qmax + 1 buckets
     const bool direct = d <= QDIRECT_MAX_D;
-    const float pscale = ldexpf(1.0f, hbits - 62);   // P * 2^-S / 2^e for the fp32 screen
 
     int bad = 0;
     float ssum = 0.0f, scomp = 0.0f, am = 0.0f;
@@ -524,7 +524,11 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             const float ism = __frcp_rn(smax);
             int e;
             frexpf(m, &e);                      // m < 2^e
-            const int S = 62 - e - hbits;       // sum_j R_j c_j < 2^62
+            // fixed point R = |r| 2^S: on the lattice, exact for every |r| that can reach bucket 1
+            // (|r| >= smax / 2G) and below 2^lat_bits; elsewhere sum_j R_j c_j < 2^62
+            const bool zs = __fmul_rn(fg(0), smax) == 0.0f;
+            const int S = (LAT && !zs) ? lat_bits - e : 62 - e - hbits;
+            const float pscale = ldexpf(1.0f, -S - e);   // P 2^-S / 2^e for the fp32 screen
             const double down = pow2d(-S);
             const float smax_e = ldexpf(smax, -e);   // smax / 2^e for the fp32 screen
             if (!direct) {
@@ -533,11 +537,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     hHi[t] = 0u;
                     hN[t] = 0;
                 }
-                if (LAT)
-                    for (int t = gt; t < nb; t += NT) {
-                        latR[t] = 0ull;
-                        latC[t] = 0;
-                    }
+                if (LAT) {
+                    for (int t = gt; t < 2 * nb; t += NT) lat[t] = 0u;
+                    if (gt == 0) sc.nq = 0;
+                }
                 gsync<WPC>(grp);
             }
             const bool zero_scale = __fmul_rn(fg(0), smax) == 0.0f;   // s_g increases with g
@@ -552,6 +555,49 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 long long Pb = 0;
                 long long Nb = 0;
                 // every level an element crosses inside the grid, one event each
+                // the event of level L of an element (c_lo < L <= c_hi): the first g whose code is
+                // below L, estimated where s_g crosses a/(L - 1/2), then settled with the exact
+                // rule (level_held is monotone in g)
+                auto event_level = [&](const float a, const int L, const unsigned int Rlo,
+                                       const unsigned int Rhi, const float ag) {
+                    int T;
+                    if (CUSTOM) {
+                        const float f_est = a * s_hinv[L] * ism;
+                        int lo = 1, hi = G - 1;
+                        while (lo < hi) {
+                            const int mid = (lo + hi) >> 1;
+                            if (fg(mid) < f_est) lo = mid + 1; else hi = mid;
+                        }
+                        T = lo;
+                    } else {
+                        // s_g = (g+1)/G * smax up to two fp32 roundings and x is a*G/(smax*h)
+                        // up to 2^-22, so unless x is within 2^-20 x of an integer, level L
+                        // is held exactly for g + 1 < x: T = floor(x) with no further check.
+                        const float x = ag * s_hinv[L];
+                        const float fx = floorf(x);
+                        const float tolx = MPQ_FAST_REL * x;
+                        T = (int)fminf(fmaxf(fx, 1.0f), (float)(G - 1));
+                        if (x - fx > tolx && fx + 1.0f - x > tolx && fx >= 1.0f &&
+                            fx <= (float)(G - 1)) {
+                            add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
+                            return;
+                        }
+                    }
+#define MPQ_HELD(t) level_held(a, __fmul_rn(fg(t), smax), fi(t) * ism, L)
+                    const bool up = (T < G - 1) && MPQ_HELD(T);
+                    const bool dn = !up && (T > 1) && !MPQ_HELD(T - 1);
+                    if (up) {
+                        ++T;
+                        while (T < G - 1 && MPQ_HELD(T)) ++T;
+                    } else if (dn) {
+                        --T;
+                        while (T > 1 && !MPQ_HELD(T - 1)) --T;
+                    }
+#undef MPQ_HELD
+                    add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
+                };
+                // every level an element crosses inside the grid, one event each; the levels held
+                // at the largest scale go to the base sums
                 auto events = [&](const float a) {
                     const int c_hi = code_fast(a, s0, i0, qmaxf);
                     if (c_hi == 0) return;   // code 0 at every scale: no contribution
@@ -562,46 +608,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     const unsigned int Rlo = (unsigned int)R;
                     const unsigned int Rhi = (unsigned int)((unsigned long long)R >> 32);
                     const float ag = a * g_per_a;
-                    for (int L = c_lo + 1; L <= c_hi; ++L) {
-                        // first g whose code is below L: estimate where s_g crosses a/(L - 1/2),
-                        // then settle with the exact rule (level_held is monotone in g)
-                        int T;
-                        if (CUSTOM) {
-                            const float f_est = a * s_hinv[L] * ism;
-                            int lo = 1, hi = G - 1;
-                            while (lo < hi) {
-                                const int mid = (lo + hi) >> 1;
-                                if (fg(mid) < f_est) lo = mid + 1; else hi = mid;
-                            }
-                            T = lo;
-                        } else {
-                            // s_g = (g+1)/G * smax up to two fp32 roundings and x is a*G/(smax*h)
-                            // up to 2^-22, so unless x is within 2^-20 x of an integer, level L
-                            // is held exactly for g + 1 < x: T = floor(x) with no further check.
-                            const float x = ag * s_hinv[L];
-                            const float fx = floorf(x);
-                            const float tolx = MPQ_FAST_REL * x;
-                            T = (int)fminf(fmaxf(fx, 1.0f), (float)(G - 1));
-                            if (x - fx > tolx && fx + 1.0f - x > tolx && fx >= 1.0f &&
-                                fx <= (float)(G - 1)) {
-                                add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
-                                continue;
-                            }
-                        }
-#define MPQ_HELD(t) level_held(a, __fmul_rn(fg(t), smax), fi(t) * ism, L)
-                        const bool up = (T < G - 1) && MPQ_HELD(T);
-                        const bool dn = !up && (T > 1) && !MPQ_HELD(T - 1);
-                        if (up) {
-                            ++T;
-                            while (T < G - 1 && MPQ_HELD(T)) ++T;
-                        } else if (dn) {
-                            --T;
-                            while (T > 1 && !MPQ_HELD(T - 1)) --T;
-                        }
-#undef MPQ_HELD
-                        add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
-                    }
+                    for (int L = c_lo + 1; L <= c_hi; ++L) event_level(a, L, Rlo, Rhi, ag);
                 };
+                // 2u within 2^-20 (relative) of an integer: its bucket is not decided exactly
+                auto near_lattice = [](float x) { return !(fabsf(x - rintf(x)) > MPQ_FAST_REL * x); };
                 if (direct) {
                     // Short rows: every candidate's P_g and N_g straight from the codes, exact
                     // (the codes as the update emits them; P in the same fixed point), into the
@@ -637,24 +647,52 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
 #pragma unroll
                         for (int u = 0; u < U; ++u) {
                             if (av[u] == 0.0f) continue;
-                            if (fabsf(u2[u] - rintf(u2[u])) > MPQ_FAST_REL * u2[u]) {
+                            if (!near_lattice(u2[u])) {
                                 const int b = (int)floorf(u2[u]);
                                 if (b >= 1) {
                                     const int bb = b < nb - 1 ? b : nb - 1;
-                                    // two 32-bit atomics: measurably cheaper than one 64-bit
+                                    // two 32-bit atomics: the low word's old value gives
+                                    // its carry, which the high word takes with the count
                                     const unsigned long long R =
                                         (unsigned long long)fixed_point(av[u], S);
-                                    unsigned int *Rw = reinterpret_cast<unsigned int *>(&latR[bb]);
-                                    add64(&Rw[0], &Rw[1], (unsigned int)R, (unsigned int)(R >> 32));
-                                    if (TABLE)
-                                        atomicAdd(reinterpret_cast<unsigned int *>(latC) + bb, 1u);
-                                    else   // 16-bit count in its word (no carry: count <= d)
-                                        atomicAdd(reinterpret_cast<unsigned int *>(latC) + (bb >> 1),
-                                                  1u << ((bb & 1) * 16));
+                                    const unsigned Rlo = (unsigned)R;
+                                    const unsigned old = atomicAdd(&lat[2 * bb], Rlo);
+                                    atomicAdd(&lat[2 * bb + 1], (unsigned)(R >> 32) +
+                                                                    (old + Rlo < old ? 1u : 0u) +
+                                                                    cnt_one);
                                 }
                             } else {
-                                events(av[u]);
+                                // within 2^-20 of a lattice point: queued, and settled level by
+                                // level by the whole group after the pass, so that one lane's
+                                // exact rule holds neither its warp nor the loop's registers
+                                const int slot = atomicAdd(&sc.nq, 1);
+                                if (slot < QNEAR) sc.nearq[slot] = av[u];
                             }
+                        }
+                    }
+                    gsync<WPC>(grp);
+                    const int nq = sc.nq;
+                    if (nq <= QNEAR) {
+                        // (queued element, level) pairs over the group's threads
+                        for (int it = gt; it < nq * qmax; it += NT) {
+                            const int q = it / qmax, L = it - q * qmax + 1;
+                            const float a = sc.nearq[q];
+                            const int c_hi = code_fast(a, s0, i0, qmaxf);
+                            if (c_hi == 0) continue;
+                            const int c_lo = code_fast(a, sG, iG, qmaxf);
+                            const long long R = fixed_point(a, S);
+                            if (L == 1) {
+                                Pb += R * (long long)c_lo;
+                                Nb += (long long)c_lo * c_lo;
+                            }
+                            if (L > c_lo && L <= c_hi)
+                                event_level(a, L, (unsigned int)R,
+                                            (unsigned int)((unsigned long long)R >> 32), a * g_per_a);
+                        }
+                    } else {   // the queue overflowed (never seen): every such element again
+                        for (int j = gt; j < d; j += NT) {
+                            const float a = fabsf(sr[j]);
+                            if (a != 0.0f && near_lattice(2.0f * (a * g_per_a))) events(a);
                         }
                     }
                 } else {
@@ -687,12 +725,13 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     mN[t] = (int)q;
                 };
                 auto lat_load = [&](int t, unsigned long long &p, long long &q) {
-                    p = latR[t];
-                    q = latC[t];
+                    const unsigned hi = lat[2 * t + 1];
+                    p = ((unsigned long long)(hi & hmask) << 32) | lat[2 * t];
+                    q = hi >> cnt_bit;
                 };
                 auto lat_store = [&](int t, unsigned long long p, long long q) {
-                    latR[t] = p;
-                    latC[t] = (Count)q;
+                    lat[2 * t] = (unsigned)p;
+                    lat[2 * t + 1] = (unsigned)(p >> 32) | ((unsigned)q << cnt_bit);
                 };
                 // with the lattice: warp 0 scans the bins while the other warps scan the lattice
                 // together (named barrier 8 + grp: gsync takes 0 or 1..4), or one warp both;
@@ -720,8 +759,9 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                         long long n = mN[g + 1];
                         for (int L = 1; L <= qmax; ++L) {
                             const int b = (g + 1) * (2 * L - 1);
-                            p += (long long)latR[b];
-                            n += (long long)(2 * L - 1) * latC[b];
+                            const unsigned hi = lat[2 * b + 1];
+                            p += (long long)(((unsigned long long)(hi & hmask) << 32) | lat[2 * b]);
+                            n += (long long)(2 * L - 1) * (hi >> cnt_bit);
                         }
                         mLo[g + 1] = (unsigned int)p;
                         mHi[g + 1] = (unsigned int)((unsigned long long)p >> 32);
@@ -802,7 +842,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             qi[j] = (int8_t)q;
             sr[j] = v;
             if (ri) ri[j] = v;
-            kahan_add(ssum, scomp, v * v);
+            // ||r||^2: a thread's share of at most 64 squares summed plainly (relative error
+            // below 2^-18 with the group's tree), longer shares compensated
+            if (short_share) ssum = __fmaf_rn(v, v, ssum);
+            else kahan_add(ssum, scomp, v * v);
             am = fmaxf(am, fabsf(v));
         }
         if (gt == 0) scales[(size_t)k * k_max + i] = s_best;
@@ -822,17 +865,37 @@ int ceil_log2(long long x)
     return b;
 }
 
+// Bit layout of the lattice buckets (2 G Qmax + 1 of them): R = |r| 2^S < 2^lat_bits, exact for
+// every |r| >= smax / 2G (the smallest magnitude that reaches bucket 1: its exponent is at least
+// e - 2 - ceil(log2(2 G Qmax)) for max|r| < 2^e, so 25 + that many bits hold its mantissa, one
+// more for margin); a bucket's high word holds its R sum's high part plus carries (at most
+// d 2^(lat_bits - 32) + d) below bit cnt_bit and its count (at most d) above.  Returns false when
+// the two fields do not fit one word (the event form runs then).
+struct LatBits {
+    int lat_bits, cnt_bit;
+};
+
+bool lattice_bits(int d, int qmax, int G, LatBits *lb)
+{
+    lb->lat_bits = 26 + ceil_log2(2LL * G * qmax);
+    const long long hi_part = lb->lat_bits > 32 ? (1LL << (lb->lat_bits - 32)) - 1 : 0;
+    const long long hi_max = (long long)d * hi_part + d;
+    lb->cnt_bit = ceil_log2(hi_max + 1);
+    return lb->cnt_bit + ceil_log2((long long)d + 1) <= 32;
+}
+
 template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
 mpq_status launch_wpc(const float *W, int C, int d, int qmax, int G, const Grid<CUSTOM> &grid,
                       int k_max, int8_t *codes, float *scales, float *resid_sq, float *residuals,
-                      int hbits, size_t smem, cudaStream_t stream)
+                      int hbits, LatBits lb, size_t smem, cudaStream_t stream)
 {
     constexpr int GPC = 8 / WPC;
     cudaError_t e = cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e == cudaSuccess) {
         quantize_kernel<WPC, CUSTOM, LAT, TABLE><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
-            W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, hbits);
+            W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, hbits, lb.lat_bits,
+            lb.cnt_bit);
         e = cudaGetLastError();
     }
     return cuda_status(e, "quantize kernel launch");
@@ -855,26 +918,25 @@ int quantize_ctas_per_sm(size_t smem)
 template <int WPC, bool CUSTOM>
 mpq_status launch_lat(bool lat, const float *W, int C, int d, int qmax, int G,
                       const Grid<CUSTOM> &grid, int k_max, int8_t *codes, float *scales,
-                      float *resid_sq, float *residuals, int hbits, size_t smem,
+                      float *resid_sq, float *residuals, int hbits, LatBits lb, size_t smem,
                       cudaStream_t stream)
 {
     if constexpr (!CUSTOM) {
         if (lat) {
-            // the lattice form on the linear grid: no grid table and packed counts when that fits
-            // one more CTA on an SM (it costs some arithmetic per candidate otherwise)
-            const int nb = 2 * G * qmax + 1;
-            const size_t packed = (size_t)(8 / WPC) * group_words(G, d, 1, nb, true) * 4;
-            if (quantize_ctas_per_sm<WPC, false, true, false>(packed) >
+            // the lattice form on the linear grid: no grid table when that fits one more CTA on
+            // an SM (it costs some arithmetic per candidate otherwise)
+            const size_t notab = smem - (size_t)2 * G * sizeof(float);
+            if (quantize_ctas_per_sm<WPC, false, true, false>(notab) >
                 quantize_ctas_per_sm<WPC, false, true, true>(smem))
                 return launch_wpc<WPC, false, true, false>(W, C, d, qmax, G, grid, k_max, codes,
-                                                           scales, resid_sq, residuals, hbits,
-                                                           packed, stream);
+                                                           scales, resid_sq, residuals, hbits, lb,
+                                                           notab, stream);
             return launch_wpc<WPC, false, true, true>(W, C, d, qmax, G, grid, k_max, codes, scales,
-                                                      resid_sq, residuals, hbits, smem, stream);
+                                                      resid_sq, residuals, hbits, lb, smem, stream);
         }
     }
     return launch_wpc<WPC, CUSTOM, false, true>(W, C, d, qmax, G, grid, k_max, codes, scales,
-                                                resid_sq, residuals, hbits, smem, stream);
+                                                resid_sq, residuals, hbits, lb, smem, stream);
 }
 
 template <bool CUSTOM>
@@ -883,8 +945,10 @@ mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid
                        cudaStream_t stream)
 {
     const int hbits = ceil_log2((long long)d * qmax) + 1;
-    // lattice form on the linear grid when its buckets fit (48 KB)
-    const bool lat = !CUSTOM && (long long)2 * G * qmax + 1 <= 4096;
+    // lattice form on the linear grid when its buckets fit (32 KB) and their fields one word
+    LatBits lb;
+    const bool lat = !CUSTOM && (long long)2 * G * qmax + 1 <= 4096 && lattice_bits(d, qmax, G, &lb);
+    if (!lat) lb = LatBits{0, 31};
     const int nb = lat ? 2 * G * qmax + 1 : 0;
     const size_t per_group = group_words(G, d, 1, nb) * 4;
     const long long smem_cap = max_smem_optin();
@@ -907,16 +971,16 @@ mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid
             switch (wpc) {
             case 1:
                 return launch_lat<1, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, smem, stream);
+                                             resid_sq, residuals, hbits, lb, smem, stream);
             case 2:
                 return launch_lat<2, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, smem, stream);
+                                             resid_sq, residuals, hbits, lb, smem, stream);
             case 4:
                 return launch_lat<4, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, smem, stream);
+                                             resid_sq, residuals, hbits, lb, smem, stream);
             default:
                 return launch_lat<8, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, smem, stream);
+                                             resid_sq, residuals, hbits, lb, smem, stream);
             }
         }
     }
