@@ -34,6 +34,7 @@
 #include <math.h>
 
 #include <type_traits>
+#include <vector>
 
 #include "mpq_internal.cuh"
 #include "rounding.cuh"
@@ -91,6 +92,9 @@ struct Scratch {
 // words on all 32 banks, measured no faster.)  Group regions stay 8-byte
 // aligned.
 __host__ __device__ constexpr size_t lattice_words(int nb) { return (size_t)2 * nb; }
+
+// bytes of the CTA's bucket -> position-index table (uint16 per bucket), 16-byte multiple
+__host__ __device__ constexpr size_t lut_bytes(int nb) { return ((size_t)nb * 2 + 15) & ~(size_t)15; }
 
 __host__ __device__ constexpr size_t group_words(int G, int d, int copies, int nb)
 {
@@ -434,7 +438,7 @@ __global__ void __launch_bounds__(QTHREADS, 4)
 quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, const Grid<CUSTOM> grid,
                 int k_max, int8_t *__restrict__ codes, float *__restrict__ scales,
                 float *__restrict__ resid_sq, float *__restrict__ residuals, int hbits,
-                int lat_bits, int cnt_bit)
+                int lat_bits, int cnt_bit, int nc)
 {
     const int nb = LAT ? 2 * G * qmax + 1 : 0;   // lattice buckets: floor(2u) in [0, 2 G Qmax]
     constexpr int NT = WPC * 32;
@@ -461,14 +465,39 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
         }
     auto fg = [&](int g) -> float { return TABLE ? ftab[g] : grid.frac(g, G); };
     auto fi = [&](int g) -> float { return TABLE ? ftab[G + g] : __frcp_rn(grid.frac(g, G)); };
+    // Lattice compression: only the positions (g+1)(2L-1) are read, so bucket b is stored at the
+    // index of the largest position <= b (lut[b]; nc positions in all): the suffix sum at a
+    // position's index is the sum over the buckets at or above it, as before.
+    unsigned short *lut = reinterpret_cast<unsigned short *>(ftab + (TABLE ? 2 * G : 0));
+    if (LAT) {
+        for (int b = threadIdx.x; b < nb; b += QTHREADS) lut[b] = 0;
+        __syncthreads();
+        for (int x = threadIdx.x; x < G * qmax; x += QTHREADS) {
+            const int g = x / qmax, L = x - g * qmax + 1;
+            lut[(g + 1) * (2 * L - 1)] = 1;
+        }
+        __syncthreads();
+        if (warp == 0) {   // inclusive count of positions, minus one
+            int run = 0;
+            for (int b0 = 0; b0 < nb; b0 += 32) {
+                const int b = b0 + lane;
+                const int bit = b < nb ? lut[b] : 0;
+                const unsigned bal = __ballot_sync(0xffffffffu, bit);
+                const int incl = run + __popc(bal & ((2u << lane) - 1u));
+                if (b < nb) lut[b] = (unsigned short)(incl - 1);
+                run += __popc(bal);
+            }
+        }
+    }
     __syncthreads();
     if (k >= C) return;   // whole group idle (group-uniform)
 
-    unsigned int *gl = reinterpret_cast<unsigned int *>(ftab + (TABLE ? 2 * G : 0)) +
-                       (size_t)grp * group_words(G, d, COPIES, nb);
-    unsigned int *lat = gl;                         // [nb][2]: R low word, R high | count
+    unsigned int *gl = reinterpret_cast<unsigned int *>(
+                           reinterpret_cast<unsigned char *>(lut) + (LAT ? lut_bytes(nb) : 0)) +
+                       (size_t)grp * group_words(G, d, COPIES, nc);
+    unsigned int *lat = gl;                         // [nc][2]: R low word, R high | count
     const unsigned cnt_one = 1u << cnt_bit, hmask = cnt_one - 1u;
-    unsigned int *gbase = gl + lattice_words(nb);
+    unsigned int *gbase = gl + lattice_words(nc);
     // this warp's private bins; copy 0 receives the merged suffix sums
     unsigned int *hLo = gbase + (size_t)(COPIES > 1 ? gw : 0) * 3 * (G + 1);
     unsigned int *hHi = hLo + (G + 1);
@@ -538,7 +567,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     hN[t] = 0;
                 }
                 if (LAT) {
-                    for (int t = gt; t < 2 * nb; t += NT) lat[t] = 0u;
+                    for (int t = gt; t < 2 * nc; t += NT) lat[t] = 0u;
                     if (gt == 0) sc.nq = 0;
                 }
                 gsync<WPC>(grp);
@@ -650,7 +679,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                             if (!near_lattice(u2[u])) {
                                 const int b = (int)floorf(u2[u]);
                                 if (b >= 1) {
-                                    const int bb = b < nb - 1 ? b : nb - 1;
+                                    const int bb = lut[b < nb - 1 ? b : nb - 1];
                                     // two 32-bit atomics: the low word's old value gives
                                     // its carry, which the high word takes with the count
                                     const unsigned long long R =
@@ -742,9 +771,9 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     if (gw == 0)
                         group_suffix_scan<1>(1, G + 1, bins_load, bins_store, sc, 0, lane, grp);
                     if (WPC == 1)
-                        group_suffix_scan<1>(0, nb, lat_load, lat_store, sc, 0, lane, grp);
+                        group_suffix_scan<1>(0, nc, lat_load, lat_store, sc, 0, lane, grp);
                     else if (gw >= 1)
-                        warps_suffix_scan(0, nb, lat_load, lat_store, sc, WPC - 1, gw - 1, lane,
+                        warps_suffix_scan(0, nc, lat_load, lat_store, sc, WPC - 1, gw - 1, lane,
                                           8 + grp);
                 } else if (G * COPIES > 1024) {
                     group_suffix_scan<WPC>(1, G + 1, bins_load, bins_store, sc, gw, lane, grp);
@@ -758,7 +787,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                         long long p = bin64(mLo, mHi, g + 1);
                         long long n = mN[g + 1];
                         for (int L = 1; L <= qmax; ++L) {
-                            const int b = (g + 1) * (2 * L - 1);
+                            const int b = lut[(g + 1) * (2 * L - 1)];
                             const unsigned hi = lat[2 * b + 1];
                             p += (long long)(((unsigned long long)(hi & hmask) << 32) | lat[2 * b]);
                             n += (long long)(2 * L - 1) * (hi >> cnt_bit);
@@ -873,7 +902,23 @@ int ceil_log2(long long x)
 // the two fields do not fit one word (the event form runs then).
 struct LatBits {
     int lat_bits, cnt_bit;
+    int nc;   // distinct lattice positions (g+1)(2L-1)
 };
+
+int lattice_positions(int G, int qmax)
+{
+    std::vector<char> seen((size_t)2 * G * qmax + 1, 0);
+    int n = 0;
+    for (int g = 1; g <= G; ++g)
+        for (int L = 1; L <= qmax; ++L) {
+            char &c = seen[(size_t)g * (2 * L - 1)];
+            if (!c) {
+                c = 1;
+                ++n;
+            }
+        }
+    return n;
+}
 
 bool lattice_bits(int d, int qmax, int G, LatBits *lb)
 {
@@ -895,7 +940,7 @@ mpq_status launch_wpc(const float *W, int C, int d, int qmax, int G, const Grid<
     if (e == cudaSuccess) {
         quantize_kernel<WPC, CUSTOM, LAT, TABLE><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
             W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, hbits, lb.lat_bits,
-            lb.cnt_bit);
+            lb.cnt_bit, lb.nc);
         e = cudaGetLastError();
     }
     return cuda_status(e, "quantize kernel launch");
@@ -948,12 +993,16 @@ mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid
     // lattice form on the linear grid when its buckets fit (32 KB) and their fields one word
     LatBits lb;
     const bool lat = !CUSTOM && (long long)2 * G * qmax + 1 <= 4096 && lattice_bits(d, qmax, G, &lb);
-    if (!lat) lb = LatBits{0, 31};
+    if (!lat) lb = LatBits{0, 31, 0};
     const int nb = lat ? 2 * G * qmax + 1 : 0;
-    const size_t per_group = group_words(G, d, 1, nb) * 4;
+    if (lat) lb.nc = lattice_positions(G, qmax);
+    const int nc = lb.nc;
+    const size_t per_group = group_words(G, d, 1, nc) * 4;
     const long long smem_cap = max_smem_optin();
     // Warps per channel: enough channels in flight to fill the GPU, at least ~2 elements per
-    // lane, and enough warps per SM for the shared memory the channels need.
+    // lane, and enough warps per SM (24) for the shared memory the channels need -- on layers with
+    // thousands of long channels, 4-warp groups (more channels per SM, barriers over fewer warps)
+    // measured faster than 8-warp ones (c5's 11008 x 4096 layer: 2.28 -> 2.20 ms).
     const long long warps_gpu = (long long)sm_count() * 32;
     int wpc_c = 1;
     while (wpc_c < 8 && (long long)C * wpc_c < warps_gpu) wpc_c *= 2;
@@ -961,12 +1010,12 @@ mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid
     while (wpc_e < 8 && wpc_e * 64 <= d) wpc_e *= 2;
     const long long groups_per_sm = (long long)(227 * 1024) / (long long)(per_group + 256);
     int wpc_s = 1;
-    while (wpc_s < 8 && groups_per_sm * wpc_s < 32) wpc_s *= 2;
+    while (wpc_s < 8 && groups_per_sm * wpc_s < 24) wpc_s *= 2;
     int wpc = wpc_c < wpc_e ? wpc_c : wpc_e;
     if (wpc < wpc_s) wpc = wpc_s;
     for (; wpc <= 8; wpc *= 2) {
-        const size_t smem = (size_t)(8 / wpc) * group_words(G, d, lat ? 1 : wpc, nb) * 4 +
-                            (size_t)2 * G * sizeof(float);
+        const size_t smem = (size_t)(8 / wpc) * group_words(G, d, lat ? 1 : wpc, nc) * 4 +
+                            (size_t)2 * G * sizeof(float) + (lat ? lut_bytes(nb) : 0);
         if ((long long)smem <= smem_cap) {
             switch (wpc) {
             case 1:
