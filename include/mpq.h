@@ -94,10 +94,13 @@ typedef enum {
  *   resid_sq   out [C][k_max+1] fp32, nullable: ||r_{k,n+1}||^2 for n = 0..k_max points
  *              (n = 0 is ||w_k||^2).
  *   residuals  out [k_max][C][d] fp32, nullable: residuals[i][k][:] = r_{k,i+2}.
+ *   rmax       out [C][k_max+1] fp32, nullable: max_j |r_{k,n+1,j}| for n = 0..k_max points
+ *              (n = 0 is max_j |w_kj|; NaN for a channel with a non-finite weight) -- the
+ *              operand ranges mpq_output_error can take instead of measuring them.
  */
 mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
                               const float *grid_frac, int k_max, int8_t *codes, float *scales,
-                              float *resid_sq, float *residuals, void *stream);
+                              float *resid_sq, float *residuals, float *rmax, void *stream);
 
 /*
  * mpq_output_error -- output error of every channel for every point count (Sec. 3.3, Eq. 11):
@@ -111,21 +114,26 @@ mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
  *   N       calibration rows, >= 1.
  *   groups  1 or C.
  *   W, codes, scales, C, d, k_max   as produced by / passed to mpq_quantize_layer.
+ *   rmax    [C][k_max+1] fp32 or NULL: the rmax output of the mpq_quantize_layer call that made
+ *           codes and scales (max |r| of every residual vector).  Given, the tensor-core path's
+ *           range pass reads X alone instead of X, W and every code plane; NULL, it measures the
+ *           ranges itself.  The results are the same either way.
  *   err     out [C][k_max+1] fp32.
  *
  * Scratch: with groups == 1, d a multiple of 16 and X, W, codes 16-byte aligned (the tensor-core
- * path with scaled fp16 operands), the call takes 4 (1 + C (k_max+1)) bytes from the current
- * device's default stream-ordered memory pool with cudaMallocAsync on `stream` and returns them
- * with cudaFreeAsync on `stream` -- concurrent calls on other streams each get their own, and a
- * CUDA graph capture records them as the graph's allocation nodes.  MPQ_ERR_NOMEM if that
- * allocation fails (nothing else is enqueued then).  The first such call in a process made
- * outside a stream capture raises that pool's release threshold (cudaMemPoolAttrReleaseThreshold) to keep freed blocks cached in
- * the pool instead of returning them to the driver at every synchronization; a process that
- * manages the default pool itself can call mpq_output_error_noalloc instead.
+ * path with scaled fp16 operands), the call takes 4 (1 + C (k_max+1)) bytes (4 bytes with rmax)
+ * from the current device's default stream-ordered memory pool with cudaMallocAsync on `stream`
+ * and returns them with cudaFreeAsync on `stream` -- concurrent calls on other streams each get
+ * their own, and a CUDA graph capture records them as the graph's allocation nodes.
+ * MPQ_ERR_NOMEM if that allocation fails (nothing else is enqueued then).  The first such call in
+ * a process made outside a stream capture raises that pool's release threshold
+ * (cudaMemPoolAttrReleaseThreshold) to keep freed blocks cached in the pool instead of returning
+ * them to the driver at every synchronization; a process that manages the default pool itself
+ * can call mpq_output_error_noalloc instead.
  */
 mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
-                            const int8_t *codes, const float *scales, int C, int d, int k_max,
-                            float *err, void *stream);
+                            const int8_t *codes, const float *scales, const float *rmax, int C,
+                            int d, int k_max, float *err, void *stream);
 
 /* Most code-level thresholds (d * Qmax) one step of mpq_quantize_layer_adaptive sorts. */
 #define MPQ_ADAPTIVE_MAX_THRESHOLDS 65536
@@ -171,8 +179,8 @@ mpq_status mpq_quantize_layer_adaptive(const float *W, int C, int d, int bits, i
  * device memory while they run -- a process whose memory is budgeted up front by its owner, a
  * framework whose allocator owns the stream-ordered pool, or a pool that is switched off.
  *
- * Same arguments, layouts, validation, results (bit for bit) and errors as mpq_output_error,
- * except for the scratch: the tensor-core path's range table (1 + C (k_max+1) words) lives in one
+ * Same arguments (without rmax: the ranges are always measured), layouts, validation, results
+ * (bit for bit) and errors as mpq_output_error, except for the scratch: the tensor-core path's range table (1 + C (k_max+1) words) lives in one
  * fixed device array of MPQ_NOALLOC_RANGE_WORDS words (4 MiB) inside the library, which every
  * device that loads the library's module keeps until the process exits.  The call zeroes the
  * part of the table it uses before filling it.  Therefore:

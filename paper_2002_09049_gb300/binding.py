@@ -47,10 +47,10 @@ class PackedLayout(ctypes.Structure):
 _L = ctypes.POINTER(PackedLayout)
 
 SIGNATURES = {
-    "mpq_quantize_layer": ([_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P], _I),
+    "mpq_quantize_layer": ([_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P, _P], _I),
     "mpq_quantize_layer_adaptive": ([_P, _I, _I, _I, _I, _D, ctypes.c_longlong, _P, _P, _P, _P,
                                      _P], _I),
-    "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_output_error_noalloc": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
     "mpq_reconstruct": ([_P, _P, _P, _P, _I, _I, _I, _P, _P], _I),
@@ -131,11 +131,12 @@ def _dev(t, name, dtype, shape=None):
 
 def mpq_quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, codes=None,
                        scales=None, resid_sq=None, residuals=None, want_resid_sq=True,
-                       stream=None):
+                       rmax=None, stream=None):
     """Greedy multipoint construction (Algorithm 1) of every channel of W [C][d] fp32.
 
     Returns (codes [k_max][C][d] int8, scales [C][k_max] fp32, resid_sq [C][k_max+1] or None,
-    residuals or None).  grid_frac: optional host sequence of G fractions in (0, 1]."""
+    residuals or None).  grid_frac: optional host sequence of G fractions in (0, 1].  rmax: an
+    optional [C][k_max+1] fp32 tensor that receives max |r| of every residual vector."""
     _dev(W, "W", torch.float32)
     C, d = W.shape
     dev = W.device
@@ -150,6 +151,8 @@ def mpq_quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, codes=N
         _dev(resid_sq, "resid_sq", torch.float32, (C, k_max + 1))
     if residuals is not None:
         _dev(residuals, "residuals", torch.float32, (k_max, C, d))
+    if rmax is not None:
+        _dev(rmax, "rmax", torch.float32, (C, k_max + 1))
     gf = None
     if grid_frac is not None:
         gf_list = [float(x) for x in grid_frac]
@@ -157,7 +160,7 @@ def mpq_quantize_layer(W, bits: int, G: int, k_max: int, grid_frac=None, codes=N
             raise ValueError("grid_frac must have G entries")
         gf = (ctypes.c_float * G)(*gf_list)
     st = load().mpq_quantize_layer(_ptr(W), C, d, bits, G, gf, k_max, _ptr(codes), _ptr(scales),
-                                   _ptr(resid_sq), _ptr(residuals), _stream(stream))
+                                   _ptr(resid_sq), _ptr(residuals), _ptr(rmax), _stream(stream))
     _check(st, "mpq_quantize_layer")
     return codes, scales, resid_sq, residuals
 
@@ -191,7 +194,7 @@ def mpq_quantize_layer_adaptive(W, bits: int, k_max: int, eta: float = ETA,
     return codes, scales, resid_sq, ncand
 
 
-def _output_error(entry, X, W, codes, scales, k_max, groups, err, stream):
+def _output_error(entry, X, W, codes, scales, k_max, groups, err, stream, rmax=None):
     _dev(W, "W", torch.float32)
     C, d = W.shape
     _dev(X, "X", torch.float32)
@@ -208,15 +211,24 @@ def _output_error(entry, X, W, codes, scales, k_max, groups, err, stream):
     err = err if err is not None else torch.empty((C, k_max + 1), dtype=torch.float32,
                                                   device=W.device)
     _dev(err, "err", torch.float32, (C, k_max + 1))
-    st = getattr(load(), entry)(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales), C, d,
-                                k_max, _ptr(err), _stream(stream))
+    if entry == "mpq_output_error":
+        if rmax is not None:
+            _dev(rmax, "rmax", torch.float32, (C, k_max + 1))
+        st = load().mpq_output_error(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales),
+                                     _ptr(rmax), C, d, k_max, _ptr(err), _stream(stream))
+    else:
+        st = getattr(load(), entry)(_ptr(X), N, groups, _ptr(W), _ptr(codes), _ptr(scales), C,
+                                    d, k_max, _ptr(err), _stream(stream))
     _check(st, entry)
     return err
 
 
-def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None, stream=None):
-    """Output error (Eq. 11) for n = 0..k_max points: err [C][k_max+1] fp32."""
-    return _output_error("mpq_output_error", X, W, codes, scales, k_max, groups, err, stream)
+def mpq_output_error(X, W, codes, scales, k_max: int, groups: int = 1, err=None, stream=None,
+                     rmax=None):
+    """Output error (Eq. 11) for n = 0..k_max points: err [C][k_max+1] fp32.  rmax: the greedy
+    search's max |r| per residual vector, if kept (the ranges are then not measured again)."""
+    return _output_error("mpq_output_error", X, W, codes, scales, k_max, groups, err, stream,
+                         rmax)
 
 
 def mpq_output_error_noalloc(X, W, codes, scales, k_max: int, groups: int = 1, err=None,

@@ -99,7 +99,7 @@ static mpq_status check_common(int C, int d, int k_max)
 extern "C" mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
                                          const float *grid_frac, int k_max, int8_t *codes,
                                          float *scales, float *resid_sq, float *residuals,
-                                         void *stream)
+                                         float *rmax, void *stream)
 {
     CallRange range_("mpq_quantize_layer");
     g_msg[0] = 0;
@@ -131,7 +131,7 @@ extern "C" mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits,
     }
     int qmax = (1 << (bits - 1)) - 1;
     return launch_quantize(W, C, d, qmax, G, grid_frac ? &gf : nullptr, k_max, codes, scales,
-                           resid_sq, residuals, (cudaStream_t)stream);
+                           resid_sq, residuals, rmax, (cudaStream_t)stream);
 }
 
 extern "C" mpq_status mpq_quantize_layer_adaptive(const float *W, int C, int d, int bits,
@@ -177,15 +177,15 @@ static mpq_status check_output_error(const float *X, int N, int groups, const fl
 }
 
 extern "C" mpq_status mpq_output_error(const float *X, int N, int groups, const float *W,
-                                       const int8_t *codes, const float *scales, int C, int d,
-                                       int k_max, float *err, void *stream)
+                                       const int8_t *codes, const float *scales, const float *rmax,
+                                       int C, int d, int k_max, float *err, void *stream)
 {
     CallRange range_("mpq_output_error");
     g_msg[0] = 0;
     const mpq_status st = check_output_error(X, N, groups, W, codes, scales, C, d, k_max, err);
     if (st != MPQ_OK || C == 0) return st;
     return launch_output_error(X, N, groups, W, codes, scales, C, d, k_max, err,
-                               (cudaStream_t)stream);
+                               (cudaStream_t)stream, nullptr, rmax);
 }
 
 // The fixed scratch of mpq_output_error_noalloc: one array for every call of that entry point

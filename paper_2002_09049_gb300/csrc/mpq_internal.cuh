@@ -50,13 +50,16 @@ struct GridFrac {
 // --- launchers, one per kernel family; arguments are already validated ----------------------
 mpq_status launch_quantize(const float *W, int C, int d, int qmax, int G, const GridFrac *grid,
                            int k_max, int8_t *codes, float *scales, float *resid_sq,
-                           float *residuals, cudaStream_t stream);
+                           float *residuals, float *rmax, cudaStream_t stream);
 
 // range: scratch of output_error_scratch_words() words for the pair kernel's operand ranges, or
-// NULL to take it from the device's stream-ordered pool on `stream`.
+// NULL to take it from the device's stream-ordered pool on `stream`.  rmax (nullable): max |r| of
+// every residual vector ([C][k_max+1], from mpq_quantize_layer); the range pre-pass then reads X
+// alone and the table holds one word.
 mpq_status launch_output_error(const float *X, int N, int groups, const float *W,
                                const int8_t *codes, const float *scales, int C, int d, int k_max,
-                               float *err, cudaStream_t stream, unsigned *range = nullptr);
+                               float *err, cudaStream_t stream, unsigned *range = nullptr,
+                               const float *rmax = nullptr);
 // Words of range scratch a call needs (0 where it takes no scratch).
 size_t output_error_scratch_words(const float *X, int groups, const float *W,
                                   const int8_t *codes, int C, int d, int k_max);
@@ -69,7 +72,7 @@ mpq_status launch_output_error_tc(const float *X, int N, const float *W, const i
 bool output_error_pair_ok(const float *X, const float *W, const int8_t *codes, int d);
 mpq_status launch_output_error_pair(const float *X, int N, const float *W, const int8_t *codes,
                                     const float *scales, int C, int d, int k_max, float *err,
-                                    cudaStream_t stream, unsigned *range);
+                                    cudaStream_t stream, unsigned *range, const float *rmax);
 
 mpq_status launch_clip_pair(const float *X, int N, const float *W, const float *clip, int C, int d,
                             int qmax, int n_cand, float *err, cudaStream_t stream);

@@ -134,12 +134,13 @@ size_t output_error_scratch_words(const float *X, int groups, const float *W,
 
 mpq_status launch_output_error(const float *X, int N, int groups, const float *W,
                                const int8_t *codes, const float *scales, int C, int d, int k_max,
-                               float *err, cudaStream_t stream, unsigned *range)
+                               float *err, cudaStream_t stream, unsigned *range,
+                               const float *rmax)
 {
     if (groups == 1) {
         if (output_error_pair_ok(X, W, codes, d))
             return launch_output_error_pair(X, N, W, codes, scales, C, d, k_max, err, stream,
-                                            range);
+                                            range, rmax);
         return launch_output_error_tc(X, N, W, codes, scales, C, d, k_max, err, stream);
     }
     switch (k_max + 1) {

@@ -324,7 +324,8 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh,
 template <int KP1, bool CLIP>
 __global__ void __launch_bounds__(PRoles<CLIP>::THREADS, 1)
 output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, int qmax,
-                         const unsigned *__restrict__ range, float *__restrict__ err, int split,
+                         const unsigned *__restrict__ xrange, const unsigned *__restrict__ vrange,
+                         float *__restrict__ err, int split,
                          const WaitCtl wc, const __grid_constant__ CUtensorMap tmX,
                          const __grid_constant__ CUtensorMap tmW,
                          const __grid_constant__ CUtensorMap tmQ)
@@ -382,12 +383,12 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         }
     } else {
         for (int i = threadIdx.x; i < nvec; i += PR::THREADS) {
-            const int e = f16_scale_exp(__uint_as_float(__ldg(range + 1 + (size_t)k0 * KP1 + i)));
+            const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * KP1 + i)));
             ctl.vexp[i] = e;
             ctl.vscale[i] = pow2f(e);
         }
         if (threadIdx.x == 0) {
-            const int e = f16_scale_exp(__uint_as_float(__ldg(range)));
+            const int e = f16_scale_exp(__uint_as_float(__ldg(xrange)));
             ctl.xexp = e;
             ctl.xscale = pow2f(e);
         }
@@ -460,6 +461,9 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 if (stop) break;
                 tc_fence_after();
                 const bool first = (sg == 0), last = (sg == nseg - 1);
+                // the previous drain's running-sum stores land before they are read back (the MMA
+                // never writes those columns, so the segment was released without waiting)
+                if (!first) tmem_wait_st();
 #pragma unroll 1
                 for (int cb = 0; cb < P_N / 64; ++cb) {
                     const uint32_t col = (uint32_t)(cb * 32);
@@ -481,12 +485,12 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                         tmem_st_32x32b_x32(lane_base + P_RUN_COL + col, v);
                     }
                 }
-                if (!last) tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_cluster(&ctl.segempty, leader);
             }
         }
+        tmem_wait_st();   // nothing of this warp's is in flight when tensor memory is released
         ctl.part[h][q * 32 + lane] = *abort_flag ? (double)NAN : acc;
     } else if (warp == PR::MMA_WARP) {
         // ---------------------------------------------------------------- MMA issuer (even CTA)
@@ -709,7 +713,7 @@ bool pair_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *ba
 template <int KP1, bool CLIP>
 mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *codes,
                        const float *scales, int C, int d, int qmax, float *err, cudaStream_t stream,
-                       unsigned *ext_range = nullptr)
+                       unsigned *ext_range = nullptr, const float *rmax = nullptr)
 {
     using G = PGeo<KP1, CLIP>;
     const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
@@ -784,25 +788,28 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     if (wst != MPQ_OK) return wst;
     unsigned *range = ext_range;
     if constexpr (!CLIP) {
-        // fp16 operands: the ranges of X and of every residual vector first
+        // fp16 operands: the ranges of X and of every residual vector first (the residual vectors'
+        // from rmax when the greedy search gave them: then the pre-pass reads X alone)
+        const size_t words = rmax ? 1 : 1 + (size_t)C * KP1;
         if (!ext_range) {
-            mpq_status st = pool_scratch(reinterpret_cast<void **>(&range),
-                                         (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
+            mpq_status st = pool_scratch(reinterpret_cast<void **>(&range), words * sizeof(unsigned),
+                                         stream);
             if (st != MPQ_OK) return st;
         }
         const long long nx4 = (long long)N * d / 4;
         const int xb = (int)std::min<long long>((nx4 + 1023) / 1024, 4LL * sm_count());
         const int rsplit = std::min(8, std::max(1, (d / 4 + 255) / 256));   // >= 8 loads per lane
-        const long long cb = ((long long)C * rsplit + 7) / 8;
-        e = cudaMemsetAsync(range, 0, (1 + (size_t)C * KP1) * sizeof(unsigned), stream);
+        const long long cb = rmax ? 0 : ((long long)C * rsplit + 7) / 8;
+        e = cudaMemsetAsync(range, 0, words * sizeof(unsigned), stream);
         if (e == cudaSuccess) {
             pair_range_kernel<KP1><<<(unsigned)(xb + cb), 256, 0, stream>>>(
                 reinterpret_cast<const float4 *>(X), nx4, xb, W, codes, scales, C, d, rsplit, range);
             e = cudaGetLastError();
         }
+        const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : range + 1;
         if (e == cudaSuccess)
             e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
-                                   (const unsigned *)range, err, split, wc, tmX, tmW, tmQ);
+                                   (const unsigned *)range, vr, err, split, wc, tmX, tmW, tmQ);
         if (!ext_range) {
             const cudaError_t ef = cudaFreeAsync(range, stream);
             if (e == cudaSuccess) e = ef;
@@ -810,7 +817,8 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         return cuda_status(e, "pair output-error kernel launch");
     }
     e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
-                           (const unsigned *)nullptr, err, split, wc, tmX, tmW, tmQ);
+                           (const unsigned *)nullptr, (const unsigned *)nullptr, err, split, wc,
+                           tmX, tmW, tmQ);
     return cuda_status(e, "pair output-error kernel launch");
 }
 
@@ -855,11 +863,11 @@ bool output_error_pair_ok(const float *X, const float *W, const int8_t *codes, i
 
 mpq_status launch_output_error_pair(const float *X, int N, const float *W, const int8_t *codes,
                                     const float *scales, int C, int d, int k_max, float *err,
-                                    cudaStream_t stream, unsigned *range)
+                                    cudaStream_t stream, unsigned *range, const float *rmax)
 {
     switch (k_max + 1) {
 #define MPQ_CASE(n) \
-    case n: return launch_pair<n, false>(X, N, W, codes, scales, C, d, 0, err, stream, range);
+    case n: return launch_pair<n, false>(X, N, W, codes, scales, C, d, 0, err, stream, range, rmax);
         MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7) MPQ_CASE(8)
         MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14) MPQ_CASE(15)
         MPQ_CASE(16) MPQ_CASE(17)

@@ -437,7 +437,8 @@ template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
 __global__ void __launch_bounds__(QTHREADS, 4)
 quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, const Grid<CUSTOM> grid,
                 int k_max, int8_t *__restrict__ codes, float *__restrict__ scales,
-                float *__restrict__ resid_sq, float *__restrict__ residuals, int hbits,
+                float *__restrict__ resid_sq, float *__restrict__ residuals,
+                float *__restrict__ rmax, int hbits,
                 int lat_bits, int cnt_bit, int nc)
 {
     const int nb = LAT ? 2 * G * qmax + 1 : 0;   // lattice buckets: floor(2u) in [0, 2 G Qmax]
@@ -529,6 +530,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
     group_max_sum_or<WPC>(m, r2, bad, sc, gw, lane, grp);
     if (WPC == 1) __syncwarp();
     if (resid_sq && gt == 0) resid_sq[(size_t)k * (k_max + 1)] = bad ? NAN : r2;
+    if (rmax && gt == 0) rmax[(size_t)k * (k_max + 1)] = bad ? NAN : m;
 
     for (int i = 0; i < k_max; ++i) {
         int8_t *qi = codes + (size_t)i * plane + (size_t)k * d;
@@ -541,6 +543,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             if (gt == 0) {
                 scales[(size_t)k * k_max + i] = NAN;
                 if (resid_sq) resid_sq[(size_t)k * (k_max + 1) + i + 1] = NAN;
+                if (rmax) rmax[(size_t)k * (k_max + 1) + i + 1] = NAN;
             }
             continue;
         }
@@ -884,6 +887,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
         group_max_sum_or<WPC>(m, r2, none, sc, gw, lane, grp);   // orders the sr[] writes too
         if (WPC == 1) __syncwarp();
         if (resid_sq && gt == 0) resid_sq[(size_t)k * (k_max + 1) + i + 1] = r2;
+        if (rmax && gt == 0) rmax[(size_t)k * (k_max + 1) + i + 1] = m;
     }
 }
 
@@ -932,14 +936,14 @@ bool lattice_bits(int d, int qmax, int G, LatBits *lb)
 template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
 mpq_status launch_wpc(const float *W, int C, int d, int qmax, int G, const Grid<CUSTOM> &grid,
                       int k_max, int8_t *codes, float *scales, float *resid_sq, float *residuals,
-                      int hbits, LatBits lb, size_t smem, cudaStream_t stream)
+                      float *rmax, int hbits, LatBits lb, size_t smem, cudaStream_t stream)
 {
     constexpr int GPC = 8 / WPC;
     cudaError_t e = cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e == cudaSuccess) {
         quantize_kernel<WPC, CUSTOM, LAT, TABLE><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
-            W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, hbits, lb.lat_bits,
+            W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, rmax, hbits, lb.lat_bits,
             lb.cnt_bit, lb.nc);
         e = cudaGetLastError();
     }
@@ -963,8 +967,8 @@ int quantize_ctas_per_sm(size_t smem)
 template <int WPC, bool CUSTOM>
 mpq_status launch_lat(bool lat, const float *W, int C, int d, int qmax, int G,
                       const Grid<CUSTOM> &grid, int k_max, int8_t *codes, float *scales,
-                      float *resid_sq, float *residuals, int hbits, LatBits lb, size_t smem,
-                      cudaStream_t stream)
+                      float *resid_sq, float *residuals, float *rmax, int hbits, LatBits lb,
+                      size_t smem, cudaStream_t stream)
 {
     if constexpr (!CUSTOM) {
         if (lat) {
@@ -974,20 +978,20 @@ mpq_status launch_lat(bool lat, const float *W, int C, int d, int qmax, int G,
             if (quantize_ctas_per_sm<WPC, false, true, false>(notab) >
                 quantize_ctas_per_sm<WPC, false, true, true>(smem))
                 return launch_wpc<WPC, false, true, false>(W, C, d, qmax, G, grid, k_max, codes,
-                                                           scales, resid_sq, residuals, hbits, lb,
+                                                           scales, resid_sq, residuals, rmax, hbits, lb,
                                                            notab, stream);
             return launch_wpc<WPC, false, true, true>(W, C, d, qmax, G, grid, k_max, codes, scales,
-                                                      resid_sq, residuals, hbits, lb, smem, stream);
+                                                      resid_sq, residuals, rmax, hbits, lb, smem, stream);
         }
     }
     return launch_wpc<WPC, CUSTOM, false, true>(W, C, d, qmax, G, grid, k_max, codes, scales,
-                                                resid_sq, residuals, hbits, lb, smem, stream);
+                                                resid_sq, residuals, rmax, hbits, lb, smem, stream);
 }
 
 template <bool CUSTOM>
 mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid<CUSTOM> &grid,
                        int k_max, int8_t *codes, float *scales, float *resid_sq, float *residuals,
-                       cudaStream_t stream)
+                       float *rmax, cudaStream_t stream)
 {
     const int hbits = ceil_log2((long long)d * qmax) + 1;
     // lattice form on the linear grid when its buckets fit (32 KB) and their fields one word
@@ -1020,16 +1024,16 @@ mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid
             switch (wpc) {
             case 1:
                 return launch_lat<1, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, lb, smem, stream);
+                                             resid_sq, residuals, rmax, hbits, lb, smem, stream);
             case 2:
                 return launch_lat<2, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, lb, smem, stream);
+                                             resid_sq, residuals, rmax, hbits, lb, smem, stream);
             case 4:
                 return launch_lat<4, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, lb, smem, stream);
+                                             resid_sq, residuals, rmax, hbits, lb, smem, stream);
             default:
                 return launch_lat<8, CUSTOM>(lat, W, C, d, qmax, G, grid, k_max, codes, scales,
-                                             resid_sq, residuals, hbits, lb, smem, stream);
+                                             resid_sq, residuals, rmax, hbits, lb, smem, stream);
             }
         }
     }
@@ -1041,16 +1045,16 @@ mpq_status launch_grid(const float *W, int C, int d, int qmax, int G, const Grid
 
 mpq_status launch_quantize(const float *W, int C, int d, int qmax, int G, const GridFrac *grid,
                            int k_max, int8_t *codes, float *scales, float *resid_sq,
-                           float *residuals, cudaStream_t stream)
+                           float *residuals, float *rmax, cudaStream_t stream)
 {
     if (grid) {
         Grid<true> g;
         g.gf = *grid;
         return launch_grid<true>(W, C, d, qmax, G, g, k_max, codes, scales, resid_sq, residuals,
-                                 stream);
+                                 rmax, stream);
     }
     return launch_grid<false>(W, C, d, qmax, G, Grid<false>(), k_max, codes, scales, resid_sq,
-                              residuals, stream);
+                              residuals, rmax, stream);
 }
 
 }  // namespace mpq

@@ -38,6 +38,9 @@ class LayerPlan:
         self.codes = torch.empty((s.k_max, s.C, s.d), dtype=torch.int8, device=dev)
         self.scales = torch.empty((s.C, s.k_max), dtype=torch.float32, device=dev)
         self.resid_sq = torch.empty((s.C, s.k_max + 1), dtype=torch.float32, device=dev)
+        # max |r| of every residual vector: the output error's operand ranges, kept from the
+        # greedy search so that they are not measured again
+        self.rmax = torch.empty((s.C, s.k_max + 1), dtype=torch.float32, device=dev)
         self.err = torch.empty((s.C, s.k_max + 1), dtype=torch.float32, device=dev)
         self.npoints = torch.empty((s.C,), dtype=torch.int32, device=dev)
         self.points_used = torch.empty((1,), dtype=torch.int32, device=dev)
@@ -65,12 +68,13 @@ class LayerPlan:
             W = self.Wc
         tick(1)
         binding.mpq_quantize_layer(W, s.bits, s.G, s.k_max, grid_frac=grid_frac, codes=self.codes,
-                                   scales=self.scales, resid_sq=self.resid_sq, stream=stream)
+                                   scales=self.scales, resid_sq=self.resid_sq, rmax=self.rmax,
+                                   stream=stream)
         tick(2)
         if x_ready is not None:
             (stream or torch.cuda.current_stream()).wait_event(x_ready)
         binding.mpq_output_error(X, W, self.codes, self.scales, s.k_max, groups=s.groups,
-                                 err=self.err, stream=stream)
+                                 err=self.err, stream=stream, rmax=self.rmax)
         tick(3)
         binding.mpq_allocate_points(self.err, s.k_max, s.mode, s.budget_or_eps,
                                     npoints=self.npoints, points_used=self.points_used,

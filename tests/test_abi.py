@@ -61,7 +61,7 @@ def test_quantize_validation(lib, kwargs, status):
     a = dict(W=FAKE, C=4, d=16, bits=4, G=8, grid=None, k_max=2, codes=FAKE, scales=FAKE)
     a.update(kwargs)
     st = lib.mpq_quantize_layer(a["W"], a["C"], a["d"], a["bits"], a["G"], a["grid"], a["k_max"],
-                                a["codes"], a["scales"], None, None, None)
+                                a["codes"], a["scales"], None, None, None, None)
     assert st == status
     assert lib.mpq_last_error() != b""
 
@@ -70,13 +70,14 @@ def test_quantize_validation(lib, kwargs, status):
                                   [0.5, 0.75, 1.5], [0.5, float("nan"), 1.0]])
 def test_quantize_rejects_bad_grid(lib, grid):
     g = (ctypes.c_float * 3)(*grid)
-    st = lib.mpq_quantize_layer(FAKE, 4, 16, 4, 3, g, 2, FAKE, FAKE, None, None, None)
+    st = lib.mpq_quantize_layer(FAKE, 4, 16, 4, 3, g, 2, FAKE, FAKE, None, None, None, None)
     assert st == 1
 
 
 def test_empty_layer_is_a_no_op(lib):
-    assert lib.mpq_quantize_layer(None, 0, 16, 4, 8, None, 2, None, None, None, None, None) == 0
-    assert lib.mpq_output_error(None, 5, 1, None, None, None, 0, 16, 2, None, None) == 0
+    assert lib.mpq_quantize_layer(None, 0, 16, 4, 8, None, 2, None, None, None, None, None,
+                                  None) == 0
+    assert lib.mpq_output_error(None, 5, 1, None, None, None, None, 0, 16, 2, None, None) == 0
     assert lib.mpq_reconstruct(None, None, None, None, 0, 16, 2, None, None) == 0
     assert lib.mpq_center_weights(None, 0, 16, 0, None, None, None) == 0
 
@@ -88,7 +89,7 @@ def test_empty_layer_is_a_no_op(lib):
     ((FAKE, 8, 1, FAKE, FAKE, FAKE, 4, 16, 2, None), 1),    # err NULL
 ])
 def test_output_error_validation(lib, args, status):
-    assert lib.mpq_output_error(*args, None) == status
+    assert lib.mpq_output_error(*args[:6], None, *args[6:], None) == status
 
 
 def test_output_error_noalloc_validation(lib):

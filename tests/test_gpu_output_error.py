@@ -109,3 +109,30 @@ def test_nonfinite_on_the_pair_path(gpu, oracle):
     compare_err(e, oracle.output_error(X, 1, W, q["codes"], q["scales"], 3))
     X[100, 10] = np.nan
     assert np.all(np.isnan(gpu_err(X, W, q["codes"], q["scales"], 3)))
+
+
+@pytest.mark.parametrize("C,d,N,K,bits", [(130, 256, 600, 4, 4), (64, 576, 1024, 8, 4),
+                                          (9, 32, 300, 16, 3), (3, 147, 100, 4, 4)])
+def test_ranges_from_the_greedy_search(gpu, oracle, C, d, N, K, bits):
+    """mpq_quantize_layer's rmax output is max |r| of every residual vector (w, then each step's
+    residual, exactly as the oracle's recursion gives them), and mpq_output_error with it gives
+    bit for bit the errors it gives measuring the ranges itself (also for rows the tensor-core
+    path cannot take, which ignore it), within 1e-5 of the oracle."""
+    W = wlm.random_weights(C, d, 3 * C + d, "normal")
+    W[1, 3] = np.nan                                   # a non-finite channel: NaN ranges
+    X = wlm.random_calibration(N, d, 11 + d)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(gpu)
+    rmax = torch.empty((C, K + 1), dtype=torch.float32, device=gpu)
+    codes, scales, _, _ = binding.mpq_quantize_layer(t(W), bits, 64, K, rmax=rmax)
+    e1 = binding.mpq_output_error(t(X), t(W), codes, scales, K, rmax=rmax)
+    e0 = binding.mpq_output_error(t(X), t(W), codes, scales, K)
+    torch.cuda.synchronize()
+    o = oracle.quantize_layer(W, bits, 64, K)
+    want = np.concatenate([np.abs(W).max(axis=1, keepdims=True),
+                           np.abs(o["residuals"]).max(axis=2).T], axis=1)
+    want[1, :] = np.nan
+    np.testing.assert_array_equal(rmax.cpu().numpy(), want.astype(np.float32))
+    assert torch.equal(torch.nan_to_num(e1, nan=-1.0), torch.nan_to_num(e0, nan=-1.0))
+    keep = np.arange(C) != 1
+    e_or = oracle.output_error(X, 1, W[keep], o["codes"][:, keep], o["scales"][keep], K)
+    compare_err(e1.cpu().numpy()[keep], e_or)
