@@ -37,7 +37,8 @@ KERNEL_SOURCES = {
                      "paper_2002_09049_gb300/csrc/output_error_pair.cu",
                      "paper_2002_09049_gb300/csrc/output_error_tc.cu",
                      "paper_2002_09049_gb300/csrc/sm100.cuh",
-                     "paper_2002_09049_gb300/csrc/tf32_operands.cuh"),
+                     "paper_2002_09049_gb300/csrc/tf32_operands.cuh",
+                     "paper_2002_09049_gb300/csrc/waits.cuh"),
     "quantize": ("paper_2002_09049_gb300/csrc/quantize.cu",
                  "paper_2002_09049_gb300/csrc/rounding.cuh"),
     "allocate": "paper_2002_09049_gb300/csrc/allocate.cu",
