@@ -64,6 +64,8 @@ def parse():
                     help="replay the multi-stream step as a captured CUDA graph (1) or launch it (0)")
     ap.add_argument("--streams", type=int, default=12,
                     help="CUDA streams the independent layers are spread over")
+    ap.add_argument("--batch-alloc", type=int, default=1,
+                    help="allocate every layer's points in one launch (1) or one launch per layer")
     ap.add_argument("--layers", default=None,
                     help="comma-separated layer indices to run (profiling a subset); default all")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
@@ -252,7 +254,8 @@ def run_ours(args, world, rank, local):
         Xhs.append(torch.from_numpy(X).pin_memory())
         Ws.append(Whs[-1].to(dev))
         Xs.append(Xhs[-1].to(dev))
-    net = pipeline.NetworkPlan(specs, dev, n_streams=args.streams)
+    net = pipeline.NetworkPlan(specs, dev, n_streams=args.streams,
+                               batch_alloc=bool(args.batch_alloc))
     units_per_step = sum(kernel_units(wl, l) for l in layers) * len(wl.bits)
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 512 MB > L2
     stream = torch.cuda.current_stream()
@@ -270,7 +273,8 @@ def run_ours(args, world, rank, local):
                 plan_b = net
             else:
                 plan_b = pipeline.NetworkPlan([dataclasses.replace(sp, bits=b) for sp in specs],
-                                              dev, n_streams=args.streams)
+                                              dev, n_streams=args.streams,
+                                              batch_alloc=bool(args.batch_alloc))
             graphs.append(pipeline.CapturedNetwork(plan_b, Ws, Xs))
     graph_streams = [torch.cuda.Stream(dev) for _ in graphs]
 
@@ -299,7 +303,9 @@ def run_ours(args, world, rank, local):
     # one kernel per call, plus the range pre-pass of every output error on the CTA-pair kernel
     # (shared calibration input, rows a multiple of 16 elements; torch buffers are 16-byte aligned)
     range_launches = sum(1 for l in layers if l.groups == 1 and l.d % 16 == 0)
-    launches_per_step = ((4 + center_launches) * len(layers) + range_launches) * len(wl.bits)
+    alloc_launches = 1 if net.batch_alloc else len(layers)
+    launches_per_step = ((3 + center_launches) * len(layers) + alloc_launches +
+                         range_launches) * len(wl.bits)
 
     for _ in range(args.warmup):
         step()
@@ -334,7 +340,18 @@ def run_ours(args, world, rank, local):
             for i in net.order:
                 evs[i] = [torch.cuda.Event(enable_timing=True) for _ in range(len(families) + 1)]
                 net.plans[i].run_device(Ws[i], Xs[i], stream=stream,
-                                        timing=lambda ph, e=evs[i]: e[ph].record(stream))
+                                        timing=lambda ph, e=evs[i]: e[ph].record(stream),
+                                        finish=not net.batch_alloc)
+            if net.batch_alloc:   # one allocation launch for every layer, then the reconstructions
+                ab = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+                ab[0].record(stream)
+                net.allocate_all(stream)
+                ab[1].record(stream)
+                for i in net.order:
+                    evs[i][4].record(stream)
+                    net.plans[i].run_reconstruct(stream)
+                    evs[i][5].record(stream)
+                evs["batch_alloc"] = ab
             rec.append(evs)
         torch.cuda.synchronize()
         recs.append(rec)
@@ -349,9 +366,14 @@ def run_ours(args, world, rank, local):
     fam_bytes = {f: 0.0 for f in families}    # algorithmic HBM bytes of every family
     for rec in recs:
         for evs in rec:
+            ab = evs.pop("batch_alloc", None)
+            if ab is not None:
+                fam_ms["allocate"] += ab[0].elapsed_time(ab[1])
             for i, e in evs.items():
                 layer = layers[i]
                 for k, f in enumerate(families):
+                    if ab is not None and f == "allocate":
+                        continue   # timed once for all layers above
                     fam_ms[f] += e[k].elapsed_time(e[k + 1])
                 fam_work["output_error"] += contraction_flops(wl, layer)
                 fam_work["quantize"] += quantize_ops(wl, layer, wl.bits[0])
@@ -401,6 +423,7 @@ def run_ours(args, world, rank, local):
                    "G": wl.G, "k_max": wl.k_max, "budget": wl.beta, "calib_rows": wl.n_calib,
                    "units_per_step": units_per_step, "l2": "flushed between steps (512 MB write)",
                    "streams": args.streams, "cuda_graph": bool(args.graph),
+                   "batched_allocation": net.batch_alloc,
                    "center": args.center, "parallelism": f"replicas x{world}"},
         "roofline": roofline,
         "roofline_greedy": roofline_greedy,

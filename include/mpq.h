@@ -219,6 +219,29 @@ mpq_status mpq_output_error_noalloc(const float *X, int N, int groups, const flo
 mpq_status mpq_allocate_points(const float *err, int C, int k_max, int mode, double budget_or_eps,
                                int *npoints, int *points_used, void *stream);
 
+/* Most layers one mpq_allocate_points_batched call takes. */
+#define MPQ_MAX_BATCH 64
+
+/*
+ * mpq_allocate_points_batched -- mpq_allocate_points for n layers in one launch, one CTA per layer
+ * (a network's small layers each leave most of the GPU idle on their own).  Every layer gets
+ * exactly what mpq_allocate_points gives it for the same arguments (each layer has its own budget
+ * or threshold; Algorithm 2 per layer).
+ *
+ *   n              number of layers, 0..MPQ_MAX_BATCH.
+ *   err            HOST array of n device pointers: layer l's [C[l]][k_max+1] fp32 error table.
+ *   C              HOST array of n channel counts (0 is an empty layer).
+ *   k_max, mode    shared by every layer (mode as for mpq_allocate_points).
+ *   budget_or_eps  HOST array of n values: each layer's beta (budget mode) or eps (threshold).
+ *   npoints        HOST array of n device pointers: out [C[l]] int32.
+ *   points_used    HOST array of n device pointers (each nullable), or NULL.
+ * Arguments are validated for every layer before anything is enqueued.
+ */
+mpq_status mpq_allocate_points_batched(int n, const float *const *err, const int *C, int k_max,
+                                       int mode, const double *budget_or_eps,
+                                       int *const *npoints, int *const *points_used,
+                                       void *stream);
+
 /*
  * mpq_reconstruct -- multipoint weights (Eq. 4): W_hat[k][j] = B_k + sum_{i=1..n_k} s_{k,i} q_{k,i,j},
  * accumulated as acc = fmaf(s_{k,i}, q_{k,i,j}, acc) from acc = B_k (the centre of an asymmetric

@@ -53,6 +53,7 @@ SIGNATURES = {
     "mpq_output_error": ([_P, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_output_error_noalloc": ([_P, _I, _I, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_allocate_points": ([_P, _I, _I, _I, _D, _P, _P, _P], _I),
+    "mpq_allocate_points_batched": ([_I, _P, _P, _I, _I, _P, _P, _P, _P], _I),
     "mpq_reconstruct": ([_P, _P, _P, _P, _I, _I, _I, _P, _P], _I),
     "mpq_center_weights": ([_P, _I, _I, _I, _P, _P, _P], _I),
     "mpq_clip_search": ([_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P], _I),
@@ -342,6 +343,41 @@ def mpq_allocate_points(err, k_max: int, mode: int = MPQ_ALLOC_BUDGET,
     st = load().mpq_allocate_points(_ptr(err), C, k_max, mode, float(budget_or_eps),
                                     _ptr(npoints), _ptr(points_used), _stream(stream))
     _check(st, "mpq_allocate_points")
+    return npoints, points_used
+
+
+MPQ_MAX_BATCH = 64
+
+
+def mpq_allocate_points_batched(errs, k_max: int, mode: int, budgets, npoints=None,
+                                points_used=None, stream=None):
+    """Algorithm 2 for several layers in one launch: errs[l] is layer l's [C_l][k_max+1] fp32
+    error table, budgets[l] its beta (budget mode) or eps.  Returns (npoints list, points_used
+    list); pass lists of preallocated tensors to write into them instead."""
+    n = len(errs)
+    if n > MPQ_MAX_BATCH:
+        raise ValueError(f"at most {MPQ_MAX_BATCH} layers per call")
+    Cs = []
+    for e in errs:
+        _dev(e, "err", torch.float32)
+        if e.dim() != 2 or e.shape[1] != k_max + 1:
+            raise ValueError("every err must be [C][k_max+1]")
+        Cs.append(e.shape[0])
+    if npoints is None:
+        npoints = [torch.empty((c,), dtype=torch.int32, device=e.device) for c, e in zip(Cs, errs)]
+    if points_used is None:
+        points_used = [torch.empty((1,), dtype=torch.int32, device=e.device) for e in errs]
+    for c, t in zip(Cs, npoints):
+        _dev(t, "npoints", torch.int32, (c,))
+    for t in points_used:
+        _dev(t, "points_used", torch.int32, (1,))
+    P = ctypes.c_void_p * max(1, n)
+    st = load().mpq_allocate_points_batched(
+        n, P(*[e.data_ptr() for e in errs]), (ctypes.c_int * max(1, n))(*Cs), k_max, mode,
+        (ctypes.c_double * max(1, n))(*[float(b) for b in budgets]),
+        P(*[t.data_ptr() for t in npoints]), P(*[t.data_ptr() for t in points_used]),
+        _stream(stream))
+    _check(st, "mpq_allocate_points_batched")
     return npoints, points_used
 
 

@@ -50,11 +50,12 @@ constexpr int KEY_CACHE = 12288;   // keys held in shared memory (96 KB) when th
 
 // Radix select of the rank-th smallest selectable key, MSB first, 8 bits per pass.  A pass whose
 // target bucket holds one key ends the search with that key (recorded as the bucket's witness).
-__global__ void __launch_bounds__(AB_THREADS)
-allocate_budget_kernel(const float *__restrict__ err, int C, int k_max, long long extra,
-                       int *__restrict__ npoints, int *__restrict__ points_used, bool cached)
+// One CTA of AB_THREADS threads allocates one layer; skeys: dynamic shared memory for its keys.
+__device__ __forceinline__ void allocate_budget_cta(const float *__restrict__ err, int C, int k_max,
+                                                    long long extra, int *__restrict__ npoints,
+                                                    int *__restrict__ points_used, bool cached,
+                                                    unsigned long long *skeys)
 {
-    extern __shared__ unsigned long long skeys[];   // [C * (k_max - 1)] when cached
     __shared__ unsigned int hist[256];
     __shared__ unsigned long long witness[256];
     __shared__ unsigned long long s_prefix, s_T, s_total;
@@ -178,6 +179,70 @@ allocate_budget_kernel(const float *__restrict__ err, int C, int k_max, long lon
     }
 }
 
+__global__ void __launch_bounds__(AB_THREADS)
+allocate_budget_kernel(const float *__restrict__ err, int C, int k_max, long long extra,
+                       int *__restrict__ npoints, int *__restrict__ points_used, bool cached)
+{
+    extern __shared__ unsigned long long skeys[];   // [C * (k_max - 1)] when cached
+    allocate_budget_cta(err, C, k_max, extra, npoints, points_used, cached, skeys);
+}
+
+// Threshold mode (Algorithm 2 as printed) for one layer by one CTA, the total by a block sum.
+__device__ __forceinline__ void allocate_threshold_cta(const float *__restrict__ err, int C,
+                                                       int k_max, double eps,
+                                                       int *__restrict__ npoints,
+                                                       int *__restrict__ points_used)
+{
+    __shared__ int s_used;
+    if (threadIdx.x == 0) s_used = 0;
+    __syncthreads();
+    int used = 0;
+    for (int k = threadIdx.x; k < C; k += blockDim.x) {
+        const float *e = err + (size_t)k * (k_max + 1);
+        int n = k_max;
+        for (int m = 1; m <= k_max; ++m) {
+            if ((double)e[m] < eps) {
+                n = m;
+                break;
+            }
+        }
+        npoints[k] = n;
+        used += n;
+    }
+    if (points_used) {
+        for (int o = 16; o > 0; o >>= 1) used += __shfl_xor_sync(0xffffffffu, used, o);
+        if ((threadIdx.x & 31) == 0) atomicAdd(&s_used, used);   // integer sum: order-free
+        __syncthreads();
+        if (threadIdx.x == 0) *points_used = s_used;
+    }
+}
+
+// Several layers in one launch: CTA b allocates layer order[b] (largest first, so the longest
+// CTAs start first).
+struct AllocBatch {
+    const float *err[MPQ_MAX_BATCH];
+    int *npoints[MPQ_MAX_BATCH];
+    int *points_used[MPQ_MAX_BATCH];
+    double param[MPQ_MAX_BATCH];     // threshold mode: eps
+    long long extra[MPQ_MAX_BATCH];  // budget mode
+    int C[MPQ_MAX_BATCH];
+    unsigned char cached[MPQ_MAX_BATCH];
+    unsigned char order[MPQ_MAX_BATCH];
+};
+
+__global__ void __launch_bounds__(AB_THREADS)
+allocate_batch_kernel(const __grid_constant__ AllocBatch b, int k_max, int mode)
+{
+    extern __shared__ unsigned long long skeys[];
+    const int l = b.order[blockIdx.x];
+    if (mode == MPQ_ALLOC_BUDGET)
+        allocate_budget_cta(b.err[l], b.C[l], k_max, b.extra[l], b.npoints[l], b.points_used[l],
+                            b.cached[l] != 0, skeys);
+    else
+        allocate_threshold_cta(b.err[l], b.C[l], k_max, b.param[l], b.npoints[l],
+                               b.points_used[l]);
+}
+
 constexpr int AT_THREADS = 256;
 
 __global__ void __launch_bounds__(AT_THREADS)
@@ -211,15 +276,51 @@ mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long 
     const long long nkeys = (long long)C * (k_max - 1);
     const bool cached = nkeys <= KEY_CACHE;
     const size_t smem = cached ? (size_t)nkeys * sizeof(unsigned long long) : 0;
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(allocate_budget_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
-        if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
-    }
+    // always set: the kernel's static shared memory counts against the 48 KB default too
+    cudaError_t e = cudaFuncSetAttribute(allocate_budget_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
     allocate_budget_kernel<<<1, AB_THREADS, smem, stream>>>(err, C, k_max, extra, npoints,
                                                             points_used, cached);
     return cuda_status(cudaGetLastError(), "allocation kernel launch");
+}
+
+mpq_status launch_allocate_batch(int n, const float *const *err, const int *C, int k_max,
+                                 int mode, const long long *extra, const double *eps,
+                                 int *const *npoints, int *const *points_used, cudaStream_t stream)
+{
+    AllocBatch b;
+    size_t smem = 0;
+    int m = 0;
+    for (int l = 0; l < n; ++l) {
+        if (C[l] == 0) continue;   // nothing to allocate (points_used zeroed by the caller)
+        b.err[l] = err[l];
+        b.npoints[l] = npoints[l];
+        b.points_used[l] = points_used ? points_used[l] : nullptr;
+        b.C[l] = C[l];
+        b.extra[l] = extra ? extra[l] : 0;
+        b.param[l] = eps ? eps[l] : 0.0;
+        const long long nkeys = (long long)C[l] * (k_max - 1);
+        const bool cached = mode == MPQ_ALLOC_BUDGET && nkeys <= KEY_CACHE;
+        b.cached[l] = cached;
+        if (cached && (size_t)nkeys * sizeof(unsigned long long) > smem)
+            smem = (size_t)nkeys * sizeof(unsigned long long);
+        b.order[m++] = (unsigned char)l;
+    }
+    if (m == 0) return MPQ_OK;
+    // largest layers first
+    for (int i = 1; i < m; ++i)
+        for (int j = i; j > 0 && b.C[b.order[j]] > b.C[b.order[j - 1]]; --j) {
+            const unsigned char t = b.order[j];
+            b.order[j] = b.order[j - 1];
+            b.order[j - 1] = t;
+        }
+    const cudaError_t e = cudaFuncSetAttribute(allocate_batch_kernel,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)smem);
+    if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
+    allocate_batch_kernel<<<m, AB_THREADS, smem, stream>>>(b, k_max, mode);
+    return cuda_status(cudaGetLastError(), "batched allocation kernel launch");
 }
 
 mpq_status launch_allocate_threshold(const float *err, int C, int k_max, double eps,

@@ -352,6 +352,49 @@ extern "C" mpq_status mpq_allocate_points(const float *err, int C, int k_max, in
                                   (cudaStream_t)stream);
 }
 
+extern "C" mpq_status mpq_allocate_points_batched(int n, const float *const *err, const int *C,
+                                                  int k_max, int mode,
+                                                  const double *budget_or_eps,
+                                                  int *const *npoints, int *const *points_used,
+                                                  void *stream)
+{
+    CallRange range_("mpq_allocate_points_batched");
+    g_msg[0] = 0;
+    REQUIRE(n >= 0, MPQ_ERR_INVALID_ARG, "n = %d must be >= 0", n);
+    REQUIRE(n <= MPQ_MAX_BATCH, MPQ_ERR_UNSUPPORTED, "n = %d exceeds MPQ_MAX_BATCH = %d", n,
+            MPQ_MAX_BATCH);
+    if (n == 0) return MPQ_OK;
+    REQUIRE(err && C && budget_or_eps && npoints, MPQ_ERR_INVALID_ARG,
+            "err, C, budget_or_eps and npoints must be non-NULL host arrays");
+    REQUIRE(mode == MPQ_ALLOC_BUDGET || mode == MPQ_ALLOC_THRESHOLD, MPQ_ERR_INVALID_ARG,
+            "mode = %d must be MPQ_ALLOC_BUDGET (0) or MPQ_ALLOC_THRESHOLD (1)", mode);
+    long long extra[MPQ_MAX_BATCH];
+    for (int l = 0; l < n; ++l) {
+        mpq_status st = check_common(C[l], 1, k_max);
+        if (st != MPQ_OK) return st;
+        const double v = budget_or_eps[l];
+        REQUIRE(!isnan(v), MPQ_ERR_NONFINITE, "budget_or_eps[%d] is NaN", l);
+        if (mode == MPQ_ALLOC_BUDGET) {
+            REQUIRE(isfinite(v), MPQ_ERR_NONFINITE, "budget[%d] must be finite", l);
+            REQUIRE(v >= 0.0, MPQ_ERR_INVALID_ARG, "budget[%d] = %g must be >= 0", l, v);
+        }
+        REQUIRE(C[l] == 0 || (err[l] && npoints[l]), MPQ_ERR_INVALID_ARG,
+                "err[%d] and npoints[%d] must be non-NULL", l, l);
+        long long e = (long long)floor(v * (double)C[l] + 0.5) - (long long)C[l];
+        const long long cap = (long long)C[l] * (k_max - 1);
+        extra[l] = e < 0 ? 0 : (e > cap ? cap : e);
+    }
+    for (int l = 0; l < n; ++l)   // empty layers: no CTA, a zero total
+        if (C[l] == 0 && points_used && points_used[l]) {
+            const mpq_status st = cuda_status(
+                cudaMemsetAsync(points_used[l], 0, sizeof(int), (cudaStream_t)stream),
+                "cudaMemsetAsync");
+            if (st != MPQ_OK) return st;
+        }
+    return launch_allocate_batch(n, err, C, k_max, mode, extra, budget_or_eps, npoints,
+                                 points_used, (cudaStream_t)stream);
+}
+
 extern "C" mpq_status mpq_reconstruct(const int8_t *codes, const float *scales, const int *npoints,
                                       const float *center, int C, int d, int k_max, float *W_hat,
                                       void *stream)

@@ -91,6 +91,11 @@ mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_lay
 mpq_status launch_allocate_budget(const float *err, int C, int k_max, long long extra,
                                   int *npoints, int *points_used, cudaStream_t stream);
 
+// Several layers, one CTA each (n <= MPQ_MAX_BATCH; extra for budget mode, eps for threshold mode).
+mpq_status launch_allocate_batch(int n, const float *const *err, const int *C, int k_max,
+                                 int mode, const long long *extra, const double *eps,
+                                 int *const *npoints, int *const *points_used, cudaStream_t stream);
+
 mpq_status launch_allocate_threshold(const float *err, int C, int k_max, double eps,
                                      int *npoints, int *points_used, cudaStream_t stream);
 

@@ -53,13 +53,15 @@ class LayerPlan:
         self._host = None
 
     # -- device-resident inputs ---------------------------------------------------------------
-    def run_device(self, W, X, stream=None, grid_frac=None, timing=None, x_ready=None):
+    def run_device(self, W, X, stream=None, grid_frac=None, timing=None, x_ready=None,
+                   finish=True):
         """Enqueue the four calls (five with centring) on ``stream``.  timing(phase), if given, is
         called before the first call (phase 0) and after the centring (1, also when there is
         none), the greedy points (2), the output error (3), the allocation (4) and the
         reconstruction (5), e.g. to record CUDA events.  x_ready, if given, is a CUDA event the
         stream waits on before the output error, the first call that reads X (its copy may still
-        be in flight while the greedy search runs)."""
+        be in flight while the greedy search runs).  finish=False stops after the output error
+        (a network plan then allocates every layer's points in one call, and reconstructs)."""
         s = self.spec
         tick = timing or (lambda ph: None)
         tick(0)
@@ -76,14 +78,21 @@ class LayerPlan:
         binding.mpq_output_error(X, W, self.codes, self.scales, s.k_max, groups=s.groups,
                                  err=self.err, stream=stream, rmax=self.rmax)
         tick(3)
+        if not finish:
+            return self
         binding.mpq_allocate_points(self.err, s.k_max, s.mode, s.budget_or_eps,
                                     npoints=self.npoints, points_used=self.points_used,
                                     stream=stream)
         tick(4)
+        self.run_reconstruct(stream)
+        tick(5)
+        return self
+
+    def run_reconstruct(self, stream=None):
+        """The multipoint weights (Eq. 4) from the allocated point counts, if kept."""
         if self.W_hat is not None:
             binding.mpq_reconstruct(self.codes, self.scales, self.npoints, W_hat=self.W_hat,
                                     stream=stream, center=self.center)
-        tick(5)
         return self
 
     # -- host inputs / outputs (end to end) ----------------------------------------------------
@@ -135,9 +144,14 @@ class NetworkPlan:
     to the caller's stream, so the call as a whole is ordered like any single launch on it.
     """
 
-    def __init__(self, specs, device, n_streams: int = 8, with_reconstruct: bool = True):
+    def __init__(self, specs, device, n_streams: int = 8, with_reconstruct: bool = True,
+                 batch_alloc: bool = True):
         self.device = torch.device(device)
         self.plans = [LayerPlan(s, self.device, with_reconstruct) for s in specs]
+        # every layer's allocation in one launch (one CTA per layer) once all output errors are
+        # in, instead of one single-CTA launch per layer -- where the layers share k_max and mode
+        self.batch_alloc = (batch_alloc and len(specs) <= binding.MPQ_MAX_BATCH and
+                            len({(s.k_max, s.mode) for s in specs}) == 1)
         work = [s.C * s.d * s.G * s.k_max + s.C * s.d * s.N for s in specs]
         self.order = sorted(range(len(specs)), key=lambda i: -work[i])
         self.streams = [torch.cuda.Stream(self.device) for _ in range(max(1, n_streams))]
@@ -166,9 +180,32 @@ class NetworkPlan:
         for n, i in enumerate(self.order):
             st = self.streams[n % len(self.streams)]
             hook = None if on_layer is None else (lambda ph, st=st, i=i: on_layer(i, st, ph))
-            self.plans[i].run_device(Ws[i], Xs[i], stream=st, timing=hook)
+            self.plans[i].run_device(Ws[i], Xs[i], stream=st, timing=hook,
+                                     finish=not self.batch_alloc)
         self._join(main)
+        if self.batch_alloc:
+            self.allocate_all(main)
+            self._fork(main)
+            for n, i in enumerate(self.order):
+                self.plans[i].run_reconstruct(self.streams[n % len(self.streams)])
+            self._join(main)
         return self
+
+    def allocate_all(self, stream):
+        """Algorithm 2 for every layer in one launch (mpq_allocate_points_batched)."""
+        p0 = self.plans[0].spec
+        binding.mpq_allocate_points_batched([p.err for p in self.plans], p0.k_max, p0.mode,
+                                            [p.spec.budget_or_eps for p in self.plans],
+                                            npoints=[p.npoints for p in self.plans],
+                                            points_used=[p.points_used for p in self.plans],
+                                            stream=stream)
+
+    def _counts_out(self, p, h):
+        with torch.cuda.stream(self.copy_out):
+            h["npoints"].copy_(p.npoints, non_blocking=True)
+            h["points_used"].copy_(p.points_used, non_blocking=True)
+            if p.center is not None:
+                h["center"].copy_(p.center, non_blocking=True)
 
     def run_host(self, W_hosts, X_hosts, W_devs, X_devs, stream=None, copy_inputs=True):
         """End to end: per layer, H2D of W and X from pinned memory, the path, D2H of codes,
@@ -211,17 +248,27 @@ class NetworkPlan:
                     h["codes"].copy_(p.codes, non_blocking=True)
                     h["scales"].copy_(p.scales, non_blocking=True)
 
-            p.run_device(W_devs[i], X_devs[i], stream=st, x_ready=x_landed[i], timing=points_out)
+            p.run_device(W_devs[i], X_devs[i], stream=st, x_ready=x_landed[i], timing=points_out,
+                         finish=not self.batch_alloc)
+            outs[i] = h
+            if self.batch_alloc:
+                continue
             done = torch.cuda.Event()
             done.record(st)
             self.copy_out.wait_event(done)
-            with torch.cuda.stream(self.copy_out):
-                h["npoints"].copy_(p.npoints, non_blocking=True)
-                h["points_used"].copy_(p.points_used, non_blocking=True)
-                if p.center is not None:
-                    h["center"].copy_(p.center, non_blocking=True)
-            outs[i] = h
+            self._counts_out(p, h)
         self._join(main)
+        if self.batch_alloc:
+            self.allocate_all(main)
+            done = torch.cuda.Event()
+            done.record(main)
+            self.copy_out.wait_event(done)
+            for i in self.order:
+                self._counts_out(self.plans[i], outs[i])
+            self._fork(main)
+            for n, i in enumerate(self.order):
+                self.plans[i].run_reconstruct(self.streams[n % len(self.streams)])
+            self._join(main)
         for s in (self.copy_in, self.copy_out):
             e = torch.cuda.Event()
             e.record(s)

@@ -206,3 +206,22 @@ def test_pack_and_linear_validation(lib):
     assert lib.mpq_multipoint_linear(FAKE, 0, ctypes.byref(lay), FAKE, FAKE, None) == 1
     assert lib.mpq_multipoint_linear(None, 4, ctypes.byref(lay), FAKE, FAKE, None) == 1
     assert lib.mpq_multipoint_linear(FAKE, 4, None, FAKE, FAKE, None) == 1
+
+
+def test_batched_allocation_validation(lib):
+    f = lib.mpq_allocate_points_batched
+    errs = (ctypes.c_void_p * 2)(0x1000, 0x2000)
+    Cs = (ctypes.c_int * 2)(4, 8)
+    vals = (ctypes.c_double * 2)(1.5, 1.5)
+    npts = (ctypes.c_void_p * 2)(0x3000, 0x4000)
+    assert f(0, None, None, 4, 0, None, None, None, None) == 0                      # nothing
+    assert f(65, errs, Cs, 4, 0, vals, npts, None, None) == 3                      # > MPQ_MAX_BATCH
+    assert f(2, None, Cs, 4, 0, vals, npts, None, None) == 1                       # err array NULL
+    assert f(2, errs, Cs, 4, 2, vals, npts, None, None) == 1                       # bad mode
+    assert f(2, errs, Cs, 0, 0, vals, npts, None, None) == 1                       # k_max = 0
+    bad = (ctypes.c_double * 2)(1.5, float("nan"))
+    assert f(2, errs, Cs, 4, 0, bad, npts, None, None) == 2                        # NaN budget
+    neg = (ctypes.c_double * 2)(-1.0, 1.5)
+    assert f(2, errs, Cs, 4, 0, neg, npts, None, None) == 1                        # budget < 0
+    nulls = (ctypes.c_void_p * 2)(0x3000, None)
+    assert f(2, errs, Cs, 4, 0, vals, nulls, None, None) == 1                      # npoints[1] NULL

@@ -94,3 +94,44 @@ def test_reconstruct_equals_weight_minus_residual(gpu, oracle):
                                    t(np.full(8, 4, np.int32))).cpu().numpy()
     ulp = np.spacing(np.abs(W).max(1, keepdims=True).astype(np.float32))
     assert np.all(np.abs(W.astype(np.float64) - What - q["residuals"][3]) <= 4 * ulp)
+
+
+@pytest.mark.parametrize("K", [4, 8])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_batched_allocation_matches_per_layer(gpu, oracle, K, mode):
+    """mpq_allocate_points_batched: every layer's point counts and total equal the oracle's
+    Algorithm 2 for that layer (budget or threshold, its own beta / eps), for layers of very
+    different sizes in one launch (an empty one included), tie-heavy tables among them."""
+    rng = np.random.default_rng(K + 10 * mode)
+    sizes = [64, 1, 0, 512, 1000, 7, 2048, 300, 11008, 33]
+    errs, vals = [], []
+    for i, C in enumerate(sizes):
+        if i % 3 == 1:
+            e = rng.integers(0, 6, size=(C, K + 1)).astype(np.float32)
+        else:
+            e = (np.sort(rng.random((C, K + 1)), 1)[:, ::-1] *
+                 rng.lognormal(0, 2, (C, 1))).astype(np.float32)
+        errs.append(np.ascontiguousarray(e))
+        vals.append([1.0, 1.25, 1.5, 2.0, 3.7][i % 5] if mode == 0 else
+                    float(np.median(e)) if C else 0.5)
+    t = [torch.from_numpy(e).to(gpu) for e in errs]
+    n_gpu, used_gpu = binding.mpq_allocate_points_batched(t, K, mode, vals)
+    torch.cuda.synchronize()
+    for e, v, n, u in zip(errs, vals, n_gpu, used_gpu):
+        if mode == 0:
+            n_or, used_or = oracle.allocate_budget(e, K, v)
+        else:
+            n_or, used_or = oracle.allocate_threshold(e, K, v)
+        assert np.array_equal(n.cpu().numpy(), n_or)
+        assert int(u.item()) == used_or
+
+
+@pytest.mark.parametrize("C,K", [(2048, 4), (6144, 2), (1536, 5)])
+def test_budget_keys_at_the_default_shared_memory_limit(gpu, oracle, C, K):
+    """C (k_max - 1) keys of exactly 48 KB (the kernel's own shared memory comes on top): the
+    launch raises its shared-memory limit instead of failing."""
+    rng = np.random.default_rng(C + K)
+    err = (np.sort(rng.random((C, K + 1)), 1)[:, ::-1] * rng.lognormal(0, 1, (C, 1))).astype(np.float32)
+    n_or, used_or = oracle.allocate_budget(err, K, 1.5)
+    n_gpu, used_gpu = gpu_alloc(err, K, binding.MPQ_ALLOC_BUDGET, 1.5)
+    assert np.array_equal(n_gpu, n_or) and used_gpu == used_or

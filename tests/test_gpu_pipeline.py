@@ -105,10 +105,14 @@ def test_network_plan_streams_match_single_stream(gpu):
         Xs.append(torch.from_numpy(wlm.make_calibration(wl, li)).to(gpu))
     many = pipeline.NetworkPlan(specs, gpu, n_streams=8).run_device(Ws, Xs)
     one = pipeline.NetworkPlan(specs, gpu, n_streams=1).run_device(Ws, Xs)
+    # every layer's allocation per layer instead of in one batched launch
+    per_layer = pipeline.NetworkPlan(specs, gpu, n_streams=8, batch_alloc=False).run_device(Ws, Xs)
     torch.cuda.synchronize()
-    for a, b in zip(many.plans, one.plans):
+    assert many.batch_alloc and not per_layer.batch_alloc
+    for a, b, c in zip(many.plans, one.plans, per_layer.plans):
         for name in ("codes", "scales", "resid_sq", "err", "npoints", "points_used", "W_hat"):
             assert torch.equal(getattr(a, name), getattr(b, name)), name
+            assert torch.equal(getattr(a, name), getattr(c, name)), name
 
 
 def test_captured_graph_matches_launches(gpu):
