@@ -370,6 +370,15 @@ __device__ __forceinline__ long long fixed_point(float a, int S)
     return sh > -40 ? (M >> -sh) : 0;
 }
 
+// The same for a normal |r| whose shift is known to be in [0, 40) (lattice elements: |r| >=
+// smax / 2G, scaled to lat_bits): no branches.
+__device__ __forceinline__ unsigned long long fixed_point_lat(float a, int S)
+{
+    const uint32_t bits = __float_as_uint(a);
+    const unsigned long long M = (unsigned long long)((bits & 0x7FFFFFu) | 0x800000u);
+    return M << ((int)(bits >> 23) - 150 + S);
+}
+
 // 2^k as a double, built from its bits (k within the normal range).
 __device__ __forceinline__ double pow2d(int k)
 {
@@ -561,6 +570,9 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             const bool zs = __fmul_rn(fg(0), smax) == 0.0f;
             const int S = (LAT && !zs) ? lat_bits - e : 62 - e - hbits;
             const float pscale = ldexpf(1.0f, -S - e);   // P 2^-S / 2^e for the fp32 screen
+            // lattice elements (|r| >= smax / 2G >= 2^(e - 2 - log2(2 G Qmax))) are normal floats
+            // unless max|r| itself is below ~2^-100
+            const bool lat_normal = LAT && !zs && e > -100;
             const double down = pow2d(-S);
             const float smax_e = ldexpf(smax, -e);   // smax / 2^e for the fp32 screen
             if (!direct) {
@@ -686,7 +698,8 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                                     // two 32-bit atomics: the low word's old value gives
                                     // its carry, which the high word takes with the count
                                     const unsigned long long R =
-                                        (unsigned long long)fixed_point(av[u], S);
+                                        lat_normal ? fixed_point_lat(av[u], S)
+                                                   : (unsigned long long)fixed_point(av[u], S);
                                     const unsigned Rlo = (unsigned)R;
                                     const unsigned old = atomicAdd(&lat[2 * bb], Rlo);
                                     atomicAdd(&lat[2 * bb + 1], (unsigned)(R >> 32) +

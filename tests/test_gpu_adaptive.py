@@ -107,3 +107,19 @@ def test_adaptive_refused_and_nonfinite(gpu, oracle):
     sub = dict(codes=g["codes"][:, keep], scales=g["scales"][keep], resid_sq=g["resid_sq"][keep],
                ncand=g["ncand"][keep])
     compare_adaptive(sub, o, 4, oracle)
+
+
+def test_adaptive_tiny_gap_zero_scales(gpu, oracle):
+    """Subnormal weights: the minimal gap is a few 2^-149, so gamma is below the fp32 range and
+    the grid's first scales fl(m gamma / Qmax) are 0 (codes 0, the objective ||r||^2) before
+    the positive ones -- a case the definition decides among scale 0 and positive scales."""
+    rng = np.random.default_rng(7)
+    ints = rng.integers(-60, 61, size=(6, 12)).astype(np.float64)
+    ints[0, :2] = [37, 38]                     # neighbouring magnitudes: the smallest gap
+    W = (ints * 2.0 ** -149).astype(np.float32)
+    assert np.all(np.abs(W[W != 0]) < np.finfo(np.float32).tiny)
+    for bits in (2, 4):
+        o = oracle.quantize_adaptive(W, bits, 3, max_candidates=10 ** 7, refuse="mark")
+        assert np.any(np.float32(o["gamma"][:, 0] / (2 ** (bits - 1) - 1)) == 0.0)
+        g = run(W, bits, 3, max_cand=10 ** 7)
+        compare_adaptive(g, o, bits, oracle)
