@@ -31,7 +31,9 @@ class LayerSpec:
 
 
 class LayerPlan:
-    def __init__(self, spec: LayerSpec, device, with_reconstruct: bool = True):
+    def __init__(self, spec: LayerSpec, device, with_reconstruct: bool = True, counts=None):
+        """counts, if given: (npoints [C], points_used [1]) int32 device views to write the
+        point counts into (a network plan keeps every layer's counts in one buffer)."""
         self.spec = spec
         s = spec
         dev = torch.device(device)
@@ -42,8 +44,11 @@ class LayerPlan:
         # greedy search so that they are not measured again
         self.rmax = torch.empty((s.C, s.k_max + 1), dtype=torch.float32, device=dev)
         self.err = torch.empty((s.C, s.k_max + 1), dtype=torch.float32, device=dev)
-        self.npoints = torch.empty((s.C,), dtype=torch.int32, device=dev)
-        self.points_used = torch.empty((1,), dtype=torch.int32, device=dev)
+        if counts is None:
+            self.npoints = torch.empty((s.C,), dtype=torch.int32, device=dev)
+            self.points_used = torch.empty((1,), dtype=torch.int32, device=dev)
+        else:
+            self.npoints, self.points_used = counts
         self.W_hat = torch.empty((s.C, s.d), dtype=torch.float32, device=dev) \
             if with_reconstruct else None
         self.center = self.Wc = None
@@ -96,15 +101,17 @@ class LayerPlan:
         return self
 
     # -- host inputs / outputs (end to end) ----------------------------------------------------
-    def host_buffers(self, pin: bool = True):
-        """Pinned host buffers for the durable result of one run."""
+    def host_buffers(self, pin: bool = True, counts=None):
+        """Pinned host buffers for the durable result of one run (counts: host views for the
+        point counts, as in __init__)."""
         if self._host is None:
             s = self.spec
             mk = lambda shape, dt: torch.empty(shape, dtype=dt, pin_memory=pin)
+            npts, used = counts if counts is not None else (mk((s.C,), torch.int32),
+                                                            mk((1,), torch.int32))
             self._host = dict(codes=mk((s.k_max, s.C, s.d), torch.int8),
                               scales=mk((s.C, s.k_max), torch.float32),
-                              npoints=mk((s.C,), torch.int32),
-                              points_used=mk((1,), torch.int32))
+                              npoints=npts, points_used=used)
             if self.center is not None:
                 self._host["center"] = mk((s.C,), torch.float32)
         return self._host
@@ -147,7 +154,18 @@ class NetworkPlan:
     def __init__(self, specs, device, n_streams: int = 8, with_reconstruct: bool = True,
                  batch_alloc: bool = True):
         self.device = torch.device(device)
-        self.plans = [LayerPlan(s, self.device, with_reconstruct) for s in specs]
+        # every layer's point counts in one buffer: [sum of C] npoints, then one total per layer
+        # (one copy brings all of them back to the host)
+        tot = sum(s.C for s in specs)
+        self.counts = torch.empty((tot + len(specs),), dtype=torch.int32, device=self.device)
+        self._counts_host = None
+        offs = [0]
+        for s in specs:
+            offs.append(offs[-1] + s.C)
+        self._count_views = [(offs[i], offs[i + 1], tot + i) for i in range(len(specs))]
+        self.plans = [LayerPlan(s, self.device, with_reconstruct,
+                                counts=(self.counts[a:b], self.counts[u:u + 1]))
+                      for s, (a, b, u) in zip(specs, self._count_views)]
         # every layer's allocation in one launch (one CTA per layer) once all output errors are
         # in, instead of one single-CTA launch per layer -- where the layers share k_max and mode
         self.batch_alloc = (batch_alloc and len(specs) <= binding.MPQ_MAX_BATCH and
@@ -200,6 +218,16 @@ class NetworkPlan:
                                             points_used=[p.points_used for p in self.plans],
                                             stream=stream)
 
+    def _host_counts(self):
+        """Pinned host copy of the count buffer, and every plan's host views into it."""
+        if self._counts_host is None:
+            self._counts_host = torch.empty(self.counts.shape, dtype=torch.int32, pin_memory=True)
+            for p, (a, b, u) in zip(self.plans, self._count_views):
+                h = p.host_buffers(counts=(self._counts_host[a:b], self._counts_host[u:u + 1]))
+                h["npoints"] = self._counts_host[a:b]            # also if made before
+                h["points_used"] = self._counts_host[u:u + 1]
+        return self._counts_host
+
     def _counts_out(self, p, h):
         with torch.cuda.stream(self.copy_out):
             h["npoints"].copy_(p.npoints, non_blocking=True)
@@ -220,6 +248,7 @@ class NetworkPlan:
         earlier call copied in (e.g. a second bit width over the same weights).  The caller
         synchronizes ``stream`` before reading the host outputs."""
         main = stream or torch.cuda.current_stream(self.device)
+        counts_host = self._host_counts()
         self._fork(main)
         for s in (self.copy_in, self.copy_out):
             s.wait_stream(main)
@@ -263,8 +292,11 @@ class NetworkPlan:
             done = torch.cuda.Event()
             done.record(main)
             self.copy_out.wait_event(done)
-            for i in self.order:
-                self._counts_out(self.plans[i], outs[i])
+            with torch.cuda.stream(self.copy_out):   # every layer's counts in one copy
+                counts_host.copy_(self.counts, non_blocking=True)
+                for p, h in zip(self.plans, outs):
+                    if p.center is not None:
+                        h["center"].copy_(p.center, non_blocking=True)
             self._fork(main)
             for n, i in enumerate(self.order):
                 self.plans[i].run_reconstruct(self.streams[n % len(self.streams)])
