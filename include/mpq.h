@@ -45,7 +45,8 @@ typedef enum {
     MPQ_ERR_UNSUPPORTED = 3,  /* valid for the method but beyond this library's limits below */
     MPQ_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
     MPQ_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up (mpq_device_status) */
-    MPQ_ERR_NOMEM = 6         /* mpq_output_error's stream-ordered scratch allocation failed */
+    MPQ_ERR_NOMEM = 6,        /* mpq_output_error's stream-ordered scratch allocation failed */
+    MPQ_ERR_BOUNDS = 7        /* the checked build skipped an out-of-range access (mpq_device_status) */
 } mpq_status;
 
 /* Library limits. */
@@ -378,11 +379,29 @@ mpq_status mpq_multipoint_linear(const int8_t *X, int T, const mpq_packed_layout
 #define MPQ_TIMEOUT_DRAIN 0x100u        /* a wait for the kernel's own copies or MMAs also gave up */
 
 /*
+ * The checked build.  Compiled with -DMPQ_CHECK_BOUNDS (paper_2002_09049_gb300._build:
+ * build(checked=True) -> libmpq_checked.so), every kernel checks the indices it computes before
+ * it uses them: each global store against the extent its arguments give the output, the
+ * data-dependent shared-memory indices (lattice buckets, event bins, queue slots, sort keys)
+ * against their arrays, the carve-up of dynamic shared memory against the launch's share, and
+ * every tile copy's coordinates against the rule that its first element be 16-byte aligned.  A
+ * failed check is counted and the access skipped -- the kernel never traps -- so a bad index
+ * shows as MPQ_FAULT_BOUNDS from mpq_device_status (with the first failing source line in
+ * mpq_last_error) and as wrong or NaN outputs, never as a fault.  A skipped tile copy leaves its
+ * barrier unsatisfied, so that kernel's bounded wait gives up too (MPQ_TIMEOUT_*).  The checks
+ * cost time: the checked build is for tests, the normal build's kernels carry none.
+ */
+#define MPQ_FAULT_BOUNDS 0x10000u        /* mpq_device_status: the checked build skipped accesses */
+#define MPQ_BUILD_CHECK_BOUNDS 0x1u      /* mpq_build_options: this is the checked build */
+
+/*
  * mpq_device_status -- synchronizes `stream`, then takes the current device's timeout word
- * (reads and clears it in one atomic exchange on the device): MPQ_OK if no bounded wait gave up
- * since the last call, else MPQ_ERR_TIMEOUT with the MPQ_TIMEOUT_* bits in *flags (nullable; 0 on
- * MPQ_OK).  It covers the kernels that have finished when the exchange runs: synchronize the
- * other streams first to include their calls.  Synchronous.
+ * (reads and clears it in one atomic exchange on the device), and in the checked build every
+ * kernel unit's count of skipped accesses likewise: MPQ_OK if no bounded wait gave up and no
+ * check failed since the last call; else MPQ_ERR_TIMEOUT if a wait gave up (it takes precedence),
+ * else MPQ_ERR_BOUNDS.  *flags (nullable; 0 on MPQ_OK) receives the MPQ_TIMEOUT_* bits, plus
+ * MPQ_FAULT_BOUNDS if a check failed.  It covers the kernels that have finished when the exchange
+ * runs: synchronize the other streams first to include their calls.  Synchronous.
  */
 mpq_status mpq_device_status(void *stream, unsigned *flags);
 
@@ -401,6 +420,9 @@ mpq_status mpq_set_wait_limit(long long clocks);
  * through mpq_device_status.  Off (0) by default; never on outside tests of the timeout path.
  */
 mpq_status mpq_test_withhold_copies(int on);
+
+/* MPQ_BUILD_* bits of the options this library was compiled with (0 for the normal build). */
+unsigned mpq_build_options(void);
 
 /* Name of a status code (static string). */
 const char *mpq_status_string(mpq_status s);

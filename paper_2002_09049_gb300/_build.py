@@ -2,6 +2,8 @@
 
 Translation units compile in parallel, then link into one shared library with the CUDA runtime
 linked statically.  Run ``python -m paper_2002_09049_gb300._build`` or call ``build()``.
+``build(checked=True)`` (``--checked``) builds the checked library, libmpq_checked.so: the same
+sources with -DMPQ_CHECK_BOUNDS, whose kernels count and skip out-of-range accesses.
 """
 from __future__ import annotations
 
@@ -17,6 +19,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmpq.so")
+CHECKED_LIB = os.path.join(PKG, "libmpq_checked.so")
 ROOT = os.path.dirname(PKG)
 INCLUDE = os.path.join(ROOT, "include")
 
@@ -41,24 +44,30 @@ def _deps():
     return _sources() + glob.glob(os.path.join(CSRC, "*.cuh")) + [os.path.join(INCLUDE, "mpq.h")]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(lib: str = LIB) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
-    """Compile csrc/*.cu -> libmpq.so (skipped when up to date).  Returns the library path."""
+def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False,
+          checked: bool = False) -> str:
+    """Compile csrc/*.cu -> libmpq.so, or with checked=True -> libmpq_checked.so (skipped when
+    up to date).  Returns the library path."""
+    lib = CHECKED_LIB if checked else LIB
+    obj_dir = os.path.join(BUILD, "checked") if checked else BUILD
     with _lock:
-        if not force and up_to_date():
-            return LIB
-        os.makedirs(BUILD, exist_ok=True)
+        if not force and up_to_date(lib):
+            return lib
+        os.makedirs(obj_dir, exist_ok=True)
         exe = nvcc()
         extra = ["-Xptxas", "-v"] if ptxas_info else []
+        if checked:
+            extra += ["-DMPQ_CHECK_BOUNDS"]
 
         def compile_one(src):
-            obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+            obj = os.path.join(obj_dir, os.path.basename(src)[:-3] + ".o")
             cmd = [exe, *ARCH, *NVCC_FLAGS, *extra, "-c", src, "-o", obj]
             res = subprocess.run(cmd, capture_output=True, text=True)
             if res.returncode != 0:
@@ -69,14 +78,15 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
 
         with ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 4)) as ex:
             objs = list(ex.map(compile_one, _sources()))
-        tmp = LIB + f".{os.getpid()}.tmp"
+        tmp = lib + f".{os.getpid()}.tmp"
         cmd = [exe, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
             raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")
-        os.replace(tmp, LIB)
-        return LIB
+        os.replace(tmp, lib)
+        return lib
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose=True, ptxas_info="--ptxas" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose=True, ptxas_info="--ptxas" in sys.argv,
+                checked="--checked" in sys.argv))

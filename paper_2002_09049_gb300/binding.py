@@ -26,10 +26,12 @@ MPQ_TIMEOUT_OUTPUT_ERROR = 0x1        # timeout bits of mpq_device_status
 MPQ_TIMEOUT_CLIP = 0x2
 MPQ_TIMEOUT_INFERENCE = 0x4
 MPQ_TIMEOUT_DRAIN = 0x100
+MPQ_FAULT_BOUNDS = 0x10000            # mpq_device_status: the checked build skipped accesses
+MPQ_BUILD_CHECK_BOUNDS = 0x1          # mpq_build_options: the checked build
 
 MPQ_STATUS = {0: "MPQ_OK", 1: "MPQ_ERR_INVALID_ARG", 2: "MPQ_ERR_NONFINITE",
               3: "MPQ_ERR_UNSUPPORTED", 4: "MPQ_ERR_CUDA", 5: "MPQ_ERR_TIMEOUT",
-              6: "MPQ_ERR_NOMEM"}
+              6: "MPQ_ERR_NOMEM", 7: "MPQ_ERR_BOUNDS"}
 
 # name -> (argtypes, restype), in the order of include/mpq.h
 _P, _I, _D = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
@@ -63,6 +65,7 @@ SIGNATURES = {
     "mpq_device_status": ([_P, _P], _I),
     "mpq_set_wait_limit": ([ctypes.c_longlong], _I),
     "mpq_test_withhold_copies": ([_I], _I),
+    "mpq_build_options": ([], ctypes.c_uint),
     "mpq_status_string": ([_I], ctypes.c_char_p),
     "mpq_last_error": ([], ctypes.c_char_p),
     "mpq_version": ([], _I),
@@ -82,11 +85,12 @@ def lib_path() -> str:
 
 
 def load(path: str | None = None):
-    """Loads libmpq.so (built by __graft_entry__.build() / paper_2002_09049_gb300._build)."""
+    """Loads libmpq.so (built by __graft_entry__.build() / paper_2002_09049_gb300._build), or the
+    library the MPQ_LIBRARY environment variable names (the checked build, libmpq_checked.so)."""
     global _lib
     if _lib is not None and path is None:
         return _lib
-    p = path or _build.LIB
+    p = path or os.environ.get("MPQ_LIBRARY") or _build.LIB
     if not os.path.exists(p):
         raise RuntimeError(f"{p} is missing: build it with paper_2002_09049_gb300._build.build() "
                            "(there is no CPU fallback)")
@@ -423,13 +427,23 @@ def mpq_version() -> int:
 
 
 def mpq_device_status(stream=None):
-    """Synchronizes the stream and takes the current device's timeout word: 0 if no bounded wait
-    of a tensor-core kernel gave up since the last call, else the MPQ_TIMEOUT_* bits."""
+    """Synchronizes the stream and takes the current device's timeout word (and, in the checked
+    build, the bounds-check counts): 0 if no bounded wait of a tensor-core kernel gave up and no
+    check failed since the last call, else the MPQ_TIMEOUT_* bits | MPQ_FAULT_BOUNDS."""
     flags = ctypes.c_uint(0)
     st = load().mpq_device_status(_stream(stream), ctypes.byref(flags))
-    if st not in (0, 5):
+    if st not in (0, 5, 7):
         _check(st, "mpq_device_status")
     return int(flags.value)
+
+
+def mpq_build_options() -> int:
+    """MPQ_BUILD_* bits of the loaded library (MPQ_BUILD_CHECK_BOUNDS for the checked build)."""
+    return int(load().mpq_build_options())
+
+
+def mpq_last_error() -> str:
+    return load().mpq_last_error().decode(errors="replace")
 
 
 def mpq_set_wait_limit(clocks: int):

@@ -32,6 +32,8 @@
 
 #include "mpq_internal.cuh"
 
+MPQ_CHECKED_UNIT("adaptive.cu");
+
 namespace mpq {
 namespace {
 
@@ -202,7 +204,8 @@ __device__ uint2 *ad_sort(uint2 *a, uint2 *b, int n, ASort &st)
             if (i < w1) e = a[i];
             const unsigned dg = i < w1 ? (e.x >> shift) & 255u : 256u;
             const unsigned m = __match_any_sync(0xffffffffu, dg);
-            if (dg < 256u) b[st.hist[w][dg] + __popc(m & lt)] = e;
+            if (dg < 256u && MPQ_IN(st.hist[w][dg] + __popc(m & lt), n))
+                b[st.hist[w][dg] + __popc(m & lt)] = e;
             __syncwarp();
             if (dg < 256u && (m & lt) == 0u) st.hist[w][dg] += __popc(m);
             __syncwarp();
@@ -382,13 +385,16 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
     uint2 *bufB = bufA + cap;
     double *sq = reinterpret_cast<double *>(bufB);   // r_j^2 for the serial sum (cap >= d)
     const size_t plane = (size_t)C * d;
+    const size_t n_codes = (size_t)k_max * plane, n_sc = (size_t)C * k_max;
+    const size_t n_rs = (size_t)C * (k_max + 1);
+    if (!MPQ_CHECK_SMEM_END(4 * (size_t)d) || !MPQ_CHECK(d <= cap)) return;
 
     for (int k = blockIdx.x; k < C; k += gridDim.x) {
         if (t == 0) sh.finite = 1;
         __syncthreads();
         int fin = 1;
         for (int j = t; j < d; j += AT) {
-            const float v = W[(size_t)k * d + j];
+            const float v = MPQ_IN((size_t)k * d + j, plane) ? W[(size_t)k * d + j] : 0.0f;
             r[j] = v;
             sq[j] = __dmul_rn((double)v, (double)v);   // exact: 24-bit times 24-bit
             fin &= isfinite(v);
@@ -399,7 +405,8 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
             const double r2 = ad_serial_sum(sq, d);
             sh.r2 = r2;
             sh.state = sh.finite ? 0 : 2;
-            if (resid_sq) resid_sq[(size_t)k * (k_max + 1)] = sh.finite ? (float)r2 : NAN;
+            if (resid_sq && MPQ_IN((size_t)k * (k_max + 1), n_rs))
+                resid_sq[(size_t)k * (k_max + 1)] = sh.finite ? (float)r2 : NAN;
         }
         __syncthreads();
         bool dead = sh.state == 2;
@@ -477,8 +484,10 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                 }
             }
             if (dead) {
-                for (int j = t; j < d; j += AT) qi[j] = 0;
-                if (t == 0) {
+                for (int j = t; j < d; j += AT)
+                    if (MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes)) qi[j] = 0;
+                if (t == 0 && MPQ_IN((size_t)k * k_max + i, n_sc) &&
+                    MPQ_IN((size_t)k * (k_max + 1) + i + 1, n_rs)) {
                     scales[(size_t)k * k_max + i] = NAN;
                     if (ncand) ncand[(size_t)k * k_max + i] = refused_now ? -1 : 0;
                     if (resid_sq) resid_sq[(size_t)k * (k_max + 1) + i + 1] = NAN;
@@ -506,7 +515,9 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                         const float tau = ad_threshold(a, L);
                         if (!(tau >= spos)) break;   // tau is non-increasing in L
                         const int pos = atomicAdd(&sh.nev, 1);
-                        bufA[pos] = make_uint2(__float_as_uint(tau), ((unsigned)j << 8) | (unsigned)L);
+                        if (MPQ_IN(pos, cap))
+                            bufA[pos] = make_uint2(__float_as_uint(tau),
+                                                   ((unsigned)j << 8) | (unsigned)L);
                         p0 += R;
                         n0 += 2 * L - 1;
                     }
@@ -530,7 +541,8 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                     N0 += sh.part[x][1];
                 }
                 __syncthreads();
-                const int n = sh.nev;
+                int n = sh.nev;
+                if (!MPQ_CHECK(n <= cap)) n = cap;
                 const uint2 *ev = ad_sort(bufA, bufB, n, sh.sort);
                 // ---- pieces e = 0..n: scales (lo, hi] with the first e thresholds passed
                 const int chunk = (n + 1 + AT - 1) / AT;
@@ -538,6 +550,7 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                 long long pre_p = 0, pre_n = 0;
                 for (int x = e0; x < min(e1, n); ++x) {
                     const unsigned v = ev[x].y;
+                    if (!MPQ_IN(v >> 8, d)) continue;
                     pre_p += ad_fixed(fabsf(r[v >> 8]), S);
                     pre_n += 2 * (int)(v & 255u) - 1;
                 }
@@ -550,6 +563,7 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                 auto advance = [&](int x, long long &cp, long long &cn) {
                     if (x < n) {
                         const unsigned v = ev[x].y;
+                        if (!MPQ_IN(v >> 8, d)) return;
                         cp += ad_fixed(fabsf(r[v >> 8]), S);
                         cn += 2 * (int)(v & 255u) - 1;
                     }
@@ -651,18 +665,21 @@ adaptive_kernel(const float *__restrict__ W, int C, int d, int qmax, int k_max, 
                 const float v = r[j];
                 int q = ad_code_mag(fabsf(v), sbest, qmax);
                 q = v < 0.0f ? -q : q;
-                qi[j] = (int8_t)q;
+                if (MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes)) qi[j] = (int8_t)q;
                 const float nv = __fmaf_rn(-sbest, (float)q, v);
                 r[j] = nv;
                 sq[j] = __dmul_rn((double)nv, (double)nv);
             }
             __syncthreads();
             if (t == 0) {
-                scales[(size_t)k * k_max + i] = sbest;
-                if (ncand) ncand[(size_t)k * k_max + i] = sh.M;
+                if (MPQ_IN((size_t)k * k_max + i, n_sc)) {
+                    scales[(size_t)k * k_max + i] = sbest;
+                    if (ncand) ncand[(size_t)k * k_max + i] = sh.M;
+                }
                 const double r2 = ad_serial_sum(sq, d);
                 sh.r2 = r2;
-                if (resid_sq) resid_sq[(size_t)k * (k_max + 1) + i + 1] = (float)r2;
+                if (resid_sq && MPQ_IN((size_t)k * (k_max + 1) + i + 1, n_rs))
+                    resid_sq[(size_t)k * (k_max + 1) + i + 1] = (float)r2;
             }
             __syncthreads();
         }

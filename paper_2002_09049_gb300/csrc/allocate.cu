@@ -17,6 +17,8 @@
 
 #include "mpq_internal.cuh"
 
+MPQ_CHECKED_UNIT("allocate.cu");
+
 namespace mpq {
 namespace {
 
@@ -63,6 +65,8 @@ __device__ __forceinline__ void allocate_budget_cta(const float *__restrict__ er
     __shared__ int s_done, s_used;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int KM1 = k_max - 1;
+    // the cached keys within the launch's shared memory, else read again from err
+    if (cached && !MPQ_CHECK_SMEM_END(8 * (size_t)C * KM1)) cached = false;
 
     if (tid == 0) {
         s_total = 0;
@@ -234,6 +238,7 @@ __global__ void __launch_bounds__(AB_THREADS)
 allocate_batch_kernel(const __grid_constant__ AllocBatch b, int k_max, int mode)
 {
     extern __shared__ unsigned long long skeys[];
+    if (!MPQ_IN(blockIdx.x, MPQ_MAX_BATCH) || !MPQ_IN(b.order[blockIdx.x], MPQ_MAX_BATCH)) return;
     const int l = b.order[blockIdx.x];
     if (mode == MPQ_ALLOC_BUDGET)
         allocate_budget_cta(b.err[l], b.C[l], k_max, b.extra[l], b.npoints[l], b.points_used[l],

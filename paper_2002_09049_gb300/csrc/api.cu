@@ -434,6 +434,7 @@ extern "C" const char *mpq_status_string(mpq_status s)
     case MPQ_ERR_CUDA: return "MPQ_ERR_CUDA";
     case MPQ_ERR_TIMEOUT: return "MPQ_ERR_TIMEOUT";
     case MPQ_ERR_NOMEM: return "MPQ_ERR_NOMEM";
+    case MPQ_ERR_BOUNDS: return "MPQ_ERR_BOUNDS";
     }
     return "MPQ_ERR_UNKNOWN";
 }

@@ -8,6 +8,8 @@
 
 #include "mpq_internal.cuh"
 
+MPQ_CHECKED_UNIT("center.cu");
+
 namespace mpq {
 namespace {
 
@@ -71,7 +73,8 @@ center_channel_kernel(const float *__restrict__ W, int C, int d, int pass, float
         if (lane == 0) center[k] = b;
     }
     float *out = Wc + (size_t)k * d;
-    for (int j = lane; j < d; j += 32) out[j] = __fsub_rn(w[j], b);
+    for (int j = lane; j < d; j += 32)
+        if (MPQ_IN((size_t)k * d + j, (size_t)C * d)) out[j] = __fsub_rn(w[j], b);
 }
 
 // One CTA: the layer's B from the channels' ranges, written to every center[k].

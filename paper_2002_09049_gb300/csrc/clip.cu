@@ -18,6 +18,8 @@
 #include "mpq_internal.cuh"
 #include "rounding.cuh"
 
+MPQ_CHECKED_UNIT("clip.cu");
+
 namespace mpq {
 namespace {
 
@@ -103,6 +105,7 @@ clip_errors_kernel(const float *__restrict__ X, int N, int groups, const float *
     __shared__ float red[CL_THREADS / 32][CL_CHUNK];
     const int k = blockIdx.x, c0 = blockIdx.y * CL_CHUNK;
     const int nc = min(CL_CHUNK, n_cand - c0);
+    if (!MPQ_IN(k, C) || !MPQ_CHECK(nc >= 1) || !MPQ_CHECK_SMEM_END(4 * (size_t)nc * d)) return;
     const float qmaxf = (float)qmax;
     const float *w = W + (size_t)k * d;
     for (int i = threadIdx.x; i < nc * d; i += CL_THREADS) {
@@ -160,7 +163,8 @@ clip_errors_kernel(const float *__restrict__ X, int N, int groups, const float *
         for (int i = 0; i < CL_THREADS / 32; ++i) v[i] = red[i][threadIdx.x];
         for (int w = CL_THREADS / 64; w > 0; w >>= 1)   // tree over the warps
             for (int i = 0; i < w; ++i) v[i] += v[i + w];
-        err[(size_t)k * n_cand + c0 + threadIdx.x] = mean_of_sum(v[0], N);
+        if (MPQ_IN((size_t)k * n_cand + c0 + threadIdx.x, (size_t)C * n_cand))
+            err[(size_t)k * n_cand + c0 + threadIdx.x] = mean_of_sum(v[0], N);
     }
 }
 

@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "checks.cuh"
 #include "mpq.h"
 
 namespace mpq {

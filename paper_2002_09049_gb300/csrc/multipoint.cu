@@ -44,6 +44,8 @@
 #include "tf32_operands.cuh"
 #include "waits.cuh"
 
+MPQ_CHECKED_UNIT("multipoint.cu");
+
 namespace mpq {
 namespace {
 
@@ -148,7 +150,7 @@ __global__ void pack_kernel(const int8_t *__restrict__ codes, const float *__res
 {
     const int r = blockIdx.x;
     const int k = v.chan[r], i = v.point[r];
-    const bool live = k >= 0 && i >= 0;
+    const bool live = k >= 0 && i >= 0 && MPQ_IN(k, C) && MPQ_IN(i, k_max);
     if (threadIdx.x == 0) v.coef[r] = live ? fixed_coeff(scales[(size_t)k * k_max + i], p, v.flag) : 0;
     const int8_t *q = live ? codes + (size_t)i * C * d + (size_t)k * d : nullptr;
     for (int j = threadIdx.x; j < d_pad; j += blockDim.x)
@@ -165,7 +167,7 @@ __device__ __forceinline__ uint32_t bf16x2_from_biased(uint32_t biased, int b0)
 
 template <int RT>
 __global__ void __launch_bounds__(L_THREADS, 1)
-multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restrict__ coef,
+multipoint_linear_kernel(int T, int C, int tiles, int n_kc, int p, const int *__restrict__ coef,
                          const int *__restrict__ chan, const int *__restrict__ tile_R,
                          const int *__restrict__ center_coef,
                          int32_t *__restrict__ Y, const WaitCtl wc,
@@ -185,6 +187,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
     // inputs vary fastest: the CTAs sharing a row tile run together and read its codes from L2
     const int tile0 = blockIdx.y * RT, n0 = blockIdx.x * L_N;
     const int nt = min(RT, tiles - tile0);          // row tiles of this CTA (the last may hold one)
+    if (!MPQ_CHECK_SMEM_END((size_t)pad + L_CTRL_BYTES + (size_t)G::BYTES)) return;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < G::A_SLOTS; ++i) {
@@ -302,7 +305,8 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
             const int r = ew * 32 + lane;
             const int k = chan[(size_t)(tile0 + u) * L_M + r];
             const long long a = ctl.coef[u][r];
-            const long long ab = centered && k >= 0 ? (long long)center_coef[k] : 0;
+            const long long ab =
+                centered && k >= 0 && MPQ_IN(k, C) ? (long long)center_coef[k] : 0;
             const uint32_t lane_base = tmem + ((uint32_t)(ew * 32) << 16) + (uint32_t)(u * L_N);
             // the rows this warp writes: one per channel (its first lane), -1 for none
             ctl.kch[ew][lane] = (lane & (R - 1)) == 0 ? k : -1;
@@ -348,7 +352,7 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                 if (t < T) {
 #pragma unroll
                     for (int L = 0; L < 32; ++L)
-                        if (kv[L] >= 0) Y[(size_t)kv[L] * T + t] = ov[L];
+                        if (kv[L] >= 0 && MPQ_IN(kv[L], C)) Y[(size_t)kv[L] * T + t] = ov[L];
                 }
             }
         }
@@ -395,6 +399,11 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                     note_timeout(wc, MPQ_TIMEOUT_INFERENCE);
                 }
                 if (*abort_flag) break;
+                // 16-byte aligned tile copies (bf16 codes: x a multiple of 8)
+                if (!MPQ_CHECK(((kc * L_KC) & 7) == 0 && ((a_u32 + as * G::A_SLOT) & 15u) == 0u)) {
+                    *abort_flag = 1;
+                    break;
+                }
                 mbar_arrive_expect_tx(&ctl.a_full[as], (uint32_t)(nt * L_A_BYTES));
                 for (int u = 0; u < nt; ++u)
                     tma_load_2d(a_u32 + as * G::A_SLOT + u * L_A_BYTES, &tmA, kc * L_KC,
@@ -420,6 +429,11 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
                     note_timeout(wc, MPQ_TIMEOUT_INFERENCE);
                 }
                 if (*abort_flag) break;
+                // 16-byte aligned tile copies (int8 inputs: x a multiple of 16)
+                if (!MPQ_CHECK(((kc * L_KC) & 15) == 0 && ((x_u32 + rs * L_RAW_BYTES) & 15u) == 0u)) {
+                    *abort_flag = 1;
+                    break;
+                }
                 mbar_arrive_expect_tx(&ctl.r_full[rs], (uint32_t)L_RAW_BYTES);
                 tma_load_2d(x_u32 + rs * L_RAW_BYTES, &tmX, kc * L_KC, n0, &ctl.r_full[rs]);
                 issued = kc + 1;
@@ -442,7 +456,8 @@ multipoint_linear_kernel(int T, int tiles, int n_kc, int p, const int *__restric
 }
 
 // The same integer arithmetic on CUDA cores: one thread per (channel, input).
-__global__ void multipoint_linear_simt(const int8_t *__restrict__ X, int T, int d, int d_pad, int rows,
+__global__ void multipoint_linear_simt(const int8_t *__restrict__ X, int T, int C, int d, int d_pad,
+                                       int rows,
                                        int p, const int *__restrict__ coef,
                                        const int *__restrict__ chan,
                                        const __nv_bfloat16 *__restrict__ codes,
@@ -455,7 +470,7 @@ __global__ void multipoint_linear_simt(const int8_t *__restrict__ X, int T, int 
     const int R = tile_R[slot_row / L_M];
     if (slot_row % R != 0) return;
     const int k = chan[slot_row];
-    if (k < 0) return;
+    if (k < 0 || !MPQ_IN(k, C)) return;
     const int8_t *x = X + (size_t)t * d;
     long long sum = 0;
     for (int i = 0; i < R; ++i) {
@@ -652,14 +667,14 @@ mpq_status launch_multipoint_linear(const int8_t *X, int T, const mpq_packed_lay
         WaitCtl wc;
         const mpq_status wst = wait_ctl(&wc);
         if (wst != MPQ_OK) return wst;
-        kernel<<<grid, L_THREADS, smem, stream>>>(T, L->tiles, L->d_pad / L_KC, L->p, v.coef,
+        kernel<<<grid, L_THREADS, smem, stream>>>(T, L->C, L->tiles, L->d_pad / L_KC, L->p, v.coef,
                                                   v.chan, v.tile_R, v.center, Y, wc, tmA, tmX);
         return cuda_status(cudaGetLastError(), "multipoint linear kernel launch");
     }
     const size_t n = (size_t)L->rows * T;
     if (n == 0) return MPQ_OK;
     multipoint_linear_simt<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(
-        X, T, d, L->d_pad, L->rows, L->p, v.coef, v.chan, v.codes, v.tile_R, v.center, Y);
+        X, T, L->C, d, L->d_pad, L->rows, L->p, v.coef, v.chan, v.codes, v.tile_R, v.center, Y);
     return cuda_status(cudaGetLastError(), "multipoint linear (integer) kernel launch");
 }
 

@@ -12,6 +12,8 @@
 
 #include "mpq_internal.cuh"
 
+MPQ_CHECKED_UNIT("output_error.cu");
+
 namespace mpq {
 namespace {
 
@@ -31,6 +33,10 @@ output_error_grouped_kernel(const float *__restrict__ X, int N, const float *__r
     const int tid = threadIdx.x;
     const int k_max = KP1 - 1;
     const size_t plane = (size_t)C * d;
+    // the residual rows and one staged chunk of X within the launch's shared memory
+    if (!MPQ_IN(k, C) || !MPQ_CHECK(d <= GR_X_FLOATS) ||
+        !MPQ_CHECK_SMEM_END(4 * ((size_t)((KP1 * d + 3) & ~3) + GR_X_FLOATS)))
+        return;
 
     for (int j = tid; j < d; j += GR_THREADS) {
         float r = W[(size_t)k * d + j];
@@ -100,7 +106,8 @@ output_error_grouped_kernel(const float *__restrict__ X, int N, const float *__r
         for (int i = 0; i < GR_THREADS / 32; ++i) v[i] = red[i][tid];
         for (int w = GR_THREADS / 64; w > 0; w >>= 1)   // tree over the warps
             for (int i = 0; i < w; ++i) v[i] += v[i + w];
-        err[(size_t)k * KP1 + tid] = mean_of_sum(v[0], N);
+        if (MPQ_IN((size_t)k * KP1 + tid, (size_t)C * KP1))
+            err[(size_t)k * KP1 + tid] = mean_of_sum(v[0], N);
     }
 }
 

@@ -50,6 +50,8 @@
 #include "tf32_operands.cuh"
 #include "waits.cuh"
 
+MPQ_CHECKED_UNIT("output_error_pair.cu");
+
 namespace mpq {
 namespace {
 
@@ -358,6 +360,11 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
     const int n_kc = (d + P_KC - 1) / P_KC;
     const int nseg = (n_kc + SEG - 1) / SEG;
     const int total = my_rt * n_kc;
+    // control block, tile sets and the raw-tile ring within the launch's shared memory (the same
+    // in every CTA, so the whole cluster leaves together)
+    if (!MPQ_CHECK_SMEM_END((size_t)pad + P_CTRL_BYTES + (size_t)P_TILE_SETS * P_STAGE_BYTES +
+                            (size_t)R * G::RAW_BYTES))
+        return;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NST; ++s) {
@@ -383,6 +390,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         }
     } else {
         for (int i = threadIdx.x; i < nvec; i += PR::THREADS) {
+            if (!MPQ_IN((size_t)k0 * KP1 + i, (size_t)C * KP1)) continue;
             const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * KP1 + i)));
             ctl.vexp[i] = e;
             ctl.vscale[i] = pow2f(e);
@@ -571,6 +579,13 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 const uint32_t dst = ring_u32 + slot * G::RAW_BYTES;
                 const int x = (f % n_kc) * P_KC;
                 const int row0 = (pr + (f / n_kc) * split) * P_N + half * P_ROWS;
+                // a tile copy starts 16-byte aligned (x counts int8 codes in the code map) into a
+                // 16-byte aligned destination; a copy that would not is not issued, and the
+                // consumers' bounded waits end the launch
+                if (!MPQ_CHECK((x & 15) == 0 && (dst & 15u) == 0u && x < d)) {
+                    *abort_flag = 1;
+                    break;
+                }
                 mbar_arrive_expect_tx(&ctl.raw_full[slot], G::RAW_TX);
                 tma_load_2d(dst, &tmX, x, row0, &ctl.raw_full[slot]);
                 tma_load_2d(dst + G::RAW_W, &tmW, x, k0, &ctl.raw_full[slot]);
@@ -596,7 +611,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             }
             double v = s / (double)N;
             if (F16) v *= pow2d(-2 * (ctl.xexp + ctl.vexp[m]));   // exact: undo the operand scales
-            err[(size_t)k0 * KP1 + m] = (float)v;
+            if (MPQ_IN((size_t)k0 * KP1 + m, (size_t)C * KP1)) err[(size_t)k0 * KP1 + m] = (float)v;
         }
     }
     cluster_sync();
@@ -659,6 +674,9 @@ pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const flo
     const int gw = ((int)blockIdx.x - xb) * 8 + warp;
     const int k = gw / split, part = gw - k * split;
     if (k >= C) return;
+    // 16-byte row loads and 4-byte code loads need d % 4 == 0 and aligned bases
+    if (!MPQ_CHECK((d & 3) == 0 && ((uintptr_t)W & 15) == 0 && ((uintptr_t)codes & 3) == 0))
+        return;
     float sc[K > 0 ? K : 1], mx[KP1];
 #pragma unroll
     for (int n = 0; n < K; ++n) sc[n] = __ldg(scales + (size_t)k * K + n);
@@ -678,7 +696,8 @@ pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const flo
     for (int n = 0; n < KP1; ++n) {
         float m = mx[n];
         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-        if (lane == 0) atomicMax(range + 1 + (size_t)k * KP1 + n, __float_as_uint(m));
+        if (lane == 0 && MPQ_IN((size_t)k * KP1 + n, (size_t)C * KP1))
+            atomicMax(range + 1 + (size_t)k * KP1 + n, __float_as_uint(m));
     }
 }
 

@@ -38,6 +38,8 @@
 #include "tf32_operands.cuh"
 #include "waits.cuh"
 
+MPQ_CHECKED_UNIT("output_error_tc.cu");
+
 namespace mpq {
 namespace {
 
@@ -82,7 +84,8 @@ constexpr int TC_SMEM = 1024 /* alignment slack */ + CTRL_BYTES + TC_STAGES * ST
 __device__ __forceinline__ float4 load4_guarded(const float *__restrict__ p, int j, int d,
                                                 bool vec_ok)
 {
-    if (vec_ok && j + 3 < d) return __ldg(reinterpret_cast<const float4 *>(p + j));
+    if (vec_ok && j + 3 < d && MPQ_CHECK(((uintptr_t)(p + j) & 15) == 0))
+        return __ldg(reinterpret_cast<const float4 *>(p + j));
     float4 v;
     v.x = (j + 0 < d) ? __ldg(p + j + 0) : 0.0f;
     v.y = (j + 1 < d) ? __ldg(p + j + 1) : 0.0f;
@@ -95,7 +98,8 @@ __device__ __forceinline__ float4 load4_guarded(const float *__restrict__ p, int
 __device__ __forceinline__ uint32_t codes4_guarded(const int8_t *__restrict__ p, int j, int d,
                                                    bool vec_ok)
 {
-    if (vec_ok && j + 3 < d) return __ldg(reinterpret_cast<const unsigned int *>(p + j));
+    if (vec_ok && j + 3 < d && MPQ_CHECK(((uintptr_t)(p + j) & 3) == 0))
+        return __ldg(reinterpret_cast<const unsigned int *>(p + j));
     uint32_t w = 0;
 #pragma unroll
     for (int b = 0; b < 4; ++b)
@@ -222,6 +226,8 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
     const int nseg = (n_kc + SEG_CHUNKS - 1) / SEG_CHUNKS;
     const int total = my_rt * n_kc;
     const size_t plane = (size_t)C * d;
+    // control block and stages within the launch's shared memory (uniform over the cluster)
+    if (!MPQ_CHECK_SMEM_END((size_t)pad + CTRL_BYTES + (size_t)TC_STAGES * STAGE_BYTES)) return;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < TC_STAGES; ++s) {
@@ -385,7 +391,8 @@ output_error_tc_kernel(const float *__restrict__ X, int N, const float *__restri
             if (m < nvec) {
                 double s = 0.0;
                 for (int c = 0; c < split; ++c) s += ld_dsmem_f64(&ctl.part[m], (uint32_t)c);
-                err[(size_t)k0 * KP1 + m] = (float)(s / (double)N);
+                if (MPQ_IN((size_t)k0 * KP1 + m, (size_t)C * KP1))
+                    err[(size_t)k0 * KP1 + m] = (float)(s / (double)N);
             }
         }
     }

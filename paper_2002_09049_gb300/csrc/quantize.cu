@@ -39,6 +39,8 @@
 #include "mpq_internal.cuh"
 #include "rounding.cuh"
 
+MPQ_CHECKED_UNIT("quantize.cu");
+
 namespace mpq {
 namespace {
 
@@ -423,8 +425,9 @@ __device__ __forceinline__ void add64(unsigned int *lo_word, unsigned int *hi_wo
 }
 
 __device__ __forceinline__ void add_event(unsigned int *hLo, unsigned int *hHi, int *hN, int T,
-                                          unsigned int Rlo, unsigned int Rhi, int L)
+                                          unsigned int Rlo, unsigned int Rhi, int L, int G)
 {
+    if (!MPQ_IN(T, G + 1)) return;
     add64(&hLo[T], &hHi[T], Rlo, Rhi);
     atomicAdd(&hN[T], 2 * L - 1);
 }
@@ -473,6 +476,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             ftab[g] = f;
             ftab[G + g] = __frcp_rn(f);
         }
+    // the last group's region ends the carve-up of dynamic shared memory
+    if (!MPQ_CHECK_SMEM_END((TABLE ? 8 * (size_t)G : 0) + (LAT ? lut_bytes(nb) : 0) +
+                            4 * (size_t)GPC * group_words(G, d, COPIES, nc)))
+        return;
     auto fg = [&](int g) -> float { return TABLE ? ftab[g] : grid.frac(g, G); };
     auto fi = [&](int g) -> float { return TABLE ? ftab[G + g] : __frcp_rn(grid.frac(g, G)); };
     // Lattice compression: only the positions (g+1)(2L-1) are read, so bucket b is stored at the
@@ -484,7 +491,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
         __syncthreads();
         for (int x = threadIdx.x; x < G * qmax; x += QTHREADS) {
             const int g = x / qmax, L = x - g * qmax + 1;
-            lut[(g + 1) * (2 * L - 1)] = 1;
+            if (MPQ_IN((g + 1) * (2 * L - 1), nb)) lut[(g + 1) * (2 * L - 1)] = 1;
         }
         __syncthreads();
         if (warp == 0) {   // inclusive count of positions, minus one
@@ -528,7 +535,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
     int bad = 0;
     float ssum = 0.0f, scomp = 0.0f, am = 0.0f;
     for (int j = gt; j < d; j += NT) {
-        const float v = w[j];
+        const float v = MPQ_IN((size_t)k * d + j, plane) ? w[j] : 0.0f;
         sr[j] = v;
         bad |= !isfinite(v);
         kahan_add(ssum, scomp, v * v);
@@ -538,21 +545,27 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
     float r2 = ssum;
     group_max_sum_or<WPC>(m, r2, bad, sc, gw, lane, grp);
     if (WPC == 1) __syncwarp();
-    if (resid_sq && gt == 0) resid_sq[(size_t)k * (k_max + 1)] = bad ? NAN : r2;
-    if (rmax && gt == 0) rmax[(size_t)k * (k_max + 1)] = bad ? NAN : m;
+    const size_t n_rs = (size_t)C * (k_max + 1), n_codes = (size_t)k_max * plane;
+    if (resid_sq && gt == 0 && MPQ_IN((size_t)k * (k_max + 1), n_rs))
+        resid_sq[(size_t)k * (k_max + 1)] = bad ? NAN : r2;
+    if (rmax && gt == 0 && MPQ_IN((size_t)k * (k_max + 1), n_rs))
+        rmax[(size_t)k * (k_max + 1)] = bad ? NAN : m;
 
     for (int i = 0; i < k_max; ++i) {
         int8_t *qi = codes + (size_t)i * plane + (size_t)k * d;
         float *ri = residuals ? residuals + (size_t)i * plane + (size_t)k * d : nullptr;
         if (bad) {
             for (int j = gt; j < d; j += NT) {
+                if (!MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes)) continue;
                 qi[j] = 0;
                 if (ri) ri[j] = sr[j];
             }
             if (gt == 0) {
-                scales[(size_t)k * k_max + i] = NAN;
-                if (resid_sq) resid_sq[(size_t)k * (k_max + 1) + i + 1] = NAN;
-                if (rmax) rmax[(size_t)k * (k_max + 1) + i + 1] = NAN;
+                const bool in_s = MPQ_IN((size_t)k * k_max + i, (size_t)C * k_max);
+                const bool in_r = MPQ_IN((size_t)k * (k_max + 1) + i + 1, n_rs);
+                if (in_s) scales[(size_t)k * k_max + i] = NAN;
+                if (resid_sq && in_r) resid_sq[(size_t)k * (k_max + 1) + i + 1] = NAN;
+                if (rmax && in_r) rmax[(size_t)k * (k_max + 1) + i + 1] = NAN;
             }
             continue;
         }
@@ -623,7 +636,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                         T = (int)fminf(fmaxf(fx, 1.0f), (float)(G - 1));
                         if (x - fx > tolx && fx + 1.0f - x > tolx && fx >= 1.0f &&
                             fx <= (float)(G - 1)) {
-                            add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
+                            add_event(hLo, hHi, hN, T, Rlo, Rhi, L, G);
                             return;
                         }
                     }
@@ -638,7 +651,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                         while (T > 1 && !MPQ_HELD(T - 1)) --T;
                     }
 #undef MPQ_HELD
-                    add_event(hLo, hHi, hN, T, Rlo, Rhi, L);
+                    add_event(hLo, hHi, hN, T, Rlo, Rhi, L, G);
                 };
                 // every level an element crosses inside the grid, one event each; the levels held
                 // at the largest scale go to the base sums
@@ -695,6 +708,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                                 const int b = (int)floorf(u2[u]);
                                 if (b >= 1) {
                                     const int bb = lut[b < nb - 1 ? b : nb - 1];
+                                    if (!MPQ_IN(bb, nc)) continue;
                                     // two 32-bit atomics: the low word's old value gives
                                     // its carry, which the high word takes with the count
                                     const unsigned long long R =
@@ -721,6 +735,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                         // (queued element, level) pairs over the group's threads
                         for (int it = gt; it < nq * qmax; it += NT) {
                             const int q = it / qmax, L = it - q * qmax + 1;
+                            if (!MPQ_IN(q, QNEAR)) continue;
                             const float a = sc.nearq[q];
                             const int c_hi = code_fast(a, s0, i0, qmaxf);
                             if (c_hi == 0) continue;
@@ -804,6 +819,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                         long long n = mN[g + 1];
                         for (int L = 1; L <= qmax; ++L) {
                             const int b = lut[(g + 1) * (2 * L - 1)];
+                            if (!MPQ_IN(b, nc)) continue;
                             const unsigned hi = lat[2 * b + 1];
                             p += (long long)(((unsigned long long)(hi & hmask) << 32) | lat[2 * b]);
                             n += (long long)(2 * L - 1) * (hi >> cnt_bit);
@@ -884,23 +900,26 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 q = (v < 0.0f) ? -c : c;
                 v = __fmaf_rn(-s_best, (float)q, v);
             }
-            qi[j] = (int8_t)q;
+            const bool in = MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes);
+            if (in) qi[j] = (int8_t)q;
             sr[j] = v;
-            if (ri) ri[j] = v;
+            if (ri && in) ri[j] = v;
             // ||r||^2: a thread's share of at most 64 squares summed plainly (relative error
             // below 2^-18 with the group's tree), longer shares compensated
             if (short_share) ssum = __fmaf_rn(v, v, ssum);
             else kahan_add(ssum, scomp, v * v);
             am = fmaxf(am, fabsf(v));
         }
-        if (gt == 0) scales[(size_t)k * k_max + i] = s_best;
+        if (gt == 0 && MPQ_IN((size_t)k * k_max + i, (size_t)C * k_max))
+            scales[(size_t)k * k_max + i] = s_best;
         m = am;
         r2 = ssum;
         int none = 0;
         group_max_sum_or<WPC>(m, r2, none, sc, gw, lane, grp);   // orders the sr[] writes too
         if (WPC == 1) __syncwarp();
-        if (resid_sq && gt == 0) resid_sq[(size_t)k * (k_max + 1) + i + 1] = r2;
-        if (rmax && gt == 0) rmax[(size_t)k * (k_max + 1) + i + 1] = m;
+        const bool in_r = MPQ_IN((size_t)k * (k_max + 1) + i + 1, n_rs);
+        if (resid_sq && gt == 0 && in_r) resid_sq[(size_t)k * (k_max + 1) + i + 1] = r2;
+        if (rmax && gt == 0 && in_r) rmax[(size_t)k * (k_max + 1) + i + 1] = m;
     }
 }
 

@@ -5,6 +5,8 @@
 // when d allows 16-byte stores.
 #include "mpq_internal.cuh"
 
+MPQ_CHECKED_UNIT("reconstruct.cu");
+
 namespace mpq {
 namespace {
 
@@ -20,6 +22,7 @@ reconstruct_kernel(const int8_t *__restrict__ codes, const float *__restrict__ s
     for (size_t idx = (size_t)blockIdx.x * RC_THREADS + threadIdx.x; idx < total;
          idx += (size_t)gridDim.x * RC_THREADS) {
         const int k = (int)(idx / d);
+        if (!MPQ_IN(k, C)) continue;
         int n = npoints[k];
         n = n < 0 ? 0 : (n > k_max ? k_max : n);
         float acc = center ? center[k] : 0.0f;
@@ -42,6 +45,10 @@ reconstruct_vec4_kernel(const int8_t *__restrict__ codes, const float *__restric
          q += (size_t)gridDim.x * RC_THREADS) {
         const size_t idx = q * 4;
         const int k = (int)(idx / d);
+        // four elements of one channel, 4-byte code and 16-byte output alignment
+        if (!MPQ_IN(k, C) || !MPQ_IN(idx + 3, plane) || !MPQ_CHECK(idx / d == (idx + 3) / d) ||
+            !MPQ_CHECK(((uintptr_t)codes & 3) == 0 && ((uintptr_t)(W_hat + idx) & 15) == 0))
+            continue;
         int n = npoints[k];
         n = n < 0 ? 0 : (n > k_max ? k_max : n);
         const float b = center ? center[k] : 0.0f;

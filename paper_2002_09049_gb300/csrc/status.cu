@@ -1,11 +1,15 @@
-// Device-side timeout reporting (include/mpq.h: mpq_device_status, mpq_set_wait_limit,
-// mpq_test_withhold_copies).  One word per device collects the MPQ_TIMEOUT_* bits of kernels whose
-// bounded waits gave up; mpq_device_status takes it (reads and clears it in one atomic exchange on
-// the device).  The word's device address is looked up once per device, with that device current,
-// and handed to every tensor-core launch.
+// Device-side status (include/mpq.h: mpq_device_status, mpq_set_wait_limit,
+// mpq_test_withhold_copies, mpq_build_options).  One word per device collects the MPQ_TIMEOUT_*
+// bits of kernels whose bounded waits gave up; mpq_device_status takes it (reads and clears it in
+// one atomic exchange on the device).  The word's device address is looked up once per device,
+// with that device current, and handed to every tensor-core launch.  In the checked build
+// (MPQ_CHECK_BOUNDS) every kernel unit also keeps a count of the accesses its bounds checks
+// skipped, taken by the same call.
 #include <atomic>
 #include <mutex>
+#include <vector>
 
+#include "checks.cuh"
 #include "mpq_internal.cuh"
 #include "waits.cuh"
 
@@ -42,6 +46,22 @@ static mpq_status timeout_word(unsigned **out)
     return MPQ_OK;
 }
 
+struct BoundsUnit {
+    const char *name;
+    BoundsTake take;
+};
+
+static std::vector<BoundsUnit> &bounds_units()
+{
+    static std::vector<BoundsUnit> units;   // filled while the library loads, read-only after
+    return units;
+}
+
+void register_bounds_unit(const char *name, BoundsTake take)
+{
+    bounds_units().push_back({name, take});
+}
+
 mpq_status wait_ctl(WaitCtl *out)
 {
     const mpq_status st = timeout_word(&out->status);
@@ -70,12 +90,41 @@ extern "C" mpq_status mpq_device_status(void *stream, unsigned *flags)
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     st = cuda_status(e, "reading the timeout word");
     if (st != MPQ_OK) return st;
+    // the checked build's bounds counts, unit by unit (none are registered in the normal build)
+    unsigned skipped = 0, first_line = 0;
+    const char *first_unit = nullptr;
+    for (const BoundsUnit &u : bounds_units()) {
+        unsigned c = 0, line = 0;
+        st = cuda_status(u.take(s, &c, &line), "reading the bounds-check words");
+        if (st != MPQ_OK) return st;
+        if (c != 0 && !first_unit) {
+            first_unit = u.name;
+            first_line = line;
+        }
+        skipped += c;
+    }
+    if (skipped != 0) h |= MPQ_FAULT_BOUNDS;
     if (flags) *flags = h;
-    if (h != 0) {
-        set_error("a bounded device-side wait gave up (MPQ_TIMEOUT bits 0x%x)", h);
+    if (h & ~MPQ_FAULT_BOUNDS) {
+        set_error("a bounded device-side wait gave up (MPQ_TIMEOUT bits 0x%x)",
+                  h & ~MPQ_FAULT_BOUNDS);
         return MPQ_ERR_TIMEOUT;
     }
+    if (skipped != 0) {
+        set_error("bounds checks skipped %u accesses (the first at %s:%u)", skipped, first_unit,
+                  first_line);
+        return MPQ_ERR_BOUNDS;
+    }
     return MPQ_OK;
+}
+
+extern "C" unsigned mpq_build_options(void)
+{
+#ifdef MPQ_CHECK_BOUNDS
+    return MPQ_BUILD_CHECK_BOUNDS;
+#else
+    return 0u;
+#endif
 }
 
 extern "C" mpq_status mpq_set_wait_limit(long long clocks)

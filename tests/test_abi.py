@@ -45,7 +45,19 @@ def test_every_declared_symbol_is_exported(lib):
 def test_status_strings(lib):
     assert lib.mpq_status_string(0) == b"MPQ_OK"
     assert lib.mpq_status_string(3) == b"MPQ_ERR_UNSUPPORTED"
+    assert lib.mpq_status_string(7) == b"MPQ_ERR_BOUNDS"
     assert lib.mpq_version() >= 100
+
+
+def test_checked_build_exports_and_reports_its_option(lib):
+    """The checked build (-DMPQ_CHECK_BOUNDS) compiles, loads without a GPU, exports every
+    declared symbol and says what it is through mpq_build_options; the normal build says 0."""
+    raw = ctypes.CDLL(_build.build(checked=True))
+    for name in declared_functions():
+        assert hasattr(raw, name), name
+    raw.mpq_build_options.restype = ctypes.c_uint
+    assert raw.mpq_build_options() == binding.MPQ_BUILD_CHECK_BOUNDS
+    assert binding.mpq_build_options() == 0
 
 
 P = ctypes.c_void_p
