@@ -1,6 +1,11 @@
 // Output error (Sec. 3.3, Eq. 11) as a CTA-pair tcgen05 contraction:
 //   err[k][n] = (1/N) sum_t (x_t . r_{k,n+1})^2,  n = 0..k_max.
 //
+// This file holds the contraction for the clipping search (tf32 operands) and for the output error
+// entry point with a fixed range table (fp16 operands, X split by the producers: it needs no
+// scratch beyond that table); the output error with pooled scratch runs output_error_f16.cu, the
+// same contraction with X split ahead and the layout its measurements favoured.
+//
 // Y = R X^T with R the C*(k_max+1) residual vectors and X the N calibration rows (length d);
 // err is the row-wise mean of Y^2.  Two CTAs on neighbouring SMs (cluster ranks 2p, 2p+1) form one
 // UMMA of M = 256 residual vectors by N = 256 calibration rows: each CTA holds 128 vectors (whole
@@ -45,6 +50,7 @@
 #include <atomic>
 
 #include "mpq_internal.cuh"
+#include "pair_common.cuh"
 #include "rounding.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
@@ -122,35 +128,6 @@ struct PairCtrl {
 constexpr int P_CTRL_BYTES = (sizeof(PairCtrl) + 1023) / 1024 * 1024;
 constexpr int P_BASE_SMEM = 1024 /* alignment slack */ + P_CTRL_BYTES + P_TILE_SETS * P_STAGE_BYTES;
 
-// fp16 operands: exponent e with m * 2^e in [2^14, 2^15) for the largest magnitude m of a residual
-// vector or of X, so that the vector's hi and lo halves are normal fp16 numbers down to 2^-7 of its
-// largest element (and nothing overflows).  0 for m = 0, NaN or inf (which then propagate); capped
-// at 126 so that 2^e stays a normal float (only vectors below 2^-111 are scaled less).
-__device__ __forceinline__ int f16_scale_exp(float m)
-{
-    if (!(m > 0.0f) || !isfinite(m)) return 0;
-    int E;
-    (void)frexpf(m, &E);              // m = f 2^E, f in [0.5, 1)
-    return min(15 - E, 126);
-}
-
-__device__ __forceinline__ float pow2f(int e) { return __int_as_float((127 + e) << 23); }
-
-__device__ __forceinline__ double pow2d(int e)
-{
-    return __longlong_as_double((long long)(1023 + e) << 52);
-}
-
-// x * 2^e (exact) split into fp16 hi + lo: hi = fl16(x), lo = fl16(x - hi) (x - hi is exact in fp32).
-__device__ __forceinline__ void split_f16x2(float a, float b, uint32_t &hi, uint32_t &lo)
-{
-    const __half2 h = __floats2half2_rn(a, b);
-    const float2 hf = __half22float2(h);
-    const __half2 l = __floats2half2_rn(__fsub_rn(a, hf.x), __fsub_rn(b, hf.y));
-    hi = *reinterpret_cast<const uint32_t *>(&h);
-    lo = *reinterpret_cast<const uint32_t *>(&l);
-}
-
 // Per-KP1 geometry and the raw slot layout, in the order the tile copies write it:
 // X chunk [128 rows][32] fp32, W chunk [CH][32] fp32, codes [K][CH][32] int8.  KP1 is the number of
 // residual vectors per channel: k_max + 1 greedy residuals, or (CLIP) one per candidate clipping
@@ -178,29 +155,13 @@ struct PGeo {
 // 0-15 or 16-31 by bit 2 of its row.  A store wavefront serves 128 bytes: a half warp's 8-byte
 // stores, or a whole warp's 4-byte stores.  So that each of them reaches both bank halves:
 // X item q (8 bytes per operand half) of a warp's 32 items goes to rows r, r+4 (lanes 0-15) and
-// r+1, r+5 (lanes 16-31) of an 8-row atom ...
+// r+1, r+5 (lanes 16-31) of an 8-row atom (the residual items' channels are paired by
+// pair_channel for the same reason).
 __device__ __forceinline__ int pair_x_item(int q)
 {
     const int g = q >> 5, j = (q & 31) >> 3;
     const int row = (g >> 1) * 8 + (g & 1) * 2 + (j >> 1) + (j & 1) * 4;
     return row * P_KC4 + (q & 7);
-}
-
-// ... and the two channels of a warp's residual items (slots j = 2t, 2t+1: lanes 0-15 and 16-31)
-// are D apart, with D (k_max+1) = 4 (mod 8) where possible, so that their rows differ in bit 2.
-// A bijection of the slots 0..nch-1: blocks of 2D slots pair channel i with i + D; a last partial
-// block of T slots pairs its first T - D channels so and keeps the rest in place.
-template <int KP1>
-__device__ __forceinline__ int pair_channel(int j, int nch)
-{
-    constexpr int D = (KP1 & 1) ? 4 : ((KP1 & 3) == 2 ? 2 : 1);
-    const int F = nch / (2 * D) * (2 * D);
-    if (j < F) {
-        const int w = j % (2 * D);
-        return j - w + (w >> 1) + (w & 1) * D;
-    }
-    const int T = nch - F, m = T > D ? T - D : 0, s = j - F;
-    return s < 2 * m ? F + (s >> 1) + (s & 1) * D : F + m + (s - 2 * m);
 }
 
 // Raw slot -> operand stage (tile set `sb`, row half `hh` with fp16 operands): X rows -> B tiles;
@@ -701,39 +662,64 @@ pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const flo
     }
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 pair_map_encoder()
+// The range pre-pass into `range` (zeroed here): max|X| into range[0] and, without rmax, max|r| of
+// every residual vector into range[1 + k (k_max+1) + n].
+template <int KP1>
+cudaError_t launch_ranges(const float *X, int N, const float *W, const int8_t *codes,
+                          const float *scales, int C, int d, const float *rmax, unsigned *range,
+                          cudaStream_t stream)
 {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                             &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-        return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
-    }();
-    return fn;
+    const size_t words = rmax ? 1 : 1 + (size_t)C * KP1;
+    const long long nx4 = (long long)N * d / 4;
+    const int xb = (int)std::min<long long>((nx4 + 1023) / 1024, 4LL * sm_count());
+    const int rsplit = std::min(8, std::max(1, (d / 4 + 255) / 256));   // >= 8 loads per lane
+    const long long cb = rmax ? 0 : ((long long)C * rsplit + 7) / 8;
+    cudaError_t e = cudaMemsetAsync(range, 0, words * sizeof(unsigned), stream);
+    if (e != cudaSuccess) return e;
+    pair_range_kernel<KP1><<<(unsigned)(xb + cb), 256, 0, stream>>>(
+        reinterpret_cast<const float4 *>(X), nx4, xb, W, codes, scales, C, d, rsplit, range);
+    return cudaGetLastError();
 }
 
-// Tile map over a row-major tensor (dims[0] contiguous, byte strides for dims 1..), zero fill.
-bool pair_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *base,
-              const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box)
+// The greedy residuals' output error with scratch from the stream-ordered pool: the range table
+// and the split X planes (2 N d fp16) in one block, the range pre-pass, then output_error_f16.cu's
+// contraction.
+template <int KP1>
+mpq_status launch_pooled_f16(const float *X, int N, const float *W, const int8_t *codes,
+                             const float *scales, int C, int d, float *err, cudaStream_t stream,
+                             const float *rmax)
 {
-    PFN_cuTensorMapEncodeTiled_v12000 enc = pair_map_encoder();
-    if (!enc) return false;
-    const cuuint32_t estr[3] = {1, 1, 1};
-    return enc(m, type, (cuuint32_t)rank, const_cast<void *>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    const size_t words = rmax ? 1 : 1 + (size_t)C * KP1;
+    const size_t range_bytes = (words * sizeof(unsigned) + 255) / 256 * 256;
+    const size_t xs_bytes = (size_t)N * d * 2 * sizeof(uint16_t);
+    void *scratch = nullptr;
+    const mpq_status st = pool_scratch(&scratch, range_bytes + xs_bytes, stream);
+    if (st != MPQ_OK) return st;
+    unsigned *range = static_cast<unsigned *>(scratch);
+    uint16_t *xs = reinterpret_cast<uint16_t *>(static_cast<char *>(scratch) + range_bytes);
+    const cudaError_t e = launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax, range, stream);
+    mpq_status r = cuda_status(e, "output-error range pre-pass");
+    if (r == MPQ_OK) {
+        const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : range + 1;
+        r = launch_output_error_f16(X, N, W, codes, scales, C, d, KP1 - 1, err, range, vr, xs,
+                                    stream);
+    }
+    const cudaError_t ef = cudaFreeAsync(scratch, stream);
+    if (r == MPQ_OK) r = cuda_status(ef, "scratch release (cudaFreeAsync)");
+    return r;
 }
 
-// ext_range: caller-provided range scratch (fp16 operands), or NULL for the stream-ordered pool.
+// ext_range: caller-provided range scratch (fp16 operands: this kernel), or NULL (fp16 operands:
+// the pooled path of output_error_f16.cu).
 template <int KP1, bool CLIP>
 mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *codes,
                        const float *scales, int C, int d, int qmax, float *err, cudaStream_t stream,
                        unsigned *ext_range = nullptr, const float *rmax = nullptr)
 {
+    if constexpr (!CLIP) {
+        if (!ext_range)
+            return launch_pooled_f16<KP1>(X, N, W, codes, scales, C, d, err, stream, rmax);
+    }
     using G = PGeo<KP1, CLIP>;
     const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
     const int n_rt = (N + P_N - 1) / P_N;
@@ -749,9 +735,9 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)C, (cuuint64_t)G::K};
     const cuuint64_t sq[2] = {(cuuint64_t)d, (cuuint64_t)C * d};
     const cuuint32_t bq[3] = {P_KC, (cuuint32_t)G::CH, (cuuint32_t)G::K};
-    if (!pair_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, X, dx, sx, bx) ||
-        !pair_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw) ||
-        (!CLIP && !pair_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq))) {
+    if (!encode_tile_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, X, dx, sx, bx) ||
+        !encode_tile_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw) ||
+        (!CLIP && !encode_tile_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq))) {
         set_error("output error: tensor map encoding failed");
         return MPQ_ERR_CUDA;
     }
@@ -805,34 +791,15 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     WaitCtl wc;
     mpq_status wst = wait_ctl(&wc);
     if (wst != MPQ_OK) return wst;
-    unsigned *range = ext_range;
     if constexpr (!CLIP) {
-        // fp16 operands: the ranges of X and of every residual vector first (the residual vectors'
-        // from rmax when the greedy search gave them: then the pre-pass reads X alone)
-        const size_t words = rmax ? 1 : 1 + (size_t)C * KP1;
-        if (!ext_range) {
-            mpq_status st = pool_scratch(reinterpret_cast<void **>(&range), words * sizeof(unsigned),
-                                         stream);
-            if (st != MPQ_OK) return st;
-        }
-        const long long nx4 = (long long)N * d / 4;
-        const int xb = (int)std::min<long long>((nx4 + 1023) / 1024, 4LL * sm_count());
-        const int rsplit = std::min(8, std::max(1, (d / 4 + 255) / 256));   // >= 8 loads per lane
-        const long long cb = rmax ? 0 : ((long long)C * rsplit + 7) / 8;
-        e = cudaMemsetAsync(range, 0, words * sizeof(unsigned), stream);
-        if (e == cudaSuccess) {
-            pair_range_kernel<KP1><<<(unsigned)(xb + cb), 256, 0, stream>>>(
-                reinterpret_cast<const float4 *>(X), nx4, xb, W, codes, scales, C, d, rsplit, range);
-            e = cudaGetLastError();
-        }
-        const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : range + 1;
+        // fp16 operands (the fixed-scratch entry point): the ranges of X and of every residual
+        // vector first, into the caller's table (the residual vectors' from rmax when the greedy
+        // search gave them: then the pre-pass reads X alone)
+        e = launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax, ext_range, stream);
+        const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : ext_range + 1;
         if (e == cudaSuccess)
             e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
-                                   (const unsigned *)range, vr, err, split, wc, tmX, tmW, tmQ);
-        if (!ext_range) {
-            const cudaError_t ef = cudaFreeAsync(range, stream);
-            if (e == cudaSuccess) e = ef;
-        }
+                                   (const unsigned *)ext_range, vr, err, split, wc, tmX, tmW, tmQ);
         return cuda_status(e, "pair output-error kernel launch");
     }
     e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
@@ -842,6 +809,34 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
 }
 
 }  // namespace
+
+namespace {
+PFN_cuTensorMapEncodeTiled_v12000 tile_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+        return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+    }();
+    return fn;
+}
+}  // namespace
+
+bool encode_tile_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *base,
+                     const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box,
+                     CUtensorMapSwizzle swizzle)
+{
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tile_map_encoder();
+    if (!enc) return false;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, type, (cuuint32_t)rank, const_cast<void *>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 // Scratch (the fp16 contraction's range table, the adaptive grid's event lists) comes from the device's stream-ordered pool (allocated and
 // freed on the call's stream, so concurrent calls on other streams never share it; inside a CUDA
