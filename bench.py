@@ -34,7 +34,9 @@ UNIT = "elem*cand*pt/s"
 PROFILES = os.path.join(ROOT, "profiles")
 KERNEL_SOURCES = {
     "output_error": ("paper_2002_09049_gb300/csrc/output_error.cu",
+                     "paper_2002_09049_gb300/csrc/output_error_f16.cu",
                      "paper_2002_09049_gb300/csrc/output_error_pair.cu",
+                     "paper_2002_09049_gb300/csrc/pair_common.cuh",
                      "paper_2002_09049_gb300/csrc/output_error_tc.cu",
                      "paper_2002_09049_gb300/csrc/sm100.cuh",
                      "paper_2002_09049_gb300/csrc/tf32_operands.cuh",
@@ -300,9 +302,10 @@ def run_ours(args, world, rank, local):
             net.run_device(Ws, Xs, stream=stream)
 
     center_launches = {"none": 0, "channel": 1, "layer": 3}[args.center]
-    # one kernel per call, plus the range pre-pass of every output error on the CTA-pair kernel
-    # (shared calibration input, rows a multiple of 16 elements; torch buffers are 16-byte aligned)
-    range_launches = sum(1 for l in layers if l.groups == 1 and l.d % 16 == 0)
+    # one kernel per call, plus the two pre-passes (ranges, X split) of every output error on the
+    # CTA-pair kernel (shared calibration input, rows a multiple of 16 elements; torch buffers are
+    # 16-byte aligned)
+    range_launches = 2 * sum(1 for l in layers if l.groups == 1 and l.d % 16 == 0)
     alloc_launches = 1 if net.batch_alloc else len(layers)
     launches_per_step = ((3 + center_launches) * len(layers) + alloc_launches +
                          range_launches) * len(wl.bits)
@@ -474,9 +477,10 @@ def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_
     if dominant == "output_error":
         peak = peaks["bf16_tflops"]
         ach = fam_work[dominant] / t_s / 1e12
-        return {"kernel": "output_error_pair_kernel (Eq. 11, tcgen05 cta_group::2 kind::f16, "
-                          "scaled fp16 hi/lo operands, 3 passes; after pair_range_kernel; "
-                          "output_error_tc_kernel for rows not 16-byte multiples)",
+        return {"kernel": "output_error_f16_kernel (Eq. 11, tcgen05 cta_group::2 kind::f16, "
+                          "scaled fp16 hi/lo operands, 3 passes, X split ahead; after "
+                          "pair_range_kernel and f16_split_kernel; output_error_tc_kernel for rows "
+                          "not 16-byte multiples)",
                 "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
                 "frac": ach / peak, "traffic": traffic,
                 "peak_source": f"{peak_src} bf16 dense burst (the fp16 rate of kind::f16)"}
