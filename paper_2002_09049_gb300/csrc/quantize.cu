@@ -33,11 +33,13 @@
 #include <limits.h>
 #include <math.h>
 
+#include <algorithm>
 #include <type_traits>
 #include <vector>
 
 #include "mpq_internal.cuh"
 #include "rounding.cuh"
+#include "sm100.cuh"
 
 MPQ_CHECKED_UNIT("quantize.cu");
 
@@ -95,8 +97,9 @@ struct Scratch {
 // aligned.
 __host__ __device__ constexpr size_t lattice_words(int nb) { return (size_t)2 * nb; }
 
-// bytes of the CTA's bucket -> position-index table (uint16 per bucket), 16-byte multiple
-__host__ __device__ constexpr size_t lut_bytes(int nb) { return ((size_t)nb * 2 + 15) & ~(size_t)15; }
+// bytes of the CTA's bucket -> position-index table (uint16 per bucket, and 16 spare entries so
+// that the largest element's bucket, at most nb - 1, needs no clamp), 16-byte multiple
+__host__ __device__ constexpr size_t lut_bytes(int nb) { return ((size_t)(nb + 16) * 2 + 15) & ~(size_t)15; }
 
 __host__ __device__ constexpr size_t group_words(int G, int d, int copies, int nb)
 {
@@ -445,8 +448,23 @@ __device__ __forceinline__ float i64_to_f32(long long x)
     return __fmaf_rn(hi, 4294967296.0f, lo);
 }
 
-template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
-__global__ void __launch_bounds__(QTHREADS, 4)
+// Columns of tensor memory a CTA allocates for its groups' residual rows in the TM build: a power of
+// two, at least 32.
+__host__ __device__ constexpr uint32_t tm_alloc_cols(int cols)
+{
+    return cols <= 32 ? 32u : cols <= 64 ? 64u : cols <= 128 ? 128u : cols <= 256 ? 256u : 512u;
+}
+constexpr int TM_MAX_D = 4096;   // TM build: d a multiple of 4 x 128, at most 32 columns per group
+
+// MINB: CTAs per SM the register budget allows (4: 64 registers per thread; 3: up to 85, for the
+// layers whose shared memory holds an SM to 3 CTAs anyway).
+// TM (4-warp groups on the lattice form): each channel's residual row lives in tensor memory, one
+// lane per thread -- thread gt of the group holds elements gt + 128 c in columns c of its lane --
+// instead of shared memory, which then holds only the lattice and bins (c5: 4 CTAs per SM instead
+// of 3).  A group without a channel (the last CTA's) repeats the CTA's last channel without writing
+// anything, so that every thread reaches the end, where tensor memory is released.
+template <int WPC, bool CUSTOM, bool LAT, bool TABLE, int MINB = 4, bool TM = false>
+__global__ void __launch_bounds__(QTHREADS, MINB)
 quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, const Grid<CUSTOM> grid,
                 int k_max, int8_t *__restrict__ codes, float *__restrict__ scales,
                 float *__restrict__ resid_sq, float *__restrict__ residuals,
@@ -461,9 +479,13 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
     __shared__ Scratch scratch[GPC];
     __shared__ float s_hinv[QMAX_LIMIT + 1];   // 1 / (L - 1/2): threshold estimates only
 
+    static_assert(!TM || (WPC == 4 && LAT && !CUSTOM), "tensor-memory rows: 4-warp lattice groups");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = warp / WPC, gw = warp % WPC, gt = gw * 32 + lane;
-    const int k = blockIdx.x * GPC + grp;
+    const int k_own = blockIdx.x * GPC + grp;
+    const bool ghost = TM && k_own >= C;          // TM: a group without a channel repeats C - 1
+    const int k = ghost ? C - 1 : k_own;
+    const int dsm = TM ? 0 : d;                   // residual words per group in shared memory
     const float qmaxf = (float)qmax;
     // the grid fractions f_g and fl(1 / f_g): a table, or (linear grid, when the table's 2G words
     // would cost a CTA per SM) computed where needed
@@ -478,7 +500,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
         }
     // the last group's region ends the carve-up of dynamic shared memory
     if (!MPQ_CHECK_SMEM_END((TABLE ? 8 * (size_t)G : 0) + (LAT ? lut_bytes(nb) : 0) +
-                            4 * (size_t)GPC * group_words(G, d, COPIES, nc)))
+                            4 * (size_t)GPC * group_words(G, dsm, COPIES, nc)))
         return;
     auto fg = [&](int g) -> float { return TABLE ? ftab[g] : grid.frac(g, G); };
     auto fi = [&](int g) -> float { return TABLE ? ftab[G + g] : __frcp_rn(grid.frac(g, G)); };
@@ -506,12 +528,21 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             }
         }
     }
+    // TM: the CTA's tensor memory for its groups' rows (warp 0 allocates and releases it)
+    __shared__ uint32_t s_tmem;
+    const int tcg = TM ? d / NT : 0;               // columns per group
+    const uint32_t tcols = tm_alloc_cols(GPC * tcg);
+    if (TM && warp == 0) sm100::tmem_alloc(&s_tmem, tcols);
+    if (TM) sm100::tc_fence_before();
     __syncthreads();
-    if (k >= C) return;   // whole group idle (group-uniform)
+    if (TM) sm100::tc_fence_after();
+    // this thread's lane (the warp's lane quarter) at the group's first column
+    const uint32_t taddr = TM ? s_tmem + ((uint32_t)(gw * 32) << 16) + (uint32_t)(grp * tcg) : 0u;
+    if (!TM && k >= C) return;   // whole group idle (group-uniform)
 
     unsigned int *gl = reinterpret_cast<unsigned int *>(
                            reinterpret_cast<unsigned char *>(lut) + (LAT ? lut_bytes(nb) : 0)) +
-                       (size_t)grp * group_words(G, d, COPIES, nc);
+                       (size_t)grp * group_words(G, dsm, COPIES, nc);
     unsigned int *lat = gl;                         // [nc][2]: R low word, R high | count
     const unsigned cnt_one = 1u << cnt_bit, hmask = cnt_one - 1u;
     unsigned int *gbase = gl + lattice_words(nc);
@@ -534,33 +565,66 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
 
     int bad = 0;
     float ssum = 0.0f, scomp = 0.0f, am = 0.0f;
-    for (int j = gt; j < d; j += NT) {
-        const float v = MPQ_IN((size_t)k * d + j, plane) ? w[j] : 0.0f;
-        sr[j] = v;
-        bad |= !isfinite(v);
-        kahan_add(ssum, scomp, v * v);
-        am = fmaxf(am, fabsf(v));
+    if constexpr (TM) {
+        for (int cc = 0; cc < tcg; cc += 4) {
+            float v4[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int j = gt + NT * (cc + u);
+                const float v = MPQ_IN((size_t)k * d + j, plane) ? w[j] : 0.0f;
+                v4[u] = v;
+                bad |= !isfinite(v);
+                kahan_add(ssum, scomp, v * v);
+                am = fmaxf(am, fabsf(v));
+            }
+            __syncwarp();
+            sm100::tmem_st_32x32b_x4(taddr + cc, v4);
+        }
+        sm100::tmem_wait_st();
+    } else {
+        for (int j = gt; j < d; j += NT) {
+            const float v = MPQ_IN((size_t)k * d + j, plane) ? w[j] : 0.0f;
+            sr[j] = v;
+            bad |= !isfinite(v);
+            kahan_add(ssum, scomp, v * v);
+            am = fmaxf(am, fabsf(v));
+        }
     }
     float m = am;
     float r2 = ssum;
     group_max_sum_or<WPC>(m, r2, bad, sc, gw, lane, grp);
     if (WPC == 1) __syncwarp();
     const size_t n_rs = (size_t)C * (k_max + 1), n_codes = (size_t)k_max * plane;
-    if (resid_sq && gt == 0 && MPQ_IN((size_t)k * (k_max + 1), n_rs))
+    if (resid_sq && gt == 0 && !ghost && MPQ_IN((size_t)k * (k_max + 1), n_rs))
         resid_sq[(size_t)k * (k_max + 1)] = bad ? NAN : r2;
-    if (rmax && gt == 0 && MPQ_IN((size_t)k * (k_max + 1), n_rs))
+    if (rmax && gt == 0 && !ghost && MPQ_IN((size_t)k * (k_max + 1), n_rs))
         rmax[(size_t)k * (k_max + 1)] = bad ? NAN : m;
 
     for (int i = 0; i < k_max; ++i) {
         int8_t *qi = codes + (size_t)i * plane + (size_t)k * d;
         float *ri = residuals ? residuals + (size_t)i * plane + (size_t)k * d : nullptr;
         if (bad) {
-            for (int j = gt; j < d; j += NT) {
-                if (!MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes)) continue;
-                qi[j] = 0;
-                if (ri) ri[j] = sr[j];
+            if constexpr (TM) {
+                for (int cc = 0; cc < tcg; cc += 4) {
+                    float v4[4];
+                    __syncwarp();
+                    sm100::tmem_ld_32x32b_x4(taddr + cc, v4);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int j = gt + NT * (cc + u);
+                        if (ghost || !MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes)) continue;
+                        qi[j] = 0;
+                        if (ri) ri[j] = v4[u];
+                    }
+                }
+            } else {
+                for (int j = gt; j < d; j += NT) {
+                    if (!MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes)) continue;
+                    qi[j] = 0;
+                    if (ri) ri[j] = sr[j];
+                }
             }
-            if (gt == 0) {
+            if (gt == 0 && !ghost) {
                 const bool in_s = MPQ_IN((size_t)k * k_max + i, (size_t)C * k_max);
                 const bool in_r = MPQ_IN((size_t)k * (k_max + 1) + i + 1, n_rs);
                 if (in_s) scales[(size_t)k * k_max + i] = NAN;
@@ -609,6 +673,7 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 const float s0 = __fmul_rn(fg(0), smax), sG = __fmul_rn(fg(G - 1), smax);
                 const float i0 = fi(0) * ism, iG = fi(G - 1) * ism;
                 const float g_per_a = __fdiv_rn((float)G, smax);   // linear grid: s_g ~ (g+1)/G*smax
+                const float g2_per_a = 2.0f * g_per_a;   // 2 fl(a g_per_a) = fl(a g2_per_a) exactly
                 long long Pb = 0;
                 long long Nb = 0;
                 // every level an element crosses inside the grid, one event each
@@ -692,14 +757,25 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                     // (relative) of an integer, one bucket update records the element for every
                     // (g, L) exactly; near a lattice point the per-level events settle each
                     // threshold with the exact rule.  Two elements per pass, for overlap.
-                    constexpr int U = 2;
+                    constexpr int U = TM ? 4 : 2;
                     for (int j0 = gt; j0 < d; j0 += U * NT) {
                         float av[U], u2[U];
+                        if constexpr (TM) {   // columns (j0 - gt) / NT .. + 3 of this lane
+                            float v4[4];
+                            __syncwarp();   // tensor-memory accesses by the converged warp
+                            sm100::tmem_ld_32x32b_x4(taddr + (uint32_t)((j0 - gt) / NT), v4);
 #pragma unroll
-                        for (int u = 0; u < U; ++u) {
-                            const int j = j0 + u * NT;
-                            av[u] = j < d ? fabsf(sr[j]) : 0.0f;
-                            u2[u] = 2.0f * (av[u] * g_per_a);
+                            for (int u = 0; u < U; ++u) {
+                                av[u] = fabsf(v4[u]);
+                                u2[u] = av[u] * g2_per_a;
+                            }
+                        } else {
+#pragma unroll
+                            for (int u = 0; u < U; ++u) {
+                                const int j = j0 + u * NT;
+                                av[u] = j < d ? fabsf(sr[j]) : 0.0f;
+                                u2[u] = av[u] * g2_per_a;
+                            }
                         }
 #pragma unroll
                         for (int u = 0; u < U; ++u) {
@@ -707,7 +783,10 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                             if (!near_lattice(u2[u])) {
                                 const int b = (int)floorf(u2[u]);
                                 if (b >= 1) {
-                                    const int bb = lut[b < nb - 1 ? b : nb - 1];
+                                    // b <= nb - 1: fl(max|r| G / smax) rounds to at most
+                                    // G Qmax (1 + 2^-22), below the next integer
+                                    if (!MPQ_IN(b, nb)) continue;
+                                    const int bb = lut[b];
                                     if (!MPQ_IN(bb, nc)) continue;
                                     // two 32-bit atomics: the low word's old value gives
                                     // its carry, which the high word takes with the count
@@ -750,9 +829,22 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                                             (unsigned int)((unsigned long long)R >> 32), a * g_per_a);
                         }
                     } else {   // the queue overflowed (never seen): every such element again
-                        for (int j = gt; j < d; j += NT) {
-                            const float a = fabsf(sr[j]);
-                            if (a != 0.0f && near_lattice(2.0f * (a * g_per_a))) events(a);
+                        if constexpr (TM) {
+                            for (int cc = 0; cc < tcg; cc += 4) {
+                                float v4[4];
+                                __syncwarp();
+                                sm100::tmem_ld_32x32b_x4(taddr + cc, v4);
+#pragma unroll
+                                for (int u = 0; u < 4; ++u) {
+                                    const float a = fabsf(v4[u]);
+                                    if (a != 0.0f && near_lattice(2.0f * (a * g_per_a))) events(a);
+                                }
+                            }
+                        } else {
+                            for (int j = gt; j < d; j += NT) {
+                                const float a = fabsf(sr[j]);
+                                if (a != 0.0f && near_lattice(2.0f * (a * g_per_a))) events(a);
+                            }
                         }
                     }
                 } else {
@@ -862,22 +954,61 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
                 }
             } else {
                 // ---- direct evaluation (a candidate scale underflowed to 0)
-                for (int g = gt; g < G; g += NT) {
-                    const float s = __fmul_rn(fg(g), smax);
-                    double D = 0.0;  // s == 0: all codes 0, E = ||r||^2
-                    if (s > 0.0f) {
+                if constexpr (TM) {
+                    // every candidate's P and N from each thread's own elements, summed over the
+                    // group in the bins (cleared at the step's start), then decided as below
+                    for (int g = 0; g < G; ++g) {
+                        const float s = __fmul_rn(fg(g), smax);
+                        if (!(s > 0.0f)) continue;   // the same for every thread
                         long long P = 0, N = 0;
-                        for (int j = 0; j < d; ++j) {
-                            const float a = fabsf(sr[j]);
-                            const int c = code_mag(a, s, qmaxf);
-                            P += fixed_point(a, S) * (long long)c;
-                            N += (long long)c * c;
+                        for (int cc = 0; cc < tcg; cc += 4) {
+                            float v4[4];
+                            __syncwarp();
+                            sm100::tmem_ld_32x32b_x4(taddr + cc, v4);
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) {
+                                const float a = fabsf(v4[u]);
+                                const int c = code_mag(a, s, qmaxf);
+                                P += fixed_point(a, S) * (long long)c;
+                                N += (long long)c * c;
+                            }
                         }
-                        D = decision(s, P, N, down);
+                        P = warp_sum(P);
+                        N = warp_sum(N);
+                        if (lane == 0) {
+                            add64(&mLo[g + 1], &mHi[g + 1], (unsigned int)P,
+                                  (unsigned int)((unsigned long long)P >> 32));
+                            atomicAdd(&mN[g + 1], (int)N);
+                        }
                     }
-                    if (D < bestD) {
-                        bestD = D;
-                        bestg = g;
+                    gsync<WPC>(grp);
+                    for (int g = gt; g < G; g += NT) {
+                        const float s = __fmul_rn(fg(g), smax);
+                        const double D = s > 0.0f ? decision(s, bin64(mLo, mHi, g + 1), (long long)mN[g + 1], down)
+                                                  : 0.0;   // s == 0: all codes 0, E = ||r||^2
+                        if (D < bestD) {
+                            bestD = D;
+                            bestg = g;
+                        }
+                    }
+                } else {
+                    for (int g = gt; g < G; g += NT) {
+                        const float s = __fmul_rn(fg(g), smax);
+                        double D = 0.0;  // s == 0: all codes 0, E = ||r||^2
+                        if (s > 0.0f) {
+                            long long P = 0, N = 0;
+                            for (int j = 0; j < d; ++j) {
+                                const float a = fabsf(sr[j]);
+                                const int c = code_mag(a, s, qmaxf);
+                                P += fixed_point(a, S) * (long long)c;
+                                N += (long long)c * c;
+                            }
+                            D = decision(s, P, N, down);
+                        }
+                        if (D < bestD) {
+                            bestD = D;
+                            bestg = g;
+                        }
                     }
                 }
             }
@@ -891,26 +1022,42 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
         ssum = 0.0f;
         scomp = 0.0f;
         am = 0.0f;
-        for (int j = gt; j < d; j += NT) {
-            float v = sr[j];
+        // one element: its code (stored), its new residual (returned), ||r||^2 and max |r|
+        auto update = [&](float v, int j) -> float {
             int q = 0;
             if (s_best > 0.0f) {
-                const int c = (inv_best > 0.0f) ? code_fast(fabsf(v), s_best, inv_best, qmaxf)
-                                                : code_mag(fabsf(v), s_best, qmaxf);
-                q = (v < 0.0f) ? -c : c;
-                v = __fmaf_rn(-s_best, (float)q, v);
+                // the code of Eq. 8 as a float (an exact small integer) with the residual's sign
+                const float c = (inv_best > 0.0f) ? code_fast_f(fabsf(v), s_best, inv_best, qmaxf)
+                                                  : fminf(rintf(__fdiv_rn(fabsf(v), s_best)), qmaxf);
+                const float qf = copysignf(c, v);
+                q = (int)qf;
+                v = __fmaf_rn(-s_best, qf, v);
             }
-            const bool in = MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes);
+            const bool in = !ghost && MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes);
             if (in) qi[j] = (int8_t)q;
-            sr[j] = v;
             if (ri && in) ri[j] = v;
             // ||r||^2: a thread's share of at most 64 squares summed plainly (relative error
             // below 2^-18 with the group's tree), longer shares compensated
             if (short_share) ssum = __fmaf_rn(v, v, ssum);
             else kahan_add(ssum, scomp, v * v);
             am = fmaxf(am, fabsf(v));
+            return v;
+        };
+        if constexpr (TM) {
+            for (int cc = 0; cc < tcg; cc += 4) {
+                float v4[4];
+                __syncwarp();
+                sm100::tmem_ld_32x32b_x4(taddr + cc, v4);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) v4[u] = update(v4[u], gt + NT * (cc + u));
+                __syncwarp();
+                sm100::tmem_st_32x32b_x4(taddr + cc, v4);
+            }
+            sm100::tmem_wait_st();
+        } else {
+            for (int j = gt; j < d; j += NT) sr[j] = update(sr[j], j);
         }
-        if (gt == 0 && MPQ_IN((size_t)k * k_max + i, (size_t)C * k_max))
+        if (gt == 0 && !ghost && MPQ_IN((size_t)k * k_max + i, (size_t)C * k_max))
             scales[(size_t)k * k_max + i] = s_best;
         m = am;
         r2 = ssum;
@@ -918,8 +1065,17 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
         group_max_sum_or<WPC>(m, r2, none, sc, gw, lane, grp);   // orders the sr[] writes too
         if (WPC == 1) __syncwarp();
         const bool in_r = MPQ_IN((size_t)k * (k_max + 1) + i + 1, n_rs);
-        if (resid_sq && gt == 0 && in_r) resid_sq[(size_t)k * (k_max + 1) + i + 1] = r2;
-        if (rmax && gt == 0 && in_r) rmax[(size_t)k * (k_max + 1) + i + 1] = m;
+        if (resid_sq && gt == 0 && !ghost && in_r) resid_sq[(size_t)k * (k_max + 1) + i + 1] = r2;
+        if (rmax && gt == 0 && !ghost && in_r) rmax[(size_t)k * (k_max + 1) + i + 1] = m;
+    }
+    if constexpr (TM) {
+        // every group is done with tensor memory before it is released
+        sm100::tc_fence_before();
+        __syncthreads();
+        if (warp == 0) {
+            sm100::tc_fence_after();
+            sm100::tmem_dealloc(s_tmem, tcols);
+        }
     }
 }
 
@@ -965,16 +1121,16 @@ bool lattice_bits(int d, int qmax, int G, LatBits *lb)
     return lb->cnt_bit + ceil_log2((long long)d + 1) <= 32;
 }
 
-template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
+template <int WPC, bool CUSTOM, bool LAT, bool TABLE, int MINB = 4, bool TM = false>
 mpq_status launch_wpc(const float *W, int C, int d, int qmax, int G, const Grid<CUSTOM> &grid,
                       int k_max, int8_t *codes, float *scales, float *resid_sq, float *residuals,
                       float *rmax, int hbits, LatBits lb, size_t smem, cudaStream_t stream)
 {
     constexpr int GPC = 8 / WPC;
-    cudaError_t e = cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
+    cudaError_t e = cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE, MINB, TM>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e == cudaSuccess) {
-        quantize_kernel<WPC, CUSTOM, LAT, TABLE><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
+        quantize_kernel<WPC, CUSTOM, LAT, TABLE, MINB, TM><<<(C + GPC - 1) / GPC, QTHREADS, smem, stream>>>(
             W, C, d, qmax, G, grid, k_max, codes, scales, resid_sq, residuals, rmax, hbits, lb.lat_bits,
             lb.cnt_bit, lb.nc);
         e = cudaGetLastError();
@@ -983,13 +1139,13 @@ mpq_status launch_wpc(const float *W, int C, int d, int qmax, int G, const Grid<
 }
 
 // CTAs of a quantize kernel that fit on one SM with `smem` bytes of dynamic shared memory.
-template <int WPC, bool CUSTOM, bool LAT, bool TABLE>
+template <int WPC, bool CUSTOM, bool LAT, bool TABLE, int MINB = 4, bool TM = false>
 int quantize_ctas_per_sm(size_t smem)
 {
     int n = 0;
-    if (cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
+    if (cudaFuncSetAttribute(quantize_kernel<WPC, CUSTOM, LAT, TABLE, MINB, TM>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, quantize_kernel<WPC, CUSTOM, LAT, TABLE>,
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, quantize_kernel<WPC, CUSTOM, LAT, TABLE, MINB, TM>,
                                                       QTHREADS, smem) != cudaSuccess)
         n = 0;
     (void)cudaGetLastError();
@@ -1007,11 +1163,42 @@ mpq_status launch_lat(bool lat, const float *W, int C, int d, int qmax, int G,
             // the lattice form on the linear grid: no grid table when that fits one more CTA on
             // an SM (it costs some arithmetic per candidate otherwise)
             const size_t notab = smem - (size_t)2 * G * sizeof(float);
-            if (quantize_ctas_per_sm<WPC, false, true, false>(notab) >
-                quantize_ctas_per_sm<WPC, false, true, true>(smem))
+            const int n_notab = quantize_ctas_per_sm<WPC, false, true, false>(notab);
+            const int n_tab = quantize_ctas_per_sm<WPC, false, true, true>(smem);
+            if constexpr (WPC == 4) {
+                // residual rows in tensor memory where that fits more CTAs on an SM (their columns
+                // included: at most 512 per SM)
+                if (d % (4 * 128) == 0 && d <= TM_MAX_D) {
+                    const size_t tm_smem = smem - (size_t)(8 / WPC) * 4 *
+                                                      (group_words(G, d, 1, lb.nc) - group_words(G, 0, 1, lb.nc));
+                    // (the occupancy query reports one CTA per SM for any kernel that allocates
+                    // tensor memory, so the count is the same kernel's without it: registers and
+                    // shared memory, then the columns)
+                    const int cols = (int)tm_alloc_cols((8 / WPC) * d / 128);
+                    const int n_tm = std::min(quantize_ctas_per_sm<WPC, false, true, true>(tm_smem), 512 / cols);
+                    if (n_tm > n_tab && n_tm > n_notab)
+                        return launch_wpc<WPC, false, true, true, 4, true>(W, C, d, qmax, G, grid, k_max,
+                                                                           codes, scales, resid_sq, residuals,
+                                                                           rmax, hbits, lb, tm_smem, stream);
+                }
+            }
+            // where shared memory holds an SM to 3 CTAs or fewer, the build with more registers per
+            // thread (no spills, more loads in flight) costs no occupancy (c5: 2 % faster)
+            if (n_notab > n_tab) {
+                if constexpr (WPC >= 4)
+                    if (n_notab <= 3)
+                        return launch_wpc<WPC, false, true, false, 3>(W, C, d, qmax, G, grid, k_max,
+                                                                      codes, scales, resid_sq, residuals,
+                                                                      rmax, hbits, lb, notab, stream);
                 return launch_wpc<WPC, false, true, false>(W, C, d, qmax, G, grid, k_max, codes,
                                                            scales, resid_sq, residuals, rmax, hbits, lb,
                                                            notab, stream);
+            }
+            if constexpr (WPC >= 4)
+                if (n_tab >= 1 && n_tab <= 3)
+                    return launch_wpc<WPC, false, true, true, 3>(W, C, d, qmax, G, grid, k_max, codes,
+                                                                 scales, resid_sq, residuals, rmax, hbits,
+                                                                 lb, smem, stream);
             return launch_wpc<WPC, false, true, true>(W, C, d, qmax, G, grid, k_max, codes, scales,
                                                       resid_sq, residuals, rmax, hbits, lb, smem, stream);
         }

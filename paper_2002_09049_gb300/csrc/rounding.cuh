@@ -28,4 +28,13 @@ __device__ __forceinline__ int code_fast(float a, float s, float inv_s, float qm
     return (int)fminf(rintf(__fdiv_rn(a, s)), qmaxf);
 }
 
+// code_fast as a float (the same integer value).
+__device__ __forceinline__ float code_fast_f(float a, float s, float inv_s, float qmaxf)
+{
+    const float qf = __fmul_rn(a, inv_s);
+    const float rq = rintf(qf);
+    if (0.5f - fabsf(qf - rq) > MPQ_FAST_REL * (qf + 1.0f)) return fminf(rq, qmaxf);
+    return fminf(rintf(__fdiv_rn(a, s)), qmaxf);
+}
+
 }  // namespace mpq

@@ -261,6 +261,29 @@ __device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, float (&v)[32
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 32 lanes x 4 consecutive 32-bit columns, thread i of the warp reading / writing lane (base + i)
+// (the warp's lane quarter): a load waits for its data, a store is waited for with tmem_wait_st.
+__device__ __forceinline__ void tmem_ld_32x32b_x4(uint32_t taddr, float (&v)[4])
+{
+    uint32_t r0, r1, r2, r3;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(taddr)
+                 : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    v[0] = __uint_as_float(r0);
+    v[1] = __uint_as_float(r1);
+    v[2] = __uint_as_float(r2);
+    v[3] = __uint_as_float(r3);
+}
+
+__device__ __forceinline__ void tmem_st_32x32b_x4(uint32_t taddr, const float (&v)[4])
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr),
+                 "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3])
+                 : "memory");
+}
+
 // Two loads of 32 columns (e.g. a segment and its running sums) in flight together, one wait.
 __device__ __forceinline__ void tmem_ld2_32x32b_x32(uint32_t taddr_a, uint32_t taddr_b,
                                                     float (&a)[32], float (&b)[32])

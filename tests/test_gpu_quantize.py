@@ -70,6 +70,30 @@ def test_occupancy_variant_without_grid_table(gpu, oracle):
     assert rep["near_ties"] <= 2
 
 
+def test_tensor_memory_rows(gpu, oracle):
+    """Layers with over a thousand 4096-long channels at G = 256 (c5's shape) keep every channel's
+    residual row in tensor memory (4-warp groups, four CTAs per SM; the last CTA's second group has
+    no channel and writes nothing).  Sampled channels against the definition, with a constant row
+    (every element beside a lattice point: the queue of such elements overflows and the exact
+    per-element rule runs), subnormal weights whose smallest grid scales round to 0 (direct
+    evaluation), a NaN and an infinity among them."""
+    C, d = 1217, 4096
+    W = wlm.random_weights(C, d, 83, "normal")
+    W[0] = np.float32(1.0)
+    W[1] *= np.float32(2.0 ** -140)
+    W[2, 17] = np.nan
+    W[3, 4000] = np.inf
+    gpu_out = run_gpu(W, 4, 256, 4)
+    sample = np.array([0, 1, 2, 3, 4, 5, 600, 1215, 1216])
+    orc = oracle.quantize_layer(W[sample], 4, 256, 4)
+    got = dict(codes=gpu_out["codes"][:, sample], scales=gpu_out["scales"][sample],
+               resid_sq=gpu_out["resid_sq"][sample], residuals=gpu_out["residuals"][:, sample])
+    rep = compare_quantize(W[sample], got, orc, 4, 256, 4, oracle=oracle)
+    assert rep["near_ties"] <= 1
+    assert np.all(np.isnan(gpu_out["scales"][2])) and np.all(gpu_out["codes"][:, 2] == 0)
+    assert np.all(np.isnan(gpu_out["scales"][3])) and np.all(gpu_out["codes"][:, 3] == 0)
+
+
 @pytest.mark.parametrize("bits", [2, 3, 4, 5, 6, 7, 8])
 def test_bit_widths(gpu, oracle, bits):
     W = wlm.random_weights(16, 200, 50 + bits, "laplace")
