@@ -70,21 +70,21 @@ def test_occupancy_variant_without_grid_table(gpu, oracle):
     assert rep["near_ties"] <= 2
 
 
-def test_tensor_memory_rows(gpu, oracle):
-    """Layers with over a thousand 4096-long channels at G = 256 (c5's shape) keep every channel's
-    residual row in tensor memory (4-warp groups, four CTAs per SM; the last CTA's second group has
-    no channel and writes nothing).  Sampled channels against the definition, with a constant row
-    (every element beside a lattice point: the queue of such elements overflows and the exact
-    per-element rule runs), subnormal weights whose smallest grid scales round to 0 (direct
-    evaluation), a NaN and an infinity among them."""
-    C, d = 1217, 4096
-    W = wlm.random_weights(C, d, 83, "normal")
+@pytest.mark.parametrize("C,d", [(1217, 4096), (1301, 3072)])
+def test_tensor_memory_rows(gpu, oracle, C, d):
+    """Layers with over a thousand long channels (4096: c5's shape; 3072: 24 columns per group) at
+    G = 256 keep every channel's residual row in tensor memory (4-warp groups, four CTAs per SM;
+    the last CTA's second group has no channel and writes nothing).  Sampled channels against the
+    definition, with a constant row (every element beside a lattice point: the queue of such
+    elements overflows and the exact per-element rule runs), subnormal weights whose smallest grid
+    scales round to 0 (direct evaluation), a NaN and an infinity among them."""
+    W = wlm.random_weights(C, d, 83 + d, "normal")
     W[0] = np.float32(1.0)
     W[1] *= np.float32(2.0 ** -140)
     W[2, 17] = np.nan
-    W[3, 4000] = np.inf
+    W[3, d - 96] = np.inf
     gpu_out = run_gpu(W, 4, 256, 4)
-    sample = np.array([0, 1, 2, 3, 4, 5, 600, 1215, 1216])
+    sample = np.array([0, 1, 2, 3, 4, 5, 600, C - 2, C - 1])
     orc = oracle.quantize_layer(W[sample], 4, 256, 4)
     got = dict(codes=gpu_out["codes"][:, sample], scales=gpu_out["scales"][sample],
                resid_sq=gpu_out["resid_sq"][sample], residuals=gpu_out["residuals"][:, sample])
