@@ -453,7 +453,6 @@ def run_ours(args, world, rank, local):
     return out if rank == 0 else None
 
 
-TF32_PER_BF16 = 1.1 / 2.25   # nominal dense tf32 / bf16 tensor rates of the part
 
 
 def dominant_roofline(dominant, fam_ms, fam_work, peaks, peak_src, wl, args, sm_count=152):
@@ -901,14 +900,14 @@ def run_clip(args, world, rank, local):
     ms = dist_helpers.max_over_ranks(float(np.mean(step_ms)), device=dev)
     value = dist_helpers.aggregate_throughput(units_per_step, ms, world)
     t1 = float(np.mean(one_ms)) / 1e3
-    peak = peaks["bf16_tflops"] * TF32_PER_BF16
+    peak = peaks["bf16_tflops"]
     ach = flops_per_step / t1 / 1e12
-    roofline = {"kernel": "output_error_pair_kernel in clip mode (Eq. 12 residuals generated on chip, "
-                          "tcgen05 cta_group::2 kind::tf32, 3-pass split) + candidate and argmin kernels",
+    roofline = {"kernel": "output_error_f16_kernel in clip mode (Eq. 12 residuals generated on chip, "
+                          "tcgen05 cta_group::2 kind::f16, 3-pass hi/lo split) + candidate, X range, "
+                          "X split and argmin kernels",
                 "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
                 "frac": ach / peak, "traffic": None,
-                "peak_source": f"{peak_src} bf16 dense burst x nominal tf32/bf16 ratio "
-                               f"{TF32_PER_BF16:.3f}",
+                "peak_source": f"{peak_src} bf16 dense burst (fp16 operands: the same rate)",
                 "timing": "whole calls (candidates, errors, argmin) on one stream, CUDA events; "
                           "achieved = algorithmic flops 2*N*d*C*n_cand / that time",
                 "single_stream_ms_per_step": t1 * 1e3}
@@ -921,7 +920,8 @@ def run_clip(args, world, rank, local):
                       "bits": bits, "calib_rows": wl.n_calib, "units_per_step": units_per_step,
                       "l2": "flushed between steps (512 MB write)", "streams": args.streams,
                       "parallelism": f"replicas x{world}"},
-           "roofline": roofline, "gpu_launches": 3 * len(layers) * args.steps,
+           "roofline": roofline,
+           "gpu_launches": sum(5 if l.groups == 1 and l.d % 16 == 0 else 3 for l in layers) * args.steps,
            "clocks": clk.summary()}
     if not args.no_e2e:
         def e2e_step():

@@ -9,9 +9,11 @@
 //   1. candidates: one warp per channel takes max|w| (NaN if a weight is non-finite); per-layer
 //      sets reduce the channels' maxima in one CTA;
 //   2. errors: the CTA-pair tensor-core contraction with residuals generated from W and the
-//      candidate scales on chip (output_error_pair.cu), or, for rows that are not 16-byte
-//      multiples and for per-channel inputs, one CTA per channel and candidate chunk with the
-//      residuals in shared memory and threads over the calibration rows;
+//      candidate scales on chip (output_error_f16.cu: fp16 hi/lo operands, each residual vector
+//      scaled by a power of two from the bound max(s/2, max|w| - Qmax s) on its elements), or,
+//      for rows that are not 16-byte multiples and for per-channel inputs, one CTA per channel
+//      and candidate chunk with the residuals in shared memory and threads over the calibration
+//      rows;
 //   3. argmin: per channel, or per layer over the channel sums (double, channels in order).
 #include <math.h>
 
@@ -31,10 +33,11 @@ __device__ __forceinline__ float candidate_fraction(int c, int n_cand)
     return __fdiv_rn((float)(c + 1), (float)n_cand);
 }
 
-// One warp per channel: m = max|w| (NaN when a weight is not finite).  Per channel, the candidate
-// row K_c = f_c m; per layer, m is parked in column 0 for clip_layer_kernel.
+// One warp per channel: m = max|w| (NaN when a weight is not finite), also into chmax[k] when
+// given.  Per channel, the candidate row K_c = f_c m; per layer, m is parked in column 0 for
+// clip_layer_kernel.
 __global__ void clip_channel_kernel(const float *__restrict__ W, int C, int d, int n_cand, int mode,
-                                    float *__restrict__ clip)
+                                    float *__restrict__ clip, float *__restrict__ chmax)
 {
     const int k = (int)((blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5);
     const int lane = threadIdx.x & 31;
@@ -52,6 +55,7 @@ __global__ void clip_channel_kernel(const float *__restrict__ W, int C, int d, i
         bad |= __shfl_xor_sync(0xffffffffu, bad, o);
     }
     if (bad) m = NAN;
+    if (chmax && lane == 0) chmax[k] = m;
     if (mode == MPQ_CLIP_PER_CHANNEL) {
         for (int c = lane; c < n_cand; c += 32)
             clip[(size_t)k * n_cand + c] = __fmul_rn(candidate_fraction(c, n_cand), m);
@@ -221,20 +225,36 @@ mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C,
                        int n_cand, int mode, float *clip, float *err, int *best,
                        cudaStream_t stream)
 {
+    // the tensor-core path takes scratch from the stream-ordered pool: channel maxima, the X range
+    // word and the split X planes (2 N d fp16)
+    const bool tc = groups == 1 && output_error_pair_ok(X, W, reinterpret_cast<const int8_t *>(W), d);
+    const size_t max_bytes = ((size_t)C * sizeof(float) + 255) / 256 * 256;
+    char *scratch = nullptr;
+    if (tc) {
+        const mpq_status st = pool_scratch(reinterpret_cast<void **>(&scratch),
+                                           max_bytes + 256 + (size_t)N * d * 2 * sizeof(uint16_t),
+                                           stream);
+        if (st != MPQ_OK) return st;
+    }
+    float *chmax = reinterpret_cast<float *>(scratch);
     const unsigned blocks = (unsigned)(((size_t)C * 32 + CL_THREADS - 1) / CL_THREADS);
-    clip_channel_kernel<<<blocks, CL_THREADS, 0, stream>>>(W, C, d, n_cand, mode, clip);
+    clip_channel_kernel<<<blocks, CL_THREADS, 0, stream>>>(W, C, d, n_cand, mode, clip, chmax);
     cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_status(e, "clip candidate kernel launch");
-    if (mode == MPQ_CLIP_PER_LAYER) {
+    if (e == cudaSuccess && mode == MPQ_CLIP_PER_LAYER) {
         clip_layer_kernel<<<1, 1024, 0, stream>>>(C, n_cand, clip);
         e = cudaGetLastError();
-        if (e != cudaSuccess) return cuda_status(e, "clip layer kernel launch");
     }
-
-    if (groups == 1 && output_error_pair_ok(X, W, reinterpret_cast<const int8_t *>(W), d)) {
-        const mpq_status st = launch_clip_pair(X, N, W, clip, C, d, qmax, n_cand, err, stream);
+    if (tc) {
+        mpq_status st = cuda_status(e, "clip candidate kernel launch");
+        if (st == MPQ_OK)
+            st = launch_clip_f16(X, N, W, clip, chmax, C, d, qmax, n_cand, err,
+                                 reinterpret_cast<unsigned *>(scratch + max_bytes),
+                                 reinterpret_cast<uint16_t *>(scratch + max_bytes + 256), stream);
+        const cudaError_t ef = cudaFreeAsync(scratch, stream);
+        if (st == MPQ_OK) st = cuda_status(ef, "scratch release (cudaFreeAsync)");
         if (st != MPQ_OK) return st;
     } else {
+        if (e != cudaSuccess) return cuda_status(e, "clip candidate kernel launch");
         const size_t smem = (size_t)CL_CHUNK * d * sizeof(float);
         if ((long long)smem > max_smem_optin()) {
             set_error("clip search with d = %d needs %zu bytes of shared memory", d, smem);

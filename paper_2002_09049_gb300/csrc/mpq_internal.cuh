@@ -75,8 +75,12 @@ mpq_status launch_output_error_pair(const float *X, int N, const float *W, const
                                     const float *scales, int C, int d, int k_max, float *err,
                                     cudaStream_t stream, unsigned *range, const float *rmax);
 
-mpq_status launch_clip_pair(const float *X, int N, const float *W, const float *clip, int C, int d,
-                            int qmax, int n_cand, float *err, cudaStream_t stream);
+// Clipping-search errors on the CTA-pair fp16 contraction (output_error_f16.cu): chmax = max|w|
+// per channel; xrange (one word) and xs (2 N d fp16) scratch on `stream`.  Needs
+// output_error_pair_ok(X, W, W, d).
+mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *clip,
+                           const float *chmax, int C, int d, int qmax, int n_cand, float *err,
+                           unsigned *xrange, uint16_t *xs, cudaStream_t stream);
 mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C, int d, int qmax,
                        int n_cand, int mode, float *clip, float *err, int *best,
                        cudaStream_t stream);

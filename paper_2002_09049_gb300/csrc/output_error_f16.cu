@@ -39,6 +39,7 @@
 
 #include "mpq_internal.cuh"
 #include "pair_common.cuh"
+#include "rounding.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
 #include "waits.cuh"
@@ -91,6 +92,9 @@ struct F16Ctrl {
     float vscale[F_VEC];           // 2^e per residual vector
     int vexp[F_VEC];
     int xexp;
+    // clipping search, per residual vector: scale s = K / Qmax, fl(1 / s), 2^e, and the byte
+    // offset of its channel's W row in a raw slot (int bits)
+    float4 clip_row[F_VEC];
 };
 constexpr int F_CTRL_BYTES = (sizeof(F16Ctrl) + 1023) / 1024 * 1024;
 constexpr int F_BASE_SMEM = 1024 /* alignment slack */ + F_CTRL_BYTES + F_ASETS * F_SET +
@@ -112,6 +116,45 @@ struct FGeo {
     static_assert(RAW >= 2, "raw ring needs two slots");
 };
 
+// Clipping search (Eq. 12): n_cand residual vectors per channel, so at most 128 / n_cand
+// channels per CTA, capped at 64 so that two raw slots of W rows fit beside the operand tiles.
+// A raw slot holds W only: [ch][64] fp32.
+__host__ __device__ constexpr int clip_channels(int n_cand)
+{
+    return 128 / n_cand < 64 ? 128 / n_cand : 64;
+}
+
+__host__ __device__ constexpr int clip_raw_bytes(int ch) { return (ch * F_KS * 4 + 1023) / 1024 * 1024; }
+
+__host__ __device__ constexpr int clip_raw_slots(int ch)
+{
+    return (F_SMEM_LIMIT - F_BASE_SMEM) / clip_raw_bytes(ch) < F_MAX_RAW
+               ? (F_SMEM_LIMIT - F_BASE_SMEM) / clip_raw_bytes(ch)
+               : F_MAX_RAW;
+}
+static_assert(clip_raw_slots(64) >= 2, "clipping search: raw ring needs two slots");
+
+// Per-launch sizes: compile-time for the greedy residuals, from n_cand for the clipping search.
+template <int KP1, bool CLIP>
+struct FShape {
+    static constexpr int kp1 = KP1, ch = FGeo<KP1>::CH, raw = FGeo<KP1>::RAW;
+    static constexpr int raw_bytes = FGeo<KP1>::RAW_BYTES, smem = FGeo<KP1>::SMEM;
+    static constexpr uint32_t raw_tx = FGeo<KP1>::RAW_TX;
+    __host__ __device__ explicit FShape(int) {}
+};
+
+template <int KP1>
+struct FShape<KP1, true> {
+    int kp1, ch, raw, raw_bytes, smem;
+    uint32_t raw_tx;
+    __host__ __device__ explicit FShape(int n_cand)
+        : kp1(n_cand), ch(clip_channels(n_cand)), raw(clip_raw_slots(ch)),
+          raw_bytes(clip_raw_bytes(ch)), smem(F_BASE_SMEM + raw * raw_bytes),
+          raw_tx((uint32_t)(ch * F_KS * 4))
+    {
+    }
+};
+
 template <int N>
 __device__ __forceinline__ void setmaxnreg_inc()
 {
@@ -123,6 +166,19 @@ __device__ __forceinline__ void setmaxnreg_dec()
 {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
+
+// A producer thread's greedy items (channel, point scales, 2^e of the residual vectors), the same
+// for every step; none in the clipping search.
+template <int KP1, bool CLIP>
+struct FItems {
+    float sc[FGeo<KP1>::ITEMS][KP1 - 1];
+    float vf[FGeo<KP1>::ITEMS][KP1];
+    int chs[FGeo<KP1>::ITEMS];
+};
+
+template <int KP1>
+struct FItems<KP1, true> {
+};
 
 // Raw slot -> A tiles of one step (tile set `aset`): for every (channel, element pair) item of
 // both 32-element halves the residuals r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7), each scaled by
@@ -174,20 +230,82 @@ __device__ __forceinline__ void f16_make_a(uint32_t slot, uint32_t aset, int pt,
     }
 }
 
-// scales: [C][k_max] point scales; xrange[0]: max|X| as float bits; vrange: max|r| per residual
-// vector ([C][k_max+1], float bits); tmX: the split X planes [2][N][d] fp16.
-template <int KP1>
+// Raw slot -> A tiles of one step for the clipping search (Eq. 12): row v of the CTA is the
+// residual r = w - s q of channel v / n_cand under candidate v mod n_cand (scale s, codes q of
+// Eq. 8; q = 0 where s is 0 or NaN, so that r = w or NaN), scaled by its 2^e and split into fp16
+// hi/lo halves.  Warp j takes the rows v = j (mod 7); lane l takes elements 2l and 2l + 1 of the
+// step, so a warp's stores fill one 128-byte row of each tile.  Four rows at a time: their reads,
+// then their codes from a multiply by 1/s without a branch, redone with the correctly rounded
+// division when any lane's quotient lies near a rounding boundary (a warp-uniform branch), then
+// the residuals and stores.
+__device__ __forceinline__ void f16_make_a_clip(uint32_t slot, uint32_t aset, int warp, int lane,
+                                                int nvec, uint32_t rows, float qmaxf, float qlim,
+                                                float tband)
+{
+    constexpr int U = 4, STEP = F_PROD_WARPS;
+    const uint32_t lofs = (uint32_t)lane * 8u, cofs = (uint32_t)(lane & 3) * 4u;
+    for (int v0 = warp; v0 < nvec; v0 += U * STEP) {
+        float4 p[U];
+        float2 w[U], q[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int v = v0 + u * STEP;
+            if (v < nvec) {
+                p[u] = ld_shared_v4(rows + (uint32_t)v * 16u);
+                w[u] = ld_shared_v2(slot + (uint32_t)__float_as_int(p[u].w) + lofs);
+            }
+        }
+        bool unsure = false;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (v0 + u * STEP < nvec) {
+                q[u].x = code_signed_fast(w[u].x, p[u].y, qmaxf, qlim, tband, unsure);
+                q[u].y = code_signed_fast(w[u].y, p[u].y, qmaxf, qlim, tband, unsure);
+            }
+        }
+        if (__any_sync(0xffffffffu, unsure)) {
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                if (v0 + u * STEP < nvec) {
+                    q[u].x = code_signed_exact(w[u].x, p[u].x, qmaxf);
+                    q[u].y = code_signed_exact(w[u].y, p[u].x, qmaxf);
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int v = v0 + u * STEP;
+            if (v < nvec) {
+                const float s = p[u].x, vf = p[u].z;
+                uint32_t hi, lo;
+                split_f16x2(__fmul_rn(__fmaf_rn(-s, q[u].x, w[u].x), vf),
+                            __fmul_rn(__fmaf_rn(-s, q[u].y, w[u].y), vf), hi, lo);
+                const uint32_t off = sw128_offset(v, lane >> 2) + cofs;
+                st_shared_u32(aset + off, hi);
+                st_shared_u32(aset + F_TILE + off, lo);
+            }
+        }
+    }
+}
+
+// Greedy residuals (CLIP false): scales [C][k_max] point scales; vrange: max|r| per residual
+// vector ([C][k_max+1], float bits); tmQ: the codes.  Clipping search (CLIP, KP1 unused): scales
+// [C][n_cand] candidate clipping factors K; chmax: max|w| per channel; qmax: the code range.
+// Both: xrange[0]: max|X| as float bits; tmX: the split X planes [2][N][d] fp16; tmW: W.
+template <int KP1, bool CLIP>
 __global__ void __launch_bounds__(F_THREADS, 1)
-output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
-                        const unsigned *__restrict__ xrange, const unsigned *__restrict__ vrange,
-                        float *__restrict__ err, int split, const WaitCtl wc,
+output_error_f16_kernel(const float *__restrict__ scales, const float *__restrict__ chmax, int C,
+                        int N, int d, int n_cand, int qmax, const unsigned *__restrict__ xrange,
+                        const unsigned *__restrict__ vrange, float *__restrict__ err, int split,
+                        const WaitCtl wc,
                         const __grid_constant__ CUtensorMap tmX,
                         const __grid_constant__ CUtensorMap tmW,
                         const __grid_constant__ CUtensorMap tmQ)
 {
-    using G = FGeo<KP1>;
-    constexpr int NA = F_ASETS, NB = F_BSLOTS, SEG = F_SEG, R = G::RAW, K = G::K;
-    constexpr unsigned KBIT = MPQ_TIMEOUT_OUTPUT_ERROR;
+    constexpr int NA = F_ASETS, NB = F_BSLOTS, SEG = F_SEG;
+    constexpr unsigned KBIT = CLIP ? MPQ_TIMEOUT_CLIP : MPQ_TIMEOUT_OUTPUT_ERROR;
+    const FShape<KP1, CLIP> S(n_cand);
+    const int R = S.raw, kp1 = S.kp1;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
@@ -203,9 +321,9 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
     const uint16_t pair_mask = (uint16_t)(3u << leader);
     const int pr = (int)(crank >> 1);                // pair index in the cluster: row-tile phase
     const int pair_tile = blockIdx.x / (2 * split);
-    const int k0 = (pair_tile * 2 + half) * G::CH;   // first channel of this CTA
-    const int nch = max(0, min(G::CH, C - k0));
-    const int nvec = nch * KP1;
+    const int k0 = (pair_tile * 2 + half) * S.ch;    // first channel of this CTA
+    const int nch = max(0, min(S.ch, C - k0));
+    const int nvec = nch * kp1;
     const int n_rt = (N + F_N - 1) / F_N;
     const int my_rt = (n_rt - pr + split - 1) / split;
     const int n_ks = (d + F_KS - 1) / F_KS;          // steps per row tile
@@ -214,7 +332,7 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
     // control block, operand tiles and the raw ring within the launch's shared memory (the same in
     // every CTA, so the whole cluster leaves together)
     if (!MPQ_CHECK_SMEM_END((size_t)pad + F_CTRL_BYTES + (size_t)(NA + NB) * F_SET +
-                            (size_t)R * G::RAW_BYTES))
+                            (size_t)R * S.raw_bytes))
         return;
 
     if (threadIdx.x == 0) {
@@ -238,11 +356,30 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
         ctl.abort = 0;
         fence_barrier_init();
     }
-    for (int i = threadIdx.x; i < nvec; i += F_THREADS) {
-        if (!MPQ_IN((size_t)k0 * KP1 + i, (size_t)C * KP1)) continue;
-        const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * KP1 + i)));
-        ctl.vexp[i] = e;
-        ctl.vscale[i] = pow2f(e);
+    if constexpr (CLIP) {
+        // s = K / Qmax; every residual |w - s q| is at most s/2 (q the nearest code) or, where the
+        // code is clamped, max|w| - Qmax s: that bound sets the operand scale (a residual a
+        // rounding above it still fits fp16, whose range reaches 2^16)
+        const float qmaxf = (float)qmax;
+        for (int i = threadIdx.x; i < nvec; i += F_THREADS) {
+            const size_t v = (size_t)k0 * kp1 + i;
+            if (!MPQ_IN(v, (size_t)C * kp1)) continue;
+            const int ch = i / kp1;
+            const float sv = __fdiv_rn(__ldg(scales + v), qmaxf);
+            const float bound = fmaxf(__fmul_rn(0.5f, sv),
+                                      __fmaf_rn(-qmaxf, sv, __ldg(chmax + (size_t)k0 + ch)));
+            const int e = f16_scale_exp(bound);
+            ctl.vexp[i] = e;
+            ctl.clip_row[i] = make_float4(sv, sv > 0.0f ? __frcp_rn(sv) : 0.0f, pow2f(e),
+                                          __int_as_float(ch * F_KS * 4));
+        }
+    } else {
+        for (int i = threadIdx.x; i < nvec; i += F_THREADS) {
+            if (!MPQ_IN((size_t)k0 * KP1 + i, (size_t)C * KP1)) continue;
+            const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * KP1 + i)));
+            ctl.vexp[i] = e;
+            ctl.vscale[i] = pow2f(e);
+        }
     }
     if (threadIdx.x == 0) ctl.xexp = f16_scale_exp(__uint_as_float(__ldg(xrange)));
     if (warp == F_MMA_WARP) {
@@ -260,20 +397,26 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
         if (warp < F_PROD_WARPS) {
             // ------------------------------------------------------------ producers
             const int pt = threadIdx.x;
-            float sc[G::ITEMS][K];      // scales of this thread's items, the same for every step
-            float vf[G::ITEMS][KP1];    // 2^e of the items' residual vectors
-            int chs[G::ITEMS];          // channel of each item
+            FItems<KP1, CLIP> its;
+            if constexpr (!CLIP) {
+                using G = FGeo<KP1>;
+                constexpr int K = G::K;
 #pragma unroll
-            for (int i = 0; i < G::ITEMS; ++i) {
-                const int p = pt + i * F_PT;
-                chs[i] = pair_channel<KP1>(p / 16, nch);
-                const bool own = p < nch * 16;
-                const int k = k0 + chs[i];
+                for (int i = 0; i < G::ITEMS; ++i) {
+                    const int p = pt + i * F_PT;
+                    its.chs[i] = pair_channel<KP1>(p / 16, nch);
+                    const bool own = p < nch * 16;
+                    const int k = k0 + its.chs[i];
 #pragma unroll
-                for (int n = 0; n < K; ++n) sc[i][n] = own ? __ldg(scales + (size_t)k * K + n) : 0.0f;
+                    for (int n = 0; n < K; ++n)
+                        its.sc[i][n] = own ? __ldg(scales + (size_t)k * K + n) : 0.0f;
 #pragma unroll
-                for (int n = 0; n < KP1; ++n) vf[i][n] = own ? ctl.vscale[chs[i] * KP1 + n] : 0.0f;
+                    for (int n = 0; n < KP1; ++n)
+                        its.vf[i][n] = own ? ctl.vscale[its.chs[i] * KP1 + n] : 0.0f;
+                }
             }
+            const float qmaxf = (float)qmax, qlim = qmaxf + 1.0f;
+            const float tband = 0.5f - MPQ_FAST_REL * (qlim + 1.0f);
             int s = 0, slot = 0, sb = 0;
             uint32_t aph = 0, rph = 0, bph = 0;    // phase parities of stage s, slot, B slot sb
             for (int it = 0; it < total; ++it) {
@@ -284,7 +427,12 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
                     note_timeout(wc, KBIT);
                 }
                 if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-                f16_make_a<KP1>(ring_u32 + slot * G::RAW_BYTES, a_u32 + s * F_SET, pt, nch, chs, sc, vf);
+                if constexpr (CLIP)
+                    f16_make_a_clip(ring_u32 + slot * S.raw_bytes, a_u32 + s * F_SET, warp, lane,
+                                    nvec, smem_u32(ctl.clip_row), qmaxf, qlim, tband);
+                else
+                    f16_make_a<KP1>(ring_u32 + slot * S.raw_bytes, a_u32 + s * F_SET, pt, nch,
+                                    its.chs, its.sc, its.vf);
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&ctl.raw_empty[slot]);
@@ -390,7 +538,7 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
         if (copier && lane == 0) {
             prefetch_tensormap(&tmX);
             prefetch_tensormap(&tmW);
-            prefetch_tensormap(&tmQ);
+            if constexpr (!CLIP) prefetch_tensormap(&tmQ);
         }
         for (int g = 0; g < nseg_all; ++g) {
             const uint32_t b = (uint32_t)g & 1u, par = (uint32_t)(g >> 1) & 1u;
@@ -400,20 +548,23 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
                     if (lane == 0) {
                         const int f = next, x = (f % n_ks) * F_KS;
                         const int rslot = f % R, bslot = f % NB;
-                        const uint32_t rdst = ring_u32 + rslot * G::RAW_BYTES;
+                        const uint32_t rdst = ring_u32 + rslot * S.raw_bytes;
                         const uint32_t bdst = b_u32 + bslot * F_SET;
                         const int row0 = (pr + (f / n_ks) * split) * F_N + half * F_ROWS;
                         // a tile copy starts 16-byte aligned (x counts int8 codes in the code
                         // map) into a 1024-byte aligned destination (128-byte swizzle), or is not
-                        // issued and the launch ends through the bounded waits
+                        // issued and the launch ends through the bounded waits; the raw slot
+                        // takes W rows (and the codes of the greedy residuals)
                         ok = MPQ_CHECK((x & 15) == 0 && (rdst & 15u) == 0u && (bdst & 1023u) == 0u &&
                                        x < d);
                         if (ok && f >= R)
                             ok = mbar_wait(&ctl.raw_empty[rslot], (uint32_t)((f - R) / R) & 1u, wc.budget);
                         if (ok) {
-                            mbar_arrive_expect_tx(&ctl.raw_full[rslot], G::RAW_TX);
+                            mbar_arrive_expect_tx(&ctl.raw_full[rslot], S.raw_tx);
                             tma_load_2d(rdst, &tmW, x, k0, &ctl.raw_full[rslot]);
-                            tma_load_3d(rdst + G::RAW_Q, &tmQ, x, k0, 0, &ctl.raw_full[rslot]);
+                            if constexpr (!CLIP)
+                                tma_load_3d(rdst + FGeo<KP1>::RAW_Q, &tmQ, x, k0, 0,
+                                            &ctl.raw_full[rslot]);
                             raw_issued = f + 1;
                         }
                         if (ok && f >= NB)
@@ -493,7 +644,7 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
             }
             double v = s / (double)N;
             v *= pow2d(-2 * (ctl.xexp + ctl.vexp[m]));   // exact: undo the operand scales
-            if (MPQ_IN((size_t)k0 * KP1 + m, (size_t)C * KP1)) err[(size_t)k0 * KP1 + m] = (float)v;
+            if (MPQ_IN((size_t)k0 * kp1 + m, (size_t)C * kp1)) err[(size_t)k0 * kp1 + m] = (float)v;
         }
     }
     cluster_sync();
@@ -523,13 +674,14 @@ f16_split_kernel(const float4 *__restrict__ X, long long n8, const unsigned *__r
     }
 }
 
-template <int KP1>
+template <int KP1, bool CLIP>
 mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes,
-                      const float *scales, int C, int d, float *err, const unsigned *xrange,
-                      const unsigned *vrange, uint16_t *xs, cudaStream_t stream)
+                      const float *scales, const float *chmax, int C, int d, int n_cand, int qmax,
+                      float *err, const unsigned *xrange, const unsigned *vrange, uint16_t *xs,
+                      cudaStream_t stream)
 {
-    using G = FGeo<KP1>;
-    const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
+    const FShape<KP1, CLIP> S(n_cand);
+    const int n_pairs = (C + 2 * S.ch - 1) / (2 * S.ch);
     const int n_rt = (N + F_N - 1) / F_N;
 
     CUtensorMap tmX, tmW, tmQ;
@@ -540,28 +692,32 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
     const cuuint64_t sx[2] = {(cuuint64_t)d * 2, (cuuint64_t)N * d * 2};
     const cuuint32_t bx[3] = {F_KS, F_ROWS, 2};
     const cuuint64_t dw[2] = {(cuuint64_t)d, (cuuint64_t)C}, sw[1] = {(cuuint64_t)d * 4};
-    const cuuint32_t bw[2] = {F_KS, (cuuint32_t)G::CH};
-    const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)C, (cuuint64_t)G::K};
-    const cuuint64_t sq[2] = {(cuuint64_t)d, (cuuint64_t)C * d};
-    const cuuint32_t bq[3] = {F_KS, (cuuint32_t)G::CH, (cuuint32_t)G::K};
-    if (!encode_tile_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, xs, dx, sx, bx,
-                         CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_tile_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw) ||
-        !encode_tile_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq)) {
+    const cuuint32_t bw[2] = {F_KS, (cuuint32_t)S.ch};
+    bool maps = encode_tile_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, xs, dx, sx, bx,
+                                CU_TENSOR_MAP_SWIZZLE_128B) &&
+                encode_tile_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw);
+    if constexpr (!CLIP) {
+        using G = FGeo<KP1>;
+        const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)C, (cuuint64_t)G::K};
+        const cuuint64_t sq[2] = {(cuuint64_t)d, (cuuint64_t)C * d};
+        const cuuint32_t bq[3] = {F_KS, (cuuint32_t)G::CH, (cuuint32_t)G::K};
+        maps = maps && encode_tile_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq);
+    }
+    if (!maps) {
         set_error("output error: tensor map encoding failed");
         return MPQ_ERR_CUDA;
     }
-    if ((long long)G::SMEM > max_smem_optin()) {
-        set_error("fp16 output error needs %d bytes of shared memory", G::SMEM);
+    if ((long long)S.smem > max_smem_optin()) {
+        set_error("fp16 output error needs %d bytes of shared memory", (int)S.smem);
         return MPQ_ERR_UNSUPPORTED;
     }
-    cudaError_t e = cudaFuncSetAttribute(output_error_f16_kernel<KP1>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(output_error_f16_kernel<KP1, CLIP>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)S.smem);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
 
     cudaLaunchConfig_t cfg = {};
     cfg.blockDim = dim3(F_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = (size_t)G::SMEM;
+    cfg.dynamicSmemBytes = (size_t)S.smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -572,7 +728,8 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
 
     // Row tiles split over `split` pairs per cluster (clusters of 2 * split CTAs): the split with
     // the least (waves of resident clusters) x (row tiles per CTA), ties to the smaller cluster;
-    // resident clusters per cluster size queried once per process (one device per process).
+    // resident clusters per cluster size queried once per process (one device per process; the
+    // 512 threads x 128 registers of a CTA fill an SM whatever its shared memory).
     static std::atomic<int> resident[3] = {{0}, {0}, {0}};
     int split = 1;
     long long best = -1;
@@ -581,7 +738,7 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
         cfg.gridDim = dim3((unsigned)(n_pairs * 2 * sp), 1, 1);
         int active = resident[i].load(std::memory_order_relaxed);
         if (active == 0) {
-            if (cudaOccupancyMaxActiveClusters(&active, output_error_f16_kernel<KP1>, &cfg) !=
+            if (cudaOccupancyMaxActiveClusters(&active, output_error_f16_kernel<KP1, CLIP>, &cfg) !=
                 cudaSuccess)
                 active = -1;
             (void)cudaGetLastError();
@@ -608,8 +765,8 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
         reinterpret_cast<uint4 *>(xs + (size_t)N * d));
     e = cudaGetLastError();
     if (e == cudaSuccess)
-        e = cudaLaunchKernelEx(&cfg, output_error_f16_kernel<KP1>, scales, C, N, d, xrange, vrange,
-                               err, split, wc, tmX, tmW, tmQ);
+        e = cudaLaunchKernelEx(&cfg, output_error_f16_kernel<KP1, CLIP>, scales, chmax, C, N, d,
+                               n_cand, qmax, xrange, vrange, err, split, wc, tmX, tmW, tmQ);
     return cuda_status(e, "fp16 output-error kernel launch");
 }
 
@@ -621,8 +778,10 @@ mpq_status launch_output_error_f16(const float *X, int N, const float *W, const 
                                    cudaStream_t stream)
 {
     switch (k_max + 1) {
-#define MPQ_CASE(n) \
-    case n: return launch_f16<n>(X, N, W, codes, scales, C, d, err, xrange, vrange, xs, stream);
+#define MPQ_CASE(n)                                                                             \
+    case n:                                                                                     \
+        return launch_f16<n, false>(X, N, W, codes, scales, nullptr, C, d, 0, 0, err, xrange,  \
+                                    vrange, xs, stream);
         MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7) MPQ_CASE(8)
         MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14) MPQ_CASE(15)
         MPQ_CASE(16) MPQ_CASE(17)
@@ -630,6 +789,16 @@ mpq_status launch_output_error_f16(const float *X, int N, const float *W, const 
     }
     set_error("k_max = %d unsupported", k_max);
     return MPQ_ERR_UNSUPPORTED;
+}
+
+mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *clip,
+                           const float *chmax, int C, int d, int qmax, int n_cand, float *err,
+                           unsigned *xrange, uint16_t *xs, cudaStream_t stream)
+{
+    const mpq_status st = launch_x_range(X, N, d, xrange, stream);
+    if (st != MPQ_OK) return st;
+    return launch_f16<1, true>(X, N, W, nullptr, clip, chmax, C, d, n_cand, qmax, err, xrange,
+                               nullptr, xs, stream);
 }
 
 }  // namespace mpq

@@ -662,18 +662,18 @@ pair_range_kernel(const float4 *__restrict__ X, long long nx4, int xb, const flo
     }
 }
 
-// The range pre-pass into `range` (zeroed here): max|X| into range[0] and, without rmax, max|r| of
-// every residual vector into range[1 + k (k_max+1) + n].
+// The range pre-pass into `range` (zeroed here): max|X| into range[0] and, with `residuals`, max|r|
+// of every residual vector into range[1 + k (k_max+1) + n].
 template <int KP1>
 cudaError_t launch_ranges(const float *X, int N, const float *W, const int8_t *codes,
-                          const float *scales, int C, int d, const float *rmax, unsigned *range,
+                          const float *scales, int C, int d, bool residuals, unsigned *range,
                           cudaStream_t stream)
 {
-    const size_t words = rmax ? 1 : 1 + (size_t)C * KP1;
+    const size_t words = residuals ? 1 + (size_t)C * KP1 : 1;
     const long long nx4 = (long long)N * d / 4;
     const int xb = (int)std::min<long long>((nx4 + 1023) / 1024, 4LL * sm_count());
     const int rsplit = std::min(8, std::max(1, (d / 4 + 255) / 256));   // >= 8 loads per lane
-    const long long cb = rmax ? 0 : ((long long)C * rsplit + 7) / 8;
+    const long long cb = residuals ? ((long long)C * rsplit + 7) / 8 : 0;
     cudaError_t e = cudaMemsetAsync(range, 0, words * sizeof(unsigned), stream);
     if (e != cudaSuccess) return e;
     pair_range_kernel<KP1><<<(unsigned)(xb + cb), 256, 0, stream>>>(
@@ -697,7 +697,8 @@ mpq_status launch_pooled_f16(const float *X, int N, const float *W, const int8_t
     if (st != MPQ_OK) return st;
     unsigned *range = static_cast<unsigned *>(scratch);
     uint16_t *xs = reinterpret_cast<uint16_t *>(static_cast<char *>(scratch) + range_bytes);
-    const cudaError_t e = launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax, range, stream);
+    const cudaError_t e =
+        launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax == nullptr, range, stream);
     mpq_status r = cuda_status(e, "output-error range pre-pass");
     if (r == MPQ_OK) {
         const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : range + 1;
@@ -795,7 +796,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         // fp16 operands (the fixed-scratch entry point): the ranges of X and of every residual
         // vector first, into the caller's table (the residual vectors' from rmax when the greedy
         // search gave them: then the pre-pass reads X alone)
-        e = launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax, ext_range, stream);
+        e = launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax == nullptr, ext_range, stream);
         const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : ext_range + 1;
         if (e == cudaSuccess)
             e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
@@ -891,21 +892,10 @@ mpq_status launch_output_error_pair(const float *X, int N, const float *W, const
     return MPQ_ERR_UNSUPPORTED;
 }
 
-mpq_status launch_clip_pair(const float *X, int N, const float *W, const float *clip, int C, int d,
-                            int qmax, int n_cand, float *err, cudaStream_t stream)
+mpq_status launch_x_range(const float *X, int N, int d, unsigned *range, cudaStream_t stream)
 {
-    switch (n_cand) {
-#define MPQ_CASE(n) \
-    case n: return launch_pair<n, true>(X, N, W, nullptr, clip, C, d, qmax, err, stream);
-        MPQ_CASE(1) MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7)
-        MPQ_CASE(8) MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14)
-        MPQ_CASE(15) MPQ_CASE(16) MPQ_CASE(17) MPQ_CASE(18) MPQ_CASE(19) MPQ_CASE(20) MPQ_CASE(21)
-        MPQ_CASE(22) MPQ_CASE(23) MPQ_CASE(24) MPQ_CASE(25) MPQ_CASE(26) MPQ_CASE(27) MPQ_CASE(28)
-        MPQ_CASE(29) MPQ_CASE(30) MPQ_CASE(31) MPQ_CASE(32)
-#undef MPQ_CASE
-    }
-    set_error("n_cand = %d unsupported", n_cand);
-    return MPQ_ERR_UNSUPPORTED;
+    return cuda_status(launch_ranges<2>(X, N, nullptr, nullptr, nullptr, 0, d, false, range, stream),
+                       "X range pass");
 }
 
 }  // namespace mpq

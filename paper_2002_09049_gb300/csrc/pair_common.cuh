@@ -68,6 +68,9 @@ bool encode_tile_map(CUtensorMap *m, CUtensorMapDataType type, int rank, const v
                      const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box,
                      CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_NONE);
 
+// Host: max|X| (float bits) into range[0], zeroed first (N d a multiple of 4, X 16-byte aligned).
+mpq_status launch_x_range(const float *X, int N, int d, unsigned *range, cudaStream_t stream);
+
 // Host: the output error of the greedy residuals on output_error_f16.cu's kernel, with its range
 // table ready on `stream` (xrange[0] = max|X|, vrange = max|r| per residual vector, float bits)
 // and `xs` scratch of 2 N d fp16 for the split X planes.

@@ -37,4 +37,24 @@ __device__ __forceinline__ float code_fast_f(float a, float s, float inv_s, floa
     return fminf(rintf(__fdiv_rn(a, s)), qmaxf);
 }
 
+// Signed code clamp(rint(w (1/s)), -Qmax, Qmax) without a branch, for clamp(rint(fl(w/s)), ...)
+// (Eq. 8 with the sign of w; rint and fl are symmetric).  `unsure` is set where the two may differ:
+// |q'| < Qmax + 1 = qlim and q' within 0.5 - tband of a half-integer, tband = 0.5 - 2^-20 (qlim + 1)
+// (at least MPQ_FAST_REL (|q'| + 1) for every |q'| < qlim).  At |q'| >= qlim both clamp to +-Qmax.
+// inv_s = 0 gives q = 0 (scales 0 or NaN).
+__device__ __forceinline__ float code_signed_fast(float w, float inv_s, float qmaxf, float qlim,
+                                                  float tband, bool &unsure)
+{
+    const float qf = __fmul_rn(w, inv_s);
+    const float rq = rintf(qf);
+    unsure |= fabsf(__fsub_rn(qf, rq)) >= tband && fabsf(qf) < qlim;
+    return fminf(fmaxf(rq, -qmaxf), qmaxf);
+}
+
+// The exact signed code clamp(rint(fl(w/s)), -Qmax, Qmax) for s > 0, 0 otherwise.
+__device__ __forceinline__ float code_signed_exact(float w, float s, float qmaxf)
+{
+    return s > 0.0f ? fminf(fmaxf(rintf(__fdiv_rn(w, s)), -qmaxf), qmaxf) : 0.0f;
+}
+
 }  // namespace mpq
