@@ -55,7 +55,8 @@ constexpr int F_VEC = 128;                 // residual vectors per CTA (TMEM lan
 constexpr int F_ROWS = 128;                // calibration rows per CTA
 constexpr int F_N = 2 * F_ROWS;            // rows per pair row tile (UMMA N)
 constexpr int F_KS = 64;                   // elements per step: one 128-byte fp16 row
-constexpr int F_ASETS = 2;                 // A operand stages (tile sets)
+constexpr int F_ASETS = 2;                 // A operand stages (tile sets) written by the producers
+constexpr int F_PRE_ASETS = 3;             // A operand stages filled by tile copies (clipping search)
 constexpr int F_BSLOTS = 3;                // B operand slots
 constexpr int F_SEG = 4;                   // steps per accumulation segment (256 elements)
 constexpr int F_PROD_WARPS = 7;
@@ -77,8 +78,9 @@ constexpr uint32_t F_TMEM_COLS = 512;
 constexpr int F_SMEM_LIMIT = 232448;       // opt-in shared memory per CTA on sm_100 parts
 
 struct F16Ctrl {
-    uint64_t full[F_ASETS];        // even CTA: both CTAs' producer warps (A written, B landed)
-    uint64_t empty[F_ASETS];       // both CTAs: pair MMA commit (A stage free)
+    uint64_t full[F_PRE_ASETS];    // even CTA: both CTAs' producer warps (A written, B landed)
+    uint64_t empty[F_PRE_ASETS];   // both CTAs: pair MMA commit (A stage free)
+    uint64_t afull[F_PRE_ASETS];   // this CTA's A tile copy (clipping search)
     uint64_t bfull[F_BSLOTS];      // this CTA's B tile copy
     uint64_t bempty[F_BSLOTS];     // both CTAs: pair MMA commit (B slot free)
     uint64_t raw_full[F_MAX_RAW];  // this CTA's W and code tile copies
@@ -92,9 +94,6 @@ struct F16Ctrl {
     float vscale[F_VEC];           // 2^e per residual vector
     int vexp[F_VEC];
     int xexp;
-    // clipping search, per residual vector: scale s = K / Qmax, fl(1 / s), 2^e, and the byte
-    // offset of its channel's W row in a raw slot (int bits)
-    float4 clip_row[F_VEC];
 };
 constexpr int F_CTRL_BYTES = (sizeof(F16Ctrl) + 1023) / 1024 * 1024;
 constexpr int F_BASE_SMEM = 1024 /* alignment slack */ + F_CTRL_BYTES + F_ASETS * F_SET +
@@ -116,44 +115,23 @@ struct FGeo {
     static_assert(RAW >= 2, "raw ring needs two slots");
 };
 
-// Clipping search (Eq. 12): n_cand residual vectors per channel, so at most 128 / n_cand
-// channels per CTA, capped at 64 so that two raw slots of W rows fit beside the operand tiles.
-// A raw slot holds W only: [ch][64] fp32.
-__host__ __device__ constexpr int clip_channels(int n_cand)
-{
-    return 128 / n_cand < 64 ? 128 / n_cand : 64;
-}
-
-__host__ __device__ constexpr int clip_raw_bytes(int ch) { return (ch * F_KS * 4 + 1023) / 1024 * 1024; }
-
-__host__ __device__ constexpr int clip_raw_slots(int ch)
-{
-    return (F_SMEM_LIMIT - F_BASE_SMEM) / clip_raw_bytes(ch) < F_MAX_RAW
-               ? (F_SMEM_LIMIT - F_BASE_SMEM) / clip_raw_bytes(ch)
-               : F_MAX_RAW;
-}
-static_assert(clip_raw_slots(64) >= 2, "clipping search: raw ring needs two slots");
-
-// Per-launch sizes: compile-time for the greedy residuals, from n_cand for the clipping search.
+// Per-launch sizes.  Greedy residuals: whole channels of k_max + 1 vectors per CTA, W and codes
+// through the raw ring, A written by the producers.  Clipping search: 128 residual vectors per CTA
+// whatever their channel, A tiles copied from the residual planes (no raw ring).
 template <int KP1, bool CLIP>
 struct FShape {
-    static constexpr int kp1 = KP1, ch = FGeo<KP1>::CH, raw = FGeo<KP1>::RAW;
+    static constexpr int kp1 = KP1, ch = FGeo<KP1>::CH, raw = FGeo<KP1>::RAW, na = F_ASETS;
     static constexpr int raw_bytes = FGeo<KP1>::RAW_BYTES, smem = FGeo<KP1>::SMEM;
     static constexpr uint32_t raw_tx = FGeo<KP1>::RAW_TX;
-    __host__ __device__ explicit FShape(int) {}
 };
 
 template <int KP1>
 struct FShape<KP1, true> {
-    int kp1, ch, raw, raw_bytes, smem;
-    uint32_t raw_tx;
-    __host__ __device__ explicit FShape(int n_cand)
-        : kp1(n_cand), ch(clip_channels(n_cand)), raw(clip_raw_slots(ch)),
-          raw_bytes(clip_raw_bytes(ch)), smem(F_BASE_SMEM + raw * raw_bytes),
-          raw_tx((uint32_t)(ch * F_KS * 4))
-    {
-    }
+    static constexpr int kp1 = 1, ch = F_VEC, raw = 0, na = F_PRE_ASETS, raw_bytes = 0;
+    static constexpr int smem = 1024 + F_CTRL_BYTES + (F_PRE_ASETS + F_BSLOTS) * F_SET;
+    static constexpr uint32_t raw_tx = 0;
 };
+static_assert(FShape<1, true>::smem <= F_SMEM_LIMIT, "clipping search: shared memory");
 
 template <int N>
 __device__ __forceinline__ void setmaxnreg_inc()
@@ -166,19 +144,6 @@ __device__ __forceinline__ void setmaxnreg_dec()
 {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
-
-// A producer thread's greedy items (channel, point scales, 2^e of the residual vectors), the same
-// for every step; none in the clipping search.
-template <int KP1, bool CLIP>
-struct FItems {
-    float sc[FGeo<KP1>::ITEMS][KP1 - 1];
-    float vf[FGeo<KP1>::ITEMS][KP1];
-    int chs[FGeo<KP1>::ITEMS];
-};
-
-template <int KP1>
-struct FItems<KP1, true> {
-};
 
 // Raw slot -> A tiles of one step (tile set `aset`): for every (channel, element pair) item of
 // both 32-element halves the residuals r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7), each scaled by
@@ -230,82 +195,23 @@ __device__ __forceinline__ void f16_make_a(uint32_t slot, uint32_t aset, int pt,
     }
 }
 
-// Raw slot -> A tiles of one step for the clipping search (Eq. 12): row v of the CTA is the
-// residual r = w - s q of channel v / n_cand under candidate v mod n_cand (scale s, codes q of
-// Eq. 8; q = 0 where s is 0 or NaN, so that r = w or NaN), scaled by its 2^e and split into fp16
-// hi/lo halves.  Warp j takes the rows v = j (mod 7); lane l takes elements 2l and 2l + 1 of the
-// step, so a warp's stores fill one 128-byte row of each tile.  Four rows at a time: their reads,
-// then their codes from a multiply by 1/s without a branch, redone with the correctly rounded
-// division when any lane's quotient lies near a rounding boundary (a warp-uniform branch), then
-// the residuals and stores.
-__device__ __forceinline__ void f16_make_a_clip(uint32_t slot, uint32_t aset, int warp, int lane,
-                                                int nvec, uint32_t rows, float qmaxf, float qlim,
-                                                float tband)
-{
-    constexpr int U = 4, STEP = F_PROD_WARPS;
-    const uint32_t lofs = (uint32_t)lane * 8u, cofs = (uint32_t)(lane & 3) * 4u;
-    for (int v0 = warp; v0 < nvec; v0 += U * STEP) {
-        float4 p[U];
-        float2 w[U], q[U];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int v = v0 + u * STEP;
-            if (v < nvec) {
-                p[u] = ld_shared_v4(rows + (uint32_t)v * 16u);
-                w[u] = ld_shared_v2(slot + (uint32_t)__float_as_int(p[u].w) + lofs);
-            }
-        }
-        bool unsure = false;
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            if (v0 + u * STEP < nvec) {
-                q[u].x = code_signed_fast(w[u].x, p[u].y, qmaxf, qlim, tband, unsure);
-                q[u].y = code_signed_fast(w[u].y, p[u].y, qmaxf, qlim, tband, unsure);
-            }
-        }
-        if (__any_sync(0xffffffffu, unsure)) {
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                if (v0 + u * STEP < nvec) {
-                    q[u].x = code_signed_exact(w[u].x, p[u].x, qmaxf);
-                    q[u].y = code_signed_exact(w[u].y, p[u].x, qmaxf);
-                }
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int v = v0 + u * STEP;
-            if (v < nvec) {
-                const float s = p[u].x, vf = p[u].z;
-                uint32_t hi, lo;
-                split_f16x2(__fmul_rn(__fmaf_rn(-s, q[u].x, w[u].x), vf),
-                            __fmul_rn(__fmaf_rn(-s, q[u].y, w[u].y), vf), hi, lo);
-                const uint32_t off = sw128_offset(v, lane >> 2) + cofs;
-                st_shared_u32(aset + off, hi);
-                st_shared_u32(aset + F_TILE + off, lo);
-            }
-        }
-    }
-}
-
 // Greedy residuals (CLIP false): scales [C][k_max] point scales; vrange: max|r| per residual
-// vector ([C][k_max+1], float bits); tmQ: the codes.  Clipping search (CLIP, KP1 unused): scales
-// [C][n_cand] candidate clipping factors K; chmax: max|w| per channel; qmax: the code range.
-// Both: xrange[0]: max|X| as float bits; tmX: the split X planes [2][N][d] fp16; tmW: W.
+// vector ([C][k_max+1], float bits); tmW: W; tmQ: the codes.  Clipping search (CLIP, KP1 unused):
+// C residual vectors, given as fp16 hi/lo planes (tmW: [2][C][d], clip_planes_kernel); vrange:
+// the bound on each vector's elements that set its operand scale.  Both: xrange[0]: max|X| as
+// float bits; tmX: the split X planes [2][N][d] fp16.
 template <int KP1, bool CLIP>
 __global__ void __launch_bounds__(F_THREADS, 1)
-output_error_f16_kernel(const float *__restrict__ scales, const float *__restrict__ chmax, int C,
-                        int N, int d, int n_cand, int qmax, const unsigned *__restrict__ xrange,
-                        const unsigned *__restrict__ vrange, float *__restrict__ err, int split,
-                        const WaitCtl wc,
+output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
+                        const unsigned *__restrict__ xrange, const unsigned *__restrict__ vrange,
+                        float *__restrict__ err, int split, const WaitCtl wc,
                         const __grid_constant__ CUtensorMap tmX,
                         const __grid_constant__ CUtensorMap tmW,
                         const __grid_constant__ CUtensorMap tmQ)
 {
-    constexpr int NA = F_ASETS, NB = F_BSLOTS, SEG = F_SEG;
+    using S = FShape<KP1, CLIP>;
+    constexpr int NA = S::na, NB = F_BSLOTS, SEG = F_SEG, R = S::raw, kp1 = S::kp1;
     constexpr unsigned KBIT = CLIP ? MPQ_TIMEOUT_CLIP : MPQ_TIMEOUT_OUTPUT_ERROR;
-    const FShape<KP1, CLIP> S(n_cand);
-    const int R = S.raw, kp1 = S.kp1;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t pad = (1024u - (raw_u32 & 1023u)) & 1023u;
@@ -321,8 +227,8 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
     const uint16_t pair_mask = (uint16_t)(3u << leader);
     const int pr = (int)(crank >> 1);                // pair index in the cluster: row-tile phase
     const int pair_tile = blockIdx.x / (2 * split);
-    const int k0 = (pair_tile * 2 + half) * S.ch;    // first channel of this CTA
-    const int nch = max(0, min(S.ch, C - k0));
+    const int k0 = (pair_tile * 2 + half) * S::ch;    // first channel (clip: vector) of this CTA
+    const int nch = max(0, min(S::ch, C - k0));
     const int nvec = nch * kp1;
     const int n_rt = (N + F_N - 1) / F_N;
     const int my_rt = (n_rt - pr + split - 1) / split;
@@ -332,13 +238,15 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
     // control block, operand tiles and the raw ring within the launch's shared memory (the same in
     // every CTA, so the whole cluster leaves together)
     if (!MPQ_CHECK_SMEM_END((size_t)pad + F_CTRL_BYTES + (size_t)(NA + NB) * F_SET +
-                            (size_t)R * S.raw_bytes))
+                            (size_t)R * S::raw_bytes))
         return;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NA; ++s) {
-            mbar_init(&ctl.full[s], 2 * F_PROD_WARPS);
+            // both CTAs' producer warps, or (CLIP) one relay warp per CTA
+            mbar_init(&ctl.full[s], CLIP ? 2 : 2 * F_PROD_WARPS);
             mbar_init(&ctl.empty[s], 1);
+            mbar_init(&ctl.afull[s], 1);
         }
         for (int s = 0; s < NB; ++s) {
             mbar_init(&ctl.bfull[s], 1);
@@ -356,30 +264,11 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
         ctl.abort = 0;
         fence_barrier_init();
     }
-    if constexpr (CLIP) {
-        // s = K / Qmax; every residual |w - s q| is at most s/2 (q the nearest code) or, where the
-        // code is clamped, max|w| - Qmax s: that bound sets the operand scale (a residual a
-        // rounding above it still fits fp16, whose range reaches 2^16)
-        const float qmaxf = (float)qmax;
-        for (int i = threadIdx.x; i < nvec; i += F_THREADS) {
-            const size_t v = (size_t)k0 * kp1 + i;
-            if (!MPQ_IN(v, (size_t)C * kp1)) continue;
-            const int ch = i / kp1;
-            const float sv = __fdiv_rn(__ldg(scales + v), qmaxf);
-            const float bound = fmaxf(__fmul_rn(0.5f, sv),
-                                      __fmaf_rn(-qmaxf, sv, __ldg(chmax + (size_t)k0 + ch)));
-            const int e = f16_scale_exp(bound);
-            ctl.vexp[i] = e;
-            ctl.clip_row[i] = make_float4(sv, sv > 0.0f ? __frcp_rn(sv) : 0.0f, pow2f(e),
-                                          __int_as_float(ch * F_KS * 4));
-        }
-    } else {
-        for (int i = threadIdx.x; i < nvec; i += F_THREADS) {
-            if (!MPQ_IN((size_t)k0 * KP1 + i, (size_t)C * KP1)) continue;
-            const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * KP1 + i)));
-            ctl.vexp[i] = e;
-            ctl.vscale[i] = pow2f(e);
-        }
+    for (int i = threadIdx.x; i < nvec; i += F_THREADS) {
+        if (!MPQ_IN((size_t)k0 * kp1 + i, (size_t)C * kp1)) continue;
+        const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * kp1 + i)));
+        ctl.vexp[i] = e;
+        ctl.vscale[i] = pow2f(e);
     }
     if (threadIdx.x == 0) ctl.xexp = f16_scale_exp(__uint_as_float(__ldg(xrange)));
     if (warp == F_MMA_WARP) {
@@ -394,29 +283,48 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
     // one setmaxnreg per warpgroup: 0-1 (producers, MMA issuer) give registers to 2-3 (epilogue)
     if (warp < F_EPI_WARP0) {
         setmaxnreg_dec<F_REGS_LOW>();
-        if (warp < F_PROD_WARPS) {
-            // ------------------------------------------------------------ producers
-            const int pt = threadIdx.x;
-            FItems<KP1, CLIP> its;
-            if constexpr (!CLIP) {
-                using G = FGeo<KP1>;
-                constexpr int K = G::K;
-#pragma unroll
-                for (int i = 0; i < G::ITEMS; ++i) {
-                    const int p = pt + i * F_PT;
-                    its.chs[i] = pair_channel<KP1>(p / 16, nch);
-                    const bool own = p < nch * 16;
-                    const int k = k0 + its.chs[i];
-#pragma unroll
-                    for (int n = 0; n < K; ++n)
-                        its.sc[i][n] = own ? __ldg(scales + (size_t)k * K + n) : 0.0f;
-#pragma unroll
-                    for (int n = 0; n < KP1; ++n)
-                        its.vf[i][n] = own ? ctl.vscale[its.chs[i] * KP1 + n] : 0.0f;
+        if (CLIP && warp == 0) {
+            // ------------------------------------------------------------ relay (clipping search)
+            // a step's A and B tiles of this CTA have landed: report the stage full
+            int s = 0, sb = 0;
+            uint32_t aph = 0, bph = 0;
+            for (int it = 0; it < total; ++it) {
+                const bool ok = mbar_wait(&ctl.afull[s], aph, wc.budget) &&
+                                mbar_wait(&ctl.bfull[sb], bph, wc.budget);
+                if (!ok) {
+                    *abort_flag = 1;
+                    note_timeout(wc, KBIT);
+                }
+                if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
+                if (lane == 0) mbar_arrive_cluster(&ctl.full[s], leader);
+                if (++s == NA) {
+                    s = 0;
+                    aph ^= 1u;
+                }
+                if (++sb == NB) {
+                    sb = 0;
+                    bph ^= 1u;
                 }
             }
-            const float qmaxf = (float)qmax, qlim = qmaxf + 1.0f;
-            const float tband = 0.5f - MPQ_FAST_REL * (qlim + 1.0f);
+        } else if (!CLIP && warp < F_PROD_WARPS) {
+            // ------------------------------------------------------------ producers
+            using G = FGeo<CLIP ? 2 : KP1>;
+            constexpr int K = G::K;
+            const int pt = threadIdx.x;
+            float sc[G::ITEMS][K];      // scales of this thread's items, the same for every step
+            float vf[G::ITEMS][K + 1];  // 2^e of the items' residual vectors
+            int chs[G::ITEMS];          // channel of each item
+#pragma unroll
+            for (int i = 0; i < G::ITEMS; ++i) {
+                const int p = pt + i * F_PT;
+                chs[i] = pair_channel<K + 1>(p / 16, nch);
+                const bool own = p < nch * 16;
+                const int k = k0 + chs[i];
+#pragma unroll
+                for (int n = 0; n < K; ++n) sc[i][n] = own ? __ldg(scales + (size_t)k * K + n) : 0.0f;
+#pragma unroll
+                for (int n = 0; n <= K; ++n) vf[i][n] = own ? ctl.vscale[chs[i] * (K + 1) + n] : 0.0f;
+            }
             int s = 0, slot = 0, sb = 0;
             uint32_t aph = 0, rph = 0, bph = 0;    // phase parities of stage s, slot, B slot sb
             for (int it = 0; it < total; ++it) {
@@ -427,12 +335,8 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
                     note_timeout(wc, KBIT);
                 }
                 if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-                if constexpr (CLIP)
-                    f16_make_a_clip(ring_u32 + slot * S.raw_bytes, a_u32 + s * F_SET, warp, lane,
-                                    nvec, smem_u32(ctl.clip_row), qmaxf, qlim, tband);
-                else
-                    f16_make_a<KP1>(ring_u32 + slot * S.raw_bytes, a_u32 + s * F_SET, pt, nch,
-                                    its.chs, its.sc, its.vf);
+                f16_make_a<K + 1>(ring_u32 + slot * G::RAW_BYTES, a_u32 + s * F_SET, pt, nch, chs,
+                                  sc, vf);
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&ctl.raw_empty[slot]);
@@ -448,7 +352,7 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
                     s = 0;
                     aph ^= 1u;
                 }
-                if (++slot == R) {
+                if (++slot == G::RAW) {
                     slot = 0;
                     rph ^= 1u;
                 }
@@ -457,7 +361,7 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
                     bph ^= 1u;
                 }
             }
-        } else if (half == 0 && lane == 0) {
+        } else if (warp == F_MMA_WARP && half == 0 && lane == 0) {
             // ------------------------------------------------------------ MMA issuer (even CTA)
             constexpr uint32_t idesc = idesc_f16(2 * F_VEC, F_N);
             bool ok = true;
@@ -547,25 +451,43 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
                 while (next < total) {
                     if (lane == 0) {
                         const int f = next, x = (f % n_ks) * F_KS;
-                        const int rslot = f % R, bslot = f % NB;
-                        const uint32_t rdst = ring_u32 + rslot * S.raw_bytes;
+                        const int bslot = f % NB;
                         const uint32_t bdst = b_u32 + bslot * F_SET;
                         const int row0 = (pr + (f / n_ks) * split) * F_N + half * F_ROWS;
                         // a tile copy starts 16-byte aligned (x counts int8 codes in the code
                         // map) into a 1024-byte aligned destination (128-byte swizzle), or is not
-                        // issued and the launch ends through the bounded waits; the raw slot
-                        // takes W rows (and the codes of the greedy residuals)
-                        ok = MPQ_CHECK((x & 15) == 0 && (rdst & 15u) == 0u && (bdst & 1023u) == 0u &&
-                                       x < d);
-                        if (ok && f >= R)
-                            ok = mbar_wait(&ctl.raw_empty[rslot], (uint32_t)((f - R) / R) & 1u, wc.budget);
-                        if (ok) {
-                            mbar_arrive_expect_tx(&ctl.raw_full[rslot], S.raw_tx);
-                            tma_load_2d(rdst, &tmW, x, k0, &ctl.raw_full[rslot]);
-                            if constexpr (!CLIP)
+                        // issued and the launch ends through the bounded waits
+                        if constexpr (CLIP) {
+                            // A tiles of step f (residual planes) into stage f % NA once the
+                            // MMAs of step f - NA have completed
+                            const int as = f % NA;
+                            const uint32_t adst = a_u32 + as * F_SET;
+                            ok = MPQ_CHECK((x & 15) == 0 && (adst & 1023u) == 0u &&
+                                           (bdst & 1023u) == 0u && x < d);
+                            if (ok && f >= NA)
+                                ok = mbar_wait_cluster(&ctl.empty[as], (uint32_t)((f - NA) / NA) & 1u,
+                                                       wc.budget);
+                            if (ok) {
+                                mbar_arrive_expect_tx(&ctl.afull[as], 2 * F_TILE);
+                                tma_load_3d(adst, &tmW, x, k0, 0, &ctl.afull[as]);
+                                raw_issued = f + 1;
+                            }
+                        } else {
+                            // the raw slot takes W rows and the codes of the greedy residuals
+                            const int rslot = f % R;
+                            const uint32_t rdst = ring_u32 + rslot * S::raw_bytes;
+                            ok = MPQ_CHECK((x & 15) == 0 && (rdst & 15u) == 0u &&
+                                           (bdst & 1023u) == 0u && x < d);
+                            if (ok && f >= R)
+                                ok = mbar_wait(&ctl.raw_empty[rslot], (uint32_t)((f - R) / R) & 1u,
+                                               wc.budget);
+                            if (ok) {
+                                mbar_arrive_expect_tx(&ctl.raw_full[rslot], S::raw_tx);
+                                tma_load_2d(rdst, &tmW, x, k0, &ctl.raw_full[rslot]);
                                 tma_load_3d(rdst + FGeo<KP1>::RAW_Q, &tmQ, x, k0, 0,
                                             &ctl.raw_full[rslot]);
-                            raw_issued = f + 1;
+                                raw_issued = f + 1;
+                            }
                         }
                         if (ok && f >= NB)
                             ok = mbar_wait_cluster(&ctl.bempty[bslot], (uint32_t)((f - NB) / NB) & 1u,
@@ -623,8 +545,13 @@ output_error_f16_kernel(const float *__restrict__ scales, const float *__restric
         }
         // no copy lands after the CTA is gone: the last copy of every slot
         if (copier && lane == 0) {
-            for (int f = raw_issued - R > 0 ? raw_issued - R : 0; f < raw_issued; ++f)
-                drain_wait(&ctl.raw_full[f % R], (uint32_t)(f / R) & 1u, wc, KBIT);
+            if constexpr (CLIP) {
+                for (int f = raw_issued - NA > 0 ? raw_issued - NA : 0; f < raw_issued; ++f)
+                    drain_wait(&ctl.afull[f % NA], (uint32_t)(f / NA) & 1u, wc, KBIT);
+            } else {
+                for (int f = raw_issued - R > 0 ? raw_issued - R : 0; f < raw_issued; ++f)
+                    drain_wait(&ctl.raw_full[f % R], (uint32_t)(f / R) & 1u, wc, KBIT);
+            }
             for (int f = b_issued - NB > 0 ? b_issued - NB : 0; f < b_issued; ++f)
                 drain_wait(&ctl.bfull[f % NB], (uint32_t)(f / NB) & 1u, wc, KBIT);
         }
@@ -674,14 +601,74 @@ f16_split_kernel(const float4 *__restrict__ X, long long n8, const unsigned *__r
     }
 }
 
-template <int KP1, bool CLIP>
-mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes,
-                      const float *scales, const float *chmax, int C, int d, int n_cand, int qmax,
-                      float *err, const unsigned *xrange, const unsigned *vrange, uint16_t *xs,
-                      cudaStream_t stream)
+// Clipping search (Eq. 12): the residual r = w - s q of channel c0 + v / n_cand under candidate
+// v mod n_cand (s = K / Qmax, the codes q of Eq. 8 with the sign of w, q = 0 where s is 0 or NaN),
+// scaled by 2^e and split into fp16 hi/lo planes ([2][M][d] as hi and lo), 8 elements a thread per
+// step.  e comes from a bound on the vector's elements, max(s/2, max|w| - Qmax s) (s/2 for a
+// nearest code, max|w| - Qmax s where the code is clamped; a residual a rounding above it still
+// fits fp16, whose range reaches 2^16), kept in vrange[v] (float bits) for the contraction.
+__global__ void __launch_bounds__(256)
+clip_planes_kernel(const float *__restrict__ W, int d, const float *__restrict__ clip,
+                   const float *__restrict__ chmax, int c0, int n_cand, int qmax, long long M,
+                   uint4 *__restrict__ hi, uint4 *__restrict__ lo, unsigned *__restrict__ vrange)
 {
-    const FShape<KP1, CLIP> S(n_cand);
-    const int n_pairs = (C + 2 * S.ch - 1) / (2 * S.ch);
+    const int d8 = d / 8;
+    const long long n = M * d8;
+    const float qmaxf = (float)qmax, qlim = qmaxf + 1.0f;
+    const float tband = 0.5f - MPQ_FAST_REL * (qlim + 1.0f);
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += stride) {
+        const long long v = t / d8;
+        const int j = (int)(t - v * d8);
+        const long long k = c0 + v / n_cand;
+        // clip row of channel k, candidate v mod n_cand: index c0 n_cand + v
+        const float sv = __fdiv_rn(__ldg(clip + (long long)c0 * n_cand + v), qmaxf);
+        const float inv = sv > 0.0f ? __frcp_rn(sv) : 0.0f;
+        const float bound = fmaxf(__fmul_rn(0.5f, sv), __fmaf_rn(-qmaxf, sv, __ldg(chmax + k)));
+        const float vf = pow2f(f16_scale_exp(bound));
+        const float4 *w4 = reinterpret_cast<const float4 *>(W + k * d) + 2 * j;
+        const float4 a = __ldg(w4), b = __ldg(w4 + 1);
+        const float w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        float q[8];
+        bool unsure = false;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) q[e] = code_signed_fast(w[e], inv, qmaxf, qlim, tband, unsure);
+        if (unsure) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) q[e] = code_signed_exact(w[e], sv, qmaxf);
+        }
+        uint32_t h[4], l[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            split_f16x2(__fmul_rn(__fmaf_rn(-sv, q[2 * e], w[2 * e]), vf),
+                        __fmul_rn(__fmaf_rn(-sv, q[2 * e + 1], w[2 * e + 1]), vf), h[e], l[e]);
+        hi[t] = make_uint4(h[0], h[1], h[2], h[3]);
+        lo[t] = make_uint4(l[0], l[1], l[2], l[3]);
+        if (j == 0) vrange[v] = __float_as_uint(bound);
+    }
+}
+
+// X split into the fp16 planes xs ([2][N][d]) on `stream`.
+cudaError_t launch_x_split(const float *X, int N, int d, const unsigned *xrange, uint16_t *xs,
+                           cudaStream_t stream)
+{
+    const long long n8 = (long long)N * d / 8;
+    const int sb = (int)std::min<long long>((n8 + 255) / 256, 4LL * sm_count());
+    f16_split_kernel<<<(unsigned)std::max(sb, 1), 256, 0, stream>>>(
+        reinterpret_cast<const float4 *>(X), n8, xrange, reinterpret_cast<uint4 *>(xs),
+        reinterpret_cast<uint4 *>(xs + (size_t)N * d));
+    return cudaGetLastError();
+}
+
+// The contraction, X already split into xs.  Greedy residuals: A = W, with codes and scales.
+// Clipping search: A = the residual planes of C vectors.
+template <int KP1, bool CLIP>
+mpq_status launch_f16(const void *A, int N, const int8_t *codes, const float *scales, int C,
+                      int d, float *err, const unsigned *xrange, const unsigned *vrange,
+                      const uint16_t *xs, cudaStream_t stream)
+{
+    using S = FShape<KP1, CLIP>;
+    const int n_pairs = (C + 2 * S::ch - 1) / (2 * S::ch);
     const int n_rt = (N + F_N - 1) / F_N;
 
     CUtensorMap tmX, tmW, tmQ;
@@ -691,33 +678,39 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
     const cuuint64_t dx[3] = {(cuuint64_t)d, (cuuint64_t)N, 2};
     const cuuint64_t sx[2] = {(cuuint64_t)d * 2, (cuuint64_t)N * d * 2};
     const cuuint32_t bx[3] = {F_KS, F_ROWS, 2};
-    const cuuint64_t dw[2] = {(cuuint64_t)d, (cuuint64_t)C}, sw[1] = {(cuuint64_t)d * 4};
-    const cuuint32_t bw[2] = {F_KS, (cuuint32_t)S.ch};
     bool maps = encode_tile_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, xs, dx, sx, bx,
-                                CU_TENSOR_MAP_SWIZZLE_128B) &&
-                encode_tile_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw);
-    if constexpr (!CLIP) {
+                                CU_TENSOR_MAP_SWIZZLE_128B);
+    if constexpr (CLIP) {
+        const cuuint64_t da[3] = {(cuuint64_t)d, (cuuint64_t)C, 2};
+        const cuuint64_t sa[2] = {(cuuint64_t)d * 2, (cuuint64_t)C * d * 2};
+        const cuuint32_t ba[3] = {F_KS, F_VEC, 2};
+        maps = maps && encode_tile_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, A, da, sa, ba,
+                                       CU_TENSOR_MAP_SWIZZLE_128B);
+    } else {
         using G = FGeo<KP1>;
+        const cuuint64_t dw[2] = {(cuuint64_t)d, (cuuint64_t)C}, sw[1] = {(cuuint64_t)d * 4};
+        const cuuint32_t bw[2] = {F_KS, (cuuint32_t)G::CH};
         const cuuint64_t dq[3] = {(cuuint64_t)d, (cuuint64_t)C, (cuuint64_t)G::K};
         const cuuint64_t sq[2] = {(cuuint64_t)d, (cuuint64_t)C * d};
         const cuuint32_t bq[3] = {F_KS, (cuuint32_t)G::CH, (cuuint32_t)G::K};
-        maps = maps && encode_tile_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq);
+        maps = maps && encode_tile_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, A, dw, sw, bw) &&
+               encode_tile_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq);
     }
     if (!maps) {
         set_error("output error: tensor map encoding failed");
         return MPQ_ERR_CUDA;
     }
-    if ((long long)S.smem > max_smem_optin()) {
-        set_error("fp16 output error needs %d bytes of shared memory", (int)S.smem);
+    if ((long long)S::smem > max_smem_optin()) {
+        set_error("fp16 output error needs %d bytes of shared memory", S::smem);
         return MPQ_ERR_UNSUPPORTED;
     }
     cudaError_t e = cudaFuncSetAttribute(output_error_f16_kernel<KP1, CLIP>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)S.smem);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, S::smem);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
 
     cudaLaunchConfig_t cfg = {};
     cfg.blockDim = dim3(F_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = (size_t)S.smem;
+    cfg.dynamicSmemBytes = (size_t)S::smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -727,9 +720,10 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
     cfg.numAttrs = 1;
 
     // Row tiles split over `split` pairs per cluster (clusters of 2 * split CTAs): the split with
-    // the least (waves of resident clusters) x (row tiles per CTA), ties to the smaller cluster;
-    // resident clusters per cluster size queried once per process (one device per process; the
-    // 512 threads x 128 registers of a CTA fill an SM whatever its shared memory).
+    // the least (waves of resident clusters) x (row tiles per CTA), ties to the smaller cluster --
+    // or, where A is copied from global memory, to the larger one, whose pairs read the same A
+    // tiles at about the same time (from L2); resident clusters per cluster size queried once per
+    // process (one device per process).
     static std::atomic<int> resident[3] = {{0}, {0}, {0}};
     int split = 1;
     long long best = -1;
@@ -747,7 +741,7 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
         if (active < 1) continue;
         const long long waves = (n_pairs + active - 1) / active;
         const long long cost = waves * ((n_rt + sp - 1) / sp);
-        if (best < 0 || cost < best) {
+        if (best < 0 || cost < best || (CLIP && cost == best)) {
             best = cost;
             split = sp;
         }
@@ -757,16 +751,8 @@ mpq_status launch_f16(const float *X, int N, const float *W, const int8_t *codes
     WaitCtl wc;
     mpq_status wst = wait_ctl(&wc);
     if (wst != MPQ_OK) return wst;
-
-    const long long n8 = (long long)N * d / 8;
-    const int sb = (int)std::min<long long>((n8 + 255) / 256, 4LL * sm_count());
-    f16_split_kernel<<<(unsigned)std::max(sb, 1), 256, 0, stream>>>(
-        reinterpret_cast<const float4 *>(X), n8, xrange, reinterpret_cast<uint4 *>(xs),
-        reinterpret_cast<uint4 *>(xs + (size_t)N * d));
-    e = cudaGetLastError();
-    if (e == cudaSuccess)
-        e = cudaLaunchKernelEx(&cfg, output_error_f16_kernel<KP1, CLIP>, scales, chmax, C, N, d,
-                               n_cand, qmax, xrange, vrange, err, split, wc, tmX, tmW, tmQ);
+    e = cudaLaunchKernelEx(&cfg, output_error_f16_kernel<KP1, CLIP>, scales, C, N, d, xrange,
+                           vrange, err, split, wc, tmX, tmW, tmQ);
     return cuda_status(e, "fp16 output-error kernel launch");
 }
 
@@ -777,17 +763,20 @@ mpq_status launch_output_error_f16(const float *X, int N, const float *W, const 
                                    const unsigned *xrange, const unsigned *vrange, uint16_t *xs,
                                    cudaStream_t stream)
 {
+    if (k_max < 1 || k_max > 16) {
+        set_error("k_max = %d unsupported", k_max);
+        return MPQ_ERR_UNSUPPORTED;
+    }
+    const cudaError_t e = launch_x_split(X, N, d, xrange, xs, stream);
+    if (e != cudaSuccess) return cuda_status(e, "X split kernel launch");
     switch (k_max + 1) {
-#define MPQ_CASE(n)                                                                             \
-    case n:                                                                                     \
-        return launch_f16<n, false>(X, N, W, codes, scales, nullptr, C, d, 0, 0, err, xrange,  \
-                                    vrange, xs, stream);
+#define MPQ_CASE(n) \
+    case n: return launch_f16<n, false>(W, N, codes, scales, C, d, err, xrange, vrange, xs, stream);
         MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7) MPQ_CASE(8)
         MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14) MPQ_CASE(15)
         MPQ_CASE(16) MPQ_CASE(17)
 #undef MPQ_CASE
     }
-    set_error("k_max = %d unsupported", k_max);
     return MPQ_ERR_UNSUPPORTED;
 }
 
@@ -795,10 +784,37 @@ mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *c
                            const float *chmax, int C, int d, int qmax, int n_cand, float *err,
                            unsigned *xrange, uint16_t *xs, cudaStream_t stream)
 {
-    const mpq_status st = launch_x_range(X, N, d, xrange, stream);
+    mpq_status st = launch_x_range(X, N, d, xrange, stream);
     if (st != MPQ_OK) return st;
-    return launch_f16<1, true>(X, N, W, nullptr, clip, chmax, C, d, n_cand, qmax, err, xrange,
-                               nullptr, xs, stream);
+    cudaError_t e = launch_x_split(X, N, d, xrange, xs, stream);
+    if (e != cudaSuccess) return cuda_status(e, "X split kernel launch");
+    // residual planes of whole channels, at most 2 GiB at a time, and their bounds
+    const long long vec_bytes = 4LL * d;
+    const int cc = (int)std::min<long long>(C, std::max(1LL, (1LL << 31) / (vec_bytes * n_cand)));
+    const long long m_max = (long long)cc * n_cand;
+    const size_t planes_bytes = (size_t)(m_max * vec_bytes);
+    void *scratch = nullptr;
+    st = pool_scratch(&scratch, planes_bytes + (size_t)(m_max * 4 + 255) / 256 * 256, stream);
+    if (st != MPQ_OK) return st;
+    uint16_t *planes = static_cast<uint16_t *>(scratch);
+    unsigned *vrange = reinterpret_cast<unsigned *>(static_cast<char *>(scratch) + planes_bytes);
+    for (int c0 = 0; c0 < C && st == MPQ_OK; c0 += cc) {
+        const int cn = std::min(cc, C - c0);
+        const long long M = (long long)cn * n_cand;
+        const long long n = M * (d / 8);
+        const int blocks = (int)std::min<long long>((n + 255) / 256, 8LL * sm_count());
+        uint4 *hi = reinterpret_cast<uint4 *>(planes);
+        clip_planes_kernel<<<(unsigned)blocks, 256, 0, stream>>>(W, d, clip, chmax, c0, n_cand,
+                                                                  qmax, M, hi, hi + n, vrange);
+        e = cudaGetLastError();
+        st = cuda_status(e, "clip residual planes kernel launch");
+        if (st == MPQ_OK)
+            st = launch_f16<1, true>(planes, N, nullptr, nullptr, (int)M, d,
+                                     err + (size_t)c0 * n_cand, xrange, vrange, xs, stream);
+    }
+    e = cudaFreeAsync(scratch, stream);
+    if (st == MPQ_OK) st = cuda_status(e, "scratch release (cudaFreeAsync)");
+    return st;
 }
 
 }  // namespace mpq
