@@ -1,10 +1,10 @@
 // Output error (Sec. 3.3, Eq. 11) as a CTA-pair tcgen05 contraction:
 //   err[k][n] = (1/N) sum_t (x_t . r_{k,n+1})^2,  n = 0..k_max.
 //
-// This file holds the contraction for the clipping search (tf32 operands) and for the output error
-// entry point with a fixed range table (fp16 operands, X split by the producers: it needs no
-// scratch beyond that table); the output error with pooled scratch runs output_error_f16.cu, the
-// same contraction with X split ahead and the layout its measurements favoured.
+// This file holds the contraction for the output error entry point with a fixed range table (X
+// split by the producers: it needs no scratch beyond that table); the output error with pooled
+// scratch and the clipping search run output_error_f16.cu, the same contraction with X split
+// ahead and the layout its measurements favoured.
 //
 // Y = R X^T with R the C*(k_max+1) residual vectors and X the N calibration rows (length d);
 // err is the row-wise mean of Y^2.  Two CTAs on neighbouring SMs (cluster ranks 2p, 2p+1) form one
@@ -19,18 +19,16 @@
 // [2^14, 2^15) and split into fp16 hi = fl16(x) and lo = fl16(x - hi), and Y = hi*hi + hi*lo + lo*hi
 // runs on kind::f16 (fp32 accumulate) -- 22 significant bits per operand like a tf32 hi/lo split,
 // at twice the tf32 rate; the reduction multiplies each mean by 2^-2(e_X + e_v) exactly, in double.
-// Clipping-search residuals keep the tf32 split (hi = x with 13 mantissa bits cleared, lo = x - hi)
-// on kind::tf32.  The accumulator restarts every 256 (fp16) or 128 (tf32) elements of d and the
-// epilogue folds each segment into fp32 running sums in tensor memory (columns [0, 256) segment,
-// [256, 512) running sums), since the tensor core's accumulation truncates.
+// The accumulator restarts every 256 elements of d and the epilogue folds each segment into fp32
+// running sums in tensor memory (columns [0, 256) segment, [256, 512) running sums), since the
+// tensor core's accumulation truncates.
 //
 // Input: one thread per CTA streams each K chunk's X rows, W rows and codes into a ring of raw
 // shared-memory slots with TMA tile copies (rows past N and channels past C read as zeros).  Eight
-// producer warps (sixteen in the clipping search) split X into the B tiles and regenerate the
-// residuals r_{n+1} = r_n - s_n q_n
+// producer warps split X into the B tiles and regenerate the residuals r_{n+1} = r_n - s_n q_n
 // (Eq. 7) from W, codes and scales into the A tiles (128-byte swizzled, K-major); residuals never
-// exist in global memory.  Two 64 KB tile sets hold the stages: with fp16 operands a 32-element
-// chunk fills a 64-byte half of every row (4 stages), with tf32 operands a whole row (2 stages).
+// exist in global memory.  Two 64 KB tile sets hold the stages: a 32-element chunk fills a 64-byte
+// half of every row (4 stages).
 // Both CTAs' producers report a full stage to the even CTA, whose MMA
 // thread issues the pair MMAs and signals both CTAs (multicast commits) when a stage or a segment
 // is consumed.  Eight epilogue warps per CTA (one per TMEM lane quarter and column half) drain the
@@ -38,8 +36,7 @@
 //
 // Row tiles (256 rows) are split over the pairs of a cluster of up to 8 CTAs; ranks 0 and 1 add
 // their peers' partial sums from distributed shared memory in rank order.  Every wait is bounded;
-// on a timeout the kernel records MPQ_TIMEOUT_OUTPUT_ERROR (or _CLIP), unwinds and the outputs
-// read NaN.
+// on a timeout the kernel records MPQ_TIMEOUT_OUTPUT_ERROR, unwinds and the outputs read NaN.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
@@ -51,7 +48,6 @@
 
 #include "mpq_internal.cuh"
 #include "pair_common.cuh"
-#include "rounding.cuh"
 #include "sm100.cuh"
 #include "tf32_operands.cuh"
 #include "waits.cuh"
@@ -78,28 +74,20 @@ constexpr int P_TILE_SETS = 2;
 constexpr int P_MAX_STAGES = 4;
 constexpr int P_EPI_WARPS = 8;                  // two per TMEM lane quarter, one per column half
 
-// Operand format per mode.  fp32 operands (the clipping search): a K chunk of 32 elements fills
-// a tile set's 128-byte rows as tf32 hi/lo parts, 2 stages, accumulator restarted every 4 chunks.
-// fp16 operands (the greedy residuals): a chunk fills half of each row (64 bytes), so the two
+// fp16 operands: a K chunk of 32 elements fills half of each 128-byte row (64 bytes), so the two
 // tile sets hold 4 stages, and the accumulator restarts every 8 chunks (256 elements).
-template <bool F16>
-struct PFmt {
-    static constexpr int STAGES = F16 ? 4 : 2;
-    static constexpr int SEG = F16 ? 8 : 4;     // chunks per accumulation segment
-};
+constexpr int P_STAGES = 4;
+constexpr int P_SEG = 8;                        // chunks per accumulation segment
 
 // Warp roles: producers first, then the epilogue warps (warp % 4 selects TMEM lanes, so the
-// producer count is a multiple of 4), the MMA warp and the TMA warp.  The clipping search's
-// producers regenerate a residual per candidate and bound that mode, so it gets 16 warps of them;
-// the greedy mode keeps 8 (more registers per thread).
-template <bool CLIP>
+// producer count is a multiple of 4), the MMA warp and the TMA warp.
 struct PRoles {
-    static constexpr int PROD_WARPS = CLIP ? 16 : 8;
+    static constexpr int PROD_WARPS = 8;
     static constexpr int PROD_THREADS = PROD_WARPS * 32;
     static constexpr int EPI_WARP0 = PROD_WARPS;
     static constexpr int MMA_WARP = EPI_WARP0 + P_EPI_WARPS;
     static constexpr int TMA_WARP = MMA_WARP + 1;
-    static constexpr int THREADS = (TMA_WARP + 1) * 32;   // 576 or 832
+    static constexpr int THREADS = (TMA_WARP + 1) * 32;   // 576
     static_assert(PROD_WARPS % 4 == 0, "epilogue warps start at a TMEM lane quarter boundary");
 };
 constexpr uint32_t P_TMEM_COLS = 512;
@@ -118,9 +106,7 @@ struct PairCtrl {
     uint32_t tmem_base;
     int abort;
     double part[2][P_VEC];        // per column half: sum over the rows' y^2
-    float clip_s[P_VEC];          // clipping search: scale K / Qmax and fl(1 / scale) per row
-    float clip_inv[P_VEC];
-    float vscale[P_VEC];          // fp16 operands: 2^e per residual vector, 2^e for X
+    float vscale[P_VEC];          // 2^e per residual vector, 2^e for X
     int vexp[P_VEC];
     float xscale;
     int xexp;
@@ -129,25 +115,23 @@ constexpr int P_CTRL_BYTES = (sizeof(PairCtrl) + 1023) / 1024 * 1024;
 constexpr int P_BASE_SMEM = 1024 /* alignment slack */ + P_CTRL_BYTES + P_TILE_SETS * P_STAGE_BYTES;
 
 // Per-KP1 geometry and the raw slot layout, in the order the tile copies write it:
-// X chunk [128 rows][32] fp32, W chunk [CH][32] fp32, codes [K][CH][32] int8.  KP1 is the number of
-// residual vectors per channel: k_max + 1 greedy residuals, or (CLIP) one per candidate clipping
-// factor, which need no codes.
-template <int KP1, bool CLIP = false>
+// X chunk [128 rows][32] fp32, W chunk [CH][32] fp32, codes [K][CH][32] int8.  KP1 = k_max + 1
+// residual vectors per channel.
+template <int KP1>
 struct PGeo {
-    static constexpr int K = CLIP ? 0 : KP1 - 1;
-    static constexpr int KQ = K > 0 ? K : 1;
-    static constexpr int VF = CLIP ? 1 : KP1;   // fp16 operand scales per item
+    static constexpr int K = KP1 - 1;
     static constexpr int CH = P_VEC / KP1;
-    static constexpr int PT = PRoles<CLIP>::PROD_THREADS;
+    static constexpr int PT = PRoles::PROD_THREADS;
     static constexpr int ITEMS2 = (CH * (P_KC / 2) + PT - 1) / PT;
     static constexpr int X_ITEMS = (P_ROWS * P_KC4 + PT - 1) / PT;
     static constexpr int RAW_W = P_ROWS * P_KC * 4;
     static constexpr int RAW_Q = (RAW_W + CH * P_KC * 4 + 127) / 128 * 128;
     static constexpr uint32_t RAW_TX = P_ROWS * P_KC * 4 + CH * P_KC * 4 + K * CH * P_KC;
-    static constexpr int RAW_BYTES = (RAW_Q + KQ * CH * P_KC + 1023) / 1024 * 1024;
+    static constexpr int RAW_BYTES = (RAW_Q + K * CH * P_KC + 1023) / 1024 * 1024;
     static constexpr int RAW_FIT = (P_SMEM_LIMIT - P_BASE_SMEM) / RAW_BYTES;
     static constexpr int RAW_STAGES = RAW_FIT < P_MAX_RAW ? RAW_FIT : P_MAX_RAW;
     static constexpr int SMEM = P_BASE_SMEM + RAW_STAGES * RAW_BYTES;
+    static_assert(K >= 1, "at least one point");
     static_assert(RAW_STAGES >= 2, "raw ring needs two slots");
 };
 
@@ -164,19 +148,16 @@ __device__ __forceinline__ int pair_x_item(int q)
     return row * P_KC4 + (q & 7);
 }
 
-// Raw slot -> operand stage (tile set `sb`, row half `hh` with fp16 operands): X rows -> B tiles;
-// for every (channel, element pair) item the residuals -> A tiles: r_0 = w, r_{n+1} = r_n - s_n q_n
-// (Eq. 7), or (CLIP) r_c = w - s_c [w / s_c]_Q for every candidate clipping factor (Eq. 12), with
-// the scales and reciprocals of `ctl`.  fp16 operands are scaled by 2^e first (xs for X, vf per
-// residual vector), which the reduction undoes exactly.
-template <int KP1, bool CLIP>
+// Raw slot -> operand stage (tile set `sb`, row half `hh`): X rows -> B tiles; for every (channel,
+// element pair) item the residuals -> A tiles: r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7).  Operands
+// are scaled by 2^e first (xs for X, vf per residual vector), which the reduction undoes exactly.
+template <int KP1>
 __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh, int pt, int nch,
-                                             const int (&chs)[PGeo<KP1, CLIP>::ITEMS2],
-                                             const float (&sc)[PGeo<KP1, CLIP>::ITEMS2][PGeo<KP1, CLIP>::KQ],
-                                             const float (&vf)[PGeo<KP1, CLIP>::ITEMS2][PGeo<KP1, CLIP>::VF],
-                                             float xs, const PairCtrl &ctl, float qmaxf)
+                                             const int (&chs)[PGeo<KP1>::ITEMS2],
+                                             const float (&sc)[PGeo<KP1>::ITEMS2][KP1 - 1],
+                                             const float (&vf)[PGeo<KP1>::ITEMS2][KP1], float xs)
 {
-    using G = PGeo<KP1, CLIP>;
+    using G = PGeo<KP1>;
     constexpr int K = G::K;
     // every shared-memory read of a group before its stores (the accessors are ordered), so the
     // reads' latencies overlap instead of adding up
@@ -185,36 +166,28 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh,
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
         const int q = pt + i * G::PT;
-        const int qi = CLIP ? q : pair_x_item(q);
+        const int qi = pair_x_item(q);
         if (G::X_ITEMS * G::PT == XN || q < XN) xr[i] = ld_shared_v4(slot + (uint32_t)qi * 16u);
     }
 #pragma unroll
     for (int i = 0; i < G::X_ITEMS; ++i) {
         const int q = pt + i * G::PT;
         if (G::X_ITEMS * G::PT != XN && q >= XN) break;
-        if constexpr (CLIP) {
-            float4 hi, lo;
-            split4(xr[i], hi, lo);
-            const uint32_t off = sw128_offset(q / P_KC4, q % P_KC4);
-            st_shared_v4(sb + P_OFF_B_HI + off, hi);
-            st_shared_v4(sb + P_OFF_B_LO + off, lo);
-        } else {
-            uint32_t h0, l0, h1, l1;
-            split_f16x2(__fmul_rn(xr[i].x, xs), __fmul_rn(xr[i].y, xs), h0, l0);
-            split_f16x2(__fmul_rn(xr[i].z, xs), __fmul_rn(xr[i].w, xs), h1, l1);
-            const int qi = pair_x_item(q), q4 = qi % P_KC4;   // 4 elements = 8 bytes of a half row
-            const uint32_t off = sw128_offset(qi / P_KC4, hh * 4 + (q4 >> 1)) + (uint32_t)(q4 & 1) * 8u;
-            st_shared_v2u(sb + P_OFF_B_HI + off, h0, h1);
-            st_shared_v2u(sb + P_OFF_B_LO + off, l0, l1);
-        }
+        uint32_t h0, l0, h1, l1;
+        split_f16x2(__fmul_rn(xr[i].x, xs), __fmul_rn(xr[i].y, xs), h0, l0);
+        split_f16x2(__fmul_rn(xr[i].z, xs), __fmul_rn(xr[i].w, xs), h1, l1);
+        const int qi = pair_x_item(q), q4 = qi % P_KC4;   // 4 elements = 8 bytes of a half row
+        const uint32_t off = sw128_offset(qi / P_KC4, hh * 4 + (q4 >> 1)) + (uint32_t)(q4 & 1) * 8u;
+        st_shared_v2u(sb + P_OFF_B_HI + off, h0, h1);
+        st_shared_v2u(sb + P_OFF_B_LO + off, l0, l1);
     }
 #pragma unroll
     for (int i = 0; i < G::ITEMS2; ++i) {
         const int p = pt + i * G::PT;
-        if (!CLIP && p < nch * (P_KC / 2)) {
+        if (p < nch * (P_KC / 2)) {
             const int ch = chs[i], e2 = p % (P_KC / 2);
             float2 r = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
-            uint32_t qb[G::KQ];
+            uint32_t qb[K];
 #pragma unroll
             for (int n = 0; n < K; ++n)
                 qb[n] = ld_shared_u16(slot + G::RAW_Q + (uint32_t)((n * G::CH + ch) * P_KC + e2 * 2)) ^
@@ -236,68 +209,23 @@ __device__ __forceinline__ void pair_consume(uint32_t slot, uint32_t sb, int hh,
             }
         }
     }
-    if constexpr (CLIP) {
-        // (candidate, channel, element pair) units over all producer threads, element pairs
-        // lane-contiguous: each warp store fills whole 128-byte rows.
-        constexpr int STEP = G::PT / (P_KC / 2);   // rows between a thread's units
-        constexpr int UNITS = (P_VEC + STEP - 1) / STEP;    // most units of one thread
-        const int rows = nch * KP1;                     // row = c * nch + ch
-        const int e2 = pt % (P_KC / 2);                  // the same for all of this thread's units
-        const int row0 = pt / (P_KC / 2);
-        int c = nch > 0 ? row0 / nch : 0, ch = nch > 0 ? row0 - c * nch : 0;
-        // all reads first (weights, scales, reciprocals of every unit), then the residuals
-        float2 w[UNITS];
-        float sv[UNITS], iv[UNITS];
-        int arow[UNITS];
-#pragma unroll
-        for (int u = 0; u < UNITS; ++u) {
-            arow[u] = ch * KP1 + c;
-            if (row0 + u * STEP < rows) {
-                w[u] = ld_shared_v2(slot + G::RAW_W + (uint32_t)(ch * P_KC + e2 * 2) * 4u);
-                sv[u] = ctl.clip_s[arow[u]];
-                iv[u] = ctl.clip_inv[arow[u]];
-            }
-            ch += STEP;                                  // next row: advance (c, ch) without dividing
-            while (ch >= nch && nch > 0) {
-                ch -= nch;
-                ++c;
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < UNITS; ++u) {
-            if (row0 + u * STEP >= rows) break;
-            const float s = sv[u], inv = iv[u];
-            // exact code of Eq. 8 (0 when the scale is 0 or NaN: the residual is then w or NaN)
-            const float qx = s > 0.0f ? copysignf((float)code_fast(fabsf(w[u].x), s, inv, qmaxf), w[u].x) : 0.0f;
-            const float qy = s > 0.0f ? copysignf((float)code_fast(fabsf(w[u].y), s, inv, qmaxf), w[u].y) : 0.0f;
-            float2 r, hi, lo;
-            r.x = __fmaf_rn(-s, qx, w[u].x);
-            r.y = __fmaf_rn(-s, qy, w[u].y);
-            split2(r, hi, lo);
-            const uint32_t off = sw128_offset(arow[u], e2 >> 1) + (uint32_t)(e2 & 1) * 8u;
-            st_shared_v2(sb + P_OFF_A_HI + off, hi);
-            st_shared_v2(sb + P_OFF_A_LO + off, lo);
-        }
-    }
 }
 
-// scales: [C][k_max] point scales, or (CLIP) [C][KP1] candidate clipping factors K; qmax: the
-// code range for CLIP; range (fp16 operands): max|X| and max|r| per residual vector, as float bits
-// (pair_range_kernel).
-template <int KP1, bool CLIP>
-__global__ void __launch_bounds__(PRoles<CLIP>::THREADS, 1)
-output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, int qmax,
+// scales: [C][k_max] point scales; xrange, vrange: max|X| and max|r| per residual vector, as
+// float bits (pair_range_kernel).
+template <int KP1>
+__global__ void __launch_bounds__(PRoles::THREADS, 1)
+output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d,
                          const unsigned *__restrict__ xrange, const unsigned *__restrict__ vrange,
                          float *__restrict__ err, int split,
                          const WaitCtl wc, const __grid_constant__ CUtensorMap tmX,
                          const __grid_constant__ CUtensorMap tmW,
                          const __grid_constant__ CUtensorMap tmQ)
 {
-    using G = PGeo<KP1, CLIP>;
-    using PR = PRoles<CLIP>;
-    constexpr bool F16 = !CLIP;
-    constexpr unsigned KBIT = CLIP ? MPQ_TIMEOUT_CLIP : MPQ_TIMEOUT_OUTPUT_ERROR;
-    constexpr int NST = PFmt<F16>::STAGES, SEG = PFmt<F16>::SEG;
+    using G = PGeo<KP1>;
+    using PR = PRoles;
+    constexpr unsigned KBIT = MPQ_TIMEOUT_OUTPUT_ERROR;
+    constexpr int NST = P_STAGES, SEG = P_SEG;
     constexpr int R = G::RAW_STAGES;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
@@ -342,25 +270,16 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
         ctl.abort = 0;
         fence_barrier_init();
     }
-    const float qmaxf = (float)qmax;
-    if (CLIP) {
-        for (int i = threadIdx.x; i < nvec; i += PR::THREADS) {
-            const float s = __fdiv_rn(__ldg(scales + (size_t)k0 * KP1 + i), qmaxf);
-            ctl.clip_s[i] = s;
-            ctl.clip_inv[i] = s > 0.0f ? __frcp_rn(s) : 0.0f;
-        }
-    } else {
-        for (int i = threadIdx.x; i < nvec; i += PR::THREADS) {
-            if (!MPQ_IN((size_t)k0 * KP1 + i, (size_t)C * KP1)) continue;
-            const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * KP1 + i)));
-            ctl.vexp[i] = e;
-            ctl.vscale[i] = pow2f(e);
-        }
-        if (threadIdx.x == 0) {
-            const int e = f16_scale_exp(__uint_as_float(__ldg(xrange)));
-            ctl.xexp = e;
-            ctl.xscale = pow2f(e);
-        }
+    for (int i = threadIdx.x; i < nvec; i += PR::THREADS) {
+        if (!MPQ_IN((size_t)k0 * KP1 + i, (size_t)C * KP1)) continue;
+        const int e = f16_scale_exp(__uint_as_float(__ldg(vrange + (size_t)k0 * KP1 + i)));
+        ctl.vexp[i] = e;
+        ctl.vscale[i] = pow2f(e);
+    }
+    if (threadIdx.x == 0) {
+        const int e = f16_scale_exp(__uint_as_float(__ldg(xrange)));
+        ctl.xexp = e;
+        ctl.xscale = pow2f(e);
     }
     if (warp == PR::MMA_WARP) {
         tmem_alloc_pair(&ctl.tmem_base, P_TMEM_COLS);
@@ -374,23 +293,23 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
     if (warp < PR::PROD_WARPS) {
         // ---------------------------------------------------------------- producers
         const int pt = threadIdx.x;
-        float sc[G::ITEMS2][G::KQ];     // scales of this thread's items, the same for every chunk
-        float vf[G::ITEMS2][G::VF];     // fp16 operands: 2^e of the items' residual vectors
+        float sc[G::ITEMS2][KP1 - 1];   // scales of this thread's items, the same for every chunk
+        float vf[G::ITEMS2][KP1];       // 2^e of the items' residual vectors
         int chs[G::ITEMS2];             // channel of each item
 #pragma unroll
         for (int i = 0; i < G::ITEMS2; ++i) {
             const int p = pt + i * PR::PROD_THREADS;
-            chs[i] = CLIP ? p / (P_KC / 2) : pair_channel<KP1>(p / (P_KC / 2), nch);
+            chs[i] = pair_channel<KP1>(p / (P_KC / 2), nch);
             const int k = k0 + chs[i];
-            const bool own = !CLIP && p < nch * (P_KC / 2);
+            const bool own = p < nch * (P_KC / 2);
 #pragma unroll
-            for (int n = 0; n < G::KQ; ++n)
-                sc[i][n] = (own && n < KP1 - 1) ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
+            for (int n = 0; n < KP1 - 1; ++n)
+                sc[i][n] = own ? __ldg(scales + (size_t)k * (KP1 - 1) + n) : 0.0f;
 #pragma unroll
-            for (int n = 0; n < G::VF; ++n)
+            for (int n = 0; n < KP1; ++n)
                 vf[i][n] = own ? ctl.vscale[chs[i] * KP1 + n] : 0.0f;
         }
-        const float xs = F16 ? ctl.xscale : 1.0f;
+        const float xs = ctl.xscale;
         for (int it = 0; it < total; ++it) {
             const int s = it % NST, slot = it % R;
             const uint32_t ph = (uint32_t)(it / NST) & 1u;
@@ -401,9 +320,8 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 note_timeout(wc, KBIT);
             }
             if (__any_sync(0xffffffffu, !ok || *abort_flag)) break;   // warp-uniform
-            const int ts = F16 ? s >> 1 : s, hh = F16 ? s & 1 : 0;
-            pair_consume<KP1, CLIP>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + ts * P_STAGE_BYTES,
-                                    hh, pt, nch, chs, sc, vf, xs, ctl, qmaxf);
+            pair_consume<KP1>(ring_u32 + slot * G::RAW_BYTES, stages_u32 + (s >> 1) * P_STAGE_BYTES,
+                              s & 1, pt, nch, chs, sc, vf, xs);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
@@ -464,7 +382,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
     } else if (warp == PR::MMA_WARP) {
         // ---------------------------------------------------------------- MMA issuer (even CTA)
         if (half == 0 && lane == 0) {
-            constexpr uint32_t idesc = F16 ? idesc_f16(2 * P_VEC, P_N) : idesc_tf32(2 * P_VEC, P_N);
+            constexpr uint32_t idesc = idesc_f16(2 * P_VEC, P_N);
             int g = 0;
             for (int lt = 0; lt < my_rt && !*abort_flag; ++lt) {
                 for (int kc = 0; kc < n_kc; ++kc) {
@@ -487,28 +405,18 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                     }
                     if (*abort_flag) break;
                     tc_fence_after();
-                    const uint32_t sb = stages_u32 + (F16 ? s >> 1 : s) * P_STAGE_BYTES;
+                    const uint32_t sb = stages_u32 + (s >> 1) * P_STAGE_BYTES;
                     const uint64_t ah = smem_desc_sw128(sb + P_OFF_A_HI);
                     const uint64_t al = smem_desc_sw128(sb + P_OFF_A_LO);
                     const uint64_t bh = smem_desc_sw128(sb + P_OFF_B_HI);
                     const uint64_t bl = smem_desc_sw128(sb + P_OFF_B_LO);
-                    if constexpr (F16) {
-                        // 32 fp16 elements of this stage's row half = two K = 16 steps of 32 bytes
+                    // 32 fp16 elements of this stage's row half = two K = 16 steps of 32 bytes
 #pragma unroll
-                        for (int kk = 0; kk < 2; ++kk) {
-                            const uint64_t o = (uint64_t)(((s & 1) * 2 + kk) * 2);   // 16 B units
-                            mma_f16_pair(tmem, al + o, bh + o, idesc, (seg_start && kk == 0) ? 0u : 1u);
-                            mma_f16_pair(tmem, ah + o, bl + o, idesc, 1u);
-                            mma_f16_pair(tmem, ah + o, bh + o, idesc, 1u);
-                        }
-                    } else {
-#pragma unroll
-                        for (int kk = 0; kk < P_KC / 8; ++kk) {
-                            const uint64_t o = (uint64_t)(kk * 2);   // 32 bytes, in 16 B units
-                            mma_tf32_pair(tmem, al + o, bh + o, idesc, (seg_start && kk == 0) ? 0u : 1u);
-                            mma_tf32_pair(tmem, ah + o, bl + o, idesc, 1u);
-                            mma_tf32_pair(tmem, ah + o, bh + o, idesc, 1u);
-                        }
+                    for (int kk = 0; kk < 2; ++kk) {
+                        const uint64_t o = (uint64_t)(((s & 1) * 2 + kk) * 2);   // 16 B units
+                        mma_f16_pair(tmem, al + o, bh + o, idesc, (seg_start && kk == 0) ? 0u : 1u);
+                        mma_f16_pair(tmem, ah + o, bl + o, idesc, 1u);
+                        mma_f16_pair(tmem, ah + o, bh + o, idesc, 1u);
                     }
                     mma_commit_pair(&ctl.empty[s], pair_mask);
                     if ((kc % SEG) == SEG - 1 || kc == n_kc - 1) {
@@ -529,7 +437,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
             prefetch_tensormap(&tmW);
             prefetch_tensormap(&tmQ);
             int issued = 0;
-            for (int f = 0; f < ((!CLIP && wc.withhold) ? 0 : total); ++f) {
+            for (int f = 0; f < (wc.withhold ? 0 : total); ++f) {
                 const int slot = f % R;
                 if (f >= R &&
                     !mbar_wait(&ctl.raw_empty[slot], (uint32_t)(f / R - 1) & 1u, wc.budget)) {
@@ -550,7 +458,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 mbar_arrive_expect_tx(&ctl.raw_full[slot], G::RAW_TX);
                 tma_load_2d(dst, &tmX, x, row0, &ctl.raw_full[slot]);
                 tma_load_2d(dst + G::RAW_W, &tmW, x, k0, &ctl.raw_full[slot]);
-                if (!CLIP) tma_load_3d(dst + G::RAW_Q, &tmQ, x, k0, 0, &ctl.raw_full[slot]);
+                tma_load_3d(dst + G::RAW_Q, &tmQ, x, k0, 0, &ctl.raw_full[slot]);
                 issued = f + 1;
             }
             // no copy may land after the CTA is gone: wait for the last copies of every slot
@@ -571,7 +479,7 @@ output_error_pair_kernel(const float *__restrict__ scales, int C, int N, int d, 
                 s += ld_dsmem_f64(&ctl.part[1][m], crank + 2u * (uint32_t)j);
             }
             double v = s / (double)N;
-            if (F16) v *= pow2d(-2 * (ctl.xexp + ctl.vexp[m]));   // exact: undo the operand scales
+            v *= pow2d(-2 * (ctl.xexp + ctl.vexp[m]));   // exact: undo the operand scales
             if (MPQ_IN((size_t)k0 * KP1 + m, (size_t)C * KP1)) err[(size_t)k0 * KP1 + m] = (float)v;
         }
     }
@@ -710,18 +618,15 @@ mpq_status launch_pooled_f16(const float *X, int N, const float *W, const int8_t
     return r;
 }
 
-// ext_range: caller-provided range scratch (fp16 operands: this kernel), or NULL (fp16 operands:
-// the pooled path of output_error_f16.cu).
-template <int KP1, bool CLIP>
+// ext_range: caller-provided range scratch (this kernel), or NULL (the pooled path of
+// output_error_f16.cu).
+template <int KP1>
 mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *codes,
-                       const float *scales, int C, int d, int qmax, float *err, cudaStream_t stream,
-                       unsigned *ext_range = nullptr, const float *rmax = nullptr)
+                       const float *scales, int C, int d, float *err, cudaStream_t stream,
+                       unsigned *ext_range, const float *rmax)
 {
-    if constexpr (!CLIP) {
-        if (!ext_range)
-            return launch_pooled_f16<KP1>(X, N, W, codes, scales, C, d, err, stream, rmax);
-    }
-    using G = PGeo<KP1, CLIP>;
+    if (!ext_range) return launch_pooled_f16<KP1>(X, N, W, codes, scales, C, d, err, stream, rmax);
+    using G = PGeo<KP1>;
     const int n_pairs = (C + 2 * G::CH - 1) / (2 * G::CH);
     const int n_rt = (N + P_N - 1) / P_N;
 
@@ -738,7 +643,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     const cuuint32_t bq[3] = {P_KC, (cuuint32_t)G::CH, (cuuint32_t)G::K};
     if (!encode_tile_map(&tmX, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, X, dx, sx, bx) ||
         !encode_tile_map(&tmW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, W, dw, sw, bw) ||
-        (!CLIP && !encode_tile_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq))) {
+        !encode_tile_map(&tmQ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, codes, dq, sq, bq)) {
         set_error("output error: tensor map encoding failed");
         return MPQ_ERR_CUDA;
     }
@@ -746,12 +651,12 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         set_error("pair output error needs %d bytes of shared memory", G::SMEM);
         return MPQ_ERR_UNSUPPORTED;
     }
-    cudaError_t e = cudaFuncSetAttribute(output_error_pair_kernel<KP1, CLIP>,
+    cudaError_t e = cudaFuncSetAttribute(output_error_pair_kernel<KP1>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute");
 
     cudaLaunchConfig_t cfg = {};
-    cfg.blockDim = dim3(PRoles<CLIP>::THREADS, 1, 1);
+    cfg.blockDim = dim3(PRoles::THREADS, 1, 1);
     cfg.dynamicSmemBytes = (size_t)G::SMEM;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -773,7 +678,7 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
         cfg.gridDim = dim3((unsigned)(n_pairs * 2 * sp), 1, 1);
         int active = resident[i].load(std::memory_order_relaxed);
         if (active == 0) {
-            if (cudaOccupancyMaxActiveClusters(&active, output_error_pair_kernel<KP1, CLIP>, &cfg) !=
+            if (cudaOccupancyMaxActiveClusters(&active, output_error_pair_kernel<KP1>, &cfg) !=
                 cudaSuccess)
                 active = -1;
             (void)cudaGetLastError();
@@ -792,20 +697,13 @@ mpq_status launch_pair(const float *X, int N, const float *W, const int8_t *code
     WaitCtl wc;
     mpq_status wst = wait_ctl(&wc);
     if (wst != MPQ_OK) return wst;
-    if constexpr (!CLIP) {
-        // fp16 operands (the fixed-scratch entry point): the ranges of X and of every residual
-        // vector first, into the caller's table (the residual vectors' from rmax when the greedy
-        // search gave them: then the pre-pass reads X alone)
-        e = launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax == nullptr, ext_range, stream);
-        const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : ext_range + 1;
-        if (e == cudaSuccess)
-            e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
-                                   (const unsigned *)ext_range, vr, err, split, wc, tmX, tmW, tmQ);
-        return cuda_status(e, "pair output-error kernel launch");
-    }
-    e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1, CLIP>, scales, C, N, d, qmax,
-                           (const unsigned *)nullptr, (const unsigned *)nullptr, err, split, wc,
-                           tmX, tmW, tmQ);
+    // the ranges of X and of every residual vector first, into the caller's table (the residual
+    // vectors' from rmax when the greedy search gave them: then the pre-pass reads X alone)
+    e = launch_ranges<KP1>(X, N, W, codes, scales, C, d, rmax == nullptr, ext_range, stream);
+    const unsigned *vr = rmax ? reinterpret_cast<const unsigned *>(rmax) : ext_range + 1;
+    if (e == cudaSuccess)
+        e = cudaLaunchKernelEx(&cfg, output_error_pair_kernel<KP1>, scales, C, N, d,
+                               (const unsigned *)ext_range, vr, err, split, wc, tmX, tmW, tmQ);
     return cuda_status(e, "pair output-error kernel launch");
 }
 
@@ -882,7 +780,7 @@ mpq_status launch_output_error_pair(const float *X, int N, const float *W, const
 {
     switch (k_max + 1) {
 #define MPQ_CASE(n) \
-    case n: return launch_pair<n, false>(X, N, W, codes, scales, C, d, 0, err, stream, range, rmax);
+    case n: return launch_pair<n>(X, N, W, codes, scales, C, d, err, stream, range, rmax);
         MPQ_CASE(2) MPQ_CASE(3) MPQ_CASE(4) MPQ_CASE(5) MPQ_CASE(6) MPQ_CASE(7) MPQ_CASE(8)
         MPQ_CASE(9) MPQ_CASE(10) MPQ_CASE(11) MPQ_CASE(12) MPQ_CASE(13) MPQ_CASE(14) MPQ_CASE(15)
         MPQ_CASE(16) MPQ_CASE(17)

@@ -194,21 +194,10 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
         : "memory");
 }
 
-// CTA-pair MMA, issued by one thread of the pair's even CTA: A is M = 256 rows, 128 in each CTA's
-// shared memory at the descriptor's offset; B is N rows, N/2 in each CTA; D lands in each CTA's
-// tensor memory (its own 128 rows x N columns) at d_tmem.
-__device__ __forceinline__ void mma_tf32_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                              uint32_t idesc, uint32_t accumulate)
-{
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::2.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
-// CTA-pair MMA of kind::f16 with fp16 A and B (fp32 accumulate); operands as in mma_tf32_pair.
+// CTA-pair MMA of kind::f16 with fp16 A and B (fp32 accumulate), issued by one thread of the
+// pair's even CTA: A is M = 256 rows, 128 in each CTA's shared memory at the descriptor's offset;
+// B is N rows, N/2 in each CTA; D lands in each CTA's tensor memory (its own 128 rows x N columns)
+// at d_tmem.
 __device__ __forceinline__ void mma_f16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                              uint32_t idesc, uint32_t accumulate)
 {

@@ -20,14 +20,6 @@ __device__ __forceinline__ void split4(const float4 x, float4 &hi, float4 &lo)
     lo.w = __fsub_rn(x.w, hi.w);
 }
 
-__device__ __forceinline__ void split2(const float2 x, float2 &hi, float2 &lo)
-{
-    hi.x = __uint_as_float(__float_as_uint(x.x) & 0xFFFFE000u);
-    hi.y = __uint_as_float(__float_as_uint(x.y) & 0xFFFFE000u);
-    lo.x = __fsub_rn(x.x, hi.x);
-    lo.y = __fsub_rn(x.y, hi.y);
-}
-
 // Code byte b (0..3) of `biased` (int8 codes XOR 0x80 per byte) as an exact float: the byte
 // becomes the low mantissa byte of 2^23, and subtracting 2^23 + 128 is exact.
 __device__ __forceinline__ float code_from_biased(uint32_t biased, int b)
