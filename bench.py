@@ -808,6 +808,17 @@ def clip_oracle_stride(wl, target_s, n_cand):
     return max(1, int(np.ceil(est / host_cores() / target_s)))
 
 
+def clip_launches(layer, n_cand):
+    """Kernels one mpq_clip_search call launches: candidates and argmin, plus (tensor-core path) the
+    X range and split and, per chunk of at most 4 GiB of residual planes, the planes and the
+    contraction; else the shared-memory error kernel."""
+    if layer.groups != 1 or layer.d % 16:
+        return 3
+    per_chunk = max(1, (1 << 32) // (4 * layer.d * n_cand))
+    chunks = -(-layer.C // min(layer.C, per_chunk))
+    return 4 + 2 * chunks
+
+
 def run_clip(args, world, rank, local):
     """Eq. 12 over every layer of the workload: mpq_clip_search (per-channel candidates, output
     errors on the tensor cores, argmin) with layers on a pool of streams."""
@@ -902,9 +913,10 @@ def run_clip(args, world, rank, local):
     t1 = float(np.mean(one_ms)) / 1e3
     peak = peaks["bf16_tflops"]
     ach = flops_per_step / t1 / 1e12
-    roofline = {"kernel": "output_error_f16_kernel in clip mode (Eq. 12 residuals generated on chip, "
-                          "tcgen05 cta_group::2 kind::f16, 3-pass hi/lo split) + candidate, X range, "
-                          "X split and argmin kernels",
+    roofline = {"kernel": "output_error_f16_kernel in clip mode (Eq. 12 residuals written once as "
+                          "fp16 hi/lo planes by clip_planes_kernel and tile-copied into a tcgen05 "
+                          "cta_group::2 kind::f16 3-pass contraction) + candidate, X range, X split "
+                          "and argmin kernels",
                 "bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
                 "frac": ach / peak, "traffic": None,
                 "peak_source": f"{peak_src} bf16 dense burst (fp16 operands: the same rate)",
@@ -921,7 +933,7 @@ def run_clip(args, world, rank, local):
                       "l2": "flushed between steps (512 MB write)", "streams": args.streams,
                       "parallelism": f"replicas x{world}"},
            "roofline": roofline,
-           "gpu_launches": sum(5 if l.groups == 1 and l.d % 16 == 0 else 3 for l in layers) * args.steps,
+           "gpu_launches": sum(clip_launches(l, nc) for l in layers) * args.steps,
            "clocks": clk.summary()}
     if not args.no_e2e:
         def e2e_step():

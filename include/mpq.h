@@ -17,8 +17,8 @@
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Every call
  *    only enqueues work on `stream` and returns; results are ready when the stream reaches them.
  *    No entry point synchronizes, and none allocates device memory except the scratch of
- *    mpq_output_error and mpq_quantize_layer_adaptive, which comes from the device's
- *    stream-ordered pool on `stream` and goes back to it on `stream` (see there).
+ *    mpq_output_error, mpq_clip_search and mpq_quantize_layer_adaptive, which comes from the
+ *    device's stream-ordered pool on `stream` and goes back to it on `stream` (see there).
  *  - Arguments are validated on the host before anything is enqueued; an invalid argument
  *    returns MPQ_ERR_INVALID_ARG / MPQ_ERR_UNSUPPORTED and leaves every output untouched.
  *    A failed kernel launch returns MPQ_ERR_CUDA.  mpq_last_error() gives a message for the
@@ -122,7 +122,8 @@ mpq_status mpq_quantize_layer(const float *W, int C, int d, int bits, int G,
  *   err     out [C][k_max+1] fp32.
  *
  * Scratch: with groups == 1, d a multiple of 16 and X, W, codes 16-byte aligned (the tensor-core
- * path with scaled fp16 operands), the call takes 4 (1 + C (k_max+1)) bytes (4 bytes with rmax)
+ * path with scaled fp16 operands), the call takes 4 (1 + C (k_max+1)) bytes (4 bytes with rmax),
+ * rounded up to 256, plus 4 N d bytes for X's fp16 hi/lo planes
  * from the current device's default stream-ordered memory pool with cudaMallocAsync on `stream`
  * and returns them with cudaFreeAsync on `stream` -- concurrent calls on other streams each get
  * their own, and a CUDA graph capture records them as the graph's allocation nodes.
@@ -301,6 +302,12 @@ mpq_status mpq_center_weights(const float *W, int C, int d, int mode, float *cen
  *   clip          out [C][n_cand] fp32: K_c of each channel (also used as working storage).
  *   err           out [C][n_cand] fp32.
  *   best          out [C] int32; the chosen factor of channel k is clip[k][best[k]].
+ * Scratch: with groups == 1, d a multiple of 16 and X, W 16-byte aligned (the tensor-core path),
+ * 4 C + 4 N d bytes (channel maxima, X's fp16 hi/lo planes) and the fp16 hi/lo planes of the
+ * candidates' residuals, 4 d n_cand bytes per channel for at most max(1, 2^32 / (4 d n_cand))
+ * channels at a time (larger layers run in chunks of whole channels), come from the current
+ * device's stream-ordered pool on `stream` (as for mpq_output_error; MPQ_ERR_NOMEM if it has no
+ * room).
  */
 mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, int C, int d,
                            int bits, int n_cand, int mode, float *clip, float *err, int *best,

@@ -603,31 +603,31 @@ f16_split_kernel(const float4 *__restrict__ X, long long n8, const unsigned *__r
 
 // Clipping search (Eq. 12): the residual r = w - s q of channel c0 + v / n_cand under candidate
 // v mod n_cand (s = K / Qmax, the codes q of Eq. 8 with the sign of w, q = 0 where s is 0 or NaN),
-// scaled by 2^e and split into fp16 hi/lo planes ([2][M][d] as hi and lo), 8 elements a thread per
-// step.  e comes from a bound on the vector's elements, max(s/2, max|w| - Qmax s) (s/2 for a
-// nearest code, max|w| - Qmax s where the code is clamped; a residual a rounding above it still
-// fits fp16, whose range reaches 2^16), kept in vrange[v] (float bits) for the contraction.
-__global__ void __launch_bounds__(256)
+// scaled by 2^e and split into fp16 hi/lo planes ([2][M][d] as hi and lo).  One CTA per vector v,
+// 8 elements a thread per step.  e comes from a bound on the vector's elements,
+// max(s/2, max|w| - Qmax s) (s/2 for a nearest code, max|w| - Qmax s where the code is clamped; a
+// residual a rounding above it still fits fp16, whose range reaches 2^16), kept in vrange[v]
+// (float bits) for the contraction.
+__global__ void __launch_bounds__(128)
 clip_planes_kernel(const float *__restrict__ W, int d, const float *__restrict__ clip,
-                   const float *__restrict__ chmax, int c0, int n_cand, int qmax, long long M,
+                   const float *__restrict__ chmax, int c0, int n_cand, int qmax, int M,
                    uint4 *__restrict__ hi, uint4 *__restrict__ lo, unsigned *__restrict__ vrange)
 {
-    const int d8 = d / 8;
-    const long long n = M * d8;
+    const int v = blockIdx.x, d8 = d / 8;
+    if (v >= M) return;
+    const long long k = c0 + v / n_cand;
     const float qmaxf = (float)qmax, qlim = qmaxf + 1.0f;
     const float tband = 0.5f - MPQ_FAST_REL * (qlim + 1.0f);
-    const long long stride = (long long)gridDim.x * blockDim.x;
-    for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += stride) {
-        const long long v = t / d8;
-        const int j = (int)(t - v * d8);
-        const long long k = c0 + v / n_cand;
-        // clip row of channel k, candidate v mod n_cand: index c0 n_cand + v
-        const float sv = __fdiv_rn(__ldg(clip + (long long)c0 * n_cand + v), qmaxf);
-        const float inv = sv > 0.0f ? __frcp_rn(sv) : 0.0f;
-        const float bound = fmaxf(__fmul_rn(0.5f, sv), __fmaf_rn(-qmaxf, sv, __ldg(chmax + k)));
-        const float vf = pow2f(f16_scale_exp(bound));
-        const float4 *w4 = reinterpret_cast<const float4 *>(W + k * d) + 2 * j;
-        const float4 a = __ldg(w4), b = __ldg(w4 + 1);
+    // clip row of channel k, candidate v mod n_cand: index c0 n_cand + v
+    const float sv = __fdiv_rn(__ldg(clip + (long long)c0 * n_cand + v), qmaxf);
+    const float inv = sv > 0.0f ? __frcp_rn(sv) : 0.0f;
+    const float bound = fmaxf(__fmul_rn(0.5f, sv), __fmaf_rn(-qmaxf, sv, __ldg(chmax + k)));
+    const float vf = pow2f(f16_scale_exp(bound));
+    if (threadIdx.x == 0) vrange[v] = __float_as_uint(bound);
+    const float4 *w4 = reinterpret_cast<const float4 *>(W + k * d);
+    const long long row = (long long)v * d8;
+    for (int j = threadIdx.x; j < d8; j += blockDim.x) {
+        const float4 a = __ldg(w4 + 2 * j), b = __ldg(w4 + 2 * j + 1);
         const float w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
         float q[8];
         bool unsure = false;
@@ -642,9 +642,8 @@ clip_planes_kernel(const float *__restrict__ W, int d, const float *__restrict__
         for (int e = 0; e < 4; ++e)
             split_f16x2(__fmul_rn(__fmaf_rn(-sv, q[2 * e], w[2 * e]), vf),
                         __fmul_rn(__fmaf_rn(-sv, q[2 * e + 1], w[2 * e + 1]), vf), h[e], l[e]);
-        hi[t] = make_uint4(h[0], h[1], h[2], h[3]);
-        lo[t] = make_uint4(l[0], l[1], l[2], l[3]);
-        if (j == 0) vrange[v] = __float_as_uint(bound);
+        hi[row + j] = make_uint4(h[0], h[1], h[2], h[3]);
+        lo[row + j] = make_uint4(l[0], l[1], l[2], l[3]);
     }
 }
 
@@ -788,9 +787,9 @@ mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *c
     if (st != MPQ_OK) return st;
     cudaError_t e = launch_x_split(X, N, d, xrange, xs, stream);
     if (e != cudaSuccess) return cuda_status(e, "X split kernel launch");
-    // residual planes of whole channels, at most 2 GiB at a time, and their bounds
+    // residual planes of whole channels, at most 4 GiB at a time, and their bounds
     const long long vec_bytes = 4LL * d;
-    const int cc = (int)std::min<long long>(C, std::max(1LL, (1LL << 31) / (vec_bytes * n_cand)));
+    const int cc = (int)std::min<long long>(C, std::max(1LL, (1LL << 32) / (vec_bytes * n_cand)));
     const long long m_max = (long long)cc * n_cand;
     const size_t planes_bytes = (size_t)(m_max * vec_bytes);
     void *scratch = nullptr;
@@ -800,16 +799,15 @@ mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *c
     unsigned *vrange = reinterpret_cast<unsigned *>(static_cast<char *>(scratch) + planes_bytes);
     for (int c0 = 0; c0 < C && st == MPQ_OK; c0 += cc) {
         const int cn = std::min(cc, C - c0);
-        const long long M = (long long)cn * n_cand;
-        const long long n = M * (d / 8);
-        const int blocks = (int)std::min<long long>((n + 255) / 256, 8LL * sm_count());
+        const int M = cn * n_cand;
+        const int threads = std::min(128, (d / 8 + 31) / 32 * 32);
         uint4 *hi = reinterpret_cast<uint4 *>(planes);
-        clip_planes_kernel<<<(unsigned)blocks, 256, 0, stream>>>(W, d, clip, chmax, c0, n_cand,
-                                                                  qmax, M, hi, hi + n, vrange);
+        clip_planes_kernel<<<(unsigned)M, (unsigned)threads, 0, stream>>>(
+            W, d, clip, chmax, c0, n_cand, qmax, M, hi, hi + (size_t)M * (d / 8), vrange);
         e = cudaGetLastError();
         st = cuda_status(e, "clip residual planes kernel launch");
         if (st == MPQ_OK)
-            st = launch_f16<1, true>(planes, N, nullptr, nullptr, (int)M, d,
+            st = launch_f16<1, true>(planes, N, nullptr, nullptr, M, d,
                                      err + (size_t)c0 * n_cand, xrange, vrange, xs, stream);
     }
     e = cudaFreeAsync(scratch, stream);

@@ -102,3 +102,23 @@ def test_full_size_sampled(gpu, oracle):
             o_err = oracle.clip_errors(X, 1, W, 4, o_clip, channels=(c0, c0 + 8), threads=8)
             compare_err(err[c0:c0 + 8], o_err[c0:c0 + 8])
         assert np.array_equal(best, oracle.clip_select(err, mode))
+
+
+def test_planes_in_chunks(gpu, oracle):
+    """Residual planes over 4 GiB (4100 channels x 32 candidates x d = 8192 x 4 bytes) are written
+    and contracted in two chunks of whole channels; channels on both sides of the boundary (4096)
+    against the oracle."""
+    C, d, N, nc = 4100, 8192, 256, 32
+    W = wlm.random_weights(C, d, 91, "laplace")
+    X = wlm.random_calibration(N, d, 92)
+    t = lambda a: torch.from_numpy(a).to("cuda:0")
+    clip, err, best = binding.mpq_clip_search(t(X), t(W), 4, nc, binding.MPQ_CLIP_PER_CHANNEL)
+    torch.cuda.synchronize()
+    clip, err, best = clip.cpu().numpy(), err.cpu().numpy(), best.cpu().numpy()
+    o_clip = oracle.clip_candidates(W, nc, binding.MPQ_CLIP_PER_CHANNEL)
+    assert np.array_equal(clip, o_clip)
+    for c0 in (0, 4090, C - 4):
+        o_err = oracle.clip_errors(X, 1, W, 4, o_clip, channels=(c0, c0 + 4), threads=8)
+        compare_err(err[c0:c0 + 4], o_err[c0:c0 + 4])
+    assert np.array_equal(best, oracle.clip_select(err, binding.MPQ_CLIP_PER_CHANNEL))
+
