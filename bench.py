@@ -42,7 +42,8 @@ KERNEL_SOURCES = {
                      "paper_2002_09049_gb300/csrc/tf32_operands.cuh",
                      "paper_2002_09049_gb300/csrc/waits.cuh"),
     "quantize": ("paper_2002_09049_gb300/csrc/quantize.cu",
-                 "paper_2002_09049_gb300/csrc/rounding.cuh"),
+                 "paper_2002_09049_gb300/csrc/rounding.cuh",
+                 "paper_2002_09049_gb300/csrc/sm100.cuh"),
     "allocate": "paper_2002_09049_gb300/csrc/allocate.cu",
     "reconstruct": "paper_2002_09049_gb300/csrc/reconstruct.cu",
     "center": "paper_2002_09049_gb300/csrc/center.cu",

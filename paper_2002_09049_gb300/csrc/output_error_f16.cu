@@ -129,7 +129,6 @@ template <int KP1>
 struct FShape<KP1, true> {
     static constexpr int kp1 = 1, ch = F_VEC, raw = 0, na = F_PRE_ASETS, raw_bytes = 0;
     static constexpr int smem = 1024 + F_CTRL_BYTES + (F_PRE_ASETS + F_BSLOTS) * F_SET;
-    static constexpr uint32_t raw_tx = 0;
 };
 static_assert(FShape<1, true>::smem <= F_SMEM_LIMIT, "clipping search: shared memory");
 
