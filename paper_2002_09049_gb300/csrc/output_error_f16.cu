@@ -22,9 +22,10 @@
 // * The tile copies are issued by one epilogue warp, which is idle between its folds: neither the
 //   producers (a stage waits for its slowest producer warp) nor the MMA thread carry them.
 //
-// Warps: 0-6 producers (224 threads: one (channel, element pair) item per 32-element half step
-// each when k_max + 1 = 9), 7 the MMA issuer (lane 0 of the even CTA), 8-15 the epilogue (lane
-// quarter warp % 4, column half; warp 15 also issues this CTA's tile copies).  Results are
+// Warps: 0-6 producers (224 threads: one (channel, 4 elements) item per step each when
+// k_max + 1 = 9; in the clipping search warp 0 only relays that a stage's tiles have landed), 7
+// the MMA issuer (lane 0 of the even CTA), 8-15 the epilogue (lane quarter warp % 4, column half;
+// warp 15 also issues this CTA's tile copies).  Results are
 // bit-identical to the fp16 mode of output_error_pair.cu: the same operands, MMAs in the same
 // order (zero-filled elements past d add exact zeros), the same fp32 additions and the same
 // reduction.  Every wait is bounded; on a timeout the kernel records MPQ_TIMEOUT_OUTPUT_ERROR,
@@ -104,7 +105,7 @@ template <int KP1>
 struct FGeo {
     static constexpr int K = KP1 - 1;
     static constexpr int CH = F_VEC / KP1;
-    static constexpr int ITEMS = (CH * 16 + F_PT - 1) / F_PT;   // 16 element pairs per half step
+    static constexpr int ITEMS = (CH * 16 + F_PT - 1) / F_PT;   // 16 items of 4 elements per step
     static constexpr int RAW_Q = CH * F_KS * 4;
     static constexpr uint32_t RAW_TX = CH * F_KS * 4 + K * CH * F_KS;
     static constexpr int RAW_BYTES = (RAW_Q + K * CH * F_KS + 1023) / 1024 * 1024;
@@ -144,11 +145,11 @@ __device__ __forceinline__ void setmaxnreg_dec()
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
 
-// Raw slot -> A tiles of one step (tile set `aset`): for every (channel, element pair) item of
-// both 32-element halves the residuals r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7), each scaled by
-// its vector's 2^e (vf) and split into fp16 hi/lo halves.  A half warp's 16 items fill 64 bytes of
-// one row; the warp's two channels are paired (pair_channel) so that their rows land in different
-// bank halves.  Every shared-memory read of an item before its stores.
+// Raw slot -> A tiles of one step (tile set `aset`): for every (channel, 4 contiguous elements)
+// item the residuals r_0 = w, r_{n+1} = r_n - s_n q_n (Eq. 7), each scaled by its vector's 2^e
+// (vf) and split into fp16 hi/lo halves.  W as one 16-byte load, each point's codes as one 4-byte
+// load, 8-byte operand stores: a half warp's 16 items fill one 128-byte row.  Every shared-memory
+// read of an item before its stores.
 template <int KP1>
 __device__ __forceinline__ void f16_make_a(uint32_t slot, uint32_t aset, int pt, int nch,
                                            const int (&chs)[FGeo<KP1>::ITEMS],
@@ -161,33 +162,28 @@ __device__ __forceinline__ void f16_make_a(uint32_t slot, uint32_t aset, int pt,
     for (int i = 0; i < G::ITEMS; ++i) {
         const int p = pt + i * F_PT;
         if (p < nch * 16) {
-            const int ch = chs[i], e2 = p % 16;
-            float2 r[2];
-            uint32_t qb[2][K];
+            const int ch = chs[i], e4 = p % 16;
+            float4 r = ld_shared_v4(slot + (uint32_t)(ch * F_KS + e4 * 4) * 4u);
+            uint32_t qb[K];
 #pragma unroll
-            for (int hh = 0; hh < 2; ++hh) {
-                const int e = hh * 32 + e2 * 2;
-                r[hh] = ld_shared_v2(slot + (uint32_t)(ch * F_KS + e) * 4u);
-#pragma unroll
-                for (int n = 0; n < K; ++n)
-                    qb[hh][n] = ld_shared_u16(slot + G::RAW_Q + (uint32_t)((n * G::CH + ch) * F_KS + e)) ^
-                                0x8080u;
-            }
-            const uint32_t cofs = (uint32_t)(e2 & 3) * 4u;   // 2 elements = 4 bytes of a 16-byte chunk
+            for (int n = 0; n < K; ++n)
+                qb[n] = ld_shared_u32(slot + G::RAW_Q + (uint32_t)((n * G::CH + ch) * F_KS + e4 * 4)) ^
+                        0x80808080u;
+            const uint32_t cofs = (uint32_t)(e4 & 1) * 8u;   // 4 elements = 8 bytes of a 16-byte chunk
 #pragma unroll
             for (int n = 0; n < KP1; ++n) {
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    uint32_t hi, lo;
-                    split_f16x2(__fmul_rn(r[hh].x, vf[i][n]), __fmul_rn(r[hh].y, vf[i][n]), hi, lo);
-                    const uint32_t off = sw128_offset(ch * KP1 + n, hh * 4 + (e2 >> 2)) + cofs;
-                    st_shared_u32(aset + off, hi);
-                    st_shared_u32(aset + F_TILE + off, lo);
-                    if (n < K) {
-                        const float sn = sc[i][n];
-                        r[hh].x = __fmaf_rn(-sn, code_from_biased(qb[hh][n], 0), r[hh].x);
-                        r[hh].y = __fmaf_rn(-sn, code_from_biased(qb[hh][n], 1), r[hh].y);
-                    }
+                uint32_t h0, l0, h1, l1;
+                split_f16x2(__fmul_rn(r.x, vf[i][n]), __fmul_rn(r.y, vf[i][n]), h0, l0);
+                split_f16x2(__fmul_rn(r.z, vf[i][n]), __fmul_rn(r.w, vf[i][n]), h1, l1);
+                const uint32_t off = sw128_offset(ch * KP1 + n, e4 >> 1) + cofs;
+                st_shared_v2u(aset + off, h0, h1);
+                st_shared_v2u(aset + F_TILE + off, l0, l1);
+                if (n < K) {
+                    const float sn = sc[i][n];
+                    r.x = __fmaf_rn(-sn, code_from_biased(qb[n], 0), r.x);
+                    r.y = __fmaf_rn(-sn, code_from_biased(qb[n], 1), r.y);
+                    r.z = __fmaf_rn(-sn, code_from_biased(qb[n], 2), r.z);
+                    r.w = __fmaf_rn(-sn, code_from_biased(qb[n], 3), r.w);
                 }
             }
         }
@@ -316,7 +312,7 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
 #pragma unroll
             for (int i = 0; i < G::ITEMS; ++i) {
                 const int p = pt + i * F_PT;
-                chs[i] = pair_channel<K + 1>(p / 16, nch);
+                chs[i] = p / 16;
                 const bool own = p < nch * 16;
                 const int k = k0 + chs[i];
 #pragma unroll

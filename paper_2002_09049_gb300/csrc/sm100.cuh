@@ -410,6 +410,13 @@ __device__ __forceinline__ void st_shared_v2u(uint32_t addr, uint32_t a, uint32_
     asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
 }
 
+__device__ __forceinline__ uint32_t ld_shared_u32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+
 __device__ __forceinline__ uint32_t ld_shared_u16(uint32_t addr)
 {
     uint16_t v;
