@@ -306,8 +306,8 @@ mpq_status mpq_center_weights(const float *W, int C, int d, int mode, float *cen
  * 4 C + 4 N d bytes (channel maxima, X's fp16 hi/lo planes) and the fp16 hi/lo planes of the
  * candidates' residuals, 4 d n_cand bytes per channel for at most max(1, 2^32 / (4 d n_cand))
  * channels at a time (larger layers run in chunks of whole channels), come from the current
- * device's stream-ordered pool on `stream` (as for mpq_output_error; MPQ_ERR_NOMEM if it has no
- * room).
+ * device's stream-ordered pool on `stream` in one allocation (as for mpq_output_error;
+ * MPQ_ERR_NOMEM if it has no room, and nothing else is enqueued then).
  */
 mpq_status mpq_clip_search(const float *X, int N, int groups, const float *W, int C, int d,
                            int bits, int n_cand, int mode, float *clip, float *err, int *best,

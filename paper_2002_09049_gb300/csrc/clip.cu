@@ -10,7 +10,8 @@
 //      sets reduce the channels' maxima in one CTA;
 //   2. errors: the CTA-pair tensor-core contraction with residuals generated from W and the
 //      candidate scales on chip (output_error_f16.cu: fp16 hi/lo operands, each residual vector
-//      scaled by a power of two from the bound max(s/2, max|w| - Qmax s) on its elements), or,
+//      scaled by a power of two from the bound max(min(max|w|, s/2), max|w| - Qmax s) on its
+//      elements), or,
 //      for rows that are not 16-byte multiples and for per-channel inputs, one CTA per channel
 //      and candidate chunk with the residuals in shared memory and threads over the calibration
 //      rows;
@@ -225,14 +226,14 @@ mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C,
                        int n_cand, int mode, float *clip, float *err, int *best,
                        cudaStream_t stream)
 {
-    // the tensor-core path takes scratch from the stream-ordered pool: channel maxima, the X range
-    // word and the split X planes (2 N d fp16)
+    // the tensor-core path takes all its scratch from the stream-ordered pool before anything is
+    // enqueued: channel maxima, then the contraction's (X range and planes, residual planes)
     const bool tc = groups == 1 && output_error_pair_ok(X, W, reinterpret_cast<const int8_t *>(W), d);
     const size_t max_bytes = ((size_t)C * sizeof(float) + 255) / 256 * 256;
     char *scratch = nullptr;
     if (tc) {
         const mpq_status st = pool_scratch(reinterpret_cast<void **>(&scratch),
-                                           max_bytes + 256 + (size_t)N * d * 2 * sizeof(uint16_t),
+                                           max_bytes + clip_f16_scratch_bytes(C, N, d, n_cand),
                                            stream);
         if (st != MPQ_OK) return st;
     }
@@ -247,9 +248,8 @@ mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C,
     if (tc) {
         mpq_status st = cuda_status(e, "clip candidate kernel launch");
         if (st == MPQ_OK)
-            st = launch_clip_f16(X, N, W, clip, chmax, C, d, qmax, n_cand, err,
-                                 reinterpret_cast<unsigned *>(scratch + max_bytes),
-                                 reinterpret_cast<uint16_t *>(scratch + max_bytes + 256), stream);
+            st = launch_clip_f16(X, N, W, clip, chmax, C, d, qmax, n_cand, err, scratch + max_bytes,
+                                 stream);
         const cudaError_t ef = cudaFreeAsync(scratch, stream);
         if (st == MPQ_OK) st = cuda_status(ef, "scratch release (cudaFreeAsync)");
         if (st != MPQ_OK) return st;

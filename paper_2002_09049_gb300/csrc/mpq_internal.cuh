@@ -76,11 +76,12 @@ mpq_status launch_output_error_pair(const float *X, int N, const float *W, const
                                     cudaStream_t stream, unsigned *range, const float *rmax);
 
 // Clipping-search errors on the CTA-pair fp16 contraction (output_error_f16.cu): chmax = max|w|
-// per channel; xrange (one word) and xs (2 N d fp16) scratch on `stream`.  Needs
+// per channel; scratch of clip_f16_scratch_bytes() bytes, 256-byte aligned, on `stream`.  Needs
 // output_error_pair_ok(X, W, W, d).
+size_t clip_f16_scratch_bytes(int C, int N, int d, int n_cand);
 mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *clip,
                            const float *chmax, int C, int d, int qmax, int n_cand, float *err,
-                           unsigned *xrange, uint16_t *xs, cudaStream_t stream);
+                           void *scratch, cudaStream_t stream);
 mpq_status launch_clip(const float *X, int N, int groups, const float *W, int C, int d, int qmax,
                        int n_cand, int mode, float *clip, float *err, int *best,
                        cudaStream_t stream);

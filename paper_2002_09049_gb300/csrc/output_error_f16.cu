@@ -600,9 +600,11 @@ f16_split_kernel(const float4 *__restrict__ X, long long n8, const unsigned *__r
 // v mod n_cand (s = K / Qmax, the codes q of Eq. 8 with the sign of w, q = 0 where s is 0 or NaN),
 // scaled by 2^e and split into fp16 hi/lo planes ([2][M][d] as hi and lo).  One CTA per vector v,
 // 8 elements a thread per step.  e comes from a bound on the vector's elements,
-// max(s/2, max|w| - Qmax s) (s/2 for a nearest code, max|w| - Qmax s where the code is clamped; a
-// residual a rounding above it still fits fp16, whose range reaches 2^16), kept in vrange[v]
-// (float bits) for the contraction.
+// max(min(max|w|, s/2), max|w| - Qmax s): an element with code 0 keeps r = w, one with a nearest
+// nonzero code |r| <= s/2, a clamped one |r| = |w| - Qmax s (a residual a rounding above the bound
+// still fits fp16, whose range reaches 2^16); kept in vrange[v] (float bits) for the contraction.
+// (With max|w| below s/2, as for a small channel under a layer-wide K, every code is 0 and the
+// bound is max|r| itself.)
 __global__ void __launch_bounds__(128)
 clip_planes_kernel(const float *__restrict__ W, int d, const float *__restrict__ clip,
                    const float *__restrict__ chmax, int c0, int n_cand, int qmax, int M,
@@ -616,7 +618,8 @@ clip_planes_kernel(const float *__restrict__ W, int d, const float *__restrict__
     // clip row of channel k, candidate v mod n_cand: index c0 n_cand + v
     const float sv = __fdiv_rn(__ldg(clip + (long long)c0 * n_cand + v), qmaxf);
     const float inv = sv > 0.0f ? __frcp_rn(sv) : 0.0f;
-    const float bound = fmaxf(__fmul_rn(0.5f, sv), __fmaf_rn(-qmaxf, sv, __ldg(chmax + k)));
+    const float m = __ldg(chmax + k);
+    const float bound = fmaxf(fminf(m, __fmul_rn(0.5f, sv)), __fmaf_rn(-qmaxf, sv, m));
     const float vf = pow2f(f16_scale_exp(bound));
     if (threadIdx.x == 0) vrange[v] = __float_as_uint(bound);
     const float4 *w4 = reinterpret_cast<const float4 *>(W + k * d);
@@ -774,24 +777,35 @@ mpq_status launch_output_error_f16(const float *X, int N, const float *W, const 
     return MPQ_ERR_UNSUPPORTED;
 }
 
+// Channels per chunk of residual planes: whole channels, at most 4 GiB of planes at a time.
+static int clip_chunk_channels(int C, int d, int n_cand)
+{
+    return (int)std::min<long long>(C, std::max(1LL, (1LL << 32) / (4LL * d * n_cand)));
+}
+
+size_t clip_f16_scratch_bytes(int C, int N, int d, int n_cand)
+{
+    const long long m_max = (long long)clip_chunk_channels(C, d, n_cand) * n_cand;
+    return 256 /* X range */ + (size_t)N * d * 4 /* X planes */ + (size_t)m_max * d * 4 /* planes */ +
+           ((size_t)m_max * 4 + 255) / 256 * 256 /* bounds */;
+}
+
 mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *clip,
                            const float *chmax, int C, int d, int qmax, int n_cand, float *err,
-                           unsigned *xrange, uint16_t *xs, cudaStream_t stream)
+                           void *scratch, cudaStream_t stream)
 {
+    // scratch: the X range word, X's planes, the residual planes of one chunk, their bounds
+    const int cc = clip_chunk_channels(C, d, n_cand);
+    char *p = static_cast<char *>(scratch);
+    unsigned *xrange = reinterpret_cast<unsigned *>(p);
+    uint16_t *xs = reinterpret_cast<uint16_t *>(p + 256);
+    uint16_t *planes = reinterpret_cast<uint16_t *>(p + 256 + (size_t)N * d * 4);
+    unsigned *vrange = reinterpret_cast<unsigned *>(p + 256 + (size_t)N * d * 4 +
+                                                    (size_t)cc * n_cand * d * 4);
     mpq_status st = launch_x_range(X, N, d, xrange, stream);
     if (st != MPQ_OK) return st;
     cudaError_t e = launch_x_split(X, N, d, xrange, xs, stream);
     if (e != cudaSuccess) return cuda_status(e, "X split kernel launch");
-    // residual planes of whole channels, at most 4 GiB at a time, and their bounds
-    const long long vec_bytes = 4LL * d;
-    const int cc = (int)std::min<long long>(C, std::max(1LL, (1LL << 32) / (vec_bytes * n_cand)));
-    const long long m_max = (long long)cc * n_cand;
-    const size_t planes_bytes = (size_t)(m_max * vec_bytes);
-    void *scratch = nullptr;
-    st = pool_scratch(&scratch, planes_bytes + (size_t)(m_max * 4 + 255) / 256 * 256, stream);
-    if (st != MPQ_OK) return st;
-    uint16_t *planes = static_cast<uint16_t *>(scratch);
-    unsigned *vrange = reinterpret_cast<unsigned *>(static_cast<char *>(scratch) + planes_bytes);
     for (int c0 = 0; c0 < C && st == MPQ_OK; c0 += cc) {
         const int cn = std::min(cc, C - c0);
         const int M = cn * n_cand;
@@ -805,8 +819,6 @@ mpq_status launch_clip_f16(const float *X, int N, const float *W, const float *c
             st = launch_f16<1, true>(planes, N, nullptr, nullptr, M, d,
                                      err + (size_t)c0 * n_cand, xrange, vrange, xs, stream);
     }
-    e = cudaFreeAsync(scratch, stream);
-    if (st == MPQ_OK) st = cuda_status(e, "scratch release (cudaFreeAsync)");
     return st;
 }
 

@@ -85,6 +85,19 @@ def test_nonfinite_and_zero_channels(gpu, oracle):
     assert np.all(best == -1) and np.all(np.isnan(err))
 
 
+def test_per_layer_small_channels(gpu, oracle):
+    """One K for the layer while some channels are orders of magnitude smaller: their candidates
+    quantize everything to 0, so their residuals are the weights themselves, far below s/2; the
+    operand scale follows their own max|w| and the errors keep the 1e-5 bar."""
+    W = wlm.random_weights(24, 256, 41, "laplace")
+    W[3] *= np.float32(1e-4)
+    W[7] *= np.float32(1e-9)
+    W[11] *= np.float32(1e-6)
+    X = wlm.random_calibration(300, 256, 42)
+    run_both(oracle, X, W, 4, 20, binding.MPQ_CLIP_PER_LAYER)
+    run_both(oracle, X, W, 4, 20, binding.MPQ_CLIP_PER_CHANNEL)
+
+
 def test_full_size_sampled(gpu, oracle):
     """c5's up_proj shape (11008 x 4096, N = 2048) in the launch the bench times, checked on
     sampled channels against the oracle; per-layer argmin recomputed from the device table."""
