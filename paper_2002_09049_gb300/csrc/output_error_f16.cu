@@ -22,14 +22,19 @@
 // * The tile copies are issued by one epilogue warp, which is idle between its folds: neither the
 //   producers (a stage waits for its slowest producer warp) nor the MMA thread carry them.
 //
+// The clipping search (Eq. 12, CLIP) runs the same contraction over every channel's n_cand
+// candidate residuals r = w - s q: clip_planes_kernel writes them once as fp16 hi/lo planes like
+// X's, and the A tiles are tile-copied from those planes like the B tiles (128 vectors per CTA,
+// regardless of channel boundaries), so no producer work remains in that mode.
+//
 // Warps: 0-6 producers (224 threads: one (channel, 4 elements) item per step each when
 // k_max + 1 = 9; in the clipping search warp 0 only relays that a stage's tiles have landed), 7
 // the MMA issuer (lane 0 of the even CTA), 8-15 the epilogue (lane quarter warp % 4, column half;
 // warp 15 also issues this CTA's tile copies).  Results are
 // bit-identical to the fp16 mode of output_error_pair.cu: the same operands, MMAs in the same
 // order (zero-filled elements past d add exact zeros), the same fp32 additions and the same
-// reduction.  Every wait is bounded; on a timeout the kernel records MPQ_TIMEOUT_OUTPUT_ERROR,
-// waits for what it issued, and the outputs read NaN.
+// reduction.  Every wait is bounded; on a timeout the kernel records MPQ_TIMEOUT_OUTPUT_ERROR (or
+// MPQ_TIMEOUT_CLIP), waits for what it issued, and the outputs read NaN.
 #include <cuda.h>
 #include <cuda_fp16.h>
 #include <math.h>
