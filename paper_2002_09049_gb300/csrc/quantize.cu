@@ -1043,19 +1043,61 @@ quantize_kernel(const float *__restrict__ W, int C, int d, int qmax, int G, cons
             am = fmaxf(am, fabsf(v));
             return v;
         };
+        // Four elements at a time where the reciprocal is usable: their signed codes
+        // clamp(rint(v (1/s))) without a branch, all four redone with the correctly rounded division
+        // when any lane's quotient lies near a rounding boundary (a warp-uniform branch), so that the
+        // four elements' arithmetic interleaves.  The codes are Eq. 8's either way.
+        const bool fastq = s_best > 0.0f && inv_best > 0.0f;
+        const float qlim = qmaxf + 1.0f, tband = 0.5f - MPQ_FAST_REL * (qlim + 1.0f);
+        auto update4 = [&](float (&v4)[4], int j0) {   // elements j0 + NT u, every lane of the warp
+            float q4[4];
+            bool unsure = false;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) q4[u] = code_signed_fast(v4[u], inv_best, qmaxf, qlim, tband, unsure);
+            if (__any_sync(0xffffffffu, unsure)) {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) q4[u] = code_signed_exact(v4[u], s_best, qmaxf);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int j = j0 + NT * u;
+                const float v = __fmaf_rn(-s_best, q4[u], v4[u]);
+                const bool in = !ghost && MPQ_IN((size_t)i * plane + (size_t)k * d + j, n_codes);
+                if (in) qi[j] = (int8_t)(int)q4[u];
+                if (ri && in) ri[j] = v;
+                if (short_share) ssum = __fmaf_rn(v, v, ssum);
+                else kahan_add(ssum, scomp, v * v);
+                am = fmaxf(am, fabsf(v));
+                v4[u] = v;
+            }
+        };
         if constexpr (TM) {
             for (int cc = 0; cc < tcg; cc += 4) {
                 float v4[4];
                 __syncwarp();
                 sm100::tmem_ld_32x32b_x4(taddr + cc, v4);
+                if (fastq) {
+                    update4(v4, gt + NT * cc);
+                } else {
 #pragma unroll
-                for (int u = 0; u < 4; ++u) v4[u] = update(v4[u], gt + NT * (cc + u));
+                    for (int u = 0; u < 4; ++u) v4[u] = update(v4[u], gt + NT * (cc + u));
+                }
                 __syncwarp();
                 sm100::tmem_st_32x32b_x4(taddr + cc, v4);
             }
             sm100::tmem_wait_st();
         } else {
-            for (int j = gt; j < d; j += NT) sr[j] = update(sr[j], j);
+            int j = gt;
+            if (fastq) {
+                // groups of four while the warp's last lane still has all four (warp-uniform)
+                for (; j - lane + 31 + 3 * NT < d; j += 4 * NT) {
+                    float v4[4] = {sr[j], sr[j + NT], sr[j + 2 * NT], sr[j + 3 * NT]};
+                    update4(v4, j);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) sr[j + NT * u] = v4[u];
+                }
+            }
+            for (; j < d; j += NT) sr[j] = update(sr[j], j);
         }
         if (gt == 0 && !ghost && MPQ_IN((size_t)k * k_max + i, (size_t)C * k_max))
             scales[(size_t)k * k_max + i] = s_best;
