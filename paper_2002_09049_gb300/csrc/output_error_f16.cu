@@ -308,7 +308,7 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
             }
         } else if (!CLIP && warp < F_PROD_WARPS) {
             // ------------------------------------------------------------ producers
-            using G = FGeo<CLIP ? 2 : KP1>;
+            using G = FGeo<CLIP ? 2 : KP1>;   // (CLIP never gets here; FGeo<2> keeps it well-formed)
             constexpr int K = G::K;
             const int pt = threadIdx.x;
             float sc[G::ITEMS][K];      // scales of this thread's items, the same for every step
@@ -455,8 +455,9 @@ output_error_f16_kernel(const float *__restrict__ scales, int C, int N, int d,
                         const uint32_t bdst = b_u32 + bslot * F_SET;
                         const int row0 = (pr + (f / n_ks) * split) * F_N + half * F_ROWS;
                         // a tile copy starts 16-byte aligned (x counts int8 codes in the code
-                        // map) into a 1024-byte aligned destination (128-byte swizzle), or is not
-                        // issued and the launch ends through the bounded waits
+                        // map, fp16 elements in the planes) into a 1024-byte aligned destination
+                        // (128-byte swizzle), or is not issued and the launch ends through the
+                        // bounded waits
                         if constexpr (CLIP) {
                             // A tiles of step f (residual planes) into stage f % NA once the
                             // MMAs of step f - NA have completed
