@@ -61,7 +61,8 @@ constexpr int F_VEC = 128;                 // residual vectors per CTA (TMEM lan
 constexpr int F_ROWS = 128;                // calibration rows per CTA
 constexpr int F_N = 2 * F_ROWS;            // rows per pair row tile (UMMA N)
 constexpr int F_KS = 64;                   // elements per step: one 128-byte fp16 row
-constexpr int F_ASETS = 2;                 // A operand stages (tile sets) written by the producers
+constexpr int F_ASETS = 2;                 // A operand stages (tile sets) at least (the producers')
+constexpr int F_MAX_ASETS = 3;             // at most: where two raw slots still fit beside them
 constexpr int F_PRE_ASETS = 3;             // A operand stages filled by tile copies (clipping search)
 constexpr int F_BSLOTS = 3;                // B operand slots
 constexpr int F_SEG = 4;                   // steps per accumulation segment (256 elements)
@@ -84,9 +85,9 @@ constexpr uint32_t F_TMEM_COLS = 512;
 constexpr int F_SMEM_LIMIT = 232448;       // opt-in shared memory per CTA on sm_100 parts
 
 struct F16Ctrl {
-    uint64_t full[F_PRE_ASETS];    // even CTA: both CTAs' producer warps (A written, B landed)
-    uint64_t empty[F_PRE_ASETS];   // both CTAs: pair MMA commit (A stage free)
-    uint64_t afull[F_PRE_ASETS];   // this CTA's A tile copy (clipping search)
+    uint64_t full[F_MAX_ASETS];    // even CTA: both CTAs' producer warps (A written, B landed)
+    uint64_t empty[F_MAX_ASETS];   // both CTAs: pair MMA commit (A stage free)
+    uint64_t afull[F_MAX_ASETS];   // this CTA's A tile copy (clipping search)
     uint64_t bfull[F_BSLOTS];      // this CTA's B tile copy
     uint64_t bempty[F_BSLOTS];     // both CTAs: pair MMA commit (B slot free)
     uint64_t raw_full[F_MAX_RAW];  // this CTA's W and code tile copies
@@ -106,6 +107,8 @@ constexpr int F_BASE_SMEM = 1024 /* alignment slack */ + F_CTRL_BYTES + F_ASETS 
                             F_BSLOTS * F_SET;
 
 // Raw slot: W step [CH][64] fp32, then codes [K][CH][64] int8, as the tile copies write them.
+// A third A stage where two raw slots still fit beside it (it gives the producers a step of slack:
+// k_max = 8 2.80 -> 2.75 ms, k_max = 6 2.39 -> 2.27 ms on an 11008 x 4096 layer), else two.
 template <int KP1>
 struct FGeo {
     static constexpr int K = KP1 - 1;
@@ -114,9 +117,12 @@ struct FGeo {
     static constexpr int RAW_Q = CH * F_KS * 4;
     static constexpr uint32_t RAW_TX = CH * F_KS * 4 + K * CH * F_KS;
     static constexpr int RAW_BYTES = (RAW_Q + K * CH * F_KS + 1023) / 1024 * 1024;
-    static constexpr int RAW_FIT = (F_SMEM_LIMIT - F_BASE_SMEM) / RAW_BYTES;
+    static constexpr int NA =
+        (F_BASE_SMEM + F_SET + 2 * RAW_BYTES <= F_SMEM_LIMIT) ? F_MAX_ASETS : F_ASETS;
+    static constexpr int BASE = F_BASE_SMEM + (NA - F_ASETS) * F_SET;
+    static constexpr int RAW_FIT = (F_SMEM_LIMIT - BASE) / RAW_BYTES;
     static constexpr int RAW = RAW_FIT < F_MAX_RAW ? RAW_FIT : F_MAX_RAW;
-    static constexpr int SMEM = F_BASE_SMEM + RAW * RAW_BYTES;
+    static constexpr int SMEM = BASE + RAW * RAW_BYTES;
     static_assert(K >= 1, "at least one point");
     static_assert(RAW >= 2, "raw ring needs two slots");
 };
@@ -126,7 +132,7 @@ struct FGeo {
 // whatever their channel, A tiles copied from the residual planes (no raw ring).
 template <int KP1, bool CLIP>
 struct FShape {
-    static constexpr int kp1 = KP1, ch = FGeo<KP1>::CH, raw = FGeo<KP1>::RAW, na = F_ASETS;
+    static constexpr int kp1 = KP1, ch = FGeo<KP1>::CH, raw = FGeo<KP1>::RAW, na = FGeo<KP1>::NA;
     static constexpr int raw_bytes = FGeo<KP1>::RAW_BYTES, smem = FGeo<KP1>::SMEM;
     static constexpr uint32_t raw_tx = FGeo<KP1>::RAW_TX;
 };
